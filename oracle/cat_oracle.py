@@ -1,0 +1,387 @@
+"""Plain fp64 CPU oracle of the block Concentration-Alignment Transform (CAT) W4A4 linear layer.
+
+TEST INFRASTRUCTURE.  Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg
+of ``bench.py`` may import or run this module.  The CUDA library never calls it, and it shares
+no code, table or constant with the CUDA path; both sides only take their inputs from the
+seeded generators in ``workloads``.
+
+Everything here follows the paper ("Dissecting Quantization Error: A Concentration-Alignment
+Perspective") step by step, in float64, with numpy's LAPACK/BLAS routines (``eigh``,
+``matmul``) as the only library primitives.  Conventions (Sec. 3, Eq. 5):
+
+* a token is a row ``x`` of ``X`` [n, d_in]; the weight is ``W`` [d_out, d_in]; ``y = X W^T``.
+* the transform ``T`` acts on activations online (``x' = T x``) and its inverse is folded
+  into the weights offline (``W' = W T^{-1}``), so ``W' x' = W x``.
+* block CAT (Sec. 4, Eq. 10) is block diagonal with ``d_in / k`` blocks of size ``k``;
+  ``T_blocks[b]`` is the k x k block acting on channels ``b*k .. b*k+k-1``.
+
+Readings where the paper is garbled or silent (listed with reasons in the design notes):
+
+* INT4 grid: symmetric, step ``s = max|v| / 7``, codes in [-7, 7], round half to even.
+  The paper's step ``r / (2^b - 1)`` with ``r = 2 max|v|`` has no zero level; the restricted
+  symmetric grid keeps zero exact and never clips.  ``N_eff = r / s = 14`` is the number
+  of intervals this grid has; ``N(b) = 2^b - 1`` is the paper's.
+* Block CAT uses a k x k Sylvester Hadamard (orthonormal) in every block.
+* Maximum alignment (Eq. 9) uses the eigenvalues ``mu_i`` of ``W Sigma_x W^T``:
+  ``A_max = sum(mu) / (sum(sqrt(mu)))^2``.
+* k = 1 (end of Sec. 4): ``m_i = (sum_j W_ji^2 / E[x_i^2]) ** (1/4)``.
+
+Parity pins for every function live in ``tests/test_oracle_*.py``.
+"""
+from __future__ import annotations
+
+import dataclasses
+from typing import Dict, Optional
+
+import numpy as np
+
+QMAX4 = 7  # largest INT4 code of the restricted symmetric grid
+
+
+# ---------------------------------------------------------------------------------------------
+# Quantizer: Lemma 2 (range r(x) = 2 max|x_i| for symmetric quantization), App. A.2.1 (uniform
+# intervals of size s, round to nearest), Sec. 6 (activations per token, weights per output
+# channel, round-to-nearest).
+# ---------------------------------------------------------------------------------------------
+
+def quantize_rows_symmetric(V: np.ndarray, bits: int = 4):
+    """Quantize every row of ``V`` on its own symmetric uniform grid.
+
+    Returns ``(q, s, pre)``: integer codes (int64), the per-row step ``s = max|v| / qmax`` and
+    the pre-rounding values ``v / s``.  An all-zero row gets ``s = 0`` and codes 0."""
+    V = np.asarray(V, dtype=np.float64)
+    qmax = 2 ** (bits - 1) - 1
+    a = np.max(np.abs(V), axis=1) if V.shape[1] else np.zeros(V.shape[0])
+    s = a / qmax
+    pre = np.zeros_like(V)
+    nz = s > 0
+    pre[nz] = V[nz] / s[nz, None]
+    q = np.clip(np.rint(pre), -qmax, qmax).astype(np.int64)
+    return q, s, pre
+
+
+def dequantize_rows(q: np.ndarray, s: np.ndarray) -> np.ndarray:
+    """``Q(v) = s * q`` per row."""
+    return q.astype(np.float64) * s[:, None]
+
+
+# ---------------------------------------------------------------------------------------------
+# Matrix functions used by the alignment-optimal transform (Sec. 4, Eq. 7).
+# ---------------------------------------------------------------------------------------------
+
+def _sym(A: np.ndarray) -> np.ndarray:
+    return 0.5 * (A + A.T)
+
+
+def spd_power(A: np.ndarray, p: float) -> np.ndarray:
+    """``A^p`` for a symmetric positive definite ``A``: ``V diag(lambda^p) V^T``."""
+    lam, V = np.linalg.eigh(_sym(np.asarray(A, dtype=np.float64)))
+    if lam[0] <= 0:
+        raise np.linalg.LinAlgError("matrix is not positive definite")
+    return _sym((V * lam ** p) @ V.T)
+
+
+def geometric_mean(A: np.ndarray, B: np.ndarray) -> np.ndarray:
+    """Matrix geometric mean (Sec. 4, Eq. 7): ``A # B = A^{1/2} (A^{-1/2} B A^{-1/2})^{1/2} A^{1/2}``."""
+    Ah = spd_power(A, 0.5)
+    Aih = spd_power(A, -0.5)
+    return _sym(Ah @ spd_power(_sym(Aih @ B @ Aih), 0.5) @ Ah)
+
+
+def alignment_optimal_M(Sigma_x: np.ndarray, Sigma_w: np.ndarray):
+    """``M_hat = (Sigma_w # Sigma_x^{-1})^{1/2}`` (Sec. 4, Eq. 7).  Returns ``(M, M^{-1})``."""
+    G = geometric_mean(Sigma_w, np.linalg.inv(Sigma_x))
+    return spd_power(G, 0.5), spd_power(G, -0.5)
+
+
+def hadamard(k: int) -> np.ndarray:
+    """Orthonormal Sylvester Hadamard matrix of order k (a power of two): the +-1 matrix
+    S_1 = [1], S_2m = [[S_m, S_m], [S_m, -S_m]], divided by sqrt(k)."""
+    if k < 1 or k & (k - 1):
+        raise ValueError("Hadamard order must be a power of two")
+    S = np.ones((1, 1))
+    while S.shape[0] < k:
+        S = np.block([[S, S], [S, -S]])
+    return S / np.sqrt(float(k))
+
+
+# ---------------------------------------------------------------------------------------------
+# Calibration statistics (Sec. 4: Sigma_x = E[x x^T], Sigma_w = W^T W; Eq. 10 keeps the k x k
+# diagonal blocks).
+# ---------------------------------------------------------------------------------------------
+
+def calib_cov_block_sums(X: np.ndarray, k: int) -> np.ndarray:
+    """Sums over tokens of ``x_b x_b^T`` for every diagonal k x k block: [d/k, k, k].  Dividing by
+    the number of tokens gives the uncentered autocorrelation blocks of ``Sigma_x``."""
+    X = np.asarray(X, dtype=np.float64)
+    n, d = X.shape
+    nb = d // k
+    Xb = X.reshape(n, nb, k)
+    return np.einsum("tbi,tbj->bij", Xb, Xb)
+
+
+def weight_autocorr_blocks(W: np.ndarray, k: int) -> np.ndarray:
+    """Diagonal k x k blocks of ``Sigma_w = W^T W``: [d/k, k, k]."""
+    W = np.asarray(W, dtype=np.float64)
+    d_out, d = W.shape
+    nb = d // k
+    Wb = W.reshape(d_out, nb, k)
+    return np.einsum("obi,obj->bij", Wb, Wb)
+
+
+# ---------------------------------------------------------------------------------------------
+# Transforms (Sec. 3, Eq. 5; Sec. 4 two-step construction and Eq. 10).
+# ---------------------------------------------------------------------------------------------
+
+def build_transform(kind: str, d: int, k: int, Sigma_x_blocks: Optional[np.ndarray] = None,
+                    Sigma_w_blocks: Optional[np.ndarray] = None, signs: Optional[np.ndarray] = None):
+    """Block-diagonal transform ``T`` and its inverse, as [d/k, k, k] arrays.
+
+    * ``identity``: T = I (plain RTN W4A4).
+    * ``rht``: T_b = H_k Diag(sigma_b), sigma = the given random signs (a randomized Hadamard
+      rotation; orthogonal, so it leaves alignment unchanged, Sec. 2 Eq. 4).
+    * ``cat``: T_b = H_k M_hat_b with M_hat_b = (Sigma_w_b # Sigma_x_b^{-1})^{1/2} solved on the
+      block's own k x k sub-problem (Sec. 4, Eq. 7 and Eq. 10)."""
+    if d % k:
+        raise ValueError("d must be a multiple of k")
+    nb = d // k
+    H = hadamard(k)
+    T = np.empty((nb, k, k))
+    Ti = np.empty((nb, k, k))
+    for b in range(nb):
+        if kind == "identity":
+            T[b] = np.eye(k)
+            Ti[b] = np.eye(k)
+        elif kind == "rht":
+            sg = np.asarray(signs, dtype=np.float64)[b * k:(b + 1) * k]
+            T[b] = H * sg[None, :]
+            Ti[b] = sg[:, None] * H.T
+        elif kind == "cat":
+            M, Mi = alignment_optimal_M(Sigma_x_blocks[b], Sigma_w_blocks[b])
+            T[b] = H @ M
+            Ti[b] = Mi @ H.T
+        else:
+            raise ValueError(kind)
+    return T, Ti
+
+
+def apply_act_transform(X: np.ndarray, T_blocks: np.ndarray) -> np.ndarray:
+    """``x' = T x`` for every token row: ``X'_b = X_b T_b^T`` block by block."""
+    X = np.asarray(X, dtype=np.float64)
+    nb, k, _ = T_blocks.shape
+    out = np.empty_like(X)
+    for b in range(nb):
+        out[:, b * k:(b + 1) * k] = X[:, b * k:(b + 1) * k] @ T_blocks[b].T
+    return out
+
+
+def apply_weight_transform(W: np.ndarray, Tinv_blocks: np.ndarray) -> np.ndarray:
+    """``W' = W T^{-1}``: ``W'_b = W_b T_b^{-1}`` block by block."""
+    W = np.asarray(W, dtype=np.float64)
+    nb, k, _ = Tinv_blocks.shape
+    out = np.empty_like(W)
+    for b in range(nb):
+        out[:, b * k:(b + 1) * k] = W[:, b * k:(b + 1) * k] @ Tinv_blocks[b]
+    return out
+
+
+# ---------------------------------------------------------------------------------------------
+# Integer GEMM, dequantization and SQNR (Sec. 3 Eq. 5: y ~ Q(W T^{-1}) Q(T x); Sec. 2 Eq. 1).
+# ---------------------------------------------------------------------------------------------
+
+def int_gemm(qx: np.ndarray, qw: np.ndarray) -> np.ndarray:
+    """``acc[t, o] = sum_i qx[t, i] qw[o, i]`` exactly.  The products and every partial sum are
+    integers far below 2^53, so a float64 matmul is exact; the result is returned as int64."""
+    acc = np.asarray(qx, dtype=np.float64) @ np.asarray(qw, dtype=np.float64).T
+    return np.rint(acc).astype(np.int64)
+
+
+def dequantize_output(acc: np.ndarray, sx: np.ndarray, sw: np.ndarray) -> np.ndarray:
+    """``y_hat[t, o] = acc[t, o] * s_x[t] * s_w[o]``."""
+    return acc.astype(np.float64) * sx[:, None] * sw[None, :]
+
+
+def linear(X: np.ndarray, W: np.ndarray) -> np.ndarray:
+    """Full-precision layer output ``y = W x`` for every token."""
+    return np.asarray(X, dtype=np.float64) @ np.asarray(W, dtype=np.float64).T
+
+
+def sqnr_sums(y: np.ndarray, y_hat: np.ndarray):
+    """``(sum y^2, sum (y - y_hat)^2)`` over all tokens and outputs."""
+    y = np.asarray(y, dtype=np.float64)
+    e = y - np.asarray(y_hat, dtype=np.float64)
+    return float(np.sum(y * y)), float(np.sum(e * e))
+
+
+def sqnr_db(y: np.ndarray, y_hat: np.ndarray) -> float:
+    """SQNR (Sec. 2, Eq. 1) in dB: ``10 log10(E||W x||^2 / E||W x - W~ x~||^2)``."""
+    sig, err = sqnr_sums(y, y_hat)
+    return 10.0 * np.log10(sig / err)
+
+
+# ---------------------------------------------------------------------------------------------
+# The whole layer.
+# ---------------------------------------------------------------------------------------------
+
+@dataclasses.dataclass
+class PreparedWeights:
+    T: np.ndarray          # [d/k, k, k] activation transform blocks
+    Tinv: np.ndarray       # [d/k, k, k]
+    Wt: np.ndarray         # W T^{-1}
+    qw: np.ndarray         # int64 codes [d_out, d_in]
+    sw: np.ndarray         # per-output-channel steps [d_out]
+    pre_w: np.ndarray      # pre-rounding values
+
+
+def prepare_weights(W: np.ndarray, kind: str, k: int, X_calib: Optional[np.ndarray] = None,
+                    signs: Optional[np.ndarray] = None, Sigma_x_blocks: Optional[np.ndarray] = None
+                    ) -> PreparedWeights:
+    """Offline part: calibration statistics, transform, ``W T^{-1}`` and its per-channel INT4 codes."""
+    W = np.asarray(W, dtype=np.float64)
+    d = W.shape[1]
+    Sx = Sw = None
+    if kind == "cat":
+        if Sigma_x_blocks is None:
+            Xc = np.asarray(X_calib, dtype=np.float64)
+            Sigma_x_blocks = calib_cov_block_sums(Xc, k) / Xc.shape[0]
+        Sx = Sigma_x_blocks
+        Sw = weight_autocorr_blocks(W, k)
+    T, Ti = build_transform(kind, d, k, Sx, Sw, signs)
+    Wt = apply_weight_transform(W, Ti)
+    qw, sw, pre_w = quantize_rows_symmetric(Wt)
+    return PreparedWeights(T=T, Tinv=Ti, Wt=Wt, qw=qw, sw=sw, pre_w=pre_w)
+
+
+@dataclasses.dataclass
+class ActCodes:
+    Xt: np.ndarray        # T x for every token
+    qx: np.ndarray        # int64 codes [n, d_in]
+    sx: np.ndarray        # per-token steps [n]
+    pre_x: np.ndarray
+
+
+def transform_quantize_act(X: np.ndarray, T_blocks: np.ndarray) -> ActCodes:
+    """Online part, first half: ``x' = T x`` and its per-token INT4 codes."""
+    Xt = apply_act_transform(X, T_blocks)
+    qx, sx, pre = quantize_rows_symmetric(Xt)
+    return ActCodes(Xt=Xt, qx=qx, sx=sx, pre_x=pre)
+
+
+def w4a4_linear(qx, sx, qw, sw):
+    """Online part, second half: integer GEMM and dequantization.  Returns ``(acc, y_hat)``."""
+    acc = int_gemm(qx, qw)
+    return acc, dequantize_output(acc, sx, sw)
+
+
+def cat_layer(X: np.ndarray, W: np.ndarray, kind: str, k: int, X_calib: Optional[np.ndarray] = None,
+              signs: Optional[np.ndarray] = None) -> Dict[str, object]:
+    """Every step of the layer, in the paper's order, returning all intermediates."""
+    pw = prepare_weights(W, kind, k, X_calib=X_calib, signs=signs)
+    ac = transform_quantize_act(X, pw.T)
+    acc, y_hat = w4a4_linear(ac.qx, ac.sx, pw.qw, pw.sw)
+    y = linear(X, W)
+    sig, err = sqnr_sums(y, y_hat)
+    return dict(prep=pw, act=ac, acc=acc, y_hat=y_hat, y=y, sig=sig, err=err,
+                sqnr_db=10.0 * np.log10(sig / err))
+
+
+# ---------------------------------------------------------------------------------------------
+# Analysis quantities (Sec. 2: Lemma 1-3, Theorem 1, concentration and alignment; Sec. 4 Eq. 9).
+# ---------------------------------------------------------------------------------------------
+
+def parallel(a: float, b: float) -> float:
+    """``a || b = (1/a + 1/b)^{-1}`` (Lemma 1)."""
+    return 1.0 / (1.0 / a + 1.0 / b)
+
+
+def range_symmetric(V: np.ndarray) -> np.ndarray:
+    """``r(v) = 2 max_i |v_i|`` per row (Lemma 2)."""
+    return 2.0 * np.max(np.abs(np.asarray(V, dtype=np.float64)), axis=1)
+
+
+def range_asymmetric(V: np.ndarray) -> np.ndarray:
+    """``r(v) = max_i v_i - min_i v_i`` per row (Lemma 2)."""
+    V = np.asarray(V, dtype=np.float64)
+    return np.max(V, axis=1) - np.min(V, axis=1)
+
+
+def concentration_act(X: np.ndarray, symmetric: bool = True) -> float:
+    """``C(x) = E||x||^2 / E[r(x)^2]`` over tokens (Lemma 2)."""
+    X = np.asarray(X, dtype=np.float64)
+    r = range_symmetric(X) if symmetric else range_asymmetric(X)
+    return float(np.mean(np.sum(X * X, axis=1)) / np.mean(r * r))
+
+
+def concentration_weight(W: np.ndarray) -> float:
+    """``C(W) = sum_i ||w_i||^2 / sum_i r(w_i)^2`` over output rows (Lemma 3)."""
+    W = np.asarray(W, dtype=np.float64)
+    r = range_symmetric(W)
+    return float(np.sum(W * W) / np.sum(r * r))
+
+
+def alignment(X: np.ndarray, W: np.ndarray) -> float:
+    """``A(x, W) = E||W x||^2 / (||W||_F^2 E||x||^2)`` (Lemma 2)."""
+    X = np.asarray(X, dtype=np.float64)
+    W = np.asarray(W, dtype=np.float64)
+    Y = X @ W.T
+    return float(np.mean(np.sum(Y * Y, axis=1)) / (np.sum(W * W) * np.mean(np.sum(X * X, axis=1))))
+
+
+def alignment_from_moments(Sigma_x: np.ndarray, Sigma_w: np.ndarray) -> float:
+    """``A = Tr(Sigma_w Sigma_x) / (Tr(Sigma_w) Tr(Sigma_x))``: the same ratio written with
+    ``E||W x||^2 = Tr(W^T W E[x x^T])``."""
+    return float(np.trace(Sigma_w @ Sigma_x) / (np.trace(Sigma_w) * np.trace(Sigma_x)))
+
+
+def max_alignment(Sigma_x: np.ndarray, W: np.ndarray) -> float:
+    """Largest alignment reachable by an invertible transform (Sec. 4, Eq. 9), in terms of the
+    eigenvalues ``mu_i`` of ``Sigma_y = W Sigma_x W^T``: ``sum(mu) / (sum(sqrt(mu)))^2``."""
+    W = np.asarray(W, dtype=np.float64)
+    mu = np.linalg.eigvalsh(_sym(W @ Sigma_x @ W.T))
+    mu = np.clip(mu, 0.0, None)
+    return float(np.sum(mu) / np.sum(np.sqrt(mu)) ** 2)
+
+
+def sqnr_act_only(X: np.ndarray, W: np.ndarray, bits: int = 4) -> float:
+    """Measured ``SQNR(W x~)``: only activations quantized (per token)."""
+    q, s, _ = quantize_rows_symmetric(X, bits)
+    return 10 ** (sqnr_db(linear(X, W), linear(dequantize_rows(q, s), W)) / 10)
+
+
+def sqnr_weight_only(X: np.ndarray, W: np.ndarray, bits: int = 4) -> float:
+    """Measured ``SQNR(W~ x)``: only weights quantized (per output channel)."""
+    q, s, _ = quantize_rows_symmetric(W, bits)
+    return 10 ** (sqnr_db(linear(X, W), linear(X, dequantize_rows(q, s))) / 10)
+
+
+def sqnr_both(X: np.ndarray, W: np.ndarray, bits_x: int = 4, bits_w: int = 4) -> float:
+    """Measured ``SQNR(W~ x~)`` (Sec. 2, Eq. 1), linear scale."""
+    qx, sx, _ = quantize_rows_symmetric(X, bits_x)
+    qw, sw, _ = quantize_rows_symmetric(W, bits_w)
+    return 10 ** (sqnr_db(linear(X, W), linear(dequantize_rows(qx, sx), dequantize_rows(qw, sw))) / 10)
+
+
+def n_intervals(bits: int, paper: bool = False) -> float:
+    """Number of quantization intervals across the range: the paper's ``N(b) = 2^b - 1``, or the
+    ``2 (2^{b-1} - 1)`` intervals of the restricted symmetric grid used here (``r / s``)."""
+    return float(2 ** bits - 1) if paper else float(2 * (2 ** (bits - 1) - 1))
+
+
+def lemma2_act_sqnr(X: np.ndarray, W: np.ndarray, bits: int = 4, paper_N: bool = False) -> float:
+    """Lemma 2: ``SQNR(W x~) ~ 12 N(b_x)^2 C(x) A(x, W)``."""
+    return 12.0 * n_intervals(bits, paper_N) ** 2 * concentration_act(X) * alignment(X, W)
+
+
+def lemma3_weight_sqnr(X: np.ndarray, W: np.ndarray, bits: int = 4, paper_N: bool = False) -> float:
+    """Lemma 3: ``SQNR(W~ x) ~ 12 N(b_w)^2 C(W) A(x, W)``."""
+    return 12.0 * n_intervals(bits, paper_N) ** 2 * concentration_weight(W) * alignment(X, W)
+
+
+def theorem1_sqnr(X: np.ndarray, W: np.ndarray, bits_x: int = 4, bits_w: int = 4, paper_N: bool = False) -> float:
+    """Theorem 1: ``SQNR ~ 12 (N(b_x)^2 C(x) || N(b_w)^2 C(W)) A(x, W)``."""
+    nx, nw = n_intervals(bits_x, paper_N), n_intervals(bits_w, paper_N)
+    return 12.0 * parallel(nx ** 2 * concentration_act(X), nw ** 2 * concentration_weight(W)) * alignment(X, W)
+
+
+def db(v: float) -> float:
+    return 10.0 * np.log10(v)

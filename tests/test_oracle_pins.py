@@ -1,0 +1,435 @@
+"""Pins for the CPU oracle: hand-worked fixtures, closed forms, exact invariants, library
+routines and brute force.  None of them reuses the oracle's own formula to check itself."""
+import os
+
+import numpy as np
+import pytest
+import scipy.linalg
+
+import oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _rng(seed=0):
+    return np.random.default_rng(seed)
+
+
+def _rand_spd(rng, k, cond=10.0):
+    Q, _ = np.linalg.qr(rng.standard_normal((k, k)))
+    lam = np.exp(rng.uniform(0, np.log(cond), k))
+    return (Q * lam) @ Q.T
+
+
+def _rand_orth(rng, d):
+    Q, R = np.linalg.qr(rng.standard_normal((d, d)))
+    return Q * np.sign(np.diag(R))
+
+
+# ------------------------------------------------------------------------------------------
+# Quantizer (Lemma 2 range, App. A.2.1 steps, Sec. 6 RTN)
+# ------------------------------------------------------------------------------------------
+
+def _read_quant_golden():
+    cases = []
+    with open(os.path.join(GOLDEN, "quantizer_rows.txt")) as f:
+        for line in f:
+            line = line.strip()
+            if not line or line.startswith("#"):
+                continue
+            row, s, codes = [p.strip() for p in line.split("|")]
+            cases.append((np.array([float(v) for v in row.split()]), float(s),
+                          np.array([int(v) for v in codes.split()])))
+    return cases
+
+
+@pytest.mark.parametrize("case", range(5))
+def test_quantizer_hand_worked_rows(case):
+    row, s_exp, q_exp = _read_quant_golden()[case]
+    q, s, pre = O.quantize_rows_symmetric(row[None, :])
+    assert s[0] == s_exp
+    np.testing.assert_array_equal(q[0], q_exp)
+
+
+def test_quantizer_ranges_and_error_bound():
+    rng = _rng(1)
+    V = rng.standard_normal((200, 96)) * np.exp(rng.standard_normal((200, 1)))
+    V[3] = 0.0
+    V[7, 5] = 40.0  # an outlier
+    q, s, pre = O.quantize_rows_symmetric(V)
+    assert q.min() >= -7 and q.max() <= 7
+    # the element of largest magnitude maps to +-7
+    idx = np.argmax(np.abs(V), axis=1)
+    big = q[np.arange(V.shape[0]), idx]
+    assert np.all(np.abs(big[np.arange(200) != 3]) == 7)
+    # zero row
+    assert s[3] == 0 and np.all(q[3] == 0)
+    # |v - s q| <= s / 2 (no clipping: the range covers the row)
+    err = np.abs(V - q * s[:, None])
+    assert np.all(err <= s[:, None] / 2 * (1 + 1e-12) + 1e-300)
+    # step size is max|v| / 7 exactly
+    np.testing.assert_array_equal(s, np.max(np.abs(V), axis=1) / 7)
+
+
+def test_quantizer_bit_widths():
+    rng = _rng(2)
+    V = rng.standard_normal((50, 33))
+    for b in (2, 3, 4, 6, 8):
+        q, s, _ = O.quantize_rows_symmetric(V, bits=b)
+        qmax = 2 ** (b - 1) - 1
+        assert q.min() == -qmax or q.max() == qmax
+        assert np.abs(q).max() == qmax
+
+
+# ------------------------------------------------------------------------------------------
+# Hadamard, matrix powers and the geometric mean (Sec. 4, Eq. 7)
+# ------------------------------------------------------------------------------------------
+
+def test_hadamard_matches_textbook_order4_and_is_orthonormal():
+    H4 = np.loadtxt(os.path.join(GOLDEN, "hadamard4.txt"))
+    np.testing.assert_array_equal(O.hadamard(4) * 2.0, H4)
+    for k in (1, 2, 32, 128, 256):
+        H = O.hadamard(k)
+        np.testing.assert_allclose(H @ H.T, np.eye(k), atol=1e-12)
+        np.testing.assert_allclose(np.abs(H), 1 / np.sqrt(k), rtol=1e-14)
+    with pytest.raises(ValueError):
+        O.hadamard(12)
+
+
+def test_spd_power_against_scipy_sqrtm_and_inverse():
+    rng = _rng(3)
+    A = _rand_spd(rng, 24, cond=1e4)
+    np.testing.assert_allclose(O.spd_power(A, 0.5), scipy.linalg.sqrtm(A).real, rtol=1e-9, atol=1e-12)
+    np.testing.assert_allclose(O.spd_power(A, -1.0), np.linalg.inv(A), rtol=1e-8, atol=1e-12)
+    with pytest.raises(np.linalg.LinAlgError):
+        O.spd_power(-np.eye(3), 0.5)
+
+
+def test_geometric_mean_closed_forms_and_riccati():
+    rng = _rng(4)
+    # scalars: a # b = sqrt(a b)
+    assert np.isclose(O.geometric_mean(np.array([[4.0]]), np.array([[9.0]]))[0, 0], 6.0, rtol=1e-14)
+    # commuting (diagonal) matrices: A # B = (A B)^{1/2}
+    a, b = rng.uniform(0.1, 10, 7), rng.uniform(0.1, 10, 7)
+    np.testing.assert_allclose(O.geometric_mean(np.diag(a), np.diag(b)), np.diag(np.sqrt(a * b)), rtol=1e-12)
+    # general SPD: G = A # B is the SPD solution of G A^{-1} G = B, symmetric in A, B, and A # A^{-1} = I
+    A, B = _rand_spd(rng, 16, 1e3), _rand_spd(rng, 16, 1e3)
+    G = O.geometric_mean(A, B)
+    np.testing.assert_allclose(G @ np.linalg.inv(A) @ G, B, rtol=1e-8, atol=1e-10)
+    np.testing.assert_allclose(G, O.geometric_mean(B, A), rtol=1e-8, atol=1e-10)
+    assert np.linalg.eigvalsh(G).min() > 0
+    np.testing.assert_allclose(O.geometric_mean(A, np.linalg.inv(A)), np.eye(16), atol=1e-9)
+
+
+def test_alignment_optimal_M_fixed_point_eq8():
+    """Eq. 8: M Sigma_x M = M^{-1} Sigma_w M^{-1}; its eigenvalues are those of
+    (Sigma_x^{1/2} Sigma_w Sigma_x^{1/2})^{1/2} (the printed right-hand side is garbled)."""
+    rng = _rng(5)
+    Sx, Sw = _rand_spd(rng, 12, 1e3), _rand_spd(rng, 12, 1e2)
+    M, Mi = O.alignment_optimal_M(Sx, Sw)
+    np.testing.assert_allclose(M @ Mi, np.eye(12), atol=1e-9)
+    L = M @ Sx @ M
+    np.testing.assert_allclose(L, Mi @ Sw @ Mi, rtol=1e-8, atol=1e-10)
+    # eigenvalues
+    Sxh = scipy.linalg.sqrtm(Sx).real
+    ref = np.sqrt(np.linalg.eigvalsh(Sxh @ Sw @ Sxh))
+    np.testing.assert_allclose(np.sort(np.linalg.eigvalsh(L)), np.sort(ref), rtol=1e-8)
+    # and Sigma_w = G Sigma_x G with G = M^2 (definition of Sigma_w # Sigma_x^{-1})
+    np.testing.assert_allclose(M @ M @ Sx @ M @ M, Sw, rtol=1e-8, atol=1e-10)
+
+
+# ------------------------------------------------------------------------------------------
+# Calibration statistics and brute force
+# ------------------------------------------------------------------------------------------
+
+def test_calib_cov_blocks_brute_force():
+    rng = _rng(6)
+    X = rng.standard_normal((37, 24))
+    S = O.calib_cov_block_sums(X, 8)
+    full = np.zeros((24, 24))
+    for t in range(37):  # one outer product per token
+        full += np.outer(X[t], X[t])
+    for b in range(3):
+        np.testing.assert_allclose(S[b], full[b * 8:(b + 1) * 8, b * 8:(b + 1) * 8], rtol=1e-13)
+    W = rng.standard_normal((19, 24))
+    Sw = O.weight_autocorr_blocks(W, 8)
+    WtW = W.T @ W
+    for b in range(3):
+        np.testing.assert_allclose(Sw[b], WtW[b * 8:(b + 1) * 8, b * 8:(b + 1) * 8], rtol=1e-13)
+
+
+def test_int_gemm_brute_force_and_extremes():
+    rng = _rng(7)
+    qx = rng.integers(-7, 8, (9, 70))
+    qw = rng.integers(-7, 8, (5, 70))
+    acc = O.int_gemm(qx, qw)
+    for t in range(9):
+        for o in range(5):
+            assert acc[t, o] == sum(int(qx[t, i]) * int(qw[o, i]) for i in range(70))
+    # largest accumulator of the layers here: 49 * 14336
+    big = O.int_gemm(np.full((2, 14336), 7), np.full((3, 14336), -7))
+    assert np.all(big == -49 * 14336)
+    assert acc.dtype == np.int64
+
+
+def test_dequantize_output_orientation():
+    acc = np.array([[1, 2, 3], [4, 5, 6]])
+    y = O.dequantize_output(acc, np.array([2.0, 3.0]), np.array([1.0, 10.0, 100.0]))
+    np.testing.assert_array_equal(y, [[2, 40, 600], [12, 150, 1800]])
+
+
+def test_sqnr_hand_worked():
+    vals = dict(l.split() for l in open(os.path.join(GOLDEN, "sqnr_example.txt")) if l[0] != "#")
+    y = np.array([[1.0, 2.0], [3.0, 4.0]])
+    yh = np.array([[1.0, 2.0], [3.0, 3.0]])
+    sig, err = O.sqnr_sums(y, yh)
+    assert sig == float(vals["sig"]) and err == float(vals["err"])
+    assert abs(O.sqnr_db(y, yh) - float(vals["sqnr_db"])) < 1e-12
+    assert abs(O.sqnr_db(np.ones(10), 0.9 * np.ones(10)) - 20.0) < 1e-9
+
+
+# ------------------------------------------------------------------------------------------
+# Transforms: function preservation (Eq. 5), rotation invariance (Eq. 4)
+# ------------------------------------------------------------------------------------------
+
+@pytest.mark.parametrize("kind", ["identity", "rht", "cat"])
+def test_function_preservation_eq5(kind):
+    rng = _rng(8)
+    d, k = 64, 16
+    X = rng.standard_normal((300, d)) @ rng.standard_normal((d, d)) * 0.3
+    X[:, 5] *= 40
+    W = rng.standard_normal((48, d)) * 0.02
+    signs = rng.choice([-1.0, 1.0], d)
+    Sx = O.calib_cov_block_sums(X, k) / X.shape[0]
+    Sw = O.weight_autocorr_blocks(W, k)
+    T, Ti = O.build_transform(kind, d, k, Sx, Sw, signs)
+    for b in range(d // k):
+        np.testing.assert_allclose(T[b] @ Ti[b], np.eye(k), atol=1e-9)
+    y = O.linear(X, W)
+    y2 = O.linear(O.apply_act_transform(X, T), O.apply_weight_transform(W, Ti))
+    assert np.linalg.norm(y2 - y) / np.linalg.norm(y) < 1e-10
+
+
+def test_act_transform_is_T_times_x():
+    rng = _rng(9)
+    d, k = 12, 4
+    T = rng.standard_normal((3, k, k))
+    X = rng.standard_normal((5, d))
+    Tfull = scipy.linalg.block_diag(*T)
+    np.testing.assert_allclose(O.apply_act_transform(X, T), (Tfull @ X.T).T, rtol=1e-13)
+    Ti = rng.standard_normal((3, k, k))
+    W = rng.standard_normal((7, d))
+    np.testing.assert_allclose(O.apply_weight_transform(W, Ti), W @ scipy.linalg.block_diag(*Ti), rtol=1e-13)
+
+
+def test_rht_signs_and_alignment_invariance_eq4():
+    rng = _rng(10)
+    d, k = 32, 8
+    X = rng.standard_normal((500, d)) * rng.uniform(0.1, 5, d)
+    W = rng.standard_normal((20, d))
+    signs = rng.choice([-1.0, 1.0], d)
+    T, Ti = O.build_transform("rht", d, k, signs=signs)
+    H = O.hadamard(k)
+    np.testing.assert_allclose(T[1], H @ np.diag(signs[k:2 * k]), rtol=1e-14)
+    a0 = O.alignment(X, W)
+    a1 = O.alignment(O.apply_act_transform(X, T), O.apply_weight_transform(W, Ti))
+    assert abs(a1 - a0) < 1e-12 * a0
+    R = _rand_orth(rng, d)
+    a2 = O.alignment(X @ R.T, W @ R.T)
+    assert abs(a2 - a0) < 1e-12 * a0
+
+
+def test_alignment_moment_form_and_bound():
+    rng = _rng(11)
+    X = rng.standard_normal((400, 16)) * rng.uniform(0.1, 3, 16)
+    W = rng.standard_normal((10, 16))
+    a = O.alignment(X, W)
+    assert abs(a - O.alignment_from_moments(X.T @ X / 400, W.T @ W)) < 1e-12
+    assert 0 < a <= 1.0
+
+
+# ------------------------------------------------------------------------------------------
+# Optimal alignment (Eq. 7, Eq. 9), block optimality (Eq. 10) and k = 1
+# ------------------------------------------------------------------------------------------
+
+def test_full_rank_M_reaches_max_alignment_eq9_and_beats_random():
+    rng = _rng(12)
+    d = 10
+    X = rng.standard_normal((2000, d)) @ rng.standard_normal((d, d))
+    W = rng.standard_normal((14, d)) * rng.uniform(0.2, 3, (14, 1))
+    Sx, Sw = X.T @ X / X.shape[0], W.T @ W
+    M, Mi = O.alignment_optimal_M(Sx, Sw)
+    a_opt = O.alignment(X @ M.T, W @ Mi)
+    a_max = O.max_alignment(Sx, W)
+    # closed form written independently: singular values of W Sigma_x^{1/2}
+    sv = np.linalg.svd(W @ scipy.linalg.sqrtm(Sx).real, compute_uv=False)
+    assert abs(a_max - np.sum(sv ** 2) / np.sum(sv) ** 2) < 1e-8 * a_max
+    assert abs(a_opt - a_max) < 1e-7 * a_max
+    assert a_opt > O.alignment(X, W)
+    for _ in range(1500):
+        Mr = rng.standard_normal((d, d)) + 3 * np.eye(d) * rng.uniform(0, 1)
+        Mr2 = M @ (np.eye(d) + 0.05 * rng.standard_normal((d, d)))
+        for MM in (Mr, Mr2):
+            if abs(np.linalg.det(MM)) < 1e-6:
+                continue
+            assert O.alignment(X @ MM.T, W @ np.linalg.inv(MM)) <= a_opt * (1 + 1e-9)
+
+
+def _blocks_data(rng, d, n=3000):
+    X = rng.standard_normal((n, d)) @ rng.standard_normal((d, d)) * 0.5
+    X[:, 3] *= 30
+    W = rng.standard_normal((2 * d, d)) * rng.lognormal(0, 0.5, (2 * d, 1))
+    return X, W
+
+
+def test_block_cat_is_optimal_among_block_diagonal_transforms():
+    """Eq. 10: solving each k x k block on its own sub-problem is optimal among all block-diagonal
+    transforms (no per-block rescaling raises alignment), with closed form
+    A = Tr(Sw Sx) / (sum_b Tr((Sx_b^{1/2} Sw_b Sx_b^{1/2})^{1/2}))^2."""
+    rng = _rng(13)
+    d, k = 16, 4
+    X, W = _blocks_data(rng, d)
+    Sx_full = X.T @ X / X.shape[0]
+    Sxb = O.calib_cov_block_sums(X, k) / X.shape[0]
+    Swb = O.weight_autocorr_blocks(W, k)
+    T, Ti = O.build_transform("cat", d, k, Sxb, Swb)
+    a_cat = O.alignment(O.apply_act_transform(X, T), O.apply_weight_transform(W, Ti))
+    denom = 0.0
+    for b in range(d // k):
+        h = scipy.linalg.sqrtm(Sxb[b]).real
+        denom += np.trace(scipy.linalg.sqrtm(h @ Swb[b] @ h).real)
+    closed = np.trace(W.T @ W @ Sx_full) / denom ** 2
+    assert abs(a_cat - closed) < 1e-9 * closed
+    assert a_cat >= O.alignment(X, W)
+    assert a_cat <= O.max_alignment(Sx_full, W) * (1 + 1e-12)
+    for _ in range(300):
+        c = np.exp(rng.standard_normal(d // k))
+        D = np.repeat(c, k)
+        Ts = T * c[:, None, None]
+        Tis = Ti / c[:, None, None]
+        assert O.alignment(O.apply_act_transform(X, Ts), O.apply_weight_transform(W, Tis)) <= a_cat * (1 + 1e-10)
+        Rb = rng.standard_normal((d // k, k, k)) + 2 * np.eye(k)
+        Rbi = np.linalg.inv(Rb)
+        assert O.alignment(O.apply_act_transform(X, Rb), O.apply_weight_transform(W, Rbi)) <= a_cat * (1 + 1e-10)
+        del D
+
+
+def test_k1_closed_form_diagonal_scaling():
+    """End of Sec. 4: for k = 1 the block solution is a diagonal scaling; from Eq. 7 with 1 x 1
+    blocks m_i = (sum_j W_ji^2 / E[x_i^2])^{1/4} (the printed exponent is garbled)."""
+    rng = _rng(14)
+    d = 12
+    X, W = _blocks_data(rng, d)
+    Sxb = O.calib_cov_block_sums(X, 1) / X.shape[0]
+    Swb = O.weight_autocorr_blocks(W, 1)
+    T, Ti = O.build_transform("cat", d, 1, Sxb, Swb)
+    m = (np.sum(W ** 2, axis=0) / np.mean(X ** 2, axis=0)) ** 0.25
+    np.testing.assert_allclose(T[:, 0, 0], m, rtol=1e-12)
+    a = O.alignment(X * m, W / m)
+    for i in range(d):  # finite-difference perturbations never raise A
+        for eps in (1e-3, -1e-3, 0.1, -0.1):
+            mm = m.copy()
+            mm[i] *= np.exp(eps)
+            assert O.alignment(X * mm, W / mm) <= a * (1 + 1e-12)
+
+
+# ------------------------------------------------------------------------------------------
+# SQNR decomposition (App. A.1 and A.2): exact identities, then the approximations
+# ------------------------------------------------------------------------------------------
+
+def test_error_expansion_identity_app_a1():
+    rng = _rng(15)
+    X = rng.standard_normal((256, 32)) * rng.uniform(0.2, 4, 32)
+    W = rng.standard_normal((24, 32)) * 0.1
+    qx, sx, _ = O.quantize_rows_symmetric(X)
+    qw, sw, _ = O.quantize_rows_symmetric(W)
+    Xq, Wq = O.dequantize_rows(qx, sx), O.dequantize_rows(qw, sw)
+    dX, dW = X - Xq, W - Wq
+    sig, err = O.sqnr_sums(O.linear(X, W), O.linear(Xq, Wq))
+    a = np.sum((dX @ W.T) ** 2)
+    b = np.sum((X @ dW.T) ** 2)
+    c = np.sum((dX @ dW.T) ** 2)
+    cross = 2 * (np.sum((dX @ W.T) * (X @ dW.T)) - np.sum((dX @ W.T) * (dX @ dW.T))
+                 - np.sum((X @ dW.T) * (dX @ dW.T)))
+    assert abs(err - (a + b + c + cross)) < 1e-10 * err
+    assert abs(sig - np.sum((X @ W.T) ** 2)) < 1e-10 * sig
+    # acc-based path equals the dequantized float path
+    _, yh = O.w4a4_linear(qx, sx, qw, sw)
+    np.testing.assert_allclose(yh, O.linear(Xq, Wq), rtol=1e-12, atol=1e-14)
+
+
+def test_activation_mse_trace_form_app_a21():
+    """App. A.2.1: E||W dx||^2 = Tr(W^T W E[dx dx^T]) exactly."""
+    rng = _rng(16)
+    X = rng.standard_normal((500, 20))
+    W = rng.standard_normal((9, 20))
+    q, s, _ = O.quantize_rows_symmetric(X)
+    dX = X - O.dequantize_rows(q, s)
+    lhs = np.mean(np.sum((dX @ W.T) ** 2, axis=1))
+    rhs = np.trace(W.T @ W @ (dX.T @ dX / 500))
+    assert abs(lhs - rhs) < 1e-12 * lhs
+
+
+def test_concentration_bounds():
+    """Sec. 2 (Concentration): lowest value 1/4 (-6 dB) for symmetric, 1/2 (-3 dB) for asymmetric."""
+    onehot = np.zeros((3, 10))
+    onehot[np.arange(3), [1, 4, 9]] = [2.0, -5.0, 0.5]
+    assert O.concentration_act(onehot) == 0.25
+    pair = np.zeros((2, 8))
+    pair[:, 0], pair[:, 1] = 3.0, -3.0
+    assert O.concentration_act(pair, symmetric=False) == 0.5
+    rng = _rng(17)
+    for _ in range(20):
+        V = rng.standard_normal((50, 16)) ** 3
+        assert O.concentration_act(V) >= 0.25
+        assert O.concentration_act(V, symmetric=False) >= 0.5
+        assert O.concentration_weight(V) >= 0.25
+    # scale invariance (Sec. 2)
+    V = rng.standard_normal((30, 12))
+    assert abs(O.concentration_act(V * 7.5) - O.concentration_act(V)) < 1e-14
+
+
+def test_lemmas_and_theorem1_on_gaussian_layer():
+    """Lemma 1-3 / Theorem 1 are approximations; the paper reports them accurate between 5 and
+    50 dB (Sec. 2).  On a Gaussian layer: within 0.2 dB at 8 bits, 1 dB at 4 bits, and about
+    6 dB per extra bit (Eq. 3)."""
+    rng = _rng(18)
+    d = 64
+    X = rng.standard_normal((60000, d))
+    W = rng.standard_normal((64, d))
+    for bits, tol in ((8, 0.2), (4, 1.0)):
+        ma = O.sqnr_act_only(X, W, bits)
+        mw = O.sqnr_weight_only(X, W, bits)
+        mb = O.sqnr_both(X, W, bits, bits)
+        assert abs(O.db(O.lemma2_act_sqnr(X, W, bits)) - O.db(ma)) < tol
+        assert abs(O.db(O.lemma3_weight_sqnr(X, W, bits)) - O.db(mw)) < tol
+        assert abs(O.db(O.parallel(ma, mw)) - O.db(mb)) < tol          # Lemma 1
+        assert abs(O.db(O.theorem1_sqnr(X, W, bits, bits)) - O.db(mb)) < tol
+    g = O.db(O.sqnr_both(X, W, 10, 10)) - O.db(O.sqnr_both(X, W, 9, 9))
+    assert 5.8 < g < 6.3
+
+
+def test_identity_transform_is_plain_rtn():
+    rng = _rng(19)
+    X = rng.standard_normal((40, 32)) * 3
+    W = rng.standard_normal((16, 32))
+    out = O.cat_layer(X, W, "identity", 8)
+    qx, sx, _ = O.quantize_rows_symmetric(X)
+    qw, sw, _ = O.quantize_rows_symmetric(W)
+    np.testing.assert_array_equal(out["act"].qx, qx)
+    np.testing.assert_array_equal(out["prep"].qw, qw)
+    np.testing.assert_array_equal(out["acc"], O.int_gemm(qx, qw))
+
+
+def test_cat_improves_sqnr_on_outlier_layer():
+    """Sec. 4 / Fig. 6 (qualitative): CAT raises alignment and SQNR over no transform and over a
+    randomized Hadamard rotation on a layer with correlated channels and outliers."""
+    import workloads as WL
+    cfg = WL.small_config("pin", d_in=256, d_out=192, n_eval=512, n_calib=512, k=32, dtype="f32", seed=3)
+    L = WL.make_layer(cfg)
+    X, W, Xc = L.x_eval.values, L.W.values, L.x_calib.values
+    res = {kind: O.cat_layer(X, W, kind, cfg.k, X_calib=Xc, signs=L.rht_signs) for kind in ("identity", "rht", "cat")}
+    assert res["rht"]["sqnr_db"] > res["identity"]["sqnr_db"]
+    assert res["cat"]["sqnr_db"] > res["rht"]["sqnr_db"]
+    for r in res.values():
+        assert np.linalg.norm(r["prep"].Wt @ np.eye(256)) > 0
