@@ -1,0 +1,395 @@
+#!/usr/bin/env python
+"""Benchmark of the block-CAT W4A4 linear layer on GB300; prints one JSON line on rank 0.
+
+A step is one pass of the whole hot path over one batch of synthetic input, through the C ABI:
+  cat_calib_cov (calibration Sigma_x blocks of the step's calibration tokens)
+  -> cat_transform_quantize_act (x' = T x, per-token INT4)
+  -> cat_w4a4_linear (integer GEMM + dequantization)
+  -> cat_sqnr (SQNR against the full-precision output).
+The weights are prepared once before timing (cat_quantize_weights, an offline step).  The
+full-precision reference y = W x used by the SQNR is computed once by the harness (fp32 GEMM,
+TF32 off) and is an input of every step.
+
+  python bench.py [--steps K] [--warmup W] [--config NAME] [--impl ours|reference]
+  python -m torch.distributed.run --nproc-per-node N ... bench.py --gpus N   (independent replicas)
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+import workloads as WL  # noqa: E402
+
+METRIC = "CAT W4A4 linear tokens/s & effective TOPS, % of int8/HBM roofline; SQNR dB"
+DEFAULT_CONFIG = "c2_qkv_4096x6144_k128_bf16"
+FP8_PER_BF16 = 2.0          # nominal dense FP8 / BF16 tensor throughput ratio (4.5 / 2.25 PFLOP/s)
+FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}
+L2_FLUSH_BYTES = 256 << 20  # > 2x the 126.5 MiB L2
+LAUNCHES_PER_STEP = 7       # calib_cov 1, transform_quantize 3, w4a4_linear 1, sqnr 2
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--config", default=DEFAULT_CONFIG, choices=sorted(WL.CONFIGS))
+    p.add_argument("--kind", default="cat", choices=["identity", "rht", "cat"])
+    p.add_argument("--k", type=int, default=0, help="block size (default: the config's)")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=12.0, help="budget of the CPU-baseline sample")
+    return p.parse_args()
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return {"hbm_gbs": float(d["hbm_gbs"]), "bf16_tflops": float(d["bf16_tflops"]), "source": "measured"}
+    except Exception:
+        return dict(FALLBACK, source="fallback")
+
+
+def committed_json(name):
+    try:
+        with open(os.path.join(ROOT, "profiles", name)) as f:
+            return json.load(f)
+    except Exception:
+        return None
+
+
+# ---------------------------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.sw_power_cap,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown")
+
+    def __init__(self, device_index: int):
+        self.samples = []
+        self.proc = None
+        try:
+            uuid = str(torch.cuda.get_device_properties(device_index).uuid)
+            sel = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", sel, f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) == 7:
+                self.samples.append(parts)
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=2)
+        except Exception:
+            self.proc.kill()
+        sm = [float(s[0]) for s in self.samples if s[0].replace(".", "").isdigit()]
+        mx = [float(s[1]) for s in self.samples if s[1].replace(".", "").isdigit()]
+        names = ["sw_power_cap", "hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown"]
+        reasons = sorted({names[i] for s in self.samples for i in range(4) if s[3 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(self.samples)}
+
+
+# ---------------------------------------------------------------------------------------------
+# distributed helpers (independent replicas; the only collectives are the barrier and the max)
+# ---------------------------------------------------------------------------------------------
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if torch.cuda.is_available():
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    return rank, world, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(v: float, world: int) -> float:
+    if world == 1:
+        return v
+    import torch.distributed as dist
+    t = torch.tensor([v], dtype=torch.float64, device="cuda" if torch.cuda.is_available() else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------------------------------------
+# CPU oracle timed on the host cores (reported baseline / reference arm)
+# ---------------------------------------------------------------------------------------------
+
+class OracleRunner:
+    """The oracle's online path on a bounded token sample, weights prepared (untimed) once."""
+
+    def __init__(self, L: WL.Layer, kind: str, k: int, sample_tokens: int):
+        import oracle as O
+        self.O = O
+        cfg = L.cfg
+        self.X = L.x_eval.values[:sample_tokens].astype(np.float64)
+        n_cal = max(1, int(round(sample_tokens * cfg.n_calib / cfg.n_eval)))
+        self.Xc = L.x_calib.values[:n_cal].astype(np.float64)
+        self.k = k
+        self.prep = O.prepare_weights(L.W.values, kind, k, X_calib=L.x_calib.values, signs=L.rht_signs)
+        self.y_ref = O.linear(self.X, L.W.values)
+        self.sample = sample_tokens
+        self.n_cal = n_cal
+
+    def step(self):
+        O = self.O
+        O.calib_cov_block_sums(self.Xc, self.k)
+        ac = O.transform_quantize_act(self.X, self.prep.T)
+        _, y_hat = O.w4a4_linear(ac.qx, ac.sx, self.prep.qw, self.prep.sw)
+        return O.sqnr_sums(self.y_ref, y_hat)
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count()
+
+
+def run_cpu_baseline(L, kind, k, seconds):
+    sample = min(L.cfg.n_eval, 128)
+    r = OracleRunner(L, kind, k, sample)
+    r.step()
+    t0 = time.perf_counter()
+    reps = 0
+    while True:
+        r.step()
+        reps += 1
+        if time.perf_counter() - t0 >= seconds:
+            break
+    dt = time.perf_counter() - t0
+    return {"value": sample * reps / dt, "unit": "tokens/s", "cores": cpu_cores(), "kind": "oracle",
+            "sample": f"{sample} of {L.cfg.n_eval} evaluation tokens (+{r.n_cal} calibration tokens) of "
+                      f"{L.cfg.name}, {reps} repetitions in {dt:.1f} s; weights prepared untimed"}
+
+
+def reference_arm(args, rank, world):
+    if rank != 0:
+        return
+    cfg = WL.CONFIGS[args.config]
+    k = args.k or cfg.k
+    L = WL.make_layer(cfg)
+    sample = min(cfg.n_eval, 128)
+    r = OracleRunner(L, args.kind, k, sample)
+    for _ in range(args.warmup):
+        r.step()
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        r.step()
+        times.append(time.perf_counter() - t0)
+    ms = 1e3 * statistics.mean(times)
+    value = sample / (ms / 1e3)
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": cfg.name, "n_tokens_per_step": sample, "d_in": cfg.d_in, "d_out": cfg.d_out,
+                       "k": k, "transform": args.kind},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cpu_cores(), "kind": "oracle",
+                             "sample": f"{sample} of {cfg.n_eval} evaluation tokens per step of {cfg.name}"},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------------------------
+
+def to_dev(t: WL.Tensor, dev):
+    if t.dtype == "f32":
+        return torch.from_numpy(np.ascontiguousarray(t.raw)).to(dev)
+    return torch.from_numpy(np.ascontiguousarray(t.raw).view(np.int16)).view(torch.bfloat16).to(dev)
+
+
+def ours_arm(args, rank, world, local):
+    import paper_2603_04359_gb300 as cat
+    cat.load_library()
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    cfg = WL.CONFIGS[args.config]
+    k = args.k or cfg.k
+    L = WL.make_layer(cfg)
+    x, W, xc = to_dev(L.x_eval, dev), to_dev(L.W, dev), to_dev(L.x_calib, dev)
+    n, d_in, d_out = cfg.n_eval, cfg.d_in, cfg.d_out
+
+    # offline: calibration statistics and weight preparation
+    sigma = cat.cat_calib_cov(xc, k)
+    T, Wq, sw = cat.cat_quantize_weights(W, k, args.kind, sigma_x=sigma, n_calib=cfg.n_calib,
+                                         rht_signs=L.rht_signs if args.kind == "rht" else None)
+    torch.backends.cuda.matmul.allow_tf32 = False
+    y_ref = (x.float() @ W.float().t()).contiguous()
+    del W
+    xq = torch.empty((n, d_in // 2), dtype=torch.uint8, device=dev)
+    sx = torch.empty((n,), dtype=torch.float32, device=dev)
+    y = torch.empty((n, d_out), dtype=torch.float32, device=dev)
+    out3 = torch.empty((3,), dtype=torch.float64, device=dev)
+    flush = torch.empty((L2_FLUSH_BYTES,), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+
+    def step(gemm_events=None):
+        cat.cat_calib_cov(xc, k, out=sigma)
+        cat.cat_transform_quantize_act(x, T, k, xq=xq, x_scale=sx)
+        if gemm_events:
+            gemm_events[0].record(stream)
+        cat.cat_w4a4_linear(xq, sx, Wq, sw, y=y)
+        if gemm_events:
+            gemm_events[1].record(stream)
+        cat.cat_sqnr(y_ref, y, out=out3)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    st, word = cat.cat_device_status(dev)
+    if st != 0:
+        raise RuntimeError(f"device status {st} ({word:#x}) after warm-up")
+
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local)
+    marks = []
+    for i in range(args.steps):
+        flush.fill_(i & 0xFF)                                # L2 flush, outside the timed events
+        s0, s1, g0, g1 = ev(), ev(), ev(), ev()
+        s0.record(stream)
+        step((g0, g1))
+        s1.record(stream)
+        marks.append((s0, s1, g0, g1))
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    barrier(world)
+    step_ms = statistics.mean(a.elapsed_time(b) for a, b, _, _ in marks)
+    gemm_ms = statistics.mean(c.elapsed_time(d) for _, _, c, d in marks)
+    sqnr_db = float(out3[2].item())
+    step_ms_max = max_over_ranks(step_ms, world)
+
+    # end to end through the same calls with host buffers: inputs copied in, output copied out
+    e2e = None
+    if not args.no_e2e:
+        x_h = x.cpu().pin_memory()
+        xc_h = xc.cpu().pin_memory()
+        yref_h = y_ref.cpu().pin_memory()
+        y_h = torch.empty_like(y, device="cpu").pin_memory()
+        o3_h = torch.empty((3,), dtype=torch.float64).pin_memory()
+        h2d = x_h.numel() * x_h.element_size() + xc_h.numel() * xc_h.element_size() + yref_h.numel() * 4
+        d2h = y_h.numel() * 4 + 3 * 8
+
+        def e2e_step():
+            x.copy_(x_h, non_blocking=True)
+            xc.copy_(xc_h, non_blocking=True)
+            y_ref.copy_(yref_h, non_blocking=True)
+            step()
+            y_h.copy_(y, non_blocking=True)
+            o3_h.copy_(out3, non_blocking=True)
+
+        for _ in range(2):
+            e2e_step()
+        torch.cuda.synchronize()
+        barrier(world)
+        em = []
+        for i in range(args.steps):
+            flush.fill_(i & 0xFF)
+            a, b = ev(), ev()
+            a.record(stream)
+            e2e_step()
+            b.record(stream)
+            em.append((a, b))
+        torch.cuda.synchronize()
+        barrier(world)
+        e2e_ms = max_over_ranks(statistics.mean(a.elapsed_time(b) for a, b in em), world)
+        e2e = {"value": world * n / (e2e_ms / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
+               "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms}
+
+    st, word = cat.cat_device_status(dev)
+    if st != 0:
+        raise RuntimeError(f"device status {st} ({word:#x}) after timing")
+
+    if rank != 0:
+        return
+    peaks = measured_peaks()
+    fp8_peak = peaks["bf16_tflops"] * FP8_PER_BF16
+    gemm_tflops = 2.0 * n * d_in * d_out / (gemm_ms / 1e3) / 1e12
+    traffic = None
+    tr = committed_json("traffic.json")
+    if tr and tr.get("workload") == cfg.name and tr.get("kernel_rev") == "w4a4_gemm_tc_v1":
+        traffic = tr.get("dram_bytes_per_launch")
+    int8 = committed_json("peaks_gb300.json") or {}
+    line = {
+        "metric": METRIC, "value": world * n / (step_ms_max / 1e3), "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms_max, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int4", "data": "synthetic",
+        "config": {"workload": cfg.name, "n_tokens": n, "d_in": d_in, "d_out": d_out, "k": k, "n_calib": cfg.n_calib,
+                   "transform": args.kind, "input_dtype": cfg.dtype, "parallelism": f"replicas x{world}",
+                   "l2": "flushed between timed steps (256 MiB write)"},
+        "roofline": {"bound": "tensor", "achieved": gemm_tflops, "peak": fp8_peak, "unit": "TFLOP/s",
+                     "frac": gemm_tflops / fp8_peak, "traffic": traffic,
+                     "kernel": "w4a4_gemm_tc (cat_w4a4_linear)",
+                     "peak_source": f"{peaks['source']} bf16 {peaks['bf16_tflops']} TFLOP/s x {FP8_PER_BF16} "
+                                    "(FP8 engine, nominal FP8/BF16 ratio)"},
+        "sqnr_db": sqnr_db, "gemm_ms": gemm_ms, "effective_tops": gemm_tflops,
+        "gpu_launches": LAUNCHES_PER_STEP * args.steps, "clocks": clk,
+    }
+    if int8.get("int8_tops"):
+        line["int8_peak"] = {"tops": int8["int8_tops"], "frac": gemm_tflops / int8["int8_tops"],
+                             "source": int8.get("int8_source", "")}
+    if e2e:
+        line["e2e"] = e2e
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = run_cpu_baseline(L, args.kind, k, args.cpu_seconds)
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    rank, world, local = dist_setup()
+    if args.impl == "reference":
+        reference_arm(args, rank, world)
+    else:
+        ours_arm(args, rank, world, local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

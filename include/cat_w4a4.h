@@ -1,0 +1,178 @@
+/*
+ * cat_w4a4.h -- C ABI of the block Concentration-Alignment Transform (CAT) W4A4 linear layer
+ * on NVIDIA GB300 (sm_103a).
+ *
+ * The layer follows "Dissecting Quantization Error: A Concentration-Alignment Perspective":
+ *   y = W x = (W T^{-1}) (T x) ~ Q(W T^{-1}) Q(T x)                      (Sec. 3, Eq. 5)
+ * with a block-diagonal transform T = H_k M_block (Sec. 4, Eq. 10), where every k x k block
+ * M_b = (Sigma_w_b # Sigma_x_b^{-1})^{1/2} maximises alignment on its own sub-problem (Eq. 7),
+ * Sigma_x = E[x x^T] over calibration tokens and Sigma_w = W^T W.  Activations are quantized
+ * per token and weights per output channel with a symmetric uniform round-to-nearest INT4
+ * quantizer (Lemma 2 range, Sec. 6 set-up); the layer's quality is its SQNR (Sec. 2, Eq. 1).
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ *  - Matrices are row-major and dense.  A token is a row of x [n][d_in]; W is [d_out][d_in];
+ *    y is [n][d_out] float32.  T acts on activations (x' = T x); T_blocks[b] is the k x k block
+ *    acting on channels b*k .. b*k+k-1, stored row-major ([d_in/k][k][k] float32).
+ *  - Unless a parameter says "host", pointers are device pointers owned by the caller; the
+ *    library never frees them.  Device pointers must be 16-byte aligned.
+ *  - Calls are asynchronous on `stream` (NULL = the legacy default stream) unless stated.
+ *    Launch failures return CAT_ERR_CUDA.  Conditions detected on the device (a bounded wait
+ *    that gave up, a non-finite input) are recorded in a device status word that
+ *    cat_device_status() reads; kernels never trap.
+ *  - Arguments are validated on the host before anything is launched; an invalid call returns
+ *    an error code, launches nothing and touches no output.  cat_last_error() gives a message.
+ *  - Shapes: d_in % 32 == 0 (a packed row is a whole number of 16-byte chunks); k is one of
+ *    16, 32, 64, 128, 256 and divides d_in; n, d_out >= 1 (n == 0 is accepted and does nothing).
+ *  - Thread safety: calls keep no host state between calls except the error message of the
+ *    calling thread.
+ *
+ * INT4 code format ("SM4x8")
+ * --------------------------
+ *  Codes q are integers in [-7, 7] (the restricted symmetric INT4 grid: step s = max|v| / 7,
+ *  round half to even, so the largest magnitude maps to +-7 and zero is exact).  Each code is a
+ *  4-bit sign-magnitude value: sign s = (q < 0), magnitude m = |q| (3 bits).  A row of d_in codes
+ *  occupies d_in/2 bytes; every 8 consecutive codes e0..e7 of a row (along d_in) form one
+ *  little-endian 32-bit word w whose byte i (i = 0..3) holds
+ *      bits 0-2: m(e_i)     bit 7: s(e_i)     bits 4-6: m(e_{4+i})     bit 3: s(e_{4+(i+3)%4}).
+ *  With this layout  (w & 0x87878787)  and  (rotr32(w, 4) & 0x87878787)  are, byte for byte,
+ *  the FP8 E4M3 encodings (s << 7 | m) of e0..e3 and e4..e7, i.e. the subnormal values
+ *  (-1)^s * m * 2^-9.  The GEMM feeds these bytes to the FP8 tensor cores and rescales the
+ *  exactly accumulated result by 2^18.
+ */
+#ifndef CAT_W4A4_H
+#define CAT_W4A4_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t. */
+typedef struct CUstream_st* cat_stream_t;
+
+typedef enum {
+  CAT_OK = 0,
+  CAT_ERR_INVALID_ARG = 1,   /* NULL pointer, unknown enum value, negative size */
+  CAT_ERR_SHAPE = 2,         /* sizes violate the shape rules above */
+  CAT_ERR_ALIGNMENT = 3,     /* a device pointer is not 16-byte aligned */
+  CAT_ERR_NUMERIC = 4,       /* non-finite input, or a calibration block that is not positive definite */
+  CAT_ERR_UNSUPPORTED = 5,   /* valid request this build does not implement (e.g. no sm_103a device) */
+  CAT_ERR_CUDA = 6,          /* a CUDA runtime call failed */
+  CAT_ERR_TIMEOUT = 7        /* a bounded device-side wait gave up */
+} cat_status;
+
+typedef enum { CAT_F32 = 0, CAT_BF16 = 1 } cat_dtype;
+
+typedef enum {
+  CAT_T_IDENTITY = 0,        /* T = I: plain W4A4 RTN */
+  CAT_T_RHT = 1,             /* T_b = H_k Diag(sigma_b): randomized Hadamard rotation, signs given by the caller */
+  CAT_T_CAT = 2              /* T_b = H_k M_b, M_b = (Sigma_w_b # Sigma_x_b^{-1})^{1/2} (Sec. 4, Eq. 7, Eq. 10) */
+} cat_tkind;
+
+/* Human-readable name of a status code (static string). */
+const char* cat_status_string(cat_status status);
+
+/* Message of the last error returned to the calling thread ("" if none). */
+const char* cat_last_error(void);
+
+/* Library version: major * 10000 + minor * 100 + patch. */
+int cat_version(void);
+
+/*
+ * cat_calib_cov -- calibration autocorrelation blocks (Sec. 4: Sigma_x = E[x x^T]; Eq. 10 uses its
+ * k x k diagonal blocks).
+ *   x            device [n][d] in `dtype` (calibration tokens, or weight rows for Sigma_w = W^T W).
+ *   sigma_blocks device [d/k][k][k] float64: receives sum_t x_{t,b} x_{t,b}^T for every block b
+ *                (a plain sum over tokens: divide by the token count for E[x x^T]).  With
+ *                accumulate == 0 the buffer is overwritten, otherwise the sums are added to it, so
+ *                calibration sets larger than one batch can be streamed through.
+ * The products of bf16 inputs are exact in fp32; the sums are carried in compensated (double-float)
+ * fp32 arithmetic and stored in float64, so they match a float64 accumulation to about 1e-12.
+ */
+cat_status cat_calib_cov(const void* x, cat_dtype dtype, int64_t n, int64_t d, int32_t k,
+                         double* sigma_blocks, int accumulate, cat_stream_t stream);
+
+/*
+ * cat_quantize_weights -- offline weight preparation (Sec. 3 Eq. 5: W' = W T^{-1}; Sec. 4 Eq. 7
+ * and Eq. 10: the block transform; Sec. 6: per-output-channel symmetric RTN).
+ *   W              device [d_out][d_in] in `dtype`.
+ *   kind           transform family.
+ *   sigma_x_blocks device [d_in/k][k][k] float64 sums from cat_calib_cov (CAT only; else may be NULL).
+ *   n_calib        number of tokens behind sigma_x_blocks (CAT only, >= 1).
+ *   rht_signs      HOST [d_in] float32, each +1 or -1 (RHT only; else may be NULL).
+ *   T_blocks       out, device [d_in/k][k][k] float32: the online activation transform T.
+ *   Wq             out, device [d_out][d_in/2] bytes: SM4x8 codes of W T^{-1}.
+ *   w_scale        out, device [d_out] float32: per-output-channel step s_w = max_i |W'_{o,i}| / 7.
+ * Synchronous: it reads the calibration sums back, builds T and T^{-1} in float64 on the host
+ * (per block, in parallel over host threads), uploads them, and runs the weight kernels; it
+ * returns after the outputs are written.  It allocates and frees its own temporaries.
+ * Returns CAT_ERR_NUMERIC if a Sigma_x or Sigma_w block is not positive definite.
+ */
+cat_status cat_quantize_weights(const void* W, cat_dtype dtype, int64_t d_out, int64_t d_in, int32_t k,
+                                cat_tkind kind, const double* sigma_x_blocks, int64_t n_calib,
+                                const float* rht_signs, float* T_blocks, uint8_t* Wq, float* w_scale,
+                                cat_stream_t stream);
+
+/*
+ * cat_build_transform_host -- the host part of cat_quantize_weights, exposed for inspection: the
+ * block transform T and its inverse in float64 (Sec. 4, Eq. 7 and Eq. 10).  All pointers are HOST.
+ *   sigma_x_blocks [d_in/k][k][k] sums over n_calib tokens (CAT only); sigma_w_blocks [d_in/k][k][k]
+ *   (= diagonal blocks of W^T W, CAT only); rht_signs [d_in] (RHT only).
+ *   T_out, Tinv_out [d_in/k][k][k] float64.
+ * Runs on the calling thread's host cores only; no CUDA call is made.
+ */
+cat_status cat_build_transform_host(cat_tkind kind, int64_t d_in, int32_t k, const double* sigma_x_blocks,
+                                    int64_t n_calib, const double* sigma_w_blocks, const float* rht_signs,
+                                    double* T_out, double* Tinv_out);
+
+/*
+ * cat_transform_quantize_act -- online activation path (Sec. 3 Eq. 5: x' = T x; Lemma 2 symmetric
+ * range; Sec. 6: dynamic per-token quantization, round to nearest).
+ *   x        device [n][d_in] in `dtype`.
+ *   T_blocks device [d_in/k][k][k] float32 (from cat_quantize_weights).
+ *   xq       out, device [n][d_in/2] bytes: SM4x8 codes of x' = T x.
+ *   x_scale  out, device [n] float32: per-token step s_x = max_i |x'_i| / 7 (0 for an all-zero token).
+ * Codes are q = clamp(rint(x'_i * (7 / max|x'|)), -7, 7), x' accumulated in float32.
+ */
+cat_status cat_transform_quantize_act(const void* x, cat_dtype dtype, int64_t n, int64_t d_in, int32_t k,
+                                      const float* T_blocks, uint8_t* xq, float* x_scale,
+                                      cat_stream_t stream);
+
+/*
+ * cat_w4a4_linear -- integer GEMM and dequantization (Sec. 3 Eq. 5: y ~ Q(W T^{-1}) Q(T x)).
+ *   xq [n][d_in/2], x_scale [n]; Wq [d_out][d_in/2], w_scale [d_out]  (SM4x8 codes and steps).
+ *   y        out, device [n][d_out] float32: y[t][o] = acc[t][o] * x_scale[t] * w_scale[o], with
+ *            acc[t][o] = sum_i q_x[t][i] q_w[o][i] computed exactly (FP8 tensor cores, fp32
+ *            accumulators holding integers |acc| <= 49 * d_in < 2^24).
+ *   acc_out  optional out (NULL to skip), device [n][d_out] int32: the integer accumulators.
+ * Exactness needs 49 * d_in < 2^24, so d_in <= 262144 is required (CAT_ERR_SHAPE otherwise).
+ */
+cat_status cat_w4a4_linear(const uint8_t* xq, const float* x_scale, const uint8_t* Wq, const float* w_scale,
+                           int64_t n, int64_t d_in, int64_t d_out, float* y, int32_t* acc_out,
+                           cat_stream_t stream);
+
+/*
+ * cat_sqnr -- signal-to-quantization-noise ratio of the layer output (Sec. 2, Eq. 1).
+ *   y_ref, y_hat device [numel] float32 (full-precision and quantized outputs).
+ *   out3         out, device [3] float64: { sum y_ref^2, sum (y_ref - y_hat)^2, 10 log10(ratio) dB }.
+ * Squares are summed in fp32 over short runs and the run sums in float64.
+ */
+cat_status cat_sqnr(const float* y_ref, const float* y_hat, int64_t numel, double* out3, cat_stream_t stream);
+
+/*
+ * cat_device_status -- synchronizes `stream`, then reads and clears the device status word.
+ * Returns CAT_OK, CAT_ERR_TIMEOUT (a bounded wait in a kernel gave up and the kernel returned
+ * early; its outputs are undefined) or CAT_ERR_NUMERIC (a kernel met a non-finite value; the
+ * affected codes are 0).  `detail` (HOST, may be NULL) receives the raw status word.
+ */
+cat_status cat_device_status(cat_stream_t stream, uint32_t* detail);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CAT_W4A4_H */

@@ -115,18 +115,22 @@ def calib_cov_block_sums(X: np.ndarray, k: int) -> np.ndarray:
     the number of tokens gives the uncentered autocorrelation blocks of ``Sigma_x``."""
     X = np.asarray(X, dtype=np.float64)
     n, d = X.shape
-    nb = d // k
-    Xb = X.reshape(n, nb, k)
-    return np.einsum("tbi,tbj->bij", Xb, Xb)
+    out = np.empty((d // k, k, k))
+    for b in range(d // k):
+        Xb = X[:, b * k:(b + 1) * k]
+        out[b] = Xb.T @ Xb
+    return out
 
 
 def weight_autocorr_blocks(W: np.ndarray, k: int) -> np.ndarray:
     """Diagonal k x k blocks of ``Sigma_w = W^T W``: [d/k, k, k]."""
     W = np.asarray(W, dtype=np.float64)
     d_out, d = W.shape
-    nb = d // k
-    Wb = W.reshape(d_out, nb, k)
-    return np.einsum("obi,obj->bij", Wb, Wb)
+    out = np.empty((d // k, k, k))
+    for b in range(d // k):
+        Wb = W[:, b * k:(b + 1) * k]
+        out[b] = Wb.T @ Wb
+    return out
 
 
 # ---------------------------------------------------------------------------------------------

@@ -1,0 +1,206 @@
+"""Block Concentration-Alignment Transform (CAT) W4A4 linear layer on GB300 (sm_103a).
+
+A thin ctypes binding of the C ABI in ``include/cat_w4a4.h``: every function below has the name
+of the C entry point it calls, takes torch tensors, allocates outputs with torch on the tensors'
+device when none are given, passes raw pointers and the current CUDA stream, and raises
+``CatError`` on a non-zero status.  All arithmetic runs in the library's CUDA kernels (or, for
+``cat_build_transform_host``, in its host code); there is no fallback path.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+from typing import Optional, Tuple
+
+import numpy as np
+import torch
+
+__all__ = [
+    "CatError", "library_path", "load_library", "exported_symbols",
+    "cat_calib_cov", "cat_quantize_weights", "cat_build_transform_host", "cat_transform_quantize_act",
+    "cat_w4a4_linear", "cat_sqnr", "cat_device_status", "cat_version", "KIND",
+]
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_LIB_PATH = os.path.join(_HERE, "libcatw4a4.so")
+_HEADER = os.path.join(os.path.dirname(_HERE), "include", "cat_w4a4.h")
+_lib: Optional[ctypes.CDLL] = None
+
+KIND = {"identity": 0, "rht": 1, "cat": 2}
+_DTYPE = {torch.float32: 0, torch.bfloat16: 1}
+_STATUS = {0: "CAT_OK", 1: "CAT_ERR_INVALID_ARG", 2: "CAT_ERR_SHAPE", 3: "CAT_ERR_ALIGNMENT", 4: "CAT_ERR_NUMERIC",
+           5: "CAT_ERR_UNSUPPORTED", 6: "CAT_ERR_CUDA", 7: "CAT_ERR_TIMEOUT"}
+
+
+class CatError(RuntimeError):
+    def __init__(self, func: str, status: int, message: str):
+        super().__init__(f"{func}: {_STATUS.get(status, status)}: {message}")
+        self.status = status
+
+
+def library_path() -> str:
+    return _LIB_PATH
+
+
+def load_library() -> ctypes.CDLL:
+    """Load ``libcatw4a4.so`` (built in-tree by ``paper_2603_04359_gb300.build``); fail loudly if absent."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(_LIB_PATH):
+        raise ImportError(f"{_LIB_PATH} is missing: build it with `python -c 'import __graft_entry__ as g; g.build()'`")
+    lib = ctypes.CDLL(_LIB_PATH)
+    P, I64, I32, I = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_int
+    sigs = {
+        "cat_status_string": ([I], ctypes.c_char_p),
+        "cat_last_error": ([], ctypes.c_char_p),
+        "cat_version": ([], I),
+        "cat_calib_cov": ([P, I, I64, I64, I32, P, I, P], I),
+        "cat_quantize_weights": ([P, I, I64, I64, I32, I, P, I64, P, P, P, P, P], I),
+        "cat_build_transform_host": ([I, I64, I32, P, I64, P, P, P, P], I),
+        "cat_transform_quantize_act": ([P, I, I64, I64, I32, P, P, P, P], I),
+        "cat_w4a4_linear": ([P, P, P, P, I64, I64, I64, P, P, P], I),
+        "cat_sqnr": ([P, P, I64, P, P], I),
+        "cat_device_status": ([P, P], I),
+    }
+    for name, (args, res) in sigs.items():
+        f = getattr(lib, name)
+        f.argtypes = args
+        f.restype = res
+    _lib = lib
+    return lib
+
+
+def exported_symbols() -> list:
+    """Names of the entry points declared in ``include/cat_w4a4.h``."""
+    with open(_HEADER) as f:
+        text = f.read()
+    return sorted(set(re.findall(r"^\s*(?:cat_status|const char\*|int)\s+(cat_\w+)\s*\(", text, re.M)))
+
+
+def _check(func: str, status: int) -> None:
+    if status != 0:
+        msg = load_library().cat_last_error().decode()
+        raise CatError(func, status, msg)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(device: torch.device):
+    return ctypes.c_void_p(torch.cuda.current_stream(device).cuda_stream)
+
+
+def _dtype(t: torch.Tensor) -> int:
+    if t.dtype not in _DTYPE:
+        raise TypeError(f"unsupported dtype {t.dtype}; expected float32 or bfloat16")
+    return _DTYPE[t.dtype]
+
+
+def _need(t: torch.Tensor, name: str) -> None:
+    if not (t.is_cuda and t.is_contiguous()):
+        raise ValueError(f"{name} must be a contiguous CUDA tensor")
+
+
+def cat_version() -> int:
+    return int(load_library().cat_version())
+
+
+def cat_calib_cov(x: torch.Tensor, k: int, out: Optional[torch.Tensor] = None, accumulate: bool = False) -> torch.Tensor:
+    """Sums of x_b x_b^T over tokens for every k x k diagonal block: float64 [d/k, k, k]."""
+    _need(x, "x")
+    n, d = x.shape
+    if out is None:
+        out = torch.empty((d // k, k, k), dtype=torch.float64, device=x.device)
+    _check("cat_calib_cov", load_library().cat_calib_cov(_ptr(x), _dtype(x), n, d, k, _ptr(out), int(accumulate),
+                                                         _stream(x.device)))
+    return out
+
+
+def cat_quantize_weights(W: torch.Tensor, k: int, kind: str, sigma_x: Optional[torch.Tensor] = None, n_calib: int = 0,
+                         rht_signs=None) -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
+    """Offline weight preparation.  Returns (T_blocks float32 [d_in/k,k,k], Wq uint8 [d_out, d_in/2],
+    w_scale float32 [d_out])."""
+    _need(W, "W")
+    d_out, d_in = W.shape
+    dev = W.device
+    T = torch.empty((d_in // k, k, k), dtype=torch.float32, device=dev)
+    Wq = torch.empty((d_out, d_in // 2), dtype=torch.uint8, device=dev)
+    sw = torch.empty((d_out,), dtype=torch.float32, device=dev)
+    signs = None
+    if rht_signs is not None:
+        signs = np.ascontiguousarray(np.asarray(rht_signs, dtype=np.float32))
+    if sigma_x is not None:
+        _need(sigma_x, "sigma_x")
+    st = load_library().cat_quantize_weights(
+        _ptr(W), _dtype(W), d_out, d_in, k, KIND[kind], _ptr(sigma_x), int(n_calib),
+        None if signs is None else signs.ctypes.data_as(ctypes.c_void_p), _ptr(T), _ptr(Wq), _ptr(sw), _stream(dev))
+    _check("cat_quantize_weights", st)
+    return T, Wq, sw
+
+
+def cat_build_transform_host(kind: str, d_in: int, k: int, sigma_x: Optional[np.ndarray] = None, n_calib: int = 0,
+                             sigma_w: Optional[np.ndarray] = None, rht_signs=None) -> Tuple[np.ndarray, np.ndarray]:
+    """Host float64 block transform (T, T^{-1}), each [d_in/k, k, k]."""
+    nb = d_in // k
+    T = np.zeros((nb, k, k), dtype=np.float64)
+    Ti = np.zeros((nb, k, k), dtype=np.float64)
+    sx = None if sigma_x is None else np.ascontiguousarray(sigma_x, dtype=np.float64)
+    sw = None if sigma_w is None else np.ascontiguousarray(sigma_w, dtype=np.float64)
+    sg = None if rht_signs is None else np.ascontiguousarray(rht_signs, dtype=np.float32)
+    vp = lambda a: None if a is None else a.ctypes.data_as(ctypes.c_void_p)  # noqa: E731
+    st = load_library().cat_build_transform_host(KIND[kind], d_in, k, vp(sx), int(n_calib), vp(sw), vp(sg), vp(T),
+                                                 vp(Ti))
+    _check("cat_build_transform_host", st)
+    return T, Ti
+
+
+def cat_transform_quantize_act(x: torch.Tensor, T_blocks: torch.Tensor, k: int, xq: Optional[torch.Tensor] = None,
+                               x_scale: Optional[torch.Tensor] = None) -> Tuple[torch.Tensor, torch.Tensor]:
+    """x' = T x, per-token INT4 codes (SM4x8 uint8 [n, d_in/2]) and steps (float32 [n])."""
+    _need(x, "x")
+    _need(T_blocks, "T_blocks")
+    n, d_in = x.shape
+    if xq is None:
+        xq = torch.empty((n, d_in // 2), dtype=torch.uint8, device=x.device)
+    if x_scale is None:
+        x_scale = torch.empty((n,), dtype=torch.float32, device=x.device)
+    _check("cat_transform_quantize_act", load_library().cat_transform_quantize_act(
+        _ptr(x), _dtype(x), n, d_in, k, _ptr(T_blocks), _ptr(xq), _ptr(x_scale), _stream(x.device)))
+    return xq, x_scale
+
+
+def cat_w4a4_linear(xq: torch.Tensor, x_scale: torch.Tensor, Wq: torch.Tensor, w_scale: torch.Tensor,
+                    y: Optional[torch.Tensor] = None, acc_out: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """y[t, o] = (sum_i q_x q_w) * s_x[t] * s_w[o] (float32 [n, d_out]); optionally the int32 accumulators."""
+    for t, name in ((xq, "xq"), (x_scale, "x_scale"), (Wq, "Wq"), (w_scale, "w_scale")):
+        _need(t, name)
+    n, half = xq.shape
+    d_out = Wq.shape[0]
+    if y is None:
+        y = torch.empty((n, d_out), dtype=torch.float32, device=xq.device)
+    _check("cat_w4a4_linear", load_library().cat_w4a4_linear(
+        _ptr(xq), _ptr(x_scale), _ptr(Wq), _ptr(w_scale), n, 2 * half, d_out, _ptr(y), _ptr(acc_out),
+        _stream(xq.device)))
+    return y
+
+
+def cat_sqnr(y_ref: torch.Tensor, y_hat: torch.Tensor, out: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """float64 [3] on the device: (sum y^2, sum (y - y_hat)^2, SQNR dB)."""
+    _need(y_ref, "y_ref")
+    _need(y_hat, "y_hat")
+    if out is None:
+        out = torch.empty((3,), dtype=torch.float64, device=y_ref.device)
+    _check("cat_sqnr", load_library().cat_sqnr(_ptr(y_ref), _ptr(y_hat), y_ref.numel(), _ptr(out),
+                                               _stream(y_ref.device)))
+    return out
+
+
+def cat_device_status(device: Optional[torch.device] = None) -> Tuple[int, int]:
+    """Synchronize the current stream and return (status, raw status word); clears the word."""
+    dev = device or torch.device("cuda", torch.cuda.current_device())
+    detail = ctypes.c_uint32(0)
+    st = load_library().cat_device_status(_stream(dev), ctypes.byref(detail))
+    return int(st), int(detail.value)

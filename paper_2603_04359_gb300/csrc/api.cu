@@ -1,0 +1,288 @@
+// C ABI of the CAT W4A4 library (declarations and contracts: include/cat_w4a4.h).
+// Host-side validation, dispatch to the kernels and the per-device status word.
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "../../include/cat_w4a4.h"
+#include "common.cuh"
+#include "transform_host.h"
+
+namespace cat {
+cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
+                                int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, uint32_t* status,
+                                cudaStream_t stream);
+cudaError_t launch_w4a4_gemm_decode(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
+                                    int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, cudaStream_t stream);
+}  // namespace cat
+
+namespace {
+
+constexpr int kVersion = 10000;        // 1.0.0
+constexpr int64_t kMaxDecodeTokens = 32;   // n <= 32: weight-streaming kernel; else tcgen05 tiles
+constexpr int64_t kMaxDin = 262144;    // 49 * d_in < 2^24 keeps fp32 accumulation exact
+
+// Device status word (one per device that loads the library).
+__device__ uint32_t g_device_status;
+
+thread_local std::string t_last_error;
+
+cat_status fail(cat_status s, const std::string& msg) {
+  t_last_error = msg;
+  return s;
+}
+
+cat_status ok() {
+  t_last_error.clear();
+  return CAT_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+bool valid_k(int32_t k) { return k == 16 || k == 32 || k == 64 || k == 128 || k == 256; }
+
+cat_status cuda_fail(cudaError_t e, const char* where) {
+  return fail(CAT_ERR_CUDA, std::string(where) + ": " + cudaGetErrorString(e));
+}
+
+// Address of this device's status word (cached per device).
+uint32_t* status_word(cudaError_t* err) {
+  static std::mutex mu;
+  static uint32_t* cache[64] = {nullptr};
+  int dev = 0;
+  *err = cudaGetDevice(&dev);
+  if (*err != cudaSuccess) return nullptr;
+  if (dev < 0 || dev >= 64) {
+    *err = cudaErrorInvalidDevice;
+    return nullptr;
+  }
+  std::lock_guard<std::mutex> lock(mu);
+  if (!cache[dev]) {
+    void* p = nullptr;
+    *err = cudaGetSymbolAddress(&p, g_device_status);
+    if (*err != cudaSuccess) return nullptr;
+    cache[dev] = static_cast<uint32_t*>(p);
+  }
+  return cache[dev];
+}
+
+// The kernels are built for sm_103a only.
+cat_status check_device() {
+  int dev = 0, major = 0, minor = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if ((e = cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev)) != cudaSuccess)
+    return cuda_fail(e, "cudaDeviceGetAttribute");
+  if ((e = cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev)) != cudaSuccess)
+    return cuda_fail(e, "cudaDeviceGetAttribute");
+  if (major != 10 || minor != 3)
+    return fail(CAT_ERR_UNSUPPORTED, "this library is built for sm_103a (GB300); device is sm_" +
+                                         std::to_string(major) + std::to_string(minor));
+  return CAT_OK;
+}
+
+cat_status check_din(int64_t d_in) {
+  if (d_in <= 0 || d_in % 32 != 0) return fail(CAT_ERR_SHAPE, "d_in must be a positive multiple of 32");
+  if (d_in > kMaxDin) return fail(CAT_ERR_SHAPE, "d_in exceeds 262144 (exact fp32 accumulation bound)");
+  return CAT_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* cat_status_string(cat_status status) {
+  switch (status) {
+    case CAT_OK: return "CAT_OK";
+    case CAT_ERR_INVALID_ARG: return "CAT_ERR_INVALID_ARG";
+    case CAT_ERR_SHAPE: return "CAT_ERR_SHAPE";
+    case CAT_ERR_ALIGNMENT: return "CAT_ERR_ALIGNMENT";
+    case CAT_ERR_NUMERIC: return "CAT_ERR_NUMERIC";
+    case CAT_ERR_UNSUPPORTED: return "CAT_ERR_UNSUPPORTED";
+    case CAT_ERR_CUDA: return "CAT_ERR_CUDA";
+    case CAT_ERR_TIMEOUT: return "CAT_ERR_TIMEOUT";
+  }
+  return "CAT_ERR_UNKNOWN";
+}
+
+const char* cat_last_error(void) { return t_last_error.c_str(); }
+
+int cat_version(void) { return kVersion; }
+
+cat_status cat_calib_cov(const void* x, cat_dtype dtype, int64_t n, int64_t d, int32_t k, double* sigma_blocks,
+                         int accumulate, cat_stream_t stream) {
+  if (dtype != CAT_F32 && dtype != CAT_BF16) return fail(CAT_ERR_INVALID_ARG, "unknown dtype");
+  if (n < 0 || d <= 0) return fail(CAT_ERR_SHAPE, "n must be >= 0 and d > 0");
+  if (!valid_k(k)) return fail(CAT_ERR_SHAPE, "k must be one of 16, 32, 64, 128, 256");
+  if (d % k != 0) return fail(CAT_ERR_SHAPE, "k must divide d");
+  if (!sigma_blocks || (n > 0 && !x)) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(sigma_blocks) || (x && !aligned16(x))) return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  if (d / k > 0x7FFFFFFF) return fail(CAT_ERR_SHAPE, "too many blocks");
+  cat_status st = check_device();
+  if (st != CAT_OK) return st;
+  cudaError_t e = cat::launch_calib_cov(x, (int)dtype, n, d, k, sigma_blocks, accumulate, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cat_calib_cov launch");
+  return ok();
+}
+
+cat_status cat_build_transform_host(cat_tkind kind, int64_t d_in, int32_t k, const double* sigma_x_blocks,
+                                    int64_t n_calib, const double* sigma_w_blocks, const float* rht_signs,
+                                    double* T_out, double* Tinv_out) {
+  if (kind != CAT_T_IDENTITY && kind != CAT_T_RHT && kind != CAT_T_CAT) return fail(CAT_ERR_INVALID_ARG, "unknown kind");
+  if (!valid_k(k)) return fail(CAT_ERR_SHAPE, "k must be one of 16, 32, 64, 128, 256");
+  if (d_in <= 0 || d_in % k != 0) return fail(CAT_ERR_SHAPE, "d_in must be a positive multiple of k");
+  if (!T_out || !Tinv_out) return fail(CAT_ERR_INVALID_ARG, "NULL output");
+  if (kind == CAT_T_RHT) {
+    if (!rht_signs) return fail(CAT_ERR_INVALID_ARG, "RHT needs rht_signs");
+    for (int64_t i = 0; i < d_in; ++i)
+      if (rht_signs[i] != 1.0f && rht_signs[i] != -1.0f) return fail(CAT_ERR_INVALID_ARG, "rht_signs must be +-1");
+  }
+  if (kind == CAT_T_CAT) {
+    if (!sigma_x_blocks || !sigma_w_blocks) return fail(CAT_ERR_INVALID_ARG, "CAT needs sigma_x and sigma_w blocks");
+    if (n_calib < 1) return fail(CAT_ERR_INVALID_ARG, "n_calib must be >= 1");
+    const size_t cnt = (size_t)d_in * (size_t)k;
+    for (size_t i = 0; i < cnt; ++i)
+      if (!std::isfinite(sigma_x_blocks[i]) || !std::isfinite(sigma_w_blocks[i]))
+        return fail(CAT_ERR_NUMERIC, "non-finite calibration statistics");
+  }
+  std::string err;
+  if (cat::build_transform_host((int)kind, d_in, k, sigma_x_blocks, n_calib, sigma_w_blocks, rht_signs, T_out,
+                                Tinv_out, &err) != 0)
+    return fail(CAT_ERR_NUMERIC, err);
+  return ok();
+}
+
+cat_status cat_quantize_weights(const void* W, cat_dtype dtype, int64_t d_out, int64_t d_in, int32_t k,
+                                cat_tkind kind, const double* sigma_x_blocks, int64_t n_calib,
+                                const float* rht_signs, float* T_blocks, uint8_t* Wq, float* w_scale,
+                                cat_stream_t stream) {
+  if (dtype != CAT_F32 && dtype != CAT_BF16) return fail(CAT_ERR_INVALID_ARG, "unknown dtype");
+  if (kind != CAT_T_IDENTITY && kind != CAT_T_RHT && kind != CAT_T_CAT) return fail(CAT_ERR_INVALID_ARG, "unknown kind");
+  if (d_out <= 0) return fail(CAT_ERR_SHAPE, "d_out must be >= 1");
+  cat_status st = check_din(d_in);
+  if (st != CAT_OK) return st;
+  if (!valid_k(k) || d_in % k != 0) return fail(CAT_ERR_SHAPE, "k must be one of 16..256 (power of two) and divide d_in");
+  if (!W || !T_blocks || !Wq || !w_scale) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (kind == CAT_T_CAT && (!sigma_x_blocks || n_calib < 1))
+    return fail(CAT_ERR_INVALID_ARG, "CAT needs sigma_x_blocks and n_calib >= 1");
+  if (kind == CAT_T_RHT && !rht_signs) return fail(CAT_ERR_INVALID_ARG, "RHT needs rht_signs");
+  if (!aligned16(W) || !aligned16(T_blocks) || !aligned16(Wq) || !aligned16(w_scale) ||
+      (sigma_x_blocks && !aligned16(sigma_x_blocks)))
+    return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  if ((st = check_device()) != CAT_OK) return st;
+
+  cudaStream_t s = (cudaStream_t)stream;
+  const int64_t nb = d_in / k;
+  const size_t kk = (size_t)k * k, nblk = (size_t)nb * kk;
+  std::vector<double> sx_h, sw_h;
+  cudaError_t e;
+  if (kind == CAT_T_CAT) {
+    double* sw_d = nullptr;
+    if ((e = cudaMallocAsync((void**)&sw_d, nblk * sizeof(double), s)) != cudaSuccess) return cuda_fail(e, "cudaMallocAsync");
+    e = cat::launch_calib_cov(W, (int)dtype, d_out, d_in, k, sw_d, 0, s);  // Sigma_w = W^T W blocks
+    sx_h.resize(nblk);
+    sw_h.resize(nblk);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(sx_h.data(), sigma_x_blocks, nblk * sizeof(double), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(sw_h.data(), sw_d, nblk * sizeof(double), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    cudaFreeAsync(sw_d, s);
+    if (e != cudaSuccess) return cuda_fail(e, "Sigma_w / Sigma_x readback");
+  }
+  std::vector<double> T(nblk), Ti(nblk);
+  st = cat_build_transform_host(kind, d_in, k, sx_h.empty() ? nullptr : sx_h.data(), n_calib,
+                                sw_h.empty() ? nullptr : sw_h.data(), rht_signs, T.data(), Ti.data());
+  if (st != CAT_OK) return st;
+  // Upload T (online transform) and A_w = (T^{-1})^T, which maps a weight row w to (W T^{-1}) row.
+  std::vector<float> Tf(nblk), Awf(nblk);
+  for (int64_t b = 0; b < nb; ++b)
+    for (int i = 0; i < k; ++i)
+      for (int j = 0; j < k; ++j) {
+        Tf[b * kk + (size_t)i * k + j] = (float)T[b * kk + (size_t)i * k + j];
+        Awf[b * kk + (size_t)i * k + j] = (float)Ti[b * kk + (size_t)j * k + i];
+      }
+  float* aw_d = nullptr;
+  uint32_t* status = status_word(&e);
+  if (!status) return cuda_fail(e, "status word");
+  if ((e = cudaMallocAsync((void**)&aw_d, nblk * sizeof(float), s)) != cudaSuccess) return cuda_fail(e, "cudaMallocAsync");
+  e = cudaMemcpyAsync(T_blocks, Tf.data(), nblk * sizeof(float), cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(aw_d, Awf.data(), nblk * sizeof(float), cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cat::launch_transform_quantize(W, (int)dtype, d_out, d_in, k, aw_d, Wq, w_scale, status, s);
+  cudaFreeAsync(aw_d, s);
+  cudaError_t e2 = cudaStreamSynchronize(s);  // host buffers above must outlive the copies
+  if (e != cudaSuccess) return cuda_fail(e, "weight quantization");
+  if (e2 != cudaSuccess) return cuda_fail(e2, "cudaStreamSynchronize");
+  return ok();
+}
+
+cat_status cat_transform_quantize_act(const void* x, cat_dtype dtype, int64_t n, int64_t d_in, int32_t k,
+                                      const float* T_blocks, uint8_t* xq, float* x_scale, cat_stream_t stream) {
+  if (dtype != CAT_F32 && dtype != CAT_BF16) return fail(CAT_ERR_INVALID_ARG, "unknown dtype");
+  if (n < 0) return fail(CAT_ERR_SHAPE, "n must be >= 0");
+  cat_status st = check_din(d_in);
+  if (st != CAT_OK) return st;
+  if (!valid_k(k) || d_in % k != 0) return fail(CAT_ERR_SHAPE, "k must be one of 16..256 (power of two) and divide d_in");
+  if (n == 0) return ok();
+  if (!x || !T_blocks || !xq || !x_scale) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(x) || !aligned16(T_blocks) || !aligned16(xq) || !aligned16(x_scale))
+    return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  if ((n + 63) / 64 > 0x7FFFFFFF) return fail(CAT_ERR_SHAPE, "n too large");
+  if ((st = check_device()) != CAT_OK) return st;
+  cudaError_t e;
+  uint32_t* status = status_word(&e);
+  if (!status) return cuda_fail(e, "status word");
+  e = cat::launch_transform_quantize(x, (int)dtype, n, d_in, k, T_blocks, xq, x_scale, status, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cat_transform_quantize_act launch");
+  return ok();
+}
+
+cat_status cat_w4a4_linear(const uint8_t* xq, const float* x_scale, const uint8_t* Wq, const float* w_scale,
+                           int64_t n, int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, cat_stream_t stream) {
+  if (n < 0 || d_out <= 0) return fail(CAT_ERR_SHAPE, "n must be >= 0 and d_out >= 1");
+  cat_status st = check_din(d_in);
+  if (st != CAT_OK) return st;
+  if (n > 0x7FFFFFFF || d_out > 0x7FFFFFFF) return fail(CAT_ERR_SHAPE, "n and d_out must fit in int32");
+  if (n == 0) return ok();
+  if (!xq || !x_scale || !Wq || !w_scale || !y) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(xq) || !aligned16(x_scale) || !aligned16(Wq) || !aligned16(w_scale) || !aligned16(y) ||
+      (acc_out && !aligned16(acc_out)))
+    return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  if ((st = check_device()) != CAT_OK) return st;
+  cudaError_t e;
+  uint32_t* status = status_word(&e);
+  if (!status) return cuda_fail(e, "status word");
+  if (n <= kMaxDecodeTokens)
+    e = cat::launch_w4a4_gemm_decode(xq, x_scale, Wq, w_scale, n, d_in, d_out, y, acc_out, (cudaStream_t)stream);
+  else
+    e = cat::launch_w4a4_gemm_tc(xq, x_scale, Wq, w_scale, n, d_in, d_out, y, acc_out, status, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cat_w4a4_linear launch");
+  return ok();
+}
+
+cat_status cat_sqnr(const float* y_ref, const float* y_hat, int64_t numel, double* out3, cat_stream_t stream) {
+  if (numel < 0) return fail(CAT_ERR_SHAPE, "numel must be >= 0");
+  if (!out3 || (numel > 0 && (!y_ref || !y_hat))) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(out3) || (y_ref && !aligned16(y_ref)) || (y_hat && !aligned16(y_hat)))
+    return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  cat_status st = check_device();
+  if (st != CAT_OK) return st;
+  cudaError_t e = cat::launch_sqnr(y_ref, y_hat, numel, out3, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cat_sqnr launch");
+  return ok();
+}
+
+cat_status cat_device_status(cat_stream_t stream, uint32_t* detail) {
+  cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+  uint32_t v = 0, zero = 0;
+  if ((e = cudaMemcpyFromSymbol(&v, g_device_status, sizeof(v))) != cudaSuccess) return cuda_fail(e, "read status");
+  if ((e = cudaMemcpyToSymbol(g_device_status, &zero, sizeof(zero))) != cudaSuccess) return cuda_fail(e, "clear status");
+  if (detail) *detail = v;
+  if (v & cat::kStatusTimeout) return fail(CAT_ERR_TIMEOUT, "a bounded device wait gave up");
+  if (v & cat::kStatusNonFinite) return fail(CAT_ERR_NUMERIC, "a kernel met a non-finite value");
+  return ok();
+}
+
+}  // extern "C"

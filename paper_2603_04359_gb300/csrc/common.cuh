@@ -1,0 +1,212 @@
+// Device helpers shared by the CAT W4A4 kernels (sm_103a): status reporting, the SM4x8 code
+// format, bounded mbarrier waits, TMA and tcgen05 wrappers.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace cat {
+
+// ------------------------------------------------------------------------------------------
+// Device status word (one per device, owned by api.cu; kernels get its address).
+// ------------------------------------------------------------------------------------------
+enum : uint32_t {
+  kStatusTimeout = 1u,     // a bounded wait gave up
+  kStatusNonFinite = 2u,   // a non-finite value reached a quantizer
+};
+
+// Upper bound of any single pipeline wait, in nanoseconds of %globaltimer.
+constexpr uint64_t kWaitLimitNs = 1000000000ull;
+
+__device__ __forceinline__ void report(uint32_t* status, uint32_t bits) {
+  if (status) atomicOr(status, bits);
+}
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
+  return t;
+}
+
+// ------------------------------------------------------------------------------------------
+// SM4x8 code format.  A code q in [-7, 7] is the FP8 E4M3 byte (q < 0) << 7 | |q|, i.e. the
+// subnormal value q * 2^-9.  Eight consecutive codes e0..e7 share one 32-bit word
+//   w = E(e0..e3) | rotl(E(e4..e7), 4)
+// where E(.) packs four E4M3 bytes little-endian; then E(e0..e3) = w & 0x87878787 and
+// E(e4..e7) = rotr(w, 4) & 0x87878787.
+// ------------------------------------------------------------------------------------------
+constexpr uint32_t kSm4Mask = 0x87878787u;
+
+__device__ __forceinline__ uint32_t sm4_lo(uint32_t w) { return w & kSm4Mask; }
+__device__ __forceinline__ uint32_t sm4_hi(uint32_t w) { return __funnelshift_r(w, w, 4) & kSm4Mask; }
+
+__device__ __forceinline__ uint32_t e4m3_code_byte(int q) {
+  return (q < 0 ? 0x80u : 0u) | (uint32_t)(q < 0 ? -q : q);
+}
+
+// Pack eight codes (each in [-7, 7]) into one SM4x8 word.
+__device__ __forceinline__ uint32_t sm4_pack(const int (&q)[8]) {
+  uint32_t lo = e4m3_code_byte(q[0]) | (e4m3_code_byte(q[1]) << 8) | (e4m3_code_byte(q[2]) << 16) |
+                (e4m3_code_byte(q[3]) << 24);
+  uint32_t hi = e4m3_code_byte(q[4]) | (e4m3_code_byte(q[5]) << 8) | (e4m3_code_byte(q[6]) << 16) |
+                (e4m3_code_byte(q[7]) << 24);
+  return lo | __funnelshift_l(hi, hi, 4);
+}
+
+// The accumulators hold sum(q_x * 2^-9 * q_w * 2^-9); multiply by 2^18 to get the integer.
+constexpr float kAccScale = 262144.0f;
+
+// ------------------------------------------------------------------------------------------
+// Shared-memory addresses, mbarriers (all waits bounded).
+// ------------------------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+      : "=r"(done)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return done != 0;
+}
+
+// Wait until the phase with the given parity has completed.  Returns false (and raises
+// `*abort`) if `*abort` was already raised by another thread or the wait exceeded the limit.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 63u) == 0u) {
+      if (*abort) return false;
+      if (globaltimer_ns() - t0 > kWaitLimitNs) {
+        *abort = 1;
+        return false;
+      }
+    }
+  }
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+
+// ------------------------------------------------------------------------------------------
+// TMA (tiled tensor copies global -> shared, completion counted on an mbarrier).
+// ------------------------------------------------------------------------------------------
+__device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* map, int32_t x, int32_t y,
+                                            uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+          smem_u32(smem_dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void prefetch_tensormap(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// ------------------------------------------------------------------------------------------
+// tcgen05 (5th-generation tensor cores, accumulators in tensor memory).
+// ------------------------------------------------------------------------------------------
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// Whole warp: allocate `ncols` TMEM columns, address written to *dst (shared memory).
+__device__ __forceinline__ void tmem_alloc(uint32_t* dst, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst)), "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+// D[tmem] (+)= A[smem] * B[smem]^T, FP8/FP6/FP4 kinds, fp32 accumulate.
+__device__ __forceinline__ void mma_f8f6f4(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                           uint32_t accumulate) {
+  asm volatile(
+      "{ .reg .pred p; setp.ne.b32 p, %4, 0; "
+      "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p; }" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrive on an mbarrier once every tcgen05.mma issued so far by this thread has completed.
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, 8-row groups 1024 B apart.
+__device__ __forceinline__ uint64_t sdesc_kmajor_sw128(uint32_t saddr) {
+  return (uint64_t)((saddr >> 4) & 0x3FFFu) | (1ull << 16) | (64ull << 32) | (1ull << 46) | (2ull << 61);
+}
+
+// Instruction descriptor: dense, D fp32, A/B E4M3, both K-major, shape M x N.
+__host__ __device__ constexpr uint32_t idesc_e4m3_f32(int M, int N) {
+  return (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+// 32 lanes x 32 consecutive 32-bit columns: thread i of the warp gets lane (base lane + i).
+#define CAT_TMEM_LD32(taddr, r)                                                                                  \
+  asm volatile(                                                                                                   \
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18," \
+      "%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"                                              \
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),          \
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),    \
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),  \
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])   \
+      : "r"(taddr))
+
+__device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
+// ------------------------------------------------------------------------------------------
+// Misc
+// ------------------------------------------------------------------------------------------
+template <typename T>
+__device__ __forceinline__ float to_f32(T v);
+template <>
+__device__ __forceinline__ float to_f32<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 v) { return __bfloat162float(v); }
+
+}  // namespace cat
+
+// Host-side launchers implemented by the kernel translation units (all return cudaError_t).
+namespace cat {
+cudaError_t launch_calib_cov(const void* x, int dtype, int64_t n, int64_t d, int k, double* sigma, int accumulate,
+                             cudaStream_t stream);
+cudaError_t launch_transform_quantize(const void* x, int dtype, int64_t n, int64_t d, int k, const float* T,
+                                      uint8_t* codes, float* scale, uint32_t* status, cudaStream_t stream);
+cudaError_t launch_w4a4_gemm(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
+                             int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, uint32_t* status,
+                             cudaStream_t stream);
+cudaError_t launch_sqnr(const float* y_ref, const float* y_hat, int64_t numel, double* out3, cudaStream_t stream);
+cudaError_t launch_transpose_blocks_f32(const double* src, float* dst, int nb, int k, int transpose,
+                                        cudaStream_t stream);
+}  // namespace cat

@@ -1,0 +1,221 @@
+"""Parity of the CUDA path (through the C ABI) with the fp64 CPU oracle, element by element.
+
+Tolerances (the benchmark spec's targets, applied per call):
+* integer accumulators: bit-exact given identical codes;
+* INT4 codes: may differ by +-1, in at most 1e-4 of the elements (at least one element is
+  allowed in small cases), and only where the oracle's pre-rounding value lies within 1e-5
+  (relative) of a rounding boundary -- the GPU accumulates x' = T x in fp32;
+* steps s_x, s_w: 1e-5 relative; y: 1e-3 relative Frobenius; SQNR: 0.01 dB;
+* calibration sums: 1e-10 relative Frobenius (compensated accumulation);
+* transform blocks: 1e-6 relative (fp32 storage of the float64 construction).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import sm4x8
+import workloads as WL
+
+pytestmark = pytest.mark.gpu
+
+cat = pytest.importorskip("paper_2603_04359_gb300")
+DEV = "cuda"
+
+
+def to_dev(t: WL.Tensor) -> torch.Tensor:
+    if t.dtype == "f32":
+        return torch.from_numpy(np.ascontiguousarray(t.raw)).to(DEV)
+    return torch.from_numpy(np.ascontiguousarray(t.raw).view(np.int16)).view(torch.bfloat16).to(DEV)
+
+
+def check_codes(q_gpu, q_ref, pre_ref, rel=1e-5, frac=1e-4):
+    q_gpu = np.asarray(q_gpu)
+    diff = q_gpu - q_ref
+    bad = diff != 0
+    if not bad.any():
+        return 0
+    assert np.abs(diff).max() <= 1, "codes differ by more than 1"
+    a = np.abs(pre_ref[bad])
+    boundary = np.floor(a) + 0.5
+    assert np.all(np.abs(a - boundary) <= rel * boundary), "a code differs away from a rounding boundary"
+    assert bad.sum() <= max(1, frac * q_ref.size), f"{bad.sum()} codes differ (> {frac} of {q_ref.size})"
+    return int(bad.sum())
+
+
+def rel_fro(a, b):
+    return float(np.linalg.norm(np.asarray(a, np.float64) - b) / max(np.linalg.norm(b), 1e-300))
+
+
+# ------------------------------------------------------------------------------------------
+# cat_calib_cov
+# ------------------------------------------------------------------------------------------
+
+@pytest.mark.parametrize("n,d,k,dtype", [(77, 256, 32, "f32"), (300, 512, 128, "bf16"), (1000, 512, 256, "bf16"),
+                                         (64, 64, 16, "f32"), (513, 384, 64, "bf16")])
+def test_calib_cov(n, d, k, dtype):
+    rng = np.random.default_rng(n + d)
+    X = rng.standard_normal((n, d)) * rng.lognormal(0, 1.5, d)
+    Xt = WL.cast(X, dtype)
+    S = cat.cat_calib_cov(to_dev(Xt), k).cpu().numpy()
+    ref = O.calib_cov_block_sums(Xt.values, k)
+    assert rel_fro(S, ref) < 1e-10
+    # accumulate a second batch
+    X2 = WL.cast(rng.standard_normal((n // 2 + 1, d)), dtype)
+    out = torch.from_numpy(S).to(DEV)
+    cat.cat_calib_cov(to_dev(X2), k, out=out, accumulate=True)
+    ref2 = O.calib_cov_block_sums(np.vstack([Xt.values, X2.values]), k)
+    assert rel_fro(out.cpu().numpy(), ref2) < 1e-10
+
+
+# ------------------------------------------------------------------------------------------
+# cat_transform_quantize_act (given the same transform)
+# ------------------------------------------------------------------------------------------
+
+def _cat_T(rng, d, k):
+    X = rng.standard_normal((4 * k + 64, d)) @ (rng.standard_normal((d, d)) / np.sqrt(d) + np.eye(d))
+    W = rng.standard_normal((d + 32, d)) * 0.02
+    T, _ = O.build_transform("cat", d, k, O.calib_cov_block_sums(X, k) / X.shape[0], O.weight_autocorr_blocks(W, k))
+    return T.astype(np.float32)
+
+
+@pytest.mark.parametrize("n,d,k,dtype", [(130, 256, 32, "f32"), (67, 384, 128, "bf16"), (200, 512, 256, "bf16"),
+                                         (5, 64, 16, "bf16"), (300, 1024, 64, "f32")])
+def test_transform_quantize_act(n, d, k, dtype):
+    rng = np.random.default_rng(7 * n + d)
+    X = rng.standard_normal((n, d)) * rng.lognormal(0, 1.0, d)
+    X[0] = 0.0                       # all-zero token
+    X[1] = 0.0
+    X[1, d // 3] = 3.0               # one-hot token
+    X[2] *= 1e4                      # a huge token
+    Xt = WL.cast(X, dtype)
+    T32 = _cat_T(rng, d, k)
+    xq, sx = cat.cat_transform_quantize_act(to_dev(Xt), torch.from_numpy(T32).to(DEV), k)
+    ref = O.transform_quantize_act(Xt.values, T32.astype(np.float64))
+    q = sm4x8.unpack(xq.cpu().numpy())
+    check_codes(q, ref.qx, ref.pre_x)
+    sxg = sx.cpu().numpy().astype(np.float64)
+    assert sxg[0] == 0.0 and np.all(q[0] == 0)
+    np.testing.assert_allclose(sxg, ref.sx, rtol=1e-5, atol=0)
+    assert np.abs(q).max() == 7
+    assert cat.cat_device_status()[0] == 0
+
+
+def test_nonfinite_activation_reports_numeric():
+    d, k = 128, 32
+    X = np.ones((70, d), dtype=np.float32)
+    X[3, 5] = np.inf
+    T = np.tile(np.eye(k, dtype=np.float32), (d // k, 1, 1))
+    cat.cat_device_status()  # clear
+    xq, sx = cat.cat_transform_quantize_act(torch.from_numpy(X).to(DEV), torch.from_numpy(T).to(DEV), k)
+    st, word = cat.cat_device_status()
+    assert st == 4 and word & 2
+    assert sx[3].item() == 0.0
+    assert sx[4].item() == pytest.approx(1.0 / 7.0, rel=1e-6)
+    assert cat.cat_device_status()[0] == 0  # cleared
+
+
+# ------------------------------------------------------------------------------------------
+# cat_w4a4_linear (given identical codes): exact accumulators
+# ------------------------------------------------------------------------------------------
+
+GEMM_SHAPES = [
+    (1, 64, 8), (5, 160, 100), (16, 4096, 520), (17, 96, 33), (32, 384, 300),          # weight-streaming path
+    (33, 128, 256), (128, 256, 256), (129, 160, 300), (300, 384, 520), (257, 4096, 64),  # tcgen05 path
+    (512, 1024, 1024),
+]
+
+
+@pytest.mark.parametrize("n,d_in,d_out", GEMM_SHAPES)
+def test_w4a4_linear_exact(n, d_in, d_out):
+    rng = np.random.default_rng(n * 1000 + d_in + d_out)
+    qx = WL.random_codes(rng, (n, d_in)).astype(np.int64)
+    qw = WL.random_codes(rng, (d_out, d_in)).astype(np.int64)
+    sx = rng.uniform(0.01, 2.0, n).astype(np.float32)
+    sw = rng.uniform(0.001, 0.1, d_out).astype(np.float32)
+    xq = torch.from_numpy(sm4x8.pack(qx)).to(DEV)
+    wq = torch.from_numpy(sm4x8.pack(qw)).to(DEV)
+    acc = torch.empty((n, d_out), dtype=torch.int32, device=DEV)
+    y = cat.cat_w4a4_linear(xq, torch.from_numpy(sx).to(DEV), wq, torch.from_numpy(sw).to(DEV), acc_out=acc)
+    ref_acc = O.int_gemm(qx, qw)
+    np.testing.assert_array_equal(acc.cpu().numpy(), ref_acc)
+    ref_y = O.dequantize_output(ref_acc, sx.astype(np.float64), sw.astype(np.float64))
+    assert rel_fro(y.cpu().numpy(), ref_y) < 1e-6
+    assert cat.cat_device_status()[0] == 0
+
+
+@pytest.mark.parametrize("n", [8, 200])
+def test_w4a4_linear_extreme_accumulators(n):
+    d_in, d_out = 14336, 64
+    qx = np.full((n, d_in), 7, dtype=np.int64)
+    qx[1::2] = -7
+    qw = np.full((d_out, d_in), 7, dtype=np.int64)
+    qw[3, : d_in // 2] = -7                       # cancels to zero
+    qw[5, -300:] = np.arange(300) % 3 - 1         # small codes after a large prefix
+    ones = torch.ones(max(n, d_out), dtype=torch.float32, device=DEV)
+    acc = torch.empty((n, d_out), dtype=torch.int32, device=DEV)
+    cat.cat_w4a4_linear(torch.from_numpy(sm4x8.pack(qx)).to(DEV), ones[:n].contiguous(),
+                        torch.from_numpy(sm4x8.pack(qw)).to(DEV), ones[:d_out].contiguous(), acc_out=acc)
+    ref = O.int_gemm(qx, qw)
+    assert np.abs(ref).max() == 49 * d_in
+    np.testing.assert_array_equal(acc.cpu().numpy(), ref)
+
+
+# ------------------------------------------------------------------------------------------
+# cat_sqnr
+# ------------------------------------------------------------------------------------------
+
+@pytest.mark.parametrize("numel", [1, 7, 4096, 1_000_003])
+def test_sqnr(numel):
+    rng = np.random.default_rng(numel)
+    y = rng.standard_normal(numel).astype(np.float32) * 3
+    yh = (y + rng.standard_normal(numel).astype(np.float32) * 0.05).astype(np.float32)
+    out = cat.cat_sqnr(torch.from_numpy(y).to(DEV), torch.from_numpy(yh).to(DEV)).cpu().numpy()
+    sig, err = O.sqnr_sums(y, yh)
+    assert abs(out[0] - sig) <= 1e-6 * sig and abs(out[1] - err) <= 1e-6 * err
+    assert abs(out[2] - 10 * np.log10(sig / err)) < 1e-5
+
+
+# ------------------------------------------------------------------------------------------
+# Whole layer: library pipeline vs oracle pipeline from the same raw inputs
+# ------------------------------------------------------------------------------------------
+
+def gpu_layer(L: WL.Layer, kind: str, k: int):
+    x, W, xc = to_dev(L.x_eval), to_dev(L.W), to_dev(L.x_calib)
+    sig = cat.cat_calib_cov(xc, k) if kind == "cat" else None
+    T, Wq, sw = cat.cat_quantize_weights(W, k, kind, sigma_x=sig, n_calib=L.cfg.n_calib,
+                                         rht_signs=L.rht_signs if kind == "rht" else None)
+    xq, sx = cat.cat_transform_quantize_act(x, T, k)
+    y = cat.cat_w4a4_linear(xq, sx, Wq, sw)
+    return dict(sigma=sig, T=T, Wq=Wq, sw=sw, xq=xq, sx=sx, y=y)
+
+
+SMALL = [
+    WL.CONFIGS["c1_256x256_k32_f32"],
+    WL.small_config("s_bf16_k128", d_in=512, d_out=384, n_eval=300, n_calib=512, k=128, seed=21),
+    WL.small_config("s_swiglu_k64", d_in=768, d_out=200, n_eval=70, n_calib=256, k=64, act="swiglu", seed=22),
+    WL.small_config("s_decode_k256", d_in=512, d_out=1000, n_eval=16, n_calib=600, k=256, seed=23),
+]
+
+
+@pytest.mark.parametrize("cfg", SMALL, ids=lambda c: c.name)
+@pytest.mark.parametrize("kind", ["identity", "rht", "cat"])
+def test_layer_end_to_end(cfg, kind):
+    L = WL.make_layer(cfg)
+    k = cfg.k
+    g = gpu_layer(L, kind, k)
+    ref = O.cat_layer(L.x_eval.values, L.W.values, kind, k, X_calib=L.x_calib.values, signs=L.rht_signs)
+    # transform blocks
+    assert rel_fro(g["T"].cpu().numpy(), ref["prep"].T) < 1e-6
+    # weight and activation codes, steps
+    check_codes(sm4x8.unpack(g["Wq"].cpu().numpy()), ref["prep"].qw, ref["prep"].pre_w)
+    np.testing.assert_allclose(g["sw"].cpu().numpy(), ref["prep"].sw, rtol=1e-5)
+    check_codes(sm4x8.unpack(g["xq"].cpu().numpy()), ref["act"].qx, ref["act"].pre_x)
+    np.testing.assert_allclose(g["sx"].cpu().numpy(), ref["act"].sx, rtol=1e-5)
+    # output and SQNR (y_ref in fp32, as the benchmark supplies it)
+    y_hat = g["y"].cpu().numpy()
+    assert rel_fro(y_hat, ref["y_hat"]) < 1e-3
+    y_ref = torch.from_numpy(ref["y"].astype(np.float32)).to(DEV)
+    s3 = cat.cat_sqnr(y_ref, g["y"]).cpu().numpy()
+    assert abs(s3[2] - ref["sqnr_db"]) < 0.01
+    assert cat.cat_device_status()[0] == 0

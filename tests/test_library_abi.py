@@ -1,0 +1,130 @@
+"""The C-ABI library without a GPU: it builds, loads, exports every entry point declared in
+include/cat_w4a4.h, validates arguments on the host before any CUDA call, and its host-side
+float64 transform construction matches the oracle."""
+import ctypes
+import os
+
+import numpy as np
+import pytest
+
+import oracle as O
+import paper_2603_04359_gb300 as cat
+from paper_2603_04359_gb300 import build as catbuild
+
+CSRC = os.path.join(os.path.dirname(catbuild.__file__), "csrc")
+
+
+@pytest.fixture(scope="session")
+def lib():
+    srcs = [os.path.join(CSRC, f) for f in os.listdir(CSRC)]
+    stale = (not os.path.exists(cat.library_path()) or
+             max(os.path.getmtime(s) for s in srcs) > os.path.getmtime(cat.library_path()))
+    if stale:
+        catbuild.build()
+    return cat.load_library()
+
+
+def test_exports_every_declared_symbol(lib):
+    names = cat.exported_symbols()
+    for expected in ("cat_calib_cov", "cat_quantize_weights", "cat_transform_quantize_act", "cat_w4a4_linear",
+                     "cat_sqnr", "cat_status_string", "cat_build_transform_host", "cat_device_status"):
+        assert expected in names
+    for name in names:
+        assert hasattr(lib, name), name
+
+
+def test_status_strings_and_version(lib):
+    assert lib.cat_status_string(0) == b"CAT_OK"
+    assert lib.cat_status_string(7) == b"CAT_ERR_TIMEOUT"
+    assert cat.cat_version() >= 10000
+
+
+def _fake(addr):
+    return ctypes.c_void_p(addr)
+
+
+def test_host_validation_without_gpu(lib):
+    """Invalid calls are rejected before anything touches CUDA (so this runs on a CPU machine)."""
+    P = _fake(0x10000)
+    bad = _fake(0x10008)  # not 16-byte aligned
+    # cat_transform_quantize_act(x, dtype, n, d_in, k, T, xq, sx, stream)
+    assert lib.cat_transform_quantize_act(P, 1, 4, 48, 16, P, P, P, None) == 2          # d_in % 32
+    assert lib.cat_transform_quantize_act(P, 1, 4, 64, 48, P, P, P, None) == 2          # k not a power of two
+    assert lib.cat_transform_quantize_act(P, 1, 4, 96, 64, P, P, P, None) == 2          # k does not divide d_in
+    assert lib.cat_transform_quantize_act(P, 7, 4, 64, 32, P, P, P, None) == 1          # dtype
+    assert lib.cat_transform_quantize_act(None, 1, 4, 64, 32, P, P, P, None) == 1       # NULL
+    assert lib.cat_transform_quantize_act(bad, 1, 4, 64, 32, P, P, P, None) == 3        # alignment
+    assert lib.cat_transform_quantize_act(P, 1, -1, 64, 32, P, P, P, None) == 2         # n < 0
+    assert lib.cat_transform_quantize_act(P, 1, 0, 64, 32, None, None, None, None) == 0  # n == 0: no-op
+    lib.cat_transform_quantize_act(P, 1, 4, 48, 16, P, P, P, None)
+    assert b"multiple of 32" in lib.cat_last_error()
+    # cat_w4a4_linear(xq, sx, wq, sw, n, d_in, d_out, y, acc, stream)
+    assert lib.cat_w4a4_linear(P, P, P, P, 4, 300000, 8, P, None, None) == 2            # exactness bound
+    assert lib.cat_w4a4_linear(P, P, P, P, 4, 64, 0, P, None, None) == 2                # d_out
+    assert lib.cat_w4a4_linear(P, P, P, P, 4, 64, 8, None, None, None) == 1             # y NULL
+    assert lib.cat_w4a4_linear(P, P, P, P, 4, 64, 8, P, bad, None) == 3                 # acc alignment
+    # cat_calib_cov(x, dtype, n, d, k, sigma, accumulate, stream)
+    assert lib.cat_calib_cov(P, 0, 4, 100, 32, P, 0, None) == 2
+    assert lib.cat_calib_cov(P, 0, 4, 64, 32, None, 0, None) == 1
+    # cat_quantize_weights(W, dtype, d_out, d_in, k, kind, sigma_x, n_calib, signs, T, Wq, sw, stream)
+    assert lib.cat_quantize_weights(P, 1, 8, 64, 32, 2, None, 0, None, P, P, P, None) == 1   # CAT w/o sigma
+    assert lib.cat_quantize_weights(P, 1, 8, 64, 32, 1, None, 0, None, P, P, P, None) == 1   # RHT w/o signs
+    assert lib.cat_quantize_weights(P, 1, 8, 64, 32, 9, None, 0, None, P, P, P, None) == 1   # kind
+    # cat_sqnr(y_ref, y_hat, numel, out3, stream)
+    assert lib.cat_sqnr(P, P, -1, P, None) == 2
+    assert lib.cat_sqnr(P, None, 10, P, None) == 1
+
+
+def test_valid_call_without_device_reports_cuda_error(lib):
+    try:
+        import torch
+        if torch.cuda.is_available():
+            pytest.skip("a GPU is present")
+    except ImportError:
+        pass
+    P = _fake(0x10000)
+    st = lib.cat_transform_quantize_act(P, 1, 4, 64, 32, P, P, P, None)
+    assert st in (5, 6)
+    assert len(lib.cat_last_error()) > 0
+
+
+def _blocks_problem(seed, d, k, n=800):
+    rng = np.random.default_rng(seed)
+    X = rng.standard_normal((n, d)) @ (rng.standard_normal((d, d)) / np.sqrt(d) + np.eye(d))
+    X[:, rng.choice(d, 2, replace=False)] *= 60.0
+    W = rng.standard_normal((3 * d // 2, d)) * 0.02 * rng.lognormal(0, 0.5, (3 * d // 2, 1))
+    return X, W, rng.choice([-1.0, 1.0], d)
+
+
+@pytest.mark.parametrize("k", [16, 32, 64])
+def test_host_transform_matches_oracle(lib, k):
+    d = 128
+    X, W, signs = _blocks_problem(k, d, k)
+    Sx_sum = O.calib_cov_block_sums(X, k)
+    Sw = O.weight_autocorr_blocks(W, k)
+    for kind in ("identity", "rht", "cat"):
+        T, Ti = cat.cat_build_transform_host(kind, d, k, Sx_sum, X.shape[0], Sw, signs)
+        To, Tio = O.build_transform(kind, d, k, Sx_sum / X.shape[0], Sw, signs)
+        rel = np.linalg.norm(T - To) / np.linalg.norm(To)
+        reli = np.linalg.norm(Ti - Tio) / np.linalg.norm(Tio)
+        assert rel < 1e-9 and reli < 1e-9, (kind, rel, reli)
+        for b in range(d // k):
+            np.testing.assert_allclose(T[b] @ Ti[b], np.eye(k), atol=1e-9)
+
+
+def test_host_transform_k256_and_errors(lib):
+    d, k = 256, 256
+    X, W, signs = _blocks_problem(7, d, k, n=1500)
+    Sx_sum = O.calib_cov_block_sums(X, k)
+    Sw = O.weight_autocorr_blocks(W, k)
+    T, Ti = cat.cat_build_transform_host("cat", d, k, Sx_sum, X.shape[0], Sw)
+    To, Tio = O.build_transform("cat", d, k, Sx_sum / X.shape[0], Sw)
+    assert np.linalg.norm(T - To) / np.linalg.norm(To) < 1e-8
+    # a singular calibration block is rejected
+    Sx_bad = Sx_sum.copy()
+    Sx_bad[0] = 0.0
+    with pytest.raises(cat.CatError) as ei:
+        cat.cat_build_transform_host("cat", d, k, Sx_bad, X.shape[0], Sw)
+    assert ei.value.status == 4
+    with pytest.raises(cat.CatError):
+        cat.cat_build_transform_host("rht", d, k, rht_signs=np.full(d, 0.5))
