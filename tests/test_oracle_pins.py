@@ -66,7 +66,10 @@ def test_quantizer_ranges_and_error_bound():
     assert s[3] == 0 and np.all(q[3] == 0)
     # |v - s q| <= s / 2 (no clipping: the range covers the row)
     err = np.abs(V - q * s[:, None])
-    assert np.all(err <= s[:, None] / 2 * (1 + 1e-12) + 1e-300)
+    assert np.all(err <= s[:, None] / 2 * (1 + 1e-6) + 1e-300)  # float32 code decision
+    # away from rounding boundaries the code is the float64 round-to-nearest of v / s
+    far = np.abs(np.abs(pre) - np.floor(np.abs(pre)) - 0.5) > 1e-5
+    np.testing.assert_array_equal(q[far], np.rint(pre[far]))
     # step size is max|v| / 7 exactly
     np.testing.assert_array_equal(s, np.max(np.abs(V), axis=1) / 7)
 
