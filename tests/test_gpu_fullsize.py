@@ -1,0 +1,77 @@
+"""Full-size parity: the five layer configurations run through the same C-ABI calls that
+bench.py times, compared with the oracle on sampled tokens and output channels (which it
+computes one by one), and -- where the oracle finishes in seconds -- on the whole output.
+
+Tolerances as in test_gpu_parity.py.  The whole-output SQNR check covers the QKV, down and
+decode layers; the 70B gate/up layer is checked on the sample only."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import sm4x8
+import workloads as WL
+from test_gpu_parity import DEV, check_codes, gpu_layer, rel_fro
+
+pytestmark = pytest.mark.gpu
+
+cat = pytest.importorskip("paper_2603_04359_gb300")
+
+FULL_OUTPUT = {"c2_qkv_4096x6144_k128_bf16", "c3_down_14336x4096_k128_bf16", "c4_decode_up_4096x14336_k128_bf16"}
+
+
+def _y_ref(L):
+    torch.backends.cuda.matmul.allow_tf32 = False
+    x = torch.from_numpy(L.x_eval.values).to(DEV)
+    W = torch.from_numpy(L.W.values).to(DEV)
+    return (x @ W.t()).contiguous()
+
+
+@pytest.mark.parametrize("name,k", [("c1_256x256_k32_f32", 32), ("c2_qkv_4096x6144_k128_bf16", 128),
+                                    ("c3_down_14336x4096_k128_bf16", 128), ("c4_decode_up_4096x14336_k128_bf16", 128),
+                                    ("c5_gateup_8192x28672_bf16", 128), ("c5_gateup_8192x28672_bf16", 256)])
+def test_full_size_layer(name, k):
+    cfg = WL.CONFIGS[name]
+    L = WL.make_layer(cfg)
+    n, d_in, d_out = cfg.n_eval, cfg.d_in, cfg.d_out
+    g = gpu_layer(L, "cat", k)
+    assert cat.cat_device_status()[0] == 0
+
+    # oracle: transform from the same calibration split
+    Xc = L.x_calib.values.astype(np.float64)
+    Sx = O.calib_cov_block_sums(Xc, k) / cfg.n_calib
+    assert rel_fro(g["sigma"].cpu().numpy(), Sx * cfg.n_calib) < 1e-10
+    Wv = L.W.values
+    Sw = O.weight_autocorr_blocks(Wv, k)
+    T, Ti = O.build_transform("cat", d_in, k, Sx, Sw)
+    assert rel_fro(g["T"].cpu().numpy(), T) < 1e-6
+
+    # sampled rows and tokens, computed one by one
+    rng = np.random.default_rng(1234)
+    ts = np.sort(rng.choice(n, min(n, 48), replace=False))
+    os_ = np.sort(rng.choice(d_out, min(d_out, 256), replace=False))
+    qw, sw, pre_w = O.quantize_rows_symmetric(O.apply_weight_transform(Wv[os_], Ti))
+    qx, sx, pre_x = O.quantize_rows_symmetric(O.apply_act_transform(L.x_eval.values[ts], T))
+    check_codes(sm4x8.unpack(g["Wq"][torch.from_numpy(os_).to(DEV)].cpu().numpy()), qw, pre_w)
+    check_codes(sm4x8.unpack(g["xq"][torch.from_numpy(ts).to(DEV)].cpu().numpy()), qx, pre_x)
+    np.testing.assert_allclose(g["sw"].cpu().numpy()[os_], sw, rtol=1e-5)
+    np.testing.assert_allclose(g["sx"].cpu().numpy()[ts], sx, rtol=1e-5)
+    y_hat_s = O.dequantize_output(O.int_gemm(qx, qw), sx, sw)
+    y_gpu = g["y"]
+    y_gpu_s = y_gpu[torch.from_numpy(ts).to(DEV)][:, torch.from_numpy(os_).to(DEV)].cpu().numpy()
+    assert rel_fro(y_gpu_s, y_hat_s) < 1e-3
+    y_s = O.linear(L.x_eval.values[ts], Wv[os_])
+    assert abs(O.sqnr_db(y_s, y_gpu_s) - O.sqnr_db(y_s, y_hat_s)) < 0.01
+
+    # whole-output SQNR through cat_sqnr (y_ref from an fp32 GEMM, as bench.py supplies it)
+    y_ref = _y_ref(L)
+    s3 = cat.cat_sqnr(y_ref, y_gpu).cpu().numpy()
+    d = (y_ref.double() - y_gpu.double())
+    assert abs(s3[1] - float((d * d).sum())) <= 1e-6 * s3[1]
+    if name in FULL_OUTPUT:
+        ref = O.transform_quantize_act(L.x_eval.values, T)
+        prep_q, prep_s, _ = O.quantize_rows_symmetric(O.apply_weight_transform(Wv, Ti))
+        _, y_hat = O.w4a4_linear(ref.qx, ref.sx, prep_q, prep_s)
+        y = O.linear(L.x_eval.values, Wv)
+        assert rel_fro(y_gpu.cpu().numpy(), y_hat) < 1e-3
+        assert abs(s3[2] - O.sqnr_db(y, y_hat)) < 0.01

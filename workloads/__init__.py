@@ -117,8 +117,8 @@ def small_config(name: str, d_in: int, d_out: int, n_eval: int, n_calib: int, k:
 def to_bf16_bits(a: np.ndarray) -> np.ndarray:
     """Round float values to bfloat16 (round to nearest, ties to even); return the uint16 bit patterns."""
     f = np.ascontiguousarray(a, dtype=np.float32)
-    u = f.view(np.uint32).astype(np.uint64)
-    rounded = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
+    u = f.view(np.uint32)  # finite values: u + 0x8000 cannot overflow 32 bits
+    rounded = (u + np.uint32(0x7FFF) + ((u >> np.uint32(16)) & np.uint32(1))) >> np.uint32(16)
     return rounded.astype(np.uint16)
 
 
