@@ -175,9 +175,22 @@ cudaError_t launch_t(const Tin* x, int64_t n, int64_t d, int k, const float* A, 
 
 }  // namespace
 
+bool transform_quantize_tc_supported(int dtype, int k, int64_t n, int64_t d);
+cudaError_t launch_transform_quantize_tc(const void* x, int64_t n, int64_t d, int k, const float* A, uint32_t* amax,
+                                         uint32_t* words, uint32_t* status, cudaStream_t stream);
+
 cudaError_t launch_transform_quantize(const void* x, int dtype, int64_t n, int64_t d, int k, const float* A,
                                       uint8_t* codes, float* scale, uint32_t* status, cudaStream_t stream) {
   if (n == 0) return cudaSuccess;
+  if (transform_quantize_tc_supported(dtype, k, n, d)) {  // bf16 rows: tensor-core path
+    uint32_t* amax = reinterpret_cast<uint32_t*>(scale);
+    cudaError_t e = cudaMemsetAsync(scale, 0, (size_t)n * sizeof(float), stream);
+    if (e == cudaSuccess) e = launch_transform_quantize_tc(x, n, d, k, A, amax, reinterpret_cast<uint32_t*>(codes),
+                                                           status, stream);
+    if (e != cudaSuccess) return e;
+    finalize_scale_kernel<<<(unsigned)((n + 255) / 256), 256, 0, stream>>>(amax, n, status);
+    return cudaGetLastError();
+  }
   if (dtype == 0) return launch_t(static_cast<const float*>(x), n, d, k, A, codes, scale, status, stream);
   return launch_t(static_cast<const __nv_bfloat16*>(x), n, d, k, A, codes, scale, status, stream);
 }

@@ -80,7 +80,8 @@ def _cat_T(rng, d, k):
 
 
 @pytest.mark.parametrize("n,d,k,dtype", [(130, 256, 32, "f32"), (67, 384, 128, "bf16"), (200, 512, 256, "bf16"),
-                                         (5, 64, 16, "bf16"), (300, 1024, 64, "f32")])
+                                         (5, 64, 16, "bf16"), (300, 1024, 64, "f32"), (300, 1024, 64, "bf16"),
+                                         (300, 640, 128, "bf16"), (1000, 256, 128, "bf16")])
 def test_transform_quantize_act(n, d, k, dtype):
     rng = np.random.default_rng(7 * n + d)
     X = rng.standard_normal((n, d)) * rng.lognormal(0, 1.0, d)
