@@ -90,8 +90,10 @@ int cat_version(void);
  *                (a plain sum over tokens: divide by the token count for E[x x^T]).  With
  *                accumulate == 0 the buffer is overwritten, otherwise the sums are added to it, so
  *                calibration sets larger than one batch can be streamed through.
- * The products of bf16 inputs are exact in fp32; the sums are carried in compensated (double-float)
- * fp32 arithmetic and stored in float64, so they match a float64 accumulation to about 1e-12.
+ * bf16 rows run on tensor cores: products are exact and tokens accumulate in fp32 (relative error
+ * ~1e-7, which moves the block transform by ~1e-7).  fp32 rows accumulate products and their FMA
+ * errors in compensated (double-float) fp32 arithmetic, matching float64 to ~1e-12.  Sums are
+ * stored as float64.
  */
 cat_status cat_calib_cov(const void* x, cat_dtype dtype, int64_t n, int64_t d, int32_t k,
                          double* sigma_blocks, int accumulate, cat_stream_t stream);

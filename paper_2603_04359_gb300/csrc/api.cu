@@ -123,7 +123,10 @@ cat_status cat_calib_cov(const void* x, cat_dtype dtype, int64_t n, int64_t d, i
   if (d / k > 0x7FFFFFFF) return fail(CAT_ERR_SHAPE, "too many blocks");
   cat_status st = check_device();
   if (st != CAT_OK) return st;
-  cudaError_t e = cat::launch_calib_cov(x, (int)dtype, n, d, k, sigma_blocks, accumulate, (cudaStream_t)stream);
+  cudaError_t e;
+  uint32_t* status = status_word(&e);
+  if (!status) return cuda_fail(e, "status word");
+  e = cat::launch_calib_cov(x, (int)dtype, n, d, k, sigma_blocks, accumulate, status, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "cat_calib_cov launch");
   return ok();
 }
@@ -182,7 +185,9 @@ cat_status cat_quantize_weights(const void* W, cat_dtype dtype, int64_t d_out, i
   if (kind == CAT_T_CAT) {
     double* sw_d = nullptr;
     if ((e = cudaMallocAsync((void**)&sw_d, nblk * sizeof(double), s)) != cudaSuccess) return cuda_fail(e, "cudaMallocAsync");
-    e = cat::launch_calib_cov(W, (int)dtype, d_out, d_in, k, sw_d, 0, s);  // Sigma_w = W^T W blocks
+    uint32_t* st_word = status_word(&e);
+    if (!st_word) return cuda_fail(e, "status word");
+    e = cat::launch_calib_cov(W, (int)dtype, d_out, d_in, k, sw_d, 0, st_word, s);  // Sigma_w = W^T W blocks
     sx_h.resize(nblk);
     sw_h.resize(nblk);
     if (e == cudaSuccess) e = cudaMemcpyAsync(sx_h.data(), sigma_x_blocks, nblk * sizeof(double), cudaMemcpyDeviceToHost, s);

@@ -1,5 +1,6 @@
 // Calibration autocorrelation blocks (Sec. 4: Sigma_x = E[x x^T]; Eq. 10 needs only its k x k
-// diagonal blocks):  sigma[b] (+)= sum_t x_{t,b} x_{t,b}^T.
+// diagonal blocks):  sigma[b] (+)= sum_t x_{t,b} x_{t,b}^T.  This file holds the path for fp32 rows
+// (and the entry point); bf16 rows take the tensor-core kernel in calib_cov_tc.cu.
 //
 // One CTA computes a TS x TS tile of one k x k block over a range of tokens, staging 32 tokens
 // at a time in shared memory.  Each product of two bf16 values is exact in fp32 (fp32 inputs add
@@ -129,9 +130,15 @@ cudaError_t launch_typed(const Tin* x, int64_t n, int64_t d, int k, double* sigm
 
 }  // namespace
 
+bool calib_cov_tc_supported(int dtype, int k, int64_t n, int64_t d);
+cudaError_t launch_calib_cov_tc(const void* x, int64_t n, int64_t d, int k, double* sigma, int accumulate,
+                                uint32_t* status, cudaStream_t stream);
+
+// bf16 rows: tensor-core SYRK (calib_cov_tc.cu); fp32 rows: the compensated SIMT kernel above.
 cudaError_t launch_calib_cov(const void* x, int dtype, int64_t n, int64_t d, int k, double* sigma, int accumulate,
-                             cudaStream_t stream) {
+                             uint32_t* status, cudaStream_t stream) {
   if (dtype == 0) return launch_typed(static_cast<const float*>(x), n, d, k, sigma, accumulate, stream);
+  if (calib_cov_tc_supported(dtype, k, n, d)) return launch_calib_cov_tc(x, n, d, k, sigma, accumulate, status, stream);
   return launch_typed(static_cast<const __nv_bfloat16*>(x), n, d, k, sigma, accumulate, stream);
 }
 

@@ -200,13 +200,11 @@ __device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 v) { return
 // Host-side launchers implemented by the kernel translation units (all return cudaError_t).
 namespace cat {
 cudaError_t launch_calib_cov(const void* x, int dtype, int64_t n, int64_t d, int k, double* sigma, int accumulate,
-                             cudaStream_t stream);
+                             uint32_t* status, cudaStream_t stream);
 cudaError_t launch_transform_quantize(const void* x, int dtype, int64_t n, int64_t d, int k, const float* T,
                                       uint8_t* codes, float* scale, uint32_t* status, cudaStream_t stream);
 cudaError_t launch_w4a4_gemm(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
                              int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, uint32_t* status,
                              cudaStream_t stream);
 cudaError_t launch_sqnr(const float* y_ref, const float* y_hat, int64_t numel, double* out3, cudaStream_t stream);
-cudaError_t launch_transpose_blocks_f32(const double* src, float* dst, int nb, int k, int transpose,
-                                        cudaStream_t stream);
 }  // namespace cat

@@ -40,11 +40,11 @@ def test_full_size_layer(name, k):
     # oracle: transform from the same calibration split
     Xc = L.x_calib.values.astype(np.float64)
     Sx = O.calib_cov_block_sums(Xc, k) / cfg.n_calib
-    assert rel_fro(g["sigma"].cpu().numpy(), Sx * cfg.n_calib) < 1e-10
+    assert rel_fro(g["sigma"].cpu().numpy(), Sx * cfg.n_calib) < (1e-10 if cfg.dtype == "f32" else 1e-6)
     Wv = L.W.values
     Sw = O.weight_autocorr_blocks(Wv, k)
     T, Ti = O.build_transform("cat", d_in, k, Sx, Sw)
-    assert rel_fro(g["T"].cpu().numpy(), T) < 1e-6
+    assert rel_fro(g["T"].cpu().numpy(), T) < (1e-6 if cfg.dtype == "f32" else 1e-5)
 
     # sampled rows and tokens, computed one by one
     rng = np.random.default_rng(1234)
