@@ -7,7 +7,8 @@
 // exact; tokens accumulate in fp32 in tensor memory.  The tensor cores' fp32 accumulation rounds
 // more coarsely than round-to-nearest, with an error that grows with the number of MMA steps, so
 // for k <= 128 the 16-token MMA steps go round-robin to NACC = 4 accumulators (512 TMEM columns),
-// each summing a quarter of the tokens, and the epilogue adds them in float64.  The result is
+// each summing a quarter of the tokens, and the epilogue adds them (fp32) before widening them to
+// float64 with integer operations (the FP64 pipe of this GPU is ~60x slower than FP32).  The result is
 // within ~1e-6 of a float64 sum, which moves the block transform by ~1e-6 (its square roots damp
 // the calibration error) -- far below the INT4 step.  Only the diagonal k x k blocks are written.
 //
@@ -52,6 +53,17 @@ struct CovBars {
 __device__ __forceinline__ uint64_t sdesc_mnmajor_sw128(uint32_t saddr, uint32_t lbo) {
   return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) | (64ull << 32) |
          (1ull << 46) | (2ull << 61);
+}
+
+// float -> double without the FP64 pipe: re-bias the exponent of a normal float (zero, subnormal,
+// inf and nan take the regular conversion).
+__device__ __forceinline__ double f32_to_f64_exact(float f) {
+  const uint32_t u = __float_as_uint(f);
+  const uint32_t e = (u >> 23) & 0xFFu;
+  if (e == 0u || e == 0xFFu) return (double)f;
+  const uint64_t bits = ((uint64_t)(u >> 31) << 63) | ((uint64_t)(e - 127u + 1023u) << 52) |
+                        ((uint64_t)(u & 0x7FFFFFu) << 29);
+  return __longlong_as_double((long long)bits);
 }
 
 __device__ __forceinline__ void mma_bf16_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
@@ -158,9 +170,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int cc = 0; cc < kw / 32; ++cc) {
           const int col = col0 + 32 * cc;
           const int jh = col / 128;
-          double v64[32];
+          float v32[32];  // the accumulators summed in fp32 (FP64 arithmetic is scarce on this GPU)
 #pragma unroll
-          for (int e = 0; e < 32; ++e) v64[e] = 0.0;
+          for (int e = 0; e < 32; ++e) v32[e] = 0.f;
           const int used = total_steps < C::NACC ? total_steps : C::NACC;  // accumulators written
 #pragma unroll 1
           for (int a = 0; a < used; ++a) {
@@ -169,7 +181,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + ((a * G2 + ih) * G2 + jh) * 128 + (col % 128), r);
             tmem_ld_wait();
 #pragma unroll
-            for (int e = 0; e < 32; ++e) v64[e] += (double)__uint_as_float(r[e]);
+            for (int e = 0; e < 32; ++e) v32[e] += __uint_as_float(r[e]);
           }
           if (ch >= d) continue;
 #pragma unroll
@@ -177,7 +189,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int jc = col + e;                      // column within the group
             if (k < 32 && (jc / k) != (row / k)) continue;  // k = 16: other half belongs to the neighbour
             double* dst = sigma + (int64_t)ch * k + (jc % k);
-            const double v = v64[e];
+            const double v = f32_to_f64_exact(v32[e]);
             if (mode == 2)
               atomicAdd(dst, v);
             else

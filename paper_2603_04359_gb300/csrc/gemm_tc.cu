@@ -8,19 +8,21 @@
 // products q_x q_w 2^-18 in fp32 tensor memory (exact: |acc| <= 49 d_in < 2^24), and the epilogue
 // multiplies by 2^18 s_x s_w.
 //
-// Shared-memory bandwidth is the budget that matters: decoding on the way into the tensor cores
-// costs a write per operand byte.  So the token operand A never touches shared memory -- each
-// decode thread owns one token row, loads its packed bytes straight from global memory, decodes
-// them in registers and writes the E4M3 row into tensor memory (tcgen05.st), from where the MMA
-// reads A -- and only the weight operand B is decoded into 128B-swizzled shared memory.
+// Data path.  The tensor cores read their shared-memory operands on a path of their own (their
+// rate does not change under concurrent LSU shared-memory traffic), an MMA with A in tensor memory
+// runs at ~93% of peak, and shared-memory stores top out near 100 B/clk/SM.  So:
+//   * packed A (128 x 64 B) and B (256 x 64 B) tiles arrive by TMA with a 64-byte swizzle, which
+//     makes one-row-per-thread 16-byte shared loads conflict-free;
+//   * A is decoded one row per thread and written to tensor memory (tcgen05.st), never to
+//     shared memory; the MMA reads A from tensor memory;
+//   * only B is decoded into 128B-swizzled shared memory (32 KiB of stores per K step).
 //
 // Persistent CTA (one per SM, 512 threads), output tile 128 tokens x 256 channels, K step 128:
-//   warp 0       TMEM allocator; lane 0 issues tcgen05.mma (4 x K=32 per K step) and commits
+//   warp 0       TMA producer (packed ring) and TMEM allocator
+//   warp 1       lane 0 issues tcgen05.mma (4 x K=32 per K step) and commits
 //   warps 4..7   epilogue: tcgen05.ld of their TMEM lane quadrant, scale, stage the rows in
 //                128B-swizzled shared memory, TMA store (plain stores when the TMA rules don't hold)
-//   warps 8..15  decode: prefetch packed A rows and B chunks two K steps ahead into registers
-//                (three rotating buffers);
-//                A -> TMEM stage, B -> shared-memory stage (4-stage ring)
+//   warps 8..15  decode: B chunks (all 8 warps) and A rows (warps 8..11, one TMEM quadrant each)
 // TMEM: accumulator columns [0, 256), A stages at 256 + 32 s.  Every mbarrier wait is bounded;
 // a wait that gives up raises the device status word and all roles drain and exit.
 #include <cstring>
@@ -33,7 +35,11 @@ namespace {
 
 constexpr int BM = 128, BN = 256, BK = 128;
 constexpr int BKP = BK / 2;                 // packed bytes per row per K step
-constexpr int SE = 4;                       // decoded stages (A in TMEM, B in shared memory)
+constexpr int SP = 3;                       // packed stages (TMA)
+constexpr int SE = 3;                       // decoded stages (A in TMEM, B in shared memory)
+constexpr uint32_t kPackedA = BM * BKP;     // 8 KiB
+constexpr uint32_t kPackedB = BN * BKP;     // 16 KiB
+constexpr uint32_t kPackedStage = kPackedA + kPackedB;
 constexpr uint32_t kStageB = BN * BK;       // 32 KiB of E4M3 per stage
 constexpr int kThreads = 512;
 constexpr int kDecWarp0 = 8, kDecWarps = 8, kDecThreads = kDecWarps * 32;
@@ -42,24 +48,27 @@ constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kAccCols = 256;
 constexpr uint32_t kIdesc = idesc_e4m3_f32(BM, BN);
 constexpr uint32_t kEpiStage = 32 * 32 * 4;                 // 32 rows x 32 fp32 columns, 4 KiB
-constexpr int kEpiBufs = 4;                                  // TMA-store staging buffers per epilogue warp
-constexpr uint32_t kEpiOffset = SE * kStageB;                // after the B stages
+constexpr int kEpiBufs = 2;                                  // TMA-store staging buffers per epilogue warp
+constexpr uint32_t kPkOffset = SE * kStageB;                 // after the decoded B stages
+constexpr uint32_t kEpiOffset = kPkOffset + SP * kPackedStage;
 constexpr uint32_t kScaleOffset = kEpiOffset + kEpiWarps * kEpiBufs * kEpiStage;
 constexpr uint32_t kBarOffset = kScaleOffset + kEpiWarps * BN * 4;
 constexpr size_t kSmemBytes = kBarOffset + 256 + 1024;      // + barriers + alignment slack
 
 struct Bars {
-  uint64_t full[SE], empty[SE], acc_full, acc_empty, mma_done;
+  uint64_t p_full[SP], p_empty[SP], full[SE], empty[SE], acc_full, acc_empty, mma_done;
   uint32_t tmem_addr;
   int abort;
 };
 
 // ---- tensor-memory stores and the TMA store path -------------------------------------------
-#define CAT_TMEM_ST16(taddr, v)                                                                              \
-  asm volatile("tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15," \
-               "%16};" ::"r"(taddr),                                                                         \
-               "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]),   \
-               "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])                  \
+#define CAT_TMEM_ST32(taddr, v)                                                                                 \
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16," \
+               "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),                   \
+               "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]),      \
+               "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]), "r"(v[16]),          \
+               "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]), "r"(v[24]),         \
+               "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])                     \
                : "memory")
 
 __device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
@@ -80,63 +89,23 @@ __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void*
                : "memory");
 }
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait_read_le3() { asm volatile("cp.async.bulk.wait_group.read 3;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read_le1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
-// Predicated 128-bit load into a zeroed destination: nothing depends on the loaded value until
-// it is consumed, so a prefetch issued here does not wait for its data.
-__device__ __forceinline__ void ldg_nc_pred(uint4& v, const uint8_t* p, bool pred) {
-  asm volatile(
-      "{ .reg .pred q; setp.ne.b32 q, %4, 0; mov.b32 %0, 0; mov.b32 %1, 0; mov.b32 %2, 0; mov.b32 %3, 0;\n"
-      "  @q ld.global.nc.v4.u32 {%0,%1,%2,%3}, [%5]; }"
-      : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-      : "r"((int)pred), "l"(p));
-}
-
-// Packed inputs of one K step for one decode thread: its A row half (2 x 16 B) and 4 B chunks.
-struct StepRegs {
-  uint4 a[2];
-  uint4 b[4];
-};
-
-struct DecodeCtx {
-  const uint8_t* xq;
-  const uint8_t* wq;
-  int64_t row_bytes;
-  int a_row;        // token row (global), this thread's TMEM lane
-  int a_half;       // which 32-byte half of the K step's 64 packed bytes
-  int n, d_out;
-  int b_row[4];     // B rows (within the tile) of this thread's 4 chunks
-  int b_chunk[4];   // 16-byte chunk (0..3) within the row's 64 bytes
-};
-
-__device__ __forceinline__ void load_step(const DecodeCtx& c, int m0, int n0, int ks, StepRegs& r) {
-  const int64_t kb = (int64_t)ks * BKP;
-  const int t = m0 + c.a_row;
-#pragma unroll
-  for (int h = 0; h < 2; ++h) {
-    const int64_t off = kb + c.a_half * 32 + h * 16;
-    const bool in = t < c.n && off < c.row_bytes;
-    ldg_nc_pred(r.a[h], c.xq + (in ? (int64_t)t * c.row_bytes + off : 0), in);
-  }
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int o = n0 + c.b_row[i];
-    const int64_t off = kb + c.b_chunk[i] * 16;
-    const bool in = o < c.d_out && off < c.row_bytes;
-    ldg_nc_pred(r.b[i], c.wq + (in ? (int64_t)o * c.row_bytes + off : 0), in);
-  }
-}
+// 64-byte swizzle of the packed TMA tiles: 16-byte chunk j of 64-byte row r sits at chunk
+// j ^ ((r >> 1) & 3), so 8 consecutive rows read at the same j touch 8 distinct bank groups.
+__device__ __forceinline__ uint32_t sw64_off(int r, int j) { return r * 64 + ((j ^ ((r >> 1) & 3)) << 4); }
 
 __global__ void __launch_bounds__(kThreads, 1)
-    w4a4_gemm_tc_kernel(const __grid_constant__ CUtensorMap tmY, const uint8_t* __restrict__ xq,
-                        const uint8_t* __restrict__ wq, const float* __restrict__ sx, const float* __restrict__ sw,
-                        int n, int d_in, int d_out, float* __restrict__ y, int32_t* __restrict__ acc_out,
-                        int use_tma_store, uint32_t* __restrict__ status) {
+    w4a4_gemm_tc_kernel(const __grid_constant__ CUtensorMap tmY, const __grid_constant__ CUtensorMap tmA,
+                        const __grid_constant__ CUtensorMap tmB, const float* __restrict__ sx,
+                        const float* __restrict__ sw, int n, int d_in, int d_out, float* __restrict__ y,
+                        int32_t* __restrict__ acc_out, int use_tma_store, uint32_t* __restrict__ status) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* bst = smem;                         // SE x [256 rows x 128 B], 128B-swizzled
-  uint8_t* epi = smem + kEpiOffset;            // 4 warps x 4 x [32 rows x 128 B], 128B-swizzled
+  uint8_t* bst = smem;                         // SE x [256 rows x 128 B] E4M3, 128B-swizzled
+  uint8_t* pk = smem + kPkOffset;              // SP x [A 128 x 64 B | B 256 x 64 B] packed, 64B-swizzled
+  uint8_t* epi = smem + kEpiOffset;            // 4 warps x 2 x [32 rows x 128 B], 128B-swizzled
   float* scl = reinterpret_cast<float*>(smem + kScaleOffset);  // 4 warps x 256 output-channel steps
   Bars* bars = reinterpret_cast<Bars*>(smem + kBarOffset);
   volatile int* abort_flag = &bars->abort;
@@ -148,6 +117,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int num_tiles = num_m * num_n;
 
   if (tid == 0) {
+    for (int s = 0; s < SP; ++s) {
+      mbar_init(&bars->p_full[s], 1);
+      mbar_init(&bars->p_empty[s], kDecWarps);
+    }
     for (int s = 0; s < SE; ++s) {
       mbar_init(&bars->full[s], kDecWarps);
       mbar_init(&bars->empty[s], 1);
@@ -166,6 +139,28 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = bars->tmem_addr;
 
   if (warp == 0) {
+    // ---------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      prefetch_tensormap(&tmA);
+      prefetch_tensormap(&tmB);
+      uint32_t it = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+        const int m = tile % num_m, nn = tile / num_m;
+        for (int ks = 0; ks < num_k; ++ks, ++it) {
+          const uint32_t s = it % SP, use = it / SP;
+          if (use > 0 && !(ok = mbar_wait_bounded(&bars->p_empty[s], (use - 1) & 1, abort_flag))) break;
+          uint8_t* dst = pk + s * kPackedStage;
+          mbar_arrive_expect_tx(&bars->p_full[s], kPackedStage);
+          tma_load_2d(dst, &tmA, ks * BKP, m * BM, &bars->p_full[s]);
+          tma_load_2d(dst + kPackedA, &tmB, ks * BKP, nn * BN, &bars->p_full[s]);
+        }
+      }
+      const uint32_t issued = it, first = issued > SP ? issued - SP : 0;
+      volatile int no_abort = 0;
+      for (uint32_t j = first; j < issued; ++j) mbar_wait_bounded(&bars->p_full[j % SP], (j / SP) & 1, &no_abort);
+    }
+  } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
     if (lane == 0) {
       uint32_t it = 0, tcount = 0;
@@ -228,7 +223,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (o0 >= d_out || row0 >= n) continue;  // warp-uniform: nothing of this chunk is in range
         if (use_tma_store) {
           uint8_t* buf = stage0 + (nstore % kEpiBufs) * kEpiStage;
-          if (lane == 0) bulk_wait_read_le3();  // the store issued kEpiBufs chunks ago has read this buffer
+          if (lane == 0) bulk_wait_read_le1();  // the store issued two chunks ago has read this buffer
           __syncwarp();
 #pragma unroll
           for (int q = 0; q < 8; ++q) {  // row `lane`, 16-byte chunk q at q ^ (lane % 8)
@@ -263,91 +258,54 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp >= kDecWarp0) {
     // ---------------------------------------------------------------- decode
     const int dt = tid - kDecWarp0 * 32;          // 0..255
+    const bool a_warp = warp < kDecWarp0 + 4;     // warps 8..11 also decode A rows
     const int quad = warp & 3;
-    DecodeCtx c;
-    c.xq = xq;
-    c.wq = wq;
-    c.row_bytes = d_in / 2;
-    c.a_row = quad * 32 + lane;
-    c.a_half = (warp - kDecWarp0) >> 2;           // warps 8..11 first half, 12..15 second half
-    c.n = n;
-    c.d_out = d_out;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int id = dt + kDecThreads * i;         // 1024 chunks = 256 rows x 4
-      c.b_row[i] = id >> 2;
-      c.b_chunk[i] = id & 3;
-    }
-    // The CTA's (tile, ks) sequence with register prefetch two steps ahead: three buffers, each
-    // loaded and then consumed two steps later (no register copies of loads in flight).
-    auto advance = [&](int& tl, int& k) {
-      if (++k == num_k) {
-        k = 0;
-        tl += gridDim.x;
-      }
-    };
-    auto load = [&](int tl, int k, StepRegs& r) {
-      if (tl < num_tiles) load_step(c, (tl % num_m) * BM, (tl / num_m) * BN, k, r);
-    };
+    const int a_row = quad * 32 + lane;           // this thread's A row = TMEM lane
     uint32_t it = 0;
     bool ok = true;
-    auto process = [&](const StepRegs& r) {
-      const uint32_t s = it % SE;
-      if (it >= SE && !(ok = mbar_wait_bounded(&bars->empty[s], ((it / SE) - 1) & 1, abort_flag))) return;
-      tc_fence_after();
-      // A: this thread's token row, 32 packed bytes -> 64 E4M3 bytes = 16 TMEM columns
-      uint32_t av[16];
-      const uint32_t aw[8] = {r.a[0].x, r.a[0].y, r.a[0].z, r.a[0].w, r.a[1].x, r.a[1].y, r.a[1].z, r.a[1].w};
+    for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+      for (int ks = 0; ks < num_k; ++ks, ++it) {
+        const uint32_t ps = it % SP, s = it % SE;
+        if (!(ok = mbar_wait_bounded(&bars->p_full[ps], (it / SP) & 1, abort_flag))) break;
+        if (it >= SE && !(ok = mbar_wait_bounded(&bars->empty[s], ((it / SE) - 1) & 1, abort_flag))) break;
+        tc_fence_after();
+        const uint8_t* pa = pk + ps * kPackedStage;
+        const uint8_t* pb = pa + kPackedA;
+        if (a_warp) {  // A: one 64-byte row per thread -> 128 E4M3 bytes = 32 TMEM columns
+          uint32_t av[32];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        av[2 * u] = sm4_lo(aw[u]);
-        av[2 * u + 1] = sm4_hi(aw[u]);
-      }
-      __syncwarp();
-      CAT_TMEM_ST16(tmem + ((uint32_t)(quad * 32) << 16) + kAccCols + 32u * s + 16u * c.a_half, av);
-      // B: 4 chunks of 16 packed bytes -> 2 x 16 E4M3 bytes each, 128B-swizzled rows
-      uint8_t* bs = bst + s * kStageB;
+          for (int j = 0; j < 4; ++j) {
+            const uint4 w = *reinterpret_cast<const uint4*>(pa + sw64_off(a_row, j));
+            av[8 * j + 0] = sm4_lo(w.x); av[8 * j + 1] = sm4_hi(w.x);
+            av[8 * j + 2] = sm4_lo(w.y); av[8 * j + 3] = sm4_hi(w.y);
+            av[8 * j + 4] = sm4_lo(w.z); av[8 * j + 5] = sm4_hi(w.z);
+            av[8 * j + 6] = sm4_lo(w.w); av[8 * j + 7] = sm4_hi(w.w);
+          }
+          __syncwarp();
+          CAT_TMEM_ST32(tmem + ((uint32_t)(quad * 32) << 16) + kAccCols + 32u * s, av);
+        }
+        // B: 1024 chunks of 16 packed bytes (256 rows x 4), 4 per thread, consecutive per warp
+        uint8_t* bs = bst + s * kStageB;
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const uint4 w = r.b[i];
-        const int row = c.b_row[i], j = c.b_chunk[i], swz = row & 7;
-        uint8_t* dst = bs + row * 128;
-        *reinterpret_cast<uint4*>(dst + (((2 * j) ^ swz) << 4)) =
-            make_uint4(sm4_lo(w.x), sm4_hi(w.x), sm4_lo(w.y), sm4_hi(w.y));
-        *reinterpret_cast<uint4*>(dst + (((2 * j + 1) ^ swz) << 4)) =
-            make_uint4(sm4_lo(w.z), sm4_hi(w.z), sm4_lo(w.w), sm4_hi(w.w));
+        for (int i = 0; i < 4; ++i) {
+          const int id = dt + kDecThreads * i;
+          const int row = id >> 2, j = id & 3, swz = row & 7;
+          const uint4 w = *reinterpret_cast<const uint4*>(pb + sw64_off(row, j));
+          uint8_t* dst = bs + row * 128;
+          *reinterpret_cast<uint4*>(dst + (((2 * j) ^ swz) << 4)) =
+              make_uint4(sm4_lo(w.x), sm4_hi(w.x), sm4_lo(w.y), sm4_hi(w.y));
+          *reinterpret_cast<uint4*>(dst + (((2 * j + 1) ^ swz) << 4)) =
+              make_uint4(sm4_lo(w.z), sm4_hi(w.z), sm4_lo(w.w), sm4_hi(w.w));
+        }
+        if (a_warp) tmem_st_wait();
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(&bars->p_empty[ps]);
+          mbar_arrive(&bars->full[s]);
+        }
       }
-      tmem_st_wait();
-      fence_proxy_async_smem();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->full[s]);
-      ++it;
-    };
-    StepRegs ra, rb, rc;
-    int tA = blockIdx.x, kA = 0;
-    int tB = tA, kB = kA;
-    advance(tB, kB);
-    int tC = tB, kC = kB;
-    advance(tC, kC);
-    load(tA, kA, ra);
-    load(tB, kB, rb);
-    while (ok) {
-      if (tA >= num_tiles) break;
-      load(tC, kC, rc);
-      process(ra);
-      tA = tC, kA = kC;
-      advance(tA, kA);
-      if (!ok || tB >= num_tiles) break;
-      load(tA, kA, ra);
-      process(rb);
-      tB = tA, kB = kA;
-      advance(tB, kB);
-      if (!ok || tC >= num_tiles) break;
-      load(tB, kB, rb);
-      process(rc);
-      tC = tB, kC = kB;
-      advance(tC, kC);
     }
   }
 
@@ -389,6 +347,19 @@ bool make_output_map(CUtensorMap* map, float* y, int64_t n, int64_t d_out) {
          CUDA_SUCCESS;
 }
 
+// Packed codes [rows][row_bytes], box [box_rows][64 bytes], 64-byte swizzle, out-of-range reads zero.
+bool make_packed_map(CUtensorMap* map, const uint8_t* base, int64_t rows, int64_t row_bytes, int box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)row_bytes, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)row_bytes};
+  cuuint32_t box[2] = {(cuuint32_t)BKP, (cuuint32_t)box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 int num_sms() {
   int dev = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return 148;
@@ -401,10 +372,12 @@ int num_sms() {
 cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
                                 int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, uint32_t* status,
                                 cudaStream_t stream) {
-  CUtensorMap ty;
+  CUtensorMap ty, ta, tb;
   memset(&ty, 0, sizeof(ty));
   int use_tma = (d_out % 4 == 0) ? 1 : 0;
   if (use_tma && !make_output_map(&ty, y, n, d_out)) use_tma = 0;
+  if (!make_packed_map(&ta, xq, n, d_in / 2, BM) || !make_packed_map(&tb, wq, d_out, d_in / 2, BN))
+    return cudaErrorInvalidValue;
   static std::once_flag attr_once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(attr_once, [] {
@@ -413,7 +386,7 @@ cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_
   if (attr_err != cudaSuccess) return attr_err;
   const int64_t tiles = ((n + BM - 1) / BM) * ((d_out + BN - 1) / BN);
   const int grid = (int)(tiles < num_sms() ? tiles : num_sms());
-  w4a4_gemm_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(ty, xq, wq, sx, sw, (int)n, (int)d_in, (int)d_out, y,
+  w4a4_gemm_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(ty, ta, tb, sx, sw, (int)n, (int)d_in, (int)d_out, y,
                                                               acc_out, use_tma, status);
   return cudaGetLastError();
 }
