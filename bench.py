@@ -38,6 +38,7 @@ FP8_PER_BF16 = 2.0          # nominal dense FP8 / BF16 tensor throughput ratio (
 FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}
 L2_FLUSH_BYTES = 256 << 20  # > 2x the 126.5 MiB L2
 LAUNCHES_PER_STEP = 7       # calib_cov 1, transform_quantize 3, w4a4_linear 1, sqnr 2
+DECODE_TOKENS = 32          # cat_w4a4_linear streams the weights (HBM-bound) up to this many tokens
 
 
 def parse_args():
@@ -63,6 +64,12 @@ def measured_peaks():
         return {"hbm_gbs": float(d["hbm_gbs"]), "bf16_tflops": float(d["bf16_tflops"]), "source": "measured"}
     except Exception:
         return dict(FALLBACK, source="fallback")
+
+
+def source_sha1(name):
+    import hashlib
+    with open(os.path.join(ROOT, "paper_2603_04359_gb300", "csrc", name), "rb") as f:
+        return hashlib.sha1(f.read()).hexdigest()
 
 
 def committed_json(name):
@@ -178,6 +185,27 @@ class OracleRunner:
         return O.sqnr_sums(self.y_ref, y_hat)
 
 
+def int8_peak_tops(dev, size=8192, reps=5):
+    """The int8 tensor-core peak of this GPU, measured with cuBLAS (outside any timed region)."""
+    try:
+        g = torch.Generator(device=dev).manual_seed(0)
+        a = torch.randint(-8, 8, (size, size), dtype=torch.int8, device=dev, generator=g)
+        b = torch.randint(-8, 8, (size, size), dtype=torch.int8, device=dev, generator=g)
+        for _ in range(2):
+            torch._int_mm(a, b)
+        best = float("inf")
+        for _ in range(reps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            torch._int_mm(a, b)
+            e1.record()
+            torch.cuda.synchronize()
+            best = min(best, e0.elapsed_time(e1))
+        return 2.0 * size ** 3 / (best / 1e3) / 1e12
+    except Exception:
+        return None
+
+
 def cpu_cores():
     try:
         return len(os.sched_getaffinity(0))
@@ -267,15 +295,22 @@ def ours_arm(args, rank, world, local):
 
     ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
 
-    def step(gemm_events=None):
+    def step(marks=None):
+        # marks: 5 events around the four calls, recorded on the launching stream
+        if marks:
+            marks[0].record(stream)
         cat.cat_calib_cov(xc, k, out=sigma)
+        if marks:
+            marks[1].record(stream)
         cat.cat_transform_quantize_act(x, T, k, xq=xq, x_scale=sx)
-        if gemm_events:
-            gemm_events[0].record(stream)
+        if marks:
+            marks[2].record(stream)
         cat.cat_w4a4_linear(xq, sx, Wq, sw, y=y)
-        if gemm_events:
-            gemm_events[1].record(stream)
+        if marks:
+            marks[3].record(stream)
         cat.cat_sqnr(y_ref, y, out=out3)
+        if marks:
+            marks[4].record(stream)
 
     for _ in range(args.warmup):
         step()
@@ -290,16 +325,16 @@ def ours_arm(args, rank, world, local):
     marks = []
     for i in range(args.steps):
         flush.fill_(i & 0xFF)                                # L2 flush, outside the timed events
-        s0, s1, g0, g1 = ev(), ev(), ev(), ev()
-        s0.record(stream)
-        step((g0, g1))
-        s1.record(stream)
-        marks.append((s0, s1, g0, g1))
+        m = [ev() for _ in range(5)]
+        step(m)
+        marks.append(m)
     torch.cuda.synchronize()
     clk = clocks.stop()
     barrier(world)
-    step_ms = statistics.mean(a.elapsed_time(b) for a, b, _, _ in marks)
-    gemm_ms = statistics.mean(c.elapsed_time(d) for _, _, c, d in marks)
+    step_ms = statistics.mean(m[0].elapsed_time(m[4]) for m in marks)
+    call_ms = {name: statistics.mean(m[j].elapsed_time(m[j + 1]) for m in marks)
+               for j, name in enumerate(("cat_calib_cov", "cat_transform_quantize_act", "cat_w4a4_linear", "cat_sqnr"))}
+    gemm_ms = call_ms["cat_w4a4_linear"]
     sqnr_db = float(out3[2].item())
     step_ms_max = max_over_ranks(step_ms, world)
 
@@ -349,11 +384,27 @@ def ours_arm(args, rank, world, local):
     peaks = measured_peaks()
     fp8_peak = peaks["bf16_tflops"] * FP8_PER_BF16
     gemm_tflops = 2.0 * n * d_in * d_out / (gemm_ms / 1e3) / 1e12
+    decode = n <= DECODE_TOKENS
+    kernel_src = "gemm_decode.cu" if decode else "gemm_tc.cu"
     traffic = None
-    tr = committed_json("traffic.json")
-    if tr and tr.get("workload") == cfg.name and tr.get("kernel_rev") == "w4a4_gemm_tc_v1":
-        traffic = tr.get("dram_bytes_per_launch")
-    int8 = committed_json("peaks_gb300.json") or {}
+    tr = committed_json("traffic.json") or {}
+    rec = tr.get(cfg.name, {})
+    if rec.get("source_sha1") == source_sha1(kernel_src):     # counters of this very kernel source
+        traffic = rec.get("dram_bytes_per_launch")
+    if decode:
+        # weight stream: packed W + w scales + packed x + x scales + y, once each
+        gemm_bytes = d_in * d_out // 2 + 4 * d_out + n * d_in // 2 + 4 * n + 4 * n * d_out
+        gbs = gemm_bytes / (gemm_ms / 1e3) / 1e9
+        roofline = {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                    "frac": gbs / peaks["hbm_gbs"], "traffic": traffic, "algorithmic_bytes": gemm_bytes,
+                    "kernel": "w4a4_gemm_decode (cat_w4a4_linear, n <= 32)",
+                    "peak_source": f"{peaks['source']} HBM copy {peaks['hbm_gbs']} GB/s"}
+    else:
+        roofline = {"bound": "tensor", "achieved": gemm_tflops, "peak": fp8_peak, "unit": "TFLOP/s",
+                    "frac": gemm_tflops / fp8_peak, "traffic": traffic,
+                    "kernel": "w4a4_gemm_tc (cat_w4a4_linear)",
+                    "peak_source": f"{peaks['source']} bf16 {peaks['bf16_tflops']} TFLOP/s x {FP8_PER_BF16} "
+                                   "(FP8 engine, nominal FP8/BF16 ratio)"}
     line = {
         "metric": METRIC, "value": world * n / (step_ms_max / 1e3), "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms_max, "higher_is_better": True,
@@ -361,17 +412,15 @@ def ours_arm(args, rank, world, local):
         "config": {"workload": cfg.name, "n_tokens": n, "d_in": d_in, "d_out": d_out, "k": k, "n_calib": cfg.n_calib,
                    "transform": args.kind, "input_dtype": cfg.dtype, "parallelism": f"replicas x{world}",
                    "l2": "flushed between timed steps (256 MiB write)"},
-        "roofline": {"bound": "tensor", "achieved": gemm_tflops, "peak": fp8_peak, "unit": "TFLOP/s",
-                     "frac": gemm_tflops / fp8_peak, "traffic": traffic,
-                     "kernel": "w4a4_gemm_tc (cat_w4a4_linear)",
-                     "peak_source": f"{peaks['source']} bf16 {peaks['bf16_tflops']} TFLOP/s x {FP8_PER_BF16} "
-                                    "(FP8 engine, nominal FP8/BF16 ratio)"},
-        "sqnr_db": sqnr_db, "gemm_ms": gemm_ms, "effective_tops": gemm_tflops,
+        "roofline": roofline,
+        "sqnr_db": sqnr_db, "gemm_ms": gemm_ms, "effective_tops": gemm_tflops, "call_ms": call_ms,
         "gpu_launches": LAUNCHES_PER_STEP * args.steps, "clocks": clk,
     }
-    if int8.get("int8_tops"):
-        line["int8_peak"] = {"tops": int8["int8_tops"], "frac": gemm_tflops / int8["int8_tops"],
-                             "source": int8.get("int8_source", "")}
+    if not decode:
+        i8 = int8_peak_tops(dev)
+        if i8:
+            line["int8_peak"] = {"tops": i8, "frac": gemm_tflops / i8,
+                                 "source": "measured now: torch._int_mm int8 8192^3, best of 5 (cuBLAS IMMA)"}
     if e2e:
         line["e2e"] = e2e
     if world == 1 and not args.no_cpu_baseline:
@@ -381,11 +430,13 @@ def ours_arm(args, rank, world, local):
 
 def main():
     args = parse_args()
-    rank, world, local = dist_setup()
     if args.impl == "reference":
-        reference_arm(args, rank, world)
-    else:
-        ours_arm(args, rank, world, local)
+        # the oracle runs on rank 0's host cores only; the other ranks exit without work and
+        # no process group is needed
+        reference_arm(args, int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")))
+        return
+    rank, world, local = dist_setup()
+    ours_arm(args, rank, world, local)
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
