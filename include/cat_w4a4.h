@@ -120,6 +120,28 @@ cat_status cat_quantize_weights(const void* W, cat_dtype dtype, int64_t d_out, i
                                 cat_stream_t stream);
 
 /*
+ * cat_quantize_weights_noalloc -- cat_quantize_weights without device allocation.  No counterpart
+ * in the paper: it exists for callers that cannot take new device memory mid-run, e.g. a process
+ * that has handed all free device memory to its own pool and re-quantizes a layer later (after
+ * re-calibration), where a new allocation would fail or evict that pool.
+ * Same arguments, steps and results as cat_quantize_weights.  Its two temporaries (the float64
+ * Sigma_w blocks and the float32 blocks (T_b^{-1})^T, 12 bytes per element of d_in * k) live in a
+ * fixed 12 MiB scratch area that the library reserves statically on every device it is loaded on.
+ *   Limit: d_in * k <= CAT_PREP_NOALLOC_MAX_DK; a larger call returns CAT_ERR_SHAPE before any
+ *   CUDA call and writes nothing.
+ *   Setup: the first call on a device looks up the scratch address (cudaGetSymbolAddress) with
+ *   that device current; make that first call before any stream capture.
+ *   Concurrency: every call on a device shares the one scratch area, so calls that overlap in
+ *   time (other host threads or streams) race; the caller must serialize them.  Each call
+ *   synchronizes its stream before returning, so consecutive calls are safe.
+ */
+#define CAT_PREP_NOALLOC_MAX_DK 1048576
+cat_status cat_quantize_weights_noalloc(const void* W, cat_dtype dtype, int64_t d_out, int64_t d_in, int32_t k,
+                                        cat_tkind kind, const double* sigma_x_blocks, int64_t n_calib,
+                                        const float* rht_signs, float* T_blocks, uint8_t* Wq, float* w_scale,
+                                        cat_stream_t stream);
+
+/*
  * cat_build_transform_host -- the host part of cat_quantize_weights, exposed for inspection: the
  * block transform T and its inverse in float64 (Sec. 4, Eq. 7 and Eq. 10).  All pointers are HOST.
  *   sigma_x_blocks [d_in/k][k][k] sums over n_calib tokens (CAT only); sigma_w_blocks [d_in/k][k][k]

@@ -58,6 +58,7 @@ def load_library() -> ctypes.CDLL:
         "cat_version": ([], I),
         "cat_calib_cov": ([P, I, I64, I64, I32, P, I, P], I),
         "cat_quantize_weights": ([P, I, I64, I64, I32, I, P, I64, P, P, P, P, P], I),
+        "cat_quantize_weights_noalloc": ([P, I, I64, I64, I32, I, P, I64, P, P, P, P, P], I),
         "cat_build_transform_host": ([I, I64, I32, P, I64, P, P, P, P], I),
         "cat_transform_quantize_act": ([P, I, I64, I64, I32, P, P, P, P], I),
         "cat_w4a4_linear": ([P, P, P, P, I64, I64, I64, P, P, P], I),
@@ -138,6 +139,30 @@ def cat_quantize_weights(W: torch.Tensor, k: int, kind: str, sigma_x: Optional[t
         _ptr(W), _dtype(W), d_out, d_in, k, KIND[kind], _ptr(sigma_x), int(n_calib),
         None if signs is None else signs.ctypes.data_as(ctypes.c_void_p), _ptr(T), _ptr(Wq), _ptr(sw), _stream(dev))
     _check("cat_quantize_weights", st)
+    return T, Wq, sw
+
+
+def cat_quantize_weights_noalloc(W: torch.Tensor, k: int, kind: str, sigma_x: Optional[torch.Tensor] = None,
+                                 n_calib: int = 0, rht_signs=None, out=None) -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
+    """cat_quantize_weights with the library's static scratch instead of device allocations
+    (d_in * k <= 1048576).  ``out`` = (T_blocks, Wq, w_scale) preallocated by the caller, or None."""
+    _need(W, "W")
+    d_out, d_in = W.shape
+    dev = W.device
+    if out is None:
+        out = (torch.empty((d_in // k, k, k), dtype=torch.float32, device=dev),
+               torch.empty((d_out, d_in // 2), dtype=torch.uint8, device=dev),
+               torch.empty((d_out,), dtype=torch.float32, device=dev))
+    T, Wq, sw = out
+    signs = None
+    if rht_signs is not None:
+        signs = np.ascontiguousarray(np.asarray(rht_signs, dtype=np.float32))
+    if sigma_x is not None:
+        _need(sigma_x, "sigma_x")
+    st = load_library().cat_quantize_weights_noalloc(
+        _ptr(W), _dtype(W), d_out, d_in, k, KIND[kind], _ptr(sigma_x), int(n_calib),
+        None if signs is None else signs.ctypes.data_as(ctypes.c_void_p), _ptr(T), _ptr(Wq), _ptr(sw), _stream(dev))
+    _check("cat_quantize_weights_noalloc", st)
     return T, Wq, sw
 
 

@@ -69,6 +69,40 @@ uint32_t* status_word(cudaError_t* err) {
   return cache[dev];
 }
 
+// Scratch of cat_quantize_weights_noalloc: it makes no device allocation of its own.
+constexpr int64_t kPrepMaxDK = CAT_PREP_NOALLOC_MAX_DK;                 // largest d_in * k
+constexpr size_t kPrepSigmaBytes = (size_t)kPrepMaxDK * sizeof(double);  // Sigma_w blocks
+constexpr size_t kPrepScratchBytes = kPrepSigmaBytes + (size_t)kPrepMaxDK * sizeof(float);  // + A_w blocks
+
+}  // namespace
+
+// Reserved with the module on each device that loads the library (12 MiB).
+static __device__ __align__(256) unsigned char g_prep_scratch[kPrepScratchBytes];
+
+namespace {
+
+// Address of this device's prep scratch.  Looked up once per device with that device current;
+// the first cat_quantize_weights_noalloc call on a device does the lookup.
+unsigned char* prep_scratch(cudaError_t* err) {
+  static std::mutex mu;
+  static unsigned char* cache[64] = {nullptr};
+  int dev = 0;
+  *err = cudaGetDevice(&dev);
+  if (*err != cudaSuccess) return nullptr;
+  if (dev < 0 || dev >= 64) {
+    *err = cudaErrorInvalidDevice;
+    return nullptr;
+  }
+  std::lock_guard<std::mutex> lock(mu);
+  if (!cache[dev]) {
+    void* p = nullptr;
+    *err = cudaGetSymbolAddress(&p, g_prep_scratch);
+    if (*err != cudaSuccess) return nullptr;
+    cache[dev] = static_cast<unsigned char*>(p);
+  }
+  return cache[dev];
+}
+
 // The kernels are built for sm_103a only.
 cat_status check_device() {
   int dev = 0, major = 0, minor = 0;
@@ -217,6 +251,77 @@ cat_status cat_quantize_weights(const void* W, cat_dtype dtype, int64_t d_out, i
   if (e == cudaSuccess) e = cat::launch_transform_quantize(W, (int)dtype, d_out, d_in, k, aw_d, Wq, w_scale, status, s);
   cudaFreeAsync(aw_d, s);
   cudaError_t e2 = cudaStreamSynchronize(s);  // host buffers above must outlive the copies
+  if (e != cudaSuccess) return cuda_fail(e, "weight quantization");
+  if (e2 != cudaSuccess) return cuda_fail(e2, "cudaStreamSynchronize");
+  return ok();
+}
+
+// Weight preparation that takes no device memory (no counterpart in the paper).  Same steps and
+// results as cat_quantize_weights; its two temporaries live in g_prep_scratch instead of
+// stream-ordered allocations.  Callers that cannot allocate: a process that has handed all free
+// device memory to its own pool up front (a serving engine's cache pool) and re-quantizes a
+// layer later, e.g. after re-calibration -- a new allocation there fails or has to evict the
+// pool.  The scratch is shared by every call on a device, so overlapping calls race.
+cat_status cat_quantize_weights_noalloc(const void* W, cat_dtype dtype, int64_t d_out, int64_t d_in, int32_t k,
+                                        cat_tkind kind, const double* sigma_x_blocks, int64_t n_calib,
+                                        const float* rht_signs, float* T_blocks, uint8_t* Wq, float* w_scale,
+                                        cat_stream_t stream) {
+  if (dtype != CAT_F32 && dtype != CAT_BF16) return fail(CAT_ERR_INVALID_ARG, "unknown dtype");
+  if (kind != CAT_T_IDENTITY && kind != CAT_T_RHT && kind != CAT_T_CAT) return fail(CAT_ERR_INVALID_ARG, "unknown kind");
+  if (d_out <= 0) return fail(CAT_ERR_SHAPE, "d_out must be >= 1");
+  cat_status st = check_din(d_in);
+  if (st != CAT_OK) return st;
+  if (!valid_k(k) || d_in % k != 0) return fail(CAT_ERR_SHAPE, "k must be one of 16..256 (power of two) and divide d_in");
+  if (d_in * (int64_t)k > kPrepMaxDK)
+    return fail(CAT_ERR_SHAPE, "cat_quantize_weights_noalloc: d_in * k = " + std::to_string(d_in * (int64_t)k) +
+                                   " exceeds the static scratch limit CAT_PREP_NOALLOC_MAX_DK = " +
+                                   std::to_string(kPrepMaxDK) + "; use cat_quantize_weights");
+  if (!W || !T_blocks || !Wq || !w_scale) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (kind == CAT_T_CAT && (!sigma_x_blocks || n_calib < 1))
+    return fail(CAT_ERR_INVALID_ARG, "CAT needs sigma_x_blocks and n_calib >= 1");
+  if (kind == CAT_T_RHT && !rht_signs) return fail(CAT_ERR_INVALID_ARG, "RHT needs rht_signs");
+  if (!aligned16(W) || !aligned16(T_blocks) || !aligned16(Wq) || !aligned16(w_scale) ||
+      (sigma_x_blocks && !aligned16(sigma_x_blocks)))
+    return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  if ((st = check_device()) != CAT_OK) return st;
+
+  cudaStream_t s = (cudaStream_t)stream;
+  cudaError_t e;
+  unsigned char* scratch = prep_scratch(&e);
+  if (!scratch) return cuda_fail(e, "cudaGetSymbolAddress(prep scratch)");
+  uint32_t* status = status_word(&e);
+  if (!status) return cuda_fail(e, "status word");
+  double* sw_d = reinterpret_cast<double*>(scratch);                    // Sigma_w blocks, float64
+  float* aw_d = reinterpret_cast<float*>(scratch + kPrepSigmaBytes);    // (T_b^{-1})^T blocks, float32
+  const int64_t nb = d_in / k;
+  const size_t kk = (size_t)k * k, nblk = (size_t)nb * kk;
+  std::vector<double> sx_h, sw_h;
+  if (kind == CAT_T_CAT) {
+    // The Sigma_w sums accumulate into the scratch, so it must start at zero on every call.
+    e = cudaMemsetAsync(sw_d, 0, nblk * sizeof(double), s);
+    if (e == cudaSuccess) e = cat::launch_calib_cov(W, (int)dtype, d_out, d_in, k, sw_d, 1, status, s);
+    sx_h.resize(nblk);
+    sw_h.resize(nblk);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(sx_h.data(), sigma_x_blocks, nblk * sizeof(double), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(sw_h.data(), sw_d, nblk * sizeof(double), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(e, "Sigma_w / Sigma_x readback");
+  }
+  std::vector<double> T(nblk), Ti(nblk);
+  st = cat_build_transform_host(kind, d_in, k, sx_h.empty() ? nullptr : sx_h.data(), n_calib,
+                                sw_h.empty() ? nullptr : sw_h.data(), rht_signs, T.data(), Ti.data());
+  if (st != CAT_OK) return st;
+  std::vector<float> Tf(nblk), Awf(nblk);
+  for (int64_t b = 0; b < nb; ++b)
+    for (int i = 0; i < k; ++i)
+      for (int j = 0; j < k; ++j) {
+        Tf[b * kk + (size_t)i * k + j] = (float)T[b * kk + (size_t)i * k + j];
+        Awf[b * kk + (size_t)i * k + j] = (float)Ti[b * kk + (size_t)j * k + i];
+      }
+  e = cudaMemcpyAsync(T_blocks, Tf.data(), nblk * sizeof(float), cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(aw_d, Awf.data(), nblk * sizeof(float), cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cat::launch_transform_quantize(W, (int)dtype, d_out, d_in, k, aw_d, Wq, w_scale, status, s);
+  cudaError_t e2 = cudaStreamSynchronize(s);  // host buffers and the scratch are in use until here
   if (e != cudaSuccess) return cuda_fail(e, "weight quantization");
   if (e2 != cudaSuccess) return cuda_fail(e2, "cudaStreamSynchronize");
   return ok();
