@@ -82,6 +82,10 @@ const char* cat_last_error(void);
 /* Library version: major * 10000 + minor * 100 + patch. */
 int cat_version(void);
 
+/* Number of kernels the library has launched in this process so far (a host counter bumped at
+ * every launch site, also during stream capture).  Diagnostic; no counterpart in the paper. */
+unsigned long long cat_kernel_launches(void);
+
 /*
  * cat_calib_cov -- calibration autocorrelation blocks (Sec. 4: Sigma_x = E[x x^T]; Eq. 10 uses its
  * k x k diagonal blocks).

@@ -56,6 +56,7 @@ def load_library() -> ctypes.CDLL:
         "cat_status_string": ([I], ctypes.c_char_p),
         "cat_last_error": ([], ctypes.c_char_p),
         "cat_version": ([], I),
+        "cat_kernel_launches": ([], ctypes.c_ulonglong),
         "cat_calib_cov": ([P, I, I64, I64, I32, P, I, P], I),
         "cat_quantize_weights": ([P, I, I64, I64, I32, I, P, I64, P, P, P, P, P], I),
         "cat_quantize_weights_noalloc": ([P, I, I64, I64, I32, I, P, I64, P, P, P, P, P], I),
@@ -77,7 +78,8 @@ def exported_symbols() -> list:
     """Names of the entry points declared in ``include/cat_w4a4.h``."""
     with open(_HEADER) as f:
         text = f.read()
-    return sorted(set(re.findall(r"^\s*(?:cat_status|const char\*|int)\s+(cat_\w+)\s*\(", text, re.M)))
+    return sorted(set(re.findall(r"^\s*(?:cat_status|const char\*|int|unsigned long long)\s+(cat_\w+)\s*\(", text,
+                                 re.M)))
 
 
 def _check(func: str, status: int) -> None:
@@ -107,6 +109,11 @@ def _need(t: torch.Tensor, name: str) -> None:
 
 def cat_version() -> int:
     return int(load_library().cat_version())
+
+
+def cat_kernel_launches() -> int:
+    """Kernels the library has launched in this process (diagnostic host counter)."""
+    return int(load_library().cat_kernel_launches())
 
 
 def cat_calib_cov(x: torch.Tensor, k: int, out: Optional[torch.Tensor] = None, accumulate: bool = False) -> torch.Tensor:

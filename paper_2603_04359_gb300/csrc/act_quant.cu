@@ -152,10 +152,13 @@ cudaError_t launch_k(const Tin* x, int64_t n, int64_t d, const float* A, uint8_t
   dim3 grid((unsigned)row_tiles, (unsigned)ny);
   uint32_t* amax = reinterpret_cast<uint32_t*>(scale);
   uint32_t* words = reinterpret_cast<uint32_t*>(codes);
+  note_launch();
   k0<<<grid, C::THREADS, C::SMEM, stream>>>(x, n, d, A, amax, words, status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  note_launch();
   k1<<<grid, C::THREADS, C::SMEM, stream>>>(x, n, d, A, amax, words, status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  note_launch();
   finalize_scale_kernel<<<(unsigned)((n + 255) / 256), 256, 0, stream>>>(amax, n, status);
   return cudaGetLastError();
 }
@@ -179,15 +182,22 @@ bool transform_quantize_tc_supported(int dtype, int k, int64_t n, int64_t d);
 cudaError_t launch_transform_quantize_tc(const void* x, int64_t n, int64_t d, int k, const float* A, uint32_t* amax,
                                          uint32_t* words, uint32_t* status, cudaStream_t stream);
 
+cudaError_t launch_transform_quantize_tc_fused(const void* x, int64_t n, int64_t d, int k, const float* A,
+                                               uint32_t* amax, uint32_t* words, uint32_t* status, cudaStream_t stream);
+
 cudaError_t launch_transform_quantize(const void* x, int dtype, int64_t n, int64_t d, int k, const float* A,
                                       uint8_t* codes, float* scale, uint32_t* status, cudaStream_t stream) {
   if (n == 0) return cudaSuccess;
   if (transform_quantize_tc_supported(dtype, k, n, d)) {  // bf16 rows: tensor-core path
     uint32_t* amax = reinterpret_cast<uint32_t*>(scale);
+    const cudaError_t ef = launch_transform_quantize_tc_fused(x, n, d, k, A, amax, reinterpret_cast<uint32_t*>(codes),
+                                                              status, stream);
+    if (ef != cudaErrorNotSupported) return ef;  // done (or failed) in one launch
     cudaError_t e = cudaMemsetAsync(scale, 0, (size_t)n * sizeof(float), stream);
     if (e == cudaSuccess) e = launch_transform_quantize_tc(x, n, d, k, A, amax, reinterpret_cast<uint32_t*>(codes),
                                                            status, stream);
     if (e != cudaSuccess) return e;
+    note_launch();
     finalize_scale_kernel<<<(unsigned)((n + 255) / 256), 256, 0, stream>>>(amax, n, status);
     return cudaGetLastError();
   }

@@ -14,6 +14,7 @@
 //   pass 0: atomicMax of the row maxima into the scale buffer (float bits, non-negative),
 //   pass 1: recompute, q = clamp(rint(v' * (7 / max)), -7, 7), pack SM4x8, store.
 // Warps: 0 TMA producer + TMEM allocator, 1 MMA issuer, 4..7 epilogue, 8..15 converters.
+#include <atomic>
 #include <cstring>
 #include <mutex>
 
@@ -26,6 +27,7 @@ constexpr int TM = 128;                 // rows per tile
 constexpr int kThreads = 512;
 constexpr int kEpiWarp0 = 4, kCvtWarp0 = 8, kCvtWarps = 8;
 constexpr int kXStages = 2;
+static_assert((64 * 64 / 8) % (kCvtWarps * 32) == 0, "converter items must divide evenly");
 
 template <int K>
 struct TcCfg {
@@ -57,9 +59,67 @@ __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint6
       : "memory");
 }
 
+// Units (block b, 128-row tile) of CTA c, block-major.  With at least as many CTAs as blocks, every
+// CTA works inside one block (its split of T_b is made once) and the CTAs of a block share its tiles
+// evenly; otherwise CTAs take contiguous ranges of units.
+__host__ __device__ inline void unit_range(int c, int grid, int nb, int tiles, int64_t* u0, int64_t* u1) {
+  if (grid >= nb) {
+    const int b = (int)((int64_t)c * nb / grid);
+    const int c_lo = (int)(((int64_t)b * grid + nb - 1) / nb);
+    const int c_hi = (int)(((int64_t)(b + 1) * grid + nb - 1) / nb);
+    const int m = c_hi - c_lo, i = c - c_lo;
+    *u0 = (int64_t)b * tiles + (int64_t)tiles * i / m;
+    *u1 = (int64_t)b * tiles + (int64_t)tiles * (i + 1) / m;
+  } else {
+    const int64_t units = (int64_t)nb * tiles;
+    *u0 = units * c / grid;
+    *u1 = units * (c + 1) / grid;
+  }
+}
+
 __device__ __forceinline__ uint32_t bf16x2_bits(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// Split the fp32 block A_b (row-major k x k, row i = output i) into bf16 H, M, L in the MMA's
+// 128B-swizzled K-major layout; `ct` is the thread's index among the converter threads.
+template <int K>
+__device__ __forceinline__ void split_block(const float* __restrict__ Ab, uint8_t* ts, int ct) {
+  using C = TcCfg<K>;
+  // all loads first (the block is read from L2/HBM once per block change: keep them in flight together)
+  constexpr int kIt = K * K / 8 / (kCvtWarps * 32);
+  float4 pv[kIt], qv[kIt];
+#pragma unroll
+  for (int it = 0; it < kIt; ++it) {  // 8 consecutive inputs of one output row per item
+    const int ch = ct + it * kCvtWarps * 32;
+    const int i = ch / (K / 8), j0 = (ch % (K / 8)) * 8;
+    pv[it] = __ldg(reinterpret_cast<const float4*>(Ab + (size_t)i * K + j0));
+    qv[it] = __ldg(reinterpret_cast<const float4*>(Ab + (size_t)i * K + j0 + 4));
+  }
+#pragma unroll
+  for (int it = 0; it < kIt; ++it) {
+    const int ch = ct + it * kCvtWarps * 32;
+    const int i = ch / (K / 8), j0 = (ch % (K / 8)) * 8;
+    const float4 p = pv[it], q = qv[it];
+    const float v[8] = {p.x, p.y, p.z, p.w, q.x, q.y, q.z, q.w};
+    uint32_t hw[4], mw[4], lw[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float a0 = v[2 * e], a1 = v[2 * e + 1];
+      const float h0 = __bfloat162float(__float2bfloat16_rn(a0)), h1 = __bfloat162float(__float2bfloat16_rn(a1));
+      const float r0 = a0 - h0, r1 = a1 - h1;  // exact
+      const float m0 = __bfloat162float(__float2bfloat16_rn(r0)), m1 = __bfloat162float(__float2bfloat16_rn(r1));
+      hw[e] = bf16x2_bits(h0, h1);
+      mw[e] = bf16x2_bits(m0, m1);
+      lw[e] = bf16x2_bits(r0 - m0, r1 - m1);
+    }
+    const int atom = j0 / 64, chunk = (j0 % 64) / 8;
+    const uint32_t off = atom * (K * 128) + i * 128 + ((chunk ^ (i & 7)) << 4);
+    *reinterpret_cast<uint4*>(ts + off) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+    *reinterpret_cast<uint4*>(ts + C::SPLIT + off) = make_uint4(mw[0], mw[1], mw[2], mw[3]);
+    *reinterpret_cast<uint4*>(ts + 2 * C::SPLIT + off) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+  }
 }
 
 template <int K, int PASS>
@@ -78,9 +138,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int nb = d / K;
   const int num_tiles = (n + TM - 1) / TM;
-  const int64_t units = (int64_t)nb * num_tiles;
-  const int64_t u0 = units * blockIdx.x / gridDim.x;
-  const int64_t u1 = units * (blockIdx.x + 1) / gridDim.x;
+  int64_t u0, u1;
+  unit_range(blockIdx.x, gridDim.x, nb, num_tiles, &u0, &u1);
 
   if (tid == 0) {
     for (int s = 0; s < kXStages; ++s) {
@@ -173,29 +232,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (b == cur_b) continue;
       if (version > 0 && !(ok = mbar_wait_bounded(&bars->t_empty, (version - 1) & 1, abort_flag))) break;
       cur_b = b;
-      const float* Ab = A + (size_t)b * K * K;
-      for (int ch = ct; ch < K * K / 8; ch += kCvtWarps * 32) {  // 8 consecutive inputs of one output row
-        const int i = ch / (K / 8), j0 = (ch % (K / 8)) * 8;
-        const float4 p = *reinterpret_cast<const float4*>(Ab + (size_t)i * K + j0);
-        const float4 q = *reinterpret_cast<const float4*>(Ab + (size_t)i * K + j0 + 4);
-        const float v[8] = {p.x, p.y, p.z, p.w, q.x, q.y, q.z, q.w};
-        uint32_t hw[4], mw[4], lw[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float a0 = v[2 * e], a1 = v[2 * e + 1];
-          const float h0 = __bfloat162float(__float2bfloat16_rn(a0)), h1 = __bfloat162float(__float2bfloat16_rn(a1));
-          const float r0 = a0 - h0, r1 = a1 - h1;  // exact
-          const float m0 = __bfloat162float(__float2bfloat16_rn(r0)), m1 = __bfloat162float(__float2bfloat16_rn(r1));
-          hw[e] = bf16x2_bits(h0, h1);
-          mw[e] = bf16x2_bits(m0, m1);
-          lw[e] = bf16x2_bits(r0 - m0, r1 - m1);
-        }
-        const int atom = j0 / 64, chunk = (j0 % 64) / 8;
-        const uint32_t off = atom * (K * 128) + i * 128 + ((chunk ^ (i & 7)) << 4);
-        *reinterpret_cast<uint4*>(ts + off) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-        *reinterpret_cast<uint4*>(ts + C::SPLIT + off) = make_uint4(mw[0], mw[1], mw[2], mw[3]);
-        *reinterpret_cast<uint4*>(ts + 2 * C::SPLIT + off) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
-      }
+      split_block<K>(A + (size_t)b * K * K, ts, ct);
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(&bars->t_full);
@@ -266,6 +303,268 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// ---- single-launch variant: x' stays in tensor memory between the two row-wide phases ---------
+//
+// When every CTA's units fit in tensor memory at once (units per CTA x K <= 512 columns), one
+// cooperative launch does both passes: phase A runs the MMAs once, keeps each unit's x' tile in its
+// own TMEM columns and records the row maxima; a grid-wide barrier; phase B reads the final maxima,
+// quantizes the tiles still in TMEM and writes the codes; a second barrier; then the CTAs holding
+// block 0 turn the row maxima into the steps s = max / 7 in place.  The barrier counters live in a
+// small static array of slots (one per launch in flight, zeroed by the preparation kernel that also
+// zeroes the maxima); every wait is bounded.
+constexpr int kSyncSlots = 64;
+__device__ __align__(16) uint32_t g_tq_sync[kSyncSlots][4];
+
+__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 2, 128;" ::: "memory"); }
+
+// All CTAs' epilogue warps meet here (the other warps of a CTA never wait on it).  Bounded: a
+// barrier that has not filled in kWaitLimitNs raises the abort flag.
+__device__ __forceinline__ void grid_barrier(uint32_t* ctr, uint32_t expected, volatile int* abort_flag, bool leader) {
+  __threadfence();
+  epi_bar();
+  if (leader) {
+    atomicAdd(ctr, 1u);
+    const uint64_t t0 = globaltimer_ns();
+    for (uint32_t it = 0; ld_acquire_gpu(ctr) < expected; ++it) {
+      if ((it & 63u) == 63u && (*abort_flag || globaltimer_ns() - t0 > kWaitLimitNs)) {
+        *abort_flag = 1;
+        break;
+      }
+    }
+    __threadfence();
+  }
+  epi_bar();
+}
+
+__global__ void tq_prep_kernel(uint32_t* __restrict__ amax_bits, int64_t n, uint32_t* __restrict__ sync) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) amax_bits[i] = 0u;
+  if (i < 4) sync[i] = 0u;
+}
+
+template <int K>
+__global__ void __launch_bounds__(kThreads, 1)
+    transform_quant_tc_fused_kernel(const __grid_constant__ CUtensorMap tmX, const float* __restrict__ A, int n,
+                                    int d, uint32_t* __restrict__ amax_bits, uint32_t* __restrict__ codes,
+                                    uint32_t* __restrict__ sync, uint32_t* __restrict__ status) {
+  using C = TcCfg<K>;
+  constexpr int kMaxUnits = 512 / K;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* xs = smem + C::X_OFF;
+  uint8_t* ts = smem + C::T_OFF;
+  TcBars* bars = reinterpret_cast<TcBars*>(smem + C::BAR_OFF);
+  uint64_t* unit_full = reinterpret_cast<uint64_t*>(bars + 1);   // one per unit (each used once)
+  volatile int* abort_flag = &bars->abort;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int nb = d / K;
+  const int num_tiles = (n + TM - 1) / TM;
+  int64_t u0, u1;
+  unit_range(blockIdx.x, gridDim.x, nb, num_tiles, &u0, &u1);
+  if (u1 - u0 > kMaxUnits) u1 = u0 + kMaxUnits;          // the launcher guarantees this never cuts
+
+  if (tid == 0) {
+    for (int st = 0; st < kXStages; ++st) {
+      mbar_init(&bars->x_full[st], 1);
+      mbar_init(&bars->x_empty[st], 1);
+    }
+    for (int j = 0; j < kMaxUnits; ++j) mbar_init(&unit_full[j], 1);
+    mbar_init(&bars->t_full, kCvtWarps);
+    mbar_init(&bars->t_empty, 1);
+    mbar_init(&bars->mma_done, 1);
+    bars->abort = 0;
+    fence_mbar_init();
+  }
+  __syncwarp();
+  if (warp == 0) tmem_alloc(&bars->tmem_addr, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bars->tmem_addr;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      prefetch_tensormap(&tmX);
+      bool ok = true;
+      uint32_t j = 0;
+      for (int64_t u = u0; u < u1 && ok; ++u, ++j) {
+        const int b = (int)(u / num_tiles), tile = (int)(u % num_tiles);
+        const uint32_t st = j % kXStages;
+        if (j >= kXStages && !(ok = mbar_wait_bounded(&bars->x_empty[st], ((j / kXStages) - 1) & 1, abort_flag))) break;
+        mbar_arrive_expect_tx(&bars->x_full[st], C::X_STAGE);
+#pragma unroll
+        for (int a = 0; a < C::ATOMS; ++a)
+          tma_load_2d(xs + st * C::X_STAGE + a * (TM * 128), &tmX, b * K + 64 * a, tile * TM, &bars->x_full[st]);
+      }
+      const uint32_t issued = j, first = issued > kXStages ? issued - kXStages : 0;
+      volatile int no_abort = 0;
+      for (uint32_t q = first; q < issued; ++q)
+        mbar_wait_bounded(&bars->x_full[q % kXStages], (q / kXStages) & 1, &no_abort);
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer: unit j -> columns j K
+    if (lane == 0) {
+      bool ok = true;
+      uint32_t j = 0, version = 0;
+      int cur_b = -1;
+      for (int64_t u = u0; u < u1 && ok; ++u, ++j) {
+        const int b = (int)(u / num_tiles);
+        if (b != cur_b) {
+          if (!(ok = mbar_wait_bounded(&bars->t_full, version & 1, abort_flag))) break;
+          ++version;
+          cur_b = b;
+        }
+        const uint32_t st = j % kXStages;
+        if (!(ok = mbar_wait_bounded(&bars->x_full[st], (j / kXStages) & 1, abort_flag))) break;
+        tc_fence_after();
+        const uint32_t dcol = tmem + j * K;
+        const uint32_t xbase = smem_u32(xs + st * C::X_STAGE);
+        const uint32_t tbase = smem_u32(ts);
+#pragma unroll
+        for (int kk = 0; kk < K / 16; ++kk) {
+          const uint32_t a_off = (kk >> 2) * (TM * 128) + (kk & 3) * 32;
+          const uint32_t b_off = (kk >> 2) * (K * 128) + (kk & 3) * 32;
+          const uint64_t da = sdesc_kmajor_sw128(xbase + a_off);
+#pragma unroll
+          for (int sp = 0; sp < 3; ++sp)
+            mma_bf16(dcol, da, sdesc_kmajor_sw128(tbase + sp * C::SPLIT + b_off), C::IDESC, (kk | sp) != 0);
+        }
+        mma_commit(&bars->x_empty[st]);
+        mma_commit(&unit_full[j]);
+        const bool last_of_block = (u + 1 >= u1) || ((int)((u + 1) / num_tiles) != b);
+        if (last_of_block) mma_commit(&bars->t_empty);
+      }
+      mma_commit(&bars->mma_done);
+      volatile int no_abort = 0;
+      mbar_wait_bounded(&bars->mma_done, 0, &no_abort);
+    }
+  } else if (warp >= kCvtWarp0) {
+    // ---------------------------------------------------------------- split A_b into bf16 H, M, L
+    const int ct = tid - kCvtWarp0 * 32;
+    bool ok = true;
+    uint32_t version = 0;
+    int cur_b = -1;
+    for (int64_t u = u0; u < u1 && ok; ++u) {
+      const int b = (int)(u / num_tiles);
+      if (b == cur_b) continue;
+      if (version > 0 && !(ok = mbar_wait_bounded(&bars->t_empty, (version - 1) & 1, abort_flag))) break;
+      cur_b = b;
+      split_block<K>(A + (size_t)b * K * K, ts, ct);
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars->t_full);
+      ++version;
+    }
+  } else if (warp >= kEpiWarp0) {
+    // ---------------------------------------------------------------- epilogue: one row per thread
+    const int quad = warp & 3;
+    const bool leader = warp == kEpiWarp0 && lane == 0;
+    const int64_t words_per_row = d / 8;
+    const int nu = (int)(u1 - u0);
+    bool finite = true;
+    // phase A: row maxima of every unit's tile
+    for (int j = 0; j < nu; ++j) {
+      const int tile = (int)((u0 + j) % num_tiles);
+      const int t = tile * TM + quad * 32 + lane;
+      const bool got = !*abort_flag && mbar_wait_bounded(&unit_full[j], 0, abort_flag);
+      if (!__all_sync(0xFFFFFFFFu, got)) break;        // warp-uniform: TMEM loads need the whole warp
+      tc_fence_after();
+      float m = 0.f;
+#pragma unroll 1
+      for (int c = 0; c < K / 32; ++c) {
+        uint32_t r[32];
+        __syncwarp();
+        CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + j * K + c * 32, r);
+        tmem_ld_wait();
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          const float v = __uint_as_float(r[e]);
+          finite &= isfinite(v);
+          m = fmaxf(m, fabsf(v));
+        }
+      }
+      if (t < n) atomicMax(&amax_bits[t], __float_as_uint(m));
+    }
+    if (!finite) report(status, kStatusNonFinite);
+    grid_barrier(&sync[0], gridDim.x, abort_flag, leader);
+    // phase B: quantize the tiles still in tensor memory with the final row maxima
+    float a_keep[kMaxUnits];
+#pragma unroll
+    for (int j = 0; j < kMaxUnits; ++j) a_keep[j] = 0.f;
+    if (!__any_sync(0xFFFFFFFFu, *abort_flag)) {
+#pragma unroll
+      for (int j = 0; j < kMaxUnits; ++j) {
+        if (j >= nu) break;
+        const int64_t u = u0 + j;
+        const int b = (int)(u / num_tiles), tile = (int)(u % num_tiles);
+        const int t = tile * TM + quad * 32 + lane;
+        float a = 0.f;
+        if (t < n) a = __uint_as_float(__ldcg(&amax_bits[t]));
+        a_keep[j] = a;
+        const float inv = (isfinite(a) && a > 0.f) ? __fdiv_rn(7.0f, a) : 0.f;
+        tc_fence_after();
+#pragma unroll 1
+        for (int c = 0; c < K / 32; ++c) {
+          uint32_t r[32];
+          __syncwarp();
+          CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + j * K + c * 32, r);
+          tmem_ld_wait();
+          if (t < n) {
+            uint32_t w[4];
+#pragma unroll
+            for (int g = 0; g < 4; ++g) {
+              int q[8];
+#pragma unroll
+              for (int e = 0; e < 8; ++e) {
+                const float v = __uint_as_float(r[8 * g + e]) * inv;
+                const int iv = isfinite(v) ? __float2int_rn(v) : 0;
+                q[e] = iv > 7 ? 7 : (iv < -7 ? -7 : iv);
+              }
+              w[g] = sm4_pack(q);
+            }
+            *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * K + c * 32) / 8) =
+                make_uint4(w[0], w[1], w[2], w[3]);
+          }
+        }
+      }
+    }
+    // every CTA has read its maxima: block 0's tiles now turn them into steps in place
+    grid_barrier(&sync[1], gridDim.x, abort_flag, leader);
+    if (!*abort_flag) {
+#pragma unroll
+      for (int j = 0; j < kMaxUnits; ++j) {
+        if (j >= nu) break;
+        const int64_t u = u0 + j;
+        const int tile = (int)(u % num_tiles);
+        const int t = tile * TM + quad * 32 + lane;
+        if (u / num_tiles != 0 || t >= n) continue;
+        const float a = a_keep[j];
+        float sc = 0.f;
+        if (isfinite(a))
+          sc = __fdiv_rn(a, 7.0f);
+        else
+          report(status, kStatusNonFinite);
+        reinterpret_cast<float*>(amax_bits)[t] = sc;
+      }
+    }
+    tc_fence_before();
+  }
+
+  __syncthreads();
+  if (bars->abort && tid == 0) report(status, kStatusTimeout);
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
@@ -317,11 +616,98 @@ cudaError_t launch_k(const __nv_bfloat16* x, int64_t n, int64_t d, const float* 
   if (attr != cudaSuccess) return attr;
   const int64_t units = (d / K) * ((n + TM - 1) / TM);
   const int grid = (int)(units < num_sms() ? units : num_sms());
+  note_launch();
   k0<<<grid, kThreads, C::SMEM, stream>>>(map, A, (int)n, (int)d, amax, words, status);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  note_launch();
   k1<<<grid, kThreads, C::SMEM, stream>>>(map, A, (int)n, (int)d, amax, words, status);
   return cudaGetLastError();
+}
+
+// Address of this device's barrier slots (looked up once per device).
+uint32_t* sync_slots(cudaError_t* err) {
+  static std::mutex mu;
+  static uint32_t* cache[64] = {nullptr};
+  int dev = 0;
+  *err = cudaGetDevice(&dev);
+  if (*err != cudaSuccess) return nullptr;
+  if (dev < 0 || dev >= 64) {
+    *err = cudaErrorInvalidDevice;
+    return nullptr;
+  }
+  std::lock_guard<std::mutex> lock(mu);
+  if (!cache[dev]) {
+    void* p = nullptr;
+    *err = cudaGetSymbolAddress(&p, g_tq_sync);
+    if (*err != cudaSuccess) return nullptr;
+    cache[dev] = static_cast<uint32_t*>(p);
+  }
+  return cache[dev];
+}
+
+bool cooperative_ok() {
+  int dev = 0, v = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  return cudaDeviceGetAttribute(&v, cudaDevAttrCooperativeLaunch, dev) == cudaSuccess && v != 0;
+}
+
+template <int K>
+cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, const float* A, uint32_t* amax,
+                           uint32_t* words, uint32_t* status, cudaStream_t stream) {
+  using C = TcCfg<K>;
+  const int nb = (int)(d / K);
+  const int tiles = (int)((n + TM - 1) / TM);
+  const int64_t units = (int64_t)nb * tiles;
+  const int grid = (int)(units < num_sms() ? units : num_sms());
+  for (int c = 0; c < grid; ++c) {  // every CTA's units must fit in tensor memory at once
+    int64_t u0, u1;
+    unit_range(c, grid, nb, tiles, &u0, &u1);
+    if (u1 - u0 > 512 / K) return cudaErrorNotSupported;
+  }
+  if (!cooperative_ok()) return cudaErrorNotSupported;
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return cudaErrorNotSupported;
+  cudaError_t e;
+  uint32_t* slots = sync_slots(&e);
+  if (!slots) return e;
+  static std::atomic<uint32_t> next_slot{0};
+  uint32_t* sync = slots + 4 * (next_slot.fetch_add(1) % kSyncSlots);
+  CUtensorMap map;
+  memset(&map, 0, sizeof(map));
+  cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)n};
+  cuuint64_t strides[1] = {(cuuint64_t)d * 2};
+  cuuint32_t box[2] = {64, TM};
+  cuuint32_t estr[2] = {1, 1};
+  if (fn(&map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<__nv_bfloat16*>(x), dims, strides, box, estr,
+         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return cudaErrorInvalidValue;
+  static std::once_flag once;
+  static cudaError_t attr = cudaSuccess;
+  std::call_once(once, [] {
+    attr = cudaFuncSetAttribute(transform_quant_tc_fused_kernel<K>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)C::SMEM);
+  });
+  if (attr != cudaSuccess) return attr;
+  const int64_t zn = n > 4 ? n : 4;
+  note_launch();
+  tq_prep_kernel<<<(unsigned)((zn + 255) / 256), 256, 0, stream>>>(amax, n, sync);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = dim3((unsigned)grid, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = C::SMEM;
+  cfg.stream = stream;
+  cudaLaunchAttribute attrs[1];
+  attrs[0].id = cudaLaunchAttributeCooperative;
+  attrs[0].val.cooperative = 1;
+  cfg.attrs = attrs;
+  cfg.numAttrs = 1;
+  note_launch();
+  return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<K>, map, A, (int)n, (int)d, amax, words, sync,
+                            status);
 }
 
 }  // namespace
@@ -339,4 +725,16 @@ cudaError_t launch_transform_quantize_tc(const void* x, int64_t n, int64_t d, in
   return cudaErrorInvalidValue;
 }
 
+}  // namespace cat
+
+namespace cat {
+// Both phases and the steps in one cooperative launch (after a preparation kernel) when every CTA's
+// units fit in tensor memory; cudaErrorNotSupported otherwise (the caller takes the two-pass path).
+cudaError_t launch_transform_quantize_tc_fused(const void* x, int64_t n, int64_t d, int k, const float* A,
+                                               uint32_t* amax, uint32_t* words, uint32_t* status, cudaStream_t stream) {
+  const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
+  if (k == 64) return launch_fused_k<64>(xb, n, d, A, amax, words, status, stream);
+  if (k == 128) return launch_fused_k<128>(xb, n, d, A, amax, words, status, stream);
+  return cudaErrorNotSupported;
+}
 }  // namespace cat

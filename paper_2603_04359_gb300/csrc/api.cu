@@ -12,11 +12,14 @@
 #include "transform_host.h"
 
 namespace cat {
+std::atomic<unsigned long long> g_kernel_launches{0};
+
 cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
                                 int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, uint32_t* status,
                                 cudaStream_t stream);
 cudaError_t launch_w4a4_gemm_decode(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
-                                    int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, cudaStream_t stream);
+                                    int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, uint32_t* status,
+                                    cudaStream_t stream);
 }  // namespace cat
 
 namespace {
@@ -145,6 +148,8 @@ const char* cat_status_string(cat_status status) {
 const char* cat_last_error(void) { return t_last_error.c_str(); }
 
 int cat_version(void) { return kVersion; }
+
+unsigned long long cat_kernel_launches(void) { return cat::g_kernel_launches.load(); }
 
 cat_status cat_calib_cov(const void* x, cat_dtype dtype, int64_t n, int64_t d, int32_t k, double* sigma_blocks,
                          int accumulate, cat_stream_t stream) {
@@ -364,7 +369,7 @@ cat_status cat_w4a4_linear(const uint8_t* xq, const float* x_scale, const uint8_
   uint32_t* status = status_word(&e);
   if (!status) return cuda_fail(e, "status word");
   if (n <= kMaxDecodeTokens)
-    e = cat::launch_w4a4_gemm_decode(xq, x_scale, Wq, w_scale, n, d_in, d_out, y, acc_out, (cudaStream_t)stream);
+    e = cat::launch_w4a4_gemm_decode(xq, x_scale, Wq, w_scale, n, d_in, d_out, y, acc_out, status, (cudaStream_t)stream);
   else
     e = cat::launch_w4a4_gemm_tc(xq, x_scale, Wq, w_scale, n, d_in, d_out, y, acc_out, status, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "cat_w4a4_linear launch");

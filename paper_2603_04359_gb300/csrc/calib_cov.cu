@@ -114,12 +114,15 @@ cudaError_t launch_typed(const Tin* x, int64_t n, int64_t d, int k, double* sigm
   dim3 grid(nb, tiles_per_dim * tiles_per_dim, (unsigned)splits);
   switch (TS) {
     case 64:
+      note_launch();
       calib_cov_kernel<Tin, 64><<<grid, 256, 0, stream>>>(x, n, d, k, tiles_per_dim, tok_per_split, sigma, use_atomic);
       break;
     case 32:
+      note_launch();
       calib_cov_kernel<Tin, 32><<<grid, 256, 0, stream>>>(x, n, d, k, tiles_per_dim, tok_per_split, sigma, use_atomic);
       break;
     case 16:
+      note_launch();
       calib_cov_kernel<Tin, 16><<<grid, 256, 0, stream>>>(x, n, d, k, tiles_per_dim, tok_per_split, sigma, use_atomic);
       break;
     default:

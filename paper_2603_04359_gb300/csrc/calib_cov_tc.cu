@@ -12,9 +12,16 @@
 // within ~1e-6 of a float64 sum, which moves the block transform by ~1e-6 (its square roots damp
 // the calibration error) -- far below the INT4 step.  Only the diagonal k x k blocks are written.
 //
-// CTA = (channel group, token split).  Warps: 0 TMA producer + TMEM allocator, 1 MMA issuer,
-// 2..5 epilogue (one TMEM lane quadrant each).  Tokens arrive in 64-row chunks of 64-channel,
-// 128B-swizzled boxes through a 4-stage ring.
+// CTA = (channel group, token split).  The token splits of a group form a thread-block cluster of
+// S <= 4 CTAs: each CTA sums its accumulators into an fp32 tile in its own shared memory, and after
+// a cluster barrier CTA r reduces rows [r 128/S, (r+1) 128/S) of the S tiles through distributed
+// shared memory and writes them as coalesced float64 rows.  More splits than one cluster (large
+// token counts) add their clusters' results with float64 atomics.  Since D = X^T X is symmetric,
+// the staged tile is the transpose of the TMEM tile (thread = TMEM row writes one shared-memory
+// column, so the stores are conflict-free) and the written blocks are D^T, equal to D up to the
+// rounding of the accumulation order.
+// Warps: 0 TMA producer + TMEM allocator, 1 MMA issuer, 2..5 epilogue (one TMEM lane quadrant
+// each).  Tokens arrive in 64-row chunks of 64-channel, 128B-swizzled boxes through a 4-stage ring.
 #include <cstring>
 #include <mutex>
 
@@ -27,6 +34,9 @@ constexpr int kChunk = 64;      // tokens per stage
 constexpr int kStages = 4;
 constexpr int kThreads = 192;
 constexpr uint32_t kBox = kChunk * 128;  // one 64-token x 64-channel bf16 box, 8 KiB
+constexpr int kMaxCluster = 4;           // token splits reduced on chip
+constexpr uint32_t kRedTile = 128 * 128 * 4;  // fp32 128 x 128 reduction tile (reuses the stage ring)
+static_assert(kStages * 2 * kBox >= kRedTile, "the reduction tile must fit in the stage ring");
 
 template <int G2>  // 128-channel tiles per dimension of a group (1: k <= 128, 2: k = 256)
 struct CovCfg {
@@ -34,7 +44,9 @@ struct CovCfg {
   static constexpr int BOXES = G / 64;
   static constexpr uint32_t STAGE = BOXES * kBox;
   static constexpr uint32_t BAR_OFF = kStages * STAGE;
-  static constexpr size_t SMEM = BAR_OFF + 256 + 1024;
+  // more than half of an SM's shared memory: one CTA per SM, so that a CTA waiting at a cluster
+  // barrier never holds tensor memory that a CTA of another cluster on the same SM is waiting for
+  static constexpr size_t SMEM = (BAR_OFF + 256 + 1024) > 120 * 1024 ? (BAR_OFF + 256 + 1024) : 120 * 1024;
   static constexpr int NACC = G2 == 1 ? 4 : 1;              // round-robin accumulators per tile
   static constexpr uint32_t TMEM_COLS = G2 * G2 * 128 * NACC;
   // kind::f16, D fp32, A = B = BF16, both MN-major (bits 15, 16), M = N = 128
@@ -64,6 +76,34 @@ __device__ __forceinline__ double f32_to_f64_exact(float f) {
   const uint64_t bits = ((uint64_t)(u >> 31) << 63) | ((uint64_t)(e - 127u + 1023u) << 52) |
                         ((uint64_t)(u & 0x7FFFFFu) << 29);
   return __longlong_as_double((long long)bits);
+}
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t cluster_nctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+  return r;
+}
+// all threads of all CTAs of the cluster; release / acquire orders the shared-memory tiles
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t map_cluster(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ float4 ld_cluster_f32x4(uint32_t caddr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(caddr)
+               : "memory");
+  return v;
 }
 
 __device__ __forceinline__ void mma_bf16_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
@@ -153,54 +193,103 @@ __global__ void __launch_bounds__(kThreads, 1)
       volatile int no_abort = 0;
       mbar_wait_bounded(&bars->mma_done, 0, &no_abort);
     }
-  } else if (chunks > 0) {
-    // epilogue: thread = one channel row of the group; keep its diagonal-block columns
-    const int quad = warp & 3;
-    if (mbar_wait_bounded(&bars->acc_full, 0, abort_flag)) {
-      __syncwarp();
-      tc_fence_after();
+  }
+
+  // ---- reduction over the cluster's token splits and the float64 store ---------------------
+  __syncthreads();
+  const bool epi = warp >= 2;
+  const int ew = warp - 2;                            // epilogue warp 0..3
+  const int quad = warp & 3;                          // the TMEM lane quadrant this warp may access
+  const uint32_t S = cluster_nctarank();
+  const uint32_t rank = cluster_ctarank();
+  const bool have_acc = chunks > 0 && !bars->abort;
+  if (epi && have_acc) {
+    if (!mbar_wait_bounded(&bars->acc_full, 0, abort_flag)) {
+      // gave up: the tile below is not written; the status word reports it
+    }
+    __syncwarp();
+    tc_fence_after();
+  }
+  float* red = reinterpret_cast<float*>(smem);        // the stage ring is idle once acc_full fired
+  const int used = total_steps < C::NACC ? total_steps : C::NACC;  // accumulators written
+  const int kw = G2 == 2 ? 128 : k;                   // needed columns per row within a tile
 #pragma unroll 1
-      for (int ih = 0; ih < G2; ++ih) {
-        const int r0 = ih * 128 + quad * 32;            // first row (within the group) of this warp
-        const int row = r0 + lane;
-        const int ch = c0 + row;                         // channel of this thread
-        const int kw = k < 32 ? 32 : k;                  // columns a warp reads for its rows
-        const int col0 = (r0 / kw) * kw;                 // first diagonal-block column (within the group)
+  for (int ih = 0; ih < G2; ++ih)
 #pragma unroll 1
-        for (int cc = 0; cc < kw / 32; ++cc) {
+    for (int jh = 0; jh < G2; ++jh) {
+      if (epi) {
+        // phase 1: this CTA's partial tile, summed over its accumulators, stored transposed
+        const int r = quad * 32 + lane;               // TMEM lane = tile row
+        const int cw = kw < 32 ? 32 : kw;             // columns a warp's 32 rows need
+        const int col0 = G2 == 2 ? 0 : ((quad * 32) / cw) * cw;
+        const bool live = have_acc && !__any_sync(0xFFFFFFFFu, *abort_flag);  // warp-uniform
+#pragma unroll 1
+        for (int cc = 0; cc < cw / 32; ++cc) {
           const int col = col0 + 32 * cc;
-          const int jh = col / 128;
-          float v32[32];  // the accumulators summed in fp32 (FP64 arithmetic is scarce on this GPU)
+          float v32[32];
 #pragma unroll
           for (int e = 0; e < 32; ++e) v32[e] = 0.f;
-          const int used = total_steps < C::NACC ? total_steps : C::NACC;  // accumulators written
+          if (live) {
 #pragma unroll 1
-          for (int a = 0; a < used; ++a) {
-            uint32_t r[32];
-            __syncwarp();
-            CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + ((a * G2 + ih) * G2 + jh) * 128 + (col % 128), r);
-            tmem_ld_wait();
+            for (int a = 0; a < used; ++a) {
+              uint32_t rr[32];
+              __syncwarp();
+              CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + ((a * G2 + ih) * G2 + jh) * 128 + col, rr);
+              tmem_ld_wait();
 #pragma unroll
-            for (int e = 0; e < 32; ++e) v32[e] += __uint_as_float(r[e]);
+              for (int e = 0; e < 32; ++e) v32[e] += __uint_as_float(rr[e]);
+            }
           }
-          if (ch >= d) continue;
 #pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            const int jc = col + e;                      // column within the group
-            if (k < 32 && (jc / k) != (row / k)) continue;  // k = 16: other half belongs to the neighbour
-            double* dst = sigma + (int64_t)ch * k + (jc % k);
-            const double v = f32_to_f64_exact(v32[e]);
-            if (mode == 2)
-              atomicAdd(dst, v);
-            else
-              *dst = (mode == 1 ? *dst : 0.0) + v;
+          for (int e = 0; e < 32; ++e) red[(col + e) * 128 + r] = v32[e];
+        }
+      }
+      __syncwarp();
+      tc_fence_before();
+      cluster_sync_all();                             // every CTA's tile is written
+      if (epi) {
+        // phase 2: rows [rank 128/S, (rank+1) 128/S) of the S tiles; lanes_per_row lanes cover a
+        // row's kw needed columns 4 at a time
+        const int rows = 128 / (int)S;
+        const int r_lo = (int)rank * rows;
+        const int lpr = kw / 4 < 32 ? kw / 4 : 32;
+        const int rpp = 32 / lpr;                     // rows per warp pass
+        const int sub = lane / lpr, l4 = lane % lpr;
+        const uint32_t red_addr = smem_u32(red);
+#pragma unroll 1
+        for (int R = r_lo + ew * rpp + sub; R < r_lo + rows; R += 4 * rpp) {
+          const int cb = G2 == 2 ? 0 : (R / k) * k;   // first column of R's diagonal block in the tile
+#pragma unroll 1
+          for (int C4 = cb + 4 * l4; C4 < cb + kw; C4 += 4 * lpr) {
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+            const uint32_t off = red_addr + (uint32_t)(R * 128 + C4) * 4u;
+            for (uint32_t src = 0; src < S; ++src) {    // fixed order: deterministic sums
+              const float4 v = ld_cluster_f32x4(map_cluster(off, src));
+              acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+            }
+            // staged tile (ih, jh) is transposed: entry (R, C) belongs to group row jh*128 + R
+            const int grow = c0 + jh * 128 + R;
+            if (grow >= d) continue;
+            double* dst = sigma + (int64_t)grow * k + ((ih * 128 + C4) % k);
+            const double v[4] = {f32_to_f64_exact(acc.x), f32_to_f64_exact(acc.y), f32_to_f64_exact(acc.z),
+                                 f32_to_f64_exact(acc.w)};
+            if (mode == 2) {
+#pragma unroll
+              for (int e = 0; e < 4; ++e) atomicAdd(dst + e, v[e]);
+            } else if (mode == 1) {
+#pragma unroll
+              for (int e = 0; e < 4; ++e) dst[e] += v[e];
+            } else {
+              reinterpret_cast<double2*>(dst)[0] = make_double2(v[0], v[1]);
+              reinterpret_cast<double2*>(dst)[1] = make_double2(v[2], v[3]);
+            }
           }
         }
       }
+      __syncwarp();
+      cluster_sync_all();                             // the tiles may be overwritten / released
     }
-  }
 
-  __syncthreads();
   if (bars->abort && tid == 0) report(status, kStatusTimeout);
   if (warp == 0) {
     tc_fence_after();
@@ -256,22 +345,41 @@ cudaError_t launch_g(const void* x, int64_t n, int64_t d, int k, double* sigma, 
   if (attr != cudaSuccess) return attr;
   const int64_t groups = (d + C::G - 1) / C::G;
   const int64_t chunks = (n + kChunk - 1) / kChunk;
-  int64_t splits = (num_sms() + groups - 1) / groups;  // fill the GPU when there are few groups
-  const int64_t min_chunks_per_split = 8;               // but keep >= 512 tokens per CTA
-  if (splits > chunks / min_chunks_per_split) splits = chunks / min_chunks_per_split;
-  if (splits < 1) splits = 1;
-  const int64_t tps = ((chunks + splits - 1) / splits) * kChunk;
-  splits = (n + tps - 1) / tps;
+  const int sms = num_sms();
+  // S token splits per group reduced on chip (a cluster), while the grid stays within one wave
+  int S = 1;
+  while (S < kMaxCluster && groups * S * 2 <= sms && chunks >= S * 2) S *= 2;
+  // more clusters per group (float64 atomics) only for long calibration runs: >= 2048 tokens per CTA
+  const int64_t per_cta = (chunks + S - 1) / S;
+  int64_t ysplits = (sms + groups * S - 1) / (groups * S);
+  if (ysplits > per_cta / 32) ysplits = per_cta / 32;
+  if (ysplits < 1) ysplits = 1;
+  const int64_t tps = ((chunks + S * ysplits - 1) / (S * ysplits)) * kChunk;
   int mode = accumulate ? 1 : 0;
-  if (splits > 1) {
+  if (ysplits > 1) {
     mode = 2;
     if (!accumulate) {
       cudaError_t e = cudaMemsetAsync(sigma, 0, (size_t)d * k * sizeof(double), stream);
       if (e != cudaSuccess) return e;
     }
   }
-  dim3 grid((unsigned)groups, (unsigned)splits);
-  calib_cov_tc_kernel<G2><<<grid, kThreads, C::SMEM, stream>>>(map, (int)n, (int)d, k, (int)tps, sigma, mode, status);
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = dim3((unsigned)groups, (unsigned)(S * ysplits), 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = C::SMEM;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr_cluster[1];
+  attr_cluster[0].id = cudaLaunchAttributeClusterDimension;
+  attr_cluster[0].val.clusterDim.x = 1;
+  attr_cluster[0].val.clusterDim.y = (unsigned)S;
+  attr_cluster[0].val.clusterDim.z = 1;
+  cfg.attrs = attr_cluster;
+  cfg.numAttrs = 1;
+  note_launch();
+  cudaError_t e = cudaLaunchKernelEx(&cfg, calib_cov_tc_kernel<G2>, map, (int)n, (int)d, k, (int)tps, sigma, mode,
+                                     status);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

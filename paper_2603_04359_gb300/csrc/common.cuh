@@ -1,6 +1,7 @@
 // Device helpers shared by the CAT W4A4 kernels (sm_103a): status reporting, the SM4x8 code
 // format, bounded mbarrier waits, TMA and tcgen05 wrappers.
 #pragma once
+#include <atomic>
 
 #include <cuda.h>
 #include <cuda_bf16.h>
@@ -8,6 +9,11 @@
 #include <stdint.h>
 
 namespace cat {
+
+// Kernels this library has launched in this process (host counter, bumped at every launch site).
+extern std::atomic<unsigned long long> g_kernel_launches;
+inline void note_launch() { g_kernel_launches.fetch_add(1, std::memory_order_relaxed); }
+
 
 // ------------------------------------------------------------------------------------------
 // Device status word (one per device, owned by api.cu; kernels get its address).

@@ -1,5 +1,6 @@
-// W4A4 GEMM for a few tokens (decode): the packed weight stream dominates and is read once from
-// HBM, so the kernel is built around that stream rather than around tensor-core tiles.
+// W4A4 GEMM for a few tokens (decode) on the legacy mma.sync path: the fallback of the tcgen05
+// weight-streaming kernel (gemm_decode_tc.cu) for token operands too large for its shared memory
+// (d_in beyond ~10k codes at 16 tokens).  The packed weight stream is read once from HBM.
 //
 //   acc[t, o] = sum_i q_x[t, i] q_w[o, i],   y[t, o] = acc * s_x[t] * s_w[o]   (Sec. 3, Eq. 5)
 //
@@ -122,15 +123,27 @@ __global__ void __launch_bounds__(kWarps * 32) w4a4_gemm_decode_kernel(
 
 }  // namespace
 
+int decode_tc_stages(int64_t n, int64_t d_in);
+cudaError_t launch_w4a4_gemm_decode_tc(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw,
+                                       int64_t n, int64_t d_in, int64_t d_out, float* y, int32_t* acc_out,
+                                       uint32_t* status, cudaStream_t stream);
+
+// n <= 32: tcgen05 weight streaming when the decoded tokens fit in shared memory, else mma.sync
+// weight streaming with registers.
 cudaError_t launch_w4a4_gemm_decode(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
-                                    int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, cudaStream_t stream) {
-  const unsigned grid = (unsigned)((d_out + kRowsPerCta - 1) / kRowsPerCta);
+                                    int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, uint32_t* status,
+                                    cudaStream_t stream) {
+  if (decode_tc_stages(n, d_in) > 0)
+    return launch_w4a4_gemm_decode_tc(xq, sx, wq, sw, n, d_in, d_out, y, acc_out, status, stream);
   const int nt8 = (int)((n + 7) / 8);
-#define CAT_DECODE_CASE(NT)                                                                                    \
-  case NT:                                                                                                     \
+#define CAT_DECODE_CASE(NT)                                                                                     \
+  case NT: {                                                                                                    \
+    const unsigned grid = (unsigned)((d_out + kRowsPerCta - 1) / kRowsPerCta);                                  \
+    note_launch();                                                                                               \
     w4a4_gemm_decode_kernel<NT><<<grid, kWarps * 32, 0, stream>>>(xq, sx, wq, sw, (int)n, (int)d_in, (int)d_out, \
-                                                                   y, acc_out);                               \
-    break;
+                                                                   y, acc_out);                                \
+    break;                                                                                                      \
+  }
   switch (nt8) {
     CAT_DECODE_CASE(1)
     CAT_DECODE_CASE(2)

@@ -1,0 +1,372 @@
+// W4A4 GEMM for a few tokens (decode, n <= 32) on 5th-generation tensor cores (sm_103a).
+//
+//   acc[t, o] = sum_i q_x[t, i] q_w[o, i],   y[t, o] = acc * s_x[t] * s_w[o]   (Sec. 3, Eq. 5)
+//
+// With a handful of tokens the packed weight stream (d_out x d_in / 2 bytes) is the whole cost, and
+// the legacy mma.sync path of this GPU is too slow to keep up with HBM, so the weights are the MMA's
+// M dimension (128 rows per unit) and the tokens its N dimension (16 or 32):
+//   * the tokens are decoded once per CTA into a resident K-major, 128B-swizzled E4M3 operand;
+//   * two producer warps stream 16 KiB packed weight tiles (128 rows x 128 bytes = 256 codes,
+//     128-byte swizzle) through a TMA ring -- two issuers, because one issuer's TMA rate is below
+//     the per-SM share of HBM bandwidth;
+//   * eight decode warps turn each tile into E4M3 in tensor memory (thread = weight row = TMEM lane,
+//     two warps per lane quadrant, each half of the 256 codes);
+//   * one thread issues tcgen05.mma (A from tensor memory, B from shared memory), accumulating the
+//     exact products q_x q_w 2^-18 in fp32 (|acc| <= 49 d_in < 2^24);
+//   * four epilogue warps read the double-buffered accumulator (thread = output channel) and write
+//     y[t][o] with consecutive o across a warp.
+// A persistent CTA per SM walks 128-row units.  Every mbarrier wait is bounded; a wait that gives up
+// raises the device status word and all roles drain and exit.
+#include <cstring>
+#include <mutex>
+
+#include "common.cuh"
+
+namespace cat {
+namespace {
+
+constexpr int UM = 128;                      // weight rows per unit (MMA M)
+constexpr int KSB = 128;                     // packed bytes per row per K step (256 codes)
+constexpr uint32_t kPkStage = UM * KSB;      // 16 KiB packed tile
+constexpr int kMaxSP = 8;                    // packed stages (runtime count <= this)
+constexpr int SE = 4;                        // decoded A stages in tensor memory, 64 columns each
+constexpr int kThreads = 512;
+constexpr int kMmaWarp = 1, kProd0 = 0, kProd1 = 2;
+constexpr int kDecWarp0 = 4, kDecWarps = 8;
+constexpr int kEpiWarp0 = 12, kEpiWarps = 4;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kAStage0 = 64;            // columns [0, 64): two accumulators of up to 32 columns
+constexpr size_t kSmemBudget = 220 * 1024;
+
+struct DecBars {
+  uint64_t p_full[kMaxSP], p_empty[kMaxSP], full[SE], empty[SE], acc_full[2], acc_empty[2], tok_ready, mma_done;
+  uint32_t tmem_addr;
+  int abort;
+};
+
+#define DEC_TMEM_ST32(taddr, v)                                                                                 \
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16," \
+               "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),                   \
+               "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]),      \
+               "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]), "r"(v[16]),          \
+               "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]), "r"(v[24]),         \
+               "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])                     \
+               : "memory")
+
+#define DEC_TMEM_LD16(taddr, r)                                                                                \
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];" \
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),      \
+                 "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]) \
+               : "r"(taddr))
+
+__device__ __forceinline__ void dec_tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+__device__ __forceinline__ void dec_mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                           uint32_t accumulate) {
+  asm volatile(
+      "{ .reg .pred p; setp.ne.b32 p, %4, 0; "
+      "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p; }" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Bytes of the resident token operand: one [NTOK rows x 128 B] block per 128-code slab.
+__host__ __device__ constexpr size_t tok_bytes(int ntok, int num_ks) { return (size_t)num_ks * 2 * ntok * 128; }
+
+template <int NTOK>
+__global__ void __launch_bounds__(kThreads, 1)
+    w4a4_gemm_decode_tc_kernel(const __grid_constant__ CUtensorMap tmW, const uint8_t* __restrict__ xq,
+                               const float* __restrict__ sx, const float* __restrict__ sw, int n, int d_in, int d_out,
+                               int sp, float* __restrict__ y, int32_t* __restrict__ acc_out,
+                               uint32_t* __restrict__ status) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int row_bytes = d_in / 2;
+  const int num_ks = (row_bytes + KSB - 1) / KSB;
+  const int num_units = (d_out + UM - 1) / UM;
+  uint8_t* bst = smem;                                            // tokens, E4M3
+  uint8_t* pk = smem + tok_bytes(NTOK, num_ks);                   // sp x 16 KiB packed weight tiles
+  DecBars* bars = reinterpret_cast<DecBars*>(pk + (size_t)sp * kPkStage);
+  float* sxs = reinterpret_cast<float*>(bars + 1);                // NTOK token steps
+  volatile int* abort_flag = &bars->abort;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+  if (tid == 0) {
+    for (int s = 0; s < sp; ++s) {
+      mbar_init(&bars->p_full[s], 1);
+      mbar_init(&bars->p_empty[s], kDecWarps);
+    }
+    for (int s = 0; s < SE; ++s) {
+      mbar_init(&bars->full[s], kDecWarps);
+      mbar_init(&bars->empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&bars->acc_full[b], 1);
+      mbar_init(&bars->acc_empty[b], kEpiWarps);
+    }
+    mbar_init(&bars->tok_ready, kDecWarps + kEpiWarps);
+    mbar_init(&bars->mma_done, 1);
+    bars->abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0) tmem_alloc(&bars->tmem_addr, kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bars->tmem_addr;
+
+  if (warp >= kDecWarp0) {
+    // resident token operand, staged by the decode and epilogue warps while the weight tiles start
+    // to stream: slab a (codes 128a .. 128a+127) of token t at a*NTOK*128 + t*128, 16-byte chunk c at
+    // c ^ (t % 8); tokens >= n and codes >= d_in are zero
+    const int slabs = 2 * num_ks;
+    const int st = tid - kDecWarp0 * 32, nst = (kDecWarps + kEpiWarps) * 32;
+    const int items = NTOK * slabs * 4;
+    for (int e0 = st; e0 < items; e0 += 4 * nst) {
+      uint4 w[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {  // four loads in flight
+        const int e = e0 + q * nst;
+        const int j = e & 3, a = (e >> 2) % slabs, t = (e >> 2) / slabs;
+        const int off = a * 64 + j * 16;                          // packed byte offset in the row
+        w[q] = make_uint4(0u, 0u, 0u, 0u);
+        if (e < items && t < n && off < row_bytes) w[q] = *reinterpret_cast<const uint4*>(xq + (int64_t)t * row_bytes + off);
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int e = e0 + q * nst;
+        if (e >= items) break;
+        const int j = e & 3, a = (e >> 2) % slabs, t = (e >> 2) / slabs;
+        uint8_t* dst = bst + (size_t)a * NTOK * 128 + t * 128;
+        const int swz = t & 7;
+        *reinterpret_cast<uint4*>(dst + (((2 * j) ^ swz) << 4)) =
+            make_uint4(sm4_lo(w[q].x), sm4_hi(w[q].x), sm4_lo(w[q].y), sm4_hi(w[q].y));
+        *reinterpret_cast<uint4*>(dst + (((2 * j + 1) ^ swz) << 4)) =
+            make_uint4(sm4_lo(w[q].z), sm4_hi(w[q].z), sm4_lo(w[q].w), sm4_hi(w[q].w));
+      }
+    }
+    if (st < NTOK) sxs[st] = st < n ? sx[st] * kAccScale : 0.f;
+    fence_proxy_async_smem();                                     // the MMA reads the tokens via the async proxy
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&bars->tok_ready);
+  }
+
+  if (warp == kProd0 || warp == kProd1) {
+    // ---------------------------------------------------------------- TMA producers (alternate K steps)
+    if (lane == 0) {
+      const uint32_t me = warp == kProd0 ? 0u : 1u;
+      if (me == 0) prefetch_tensormap(&tmW);
+      uint32_t it = 0, issued_end = 0;                  // this producer issued every K step of its parity below issued_end
+      bool ok = true;
+      for (int u = blockIdx.x; u < num_units && ok; u += gridDim.x)
+        for (int ks = 0; ks < num_ks; ++ks, ++it) {
+          if ((it & 1u) != me) continue;
+          const uint32_t s = it % sp, use = it / sp;
+          if (use > 0 && !(ok = mbar_wait_bounded(&bars->p_empty[s], (use - 1) & 1, abort_flag))) break;
+          mbar_arrive_expect_tx(&bars->p_full[s], kPkStage);
+          tma_load_2d(pk + s * kPkStage, &tmW, ks * KSB, u * UM, &bars->p_full[s]);
+          issued_end = it + 1;
+        }
+      // loads still in flight land before the CTA exits: only the last sp K steps of the whole walk
+      // (`it` steps) have stages that were not reused, so only their barriers still hold the phase
+      // to wait for; this producer waits for the ones it issued
+      volatile int no_abort = 0;
+      for (uint32_t q = it > (uint32_t)sp ? it - sp : 0; q < it && q < issued_end; ++q)
+        if ((q & 1u) == me) mbar_wait_bounded(&bars->p_full[q % sp], (q / sp) & 1, &no_abort);
+    }
+  } else if (warp == kMmaWarp) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t kIdesc = idesc_e4m3_f32(UM, NTOK);
+      const uint32_t bbase = smem_u32(bst);
+      uint32_t it = 0, tcount = 0;
+      bool ok = mbar_wait_bounded(&bars->tok_ready, 0, abort_flag);
+      tc_fence_after();
+      for (int u = blockIdx.x; u < num_units && ok; u += gridDim.x, ++tcount) {
+        const uint32_t ab = tcount & 1;
+        if (tcount >= 2 && !(ok = mbar_wait_bounded(&bars->acc_empty[ab], ((tcount >> 1) - 1) & 1, abort_flag))) break;
+        tc_fence_after();
+        for (int ks = 0; ks < num_ks; ++ks, ++it) {
+          const uint32_t s = it % SE;
+          if (!(ok = mbar_wait_bounded(&bars->full[s], (it / SE) & 1, abort_flag))) break;
+          tc_fence_after();
+          const uint32_t ta = tmem + kAStage0 + 64u * s;
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk) {  // K = 32 codes per MMA: 8 TMEM columns of A; B slab 2ks + kk/4, +32 B
+            const uint64_t db = sdesc_kmajor_sw128(bbase + (uint32_t)((2 * ks + (kk >> 2)) * NTOK * 128)) + 2 * (kk & 3);
+            dec_mma_ts(tmem + ab * 32u, ta + 8u * kk, db, kIdesc, (ks | kk) != 0);
+          }
+          mma_commit(&bars->empty[s]);
+        }
+        if (ok) mma_commit(&bars->acc_full[ab]);
+      }
+      mma_commit(&bars->mma_done);  // all MMAs complete before tensor memory is released
+      volatile int no_abort = 0;
+      mbar_wait_bounded(&bars->mma_done, 0, &no_abort);
+    }
+  } else if (warp >= kDecWarp0 && warp < kDecWarp0 + kDecWarps) {
+    // ---------------------------------------------------------------- decode: weight row = TMEM lane
+    const int quad = warp & 3, half = (warp - kDecWarp0) >> 2;
+    const int r = quad * 32 + lane;
+    uint32_t it = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; u < num_units && ok; u += gridDim.x)
+      for (int ks = 0; ks < num_ks; ++ks, ++it) {
+        const uint32_t ps = it % sp, s = it % SE;
+        if (!(ok = mbar_wait_bounded(&bars->p_full[ps], (it / sp) & 1, abort_flag))) break;
+        if (it >= SE && !(ok = mbar_wait_bounded(&bars->empty[s], ((it / SE) - 1) & 1, abort_flag))) break;
+        tc_fence_after();
+        const uint8_t* prow = pk + ps * kPkStage + r * 128;
+        uint32_t av[32];
+#pragma unroll
+        for (int jj = 0; jj < 4; ++jj) {  // 16-byte chunk j = 4 half + jj of the 128-byte row, at j ^ (r % 8)
+          const int j = 4 * half + jj;
+          const uint4 w = *reinterpret_cast<const uint4*>(prow + ((j ^ (r & 7)) << 4));
+          av[8 * jj + 0] = sm4_lo(w.x); av[8 * jj + 1] = sm4_hi(w.x);
+          av[8 * jj + 2] = sm4_lo(w.y); av[8 * jj + 3] = sm4_hi(w.y);
+          av[8 * jj + 4] = sm4_lo(w.z); av[8 * jj + 5] = sm4_hi(w.z);
+          av[8 * jj + 6] = sm4_lo(w.w); av[8 * jj + 7] = sm4_hi(w.w);
+        }
+        __syncwarp();
+        DEC_TMEM_ST32(tmem + ((uint32_t)(quad * 32) << 16) + kAStage0 + 64u * s + 32u * half, av);
+        dec_tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(&bars->p_empty[ps]);
+          mbar_arrive(&bars->full[s]);
+        }
+      }
+  } else if (warp >= kEpiWarp0) {
+    // ---------------------------------------------------------------- epilogue: output channel = TMEM lane
+    const int quad = warp & 3;
+    uint32_t tcount = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; u < num_units && ok; u += gridDim.x, ++tcount) {
+      const uint32_t ab = tcount & 1;
+      const int o = u * UM + quad * 32 + lane;
+      const float swo = o < d_out ? sw[o] : 0.f;
+      if (!(ok = mbar_wait_bounded(&bars->acc_full[ab], (tcount >> 1) & 1, abort_flag))) break;
+      __syncwarp();
+      tc_fence_after();
+      uint32_t acc[NTOK];
+#pragma unroll
+      for (int c = 0; c < NTOK / 16; ++c) {
+        uint32_t* a16 = acc + 16 * c;
+        DEC_TMEM_LD16(tmem + ((uint32_t)(quad * 32) << 16) + ab * 32u + 16u * c, a16);
+      }
+      tmem_ld_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars->acc_empty[ab]);
+      if (o < d_out) {
+#pragma unroll
+        for (int t = 0; t < NTOK; ++t) {
+          if (t >= n) break;
+          const float a = __uint_as_float(acc[t]);
+          y[(int64_t)t * d_out + o] = a * sxs[t] * swo;
+          if (acc_out) acc_out[(int64_t)t * d_out + o] = __float2int_rn(a * kAccScale);
+        }
+      }
+    }
+  }
+
+  __syncthreads();
+  if (bars->abort && tid == 0) report(status, kStatusTimeout);
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+int num_sms() {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) return 148;
+  return sms;
+}
+
+size_t smem_bytes(int ntok, int num_ks, int sp) {
+  return 1024 + tok_bytes(ntok, num_ks) + (size_t)sp * kPkStage + sizeof(DecBars) + 32 * sizeof(float);
+}
+
+template <int NTOK>
+cudaError_t launch_ntok(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
+                        int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, uint32_t* status, int sp,
+                        cudaStream_t stream) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return cudaErrorNotSupported;
+  const int64_t row_bytes = d_in / 2;
+  CUtensorMap map;
+  memset(&map, 0, sizeof(map));
+  cuuint64_t dims[2] = {(cuuint64_t)row_bytes, (cuuint64_t)d_out};
+  cuuint64_t strides[1] = {(cuuint64_t)row_bytes};
+  cuuint32_t box[2] = {(cuuint32_t)KSB, (cuuint32_t)UM};
+  cuuint32_t estr[2] = {1, 1};
+  if (fn(&map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t*>(wq), dims, strides, box, estr,
+         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return cudaErrorInvalidValue;
+  const int num_ks = (int)((row_bytes + KSB - 1) / KSB);
+  const size_t smem = smem_bytes(NTOK, num_ks, sp);
+  static std::mutex mu;
+  static size_t configured = 0;
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    if (smem > configured) {
+      cudaError_t e = cudaFuncSetAttribute(w4a4_gemm_decode_tc_kernel<NTOK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)smem);
+      if (e != cudaSuccess) return e;
+      configured = smem;
+    }
+  }
+  const int64_t units = (d_out + UM - 1) / UM;
+  const int64_t sms = num_sms();
+  const unsigned grid = (unsigned)(units < sms ? units : sms);
+  note_launch();
+  w4a4_gemm_decode_tc_kernel<NTOK><<<grid, kThreads, smem, stream>>>(map, xq, sx, sw, (int)n, (int)d_in, (int)d_out,
+                                                                      sp, y, acc_out, status);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+// Packed stages that fit beside the resident tokens; 0 when this kernel does not apply.
+int decode_tc_stages(int64_t n, int64_t d_in) {
+  if (n < 1 || n > 32) return 0;
+  const int ntok = n <= 16 ? 16 : 32;
+  const int num_ks = (int)((d_in / 2 + KSB - 1) / KSB);
+  const size_t fixed = smem_bytes(ntok, num_ks, 0);
+  if (fixed >= kSmemBudget) return 0;
+  int sp = (int)((kSmemBudget - fixed) / kPkStage);
+  if (sp > kMaxSP) sp = kMaxSP;
+  return sp >= 3 ? sp : 0;
+}
+
+cudaError_t launch_w4a4_gemm_decode_tc(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw,
+                                       int64_t n, int64_t d_in, int64_t d_out, float* y, int32_t* acc_out,
+                                       uint32_t* status, cudaStream_t stream) {
+  const int sp = decode_tc_stages(n, d_in);
+  if (sp == 0) return cudaErrorInvalidValue;
+  if (n <= 16) return launch_ntok<16>(xq, sx, wq, sw, n, d_in, d_out, y, acc_out, status, sp, stream);
+  return launch_ntok<32>(xq, sx, wq, sw, n, d_in, d_out, y, acc_out, status, sp, stream);
+}
+
+}  // namespace cat

@@ -386,6 +386,7 @@ cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_
   if (attr_err != cudaSuccess) return attr_err;
   const int64_t tiles = ((n + BM - 1) / BM) * ((d_out + BN - 1) / BN);
   const int grid = (int)(tiles < num_sms() ? tiles : num_sms());
+  note_launch();
   w4a4_gemm_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(ty, ta, tb, sx, sw, (int)n, (int)d_in, (int)d_out, y,
                                                               acc_out, use_tma, status);
   return cudaGetLastError();

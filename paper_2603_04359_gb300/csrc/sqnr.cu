@@ -1,9 +1,11 @@
 // SQNR of the layer output (Sec. 2, Eq. 1):  10 log10( sum y^2 / sum (y - y_hat)^2 ).
 //
-// HBM-bound: 8 bytes read per element.  Each thread streams float4 pairs, sums squares in fp32
-// over runs of 16 elements (short runs keep the fp32 rounding at ~1e-7 of a run) and adds the
-// run sums to float64 accumulators; warps reduce with shuffles and each CTA adds its two
-// partial sums to the float64 outputs atomically.  A one-thread kernel then forms the ratio.
+// HBM-bound: 8 bytes read per element.  Each thread issues the loads of 4 float4 pairs at once
+// (bytes in flight), sums squares in fp32 over runs of 16 elements (short runs keep the fp32
+// rounding at ~1e-7 of a run) and adds the run sums to float64 accumulators; warps reduce with
+// shuffles and each CTA adds its two partial sums to the float64 outputs atomically.  The last
+// CTA to finish (a counter kept in the third output word, which the launch zeroes with the sums)
+// forms the ratio, so the whole reduction is one launch.
 #include "common.cuh"
 
 namespace cat {
@@ -23,19 +25,23 @@ __global__ void __launch_bounds__(kThreads) sqnr_partial_kernel(const float* __r
   const int64_t n4 = numel / 4;
   const float4* r4 = reinterpret_cast<const float4*>(yr);
   const float4* h4 = reinterpret_cast<const float4*>(yh);
-  const int64_t stride = (int64_t)gridDim.x * kThreads;
   double sig = 0.0, err = 0.0;
-  int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x;
-  while (i < n4) {
+  // CTA tiles of 4 x kThreads consecutive float4 (16 KiB of each input), tiles strided by the grid
+  const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int64_t base = (int64_t)blockIdx.x * 4 * kThreads; base < n4; base += (int64_t)gridDim.x * 4 * kThreads) {
+    float4 a[4], b[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {  // all 8 loads in flight before the first use
+      const int64_t j = base + u * kThreads + threadIdx.x;
+      a[u] = j < n4 ? __ldcs(r4 + j) : zero;
+      b[u] = j < n4 ? __ldcs(h4 + j) : zero;
+    }
     float s_run = 0.f, e_run = 0.f;
 #pragma unroll
-    for (int u = 0; u < 4 && i < n4; ++u) {
-      const float4 a = __ldcs(r4 + i);
-      const float4 b = __ldcs(h4 + i);
-      const float ex = a.x - b.x, ey = a.y - b.y, ez = a.z - b.z, ew = a.w - b.w;
-      s_run += a.x * a.x + a.y * a.y + a.z * a.z + a.w * a.w;
+    for (int u = 0; u < 4; ++u) {
+      const float ex = a[u].x - b[u].x, ey = a[u].y - b[u].y, ez = a[u].z - b[u].z, ew = a[u].w - b[u].w;
+      s_run += a[u].x * a[u].x + a[u].y * a[u].y + a[u].z * a[u].z + a[u].w * a[u].w;
       e_run += ex * ex + ey * ey + ez * ez + ew * ew;
-      i += stride;
     }
     sig += (double)s_run;
     err += (double)e_run;
@@ -63,6 +69,13 @@ __global__ void __launch_bounds__(kThreads) sqnr_partial_kernel(const float* __r
     }
     atomicAdd(&out3[0], a);
     atomicAdd(&out3[1], b);
+    __threadfence();
+    unsigned long long* done = reinterpret_cast<unsigned long long*>(&out3[2]);
+    if (atomicAdd(done, 1ull) == (unsigned long long)gridDim.x - 1) {  // every CTA's sums have landed
+      __threadfence();
+      const double s_tot = atomicAdd(&out3[0], 0.0), e_tot = atomicAdd(&out3[1], 0.0);
+      out3[2] = (e_tot > 0.0) ? 10.0 * log10(s_tot / e_tot) : (s_tot > 0.0 ? HUGE_VAL : 0.0);
+    }
   }
 }
 
@@ -81,16 +94,18 @@ int num_sms() {
 }  // namespace
 
 cudaError_t launch_sqnr(const float* y_ref, const float* y_hat, int64_t numel, double* out3, cudaStream_t stream) {
-  cudaError_t e = cudaMemsetAsync(out3, 0, 2 * sizeof(double), stream);
+  cudaError_t e = cudaMemsetAsync(out3, 0, 3 * sizeof(double), stream);  // sums and the CTA counter
   if (e != cudaSuccess) return e;
-  if (numel > 0) {
-    const int64_t want = (numel / 4 + kThreads * 16 - 1) / (kThreads * 16);  // >= 16 float4 per thread
-    const int64_t cap = (int64_t)num_sms() * 8;
-    const unsigned grid = (unsigned)(want < 1 ? 1 : (want > cap ? cap : want));
-    sqnr_partial_kernel<<<grid, kThreads, 0, stream>>>(y_ref, y_hat, numel, out3);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if (numel == 0) {
+    note_launch();
+    sqnr_finalize_kernel<<<1, 1, 0, stream>>>(out3);
+    return cudaGetLastError();
   }
-  sqnr_finalize_kernel<<<1, 1, 0, stream>>>(out3);
+  const int64_t want = (numel / 4 + kThreads * 4 - 1) / (kThreads * 4);  // one 4-float4 tile per thread at least
+  const int64_t cap = (int64_t)num_sms() * 8;
+  const unsigned grid = (unsigned)(want < 1 ? 1 : (want > cap ? cap : want));
+  note_launch();
+  sqnr_partial_kernel<<<grid, kThreads, 0, stream>>>(y_ref, y_hat, numel, out3);
   return cudaGetLastError();
 }
 

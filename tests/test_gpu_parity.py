@@ -127,7 +127,8 @@ def test_nonfinite_activation_reports_numeric():
 # ------------------------------------------------------------------------------------------
 
 GEMM_SHAPES = [
-    (1, 64, 8), (5, 160, 100), (16, 4096, 520), (17, 96, 33), (32, 384, 300),          # weight-streaming path
+    (1, 64, 8), (5, 160, 100), (17, 96, 33),                                            # weight streaming, registers
+    (16, 4096, 520), (32, 384, 300), (8, 8192, 200), (24, 2048, 1000), (2, 1024, 17),   # weight streaming, bulk ring
     (33, 128, 256), (128, 256, 256), (129, 160, 300), (300, 384, 520), (257, 4096, 64),  # tcgen05 path
     (512, 1024, 1024),
 ]
@@ -151,9 +152,9 @@ def test_w4a4_linear_exact(n, d_in, d_out):
     assert cat.cat_device_status()[0] == 0
 
 
-@pytest.mark.parametrize("n", [8, 200])
-def test_w4a4_linear_extreme_accumulators(n):
-    d_in, d_out = 14336, 64
+@pytest.mark.parametrize("n,d_in", [(8, 14336), (200, 14336), (16, 4096)])
+def test_w4a4_linear_extreme_accumulators(n, d_in):
+    d_out = 64
     qx = np.full((n, d_in), 7, dtype=np.int64)
     qx[1::2] = -7
     qw = np.full((d_out, d_in), 7, dtype=np.int64)
