@@ -26,7 +26,7 @@ namespace {
 constexpr int TM = 128;                 // rows per tile
 constexpr int kThreads = 512;
 constexpr int kEpiWarp0 = 4, kCvtWarp0 = 8, kCvtWarps = 8;
-constexpr int kXStages = 2;
+constexpr int kXStages = 4;                    // every unit of a CTA in flight at once (<= 4 units at k = 128)
 static_assert((64 * 64 / 8) % (kCvtWarps * 32) == 0, "converter items must divide evenly");
 
 template <int K>
@@ -331,6 +331,7 @@ __device__ __forceinline__ void grid_barrier(uint32_t* ctr, uint32_t expected, v
     atomicAdd(ctr, 1u);
     const uint64_t t0 = globaltimer_ns();
     for (uint32_t it = 0; ld_acquire_gpu(ctr) < expected; ++it) {
+      __nanosleep(64);                                  // keep the polls off the counter's L2 slice
       if ((it & 63u) == 63u && (*abort_flag || globaltimer_ns() - t0 > kWaitLimitNs)) {
         *abort_flag = 1;
         break;
@@ -345,6 +346,66 @@ __global__ void tq_prep_kernel(uint32_t* __restrict__ amax_bits, int64_t n, uint
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i < n) amax_bits[i] = 0u;
   if (i < 4) sync[i] = 0u;
+}
+
+// Named barrier of the 12 warps that quantize (4 epilogue + 8 converter warps).
+__device__ __forceinline__ void quant_bar() { asm volatile("bar.sync 3, 384;" ::: "memory"); }
+
+// Phase B jobs of one warp: job = (unit j, 32-column chunk c), taken round-robin by the three warps
+// of a TMEM lane quadrant (slot 0: the epilogue warp, 1 and 2: converter warps).
+template <int K>
+__device__ __forceinline__ void quantize_jobs(uint32_t tmem, int64_t u0, int64_t u1, int num_tiles, int n, int d,
+                                              const uint32_t* __restrict__ amax_bits, uint32_t* __restrict__ codes,
+                                              volatile int* abort_flag, int slot) {
+  if (__any_sync(0xFFFFFFFFu, *abort_flag)) return;
+  constexpr int kMaxUnits = 512 / K;
+  const int lane = threadIdx.x & 31, quad = (threadIdx.x >> 5) & 3;
+  const int64_t words_per_row = d / 8;
+  const int nu = (int)(u1 - u0);
+  const int jobs = nu * (K / 32);
+  // this lane's row maxima of every unit, all loads in flight at once
+  float inv_u[kMaxUnits];
+#pragma unroll
+  for (int j = 0; j < kMaxUnits; ++j) {
+    const int t = (int)((u0 + j) % num_tiles) * TM + quad * 32 + lane;
+    inv_u[j] = (j < nu && t < n) ? __uint_as_float(__ldcg(&amax_bits[t])) : 0.f;
+  }
+#pragma unroll
+  for (int j = 0; j < kMaxUnits; ++j) {
+    const float a = inv_u[j];
+    inv_u[j] = (isfinite(a) && a > 0.f) ? __fdiv_rn(7.0f, a) : 0.f;
+  }
+  tc_fence_after();
+  for (int job = slot; job < jobs; job += 3) {
+    const int j = job / (K / 32), c = job % (K / 32);
+    const int64_t u = u0 + j;
+    const int b = (int)(u / num_tiles), tile = (int)(u % num_tiles);
+    const int t = tile * TM + quad * 32 + lane;
+    float inv = inv_u[0];
+#pragma unroll
+    for (int q = 1; q < kMaxUnits; ++q)
+      if (j == q) inv = inv_u[q];
+    uint32_t r[32];
+    __syncwarp();
+    CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + j * K + c * 32, r);
+    tmem_ld_wait();
+    if (t < n) {
+      uint32_t w[4];
+#pragma unroll
+      for (int g = 0; g < 4; ++g) {
+        int q[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float v = __uint_as_float(r[8 * g + e]) * inv;
+          const int iv = isfinite(v) ? __float2int_rn(v) : 0;
+          q[e] = iv > 7 ? 7 : (iv < -7 ? -7 : iv);
+        }
+        w[g] = sm4_pack(q);
+      }
+      *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * K + c * 32) / 8) =
+          make_uint4(w[0], w[1], w[2], w[3]);
+    }
+  }
 }
 
 template <int K>
@@ -462,11 +523,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) mbar_arrive(&bars->t_full);
       ++version;
     }
+    quant_bar();                                       // the epilogue warps have passed the first grid barrier
+    quantize_jobs<K>(tmem, u0, u1, num_tiles, n, d, amax_bits, codes, abort_flag, 1 + ((warp - kCvtWarp0) >> 2));
+    quant_bar();
+    tc_fence_before();
   } else if (warp >= kEpiWarp0) {
     // ---------------------------------------------------------------- epilogue: one row per thread
     const int quad = warp & 3;
     const bool leader = warp == kEpiWarp0 && lane == 0;
-    const int64_t words_per_row = d / 8;
     const int nu = (int)(u1 - u0);
     bool finite = true;
     // phase A: row maxima of every unit's tile
@@ -494,58 +558,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (!finite) report(status, kStatusNonFinite);
     grid_barrier(&sync[0], gridDim.x, abort_flag, leader);
-    // phase B: quantize the tiles still in tensor memory with the final row maxima
-    float a_keep[kMaxUnits];
-#pragma unroll
-    for (int j = 0; j < kMaxUnits; ++j) a_keep[j] = 0.f;
-    if (!__any_sync(0xFFFFFFFFu, *abort_flag)) {
-#pragma unroll
-      for (int j = 0; j < kMaxUnits; ++j) {
-        if (j >= nu) break;
-        const int64_t u = u0 + j;
-        const int b = (int)(u / num_tiles), tile = (int)(u % num_tiles);
-        const int t = tile * TM + quad * 32 + lane;
-        float a = 0.f;
-        if (t < n) a = __uint_as_float(__ldcg(&amax_bits[t]));
-        a_keep[j] = a;
-        const float inv = (isfinite(a) && a > 0.f) ? __fdiv_rn(7.0f, a) : 0.f;
-        tc_fence_after();
-#pragma unroll 1
-        for (int c = 0; c < K / 32; ++c) {
-          uint32_t r[32];
-          __syncwarp();
-          CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + j * K + c * 32, r);
-          tmem_ld_wait();
-          if (t < n) {
-            uint32_t w[4];
-#pragma unroll
-            for (int g = 0; g < 4; ++g) {
-              int q[8];
-#pragma unroll
-              for (int e = 0; e < 8; ++e) {
-                const float v = __uint_as_float(r[8 * g + e]) * inv;
-                const int iv = isfinite(v) ? __float2int_rn(v) : 0;
-                q[e] = iv > 7 ? 7 : (iv < -7 ? -7 : iv);
-              }
-              w[g] = sm4_pack(q);
-            }
-            *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * K + c * 32) / 8) =
-                make_uint4(w[0], w[1], w[2], w[3]);
-          }
-        }
-      }
-    }
+    // phase B: the tiles still in tensor memory, quantized with the final row maxima by the 12 warps
+    // that own TMEM lane quadrants (4 epilogue + 8 converter warps), a 32-column chunk per job
+    quant_bar();
+    quantize_jobs<K>(tmem, u0, u1, num_tiles, n, d, amax_bits, codes, abort_flag, 0);
+    quant_bar();                                       // all of this CTA's reads of the maxima are done
     // every CTA has read its maxima: block 0's tiles now turn them into steps in place
     grid_barrier(&sync[1], gridDim.x, abort_flag, leader);
-    if (!*abort_flag) {
-#pragma unroll
-      for (int j = 0; j < kMaxUnits; ++j) {
-        if (j >= nu) break;
-        const int64_t u = u0 + j;
+    if (!__any_sync(0xFFFFFFFFu, *abort_flag)) {
+      for (int64_t u = u0; u < u1; ++u) {
         const int tile = (int)(u % num_tiles);
         const int t = tile * TM + quad * 32 + lane;
         if (u / num_tiles != 0 || t >= n) continue;
-        const float a = a_keep[j];
+        const float a = __uint_as_float(__ldcg(&amax_bits[t]));
         float sc = 0.f;
         if (isfinite(a))
           sc = __fdiv_rn(a, 7.0f);

@@ -9,22 +9,34 @@
 // multiplies by 2^18 s_x s_w.
 //
 // Data path.  The tensor cores read their shared-memory operands on a path of their own (their
-// rate does not change under concurrent LSU shared-memory traffic), an MMA with A in tensor memory
-// runs at ~93% of peak, and shared-memory stores top out near 100 B/clk/SM.  So:
-//   * packed A (128 x 64 B) and B (256 x 64 B) tiles arrive by TMA with a 64-byte swizzle, which
-//     makes one-row-per-thread 16-byte shared loads conflict-free;
-//   * A is decoded one row per thread and written to tensor memory (tcgen05.st), never to
-//     shared memory; the MMA reads A from tensor memory;
-//   * only B is decoded into 128B-swizzled shared memory (32 KiB of stores per K step).
+// rate does not change under concurrent LSU shared-memory traffic) and an MMA with A in tensor
+// memory runs at ~93% of peak, while the decode of the packed B operand into shared memory is the
+// costliest step.  So two SMs share each output tile (a cluster pair and tcgen05.mma.cta_group::2):
+//   * the pair tile is 256 tokens x 128 channels; each CTA owns 128 tokens (the A rows, in its own
+//     tensor memory) and 64 channels (half of B, in its own shared memory), so every decoded B row
+//     serves 256 tokens and each SM decodes half the B rows a single-SM tile would need;
+//   * each K step covers 256 codes: packed A (128 x 128 B) and B (64 x 128 B) tiles arrive by TMA
+//     with a 128-byte swizzle, from two issuing warps (one per operand);
+//   * A is decoded one row per thread and written to tensor memory; B is decoded into 128B-swizzled
+//     shared memory; two groups of decode warps take alternate K steps;
+//   * the decode warps of both CTAs arrive on the even CTA's stage barrier; its MMA thread issues the
+//     pair MMAs and multicasts the completions (stage free, accumulator full) to both CTAs;
+//   * four decoded stages: the decode of a K step takes several times longer (latency: loads, fences,
+//     tensor-memory stores) than its MMAs, so four steps are decoded while one is multiplied;
+//   * the accumulator is double-buffered (2 x 128 columns), so the epilogue of one tile overlaps the
+//     MMAs of the next; each CTA drains its own 128 rows.
 //
-// Persistent CTA (one per SM, 512 threads), output tile 128 tokens x 256 channels, K step 128:
-//   warp 0       TMA producer (packed ring) and TMEM allocator
-//   warp 1       lane 0 issues tcgen05.mma (4 x K=32 per K step) and commits
+// Persistent CTA pairs (one CTA per SM, 512 threads each):
+//   warp 0       TMA producer of A tiles and TMEM allocator
+//   warp 1       lane 0 of the even CTA issues tcgen05.mma (8 x K=32 per K step) and commits
+//   warps 1, 3   lane 0 of the odd CTA forwards its decode groups' stage readiness to the even CTA
+//   warp 2       TMA producer of B tiles
 //   warps 4..7   epilogue: tcgen05.ld of their TMEM lane quadrant, scale, stage the rows in
 //                128B-swizzled shared memory, TMA store (plain stores when the TMA rules don't hold)
-//   warps 8..15  decode: B chunks (all 8 warps) and A rows (warps 8..11, one TMEM quadrant each)
-// TMEM: accumulator columns [0, 256), A stages at 256 + 32 s.  Every mbarrier wait is bounded;
-// a wait that gives up raises the device status word and all roles drain and exit.
+//   warps 8..15  decode, two groups of four warps taking alternate K steps: a whole A row per
+//                thread, and B chunks
+// TMEM: accumulators at columns [0, 128) and [128, 256), A stages at 256 + 64 s.  Every mbarrier wait
+// is bounded; a wait that gives up raises the device status word and all roles drain and exit.
 #include <cstring>
 #include <mutex>
 
@@ -33,20 +45,25 @@
 namespace cat {
 namespace {
 
-constexpr int BM = 128, BN = 256, BK = 128;
-constexpr int BKP = BK / 2;                 // packed bytes per row per K step
-constexpr int SP = 3;                       // packed stages (TMA)
-constexpr int SE = 3;                       // decoded stages (A in TMEM, B in shared memory)
-constexpr uint32_t kPackedA = BM * BKP;     // 8 KiB
-constexpr uint32_t kPackedB = BN * BKP;     // 16 KiB
+constexpr int BM = 128;                    // tokens per CTA (256 per pair)
+constexpr int BN = 128;                    // channels per pair tile
+constexpr int BNC = BN / 2;                // channels (B rows) held by each CTA
+constexpr int BK = 256;
+constexpr int BKP = BK / 2;                 // packed bytes per row per K step (128)
+constexpr int SP = 4;                       // packed stages (TMA)
+constexpr int SE = 4;                       // decoded stages (A in TMEM, B in shared memory)
+constexpr uint32_t kPackedA = BM * BKP;     // 16 KiB
+constexpr uint32_t kPackedB = BNC * BKP;    // 8 KiB
 constexpr uint32_t kPackedStage = kPackedA + kPackedB;
-constexpr uint32_t kStageB = BN * BK;       // 32 KiB of E4M3 per stage
+constexpr uint32_t kAtomB = BNC * 128;      // one 128-code K atom of decoded B (64 rows x 128 B)
+constexpr uint32_t kStageB = BNC * BK;      // 16 KiB of E4M3 per stage (two atoms)
 constexpr int kThreads = 512;
-constexpr int kDecWarp0 = 8, kDecWarps = 8, kDecThreads = kDecWarps * 32;
+constexpr int kProdA = 0, kMmaWarp = 1, kProdB = 2, kFwdWarp = 3;
+constexpr int kDecWarp0 = 8, kGroupWarps = 4, kGroupThreads = kGroupWarps * 32;  // two decode groups
 constexpr int kEpiWarp0 = 4, kEpiWarps = 4;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kAccCols = 256;
-constexpr uint32_t kIdesc = idesc_e4m3_f32(BM, BN);
+constexpr uint32_t kAccCols = 2 * BN;       // two accumulators
+constexpr uint32_t kIdesc = idesc_e4m3_f32(2 * BM, BN);
 constexpr uint32_t kEpiStage = 32 * 32 * 4;                 // 32 rows x 32 fp32 columns, 4 KiB
 constexpr int kEpiBufs = 2;                                  // TMA-store staging buffers per epilogue warp
 constexpr uint32_t kPkOffset = SE * kStageB;                 // after the decoded B stages
@@ -54,9 +71,14 @@ constexpr uint32_t kEpiOffset = kPkOffset + SP * kPackedStage;
 constexpr uint32_t kScaleOffset = kEpiOffset + kEpiWarps * kEpiBufs * kEpiStage;
 constexpr uint32_t kBarOffset = kScaleOffset + kEpiWarps * BN * 4;
 constexpr size_t kSmemBytes = kBarOffset + 256 + 1024;      // + barriers + alignment slack
+static_assert(kAccCols + SE * 64 <= kTmemCols, "tensor memory budget");
+static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+static_assert(kPackedStage % 1024 == 0 && kAtomB % 1024 == 0 && kPackedA % 1024 == 0, "128B-swizzle alignment");
+static_assert((BNC * 8) % kGroupThreads == 0, "B chunks per decode thread");
+static_assert(SP % 2 == 0 && SE % 2 == 0, "the two decode groups own alternate stages");
 
 struct Bars {
-  uint64_t p_full[SP], p_empty[SP], full[SE], empty[SE], acc_full, acc_empty, mma_done;
+  uint64_t p_full[SP], p_empty[SP], full[SE], ready[SE], empty[SE], acc_full[2], acc_empty[2], mma_done;
   uint32_t tmem_addr;
   int abort;
 };
@@ -71,16 +93,46 @@ struct Bars {
                "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])                     \
                : "memory")
 
-__device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
-
-__device__ __forceinline__ void mma_f8f6f4_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
-                                              uint32_t accumulate) {
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// arrive on the mbarrier at the same shared-memory offset in CTA `rank` of the cluster
+__device__ __forceinline__ void mbar_arrive_cluster(uint64_t* bar, uint32_t rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(bar)), "r"(rank));
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote) : "memory");
+}
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t* dst, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst)), "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+// the pair MMA: D (both CTAs' TMEM) (+)= A (both CTAs' TMEM) x B (both CTAs' shared memory)
+__device__ __forceinline__ void mma_pair_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                            uint32_t accumulate) {
   asm volatile(
       "{ .reg .pred p; setp.ne.b32 p, %4, 0; "
-      "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p; }" ::"r"(d_tmem),
+      "tcgen05.mma.cta_group::2.kind::f8f6f4 [%0], [%1], %2, %3, p; }" ::"r"(d_tmem),
       "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// arrive once on the mbarrier at this offset in both CTAs when the pair MMAs issued so far complete
+__device__ __forceinline__ void mma_commit_pair(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+                   smem_u32(bar)),
+               "h"((uint16_t)3)
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
 __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* smem_src, int32_t x, int32_t y) {
   asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
@@ -92,97 +144,120 @@ __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.comm
 __device__ __forceinline__ void bulk_wait_read_le1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
-// 64-byte swizzle of the packed TMA tiles: 16-byte chunk j of 64-byte row r sits at chunk
-// j ^ ((r >> 1) & 3), so 8 consecutive rows read at the same j touch 8 distinct bank groups.
-__device__ __forceinline__ uint32_t sw64_off(int r, int j) { return r * 64 + ((j ^ ((r >> 1) & 3)) << 4); }
-
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     w4a4_gemm_tc_kernel(const __grid_constant__ CUtensorMap tmY, const __grid_constant__ CUtensorMap tmA,
                         const __grid_constant__ CUtensorMap tmB, const float* __restrict__ sx,
                         const float* __restrict__ sw, int n, int d_in, int d_out, float* __restrict__ y,
                         int32_t* __restrict__ acc_out, int use_tma_store, uint32_t* __restrict__ status) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* bst = smem;                         // SE x [256 rows x 128 B] E4M3, 128B-swizzled
-  uint8_t* pk = smem + kPkOffset;              // SP x [A 128 x 64 B | B 256 x 64 B] packed, 64B-swizzled
+  uint8_t* bst = smem;                         // SE x 2 atoms x [128 rows x 128 B] E4M3, 128B-swizzled
+  uint8_t* pk = smem + kPkOffset;              // SP x [A 128 x 128 B | B 128 x 128 B] packed, 128B-swizzled
   uint8_t* epi = smem + kEpiOffset;            // 4 warps x 2 x [32 rows x 128 B], 128B-swizzled
   float* scl = reinterpret_cast<float*>(smem + kScaleOffset);  // 4 warps x 256 output-channel steps
   Bars* bars = reinterpret_cast<Bars*>(smem + kBarOffset);
   volatile int* abort_flag = &bars->abort;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int num_m = (n + BM - 1) / BM;
+  const uint32_t rank = cluster_rank();         // 0: the pair's MMA issuer
+  const int pair = blockIdx.x >> 1, num_pairs = gridDim.x >> 1;
+  const int num_m = (n + 2 * BM - 1) / (2 * BM);  // 256-token pair tiles
   const int num_n = (d_out + BN - 1) / BN;
   const int num_k = (d_in + BK - 1) / BK;
   const int num_tiles = num_m * num_n;
 
   if (tid == 0) {
     for (int s = 0; s < SP; ++s) {
-      mbar_init(&bars->p_full[s], 1);
-      mbar_init(&bars->p_empty[s], kDecWarps);
+      mbar_init(&bars->p_full[s], 2);          // the A and the B producer each arrive with their bytes
+      mbar_init(&bars->p_empty[s], kGroupWarps);    // the decode group of that stage
     }
     for (int s = 0; s < SE; ++s) {
-      mbar_init(&bars->full[s], kDecWarps);
-      mbar_init(&bars->empty[s], 1);
+      mbar_init(&bars->full[s], kGroupWarps + 1); // even CTA: its decode group + the odd CTA's forwarder
+      mbar_init(&bars->ready[s], kGroupWarps);    // odd CTA: its decode group (then forwarded)
+      mbar_init(&bars->empty[s], 1);              // the pair MMA's multicast commit
     }
-    mbar_init(&bars->acc_full, 1);
-    mbar_init(&bars->acc_empty, kEpiWarps);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&bars->acc_full[b], 1);
+      mbar_init(&bars->acc_empty[b], 2 * kEpiWarps);  // the epilogue warps of both CTAs (even CTA)
+    }
     mbar_init(&bars->mma_done, 1);
     bars->abort = 0;
     fence_mbar_init();
   }
   __syncwarp();
-  if (warp == 0) tmem_alloc(&bars->tmem_addr, kTmemCols);
+  if (warp == 0) tmem_alloc_pair(&bars->tmem_addr, kTmemCols);
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();                                 // both CTAs' barriers are initialized before any remote arrive
   tc_fence_after();
   const uint32_t tmem = bars->tmem_addr;
 
-  if (warp == 0) {
-    // ---------------------------------------------------------------- TMA producer
+  if (warp == kProdA || warp == kProdB) {
+    // ---------------------------------------------------------------- TMA producers (A: warp 0, B: warp 2)
     if (lane == 0) {
-      prefetch_tensormap(&tmA);
-      prefetch_tensormap(&tmB);
+      const bool is_a = warp == kProdA;
+      const CUtensorMap* map = is_a ? &tmA : &tmB;
+      prefetch_tensormap(map);
       uint32_t it = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+      for (int tile = pair; tile < num_tiles && ok; tile += num_pairs) {
         const int m = tile % num_m, nn = tile / num_m;
         for (int ks = 0; ks < num_k; ++ks, ++it) {
           const uint32_t s = it % SP, use = it / SP;
           if (use > 0 && !(ok = mbar_wait_bounded(&bars->p_empty[s], (use - 1) & 1, abort_flag))) break;
-          uint8_t* dst = pk + s * kPackedStage;
-          mbar_arrive_expect_tx(&bars->p_full[s], kPackedStage);
-          tma_load_2d(dst, &tmA, ks * BKP, m * BM, &bars->p_full[s]);
-          tma_load_2d(dst + kPackedA, &tmB, ks * BKP, nn * BN, &bars->p_full[s]);
+          uint8_t* dst = pk + s * kPackedStage + (is_a ? 0 : kPackedA);
+          mbar_arrive_expect_tx(&bars->p_full[s], is_a ? kPackedA : kPackedB);
+          tma_load_2d(dst, map, ks * BKP, is_a ? m * 2 * BM + (int)rank * BM : nn * BN + (int)rank * BNC,
+                      &bars->p_full[s]);
         }
       }
       const uint32_t issued = it, first = issued > SP ? issued - SP : 0;
       volatile int no_abort = 0;
       for (uint32_t j = first; j < issued; ++j) mbar_wait_bounded(&bars->p_full[j % SP], (j / SP) & 1, &no_abort);
     }
-  } else if (warp == 1) {
-    // ---------------------------------------------------------------- MMA issuer
+  } else if ((warp == kMmaWarp || warp == kFwdWarp) && rank == 1) {
+    // ---------------------------------------------------------------- odd CTA: forward stage readiness
+    // An arrive on the even CTA's barrier from a thread that has just written shared and tensor
+    // memory stalls it for ~1.5k cycles (the cluster-scope release drains its writes), so the decode
+    // warps arrive locally and one thread per decode group carries the stage's readiness over.
     if (lane == 0) {
+      const uint32_t grp = warp == kMmaWarp ? 0u : 1u;
+      uint32_t it = 0;
+      bool ok = true;
+      for (int tile = pair; tile < num_tiles && ok; tile += num_pairs)
+        for (int ks = 0; ks < num_k; ++ks, ++it) {
+          if ((it & 1u) != grp) continue;
+          const uint32_t s = it % SE;
+          if (!(ok = mbar_wait_bounded(&bars->ready[s], (it / SE) & 1, abort_flag))) break;
+          tc_fence_after();
+          mbar_arrive_cluster(&bars->full[s], 0);
+        }
+    }
+  } else if (warp == kMmaWarp) {
+    // ---------------------------------------------------------------- MMA issuer (even CTA)
+    if (lane == 0 && rank == 0) {
       uint32_t it = 0, tcount = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x, ++tcount) {
-        // the epilogue must have drained the accumulator of the previous tile
-        if (tcount > 0 && !(ok = mbar_wait_bounded(&bars->acc_empty, (tcount - 1) & 1, abort_flag))) break;
+      for (int tile = pair; tile < num_tiles && ok; tile += num_pairs, ++tcount) {
+        const uint32_t ab = tcount & 1;
+        // the epilogue must have drained this accumulator (used two tiles ago)
+        if (tcount >= 2 && !(ok = mbar_wait_bounded(&bars->acc_empty[ab], ((tcount >> 1) - 1) & 1, abort_flag))) break;
         tc_fence_after();
         for (int ks = 0; ks < num_k; ++ks, ++it) {
           const uint32_t s = it % SE;
           if (!(ok = mbar_wait_bounded(&bars->full[s], (it / SE) & 1, abort_flag))) break;
           tc_fence_after();
-          const uint64_t db = sdesc_kmajor_sw128(smem_u32(bst + s * kStageB));
-          const uint32_t ta = tmem + kAccCols + 32u * s;
+          const uint32_t bbase = smem_u32(bst + s * kStageB);
+          const uint32_t ta = tmem + kAccCols + 64u * s;
 #pragma unroll
-          for (int kk = 0; kk < BK / 32; ++kk)  // K = 32 bytes per MMA: 8 TMEM columns of A, +2 in B's address field
-            mma_f8f6f4_ts(tmem, ta + 8u * kk, db + 2 * kk, kIdesc, (ks | kk) != 0);
-          mma_commit(&bars->empty[s]);
+          for (int kk = 0; kk < BK / 32; ++kk) {  // K = 32 codes per MMA: 8 TMEM columns of A; B atom kk/4, +32 B
+            const uint64_t db = sdesc_kmajor_sw128(bbase + (uint32_t)(kk >> 2) * kAtomB) + 2 * (kk & 3);
+            mma_pair_ts(tmem + ab * BN, ta + 8u * kk, db, kIdesc, (ks | kk) != 0);
+          }
+          mma_commit_pair(&bars->empty[s]);
         }
-        if (ok) mma_commit(&bars->acc_full);
+        if (ok) mma_commit_pair(&bars->acc_full[ab]);
       }
-      mma_commit(&bars->mma_done);  // all MMAs complete before TMEM is released
+      mma_commit_pair(&bars->mma_done);  // all MMAs complete before TMEM is released
       volatile int no_abort = 0;
       mbar_wait_bounded(&bars->mma_done, 0, &no_abort);
     }
@@ -193,9 +268,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     float* wsc = scl + (warp - kEpiWarp0) * BN;
     uint32_t tcount = 0, nstore = 0;
     bool ok = true;
-    for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x, ++tcount) {
+    for (int tile = pair; tile < num_tiles && ok; tile += num_pairs, ++tcount) {
+      const uint32_t ab = tcount & 1;
       const int m = tile % num_m, nn = tile / num_m;
-      const int row0 = m * BM + quad * 32;
+      const int row0 = m * 2 * BM + (int)rank * BM + quad * 32;
       const int t = row0 + lane;
       const float sxt = (t < n) ? sx[t] * kAccScale : 0.f;
       __syncwarp();
@@ -205,19 +281,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         wsc[32 * i + lane] = (o < d_out) ? sw[o] : 0.f;
       }
       __syncwarp();
-      if (!(ok = mbar_wait_bounded(&bars->acc_full, tcount & 1, abort_flag))) break;
+      if (!(ok = mbar_wait_bounded(&bars->acc_full[ab], (tcount >> 1) & 1, abort_flag))) break;
       __syncwarp();
       tc_fence_after();
 #pragma unroll 1
       for (int c = 0; c < BN / 32; ++c) {
         uint32_t r[32];
         __syncwarp();
-        CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + c * 32, r);
+        CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + ab * BN + c * 32, r);
         tmem_ld_wait();
-        if (c == BN / 32 - 1) {  // accumulator fully read: let the next tile's MMAs start
+        if (c == BN / 32 - 1) {  // accumulator fully read: the MMAs of tile + 2 may use it
           tc_fence_before();
           __syncwarp();
-          if (lane == 0) mbar_arrive(&bars->acc_empty);
+          if (lane == 0) mbar_arrive_cluster(&bars->acc_empty[ab], 0);
         }
         const int o0 = nn * BN + c * 32;
         if (o0 >= d_out || row0 >= n) continue;  // warp-uniform: nothing of this chunk is in range
@@ -257,63 +333,80 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else if (warp >= kDecWarp0) {
     // ---------------------------------------------------------------- decode
-    const int dt = tid - kDecWarp0 * 32;          // 0..255
-    const bool a_warp = warp < kDecWarp0 + 4;     // warps 8..11 also decode A rows
+    // Two groups of four warps (one warp per TMEM lane quadrant each) decode alternate K steps: the
+    // decode of one step is latency-bound (shared-memory loads, tensor-memory stores and their wait,
+    // the proxy fence), so two steps are kept in flight.
+    const int grp = (warp - kDecWarp0) >> 2;      // 0: even K steps, 1: odd K steps
     const int quad = warp & 3;
+    const int gt = (warp - kDecWarp0 - 4 * grp) * 32 + lane;  // 0..127 within the group
     const int a_row = quad * 32 + lane;           // this thread's A row = TMEM lane
     uint32_t it = 0;
     bool ok = true;
-    for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+    for (int tile = pair; tile < num_tiles && ok; tile += num_pairs) {
       for (int ks = 0; ks < num_k; ++ks, ++it) {
+        if ((it & 1u) != (uint32_t)grp) continue;
         const uint32_t ps = it % SP, s = it % SE;
         if (!(ok = mbar_wait_bounded(&bars->p_full[ps], (it / SP) & 1, abort_flag))) break;
         if (it >= SE && !(ok = mbar_wait_bounded(&bars->empty[s], ((it / SE) - 1) & 1, abort_flag))) break;
         tc_fence_after();
         const uint8_t* pa = pk + ps * kPackedStage;
         const uint8_t* pb = pa + kPackedA;
-        if (a_warp) {  // A: one 64-byte row per thread -> 128 E4M3 bytes = 32 TMEM columns
+        const uint8_t* prow = pa + a_row * 128;
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {  // A: one 128-byte row per thread -> 64 TMEM columns
           uint32_t av[32];
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const uint4 w = *reinterpret_cast<const uint4*>(pa + sw64_off(a_row, j));
-            av[8 * j + 0] = sm4_lo(w.x); av[8 * j + 1] = sm4_hi(w.x);
-            av[8 * j + 2] = sm4_lo(w.y); av[8 * j + 3] = sm4_hi(w.y);
-            av[8 * j + 4] = sm4_lo(w.z); av[8 * j + 5] = sm4_hi(w.z);
-            av[8 * j + 6] = sm4_lo(w.w); av[8 * j + 7] = sm4_hi(w.w);
+          for (int jj = 0; jj < 4; ++jj) {
+            const int j = 4 * half + jj;
+            const uint4 w = *reinterpret_cast<const uint4*>(prow + ((j ^ (a_row & 7)) << 4));
+            av[8 * jj + 0] = sm4_lo(w.x); av[8 * jj + 1] = sm4_hi(w.x);
+            av[8 * jj + 2] = sm4_lo(w.y); av[8 * jj + 3] = sm4_hi(w.y);
+            av[8 * jj + 4] = sm4_lo(w.z); av[8 * jj + 5] = sm4_hi(w.z);
+            av[8 * jj + 6] = sm4_lo(w.w); av[8 * jj + 7] = sm4_hi(w.w);
           }
           __syncwarp();
-          CAT_TMEM_ST32(tmem + ((uint32_t)(quad * 32) << 16) + kAccCols + 32u * s, av);
+          CAT_TMEM_ST32(tmem + ((uint32_t)(quad * 32) << 16) + kAccCols + 64u * s + 32u * half, av);
         }
-        // B: 1024 chunks of 16 packed bytes (256 rows x 4), 4 per thread, consecutive per warp
+        // B: 512 chunks of 16 packed bytes (64 rows x 8), 4 per thread; 8 consecutive threads read
+        // one 128-byte row.  Chunk j (codes 32j .. 32j+31) becomes the 16-byte E4M3 chunks 2(j%4) and
+        // 2(j%4)+1 of atom j/4; threads of atom 1 store their odd chunk first, so the 8 threads of a
+        // row never hit the same bank group in one store
         uint8_t* bs = bst + s * kStageB;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const int id = dt + kDecThreads * i;
-          const int row = id >> 2, j = id & 3, swz = row & 7;
-          const uint4 w = *reinterpret_cast<const uint4*>(pb + sw64_off(row, j));
-          uint8_t* dst = bs + row * 128;
-          *reinterpret_cast<uint4*>(dst + (((2 * j) ^ swz) << 4)) =
-              make_uint4(sm4_lo(w.x), sm4_hi(w.x), sm4_lo(w.y), sm4_hi(w.y));
-          *reinterpret_cast<uint4*>(dst + (((2 * j + 1) ^ swz) << 4)) =
-              make_uint4(sm4_lo(w.z), sm4_hi(w.z), sm4_lo(w.w), sm4_hi(w.w));
+        for (int i = 0; i < BNC * 8 / kGroupThreads; ++i) {
+          const int id = gt + kGroupThreads * i;
+          const int row = id >> 3, j = id & 7, swz = row & 7;
+          const uint4 w = *reinterpret_cast<const uint4*>(pb + row * 128 + ((j ^ swz) << 4));
+          uint8_t* dst = bs + (j >> 2) * kAtomB + row * 128;
+          const uint4 lo = make_uint4(sm4_lo(w.x), sm4_hi(w.x), sm4_lo(w.y), sm4_hi(w.y));
+          const uint4 hi = make_uint4(sm4_lo(w.z), sm4_hi(w.z), sm4_lo(w.w), sm4_hi(w.w));
+          const int c0 = 2 * (j & 3);
+          if (j < 4) {
+            *reinterpret_cast<uint4*>(dst + ((c0 ^ swz) << 4)) = lo;
+            *reinterpret_cast<uint4*>(dst + (((c0 + 1) ^ swz) << 4)) = hi;
+          } else {
+            *reinterpret_cast<uint4*>(dst + (((c0 + 1) ^ swz) << 4)) = hi;
+            *reinterpret_cast<uint4*>(dst + ((c0 ^ swz) << 4)) = lo;
+          }
         }
-        if (a_warp) tmem_st_wait();
+        tmem_st_wait();
         fence_proxy_async_smem();
         tc_fence_before();
         __syncwarp();
         if (lane == 0) {
           mbar_arrive(&bars->p_empty[ps]);
-          mbar_arrive(&bars->full[s]);
+          mbar_arrive(rank == 0 ? &bars->full[s] : &bars->ready[s]);  // local arrives only: cheap
         }
       }
     }
   }
 
-  __syncthreads();
+  tc_fence_before();
+  cluster_sync();                                 // the pair's MMAs and both epilogues are done with TMEM
   if (bars->abort && tid == 0) report(status, kStatusTimeout);
   if (warp == 0) {
     tc_fence_after();
-    tmem_dealloc(tmem, kTmemCols);
+    tmem_dealloc_pair(tmem, kTmemCols);
   }
 }
 
@@ -347,7 +440,7 @@ bool make_output_map(CUtensorMap* map, float* y, int64_t n, int64_t d_out) {
          CUDA_SUCCESS;
 }
 
-// Packed codes [rows][row_bytes], box [box_rows][64 bytes], 64-byte swizzle, out-of-range reads zero.
+// Packed codes [rows][row_bytes], box [box_rows][128 bytes], 128-byte swizzle, out-of-range reads zero.
 bool make_packed_map(CUtensorMap* map, const uint8_t* base, int64_t rows, int64_t row_bytes, int box_rows) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
@@ -356,7 +449,7 @@ bool make_packed_map(CUtensorMap* map, const uint8_t* base, int64_t rows, int64_
   cuuint32_t box[2] = {(cuuint32_t)BKP, (cuuint32_t)box_rows};
   cuuint32_t estr[2] = {1, 1};
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t*>(base), dims, strides, box, estr,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -376,7 +469,7 @@ cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_
   memset(&ty, 0, sizeof(ty));
   int use_tma = (d_out % 4 == 0) ? 1 : 0;
   if (use_tma && !make_output_map(&ty, y, n, d_out)) use_tma = 0;
-  if (!make_packed_map(&ta, xq, n, d_in / 2, BM) || !make_packed_map(&tb, wq, d_out, d_in / 2, BN))
+  if (!make_packed_map(&ta, xq, n, d_in / 2, BM) || !make_packed_map(&tb, wq, d_out, d_in / 2, BNC))
     return cudaErrorInvalidValue;
   static std::once_flag attr_once;
   static cudaError_t attr_err = cudaSuccess;
@@ -384,8 +477,9 @@ cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_
     attr_err = cudaFuncSetAttribute(w4a4_gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
   });
   if (attr_err != cudaSuccess) return attr_err;
-  const int64_t tiles = ((n + BM - 1) / BM) * ((d_out + BN - 1) / BN);
-  const int grid = (int)(tiles < num_sms() ? tiles : num_sms());
+  const int64_t tiles = ((n + 2 * BM - 1) / (2 * BM)) * ((d_out + BN - 1) / BN);
+  const int64_t pairs_max = num_sms() / 2;
+  const int grid = 2 * (int)(tiles < pairs_max ? tiles : pairs_max);  // CTA pairs (cluster of 2)
   note_launch();
   w4a4_gemm_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(ty, ta, tb, sx, sw, (int)n, (int)d_in, (int)d_out, y,
                                                               acc_out, use_tma, status);
