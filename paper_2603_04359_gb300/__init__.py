@@ -64,6 +64,7 @@ def load_library() -> ctypes.CDLL:
         "cat_transform_quantize_act": ([P, I, I64, I64, I32, P, P, P, P], I),
         "cat_w4a4_linear": ([P, P, P, P, I64, I64, I64, P, P, P], I),
         "cat_sqnr": ([P, P, I64, P, P], I),
+        "cat_w4a4_linear_sqnr": ([P, P, P, P, I64, I64, I64, P, P, P, P], I),
         "cat_device_status": ([P, P], I),
     }
     for name, (args, res) in sigs.items():
@@ -217,6 +218,24 @@ def cat_w4a4_linear(xq: torch.Tensor, x_scale: torch.Tensor, Wq: torch.Tensor, w
         _ptr(xq), _ptr(x_scale), _ptr(Wq), _ptr(w_scale), n, 2 * half, d_out, _ptr(y), _ptr(acc_out),
         _stream(xq.device)))
     return y
+
+
+def cat_w4a4_linear_sqnr(xq: torch.Tensor, x_scale: torch.Tensor, Wq: torch.Tensor, w_scale: torch.Tensor,
+                         y_ref: torch.Tensor, y: Optional[torch.Tensor] = None,
+                         out: Optional[torch.Tensor] = None) -> Tuple[torch.Tensor, torch.Tensor]:
+    """cat_w4a4_linear and cat_sqnr against y_ref in one call: (y float32 [n, d_out], float64 [3])."""
+    for t, name in ((xq, "xq"), (x_scale, "x_scale"), (Wq, "Wq"), (w_scale, "w_scale"), (y_ref, "y_ref")):
+        _need(t, name)
+    n, half = xq.shape
+    d_out = Wq.shape[0]
+    if y is None:
+        y = torch.empty((n, d_out), dtype=torch.float32, device=xq.device)
+    if out is None:
+        out = torch.empty((3,), dtype=torch.float64, device=xq.device)
+    _check("cat_w4a4_linear_sqnr", load_library().cat_w4a4_linear_sqnr(
+        _ptr(xq), _ptr(x_scale), _ptr(Wq), _ptr(w_scale), n, 2 * half, d_out, _ptr(y), _ptr(y_ref), _ptr(out),
+        _stream(xq.device)))
+    return y, out
 
 
 def cat_sqnr(y_ref: torch.Tensor, y_hat: torch.Tensor, out: Optional[torch.Tensor] = None) -> torch.Tensor:

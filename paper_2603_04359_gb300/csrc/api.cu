@@ -15,8 +15,8 @@ namespace cat {
 std::atomic<unsigned long long> g_kernel_launches{0};
 
 cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
-                                int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, uint32_t* status,
-                                cudaStream_t stream);
+                                int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, const float* y_ref,
+                                double* sums3, uint32_t* status, cudaStream_t stream);
 cudaError_t launch_w4a4_gemm_decode(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
                                     int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, uint32_t* status,
                                     cudaStream_t stream);
@@ -371,8 +371,39 @@ cat_status cat_w4a4_linear(const uint8_t* xq, const float* x_scale, const uint8_
   if (n <= kMaxDecodeTokens)
     e = cat::launch_w4a4_gemm_decode(xq, x_scale, Wq, w_scale, n, d_in, d_out, y, acc_out, status, (cudaStream_t)stream);
   else
-    e = cat::launch_w4a4_gemm_tc(xq, x_scale, Wq, w_scale, n, d_in, d_out, y, acc_out, status, (cudaStream_t)stream);
+    e = cat::launch_w4a4_gemm_tc(xq, x_scale, Wq, w_scale, n, d_in, d_out, y, acc_out, nullptr, nullptr, status,
+                                 (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "cat_w4a4_linear launch");
+  return ok();
+}
+
+cat_status cat_w4a4_linear_sqnr(const uint8_t* xq, const float* x_scale, const uint8_t* Wq, const float* w_scale,
+                                int64_t n, int64_t d_in, int64_t d_out, float* y, const float* y_ref, double* out3,
+                                cat_stream_t stream) {
+  if (n < 0 || d_out <= 0) return fail(CAT_ERR_SHAPE, "n must be >= 0 and d_out >= 1");
+  cat_status st = check_din(d_in);
+  if (st != CAT_OK) return st;
+  if (n > 0x7FFFFFFF || d_out > 0x7FFFFFFF) return fail(CAT_ERR_SHAPE, "n and d_out must fit in int32");
+  if (!out3 || (n > 0 && (!xq || !x_scale || !Wq || !w_scale || !y || !y_ref)))
+    return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(out3) || (n > 0 && (!aligned16(xq) || !aligned16(x_scale) || !aligned16(Wq) || !aligned16(w_scale) ||
+                                     !aligned16(y) || !aligned16(y_ref))))
+    return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  if ((st = check_device()) != CAT_OK) return st;
+  cudaError_t e;
+  uint32_t* status = status_word(&e);
+  if (!status) return cuda_fail(e, "status word");
+  cudaStream_t s = (cudaStream_t)stream;
+  if (n > kMaxDecodeTokens && d_out % 4 == 0) {  // SQNR sums fused into the GEMM epilogue
+    e = cat::launch_w4a4_gemm_tc(xq, x_scale, Wq, w_scale, n, d_in, d_out, y, nullptr, y_ref, out3, status, s);
+  } else {  // the GEMM, then the separate reduction
+    e = n == 0 ? cudaSuccess
+        : n <= kMaxDecodeTokens
+            ? cat::launch_w4a4_gemm_decode(xq, x_scale, Wq, w_scale, n, d_in, d_out, y, nullptr, status, s)
+            : cat::launch_w4a4_gemm_tc(xq, x_scale, Wq, w_scale, n, d_in, d_out, y, nullptr, nullptr, nullptr, status, s);
+    if (e == cudaSuccess) e = cat::launch_sqnr(y_ref, y, n * d_out, out3, s);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, "cat_w4a4_linear_sqnr launch");
   return ok();
 }
 

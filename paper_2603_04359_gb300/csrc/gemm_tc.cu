@@ -50,7 +50,7 @@ constexpr int BN = 128;                    // channels per pair tile
 constexpr int BNC = BN / 2;                // channels (B rows) held by each CTA
 constexpr int BK = 256;
 constexpr int BKP = BK / 2;                 // packed bytes per row per K step (128)
-constexpr int SP = 4;                       // packed stages (TMA)
+constexpr int SP = 3;                       // packed stages (TMA)
 constexpr int SE = 4;                       // decoded stages (A in TMEM, B in shared memory)
 constexpr uint32_t kPackedA = BM * BKP;     // 16 KiB
 constexpr uint32_t kPackedB = BNC * BKP;    // 8 KiB
@@ -68,17 +68,19 @@ constexpr uint32_t kEpiStage = 32 * 32 * 4;                 // 32 rows x 32 fp32
 constexpr int kEpiBufs = 2;                                  // TMA-store staging buffers per epilogue warp
 constexpr uint32_t kPkOffset = SE * kStageB;                 // after the decoded B stages
 constexpr uint32_t kEpiOffset = kPkOffset + SP * kPackedStage;
-constexpr uint32_t kScaleOffset = kEpiOffset + kEpiWarps * kEpiBufs * kEpiStage;
+constexpr uint32_t kRefOffset = kEpiOffset + kEpiWarps * kEpiBufs * kEpiStage;   // y_ref tiles (SQNR)
+constexpr uint32_t kScaleOffset = kRefOffset + kEpiWarps * kEpiBufs * kEpiStage;
 constexpr uint32_t kBarOffset = kScaleOffset + kEpiWarps * BN * 4;
 constexpr size_t kSmemBytes = kBarOffset + 256 + 1024;      // + barriers + alignment slack
 static_assert(kAccCols + SE * 64 <= kTmemCols, "tensor memory budget");
 static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 static_assert(kPackedStage % 1024 == 0 && kAtomB % 1024 == 0 && kPackedA % 1024 == 0, "128B-swizzle alignment");
 static_assert((BNC * 8) % kGroupThreads == 0, "B chunks per decode thread");
-static_assert(SP % 2 == 0 && SE % 2 == 0, "the two decode groups own alternate stages");
+
 
 struct Bars {
   uint64_t p_full[SP], p_empty[SP], full[SE], ready[SE], empty[SE], acc_full[2], acc_empty[2], mma_done;
+  uint64_t ref_full[kEpiWarps][kEpiBufs];      // y_ref tile loads of each epilogue warp
   uint32_t tmem_addr;
   int abort;
 };
@@ -146,7 +148,8 @@ __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wa
 
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     w4a4_gemm_tc_kernel(const __grid_constant__ CUtensorMap tmY, const __grid_constant__ CUtensorMap tmA,
-                        const __grid_constant__ CUtensorMap tmB, const float* __restrict__ sx,
+                        const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmR,
+                        double* __restrict__ sums3, const float* __restrict__ sx,
                         const float* __restrict__ sw, int n, int d_in, int d_out, float* __restrict__ y,
                         int32_t* __restrict__ acc_out, int use_tma_store, uint32_t* __restrict__ status) {
   extern __shared__ uint8_t smem_raw[];
@@ -154,7 +157,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   uint8_t* bst = smem;                         // SE x 2 atoms x [128 rows x 128 B] E4M3, 128B-swizzled
   uint8_t* pk = smem + kPkOffset;              // SP x [A 128 x 128 B | B 128 x 128 B] packed, 128B-swizzled
   uint8_t* epi = smem + kEpiOffset;            // 4 warps x 2 x [32 rows x 128 B], 128B-swizzled
-  float* scl = reinterpret_cast<float*>(smem + kScaleOffset);  // 4 warps x 256 output-channel steps
+  uint8_t* refb = smem + kRefOffset;           // 4 warps x 2 x [32 rows x 128 B] y_ref, 128B-swizzled
+  float* scl = reinterpret_cast<float*>(smem + kScaleOffset);  // 4 warps x 128 output-channel steps
   Bars* bars = reinterpret_cast<Bars*>(smem + kBarOffset);
   volatile int* abort_flag = &bars->abort;
 
@@ -181,6 +185,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       mbar_init(&bars->acc_empty[b], 2 * kEpiWarps);  // the epilogue warps of both CTAs (even CTA)
     }
     mbar_init(&bars->mma_done, 1);
+    for (int w = 0; w < kEpiWarps; ++w)
+      for (int b = 0; b < kEpiBufs; ++b) mbar_init(&bars->ref_full[w][b], 1);
     bars->abort = 0;
     fence_mbar_init();
   }
@@ -263,11 +269,31 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     }
   } else if (warp >= kEpiWarp0 && warp < kEpiWarp0 + kEpiWarps) {
     // ---------------------------------------------------------------- epilogue
-    const int quad = warp & 3;
-    uint8_t* stage0 = epi + (warp - kEpiWarp0) * kEpiBufs * kEpiStage;
-    float* wsc = scl + (warp - kEpiWarp0) * BN;
+    const int quad = warp & 3, ew = warp - kEpiWarp0;
+    uint8_t* stage0 = epi + ew * kEpiBufs * kEpiStage;
+    uint8_t* rstage0 = refb + ew * kEpiBufs * kEpiStage;
+    float* wsc = scl + ew * BN;
+    const bool with_ref = sums3 != nullptr;
+    double sig = 0.0, err = 0.0;                   // SQNR sums of this thread's outputs
     uint32_t tcount = 0, nstore = 0;
     bool ok = true;
+    // y_ref tiles: chunk c of every tile goes through buffer c % 2; all four are loaded (out-of-range
+    // parts read as zero), so the buffer phases advance regularly
+    uint32_t nref[kEpiBufs] = {0u, 0u}, nused[kEpiBufs] = {0u, 0u};  // loads issued / consumed per buffer
+    auto load_ref = [&](int tile_, int c_) {        // called by the whole warp; lane 0 issues
+      const int m_ = tile_ % num_m, nn_ = tile_ / num_m;
+      uint64_t* bar = &bars->ref_full[ew][c_ & 1];
+      if (lane == 0) {
+        mbar_arrive_expect_tx(bar, kEpiStage);
+        tma_load_2d(rstage0 + (c_ & 1) * kEpiStage, &tmR, nn_ * BN + c_ * 32, m_ * 2 * BM + (int)rank * BM + quad * 32,
+                    bar);
+      }
+      ++nref[c_ & 1];
+    };
+    if (with_ref && pair < num_tiles) {
+      load_ref(pair, 0);
+      load_ref(pair, 1);
+    }
     for (int tile = pair; tile < num_tiles && ok; tile += num_pairs, ++tcount) {
       const uint32_t ab = tcount & 1;
       const int m = tile % num_m, nn = tile / num_m;
@@ -296,18 +322,45 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           if (lane == 0) mbar_arrive_cluster(&bars->acc_empty[ab], 0);
         }
         const int o0 = nn * BN + c * 32;
+        float v[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]) * sxt * wsc[c * 32 + i];
+        if (with_ref) {
+          // SQNR sums (Sec. 2, Eq. 1) from the y_ref tile of this chunk; out-of-range entries are zero
+          // on both sides.  Squares are summed in fp32 over the chunk's 32 values, then in float64.
+          const uint32_t use = 2 * tcount + (c >> 1);  // the use-th load into buffer c % 2
+          if (!(ok = mbar_wait_bounded(&bars->ref_full[ew][c & 1], use & 1, abort_flag))) break;
+          ++nused[c & 1];
+          const uint8_t* rb = rstage0 + (c & 1) * kEpiStage + lane * 128;
+          float s_run = 0.f, e_run = 0.f;
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            const float4 yr = *reinterpret_cast<const float4*>(rb + ((q ^ (lane & 7)) << 4));
+            const float e0 = yr.x - v[4 * q], e1 = yr.y - v[4 * q + 1], e2 = yr.z - v[4 * q + 2], e3 = yr.w - v[4 * q + 3];
+            s_run += yr.x * yr.x + yr.y * yr.y + yr.z * yr.z + yr.w * yr.w;
+            e_run += e0 * e0 + e1 * e1 + e2 * e2 + e3 * e3;
+          }
+          sig += (double)s_run;
+          err += (double)e_run;
+          // refill this buffer with the chunk two ahead (this or the next tile)
+          int nt = tile, nc = c + 2;
+          if (nc >= BN / 32) {
+            nc -= BN / 32;
+            nt = tile + num_pairs;
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (nt < num_tiles) load_ref(nt, nc);
+        }
         if (o0 >= d_out || row0 >= n) continue;  // warp-uniform: nothing of this chunk is in range
         if (use_tma_store) {
           uint8_t* buf = stage0 + (nstore % kEpiBufs) * kEpiStage;
           if (lane == 0) bulk_wait_read_le1();  // the store issued two chunks ago has read this buffer
           __syncwarp();
 #pragma unroll
-          for (int q = 0; q < 8; ++q) {  // row `lane`, 16-byte chunk q at q ^ (lane % 8)
-            const float4 s4 = *reinterpret_cast<const float4*>(wsc + c * 32 + 4 * q);
+          for (int q = 0; q < 8; ++q)  // row `lane`, 16-byte chunk q at q ^ (lane % 8)
             *reinterpret_cast<float4*>(buf + lane * 128 + ((q ^ (lane & 7)) << 4)) =
-                make_float4(__uint_as_float(r[4 * q]) * sxt * s4.x, __uint_as_float(r[4 * q + 1]) * sxt * s4.y,
-                            __uint_as_float(r[4 * q + 2]) * sxt * s4.z, __uint_as_float(r[4 * q + 3]) * sxt * s4.w);
-          }
+                make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
           fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) {
@@ -319,13 +372,38 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           float* yrow = y + (size_t)t * d_out;
 #pragma unroll
           for (int i = 0; i < 32; ++i)
-            if (o0 + i < d_out) yrow[o0 + i] = __uint_as_float(r[i]) * sxt * wsc[c * 32 + i];
+            if (o0 + i < d_out) yrow[o0 + i] = v[i];
         }
         if (acc_out && t < n) {
           int32_t* arow = acc_out + (size_t)t * d_out;
 #pragma unroll
           for (int i = 0; i < 32; ++i)
             if (o0 + i < d_out) arow[o0 + i] = __float2int_rn(__uint_as_float(r[i]) * kAccScale);
+        }
+      }
+    }
+    if (with_ref) {
+      // y_ref loads issued but not consumed (only after a wait gave up) land before the CTA exits
+      volatile int no_abort = 0;
+      for (int bb = 0; bb < kEpiBufs; ++bb)
+        if (nref[bb] > nused[bb]) mbar_wait_bounded(&bars->ref_full[ew][bb], (nref[bb] - 1) & 1, &no_abort);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        sig += __shfl_xor_sync(0xFFFFFFFFu, sig, o);
+        err += __shfl_xor_sync(0xFFFFFFFFu, err, o);
+      }
+      if (lane == 0) {
+        atomicAdd(&sums3[0], sig);
+        atomicAdd(&sums3[1], err);
+      }
+      __threadfence();
+      asm volatile("bar.sync 2, 128;" ::: "memory");  // this CTA's four epilogue warps have added theirs
+      if (ew == 0 && lane == 0) {
+        unsigned long long* done = reinterpret_cast<unsigned long long*>(&sums3[2]);
+        if (atomicAdd(done, 1ull) == (unsigned long long)gridDim.x - 1) {  // the last CTA forms the ratio
+          __threadfence();
+          const double s_tot = atomicAdd(&sums3[0], 0.0), e_tot = atomicAdd(&sums3[1], 0.0);
+          sums3[2] = (e_tot > 0.0) ? 10.0 * log10(s_tot / e_tot) : (s_tot > 0.0 ? HUGE_VAL : 0.0);
         }
       }
     }
@@ -462,13 +540,22 @@ int num_sms() {
 
 }  // namespace
 
+// y_ref != nullptr: the epilogue also accumulates the SQNR sums of y against y_ref into sums3
+// (zeroed here; sums3[2] ends as the dB value).  Needs d_out % 4 == 0 (TMA row pitch).
 cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
-                                int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, uint32_t* status,
-                                cudaStream_t stream) {
-  CUtensorMap ty, ta, tb;
+                                int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, const float* y_ref,
+                                double* sums3, uint32_t* status, cudaStream_t stream) {
+  CUtensorMap ty, ta, tb, tr;
   memset(&ty, 0, sizeof(ty));
+  memset(&tr, 0, sizeof(tr));
   int use_tma = (d_out % 4 == 0) ? 1 : 0;
   if (use_tma && !make_output_map(&ty, y, n, d_out)) use_tma = 0;
+  if (y_ref) {
+    if (d_out % 4 != 0 || !sums3 || !make_output_map(&tr, const_cast<float*>(y_ref), n, d_out))
+      return cudaErrorInvalidValue;
+    cudaError_t e = cudaMemsetAsync(sums3, 0, 3 * sizeof(double), stream);
+    if (e != cudaSuccess) return e;
+  }
   if (!make_packed_map(&ta, xq, n, d_in / 2, BM) || !make_packed_map(&tb, wq, d_out, d_in / 2, BNC))
     return cudaErrorInvalidValue;
   static std::once_flag attr_once;
@@ -481,8 +568,9 @@ cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_
   const int64_t pairs_max = num_sms() / 2;
   const int grid = 2 * (int)(tiles < pairs_max ? tiles : pairs_max);  // CTA pairs (cluster of 2)
   note_launch();
-  w4a4_gemm_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(ty, ta, tb, sx, sw, (int)n, (int)d_in, (int)d_out, y,
-                                                              acc_out, use_tma, status);
+  w4a4_gemm_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(ty, ta, tb, tr, y_ref ? sums3 : nullptr, sx, sw,
+                                                              (int)n, (int)d_in, (int)d_out, y, acc_out, use_tma,
+                                                              status);
   return cudaGetLastError();
 }
 

@@ -170,6 +170,35 @@ def test_w4a4_linear_extreme_accumulators(n, d_in):
 
 
 # ------------------------------------------------------------------------------------------
+# cat_w4a4_linear_sqnr: the GEMM with the SQNR sums formed in its epilogue
+# ------------------------------------------------------------------------------------------
+
+@pytest.mark.parametrize("n,d_in,d_out", [(300, 1024, 520), (513, 512, 256), (257, 4096, 130), (16, 1024, 200),
+                                          (129, 160, 300)])
+def test_w4a4_linear_sqnr_fused(n, d_in, d_out):
+    """y equals cat_w4a4_linear's bit for bit; the sums match the oracle's over the same outputs
+    (fused epilogue for n > 32 and d_out % 4 == 0, else the separate reduction)."""
+    rng = np.random.default_rng(n + 7 * d_in + 13 * d_out)
+    qx = WL.random_codes(rng, (n, d_in)).astype(np.int64)
+    qw = WL.random_codes(rng, (d_out, d_in)).astype(np.int64)
+    sx = rng.uniform(0.01, 2.0, n).astype(np.float32)
+    sw = rng.uniform(0.001, 0.1, d_out).astype(np.float32)
+    xq = torch.from_numpy(sm4x8.pack(qx)).to(DEV)
+    wq = torch.from_numpy(sm4x8.pack(qw)).to(DEV)
+    sx_d, sw_d = torch.from_numpy(sx).to(DEV), torch.from_numpy(sw).to(DEV)
+    y_plain = cat.cat_w4a4_linear(xq, sx_d, wq, sw_d)
+    y_ref = (y_plain.double() + torch.randn(n, d_out, device=DEV, dtype=torch.float64) * 0.05).float().contiguous()
+    for rep in range(2):                                   # twice: the sums restart from zero each call
+        y, out3 = cat.cat_w4a4_linear_sqnr(xq, sx_d, wq, sw_d, y_ref)
+        assert torch.equal(y, y_plain)
+        sig, err = O.sqnr_sums(y_ref.cpu().numpy(), y.cpu().numpy())
+        o = out3.cpu().numpy()
+        assert abs(o[0] - sig) <= 1e-6 * sig and abs(o[1] - err) <= 1e-6 * err
+        assert abs(o[2] - 10 * np.log10(sig / err)) < 1e-5
+    assert cat.cat_device_status()[0] == 0
+
+
+# ------------------------------------------------------------------------------------------
 # cat_sqnr
 # ------------------------------------------------------------------------------------------
 
