@@ -188,9 +188,10 @@ cat_status cat_w4a4_linear(const uint8_t* xq, const float* x_scale, const uint8_
  *   Same arguments as cat_w4a4_linear (without acc_out), plus
  *   y_ref  device [n][d_out] float32: the full-precision output y = W x;
  *   out3   out, device [3] float64: { sum y_ref^2, sum (y_ref - y)^2, 10 log10(ratio) dB }, as cat_sqnr.
- * y is written exactly as cat_w4a4_linear writes it.  For n > 32 and d_out % 4 == 0 the sums are formed
- * in the GEMM's epilogue while y is produced (y is not read back); otherwise the GEMM is followed by
- * the cat_sqnr reduction.  Squares are summed in fp32 over runs of 32 outputs and the runs in float64.
+ * y is written exactly as cat_w4a4_linear writes it.  The sums are formed in the GEMM's epilogue while
+ * y is produced (y is not read back) -- for n > 32 when d_out % 4 == 0, for n <= 32 when the decoded
+ * tokens fit in the weight-streaming kernel's shared memory; otherwise the GEMM is followed by the
+ * cat_sqnr reduction.  Squares are summed in fp32 over runs of at most 32 outputs, the runs in float64.
  */
 cat_status cat_w4a4_linear_sqnr(const uint8_t* xq, const float* x_scale, const uint8_t* Wq, const float* w_scale,
                                 int64_t n, int64_t d_in, int64_t d_out, float* y, const float* y_ref, double* out3,

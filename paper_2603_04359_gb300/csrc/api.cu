@@ -18,8 +18,8 @@ cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_
                                 int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, const float* y_ref,
                                 double* sums3, uint32_t* status, cudaStream_t stream);
 cudaError_t launch_w4a4_gemm_decode(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
-                                    int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, uint32_t* status,
-                                    cudaStream_t stream);
+                                    int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, const float* y_ref,
+                                    double* sums3, uint32_t* status, cudaStream_t stream);
 }  // namespace cat
 
 namespace {
@@ -369,7 +369,8 @@ cat_status cat_w4a4_linear(const uint8_t* xq, const float* x_scale, const uint8_
   uint32_t* status = status_word(&e);
   if (!status) return cuda_fail(e, "status word");
   if (n <= kMaxDecodeTokens)
-    e = cat::launch_w4a4_gemm_decode(xq, x_scale, Wq, w_scale, n, d_in, d_out, y, acc_out, status, (cudaStream_t)stream);
+    e = cat::launch_w4a4_gemm_decode(xq, x_scale, Wq, w_scale, n, d_in, d_out, y, acc_out, nullptr, nullptr, status,
+                                     (cudaStream_t)stream);
   else
     e = cat::launch_w4a4_gemm_tc(xq, x_scale, Wq, w_scale, n, d_in, d_out, y, acc_out, nullptr, nullptr, status,
                                  (cudaStream_t)stream);
@@ -396,11 +397,12 @@ cat_status cat_w4a4_linear_sqnr(const uint8_t* xq, const float* x_scale, const u
   cudaStream_t s = (cudaStream_t)stream;
   if (n > kMaxDecodeTokens && d_out % 4 == 0) {  // SQNR sums fused into the GEMM epilogue
     e = cat::launch_w4a4_gemm_tc(xq, x_scale, Wq, w_scale, n, d_in, d_out, y, nullptr, y_ref, out3, status, s);
+  } else if (n > 0 && n <= kMaxDecodeTokens) {  // weight streaming; sums in its epilogue where it can
+    e = cat::launch_w4a4_gemm_decode(xq, x_scale, Wq, w_scale, n, d_in, d_out, y, nullptr, y_ref, out3, status, s);
   } else {  // the GEMM, then the separate reduction
     e = n == 0 ? cudaSuccess
-        : n <= kMaxDecodeTokens
-            ? cat::launch_w4a4_gemm_decode(xq, x_scale, Wq, w_scale, n, d_in, d_out, y, nullptr, status, s)
-            : cat::launch_w4a4_gemm_tc(xq, x_scale, Wq, w_scale, n, d_in, d_out, y, nullptr, nullptr, nullptr, status, s);
+               : cat::launch_w4a4_gemm_tc(xq, x_scale, Wq, w_scale, n, d_in, d_out, y, nullptr, nullptr, nullptr,
+                                          status, s);
     if (e == cudaSuccess) e = cat::launch_sqnr(y_ref, y, n * d_out, out3, s);
   }
   if (e != cudaSuccess) return cuda_fail(e, "cat_w4a4_linear_sqnr launch");

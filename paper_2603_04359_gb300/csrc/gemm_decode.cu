@@ -126,15 +126,22 @@ __global__ void __launch_bounds__(kWarps * 32) w4a4_gemm_decode_kernel(
 int decode_tc_stages(int64_t n, int64_t d_in);
 cudaError_t launch_w4a4_gemm_decode_tc(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw,
                                        int64_t n, int64_t d_in, int64_t d_out, float* y, int32_t* acc_out,
-                                       uint32_t* status, cudaStream_t stream);
+                                       const float* y_ref, double* sums3, uint32_t* status, cudaStream_t stream);
 
 // n <= 32: tcgen05 weight streaming when the decoded tokens fit in shared memory, else mma.sync
 // weight streaming with registers.
+// y_ref != nullptr: also the SQNR sums of y against y_ref into sums3 (in the tcgen05 kernel's
+// epilogue, else by the separate reduction after the GEMM).
 cudaError_t launch_w4a4_gemm_decode(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
-                                    int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, uint32_t* status,
-                                    cudaStream_t stream) {
+                                    int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, const float* y_ref,
+                                    double* sums3, uint32_t* status, cudaStream_t stream) {
   if (decode_tc_stages(n, d_in) > 0)
-    return launch_w4a4_gemm_decode_tc(xq, sx, wq, sw, n, d_in, d_out, y, acc_out, status, stream);
+    return launch_w4a4_gemm_decode_tc(xq, sx, wq, sw, n, d_in, d_out, y, acc_out, y_ref, sums3, status, stream);
+  if (y_ref) {
+    const cudaError_t e = launch_w4a4_gemm_decode(xq, sx, wq, sw, n, d_in, d_out, y, acc_out, nullptr, nullptr, status,
+                                                  stream);
+    return e != cudaSuccess ? e : launch_sqnr(y_ref, y, n * d_out, sums3, stream);
+  }
   const int nt8 = (int)((n + 7) / 8);
 #define CAT_DECODE_CASE(NT)                                                                                     \
   case NT: {                                                                                                    \

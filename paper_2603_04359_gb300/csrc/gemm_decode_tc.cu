@@ -9,8 +9,8 @@
 //   * two producer warps stream 16 KiB packed weight tiles (128 rows x 128 bytes = 256 codes,
 //     128-byte swizzle) through a TMA ring -- two issuers, because one issuer's TMA rate is below
 //     the per-SM share of HBM bandwidth;
-//   * eight decode warps turn each tile into E4M3 in tensor memory (thread = weight row = TMEM lane,
-//     two warps per lane quadrant, each half of the 256 codes);
+//   * eight decode warps, in two groups taking alternate K steps, turn each tile into E4M3 in tensor
+//     memory (thread = weight row = TMEM lane, the whole 256 codes);
 //   * one thread issues tcgen05.mma (A from tensor memory, B from shared memory), accumulating the
 //     exact products q_x q_w 2^-18 in fp32 (|acc| <= 49 d_in < 2^24);
 //   * four epilogue warps read the double-buffered accumulator (thread = output channel) and write
@@ -78,6 +78,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     w4a4_gemm_decode_tc_kernel(const __grid_constant__ CUtensorMap tmW, const uint8_t* __restrict__ xq,
                                const float* __restrict__ sx, const float* __restrict__ sw, int n, int d_in, int d_out,
                                int sp, float* __restrict__ y, int32_t* __restrict__ acc_out,
+                               const float* __restrict__ y_ref, double* __restrict__ sums3,
                                uint32_t* __restrict__ status) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -94,10 +95,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (tid == 0) {
     for (int s = 0; s < sp; ++s) {
       mbar_init(&bars->p_full[s], 1);
-      mbar_init(&bars->p_empty[s], kDecWarps);
+      mbar_init(&bars->p_empty[s], kDecWarps / 2);   // the decode group of that K step
     }
     for (int s = 0; s < SE; ++s) {
-      mbar_init(&bars->full[s], kDecWarps);
+      mbar_init(&bars->full[s], kDecWarps / 2);
       mbar_init(&bars->empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
@@ -206,29 +207,36 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp >= kDecWarp0 && warp < kDecWarp0 + kDecWarps) {
     // ---------------------------------------------------------------- decode: weight row = TMEM lane
-    const int quad = warp & 3, half = (warp - kDecWarp0) >> 2;
+    // two groups of four warps (one per TMEM lane quadrant) take alternate K steps: the decode of a
+    // step is latency-bound (shared-memory loads, tensor-memory stores and their wait), so two steps
+    // are kept in flight; a thread decodes its whole 128-byte row (256 codes, 64 TMEM columns)
+    const int quad = warp & 3, grp = (warp - kDecWarp0) >> 2;
     const int r = quad * 32 + lane;
     uint32_t it = 0;
     bool ok = true;
     for (int u = blockIdx.x; u < num_units && ok; u += gridDim.x)
       for (int ks = 0; ks < num_ks; ++ks, ++it) {
+        if ((it & 1u) != (uint32_t)grp) continue;
         const uint32_t ps = it % sp, s = it % SE;
         if (!(ok = mbar_wait_bounded(&bars->p_full[ps], (it / sp) & 1, abort_flag))) break;
         if (it >= SE && !(ok = mbar_wait_bounded(&bars->empty[s], ((it / SE) - 1) & 1, abort_flag))) break;
         tc_fence_after();
         const uint8_t* prow = pk + ps * kPkStage + r * 128;
-        uint32_t av[32];
 #pragma unroll
-        for (int jj = 0; jj < 4; ++jj) {  // 16-byte chunk j = 4 half + jj of the 128-byte row, at j ^ (r % 8)
-          const int j = 4 * half + jj;
-          const uint4 w = *reinterpret_cast<const uint4*>(prow + ((j ^ (r & 7)) << 4));
-          av[8 * jj + 0] = sm4_lo(w.x); av[8 * jj + 1] = sm4_hi(w.x);
-          av[8 * jj + 2] = sm4_lo(w.y); av[8 * jj + 3] = sm4_hi(w.y);
-          av[8 * jj + 4] = sm4_lo(w.z); av[8 * jj + 5] = sm4_hi(w.z);
-          av[8 * jj + 6] = sm4_lo(w.w); av[8 * jj + 7] = sm4_hi(w.w);
+        for (int half = 0; half < 2; ++half) {
+          uint32_t av[32];
+#pragma unroll
+          for (int jj = 0; jj < 4; ++jj) {  // 16-byte chunk j of the 128-byte row, at j ^ (r % 8)
+            const int j = 4 * half + jj;
+            const uint4 w = *reinterpret_cast<const uint4*>(prow + ((j ^ (r & 7)) << 4));
+            av[8 * jj + 0] = sm4_lo(w.x); av[8 * jj + 1] = sm4_hi(w.x);
+            av[8 * jj + 2] = sm4_lo(w.y); av[8 * jj + 3] = sm4_hi(w.y);
+            av[8 * jj + 4] = sm4_lo(w.z); av[8 * jj + 5] = sm4_hi(w.z);
+            av[8 * jj + 6] = sm4_lo(w.w); av[8 * jj + 7] = sm4_hi(w.w);
+          }
+          __syncwarp();
+          DEC_TMEM_ST32(tmem + ((uint32_t)(quad * 32) << 16) + kAStage0 + 64u * s + 32u * half, av);
         }
-        __syncwarp();
-        DEC_TMEM_ST32(tmem + ((uint32_t)(quad * 32) << 16) + kAStage0 + 64u * s + 32u * half, av);
         dec_tmem_st_wait();
         tc_fence_before();
         __syncwarp();
@@ -242,6 +250,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int quad = warp & 3;
     uint32_t tcount = 0;
     bool ok = true;
+    double sig = 0.0, err = 0.0;                   // SQNR sums (Sec. 2, Eq. 1) when y_ref is given
     for (int u = blockIdx.x; u < num_units && ok; u += gridDim.x, ++tcount) {
       const uint32_t ab = tcount & 1;
       const int o = u * UM + quad * 32 + lane;
@@ -260,12 +269,44 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&bars->acc_empty[ab]);
       if (o < d_out) {
+        float yr[NTOK];                              // all y_ref loads in flight before the first use
+#pragma unroll
+        for (int t = 0; t < NTOK; ++t) yr[t] = (y_ref && t < n) ? __ldcs(y_ref + (int64_t)t * d_out + o) : 0.f;
+        float s_run = 0.f, e_run = 0.f;
 #pragma unroll
         for (int t = 0; t < NTOK; ++t) {
-          if (t >= n) break;
-          const float a = __uint_as_float(acc[t]);
-          y[(int64_t)t * d_out + o] = a * sxs[t] * swo;
-          if (acc_out) acc_out[(int64_t)t * d_out + o] = __float2int_rn(a * kAccScale);
+          if (t < n) {
+            const float a = __uint_as_float(acc[t]);
+            const float v = a * sxs[t] * swo;          // consecutive o across the warp: coalesced stores
+            y[(int64_t)t * d_out + o] = v;
+            if (acc_out) acc_out[(int64_t)t * d_out + o] = __float2int_rn(a * kAccScale);
+            const float e = yr[t] - v;
+            s_run += yr[t] * yr[t];
+            e_run += e * e;
+          }
+        }
+        sig += (double)s_run;
+        err += (double)e_run;
+      }
+    }
+    if (y_ref) {
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        sig += __shfl_xor_sync(0xFFFFFFFFu, sig, off);
+        err += __shfl_xor_sync(0xFFFFFFFFu, err, off);
+      }
+      if (lane == 0) {
+        atomicAdd(&sums3[0], sig);
+        atomicAdd(&sums3[1], err);
+      }
+      __threadfence();
+      asm volatile("bar.sync 2, 128;" ::: "memory");  // this CTA's four epilogue warps have added theirs
+      if (warp == kEpiWarp0 && lane == 0) {
+        unsigned long long* done = reinterpret_cast<unsigned long long*>(&sums3[2]);
+        if (atomicAdd(done, 1ull) == (unsigned long long)gridDim.x - 1) {  // the last CTA forms the ratio
+          __threadfence();
+          const double s_tot = atomicAdd(&sums3[0], 0.0), e_tot = atomicAdd(&sums3[1], 0.0);
+          sums3[2] = (e_tot > 0.0) ? 10.0 * log10(s_tot / e_tot) : (s_tot > 0.0 ? HUGE_VAL : 0.0);
         }
       }
     }
@@ -309,8 +350,8 @@ size_t smem_bytes(int ntok, int num_ks, int sp) {
 
 template <int NTOK>
 cudaError_t launch_ntok(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
-                        int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, uint32_t* status, int sp,
-                        cudaStream_t stream) {
+                        int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, const float* y_ref, double* sums3,
+                        uint32_t* status, int sp, cudaStream_t stream) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return cudaErrorNotSupported;
   const int64_t row_bytes = d_in / 2;
@@ -341,8 +382,12 @@ cudaError_t launch_ntok(const uint8_t* xq, const float* sx, const uint8_t* wq, c
   const int64_t sms = num_sms();
   const unsigned grid = (unsigned)(units < sms ? units : sms);
   note_launch();
+  if (y_ref) {
+    cudaError_t e = cudaMemsetAsync(sums3, 0, 3 * sizeof(double), stream);
+    if (e != cudaSuccess) return e;
+  }
   w4a4_gemm_decode_tc_kernel<NTOK><<<grid, kThreads, smem, stream>>>(map, xq, sx, sw, (int)n, (int)d_in, (int)d_out,
-                                                                      sp, y, acc_out, status);
+                                                                      sp, y, acc_out, y_ref, sums3, status);
   return cudaGetLastError();
 }
 
@@ -360,13 +405,15 @@ int decode_tc_stages(int64_t n, int64_t d_in) {
   return sp >= 3 ? sp : 0;
 }
 
+// y_ref != nullptr: the epilogue also accumulates the SQNR sums of y against y_ref into sums3
+// (zeroed here; sums3[2] ends as the dB value).
 cudaError_t launch_w4a4_gemm_decode_tc(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw,
                                        int64_t n, int64_t d_in, int64_t d_out, float* y, int32_t* acc_out,
-                                       uint32_t* status, cudaStream_t stream) {
+                                       const float* y_ref, double* sums3, uint32_t* status, cudaStream_t stream) {
   const int sp = decode_tc_stages(n, d_in);
   if (sp == 0) return cudaErrorInvalidValue;
-  if (n <= 16) return launch_ntok<16>(xq, sx, wq, sw, n, d_in, d_out, y, acc_out, status, sp, stream);
-  return launch_ntok<32>(xq, sx, wq, sw, n, d_in, d_out, y, acc_out, status, sp, stream);
+  if (n <= 16) return launch_ntok<16>(xq, sx, wq, sw, n, d_in, d_out, y, acc_out, y_ref, sums3, status, sp, stream);
+  return launch_ntok<32>(xq, sx, wq, sw, n, d_in, d_out, y, acc_out, y_ref, sums3, status, sp, stream);
 }
 
 }  // namespace cat
