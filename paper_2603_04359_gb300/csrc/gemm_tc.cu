@@ -81,6 +81,7 @@ static_assert((BNC * 8) % kGroupThreads == 0, "B chunks per decode thread");
 struct Bars {
   uint64_t p_full[SP], p_empty[SP], full[SE], ready[SE], empty[SE], acc_full[2], acc_empty[2], mma_done;
   uint64_t ref_full[kEpiWarps][kEpiBufs];      // y_ref tile loads of each epilogue warp
+  uint32_t fwd_word[SE];                         // even CTA: targets of the odd CTA's st.async per stage
   uint32_t tmem_addr;
   int abort;
 };
@@ -108,6 +109,15 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint64_t* bar, uint32_t rank
   uint32_t remote;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(bar)), "r"(rank));
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote) : "memory");
+}
+// Asynchronous 4-byte store into CTA `rank`'s shared memory whose completion is counted (complete_tx,
+// release at cluster scope) on that CTA's mbarrier; the issuing thread does not wait for it.
+__device__ __forceinline__ void st_async_signal(uint32_t* word, uint64_t* bar, uint32_t rank) {
+  uint32_t rw, rb;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(rw) : "r"(smem_u32(word)), "r"(rank));
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(rb) : "r"(smem_u32(bar)), "r"(rank));
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.u32 [%0], %1, [%2];" ::"r"(rw), "r"(1u), "r"(rb)
+               : "memory");
 }
 __device__ __forceinline__ void tmem_alloc_pair(uint32_t* dst, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst)), "r"(ncols)
@@ -176,7 +186,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       mbar_init(&bars->p_empty[s], kGroupWarps);    // the decode group of that stage
     }
     for (int s = 0; s < SE; ++s) {
-      mbar_init(&bars->full[s], kGroupWarps + 1); // even CTA: its decode group + the odd CTA's forwarder
+      mbar_init(&bars->full[s], kGroupWarps);     // even CTA: its decode group (+ 4 bytes from the odd CTA)
       mbar_init(&bars->ready[s], kGroupWarps);    // odd CTA: its decode group (then forwarded)
       mbar_init(&bars->empty[s], 1);              // the pair MMA's multicast commit
     }
@@ -224,7 +234,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     // ---------------------------------------------------------------- odd CTA: forward stage readiness
     // An arrive on the even CTA's barrier from a thread that has just written shared and tensor
     // memory stalls it for ~1.5k cycles (the cluster-scope release drains its writes), so the decode
-    // warps arrive locally and one thread per decode group carries the stage's readiness over.
+    // warps arrive locally and one thread per decode group carries the stage's readiness over with an
+    // asynchronous 4-byte store that completes bytes on the even CTA's stage barrier.
     if (lane == 0) {
       const uint32_t grp = warp == kMmaWarp ? 0u : 1u;
       uint32_t it = 0;
@@ -235,7 +246,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           const uint32_t s = it % SE;
           if (!(ok = mbar_wait_bounded(&bars->ready[s], (it / SE) & 1, abort_flag))) break;
           tc_fence_after();
-          mbar_arrive_cluster(&bars->full[s], 0);
+          st_async_signal(&bars->fwd_word[s], &bars->full[s], 0);
         }
     }
   } else if (warp == kMmaWarp) {
@@ -473,7 +484,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         __syncwarp();
         if (lane == 0) {
           mbar_arrive(&bars->p_empty[ps]);
-          mbar_arrive(rank == 0 ? &bars->full[s] : &bars->ready[s]);  // local arrives only: cheap
+          if (rank == 1)
+            mbar_arrive(&bars->ready[s]);          // local arrives only: cheap
+          else if (quad == 0)
+            mbar_arrive_expect_tx(&bars->full[s], 4u);  // the odd CTA's 4-byte signal completes the stage
+          else
+            mbar_arrive(&bars->full[s]);
         }
       }
     }
