@@ -49,6 +49,8 @@ struct TcBars {
   uint32_t tmem_addr;
   int abort;
 };
+// the barrier block and the fused kernel's per-unit barriers (<= 8) fit the 256 bytes reserved for them
+static_assert(sizeof(TcBars) + 8 * sizeof(uint64_t) <= 256, "barrier room");
 
 __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
                                          uint32_t accumulate) {

@@ -59,6 +59,7 @@ struct CovBars {
   uint32_t tmem_addr;
   int abort;
 };
+static_assert(sizeof(CovBars) <= 256, "barrier room");
 
 // MN-major operand, 128-byte swizzle: 64 contiguous channels per 128-byte row, one row per token,
 // 8-token groups 1 KiB apart (SBO), 64-channel atoms kBox bytes apart (LBO).

@@ -71,7 +71,8 @@ constexpr uint32_t kEpiOffset = kPkOffset + SP * kPackedStage;
 constexpr uint32_t kRefOffset = kEpiOffset + kEpiWarps * kEpiBufs * kEpiStage;   // y_ref tiles (SQNR)
 constexpr uint32_t kScaleOffset = kRefOffset + kEpiWarps * kEpiBufs * kEpiStage;
 constexpr uint32_t kBarOffset = kScaleOffset + kEpiWarps * BN * 4;
-constexpr size_t kSmemBytes = kBarOffset + 256 + 1024;      // + barriers + alignment slack
+constexpr uint32_t kBarBytes = 1024;                         // room reserved for the barrier block
+constexpr size_t kSmemBytes = kBarOffset + kBarBytes + 1024;  // + barriers + alignment slack
 static_assert(kAccCols + SE * 64 <= kTmemCols, "tensor memory budget");
 static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 static_assert(kPackedStage % 1024 == 0 && kAtomB % 1024 == 0 && kPackedA % 1024 == 0, "128B-swizzle alignment");
@@ -85,6 +86,7 @@ struct Bars {
   uint32_t tmem_addr;
   int abort;
 };
+static_assert(sizeof(Bars) <= kBarBytes, "barrier block must fit its reserved room");
 
 // ---- tensor-memory stores and the TMA store path -------------------------------------------
 #define CAT_TMEM_ST32(taddr, v)                                                                                 \

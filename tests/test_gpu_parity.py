@@ -130,7 +130,7 @@ GEMM_SHAPES = [
     (1, 64, 8), (5, 160, 100), (17, 96, 33),                                            # weight streaming, registers
     (16, 4096, 520), (32, 384, 300), (8, 8192, 200), (24, 2048, 1000), (2, 1024, 17),   # weight streaming, bulk ring
     (33, 128, 256), (128, 256, 256), (129, 160, 300), (300, 384, 520), (257, 4096, 64),  # tcgen05 path
-    (512, 1024, 1024),
+    (512, 1024, 1024), (1024, 512, 6144),                                                # ... several tiles per pair
 ]
 
 
@@ -174,7 +174,8 @@ def test_w4a4_linear_extreme_accumulators(n, d_in):
 # ------------------------------------------------------------------------------------------
 
 @pytest.mark.parametrize("n,d_in,d_out", [(300, 1024, 520), (513, 512, 256), (257, 4096, 130), (16, 1024, 200),
-                                          (129, 160, 300)])
+                                          (129, 160, 300),
+                                          (1024, 512, 6144)])   # several pair tiles per CTA pair
 def test_w4a4_linear_sqnr_fused(n, d_in, d_out):
     """y equals cat_w4a4_linear's bit for bit; the sums match the oracle's over the same outputs
     (fused epilogue for n > 32 and d_out % 4 == 0, else the separate reduction)."""
