@@ -127,8 +127,12 @@ def test_nonfinite_activation_reports_numeric():
 # ------------------------------------------------------------------------------------------
 
 GEMM_SHAPES = [
-    (1, 64, 8), (5, 160, 100), (17, 96, 33),                                            # weight streaming, registers
-    (16, 4096, 520), (32, 384, 300), (8, 8192, 200), (24, 2048, 1000), (2, 1024, 17),   # weight streaming, bulk ring
+    # n <= 32: tcgen05 weight streaming, tokens resident in shared memory (the last five walk many
+    # 128-row units per CTA, the last two with few packed stages beside a large token operand)
+    (1, 64, 8), (5, 160, 100), (17, 96, 33), (16, 4096, 520), (32, 384, 300), (8, 8192, 200),
+    (24, 2048, 1000), (2, 1024, 17), (3, 4096, 20000), (20, 2048, 40000), (9, 8192, 12000),
+    (16, 9216, 300), (32, 4608, 260),
+    (3, 12288, 100),                                  # n <= 32, tokens too large for shared memory: mma.sync
     (33, 128, 256), (128, 256, 256), (129, 160, 300), (300, 384, 520), (257, 4096, 64),  # tcgen05 path
     (512, 1024, 1024), (1024, 512, 6144),                                                # ... several tiles per pair
 ]
@@ -174,11 +178,12 @@ def test_w4a4_linear_extreme_accumulators(n, d_in):
 # ------------------------------------------------------------------------------------------
 
 @pytest.mark.parametrize("n,d_in,d_out", [(300, 1024, 520), (513, 512, 256), (257, 4096, 130), (16, 1024, 200),
-                                          (129, 160, 300),
+                                          (129, 160, 300), (24, 2048, 40000), (16, 9216, 300), (3, 12288, 100),
                                           (1024, 512, 6144)])   # several pair tiles per CTA pair
 def test_w4a4_linear_sqnr_fused(n, d_in, d_out):
     """y equals cat_w4a4_linear's bit for bit; the sums match the oracle's over the same outputs
-    (fused epilogue for n > 32 and d_out % 4 == 0, else the separate reduction)."""
+    (fused in the GEMM epilogue for n > 32 with d_out % 4 == 0 and in the tcgen05 decode kernel,
+    else the separate reduction)."""
     rng = np.random.default_rng(n + 7 * d_in + 13 * d_out)
     qx = WL.random_codes(rng, (n, d_in)).astype(np.int64)
     qw = WL.random_codes(rng, (d_out, d_in)).astype(np.int64)
