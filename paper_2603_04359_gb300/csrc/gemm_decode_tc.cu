@@ -5,16 +5,18 @@
 // With a handful of tokens the packed weight stream (d_out x d_in / 2 bytes) is the whole cost, and
 // the legacy mma.sync path of this GPU is too slow to keep up with HBM, so the weights are the MMA's
 // M dimension (128 rows per unit) and the tokens its N dimension (16 or 32):
-//   * the tokens are decoded once per CTA into a resident K-major, 128B-swizzled E4M3 operand;
+//   * the tokens are decoded once per CTA into a resident K-major, 128B-swizzled E4M3 operand, with
+//     every staging thread's loads in flight at once (the first MMA waits for the whole operand);
 //   * two producer warps stream 16 KiB packed weight tiles (128 rows x 128 bytes = 256 codes,
 //     128-byte swizzle) through a TMA ring -- two issuers, because one issuer's TMA rate is below
 //     the per-SM share of HBM bandwidth;
-//   * eight decode warps, in two groups taking alternate K steps, turn each tile into E4M3 in tensor
-//     memory (thread = weight row = TMEM lane, the whole 256 codes);
+//   * sixteen decode warps, in four groups taking every fourth K step (the decode of a step is a
+//     latency chain), turn each tile into E4M3 in tensor memory (thread = weight row = TMEM lane,
+//     the whole 256 codes);
 //   * one thread issues tcgen05.mma (A from tensor memory, B from shared memory), accumulating the
 //     exact products q_x q_w 2^-18 in fp32 (|acc| <= 49 d_in < 2^24);
 //   * four epilogue warps read the double-buffered accumulator (thread = output channel) and write
-//     y[t][o] with consecutive o across a warp.
+//     y[t][o] with consecutive o across a warp; y_ref, when given, is loaded while the MMAs run.
 // A persistent CTA per SM walks 128-row units.  Every mbarrier wait is bounded; a wait that gives up
 // raises the device status word and all roles drain and exit.
 #include <cstring>
@@ -29,17 +31,33 @@ constexpr int UM = 128;                      // weight rows per unit (MMA M)
 constexpr int KSB = 128;                     // packed bytes per row per K step (256 codes)
 constexpr uint32_t kPkStage = UM * KSB;      // 16 KiB packed tile
 constexpr int kMaxSP = 8;                    // packed stages (runtime count <= this)
-constexpr int SE = 4;                        // decoded A stages in tensor memory, 64 columns each
-constexpr int kThreads = 512;
-constexpr int kMmaWarp = 1, kProd0 = 0, kProd1 = 2;
-constexpr int kDecWarp0 = 4, kDecWarps = 8;
-constexpr int kEpiWarp0 = 12, kEpiWarps = 4;
+constexpr int kMaxSE = 8;                    // decoded A stages in tensor memory, 64 columns each
+constexpr int kThreads = 768;
+constexpr int kProd0 = 0, kProd1 = 2;
+constexpr int kStageWarp0 = 3;               // warps 3.. stage the token operand at the start
+constexpr int kDecWarp0 = 4, kDecWarps = 16, kDecGroups = 4;
+constexpr int kEpiWarp0 = 20, kEpiWarps = 4;
+constexpr int kTokLoads = 4;                 // token loads in flight per staging thread
+constexpr int kGroupBar0 = 4;                // named barriers 4..7: the four warps of a decode group
+
+// Tensor memory: accumulator (group g, buffer b) at column (b * kDecGroups + g) * NTOK, then the
+// decoded A stages of 64 columns.  Stage s is only ever used by group s % kDecGroups, and packed
+// stage ps only by group ps % kDecGroups (both counts are multiples of the group count): every
+// mbarrier phase a group waits for is then the one after the phase it last saw.
+template <int NTOK>
+struct TmemPlan {
+  static constexpr uint32_t kAccCols = 2u * kDecGroups * NTOK;
+  // two stages per group where they fit (a group decodes its next step while the MMAs of the last
+  // one run), else one
+  static constexpr int kSE = kAccCols + 64u * 2 * kDecGroups <= 512u ? 2 * kDecGroups : kDecGroups;
+  static_assert(kAccCols + 64u * kSE <= 512u && kSE <= kMaxSE, "tensor memory plan");
+};
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kAStage0 = 64;            // columns [0, 64): two accumulators of up to 32 columns
 constexpr size_t kSmemBudget = 220 * 1024;
 
 struct DecBars {
-  uint64_t p_full[kMaxSP], p_empty[kMaxSP], full[SE], empty[SE], acc_full[2], acc_empty[2], tok_ready, mma_done;
+  uint64_t p_full[kMaxSP], p_empty[kMaxSP], empty[kMaxSE], acc_full[2], acc_empty[2], tok_ready, mma_done;
+  double sums[4][2];                           // SQNR sums of the four epilogue warps
   uint32_t tmem_addr;
   int abort;
 };
@@ -60,6 +78,16 @@ struct DecBars {
                : "r"(taddr))
 
 __device__ __forceinline__ void dec_tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+// Named barrier over the 128 threads of a decode group; true on every thread if pred is true on any.
+__device__ __forceinline__ bool group_barrier_any(int id, bool pred) {
+  uint32_t r;
+  asm volatile("{ .reg .pred q, p; setp.ne.u32 q, %1, 0; bar.red.or.pred p, %2, 128, q; selp.u32 %0, 1, 0, p; }"
+               : "=r"(r)
+               : "r"((uint32_t)pred), "r"(id)
+               : "memory");
+  return r != 0;
+}
 
 __device__ __forceinline__ void dec_mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
                                            uint32_t accumulate) {
@@ -85,6 +113,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int row_bytes = d_in / 2;
   const int num_ks = (row_bytes + KSB - 1) / KSB;
   const int num_units = (d_out + UM - 1) / UM;
+  const int act_groups = num_ks < kDecGroups ? num_ks : kDecGroups;  // groups with K steps in a unit
+  constexpr int kSE = TmemPlan<NTOK>::kSE;
+  constexpr uint32_t kAStage0 = TmemPlan<NTOK>::kAccCols;
   uint8_t* bst = smem;                                            // tokens, E4M3
   uint8_t* pk = smem + tok_bytes(NTOK, num_ks);                   // sp x 16 KiB packed weight tiles
   DecBars* bars = reinterpret_cast<DecBars*>(pk + (size_t)sp * kPkStage);
@@ -95,18 +126,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (tid == 0) {
     for (int s = 0; s < sp; ++s) {
       mbar_init(&bars->p_full[s], 1);
-      mbar_init(&bars->p_empty[s], kDecWarps / 2);   // the decode group of that K step
+      mbar_init(&bars->p_empty[s], kDecWarps / kDecGroups);   // the decode group of that K step
     }
-    for (int s = 0; s < SE; ++s) {
-      mbar_init(&bars->full[s], kDecWarps / 2);
-      mbar_init(&bars->empty[s], 1);
-    }
+    for (int s = 0; s < kSE; ++s) mbar_init(&bars->empty[s], 1);
     for (int b = 0; b < 2; ++b) {
-      mbar_init(&bars->acc_full[b], 1);
+      mbar_init(&bars->acc_full[b], act_groups);  // the groups with K steps in a unit commit once each
       mbar_init(&bars->acc_empty[b], kEpiWarps);
     }
-    mbar_init(&bars->tok_ready, kDecWarps + kEpiWarps);
-    mbar_init(&bars->mma_done, 1);
+    mbar_init(&bars->tok_ready, kThreads / 32 - kStageWarp0);
+    mbar_init(&bars->mma_done, act_groups);
     bars->abort = 0;
     fence_mbar_init();
   }
@@ -116,17 +144,18 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = bars->tmem_addr;
 
-  if (warp >= kDecWarp0) {
-    // resident token operand, staged by the decode and epilogue warps while the weight tiles start
-    // to stream: slab a (codes 128a .. 128a+127) of token t at a*NTOK*128 + t*128, 16-byte chunk c at
-    // c ^ (t % 8); tokens >= n and codes >= d_in are zero
+  if (warp >= kStageWarp0) {
+    // resident token operand, staged by warps 3.. while the weight tiles start to stream (all of a
+    // thread's loads in flight at once: the first MMA waits for the whole operand): slab a (codes
+    // 128a .. 128a+127) of token t at a*NTOK*128 + t*128, 16-byte chunk c at c ^ (t % 8); tokens >= n
+    // and codes >= d_in are zero
     const int slabs = 2 * num_ks;
-    const int st = tid - kDecWarp0 * 32, nst = (kDecWarps + kEpiWarps) * 32;
+    const int st = tid - kStageWarp0 * 32, nst = kThreads - kStageWarp0 * 32;
     const int items = NTOK * slabs * 4;
-    for (int e0 = st; e0 < items; e0 += 4 * nst) {
-      uint4 w[4];
+    for (int e0 = st; e0 < items; e0 += kTokLoads * nst) {
+      uint4 w[kTokLoads];
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {  // four loads in flight
+      for (int q = 0; q < kTokLoads; ++q) {
         const int e = e0 + q * nst;
         const int j = e & 3, a = (e >> 2) % slabs, t = (e >> 2) / slabs;
         const int off = a * 64 + j * 16;                          // packed byte offset in the row
@@ -134,7 +163,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (e < items && t < n && off < row_bytes) w[q] = *reinterpret_cast<const uint4*>(xq + (int64_t)t * row_bytes + off);
       }
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
+      for (int q = 0; q < kTokLoads; ++q) {
         const int e = e0 + q * nst;
         if (e >= items) break;
         const int j = e & 3, a = (e >> 2) % slabs, t = (e >> 2) / slabs;
@@ -175,76 +204,80 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (uint32_t q = it > (uint32_t)sp ? it - sp : 0; q < it && q < issued_end; ++q)
         if ((q & 1u) == me) mbar_wait_bounded(&bars->p_full[q % sp], (q / sp) & 1, &no_abort);
     }
-  } else if (warp == kMmaWarp) {
-    // ---------------------------------------------------------------- MMA issuer
-    if (lane == 0) {
-      constexpr uint32_t kIdesc = idesc_e4m3_f32(UM, NTOK);
-      const uint32_t bbase = smem_u32(bst);
-      uint32_t it = 0, tcount = 0;
-      bool ok = mbar_wait_bounded(&bars->tok_ready, 0, abort_flag);
+  } else if (warp >= kDecWarp0 && warp < kDecWarp0 + kDecWarps) {
+    // ---------------------------------------------------------------- decode + MMA: weight row = TMEM lane
+    // Four groups of four warps (one per TMEM lane quadrant) take every fourth K step.  A thread
+    // decodes its whole 128-byte row (256 codes, 64 TMEM columns); then the group's leader thread
+    // issues the step's eight MMAs into the group's own accumulator.  One thread issues an MMA about
+    // every 55 cycles whatever N is, so four issuers keep the tensor core fed at N = 16; the four
+    // partial accumulators are added in the epilogue (integers times 2^-18: exact).
+    const int quad = warp & 3, grp = (warp - kDecWarp0) >> 2;
+    const bool leader = quad == 0 && lane == 0;
+    const int r = quad * 32 + lane;
+    constexpr uint32_t kIdesc = idesc_e4m3_f32(UM, NTOK);
+    const uint32_t bbase = smem_u32(bst);
+    uint32_t it = 0, tcount = 0;
+    bool stop = false;
+    if (leader) {
+      mbar_wait_bounded(&bars->tok_ready, 0, abort_flag);
       tc_fence_after();
-      for (int u = blockIdx.x; u < num_units && ok; u += gridDim.x, ++tcount) {
-        const uint32_t ab = tcount & 1;
-        if (tcount >= 2 && !(ok = mbar_wait_bounded(&bars->acc_empty[ab], ((tcount >> 1) - 1) & 1, abort_flag))) break;
-        tc_fence_after();
-        for (int ks = 0; ks < num_ks; ++ks, ++it) {
-          const uint32_t s = it % SE;
-          if (!(ok = mbar_wait_bounded(&bars->full[s], (it / SE) & 1, abort_flag))) break;
+    }
+    for (int u = blockIdx.x; u < num_units && !stop; u += gridDim.x, ++tcount) {
+      const uint32_t ab = tcount & 1;
+      const uint32_t d_acc = tmem + (ab * kDecGroups + grp) * NTOK;
+      bool first = true;                                 // the group's first K step of the unit
+      for (int ks = 0; ks < num_ks; ++ks, ++it) {
+        if (ks % kDecGroups != grp) continue;          // group g takes the steps ks = g (mod 4) of every unit
+        const uint32_t ps = it % sp, s = it % kSE;
+        const bool good = mbar_wait_bounded(&bars->p_full[ps], (it / sp) & 1, abort_flag) &&
+                          (it < (uint32_t)kSE || mbar_wait_bounded(&bars->empty[s], ((it / kSE) - 1) & 1, abort_flag));
+        if (good) {
+          tc_fence_after();
+          const uint8_t* prow = pk + ps * kPkStage + r * 128;
+#pragma unroll
+          for (int half = 0; half < 2; ++half) {
+            uint32_t av[32];
+#pragma unroll
+            for (int jj = 0; jj < 4; ++jj) {  // 16-byte chunk j of the 128-byte row, at j ^ (r % 8)
+              const int j = 4 * half + jj;
+              const uint4 w = *reinterpret_cast<const uint4*>(prow + ((j ^ (r & 7)) << 4));
+              av[8 * jj + 0] = sm4_lo(w.x); av[8 * jj + 1] = sm4_hi(w.x);
+              av[8 * jj + 2] = sm4_lo(w.y); av[8 * jj + 3] = sm4_hi(w.y);
+              av[8 * jj + 4] = sm4_lo(w.z); av[8 * jj + 5] = sm4_hi(w.z);
+              av[8 * jj + 6] = sm4_lo(w.w); av[8 * jj + 7] = sm4_hi(w.w);
+            }
+            __syncwarp();
+            DEC_TMEM_ST32(tmem + ((uint32_t)(quad * 32) << 16) + kAStage0 + 64u * s + 32u * half, av);
+          }
+          dec_tmem_st_wait();
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0 && good) mbar_arrive(&bars->p_empty[ps]);
+        // the group's four warps have stored the stage (and agree on whether to go on)
+        stop = group_barrier_any(kGroupBar0 + grp, *abort_flag != 0);
+        if (stop) break;
+        if (leader) {
+          tc_fence_after();
+          if (first && tcount >= 2) mbar_wait_bounded(&bars->acc_empty[ab], ((tcount >> 1) - 1) & 1, abort_flag);
           tc_fence_after();
           const uint32_t ta = tmem + kAStage0 + 64u * s;
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {  // K = 32 codes per MMA: 8 TMEM columns of A; B slab 2ks + kk/4, +32 B
             const uint64_t db = sdesc_kmajor_sw128(bbase + (uint32_t)((2 * ks + (kk >> 2)) * NTOK * 128)) + 2 * (kk & 3);
-            dec_mma_ts(tmem + ab * 32u, ta + 8u * kk, db, kIdesc, (ks | kk) != 0);
+            dec_mma_ts(d_acc, ta + 8u * kk, db, kIdesc, (first && kk == 0) ? 0u : 1u);
           }
           mma_commit(&bars->empty[s]);
+          if (ks + kDecGroups >= num_ks) mma_commit(&bars->acc_full[ab]);  // the group's last step of the unit
         }
-        if (ok) mma_commit(&bars->acc_full[ab]);
+        first = false;
       }
+    }
+    if (leader && grp < act_groups) {
       mma_commit(&bars->mma_done);  // all MMAs complete before tensor memory is released
       volatile int no_abort = 0;
       mbar_wait_bounded(&bars->mma_done, 0, &no_abort);
     }
-  } else if (warp >= kDecWarp0 && warp < kDecWarp0 + kDecWarps) {
-    // ---------------------------------------------------------------- decode: weight row = TMEM lane
-    // two groups of four warps (one per TMEM lane quadrant) take alternate K steps: the decode of a
-    // step is latency-bound (shared-memory loads, tensor-memory stores and their wait), so two steps
-    // are kept in flight; a thread decodes its whole 128-byte row (256 codes, 64 TMEM columns)
-    const int quad = warp & 3, grp = (warp - kDecWarp0) >> 2;
-    const int r = quad * 32 + lane;
-    uint32_t it = 0;
-    bool ok = true;
-    for (int u = blockIdx.x; u < num_units && ok; u += gridDim.x)
-      for (int ks = 0; ks < num_ks; ++ks, ++it) {
-        if ((it & 1u) != (uint32_t)grp) continue;
-        const uint32_t ps = it % sp, s = it % SE;
-        if (!(ok = mbar_wait_bounded(&bars->p_full[ps], (it / sp) & 1, abort_flag))) break;
-        if (it >= SE && !(ok = mbar_wait_bounded(&bars->empty[s], ((it / SE) - 1) & 1, abort_flag))) break;
-        tc_fence_after();
-        const uint8_t* prow = pk + ps * kPkStage + r * 128;
-#pragma unroll
-        for (int half = 0; half < 2; ++half) {
-          uint32_t av[32];
-#pragma unroll
-          for (int jj = 0; jj < 4; ++jj) {  // 16-byte chunk j of the 128-byte row, at j ^ (r % 8)
-            const int j = 4 * half + jj;
-            const uint4 w = *reinterpret_cast<const uint4*>(prow + ((j ^ (r & 7)) << 4));
-            av[8 * jj + 0] = sm4_lo(w.x); av[8 * jj + 1] = sm4_hi(w.x);
-            av[8 * jj + 2] = sm4_lo(w.y); av[8 * jj + 3] = sm4_hi(w.y);
-            av[8 * jj + 4] = sm4_lo(w.z); av[8 * jj + 5] = sm4_hi(w.z);
-            av[8 * jj + 6] = sm4_lo(w.w); av[8 * jj + 7] = sm4_hi(w.w);
-          }
-          __syncwarp();
-          DEC_TMEM_ST32(tmem + ((uint32_t)(quad * 32) << 16) + kAStage0 + 64u * s + 32u * half, av);
-        }
-        dec_tmem_st_wait();
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) {
-          mbar_arrive(&bars->p_empty[ps]);
-          mbar_arrive(&bars->full[s]);
-        }
-      }
   } else if (warp >= kEpiWarp0) {
     // ---------------------------------------------------------------- epilogue: output channel = TMEM lane
     const int quad = warp & 3;
@@ -254,54 +287,69 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int u = blockIdx.x; u < num_units && ok; u += gridDim.x, ++tcount) {
       const uint32_t ab = tcount & 1;
       const int o = u * UM + quad * 32 + lane;
-      const float swo = o < d_out ? sw[o] : 0.f;
+      const bool o_ok = o < d_out;
+      const float swo = o_ok ? sw[o] : 0.f;
+      float yr[NTOK];                                // y_ref in flight while the MMAs of the unit run
+#pragma unroll
+      for (int t = 0; t < NTOK; ++t) yr[t] = (y_ref && o_ok && t < n) ? __ldcs(y_ref + (int64_t)t * d_out + o) : 0.f;
       if (!(ok = mbar_wait_bounded(&bars->acc_full[ab], (tcount >> 1) & 1, abort_flag))) break;
       __syncwarp();
       tc_fence_after();
-      uint32_t acc[NTOK];
+      float s_run = 0.f, e_run = 0.f;
 #pragma unroll
-      for (int c = 0; c < NTOK / 16; ++c) {
-        uint32_t* a16 = acc + 16 * c;
-        DEC_TMEM_LD16(tmem + ((uint32_t)(quad * 32) << 16) + ab * 32u + 16u * c, a16);
-      }
-      tmem_ld_wait();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->acc_empty[ab]);
-      if (o < d_out) {
-        float yr[NTOK];                              // all y_ref loads in flight before the first use
+      for (int c = 0; c < NTOK / 16; ++c) {          // 16 accumulator columns at a time
+        float acc[16];
 #pragma unroll
-        for (int t = 0; t < NTOK; ++t) yr[t] = (y_ref && t < n) ? __ldcs(y_ref + (int64_t)t * d_out + o) : 0.f;
-        float s_run = 0.f, e_run = 0.f;
+        for (int j = 0; j < 16; ++j) acc[j] = 0.f;
+        for (int g = 0; g < act_groups; ++g) {         // the decode groups' partial accumulators
+          uint32_t part[16];
+          DEC_TMEM_LD16(tmem + ((uint32_t)(quad * 32) << 16) + (ab * kDecGroups + g) * NTOK + 16u * c, part);
+          tmem_ld_wait();
 #pragma unroll
-        for (int t = 0; t < NTOK; ++t) {
-          if (t < n) {
-            const float a = __uint_as_float(acc[t]);
-            const float v = a * sxs[t] * swo;          // consecutive o across the warp: coalesced stores
-            y[(int64_t)t * d_out + o] = v;
-            if (acc_out) acc_out[(int64_t)t * d_out + o] = __float2int_rn(a * kAccScale);
-            const float e = yr[t] - v;
-            s_run += yr[t] * yr[t];
-            e_run += e * e;
+          for (int j = 0; j < 16; ++j) acc[j] += __uint_as_float(part[j]);  // integers times 2^-18: exact
+        }
+        if (c == NTOK / 16 - 1) {
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&bars->acc_empty[ab]);
+        }
+        if (o_ok) {
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const int t = 16 * c + j;
+            if (t < n) {
+              const float a = acc[j];
+              const float v = a * sxs[t] * swo;        // consecutive o across the warp: coalesced stores
+              y[(int64_t)t * d_out + o] = v;
+              if (acc_out) acc_out[(int64_t)t * d_out + o] = __float2int_rn(a * kAccScale);
+              const float e = yr[t] - v;
+              s_run += yr[t] * yr[t];
+              e_run += e * e;
+            }
           }
         }
-        sig += (double)s_run;
-        err += (double)e_run;
       }
+      sig += (double)s_run;
+      err += (double)e_run;
     }
     if (y_ref) {
+      // one pair of float64 atomics per CTA: the four warps' sums meet in shared memory first
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) {
         sig += __shfl_xor_sync(0xFFFFFFFFu, sig, off);
         err += __shfl_xor_sync(0xFFFFFFFFu, err, off);
       }
       if (lane == 0) {
-        atomicAdd(&sums3[0], sig);
-        atomicAdd(&sums3[1], err);
+        bars->sums[quad][0] = sig;
+        bars->sums[quad][1] = err;
       }
-      __threadfence();
-      asm volatile("bar.sync 2, 128;" ::: "memory");  // this CTA's four epilogue warps have added theirs
+      asm volatile("bar.sync 2, 128;" ::: "memory");  // this CTA's four epilogue warps have written theirs
       if (warp == kEpiWarp0 && lane == 0) {
+        const double s_cta = (bars->sums[0][0] + bars->sums[1][0]) + (bars->sums[2][0] + bars->sums[3][0]);
+        const double e_cta = (bars->sums[0][1] + bars->sums[1][1]) + (bars->sums[2][1] + bars->sums[3][1]);
+        atomicAdd(&sums3[0], s_cta);
+        atomicAdd(&sums3[1], e_cta);
+        __threadfence();
         unsigned long long* done = reinterpret_cast<unsigned long long*>(&sums3[2]);
         if (atomicAdd(done, 1ull) == (unsigned long long)gridDim.x - 1) {  // the last CTA forms the ratio
           __threadfence();
@@ -402,7 +450,8 @@ int decode_tc_stages(int64_t n, int64_t d_in) {
   if (fixed >= kSmemBudget) return 0;
   int sp = (int)((kSmemBudget - fixed) / kPkStage);
   if (sp > kMaxSP) sp = kMaxSP;
-  return sp >= 3 ? sp : 0;
+  sp -= sp % kDecGroups;                      // a multiple of the decode groups (see TmemPlan)
+  return sp >= kDecGroups ? sp : 0;
 }
 
 // y_ref != nullptr: the epilogue also accumulates the SQNR sums of y against y_ref into sums3
