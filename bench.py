@@ -15,7 +15,8 @@ same kernels) and the graph is replayed between two CUDA events; every operand, 
 has several copies whose total exceeds 3x the L2 cache and the steps rotate through them.  The
 per-call times (and the roofline of the GEMM) come from graphs of K launches of that call alone over
 the same rotation.  The e2e number issues every call from the host through the Python binding, with
-the step's inputs copied in from pinned host memory and its outputs copied back.
+the step's inputs copied in from pinned host memory and its outputs copied back, the copies of one
+step overlapping the compute of its neighbours (three streams).
 
   python bench.py [--steps K] [--warmup W] [--config NAME] [--impl ours|reference]
   python -m torch.distributed.run --nproc-per-node N ... bench.py --gpus N   (independent replicas)
@@ -384,41 +385,69 @@ def ours_arm(args, rank, world, local):
     gemm_ms = call_ms["cat_w4a4_linear (alone)" if decode else "cat_w4a4_linear_sqnr"]
     sqnr_db = float(sets[(args.steps - 1) % n_sets].out3[2].item())
 
-    # end to end through the public API with host buffers: inputs copied in, outputs copied out,
-    # every call issued by the host (its launch overhead included)
+    # end to end through the public API with host buffers: every step copies its inputs in from pinned
+    # host memory and its outputs (y and the SQNR triple) back out, every call issued by the host (its
+    # launch overhead included).  The copies run on their own streams (one per direction), so step
+    # i + 1's inputs stream in and step i - 1's outputs stream out while step i computes; events keep
+    # each operand set's copies, compute and read-back in order.
     e2e = None
     if not args.no_e2e:
         b0 = sets[0]
         x_h = b0.x.cpu().pin_memory()
         xc_h = b0.xc.cpu().pin_memory()
         yref_h = b0.y_ref.cpu().pin_memory()
-        y_h = torch.empty_like(b0.y, device="cpu").pin_memory()
-        o3_h = torch.empty((3,), dtype=torch.float64).pin_memory()
+        y_h = [torch.empty_like(b0.y, device="cpu").pin_memory() for _ in range(n_sets)]
+        o3_h = [torch.empty((3,), dtype=torch.float64).pin_memory() for _ in range(n_sets)]
         h2d = x_h.numel() * x_h.element_size() + xc_h.numel() * xc_h.element_size() + yref_h.numel() * 4
-        d2h = y_h.numel() * 4 + 3 * 8
+        d2h = y_h[0].numel() * 4 + 3 * 8
+        s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+        ev0 = lambda: torch.cuda.Event()  # noqa: E731
+        computed = [None] * n_sets          # per set: its last step's compute is done
+        drained = [None] * n_sets           # per set: its last step's outputs are read back
 
-        def e2e_step(b):
-            b.x.copy_(x_h, non_blocking=True)
-            b.xc.copy_(xc_h, non_blocking=True)
-            b.y_ref.copy_(yref_h, non_blocking=True)
+        def e2e_step(i):
+            j = i % n_sets
+            b = sets[j]
+            with torch.cuda.stream(s_in):   # inputs of set j may be overwritten once its last compute is done
+                if computed[j] is not None:
+                    s_in.wait_event(computed[j])
+                b.x.copy_(x_h, non_blocking=True)
+                b.xc.copy_(xc_h, non_blocking=True)
+                b.y_ref.copy_(yref_h, non_blocking=True)
+                landed = ev0()
+                landed.record(s_in)
+            stream.wait_event(landed)       # compute: inputs in, and y free once it has been read back
+            if drained[j] is not None:
+                stream.wait_event(drained[j])
             step(b)
-            y_h.copy_(b.y, non_blocking=True)
-            o3_h.copy_(b.out3, non_blocking=True)
+            computed[j] = ev0()
+            computed[j].record(stream)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(computed[j])
+                y_h[j].copy_(b.y, non_blocking=True)
+                o3_h[j].copy_(b.out3, non_blocking=True)
+                drained[j] = ev0()
+                drained[j].record(s_out)
 
-        for i in range(2):
-            e2e_step(sets[i % n_sets])
+        for i in range(2 * n_sets):
+            e2e_step(i)
         torch.cuda.synchronize()
+        computed = [None] * n_sets
+        drained = [None] * n_sets
         barrier(world)
         a, b = ev(), ev()
         a.record(stream)
+        s_in.wait_stream(stream)            # the timed region starts before the first input copy
         for i in range(args.steps):
-            e2e_step(sets[i % n_sets])
+            e2e_step(i)
+        stream.wait_stream(s_out)           # ... and ends after the last read-back
         b.record(stream)
         torch.cuda.synchronize()
         barrier(world)
         e2e_ms = max_over_ranks(a.elapsed_time(b) / args.steps, world)
         e2e = {"value": world * n / (e2e_ms / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
-               "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms}
+               "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms,
+               "overlap": "inputs in, compute, outputs out on three streams (pipelined across steps)"}
 
     st, word = cat.cat_device_status(dev)
     if st != 0:
