@@ -309,13 +309,18 @@ __global__ void __launch_bounds__(kThreads, 1)
 //
 // When every CTA's units fit in tensor memory at once (units per CTA x K <= 512 columns), one
 // cooperative launch does both passes: phase A runs the MMAs once, keeps each unit's x' tile in its
-// own TMEM columns and records the row maxima; a grid-wide barrier; phase B reads the final maxima,
-// quantizes the tiles still in TMEM and writes the codes; a second barrier; then the CTAs holding
-// block 0 turn the row maxima into the steps s = max / 7 in place.  The barrier counters live in a
-// small static array of slots (one per launch in flight, zeroed by the preparation kernel that also
-// zeroes the maxima); every wait is bounded.
-constexpr int kSyncSlots = 64;
+// own TMEM columns and records the row maxima in the launch's scratch slot; a grid-wide barrier;
+// phase B reads the final maxima, quantizes the tiles still in TMEM and writes the codes, and the
+// CTAs holding block 0 write the steps s = max / 7.  The last CTA to leave zeroes the slot (maxima
+// and counters) for the next launch.  Every wait is bounded.
+// Per-launch state of the fused kernel, one slot per launch in flight (slots are handed out round
+// robin, so up to kSyncSlots launches may run at once on different streams): the grid-barrier and
+// exit counters, and the row maxima (float bits).  The last CTA to leave a launch returns its slot to
+// zero, so a launch, a graph replay of it included, always starts from a clean slot.
+constexpr int kSyncSlots = 8;
+constexpr int kAmaxRows = 1 << 17;             // rows the fused path can have (<= 608 units of 128 rows)
 __device__ __align__(16) uint32_t g_tq_sync[kSyncSlots][4];
+__device__ uint32_t g_tq_amax[kSyncSlots][kAmaxRows];
 
 __device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
   uint32_t v;
@@ -342,12 +347,6 @@ __device__ __forceinline__ void grid_barrier(uint32_t* ctr, uint32_t expected, v
     __threadfence();
   }
   epi_bar();
-}
-
-__global__ void tq_prep_kernel(uint32_t* __restrict__ amax_bits, int64_t n, uint32_t* __restrict__ sync) {
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i < n) amax_bits[i] = 0u;
-  if (i < 4) sync[i] = 0u;
 }
 
 // Four two's-complement bytes in [-7, 7] -> the SM4x8 sign-magnitude bytes (sign << 7 | magnitude).
@@ -381,6 +380,7 @@ template <int K>
 __device__ __forceinline__ void quantize_jobs(uint32_t tmem, int64_t u0, int64_t u1, int num_tiles, int n, int d,
                                               const uint32_t* __restrict__ amax_bits, uint32_t* __restrict__ codes,
                                               volatile int* abort_flag, int slot) {
+  // amax_bits: the launch's row maxima (float bits) in its scratch slot
   if (__any_sync(0xFFFFFFFFu, *abort_flag)) return;
   constexpr int kMaxUnits = 512 / K;
   const int lane = threadIdx.x & 31, quad = (threadIdx.x >> 5) & 3;
@@ -426,8 +426,9 @@ __device__ __forceinline__ void quantize_jobs(uint32_t tmem, int64_t u0, int64_t
 template <int K>
 __global__ void __launch_bounds__(kThreads, 1)
     transform_quant_tc_fused_kernel(const __grid_constant__ CUtensorMap tmX, const float* __restrict__ A, int n,
-                                    int d, uint32_t* __restrict__ amax_bits, uint32_t* __restrict__ codes,
-                                    uint32_t* __restrict__ sync, uint32_t* __restrict__ status) {
+                                    int d, float* __restrict__ scale, uint32_t* __restrict__ codes,
+                                    uint32_t* __restrict__ sync, uint32_t* __restrict__ amax_bits,
+                                    uint32_t* __restrict__ status) {
   using C = TcCfg<K>;
   constexpr int kMaxUnits = 512 / K;
   extern __shared__ uint8_t smem_raw[];
@@ -580,9 +581,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // that own TMEM lane quadrants (4 epilogue + 8 converter warps), a 32-column chunk per job
     quant_bar();
     quantize_jobs<K>(tmem, u0, u1, num_tiles, n, d, amax_bits, codes, abort_flag, 0);
-    quant_bar();                                       // all of this CTA's reads of the maxima are done
-    // every CTA has read its maxima: block 0's tiles now turn them into steps in place
-    grid_barrier(&sync[1], gridDim.x, abort_flag, leader);
+    quant_bar();
+    // the steps of the rows this CTA holds in block 0 (the maxima are final since the grid barrier)
     if (!__any_sync(0xFFFFFFFFu, *abort_flag)) {
       for (int64_t u = u0; u < u1; ++u) {
         const int tile = (int)(u % num_tiles);
@@ -594,12 +594,29 @@ __global__ void __launch_bounds__(kThreads, 1)
           sc = __fdiv_rn(a, 7.0f);
         else
           report(status, kStatusNonFinite);
-        reinterpret_cast<float*>(amax_bits)[t] = sc;
+        scale[t] = sc;
       }
     }
     tc_fence_before();
   }
 
+  // the last CTA out returns the launch's slot to zero: every CTA has passed the grid barrier and read
+  // its maxima before it counts itself out
+  __shared__ int last_out;
+  __syncthreads();
+  if (tid == 0) {
+    __threadfence();
+    last_out = atomicAdd(&sync[1], 1u) == gridDim.x - 1;
+  }
+  __syncthreads();
+  if (last_out) {
+    __threadfence();
+    for (int t = tid; t < n; t += kThreads) amax_bits[t] = 0u;
+    if (tid == 0) sync[0] = 0u;
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) sync[1] = 0u;
+  }
   __syncthreads();
   if (bars->abort && tid == 0) report(status, kStatusTimeout);
   if (warp == 0) {
@@ -669,9 +686,11 @@ cudaError_t launch_k(const __nv_bfloat16* x, int64_t n, int64_t d, const float* 
 }
 
 // Address of this device's barrier slots (looked up once per device).
-uint32_t* sync_slots(cudaError_t* err) {
+// The device's slot arrays (grid-barrier and exit counters; row maxima), looked up once per device.
+uint32_t* sync_slots(cudaError_t* err, uint32_t** amax_slots) {
   static std::mutex mu;
   static uint32_t* cache[64] = {nullptr};
+  static uint32_t* amax_cache[64] = {nullptr};
   int dev = 0;
   *err = cudaGetDevice(&dev);
   if (*err != cudaSuccess) return nullptr;
@@ -682,10 +701,13 @@ uint32_t* sync_slots(cudaError_t* err) {
   std::lock_guard<std::mutex> lock(mu);
   if (!cache[dev]) {
     void* p = nullptr;
-    *err = cudaGetSymbolAddress(&p, g_tq_sync);
-    if (*err != cudaSuccess) return nullptr;
+    void* q = nullptr;
+    if ((*err = cudaGetSymbolAddress(&p, g_tq_sync)) != cudaSuccess) return nullptr;
+    if ((*err = cudaGetSymbolAddress(&q, g_tq_amax)) != cudaSuccess) return nullptr;
     cache[dev] = static_cast<uint32_t*>(p);
+    amax_cache[dev] = static_cast<uint32_t*>(q);
   }
+  *amax_slots = amax_cache[dev];
   return cache[dev];
 }
 
@@ -711,11 +733,15 @@ cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, const f
   if (!cooperative_ok()) return cudaErrorNotSupported;
   EncodeTiledFn fn = encode_fn();
   if (!fn) return cudaErrorNotSupported;
+  if (n > kAmaxRows) return cudaErrorNotSupported;
   cudaError_t e;
-  uint32_t* slots = sync_slots(&e);
+  uint32_t* amax_slots = nullptr;
+  uint32_t* slots = sync_slots(&e, &amax_slots);
   if (!slots) return e;
   static std::atomic<uint32_t> next_slot{0};
-  uint32_t* sync = slots + 4 * (next_slot.fetch_add(1) % kSyncSlots);
+  const uint32_t slot = next_slot.fetch_add(1) % kSyncSlots;
+  uint32_t* sync = slots + 4 * slot;
+  uint32_t* amax_bits = amax_slots + (size_t)kAmaxRows * slot;
   CUtensorMap map;
   memset(&map, 0, sizeof(map));
   cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)n};
@@ -733,10 +759,6 @@ cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, const f
                                 (int)C::SMEM);
   });
   if (attr != cudaSuccess) return attr;
-  const int64_t zn = n > 4 ? n : 4;
-  note_launch();
-  tq_prep_kernel<<<(unsigned)((zn + 255) / 256), 256, 0, stream>>>(amax, n, sync);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
   cudaLaunchConfig_t cfg;
   memset(&cfg, 0, sizeof(cfg));
   cfg.gridDim = dim3((unsigned)grid, 1, 1);
@@ -749,8 +771,8 @@ cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, const f
   cfg.attrs = attrs;
   cfg.numAttrs = 1;
   note_launch();
-  return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<K>, map, A, (int)n, (int)d, amax, words, sync,
-                            status);
+  return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<K>, map, A, (int)n, (int)d,
+                            reinterpret_cast<float*>(amax), words, sync, amax_bits, status);
 }
 
 }  // namespace
@@ -771,8 +793,9 @@ cudaError_t launch_transform_quantize_tc(const void* x, int64_t n, int64_t d, in
 }  // namespace cat
 
 namespace cat {
-// Both phases and the steps in one cooperative launch (after a preparation kernel) when every CTA's
-// units fit in tensor memory; cudaErrorNotSupported otherwise (the caller takes the two-pass path).
+// Both phases and the steps in one cooperative launch when every CTA's units fit in tensor memory
+// (the row maxima go to a slot of device scratch that the launch leaves zeroed); cudaErrorNotSupported
+// otherwise (the caller takes the two-pass path).
 cudaError_t launch_transform_quantize_tc_fused(const void* x, int64_t n, int64_t d, int k, const float* A,
                                                uint32_t* amax, uint32_t* words, uint32_t* status, cudaStream_t stream) {
   const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
