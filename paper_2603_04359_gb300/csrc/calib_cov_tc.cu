@@ -232,13 +232,19 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int e = 0; e < 32; ++e) v32[e] = 0.f;
           if (live) {
 #pragma unroll 1
-            for (int a = 0; a < used; ++a) {
-              uint32_t rr[32];
+            for (int a = 0; a < used; a += 2) {      // two accumulators per tensor-memory round trip
+              uint32_t rr[32], rq[32];
               __syncwarp();
               CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + ((a * G2 + ih) * G2 + jh) * 128 + col, rr);
+              if (a + 1 < used)
+                CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + (((a + 1) * G2 + ih) * G2 + jh) * 128 + col, rq);
               tmem_ld_wait();
 #pragma unroll
               for (int e = 0; e < 32; ++e) v32[e] += __uint_as_float(rr[e]);
+              if (a + 1 < used) {
+#pragma unroll
+                for (int e = 0; e < 32; ++e) v32[e] += __uint_as_float(rq[e]);
+              }
             }
           }
 #pragma unroll
@@ -262,12 +268,19 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int cb = G2 == 2 ? 0 : (R / k) * k;   // first column of R's diagonal block in the tile
 #pragma unroll 1
           for (int C4 = cb + 4 * l4; C4 < cb + kw; C4 += 4 * lpr) {
-            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
             const uint32_t off = red_addr + (uint32_t)(R * 128 + C4) * 4u;
-            for (uint32_t src = 0; src < S; ++src) {    // fixed order: deterministic sums
-              const float4 v = ld_cluster_f32x4(map_cluster(off, src));
-              acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
-            }
+            // every CTA's value in flight at once (remote shared-memory loads are slow), then the
+            // sum in a fixed order: deterministic
+            float4 part[kMaxCluster];
+#pragma unroll
+            for (int src = 0; src < kMaxCluster; ++src)
+              part[src] = (uint32_t)src < S ? ld_cluster_f32x4(map_cluster(off, (uint32_t)src)) : make_float4(0.f, 0.f, 0.f, 0.f);
+            float4 acc = part[0];
+#pragma unroll
+            for (int src = 1; src < kMaxCluster; ++src)
+              if ((uint32_t)src < S) {
+                acc.x += part[src].x; acc.y += part[src].y; acc.z += part[src].z; acc.w += part[src].w;
+              }
             // staged tile (ih, jh) is transposed: entry (R, C) belongs to group row jh*128 + R
             const int grow = c0 + jh * 128 + R;
             if (grow >= d) continue;
