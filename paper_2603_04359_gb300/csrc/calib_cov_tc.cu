@@ -68,14 +68,24 @@ __device__ __forceinline__ uint64_t sdesc_mnmajor_sw128(uint32_t saddr, uint32_t
          (1ull << 46) | (2ull << 61);
 }
 
-// float -> double without the FP64 pipe: re-bias the exponent of a normal float (zero, subnormal,
-// inf and nan take the regular conversion).
+// float -> double without the FP64 pipe (the exact widening, done in integer registers): a normal
+// float re-biases its exponent; a subnormal is normalized (its leading one becomes the implicit
+// bit); zero keeps its sign; inf and nan keep their payload under the all-ones exponent.
 __device__ __forceinline__ double f32_to_f64_exact(float f) {
   const uint32_t u = __float_as_uint(f);
-  const uint32_t e = (u >> 23) & 0xFFu;
-  if (e == 0u || e == 0xFFu) return (double)f;
-  const uint64_t bits = ((uint64_t)(u >> 31) << 63) | ((uint64_t)(e - 127u + 1023u) << 52) |
-                        ((uint64_t)(u & 0x7FFFFFu) << 29);
+  const uint32_t e = (u >> 23) & 0xFFu, m = u & 0x7FFFFFu;
+  const uint64_t sign = (uint64_t)(u >> 31) << 63;
+  uint64_t bits;
+  if (e == 0xFFu) {
+    bits = sign | (0x7FFull << 52) | ((uint64_t)m << 29);
+  } else if (e != 0u) {
+    bits = sign | ((uint64_t)(e - 127u + 1023u) << 52) | ((uint64_t)m << 29);
+  } else if (m == 0u) {
+    bits = sign;
+  } else {                                   // m * 2^-149 with its leading one at bit p
+    const int p = 31 - __clz(m);
+    bits = sign | ((uint64_t)(p - 149 + 1023) << 52) | ((uint64_t)((m << (23 - p)) & 0x7FFFFFu) << 29);
+  }
   return __longlong_as_double((long long)bits);
 }
 
@@ -263,39 +273,53 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int rpp = 32 / lpr;                     // rows per warp pass
         const int sub = lane / lpr, l4 = lane % lpr;
         const uint32_t red_addr = smem_u32(red);
+        // kRowsInFlight rows per round: all their remote loads (S per row and 4-column group) are in
+        // flight before the first sum (remote shared-memory loads are slow); the sums run in a fixed
+        // source order, so they are deterministic
+        constexpr int kRowsInFlight = 4;
 #pragma unroll 1
-        for (int R = r_lo + ew * rpp + sub; R < r_lo + rows; R += 4 * rpp) {
-          const int cb = G2 == 2 ? 0 : (R / k) * k;   // first column of R's diagonal block in the tile
+        for (int R0 = r_lo + ew * rpp + sub; R0 < r_lo + rows; R0 += kRowsInFlight * 4 * rpp) {
 #pragma unroll 1
-          for (int C4 = cb + 4 * l4; C4 < cb + kw; C4 += 4 * lpr) {
-            const uint32_t off = red_addr + (uint32_t)(R * 128 + C4) * 4u;
-            // every CTA's value in flight at once (remote shared-memory loads are slow), then the
-            // sum in a fixed order: deterministic
-            float4 part[kMaxCluster];
+          for (int C4i = 4 * l4; C4i < kw; C4i += 4 * lpr) {
+            float4 part[kRowsInFlight][kMaxCluster];
 #pragma unroll
-            for (int src = 0; src < kMaxCluster; ++src)
-              part[src] = (uint32_t)src < S ? ld_cluster_f32x4(map_cluster(off, (uint32_t)src)) : make_float4(0.f, 0.f, 0.f, 0.f);
-            float4 acc = part[0];
+            for (int q = 0; q < kRowsInFlight; ++q) {
+              const int R = R0 + q * 4 * rpp;
+              const int cb = G2 == 2 ? 0 : (R / k) * k;   // first column of R's diagonal block in the tile
+              const uint32_t off = red_addr + (uint32_t)(R * 128 + cb + C4i) * 4u;
 #pragma unroll
-            for (int src = 1; src < kMaxCluster; ++src)
-              if ((uint32_t)src < S) {
-                acc.x += part[src].x; acc.y += part[src].y; acc.z += part[src].z; acc.w += part[src].w;
+              for (int src = 0; src < kMaxCluster; ++src)
+                part[q][src] = (R < r_lo + rows && (uint32_t)src < S) ? ld_cluster_f32x4(map_cluster(off, (uint32_t)src))
+                                                                       : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+#pragma unroll
+            for (int q = 0; q < kRowsInFlight; ++q) {
+              const int R = R0 + q * 4 * rpp;
+              if (R >= r_lo + rows) break;
+              const int cb = G2 == 2 ? 0 : (R / k) * k;
+              const int C4 = cb + C4i;
+              float4 acc = part[q][0];
+#pragma unroll
+              for (int src = 1; src < kMaxCluster; ++src)
+                if ((uint32_t)src < S) {
+                  acc.x += part[q][src].x; acc.y += part[q][src].y; acc.z += part[q][src].z; acc.w += part[q][src].w;
+                }
+              // staged tile (ih, jh) is transposed: entry (R, C) belongs to group row jh*128 + R
+              const int grow = c0 + jh * 128 + R;
+              if (grow >= d) continue;
+              double* dst = sigma + (int64_t)grow * k + ((ih * 128 + C4) % k);
+              const double v[4] = {f32_to_f64_exact(acc.x), f32_to_f64_exact(acc.y), f32_to_f64_exact(acc.z),
+                                   f32_to_f64_exact(acc.w)};
+              if (mode == 2) {
+#pragma unroll
+                for (int e = 0; e < 4; ++e) atomicAdd(dst + e, v[e]);
+              } else if (mode == 1) {
+#pragma unroll
+                for (int e = 0; e < 4; ++e) dst[e] += v[e];
+              } else {
+                reinterpret_cast<double2*>(dst)[0] = make_double2(v[0], v[1]);
+                reinterpret_cast<double2*>(dst)[1] = make_double2(v[2], v[3]);
               }
-            // staged tile (ih, jh) is transposed: entry (R, C) belongs to group row jh*128 + R
-            const int grow = c0 + jh * 128 + R;
-            if (grow >= d) continue;
-            double* dst = sigma + (int64_t)grow * k + ((ih * 128 + C4) % k);
-            const double v[4] = {f32_to_f64_exact(acc.x), f32_to_f64_exact(acc.y), f32_to_f64_exact(acc.z),
-                                 f32_to_f64_exact(acc.w)};
-            if (mode == 2) {
-#pragma unroll
-              for (int e = 0; e < 4; ++e) atomicAdd(dst + e, v[e]);
-            } else if (mode == 1) {
-#pragma unroll
-              for (int e = 0; e < 4; ++e) dst[e] += v[e];
-            } else {
-              reinterpret_cast<double2*>(dst)[0] = make_double2(v[0], v[1]);
-              reinterpret_cast<double2*>(dst)[1] = make_double2(v[2], v[3]);
             }
           }
         }
