@@ -294,7 +294,12 @@ class BufferSet:
                                                           self.sigma, self.xq, self.sx, self.y, self.out3))
 
 
-def ours_arm(args, rank, world, local):
+class DeviceTimeout(RuntimeError):
+    """A bounded wait in a kernel gave up (status word bit 0; bits 8..12 name the kernel and bits
+    16..31 the source line of the first wait that gave up)."""
+
+
+def ours_arm(args, rank, world, local, retried=None):
     import paper_2603_04359_gb300 as cat
     cat.load_library()
     dev = torch.device("cuda", local)
@@ -334,7 +339,7 @@ def ours_arm(args, rank, world, local):
     torch.cuda.synchronize()
     st, word = cat.cat_device_status(dev)
     if st != 0:
-        raise RuntimeError(f"device status {st} ({word:#x}) after warm-up")
+        raise (DeviceTimeout if word & 1 else RuntimeError)(f"device status {st} ({word:#x}) after warm-up")
 
     # the timed region: one CUDA graph of exactly `steps` steps (sets in rotation), replayed once;
     # host launch overhead is not part of the device-side number (the e2e number below has it)
@@ -451,7 +456,7 @@ def ours_arm(args, rank, world, local):
 
     st, word = cat.cat_device_status(dev)
     if st != 0:
-        raise RuntimeError(f"device status {st} ({word:#x}) after timing")
+        raise (DeviceTimeout if word & 1 else RuntimeError)(f"device status {st} ({word:#x}) after timing")
 
     if rank != 0:
         return
@@ -501,6 +506,8 @@ def ours_arm(args, rank, world, local):
                                  "source": "measured now: torch._int_mm int8 8192^3, best of 5 (cuBLAS IMMA)"}
     if e2e:
         line["e2e"] = e2e
+    if retried:
+        line["retried_after"] = retried
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = run_cpu_baseline(L, args.kind, k, args.cpu_seconds)
     print(json.dumps(line), flush=True)
@@ -514,7 +521,13 @@ def main():
         reference_arm(args, int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")))
         return
     rank, world, local = dist_setup()
-    ours_arm(args, rank, world, local)
+    try:
+        ours_arm(args, rank, world, local)
+    except DeviceTimeout as e:           # one fresh measurement on a single GPU, recorded in the line
+        if world > 1:
+            raise
+        print(f"bench: {e}; measuring once more", file=sys.stderr, flush=True)
+        ours_arm(args, rank, world, local, retried=str(e))
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()

@@ -174,7 +174,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int64_t u = u0; u < u1 && ok; ++u, ++j) {
         const int b = (int)(u / num_tiles), tile = (int)(u % num_tiles);
         const uint32_t s = j % kXStages;
-        if (j >= kXStages && !(ok = mbar_wait_bounded(&bars->x_empty[s], ((j / kXStages) - 1) & 1, abort_flag))) break;
+        if (j >= kXStages && !(ok = mbar_wait_bounded(&bars->x_empty[s], ((j / kXStages) - 1) & 1, abort_flag, __LINE__))) break;
         mbar_arrive_expect_tx(&bars->x_full[s], C::X_STAGE);
 #pragma unroll
         for (int a = 0; a < C::ATOMS; ++a)
@@ -194,13 +194,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int64_t u = u0; u < u1 && ok; ++u, ++j) {
         const int b = (int)(u / num_tiles);
         if (b != cur_b) {
-          if (!(ok = mbar_wait_bounded(&bars->t_full, version & 1, abort_flag))) break;
+          if (!(ok = mbar_wait_bounded(&bars->t_full, version & 1, abort_flag, __LINE__))) break;
           ++version;
           cur_b = b;
         }
         const uint32_t s = j % kXStages, sd = j & 1;
-        if (!(ok = mbar_wait_bounded(&bars->x_full[s], (j / kXStages) & 1, abort_flag))) break;
-        if (j >= 2 && !(ok = mbar_wait_bounded(&bars->d_empty[sd], ((j >> 1) - 1) & 1, abort_flag))) break;
+        if (!(ok = mbar_wait_bounded(&bars->x_full[s], (j / kXStages) & 1, abort_flag, __LINE__))) break;
+        if (j >= 2 && !(ok = mbar_wait_bounded(&bars->d_empty[sd], ((j >> 1) - 1) & 1, abort_flag, __LINE__))) break;
         tc_fence_after();
         const uint32_t dcol = tmem + sd * K;
         const uint32_t xbase = smem_u32(xs + s * C::X_STAGE);
@@ -232,7 +232,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int64_t u = u0; u < u1 && ok; ++u) {
       const int b = (int)(u / num_tiles);
       if (b == cur_b) continue;
-      if (version > 0 && !(ok = mbar_wait_bounded(&bars->t_empty, (version - 1) & 1, abort_flag))) break;
+      if (version > 0 && !(ok = mbar_wait_bounded(&bars->t_empty, (version - 1) & 1, abort_flag, __LINE__))) break;
       cur_b = b;
       split_block<K>(A + (size_t)b * K * K, ts, ct);
       fence_proxy_async_smem();
@@ -255,7 +255,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float a = __uint_as_float(amax_bits[t]);
         inv = (isfinite(a) && a > 0.f) ? __fdiv_rn(7.0f, a) : 0.f;
       }
-      if (!(ok = mbar_wait_bounded(&bars->d_full[sd], (j >> 1) & 1, abort_flag))) break;
+      if (!(ok = mbar_wait_bounded(&bars->d_full[sd], (j >> 1) & 1, abort_flag, __LINE__))) break;
       __syncwarp();
       tc_fence_after();
       float m = 0.f;
@@ -298,7 +298,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   __syncthreads();
-  if (bars->abort && tid == 0) report(status, kStatusTimeout);
+  if (bars->abort && tid == 0) report(status, timeout_bits(kWhereTransform2Pass, bars->abort));
   if (warp == 0) {
     tc_fence_after();
     tmem_dealloc(tmem, C::TMEM_COLS);
@@ -340,7 +340,7 @@ __device__ __forceinline__ void grid_barrier(uint32_t* ctr, uint32_t expected, v
     for (uint32_t it = 0; ld_acquire_gpu(ctr) < expected; ++it) {
       __nanosleep(64);                                  // keep the polls off the counter's L2 slice
       if ((it & 63u) == 63u && (*abort_flag || globaltimer_ns() - t0 > kWaitLimitNs)) {
-        *abort_flag = 1;
+        if (*abort_flag == 0) *abort_flag = __LINE__;
         break;
       }
     }
@@ -474,7 +474,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int64_t u = u0; u < u1 && ok; ++u, ++j) {
         const int b = (int)(u / num_tiles), tile = (int)(u % num_tiles);
         const uint32_t st = j % kXStages;
-        if (j >= kXStages && !(ok = mbar_wait_bounded(&bars->x_empty[st], ((j / kXStages) - 1) & 1, abort_flag))) break;
+        if (j >= kXStages && !(ok = mbar_wait_bounded(&bars->x_empty[st], ((j / kXStages) - 1) & 1, abort_flag, __LINE__))) break;
         mbar_arrive_expect_tx(&bars->x_full[st], C::X_STAGE);
 #pragma unroll
         for (int a = 0; a < C::ATOMS; ++a)
@@ -494,12 +494,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int64_t u = u0; u < u1 && ok; ++u, ++j) {
         const int b = (int)(u / num_tiles);
         if (b != cur_b) {
-          if (!(ok = mbar_wait_bounded(&bars->t_full, version & 1, abort_flag))) break;
+          if (!(ok = mbar_wait_bounded(&bars->t_full, version & 1, abort_flag, __LINE__))) break;
           ++version;
           cur_b = b;
         }
         const uint32_t st = j % kXStages;
-        if (!(ok = mbar_wait_bounded(&bars->x_full[st], (j / kXStages) & 1, abort_flag))) break;
+        if (!(ok = mbar_wait_bounded(&bars->x_full[st], (j / kXStages) & 1, abort_flag, __LINE__))) break;
         tc_fence_after();
         const uint32_t dcol = tmem + j * K;
         const uint32_t xbase = smem_u32(xs + st * C::X_STAGE);
@@ -531,7 +531,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int64_t u = u0; u < u1 && ok; ++u) {
       const int b = (int)(u / num_tiles);
       if (b == cur_b) continue;
-      if (version > 0 && !(ok = mbar_wait_bounded(&bars->t_empty, (version - 1) & 1, abort_flag))) break;
+      if (version > 0 && !(ok = mbar_wait_bounded(&bars->t_empty, (version - 1) & 1, abort_flag, __LINE__))) break;
       cur_b = b;
       split_block<K>(A + (size_t)b * K * K, ts, ct);
       fence_proxy_async_smem();
@@ -553,7 +553,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int j = 0; j < nu; ++j) {
       const int tile = (int)((u0 + j) % num_tiles);
       const int t = tile * TM + quad * 32 + lane;
-      const bool got = !*abort_flag && mbar_wait_bounded(&unit_full[j], 0, abort_flag);
+      const bool got = !*abort_flag && mbar_wait_bounded(&unit_full[j], 0, abort_flag, __LINE__);
       if (!__all_sync(0xFFFFFFFFu, got)) break;        // warp-uniform: TMEM loads need the whole warp
       tc_fence_after();
       float m = 0.f;
@@ -618,7 +618,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (tid == 0) sync[1] = 0u;
   }
   __syncthreads();
-  if (bars->abort && tid == 0) report(status, kStatusTimeout);
+  if (bars->abort && tid == 0) report(status, timeout_bits(kWhereTransformFused, bars->abort));
   if (warp == 0) {
     tc_fence_after();
     tmem_dealloc(tmem, 512);

@@ -167,7 +167,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       int c = 0;
       for (; c < chunks && ok; ++c) {
         const uint32_t s = c % kStages;
-        if (c >= kStages && !(ok = mbar_wait_bounded(&bars->empty[s], ((c / kStages) - 1) & 1, abort_flag))) break;
+        if (c >= kStages && !(ok = mbar_wait_bounded(&bars->empty[s], ((c / kStages) - 1) & 1, abort_flag, __LINE__))) break;
         mbar_arrive_expect_tx(&bars->full[s], C::STAGE);
         for (int bx = 0; bx < C::BOXES; ++bx)
           tma_load_2d(smem + s * C::STAGE + bx * kBox, &tmX, c0 + 64 * bx, t_begin + c * kChunk, &bars->full[s]);
@@ -181,7 +181,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int c = 0; c < chunks && ok; ++c) {
         const uint32_t s = c % kStages;
-        if (!(ok = mbar_wait_bounded(&bars->full[s], (c / kStages) & 1, abort_flag))) break;
+        if (!(ok = mbar_wait_bounded(&bars->full[s], (c / kStages) & 1, abort_flag, __LINE__))) break;
         tc_fence_after();
         const uint32_t base = smem_u32(smem + s * C::STAGE);
 #pragma unroll
@@ -215,7 +215,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t rank = cluster_ctarank();
   const bool have_acc = chunks > 0 && !bars->abort;
   if (epi && have_acc) {
-    if (!mbar_wait_bounded(&bars->acc_full, 0, abort_flag)) {
+    if (!mbar_wait_bounded(&bars->acc_full, 0, abort_flag, __LINE__)) {
       // gave up: the tile below is not written; the status word reports it
     }
     __syncwarp();
@@ -328,7 +328,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       cluster_sync_all();                             // the tiles may be overwritten / released
     }
 
-  if (bars->abort && tid == 0) report(status, kStatusTimeout);
+  if (bars->abort && tid == 0) report(status, timeout_bits(kWhereCalib, bars->abort));
   if (warp == 0) {
     tc_fence_after();
     tmem_dealloc(tmem, C::TMEM_COLS);

@@ -21,7 +21,19 @@ inline void note_launch() { g_kernel_launches.fetch_add(1, std::memory_order_rel
 enum : uint32_t {
   kStatusTimeout = 1u,     // a bounded wait gave up
   kStatusNonFinite = 2u,   // a non-finite value reached a quantizer
+  // with kStatusTimeout: the kernel (bits 8..12) and, in bits 16..31, the source line of the first
+  // wait that gave up
+  kWhereTransform2Pass = 1u << 8,
+  kWhereTransformFused = 1u << 9,
+  kWhereGemm = 1u << 10,
+  kWhereGemmDecode = 1u << 11,
+  kWhereCalib = 1u << 12,
 };
+
+// The status bits a kernel raises when a wait gave up: abort holds the line of the first one.
+__host__ __device__ constexpr uint32_t timeout_bits(uint32_t where, int abort) {
+  return kStatusTimeout | where | ((uint32_t)(abort & 0xFFFF) << 16);
+}
 
 // Upper bound of any single pipeline wait, in nanoseconds of %globaltimer.
 constexpr uint64_t kWaitLimitNs = 1000000000ull;
@@ -90,8 +102,9 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Wait until the phase with the given parity has completed.  Returns false (and raises
-// `*abort`) if `*abort` was already raised by another thread or the wait exceeded the limit.
-__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, volatile int* abort) {
+// `*abort`, to `site` if it was not raised yet) if `*abort` was already raised by another thread or
+// the wait exceeded the limit.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, volatile int* abort, int site = 1) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t it = 1;; ++it) {
@@ -99,7 +112,7 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity
     if ((it & 63u) == 0u) {
       if (*abort) return false;
       if (globaltimer_ns() - t0 > kWaitLimitNs) {
-        *abort = 1;
+        if (*abort == 0) *abort = site;
         return false;
       }
     }
@@ -125,6 +138,13 @@ __device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* m
           smem_u32(smem_dst)),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
       : "memory");
+}
+
+// Bring a tensor tile into L2 only (no shared memory, no completion to wait for).
+__device__ __forceinline__ void tma_prefetch_l2_2d(const CUtensorMap* map, int32_t x, int32_t y) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y)
+               : "memory");
 }
 
 __device__ __forceinline__ void prefetch_tensormap(const CUtensorMap* map) {

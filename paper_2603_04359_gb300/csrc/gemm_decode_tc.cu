@@ -192,7 +192,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int ks = 0; ks < num_ks; ++ks, ++it) {
           if ((it & 1u) != me) continue;
           const uint32_t s = it % sp, use = it / sp;
-          if (use > 0 && !(ok = mbar_wait_bounded(&bars->p_empty[s], (use - 1) & 1, abort_flag))) break;
+          if (use > 0 && !(ok = mbar_wait_bounded(&bars->p_empty[s], (use - 1) & 1, abort_flag, __LINE__))) break;
           mbar_arrive_expect_tx(&bars->p_full[s], kPkStage);
           tma_load_2d(pk + s * kPkStage, &tmW, ks * KSB, u * UM, &bars->p_full[s]);
           issued_end = it + 1;
@@ -219,7 +219,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t it = 0, tcount = 0;
     bool stop = false;
     if (leader) {
-      mbar_wait_bounded(&bars->tok_ready, 0, abort_flag);
+      mbar_wait_bounded(&bars->tok_ready, 0, abort_flag, __LINE__);
       tc_fence_after();
     }
     for (int u = blockIdx.x; u < num_units && !stop; u += gridDim.x, ++tcount) {
@@ -229,8 +229,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int ks = 0; ks < num_ks; ++ks, ++it) {
         if (ks % kDecGroups != grp) continue;          // group g takes the steps ks = g (mod 4) of every unit
         const uint32_t ps = it % sp, s = it % kSE;
-        const bool good = mbar_wait_bounded(&bars->p_full[ps], (it / sp) & 1, abort_flag) &&
-                          (it < (uint32_t)kSE || mbar_wait_bounded(&bars->empty[s], ((it / kSE) - 1) & 1, abort_flag));
+        const bool good = mbar_wait_bounded(&bars->p_full[ps], (it / sp) & 1, abort_flag, __LINE__) &&
+                          (it < (uint32_t)kSE || mbar_wait_bounded(&bars->empty[s], ((it / kSE) - 1) & 1, abort_flag, __LINE__));
         if (good) {
           tc_fence_after();
           const uint8_t* prow = pk + ps * kPkStage + r * 128;
@@ -259,7 +259,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (stop) break;
         if (leader) {
           tc_fence_after();
-          if (first && tcount >= 2) mbar_wait_bounded(&bars->acc_empty[ab], ((tcount >> 1) - 1) & 1, abort_flag);
+          if (first && tcount >= 2) mbar_wait_bounded(&bars->acc_empty[ab], ((tcount >> 1) - 1) & 1, abort_flag, __LINE__);
           tc_fence_after();
           const uint32_t ta = tmem + kAStage0 + 64u * s;
 #pragma unroll
@@ -292,7 +292,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       float yr[NTOK];                                // y_ref in flight while the MMAs of the unit run
 #pragma unroll
       for (int t = 0; t < NTOK; ++t) yr[t] = (y_ref && o_ok && t < n) ? __ldcs(y_ref + (int64_t)t * d_out + o) : 0.f;
-      if (!(ok = mbar_wait_bounded(&bars->acc_full[ab], (tcount >> 1) & 1, abort_flag))) break;
+      if (!(ok = mbar_wait_bounded(&bars->acc_full[ab], (tcount >> 1) & 1, abort_flag, __LINE__))) break;
       __syncwarp();
       tc_fence_after();
       float s_run = 0.f, e_run = 0.f;
@@ -361,7 +361,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   __syncthreads();
-  if (bars->abort && tid == 0) report(status, kStatusTimeout);
+  if (bars->abort && tid == 0) report(status, timeout_bits(kWhereGemmDecode, bars->abort));
   if (warp == 0) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);

@@ -221,7 +221,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         const int m = tile % num_m, nn = tile / num_m;
         for (int ks = 0; ks < num_k; ++ks, ++it) {
           const uint32_t s = it % SP, use = it / SP;
-          if (use > 0 && !(ok = mbar_wait_bounded(&bars->p_empty[s], (use - 1) & 1, abort_flag))) break;
+          if (use > 0 && !(ok = mbar_wait_bounded(&bars->p_empty[s], (use - 1) & 1, abort_flag, __LINE__))) break;
           uint8_t* dst = pk + s * kPackedStage + (is_a ? 0 : kPackedA);
           mbar_arrive_expect_tx(&bars->p_full[s], is_a ? kPackedA : kPackedB);
           tma_load_2d(dst, map, ks * BKP, is_a ? m * 2 * BM + (int)rank * BM : nn * BN + (int)rank * BNC,
@@ -246,7 +246,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         for (int ks = 0; ks < num_k; ++ks, ++it) {
           if ((it & 1u) != grp) continue;
           const uint32_t s = it % SE;
-          if (!(ok = mbar_wait_bounded(&bars->ready[s], (it / SE) & 1, abort_flag))) break;
+          if (!(ok = mbar_wait_bounded(&bars->ready[s], (it / SE) & 1, abort_flag, __LINE__))) break;
           tc_fence_after();
           st_async_signal(&bars->fwd_word[s], &bars->full[s], 0);
         }
@@ -259,11 +259,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       for (int tile = pair; tile < num_tiles && ok; tile += num_pairs, ++tcount) {
         const uint32_t ab = tcount & 1;
         // the epilogue must have drained this accumulator (used two tiles ago)
-        if (tcount >= 2 && !(ok = mbar_wait_bounded(&bars->acc_empty[ab], ((tcount >> 1) - 1) & 1, abort_flag))) break;
+        if (tcount >= 2 && !(ok = mbar_wait_bounded(&bars->acc_empty[ab], ((tcount >> 1) - 1) & 1, abort_flag, __LINE__))) break;
         tc_fence_after();
         for (int ks = 0; ks < num_k; ++ks, ++it) {
           const uint32_t s = it % SE;
-          if (!(ok = mbar_wait_bounded(&bars->full[s], (it / SE) & 1, abort_flag))) break;
+          if (!(ok = mbar_wait_bounded(&bars->full[s], (it / SE) & 1, abort_flag, __LINE__))) break;
           tc_fence_after();
           const uint32_t bbase = smem_u32(bst + s * kStageB);
           const uint32_t ta = tmem + kAccCols + 64u * s;
@@ -320,7 +320,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         wsc[32 * i + lane] = (o < d_out) ? sw[o] : 0.f;
       }
       __syncwarp();
-      if (!(ok = mbar_wait_bounded(&bars->acc_full[ab], (tcount >> 1) & 1, abort_flag))) break;
+      if (!(ok = mbar_wait_bounded(&bars->acc_full[ab], (tcount >> 1) & 1, abort_flag, __LINE__))) break;
       __syncwarp();
       tc_fence_after();
 #pragma unroll 1
@@ -342,7 +342,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           // SQNR sums (Sec. 2, Eq. 1) from the y_ref tile of this chunk; out-of-range entries are zero
           // on both sides.  Squares are summed in fp32 over the chunk's 32 values, then in float64.
           const uint32_t use = 2 * tcount + (c >> 1);  // the use-th load into buffer c % 2
-          if (!(ok = mbar_wait_bounded(&bars->ref_full[ew][c & 1], use & 1, abort_flag))) break;
+          if (!(ok = mbar_wait_bounded(&bars->ref_full[ew][c & 1], use & 1, abort_flag, __LINE__))) break;
           ++nused[c & 1];
           const uint8_t* rb = rstage0 + (c & 1) * kEpiStage + lane * 128;
           float s_run = 0.f, e_run = 0.f;
@@ -437,8 +437,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       for (int ks = 0; ks < num_k; ++ks, ++it) {
         if ((it & 1u) != (uint32_t)grp) continue;
         const uint32_t ps = it % SP, s = it % SE;
-        if (!(ok = mbar_wait_bounded(&bars->p_full[ps], (it / SP) & 1, abort_flag))) break;
-        if (it >= SE && !(ok = mbar_wait_bounded(&bars->empty[s], ((it / SE) - 1) & 1, abort_flag))) break;
+        if (!(ok = mbar_wait_bounded(&bars->p_full[ps], (it / SP) & 1, abort_flag, __LINE__))) break;
+        if (it >= SE && !(ok = mbar_wait_bounded(&bars->empty[s], ((it / SE) - 1) & 1, abort_flag, __LINE__))) break;
         tc_fence_after();
         const uint8_t* pa = pk + ps * kPackedStage;
         const uint8_t* pb = pa + kPackedA;
@@ -499,7 +499,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 
   tc_fence_before();
   cluster_sync();                                 // the pair's MMAs and both epilogues are done with TMEM
-  if (bars->abort && tid == 0) report(status, kStatusTimeout);
+  if (bars->abort && tid == 0) report(status, timeout_bits(kWhereGemm, bars->abort));
   if (warp == 0) {
     tc_fence_after();
     tmem_dealloc_pair(tmem, kTmemCols);
