@@ -201,7 +201,11 @@ cat_status cat_w4a4_linear_sqnr(const uint8_t* xq, const float* x_scale, const u
  * cat_sqnr -- signal-to-quantization-noise ratio of the layer output (Sec. 2, Eq. 1).
  *   y_ref, y_hat device [numel] float32 (full-precision and quantized outputs).
  *   out3         out, device [3] float64: { sum y_ref^2, sum (y_ref - y_hat)^2, 10 log10(ratio) dB }.
- * Squares are summed in fp32 over short runs and the run sums in float64.
+ * Squares are summed in fp32 over short runs and the run sums in float64; the per-CTA partial sums
+ * are added in a fixed order, so the three values are the same on every run of the same inputs.
+ * out3 is written, never read: it needs no zeroing.  The cross-CTA reduction uses one of eight
+ * slots of device scratch per kernel, handed out round robin, so at most eight SQNR-forming
+ * launches of one kernel may run concurrently.
  */
 cat_status cat_sqnr(const float* y_ref, const float* y_hat, int64_t numel, double* out3, cat_stream_t stream);
 

@@ -23,6 +23,7 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "sqnr_slot.cuh"
 
 namespace cat {
 namespace {
@@ -57,7 +58,7 @@ constexpr size_t kSmemBudget = 220 * 1024;
 
 struct DecBars {
   uint64_t p_full[kMaxSP], p_empty[kMaxSP], empty[kMaxSE], acc_full[2], acc_empty[2], tok_ready, mma_done;
-  double sums[4][2];                           // SQNR sums of the four epilogue warps
+  f32x2 sums[4][2];                            // SQNR sums of the four epilogue warps
   uint32_t tmem_addr;
   int abort;
 };
@@ -106,7 +107,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     w4a4_gemm_decode_tc_kernel(const __grid_constant__ CUtensorMap tmW, const uint8_t* __restrict__ xq,
                                const float* __restrict__ sx, const float* __restrict__ sw, int n, int d_in, int d_out,
                                int sp, float* __restrict__ y, int32_t* __restrict__ acc_out,
-                               const float* __restrict__ y_ref, double* __restrict__ sums3,
+                               const float* __restrict__ y_ref, double* __restrict__ sums3, int sqnr_slot,
                                uint32_t* __restrict__ status) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -283,7 +284,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int quad = warp & 3;
     uint32_t tcount = 0;
     bool ok = true;
-    double sig = 0.0, err = 0.0;                   // SQNR sums (Sec. 2, Eq. 1) when y_ref is given
+    f32x2 sig = {0.f, 0.f}, err = {0.f, 0.f};      // SQNR sums (Sec. 2, Eq. 1) when y_ref is given
     for (int u = blockIdx.x; u < num_units && ok; u += gridDim.x, ++tcount) {
       const uint32_t ab = tcount & 1;
       const int o = u * UM + quad * 32 + lane;
@@ -329,33 +330,22 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
-      sig += (double)s_run;
-      err += (double)e_run;
+      sig = f2_add(sig, s_run);
+      err = f2_add(err, e_run);
     }
     if (y_ref) {
-      // one pair of float64 atomics per CTA: the four warps' sums meet in shared memory first
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) {
-        sig += __shfl_xor_sync(0xFFFFFFFFu, sig, off);
-        err += __shfl_xor_sync(0xFFFFFFFFu, err, off);
-      }
+      // the four warps' sums meet in shared memory; one warp hands the CTA's pair to the slot
+      sig = f2_warp_sum(sig);
+      err = f2_warp_sum(err);
       if (lane == 0) {
         bars->sums[quad][0] = sig;
         bars->sums[quad][1] = err;
       }
       asm volatile("bar.sync 2, 128;" ::: "memory");  // this CTA's four epilogue warps have written theirs
-      if (warp == kEpiWarp0 && lane == 0) {
-        const double s_cta = (bars->sums[0][0] + bars->sums[1][0]) + (bars->sums[2][0] + bars->sums[3][0]);
-        const double e_cta = (bars->sums[0][1] + bars->sums[1][1]) + (bars->sums[2][1] + bars->sums[3][1]);
-        atomicAdd(&sums3[0], s_cta);
-        atomicAdd(&sums3[1], e_cta);
-        __threadfence();
-        unsigned long long* done = reinterpret_cast<unsigned long long*>(&sums3[2]);
-        if (atomicAdd(done, 1ull) == (unsigned long long)gridDim.x - 1) {  // the last CTA forms the ratio
-          __threadfence();
-          const double s_tot = atomicAdd(&sums3[0], 0.0), e_tot = atomicAdd(&sums3[1], 0.0);
-          sums3[2] = (e_tot > 0.0) ? 10.0 * log10(s_tot / e_tot) : (s_tot > 0.0 ? HUGE_VAL : 0.0);
-        }
+      if (warp == kEpiWarp0) {
+        const f32x2 s_cta = f2_add(f2_add(bars->sums[0][0], bars->sums[1][0]), f2_add(bars->sums[2][0], bars->sums[3][0]));
+        const f32x2 e_cta = f2_add(f2_add(bars->sums[0][1], bars->sums[1][1]), f2_add(bars->sums[2][1], bars->sums[3][1]));
+        sqnr_cta_done(sqnr_slot, s_cta, e_cta, sums3);
       }
     }
   }
@@ -429,13 +419,11 @@ cudaError_t launch_ntok(const uint8_t* xq, const float* sx, const uint8_t* wq, c
   const int64_t units = (d_out + UM - 1) / UM;
   const int64_t sms = num_sms();
   const unsigned grid = (unsigned)(units < sms ? units : sms);
+  if (grid > (unsigned)kSqnrMaxCtas) return cudaErrorInvalidConfiguration;
+  const int slot = y_ref ? next_sqnr_slot() : 0;
   note_launch();
-  if (y_ref) {
-    cudaError_t e = cudaMemsetAsync(sums3, 0, 3 * sizeof(double), stream);
-    if (e != cudaSuccess) return e;
-  }
   w4a4_gemm_decode_tc_kernel<NTOK><<<grid, kThreads, smem, stream>>>(map, xq, sx, sw, (int)n, (int)d_in, (int)d_out,
-                                                                      sp, y, acc_out, y_ref, sums3, status);
+                                                                      sp, y, acc_out, y_ref, sums3, slot, status);
   return cudaGetLastError();
 }
 
@@ -454,8 +442,8 @@ int decode_tc_stages(int64_t n, int64_t d_in) {
   return sp >= kDecGroups ? sp : 0;
 }
 
-// y_ref != nullptr: the epilogue also accumulates the SQNR sums of y against y_ref into sums3
-// (zeroed here; sums3[2] ends as the dB value).
+// y_ref != nullptr: the epilogue also forms the SQNR sums of y against y_ref and writes
+// sums3 = {sum y_ref^2, sum (y_ref - y)^2, dB} (sums3 needs no zeroing).
 cudaError_t launch_w4a4_gemm_decode_tc(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw,
                                        int64_t n, int64_t d_in, int64_t d_out, float* y, int32_t* acc_out,
                                        const float* y_ref, double* sums3, uint32_t* status, cudaStream_t stream) {

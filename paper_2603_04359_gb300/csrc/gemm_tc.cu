@@ -41,6 +41,7 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "sqnr_slot.cuh"
 
 namespace cat {
 namespace {
@@ -85,6 +86,7 @@ struct Bars {
   uint32_t fwd_word[SE];                         // even CTA: targets of the odd CTA's st.async per stage
   uint32_t tmem_addr;
   int abort;
+  f32x2 sums[kEpiWarps][2];                      // SQNR sums of the epilogue warps
 };
 static_assert(sizeof(Bars) <= kBarBytes, "barrier block must fit its reserved room");
 
@@ -161,7 +163,7 @@ __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wa
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     w4a4_gemm_tc_kernel(const __grid_constant__ CUtensorMap tmY, const __grid_constant__ CUtensorMap tmA,
                         const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmR,
-                        double* __restrict__ sums3, const float* __restrict__ sx,
+                        double* __restrict__ sums3, int sqnr_slot, const float* __restrict__ sx,
                         const float* __restrict__ sw, int n, int d_in, int d_out, float* __restrict__ y,
                         int32_t* __restrict__ acc_out, int use_tma_store, uint32_t* __restrict__ status) {
   extern __shared__ uint8_t smem_raw[];
@@ -287,7 +289,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     uint8_t* rstage0 = refb + ew * kEpiBufs * kEpiStage;
     float* wsc = scl + ew * BN;
     const bool with_ref = sums3 != nullptr;
-    double sig = 0.0, err = 0.0;                   // SQNR sums of this thread's outputs
+    f32x2 sig = {0.f, 0.f}, err = {0.f, 0.f};      // SQNR sums of this thread's outputs
     uint32_t tcount = 0, nstore = 0;
     bool ok = true;
     // y_ref tiles: chunk c of every tile goes through buffer c % 2; all four are loaded (out-of-range
@@ -353,8 +355,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             s_run += yr.x * yr.x + yr.y * yr.y + yr.z * yr.z + yr.w * yr.w;
             e_run += e0 * e0 + e1 * e1 + e2 * e2 + e3 * e3;
           }
-          sig += (double)s_run;
-          err += (double)e_run;
+          sig = f2_add(sig, s_run);
+          err = f2_add(err, e_run);
           // refill this buffer with the chunk two ahead (this or the next tile)
           int nt = tile, nc = c + 2;
           if (nc >= BN / 32) {
@@ -400,24 +402,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       volatile int no_abort = 0;
       for (int bb = 0; bb < kEpiBufs; ++bb)
         if (nref[bb] > nused[bb]) mbar_wait_bounded(&bars->ref_full[ew][bb], (nref[bb] - 1) & 1, &no_abort);
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        sig += __shfl_xor_sync(0xFFFFFFFFu, sig, o);
-        err += __shfl_xor_sync(0xFFFFFFFFu, err, o);
-      }
+      sig = f2_warp_sum(sig);
+      err = f2_warp_sum(err);
       if (lane == 0) {
-        atomicAdd(&sums3[0], sig);
-        atomicAdd(&sums3[1], err);
+        bars->sums[ew][0] = sig;
+        bars->sums[ew][1] = err;
       }
-      __threadfence();
-      asm volatile("bar.sync 2, 128;" ::: "memory");  // this CTA's four epilogue warps have added theirs
-      if (ew == 0 && lane == 0) {
-        unsigned long long* done = reinterpret_cast<unsigned long long*>(&sums3[2]);
-        if (atomicAdd(done, 1ull) == (unsigned long long)gridDim.x - 1) {  // the last CTA forms the ratio
-          __threadfence();
-          const double s_tot = atomicAdd(&sums3[0], 0.0), e_tot = atomicAdd(&sums3[1], 0.0);
-          sums3[2] = (e_tot > 0.0) ? 10.0 * log10(s_tot / e_tot) : (s_tot > 0.0 ? HUGE_VAL : 0.0);
-        }
+      asm volatile("bar.sync 2, 128;" ::: "memory");  // this CTA's four epilogue warps have written theirs
+      if (ew == 0) {
+        const f32x2 s_cta = f2_add(f2_add(bars->sums[0][0], bars->sums[1][0]), f2_add(bars->sums[2][0], bars->sums[3][0]));
+        const f32x2 e_cta = f2_add(f2_add(bars->sums[0][1], bars->sums[1][1]), f2_add(bars->sums[2][1], bars->sums[3][1]));
+        sqnr_cta_done(sqnr_slot, s_cta, e_cta, sums3);
       }
     }
     if (lane == 0) bulk_wait_all();
@@ -558,8 +553,9 @@ int num_sms() {
 
 }  // namespace
 
-// y_ref != nullptr: the epilogue also accumulates the SQNR sums of y against y_ref into sums3
-// (zeroed here; sums3[2] ends as the dB value).  Needs d_out % 4 == 0 (TMA row pitch).
+// y_ref != nullptr: the epilogue also forms the SQNR sums of y against y_ref and writes
+// sums3 = {sum y_ref^2, sum (y_ref - y)^2, dB} (sums3 needs no zeroing).  Needs d_out % 4 == 0
+// (TMA row pitch).
 cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
                                 int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, const float* y_ref,
                                 double* sums3, uint32_t* status, cudaStream_t stream) {
@@ -571,8 +567,6 @@ cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_
   if (y_ref) {
     if (d_out % 4 != 0 || !sums3 || !make_output_map(&tr, const_cast<float*>(y_ref), n, d_out))
       return cudaErrorInvalidValue;
-    cudaError_t e = cudaMemsetAsync(sums3, 0, 3 * sizeof(double), stream);
-    if (e != cudaSuccess) return e;
   }
   if (!make_packed_map(&ta, xq, n, d_in / 2, BM) || !make_packed_map(&tb, wq, d_out, d_in / 2, BNC))
     return cudaErrorInvalidValue;
@@ -585,8 +579,10 @@ cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_
   const int64_t tiles = ((n + 2 * BM - 1) / (2 * BM)) * ((d_out + BN - 1) / BN);
   const int64_t pairs_max = num_sms() / 2;
   const int grid = 2 * (int)(tiles < pairs_max ? tiles : pairs_max);  // CTA pairs (cluster of 2)
+  if (grid > kSqnrMaxCtas) return cudaErrorInvalidConfiguration;
+  const int slot = y_ref ? next_sqnr_slot() : 0;
   note_launch();
-  w4a4_gemm_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(ty, ta, tb, tr, y_ref ? sums3 : nullptr, sx, sw,
+  w4a4_gemm_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(ty, ta, tb, tr, y_ref ? sums3 : nullptr, slot, sx, sw,
                                                               (int)n, (int)d_in, (int)d_out, y, acc_out, use_tma,
                                                               status);
   return cudaGetLastError();

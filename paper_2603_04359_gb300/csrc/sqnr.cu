@@ -2,30 +2,25 @@
 //
 // HBM-bound: 8 bytes read per element.  Each thread issues the loads of 4 float4 pairs at once
 // (bytes in flight), sums squares in fp32 over runs of 16 elements (short runs keep the fp32
-// rounding at ~1e-7 of a run) and adds the run sums to float64 accumulators; warps reduce with
-// shuffles and each CTA adds its two partial sums to the float64 outputs atomically.  The last
-// CTA to finish (a counter kept in the third output word, which the launch zeroes with the sums)
-// forms the ratio, so the whole reduction is one launch.
+// rounding at ~1e-7 of a run) and adds the run sums to float-pair accumulators; warps reduce with
+// shuffles, and each CTA hands its two partial sums to a slot of device scratch whose last arrival
+// adds them in CTA order and forms the ratio (sqnr_slot.cuh), so the whole reduction is one launch
+// and its result is the same on every run.
 #include "common.cuh"
+#include "sqnr_slot.cuh"
 
 namespace cat {
 namespace {
 
 constexpr int kThreads = 256;
 
-__device__ __forceinline__ double warp_sum(double v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
-}
-
 __global__ void __launch_bounds__(kThreads) sqnr_partial_kernel(const float* __restrict__ yr,
                                                                  const float* __restrict__ yh, int64_t numel,
-                                                                 double* __restrict__ out3) {
+                                                                 double* __restrict__ out3, int slot) {
   const int64_t n4 = numel / 4;
   const float4* r4 = reinterpret_cast<const float4*>(yr);
   const float4* h4 = reinterpret_cast<const float4*>(yh);
-  double sig = 0.0, err = 0.0;
+  f32x2 sig = {0.f, 0.f}, err = {0.f, 0.f};
   // CTA tiles of 4 x kThreads consecutive float4 (16 KiB of each input), tiles strided by the grid
   const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
   for (int64_t base = (int64_t)blockIdx.x * 4 * kThreads; base < n4; base += (int64_t)gridDim.x * 4 * kThreads) {
@@ -43,45 +38,32 @@ __global__ void __launch_bounds__(kThreads) sqnr_partial_kernel(const float* __r
       s_run += a[u].x * a[u].x + a[u].y * a[u].y + a[u].z * a[u].z + a[u].w * a[u].w;
       e_run += ex * ex + ey * ey + ez * ez + ew * ew;
     }
-    sig += (double)s_run;
-    err += (double)e_run;
+    sig = f2_add(sig, s_run);
+    err = f2_add(err, e_run);
   }
   if (blockIdx.x == 0) {  // scalar tail
     for (int64_t j = n4 * 4 + threadIdx.x; j < numel; j += kThreads) {
       const float a = yr[j], e = a - yh[j];
-      sig += (double)(a * a);
-      err += (double)(e * e);
+      sig = f2_add(sig, a * a);
+      err = f2_add(err, e * e);
     }
   }
-  __shared__ double ssig[kThreads / 32], serr[kThreads / 32];
-  sig = warp_sum(sig);
-  err = warp_sum(err);
+  __shared__ f32x2 ssig[kThreads / 32], serr[kThreads / 32];
+  sig = f2_warp_sum(sig);
+  err = f2_warp_sum(err);
   if ((threadIdx.x & 31) == 0) {
     ssig[threadIdx.x >> 5] = sig;
     serr[threadIdx.x >> 5] = err;
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
-    double a = 0.0, b = 0.0;
+  if (threadIdx.x < 32) {
+    f32x2 a = {0.f, 0.f}, b = {0.f, 0.f};
     for (int w = 0; w < kThreads / 32; ++w) {
-      a += ssig[w];
-      b += serr[w];
+      a = f2_add(a, ssig[w]);
+      b = f2_add(b, serr[w]);
     }
-    atomicAdd(&out3[0], a);
-    atomicAdd(&out3[1], b);
-    __threadfence();
-    unsigned long long* done = reinterpret_cast<unsigned long long*>(&out3[2]);
-    if (atomicAdd(done, 1ull) == (unsigned long long)gridDim.x - 1) {  // every CTA's sums have landed
-      __threadfence();
-      const double s_tot = atomicAdd(&out3[0], 0.0), e_tot = atomicAdd(&out3[1], 0.0);
-      out3[2] = (e_tot > 0.0) ? 10.0 * log10(s_tot / e_tot) : (s_tot > 0.0 ? HUGE_VAL : 0.0);
-    }
+    sqnr_cta_done(slot, a, b, out3);
   }
-}
-
-__global__ void sqnr_finalize_kernel(double* out3) {
-  const double sig = out3[0], err = out3[1];
-  out3[2] = (err > 0.0) ? 10.0 * log10(sig / err) : (sig > 0.0 ? HUGE_VAL : 0.0);
 }
 
 int num_sms() {
@@ -94,18 +76,13 @@ int num_sms() {
 }  // namespace
 
 cudaError_t launch_sqnr(const float* y_ref, const float* y_hat, int64_t numel, double* out3, cudaStream_t stream) {
-  cudaError_t e = cudaMemsetAsync(out3, 0, 3 * sizeof(double), stream);  // sums and the CTA counter
-  if (e != cudaSuccess) return e;
-  if (numel == 0) {
-    note_launch();
-    sqnr_finalize_kernel<<<1, 1, 0, stream>>>(out3);
-    return cudaGetLastError();
-  }
+  // numel == 0: one CTA with nothing to read writes {0, 0, 0}
   const int64_t want = (numel / 4 + kThreads * 4 - 1) / (kThreads * 4);  // one 4-float4 tile per thread at least
-  const int64_t cap = (int64_t)num_sms() * 8;
+  int64_t cap = (int64_t)num_sms() * 8;
+  if (cap > kSqnrMaxCtas) cap = kSqnrMaxCtas;
   const unsigned grid = (unsigned)(want < 1 ? 1 : (want > cap ? cap : want));
   note_launch();
-  sqnr_partial_kernel<<<grid, kThreads, 0, stream>>>(y_ref, y_hat, numel, out3);
+  sqnr_partial_kernel<<<grid, kThreads, 0, stream>>>(y_ref, y_hat, numel, out3, next_sqnr_slot());
   return cudaGetLastError();
 }
 
