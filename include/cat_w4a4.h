@@ -191,7 +191,8 @@ cat_status cat_w4a4_linear(const uint8_t* xq, const float* x_scale, const uint8_
  * y is written exactly as cat_w4a4_linear writes it.  The sums are formed in the GEMM's epilogue while
  * y is produced (y is not read back) -- for n > 32 when d_out % 4 == 0, for n <= 32 when the decoded
  * tokens fit in the weight-streaming kernel's shared memory; otherwise the GEMM is followed by the
- * cat_sqnr reduction.  Squares are summed in fp32 over runs of at most 32 outputs, the runs in float64.
+ * cat_sqnr reduction.  Squares are summed in fp32 over runs of at most 32 outputs, the runs as float pairs
+ * (hi + lo, ~48 significant bits); the result does not depend on CTA timing.
  */
 cat_status cat_w4a4_linear_sqnr(const uint8_t* xq, const float* x_scale, const uint8_t* Wq, const float* w_scale,
                                 int64_t n, int64_t d_in, int64_t d_out, float* y, const float* y_ref, double* out3,
@@ -201,7 +202,8 @@ cat_status cat_w4a4_linear_sqnr(const uint8_t* xq, const float* x_scale, const u
  * cat_sqnr -- signal-to-quantization-noise ratio of the layer output (Sec. 2, Eq. 1).
  *   y_ref, y_hat device [numel] float32 (full-precision and quantized outputs).
  *   out3         out, device [3] float64: { sum y_ref^2, sum (y_ref - y_hat)^2, 10 log10(ratio) dB }.
- * Squares are summed in fp32 over short runs and the run sums in float64; the per-CTA partial sums
+ * Squares are summed in fp32 over short runs and the run sums as float pairs (hi + lo, ~48 significant
+ * bits); the dB value is formed in fp32 from the high parts (|error| ~1e-5 dB).  The per-CTA partial sums
  * are added in a fixed order, so the three values are the same on every run of the same inputs.
  * out3 is written, never read: it needs no zeroing.  The cross-CTA reduction uses one of eight
  * slots of device scratch per kernel, handed out round robin, so at most eight SQNR-forming

@@ -39,6 +39,7 @@
 // is bounded; a wait that gives up raises the device status word and all roles drain and exit.
 #include <cstring>
 #include <mutex>
+#include <type_traits>
 
 #include "common.cuh"
 #include "sqnr_slot.cuh"
@@ -160,12 +161,50 @@ __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.comm
 __device__ __forceinline__ void bulk_wait_read_le1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
+// ---- the last wave's tiles split along K -----------------------------------------------------
+// With T pair tiles on P pairs the last wave holds T mod P tiles and the other pairs idle through
+// it.  When it is at most half full, each of its tiles is split into S parts of its K steps (S a
+// power of two, at most 16), one part per pair.  Every part writes its raw accumulators to its own
+// slice of device scratch with plain stores (float32 atomics from many SMs onto one tile are an
+// order of magnitude slower), waits until all S parts of the tile have arrived (bounded; the launch
+// is cooperative, so all parts are resident), and then finishes 128 / S of the tile's channels:
+// the sum over the parts (exact in any order: integer multiples of 2^-18 below 2^6 in magnitude),
+// the scaling, y, acc_out and the SQNR sums.  Counters are per (tile, CTA, epilogue warp); the last
+// part to finish sets them back to zero.  Slots of this scratch are handed out round robin per launch.
+constexpr int kSplitSlots = 2;
+constexpr int kMaxSplitTiles = 38;            // half a wave of 76 pairs
+constexpr int kMaxSplitUnits = 80;            // tail tiles x parts <= pairs
+constexpr int kMaxSplit = 16;
+__device__ float4 g_split_part[kSplitSlots][kMaxSplitUnits][BN / 4][2 * BM];   // [part][channel/4][row]
+__device__ uint32_t g_split_cnt[kSplitSlots][kMaxSplitTiles][2][kEpiWarps][2];   // arrived, finished
+
+__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Work unit u of the launch: the n_split = tail x split parts come first (part u % split of tail
+// tile num_full + u / split, on pairs 0 .. n_split - 1, one each), then the whole tiles (tile
+// u - n_split).  Each part's sibling parts run at the same time, and the part's share of the tile is
+// finished after the pair's first whole tile, when they have long arrived.
+struct Unit {
+  int tile, k0, k1, part;                     // part < 0: the whole tile
+};
+__device__ __forceinline__ Unit unit_at(int u, int num_full, int split, int num_k, int n_split) {
+  if (u >= n_split) return {u - n_split, 0, num_k, -1};
+  const int part = u % split;
+  return {num_full + u / split, part * num_k / split, (part + 1) * num_k / split, part};
+}
+
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     w4a4_gemm_tc_kernel(const __grid_constant__ CUtensorMap tmY, const __grid_constant__ CUtensorMap tmA,
                         const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmR,
-                        double* __restrict__ sums3, int sqnr_slot, const float* __restrict__ sx,
+                        const float* __restrict__ y_ref, double* __restrict__ sums3, int sqnr_slot,
+                        const float* __restrict__ sx,
                         const float* __restrict__ sw, int n, int d_in, int d_out, float* __restrict__ y,
-                        int32_t* __restrict__ acc_out, int use_tma_store, uint32_t* __restrict__ status) {
+                        int32_t* __restrict__ acc_out, int use_tma_store, int num_full, int split, int split_slot,
+                        uint32_t* __restrict__ status) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* bst = smem;                         // SE x 2 atoms x [128 rows x 128 B] E4M3, 128B-swizzled
@@ -183,6 +222,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const int num_n = (d_out + BN - 1) / BN;
   const int num_k = (d_in + BK - 1) / BK;
   const int num_tiles = num_m * num_n;
+  const int n_split = (num_tiles - num_full) * split;   // 0 without a split
+  const int total_units = num_full + n_split;
 
   if (tid == 0) {
     for (int s = 0; s < SP; ++s) {
@@ -219,9 +260,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       prefetch_tensormap(map);
       uint32_t it = 0;
       bool ok = true;
-      for (int tile = pair; tile < num_tiles && ok; tile += num_pairs) {
-        const int m = tile % num_m, nn = tile / num_m;
-        for (int ks = 0; ks < num_k; ++ks, ++it) {
+      for (int u = pair; u < total_units && ok; u += num_pairs) {
+        const Unit w = unit_at(u, num_full, split, num_k, n_split);
+        const int m = w.tile % num_m, nn = w.tile / num_m;
+        for (int ks = w.k0; ks < w.k1; ++ks, ++it) {
           const uint32_t s = it % SP, use = it / SP;
           if (use > 0 && !(ok = mbar_wait_bounded(&bars->p_empty[s], (use - 1) & 1, abort_flag, __LINE__))) break;
           uint8_t* dst = pk + s * kPackedStage + (is_a ? 0 : kPackedA);
@@ -244,26 +286,29 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const uint32_t grp = warp == kMmaWarp ? 0u : 1u;
       uint32_t it = 0;
       bool ok = true;
-      for (int tile = pair; tile < num_tiles && ok; tile += num_pairs)
-        for (int ks = 0; ks < num_k; ++ks, ++it) {
+      for (int u = pair; u < total_units && ok; u += num_pairs) {
+        const Unit w = unit_at(u, num_full, split, num_k, n_split);
+        for (int ks = w.k0; ks < w.k1; ++ks, ++it) {
           if ((it & 1u) != grp) continue;
           const uint32_t s = it % SE;
           if (!(ok = mbar_wait_bounded(&bars->ready[s], (it / SE) & 1, abort_flag, __LINE__))) break;
           tc_fence_after();
           st_async_signal(&bars->fwd_word[s], &bars->full[s], 0);
         }
+      }
     }
   } else if (warp == kMmaWarp) {
     // ---------------------------------------------------------------- MMA issuer (even CTA)
     if (lane == 0 && rank == 0) {
       uint32_t it = 0, tcount = 0;
       bool ok = true;
-      for (int tile = pair; tile < num_tiles && ok; tile += num_pairs, ++tcount) {
+      for (int u = pair; u < total_units && ok; u += num_pairs, ++tcount) {
+        const Unit w = unit_at(u, num_full, split, num_k, n_split);
         const uint32_t ab = tcount & 1;
-        // the epilogue must have drained this accumulator (used two tiles ago)
+        // the epilogue must have drained this accumulator (used two units ago)
         if (tcount >= 2 && !(ok = mbar_wait_bounded(&bars->acc_empty[ab], ((tcount >> 1) - 1) & 1, abort_flag, __LINE__))) break;
         tc_fence_after();
-        for (int ks = 0; ks < num_k; ++ks, ++it) {
+        for (int ks = w.k0; ks < w.k1; ++ks, ++it) {
           const uint32_t s = it % SE;
           if (!(ok = mbar_wait_bounded(&bars->full[s], (it / SE) & 1, abort_flag, __LINE__))) break;
           tc_fence_after();
@@ -272,7 +317,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int kk = 0; kk < BK / 32; ++kk) {  // K = 32 codes per MMA: 8 TMEM columns of A; B atom kk/4, +32 B
             const uint64_t db = sdesc_kmajor_sw128(bbase + (uint32_t)(kk >> 2) * kAtomB) + 2 * (kk & 3);
-            mma_pair_ts(tmem + ab * BN, ta + 8u * kk, db, kIdesc, (ks | kk) != 0);
+            mma_pair_ts(tmem + ab * BN, ta + 8u * kk, db, kIdesc, (ks != w.k0 || kk != 0) ? 1u : 0u);
           }
           mma_commit_pair(&bars->empty[s]);
         }
@@ -292,8 +337,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     f32x2 sig = {0.f, 0.f}, err = {0.f, 0.f};      // SQNR sums of this thread's outputs
     uint32_t tcount = 0, nstore = 0;
     bool ok = true;
-    // y_ref tiles: chunk c of every tile goes through buffer c % 2; all four are loaded (out-of-range
-    // parts read as zero), so the buffer phases advance regularly
+    // y_ref tiles of whole-tile units: chunk c of every such tile goes through buffer c % 2; all four
+    // are loaded (out-of-range parts read as zero), so the buffer phases advance regularly.  The
+    // epilogue of a split tail tile reads y_ref with plain loads.
     uint32_t nref[kEpiBufs] = {0u, 0u}, nused[kEpiBufs] = {0u, 0u};  // loads issued / consumed per buffer
     auto load_ref = [&](int tile_, int c_) {        // called by the whole warp; lane 0 issues
       const int m_ = tile_ % num_m, nn_ = tile_ / num_m;
@@ -305,19 +351,168 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       }
       ++nref[c_ & 1];
     };
-    if (with_ref && pair < num_tiles) {
-      load_ref(pair, 0);
-      load_ref(pair, 1);
+    // y (and acc_out) of one chunk: 32 rows from row0_ (this lane: t_) x 32 channels from o0; v the
+    // outputs, a the raw accumulators
+    auto store_chunk = [&](int o0, int row0_, int t_, const float (&v)[32], const float (&a)[32]) {
+      if (o0 >= d_out || row0_ >= n) return;      // warp-uniform: nothing of this chunk is in range
+      if (use_tma_store) {
+        uint8_t* buf = stage0 + (nstore % kEpiBufs) * kEpiStage;
+        if (lane == 0) bulk_wait_read_le1();  // the store issued two chunks ago has read this buffer
+        __syncwarp();
+#pragma unroll
+        for (int q = 0; q < 8; ++q)  // row `lane`, 16-byte chunk q at q ^ (lane % 8)
+          *reinterpret_cast<float4*>(buf + lane * 128 + ((q ^ (lane & 7)) << 4)) =
+              make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_2d(&tmY, buf, o0, row0_);
+          bulk_commit();
+        }
+        ++nstore;
+      } else if (t_ < n) {
+        float* yrow = y + (size_t)t_ * d_out;
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          if (o0 + i < d_out) yrow[o0 + i] = v[i];
+      }
+      if (acc_out && t_ < n) {
+        int32_t* arow = acc_out + (size_t)t_ * d_out;
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          if (o0 + i < d_out) arow[o0 + i] = __float2int_rn(a[i] * kAccScale);
+      }
+    };
+    // tail tiles: this lane's row of part j's partial accumulators, the counters of this warp's
+    // 32-row slice of tail tile tj, and the bounded wait for all parts of the tile
+    const int my_row = (int)rank * BM + quad * 32 + lane;
+    auto cnt_of = [&](int tj, int which) { return &g_split_cnt[split_slot][tj][rank][ew][which]; };
+    auto arrive_part = [&](int tj) {                // after this lane's partial stores
+      __threadfence();
+      __syncwarp();
+      if (lane == 0) atomicAdd(cnt_of(tj, 0), 1u);
+    };
+    auto wait_parts = [&](int tj) -> bool {         // warp-uniform: true once all parts have arrived
+      uint32_t good = 1u;
+      if (lane == 0) {
+        const uint64_t t0 = globaltimer_ns();
+        for (uint32_t it = 0; ld_acquire_gpu(cnt_of(tj, 0)) < (uint32_t)split; ++it) {
+          __nanosleep(64);
+          if ((it & 63u) == 63u && (*abort_flag || globaltimer_ns() - t0 > kWaitLimitNs)) {
+            if (*abort_flag == 0) *abort_flag = __LINE__;
+            good = 0u;
+            break;
+          }
+        }
+      }
+      good = __shfl_sync(0xFFFFFFFFu, good, 0);
+      __threadfence();                              // the other parts' stores are seen from here on
+      return good != 0u;
+    };
+    auto finish_part = [&](int tj) {                // the last part to finish clears the counters
+      __syncwarp();
+      if (lane == 0 && atomicAdd(cnt_of(tj, 1), 1u) == (uint32_t)(split - 1)) {
+        *cnt_of(tj, 0) = 0u;
+        *cnt_of(tj, 1) = 0u;
+      }
+    };
+    // the share of split unit uu's tile that its part finishes: channels [128 / S * part, ...) of the
+    // tile, once all S parts' partials are out
+    auto finish_share = [&](int uu) {
+      const Unit w = unit_at(uu, num_full, split, num_k, n_split);
+      const int tj = w.tile - num_full;
+      const int m = w.tile % num_m, nn = w.tile / num_m;
+      const int t = m * 2 * BM + (int)rank * BM + quad * 32 + lane;
+      const float sxt = (t < n) ? sx[t] * kAccScale : 0.f;
+      if (wait_parts(tj)) {
+        float s_run = 0.f, e_run = 0.f;
+        auto fixup = [&](auto split_c) {
+          constexpr int S = decltype(split_c)::value;
+          constexpr int L = S >= 4 ? 16 : 8;      // loads of parts per batch
+          constexpr int G = 32 / S, PB = L / S;   // groups of the share, groups per batch
+          const int g0 = w.part * G;
+#pragma unroll 1
+          for (int b = 0; b < G; b += PB) {
+            float4 pq[L], yr[PB];
+#pragma unroll
+            for (int i = 0; i < L; ++i)
+              pq[i] = __ldcg(&g_split_part[split_slot][tj * S + i % S][g0 + b + i / S][my_row]);
+#pragma unroll
+            for (int k = 0; k < PB; ++k) {
+              const int o = nn * BN + 4 * (g0 + b + k);
+              yr[k] = (with_ref && t < n && o < d_out)
+                          ? __ldcs(reinterpret_cast<const float4*>(y_ref + (size_t)t * d_out + o))
+                          : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+#pragma unroll
+            for (int k = 0; k < PB; ++k) {
+              float4 acc4 = pq[k * S];
+#pragma unroll
+              for (int q = 1; q < S; ++q) {   // exact in any order
+                acc4.x += pq[k * S + q].x;
+                acc4.y += pq[k * S + q].y;
+                acc4.z += pq[k * S + q].z;
+                acc4.w += pq[k * S + q].w;
+              }
+              const int gl = g0 + b + k, o = nn * BN + 4 * gl;
+              const float a[4] = {acc4.x, acc4.y, acc4.z, acc4.w};
+              float v[4];
+#pragma unroll
+              for (int i = 0; i < 4; ++i) v[i] = a[i] * sxt * ((o + i < d_out) ? __ldg(sw + o + i) : 0.f);
+              if (t < n && o < d_out) {
+                float* yp = y + (size_t)t * d_out + o;
+                if ((d_out & 3) == 0) {               // a float4 is wholly in or out of range
+                  *reinterpret_cast<float4*>(yp) = make_float4(v[0], v[1], v[2], v[3]);
+                  const float e0 = yr[k].x - v[0], e1 = yr[k].y - v[1], e2 = yr[k].z - v[2], e3 = yr[k].w - v[3];
+                  s_run += yr[k].x * yr[k].x + yr[k].y * yr[k].y + yr[k].z * yr[k].z + yr[k].w * yr[k].w;
+                  e_run += e0 * e0 + e1 * e1 + e2 * e2 + e3 * e3;
+                } else {
+#pragma unroll
+                  for (int i = 0; i < 4; ++i)
+                    if (o + i < d_out) yp[i] = v[i];
+                }
+                if (acc_out) {
+#pragma unroll
+                  for (int i = 0; i < 4; ++i)
+                    if (o + i < d_out) acc_out[(size_t)t * d_out + o + i] = __float2int_rn(a[i] * kAccScale);
+                }
+              }
+            }
+          }
+        };
+        switch (split) {
+          case 2: fixup(std::integral_constant<int, 2>{}); break;
+          case 4: fixup(std::integral_constant<int, 4>{}); break;
+          case 8: fixup(std::integral_constant<int, 8>{}); break;
+          default: fixup(std::integral_constant<int, 16>{}); break;
+        }
+        if (with_ref) {
+          sig = f2_add(sig, s_run);
+          err = f2_add(err, e_run);
+        }
+      }
+      finish_part(tj);
+    };
+    // this pair's first whole tile comes after its split part, if it has one; y_ref loads and uses
+    // count whole tiles only (fcount)
+    const int u_full0 = pair < n_split ? pair + num_pairs : pair;
+    if (with_ref && u_full0 < total_units) {
+      load_ref(u_full0 - n_split, 0);
+      load_ref(u_full0 - n_split, 1);
     }
-    for (int tile = pair; tile < num_tiles && ok; tile += num_pairs, ++tcount) {
+    uint32_t fcount = 0;
+    int split_state = 0;                            // this pair's split part: 1 partials out, 2 share done
+    int u = pair;
+    for (; u < total_units; u += num_pairs, ++tcount) {
+      const Unit w = unit_at(u, num_full, split, num_k, n_split);
       const uint32_t ab = tcount & 1;
-      const int m = tile % num_m, nn = tile / num_m;
+      const int m = w.tile % num_m, nn = w.tile / num_m;
       const int row0 = m * 2 * BM + (int)rank * BM + quad * 32;
       const int t = row0 + lane;
       const float sxt = (t < n) ? sx[t] * kAccScale : 0.f;
       __syncwarp();
 #pragma unroll
-      for (int i = 0; i < BN / 32; ++i) {  // this tile's output-channel steps, staged once per tile
+      for (int i = 0; i < BN / 32; ++i) {  // this tile's output-channel steps, staged once per unit
         const int o = nn * BN + 32 * i + lane;
         wsc[32 * i + lane] = (o < d_out) ? sw[o] : 0.f;
       }
@@ -325,77 +520,94 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       if (!(ok = mbar_wait_bounded(&bars->acc_full[ab], (tcount >> 1) & 1, abort_flag, __LINE__))) break;
       __syncwarp();
       tc_fence_after();
+      if (w.part < 0) {
 #pragma unroll 1
-      for (int c = 0; c < BN / 32; ++c) {
-        uint32_t r[32];
-        __syncwarp();
-        CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + ab * BN + c * 32, r);
-        tmem_ld_wait();
-        if (c == BN / 32 - 1) {  // accumulator fully read: the MMAs of tile + 2 may use it
-          tc_fence_before();
+        for (int c = 0; c < BN / 32; ++c) {
+          uint32_t r[32];
           __syncwarp();
-          if (lane == 0) mbar_arrive_cluster(&bars->acc_empty[ab], 0);
-        }
-        const int o0 = nn * BN + c * 32;
-        float v[32];
-#pragma unroll
-        for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]) * sxt * wsc[c * 32 + i];
-        if (with_ref) {
-          // SQNR sums (Sec. 2, Eq. 1) from the y_ref tile of this chunk; out-of-range entries are zero
-          // on both sides.  Squares are summed in fp32 over the chunk's 32 values, then in float64.
-          const uint32_t use = 2 * tcount + (c >> 1);  // the use-th load into buffer c % 2
-          if (!(ok = mbar_wait_bounded(&bars->ref_full[ew][c & 1], use & 1, abort_flag, __LINE__))) break;
-          ++nused[c & 1];
-          const uint8_t* rb = rstage0 + (c & 1) * kEpiStage + lane * 128;
-          float s_run = 0.f, e_run = 0.f;
-#pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            const float4 yr = *reinterpret_cast<const float4*>(rb + ((q ^ (lane & 7)) << 4));
-            const float e0 = yr.x - v[4 * q], e1 = yr.y - v[4 * q + 1], e2 = yr.z - v[4 * q + 2], e3 = yr.w - v[4 * q + 3];
-            s_run += yr.x * yr.x + yr.y * yr.y + yr.z * yr.z + yr.w * yr.w;
-            e_run += e0 * e0 + e1 * e1 + e2 * e2 + e3 * e3;
+          CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + ab * BN + c * 32, r);
+          tmem_ld_wait();
+          if (c == BN / 32 - 1) {  // accumulator fully read: the MMAs of unit + 2 may use it
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_cluster(&bars->acc_empty[ab], 0);
           }
-          sig = f2_add(sig, s_run);
-          err = f2_add(err, e_run);
-          // refill this buffer with the chunk two ahead (this or the next tile)
-          int nt = tile, nc = c + 2;
-          if (nc >= BN / 32) {
-            nc -= BN / 32;
-            nt = tile + num_pairs;
+          const int o0 = nn * BN + c * 32;
+          float a[32], v[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            a[i] = __uint_as_float(r[i]);
+            v[i] = a[i] * sxt * wsc[c * 32 + i];
           }
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (nt < num_tiles) load_ref(nt, nc);
-        }
-        if (o0 >= d_out || row0 >= n) continue;  // warp-uniform: nothing of this chunk is in range
-        if (use_tma_store) {
-          uint8_t* buf = stage0 + (nstore % kEpiBufs) * kEpiStage;
-          if (lane == 0) bulk_wait_read_le1();  // the store issued two chunks ago has read this buffer
-          __syncwarp();
+          if (with_ref) {
+            // SQNR sums (Sec. 2, Eq. 1) from the y_ref tile of this chunk; out-of-range entries are zero
+            // on both sides.  Squares are summed in fp32 over the chunk's 32 values, then as float pairs.
+            const uint32_t use = 2 * fcount + (c >> 1);  // the use-th load into buffer c % 2
+            if (!(ok = mbar_wait_bounded(&bars->ref_full[ew][c & 1], use & 1, abort_flag, __LINE__))) break;
+            ++nused[c & 1];
+            const uint8_t* rb = rstage0 + (c & 1) * kEpiStage + lane * 128;
+            float s_run = 0.f, e_run = 0.f;
 #pragma unroll
-          for (int q = 0; q < 8; ++q)  // row `lane`, 16-byte chunk q at q ^ (lane % 8)
-            *reinterpret_cast<float4*>(buf + lane * 128 + ((q ^ (lane & 7)) << 4)) =
-                make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) {
-            tma_store_2d(&tmY, buf, o0, row0);
-            bulk_commit();
+            for (int q = 0; q < 8; ++q) {
+              const float4 yr = *reinterpret_cast<const float4*>(rb + ((q ^ (lane & 7)) << 4));
+              const float e0 = yr.x - v[4 * q], e1 = yr.y - v[4 * q + 1], e2 = yr.z - v[4 * q + 2], e3 = yr.w - v[4 * q + 3];
+              s_run += yr.x * yr.x + yr.y * yr.y + yr.z * yr.z + yr.w * yr.w;
+              e_run += e0 * e0 + e1 * e1 + e2 * e2 + e3 * e3;
+            }
+            sig = f2_add(sig, s_run);
+            err = f2_add(err, e_run);
+            // refill this buffer with the chunk two ahead (this tile or the next: whole tiles follow)
+            int nu = u, nc = c + 2;
+            if (nc >= BN / 32) {
+              nc -= BN / 32;
+              nu = u + num_pairs;
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (nu < total_units) load_ref(nu - n_split, nc);
           }
-          ++nstore;
-        } else if (t < n) {
-          float* yrow = y + (size_t)t * d_out;
-#pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (o0 + i < d_out) yrow[o0 + i] = v[i];
+          store_chunk(o0, row0, t, v, a);
         }
-        if (acc_out && t < n) {
-          int32_t* arow = acc_out + (size_t)t * d_out;
-#pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (o0 + i < d_out) arow[o0 + i] = __float2int_rn(__uint_as_float(r[i]) * kAccScale);
+        ++fcount;
+        if (!ok) break;
+        if (split_state == 1) {                     // the split part's siblings have long arrived
+          finish_share(pair);
+          split_state = 2;
         }
+      } else {
+        // a K part of a tail tile: this warp's 32 rows of raw accumulators to the part's slice
+        const int tj = w.tile - num_full, j = u;
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          uint32_t r[32];
+          __syncwarp();
+          CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + ab * BN + c * 32, r);
+          tmem_ld_wait();
+          if (c == BN / 32 - 1) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_cluster(&bars->acc_empty[ab], 0);
+          }
+#pragma unroll
+          for (int q = 0; q < 8; ++q)   // a warp stores 32 consecutive rows of one channel group: 512 B
+            __stcg(&g_split_part[split_slot][j][8 * c + q][my_row],
+                   make_float4(__uint_as_float(r[4 * q]), __uint_as_float(r[4 * q + 1]), __uint_as_float(r[4 * q + 2]),
+                               __uint_as_float(r[4 * q + 3])));
+        }
+        arrive_part(tj);
+        split_state = 1;
       }
+    }
+    if (ok && split_state == 1) {                   // no whole tile followed the split part
+      finish_share(pair);
+      split_state = 2;
+    }
+    if (!ok && pair < n_split) {
+      // a wait gave up: settle this warp's split part all the same (without data: the launch's
+      // outputs are void), so that every counter of the launch ends at zero
+      const int tj = unit_at(pair, num_full, split, num_k, n_split).tile - num_full;
+      if (split_state == 0) arrive_part(tj);
+      if (split_state <= 1) finish_part(tj);
     }
     if (with_ref) {
       // y_ref loads issued but not consumed (only after a wait gave up) land before the CTA exits
@@ -428,8 +640,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     const int a_row = quad * 32 + lane;           // this thread's A row = TMEM lane
     uint32_t it = 0;
     bool ok = true;
-    for (int tile = pair; tile < num_tiles && ok; tile += num_pairs) {
-      for (int ks = 0; ks < num_k; ++ks, ++it) {
+    for (int u = pair; u < total_units && ok; u += num_pairs) {
+      const Unit w = unit_at(u, num_full, split, num_k, n_split);
+      for (int ks = w.k0; ks < w.k1; ++ks, ++it) {
         if ((it & 1u) != (uint32_t)grp) continue;
         const uint32_t ps = it % SP, s = it % SE;
         if (!(ok = mbar_wait_bounded(&bars->p_full[ps], (it / SP) & 1, abort_flag, __LINE__))) break;
@@ -551,6 +764,32 @@ int num_sms() {
   return sms;
 }
 
+// Whether a cooperative launch of `pairs` CTA pairs of the GEMM kernel fits on this device (checked
+// once per process, on the first device asked).
+bool split_launch_ok(int64_t pairs) {
+  static int ok = -1;
+  static std::mutex mu;
+  std::lock_guard<std::mutex> lock(mu);
+  if (ok < 0) {
+    int dev = 0, coop = 0, clusters = 0;
+    ok = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess &&
+        cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) == cudaSuccess && coop &&
+        cudaFuncSetAttribute(w4a4_gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes) ==
+            cudaSuccess) {
+      cudaLaunchConfig_t cfg;
+      memset(&cfg, 0, sizeof(cfg));
+      cfg.gridDim = dim3((unsigned)(2 * pairs), 1, 1);
+      cfg.blockDim = dim3(kThreads, 1, 1);
+      cfg.dynamicSmemBytes = kSmemBytes;
+      if (cudaOccupancyMaxActiveClusters(&clusters, w4a4_gemm_tc_kernel, &cfg) == cudaSuccess && clusters >= pairs)
+        ok = 1;
+    }
+    cudaGetLastError();
+  }
+  return ok == 1;
+}
+
 }  // namespace
 
 // y_ref != nullptr: the epilogue also forms the SQNR sums of y against y_ref and writes
@@ -577,14 +816,47 @@ cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_
   });
   if (attr_err != cudaSuccess) return attr_err;
   const int64_t tiles = ((n + 2 * BM - 1) / (2 * BM)) * ((d_out + BN - 1) / BN);
+  const int64_t num_k = (d_in + BK - 1) / BK;
   const int64_t pairs_max = num_sms() / 2;
-  const int grid = 2 * (int)(tiles < pairs_max ? tiles : pairs_max);  // CTA pairs (cluster of 2)
+  // the last wave's tiles, split along K into a power-of-two number of parts when that wave is at
+  // most half full (the parts wait for one another: only with a cooperative launch)
+  const int64_t tail = tiles >= pairs_max ? tiles % pairs_max : tiles;
+  int split = 1;
+  if (tail > 0 && tail <= kMaxSplitTiles && 2 * tail <= pairs_max && split_launch_ok(pairs_max))
+    while (2 * split <= kMaxSplit && 2 * split * tail <= pairs_max && 2 * split <= num_k) split *= 2;
+  // a single partial wave has no whole tiles to hide the parts' exchange behind: split it only
+  // when that saves ten K steps or more
+  if (split > 1 && tiles < pairs_max && num_k - num_k / split < 10) split = 1;
+  const int64_t num_full = split > 1 ? tiles - tail : tiles;
+  const int64_t units = num_full + (tiles - num_full) * split;
+  if (split > 1 && (units - num_full > kMaxSplitUnits || num_full % pairs_max != 0)) return cudaErrorInvalidConfiguration;
+  const int grid = 2 * (int)(units < pairs_max ? units : pairs_max);  // CTA pairs (cluster of 2)
   if (grid > kSqnrMaxCtas) return cudaErrorInvalidConfiguration;
+  static std::atomic<unsigned> next_split{0};
+  const int split_slot = split > 1 ? (int)(next_split.fetch_add(1, std::memory_order_relaxed) % kSplitSlots) : 0;
   const int slot = y_ref ? next_sqnr_slot() : 0;
+  const double* sums = y_ref ? sums3 : nullptr;
   note_launch();
-  w4a4_gemm_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(ty, ta, tb, tr, y_ref ? sums3 : nullptr, slot, sx, sw,
-                                                              (int)n, (int)d_in, (int)d_out, y, acc_out, use_tma,
-                                                              status);
+  if (split == 1) {
+    w4a4_gemm_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(ty, ta, tb, tr, y_ref, const_cast<double*>(sums), slot,
+                                                                sx, sw, (int)n, (int)d_in, (int)d_out, y, acc_out,
+                                                                use_tma, (int)num_full, split, split_slot, status);
+    return cudaGetLastError();
+  }
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = dim3((unsigned)grid, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = stream;
+  cudaLaunchAttribute attrs[1];
+  attrs[0].id = cudaLaunchAttributeCooperative;
+  attrs[0].val.cooperative = 1;
+  cfg.attrs = attrs;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, w4a4_gemm_tc_kernel, ty, ta, tb, tr, y_ref, const_cast<double*>(sums), slot, sx, sw,
+                            (int)n, (int)d_in, (int)d_out, y, acc_out, use_tma, (int)num_full, split, split_slot,
+                            status);
   return cudaGetLastError();
 }
 

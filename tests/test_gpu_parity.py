@@ -135,6 +135,7 @@ GEMM_SHAPES = [
     (3, 12288, 100),                                  # n <= 32, tokens too large for shared memory: mma.sync
     (33, 128, 256), (128, 256, 256), (129, 160, 300), (300, 384, 520), (257, 4096, 64),  # tcgen05 path
     (512, 1024, 1024), (1024, 512, 6144),                                                # ... several tiles per pair
+    (256, 1024, 9984), (300, 2048, 5030),  # a last wave of 2 / 4 tiles on 76 pairs, split along K into 4 / 8 parts
 ]
 
 
@@ -179,7 +180,8 @@ def test_w4a4_linear_extreme_accumulators(n, d_in):
 
 @pytest.mark.parametrize("n,d_in,d_out", [(300, 1024, 520), (513, 512, 256), (257, 4096, 130), (16, 1024, 200),
                                           (129, 160, 300), (24, 2048, 40000), (16, 9216, 300), (3, 12288, 100),
-                                          (1024, 512, 6144)])   # several pair tiles per CTA pair
+                                          (1024, 512, 6144),    # several pair tiles per CTA pair
+                                          (300, 2048, 5032)])   # a split last wave
 def test_w4a4_linear_sqnr_fused(n, d_in, d_out):
     """y equals cat_w4a4_linear's bit for bit; the sums match the oracle's over the same outputs
     (fused in the GEMM epilogue for n > 32 with d_out % 4 == 0 and in the tcgen05 decode kernel,
