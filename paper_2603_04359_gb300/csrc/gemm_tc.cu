@@ -35,8 +35,9 @@
 //                128B-swizzled shared memory, TMA store (plain stores when the TMA rules don't hold)
 //   warps 8..15  decode, two groups of four warps taking alternate K steps: a whole A row per
 //                thread, and B chunks
-// TMEM: accumulators at columns [0, 128) and [128, 256), A stages at 256 + 64 s.  Every mbarrier wait
-// is bounded; a wait that gives up raises the device status word and all roles drain and exit.
+// TMEM: accumulators at columns [0, 128) and [128, 256), A stages at 256 + 64 s.  A last wave that is at
+// most half full is split along K (see the split-tail section below).  Every wait is bounded; a wait
+// that gives up raises the device status word and all roles drain and exit.
 #include <cstring>
 #include <mutex>
 #include <type_traits>
