@@ -45,6 +45,7 @@ DEFAULT_CONFIG = "c2_qkv_4096x6144_k128_bf16"
 FP8_PER_BF16 = 2.0          # nominal dense FP8 / BF16 tensor throughput ratio (4.5 / 2.25 PFLOP/s)
 FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}
 DECODE_TOKENS = 32          # cat_w4a4_linear streams the weights (HBM-bound) up to this many tokens
+SWEEP_K = (32, 64, 128, 256)
 
 
 def parse_args():
@@ -59,6 +60,9 @@ def parse_args():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="budget of the CPU-baseline sample")
+    p.add_argument("--sweep", action="store_true",
+                   help="also report the layer's SQNR for every block size in SWEEP_K and every transform "
+                        "(identity, randomized Hadamard, CAT), side by side")
     return p.parse_args()
 
 
@@ -294,6 +298,28 @@ class BufferSet:
                                                           self.sigma, self.xq, self.sx, self.y, self.out3))
 
 
+def transform_sweep(cat, L, x, W, xc, y_ref):
+    """SQNR (dB) of the library's W4A4 output against y = W x in fp32, over all n x d_out outputs,
+    for every block size in SWEEP_K and every transform kind (Sec. 4: identity, the block
+    randomized Hadamard rotation, CAT), each prepared from the same calibration split."""
+    out = {"k": list(SWEEP_K)}
+    for kind in ("identity", "rht", "cat"):
+        vals = []
+        for k in SWEEP_K:
+            sigma = cat.cat_calib_cov(xc, k) if kind == "cat" else None
+            T, Wq, sw = cat.cat_quantize_weights(W, k, kind, sigma_x=sigma, n_calib=L.cfg.n_calib,
+                                                 rht_signs=L.rht_signs if kind == "rht" else None)
+            xq, sx = cat.cat_transform_quantize_act(x, T, k)
+            _, out3 = cat.cat_w4a4_linear_sqnr(xq, sx, Wq, sw, y_ref)
+            vals.append(round(float(out3[2].item()), 3))
+            del T, Wq, sw, xq, sx
+        out[kind] = vals
+    status, detail = cat.cat_device_status()
+    if status != 0:
+        raise DeviceTimeout(f"device status 0x{detail:x} after the transform sweep")
+    return out
+
+
 class DeviceTimeout(RuntimeError):
     """A bounded wait in a kernel gave up (status word bit 0; bits 8..12 name the kernel and bits
     16..31 the source line of the first wait that gave up)."""
@@ -316,6 +342,7 @@ def ours_arm(args, rank, world, local, retried=None):
                                          rht_signs=L.rht_signs if args.kind == "rht" else None)
     torch.backends.cuda.matmul.allow_tf32 = False
     y_ref = (x.float() @ W.float().t()).contiguous()
+    sweep = transform_sweep(cat, L, x, W, xc, y_ref) if args.sweep and rank == 0 else None
     del W
     l2 = torch.cuda.get_device_properties(dev).L2_cache_size
     first = BufferSet(cat, x, xc, y_ref, T, Wq, sw, k, dev)
@@ -508,6 +535,8 @@ def ours_arm(args, rank, world, local, retried=None):
         line["e2e"] = e2e
     if retried:
         line["retried_after"] = retried
+    if sweep:
+        line["sqnr_sweep"] = dict(sweep, unit="dB", over="all n x d_out outputs, y = W x in fp32 as reference")
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = run_cpu_baseline(L, args.kind, k, args.cpu_seconds)
     print(json.dumps(line), flush=True)

@@ -264,3 +264,29 @@ def test_layer_end_to_end(cfg, kind):
     s3 = cat.cat_sqnr(y_ref, g["y"]).cpu().numpy()
     assert abs(s3[2] - ref["sqnr_db"]) < 0.01
     assert cat.cat_device_status()[0] == 0
+
+
+# ------------------------------------------------------------------------------------------
+# The gate/up layer's sweep, reduced: every block size x every transform through the library
+# ------------------------------------------------------------------------------------------
+
+SWEEP_LAYER = WL.small_config("s_gateup_sweep", d_in=1024, d_out=1792, n_eval=384, n_calib=512, k=128,
+                              outlier_frac=0.005, outlier_scale=200.0, w_std=0.01, seed=25)
+
+
+@pytest.mark.parametrize("k", [32, 64, 128, 256])
+def test_block_size_transform_sweep(k):
+    """SQNR of identity, randomized Hadamard and CAT transforms at block size k (Sec. 4) matches the
+    oracle's within 0.01 dB, and CAT beats both (Sec. 3-4: it raises concentration and alignment;
+    with outlier channels this strong the rotation alone barely moves the SQNR)."""
+    L = WL.make_layer(SWEEP_LAYER)
+    res = {}
+    for kind in ("identity", "rht", "cat"):
+        g = gpu_layer(L, kind, k)
+        ref = O.cat_layer(L.x_eval.values, L.W.values, kind, k, X_calib=L.x_calib.values, signs=L.rht_signs)
+        y_ref = torch.from_numpy(ref["y"].astype(np.float32)).to(DEV)
+        s3 = cat.cat_sqnr(y_ref, g["y"]).cpu().numpy()
+        assert abs(s3[2] - ref["sqnr_db"]) < 0.01, (kind, s3[2], ref["sqnr_db"])
+        res[kind] = float(s3[2])
+    assert res["cat"] > res["rht"] + 10.0 and res["cat"] > res["identity"] + 10.0, res
+    assert cat.cat_device_status()[0] == 0
