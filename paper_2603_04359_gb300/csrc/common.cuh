@@ -38,6 +38,25 @@ __host__ __device__ constexpr uint32_t timeout_bits(uint32_t where, int abort) {
 // Upper bound of any single pipeline wait, in nanoseconds of %globaltimer.
 constexpr uint64_t kWaitLimitNs = 1000000000ull;
 
+// Programmatic dependent launch.  A kernel launched with pdl_attr() (the two GEMMs) may be scheduled
+// while the previous kernel in the stream is still running; before its first access to global or
+// tensor memory it calls pdl_wait_then_release(), which waits until that grid has completed with
+// its writes visible, then lets the next dependent grid be scheduled.  The transform and SYRK
+// kernels call it too (without the attribute the wait returns at once) so that a GEMM after them
+// is scheduled early.  A dependent grid is scheduled
+// only once every CTA of this grid has passed that point, i.e. is resident, so waiting CTAs of
+// the next grid can never keep a CTA of this one from an SM.
+inline cudaLaunchAttribute pdl_attr() {
+  cudaLaunchAttribute a;
+  a.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  a.val.programmaticStreamSerializationAllowed = 1;
+  return a;
+}
+__device__ __forceinline__ void pdl_wait_then_release() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 __device__ __forceinline__ void report(uint32_t* status, uint32_t bits) {
   if (status) atomicOr(status, bits);
 }

@@ -139,6 +139,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     bars->abort = 0;
     fence_mbar_init();
   }
+  pdl_wait_then_release();                        // nothing global or in tensor memory before this
   if (warp == 0) tmem_alloc(&bars->tmem_addr, kTmemCols);
   tc_fence_before();
   __syncthreads();
@@ -422,9 +423,17 @@ cudaError_t launch_ntok(const uint8_t* xq, const float* sx, const uint8_t* wq, c
   if (grid > (unsigned)kSqnrMaxCtas) return cudaErrorInvalidConfiguration;
   const int slot = y_ref ? next_sqnr_slot() : 0;
   note_launch();
-  w4a4_gemm_decode_tc_kernel<NTOK><<<grid, kThreads, smem, stream>>>(map, xq, sx, sw, (int)n, (int)d_in, (int)d_out,
-                                                                      sp, y, acc_out, y_ref, sums3, slot, status);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = dim3(grid, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attrs[1] = {pdl_attr()};
+  cfg.attrs = attrs;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, w4a4_gemm_decode_tc_kernel<NTOK>, map, xq, sx, sw, (int)n, (int)d_in, (int)d_out, sp,
+                            y, acc_out, y_ref, sums3, slot, status);
 }
 
 }  // namespace

@@ -247,6 +247,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     fence_mbar_init();
   }
   __syncwarp();
+  pdl_wait_then_release();                        // nothing global or in tensor memory before this
   if (warp == 0) tmem_alloc_pair(&bars->tmem_addr, kTmemCols);
   tc_fence_before();
   cluster_sync();                                 // both CTAs' barriers are initialized before any remote arrive
@@ -838,27 +839,21 @@ cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_
   const int slot = y_ref ? next_sqnr_slot() : 0;
   const double* sums = y_ref ? sums3 : nullptr;
   note_launch();
-  if (split == 1) {
-    w4a4_gemm_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(ty, ta, tb, tr, y_ref, const_cast<double*>(sums), slot,
-                                                                sx, sw, (int)n, (int)d_in, (int)d_out, y, acc_out,
-                                                                use_tma, (int)num_full, split, split_slot, status);
-    return cudaGetLastError();
-  }
   cudaLaunchConfig_t cfg;
   memset(&cfg, 0, sizeof(cfg));
   cfg.gridDim = dim3((unsigned)grid, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = kSmemBytes;
   cfg.stream = stream;
-  cudaLaunchAttribute attrs[1];
-  attrs[0].id = cudaLaunchAttributeCooperative;
-  attrs[0].val.cooperative = 1;
+  cudaLaunchAttribute attrs[2];
+  attrs[0] = pdl_attr();
+  attrs[1].id = cudaLaunchAttributeCooperative;   // the split parts wait for one another
+  attrs[1].val.cooperative = 1;
   cfg.attrs = attrs;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = split > 1 ? 2 : 1;
   return cudaLaunchKernelEx(&cfg, w4a4_gemm_tc_kernel, ty, ta, tb, tr, y_ref, const_cast<double*>(sums), slot, sx, sw,
                             (int)n, (int)d_in, (int)d_out, y, acc_out, use_tma, (int)num_full, split, split_slot,
                             status);
-  return cudaGetLastError();
 }
 
 }  // namespace cat
