@@ -46,6 +46,7 @@ struct TcCfg {
 
 struct TcBars {
   uint64_t x_full[kXStages], x_empty[kXStages], d_full[2], d_empty[2], t_full, t_empty, mma_done;
+  uint64_t t_first;                              // fused kernel: the CTA's first T_b split is in shared memory
   uint32_t tmem_addr;
   int abort;
 };
@@ -452,6 +453,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bars->x_empty[st], 1);
     }
     for (int j = 0; j < kMaxUnits; ++j) mbar_init(&unit_full[j], 1);
+    mbar_init(&bars->t_first, kCvtWarps);
     mbar_init(&bars->t_full, kCvtWarps);
     mbar_init(&bars->t_empty, 1);
     mbar_init(&bars->mma_done, 1);
@@ -475,6 +477,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int64_t u = u0; u < u1 && ok; ++u, ++j) {
         const int b = (int)(u / num_tiles), tile = (int)(u % num_tiles);
         const uint32_t st = j % kXStages;
+        // the first unit's x tile goes out with T_b's loads; the others wait until T_b is split, so
+        // that T_b does not queue behind them in HBM and unit 0's MMAs start as early as they can
+        if (j == 1 && !(ok = mbar_wait_bounded(&bars->t_first, 0, abort_flag, __LINE__))) break;
         if (j >= kXStages && !(ok = mbar_wait_bounded(&bars->x_empty[st], ((j / kXStages) - 1) & 1, abort_flag, __LINE__))) break;
         mbar_arrive_expect_tx(&bars->x_full[st], C::X_STAGE);
 #pragma unroll
@@ -537,7 +542,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       split_block<K>(A + (size_t)b * K * K, ts, ct);
       fence_proxy_async_smem();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->t_full);
+      if (lane == 0) {
+        mbar_arrive(&bars->t_full);
+        if (version == 0) mbar_arrive(&bars->t_first);
+      }
       ++version;
     }
     quant_bar();                                       // the epilogue warps have passed the first grid barrier
