@@ -303,8 +303,12 @@ def transform_sweep(cat, L, x, W, xc, y_ref):
     for every block size in SWEEP_K and every transform kind (Sec. 4: identity, the block
     randomized Hadamard rotation, CAT), each prepared from the same calibration split."""
     out = {"k": list(SWEEP_K)}
+    diag = {}
+    n2 = float((2 * (2 ** 3 - 1)) ** 2)           # 14 intervals of the restricted INT4 grid, squared
+    db = lambda v: round(10.0 * float(np.log10(v)), 3)
     for kind in ("identity", "rht", "cat"):
         vals = []
+        dk = {"C_x_db": [], "C_w_db": [], "A_db": [], "theorem1_db": []}
         for k in SWEEP_K:
             sigma = cat.cat_calib_cov(xc, k) if kind == "cat" else None
             T, Wq, sw = cat.cat_quantize_weights(W, k, kind, sigma_x=sigma, n_calib=L.cfg.n_calib,
@@ -312,8 +316,22 @@ def transform_sweep(cat, L, x, W, xc, y_ref):
             xq, sx = cat.cat_transform_quantize_act(x, T, k)
             _, out3 = cat.cat_w4a4_linear_sqnr(xq, sx, Wq, sw, y_ref)
             vals.append(round(float(out3[2].item()), 3))
-            del T, Wq, sw, xq, sx
+            # diagnostics (Sec. 2): C(x') = sum ||x'||^2 / sum r^2, C(W') likewise over output rows,
+            # A = sum y^2 / (sum ||w'||^2 sum ||x'||^2), Theorem 1: 12 (N^2 C(x') || N^2 C(W')) A
+            Tinv = torch.linalg.inv(T.double()).float().contiguous()
+            _, _, x3 = cat.cat_block_row_stats(x, k, T)
+            _, _, w3 = cat.cat_block_row_stats(W, k, Tinv, transpose=True)
+            sx2, rx2 = float(x3[0].item()), float(x3[1].item())
+            sw2, rw2 = float(w3[0].item()), float(w3[1].item())
+            c_x, c_w, a = sx2 / rx2, sw2 / rw2, float(out3[0].item()) / (sw2 * sx2)
+            dk["C_x_db"].append(db(c_x))
+            dk["C_w_db"].append(db(c_w))
+            dk["A_db"].append(db(a))
+            dk["theorem1_db"].append(db(12.0 * a / (1.0 / (n2 * c_x) + 1.0 / (n2 * c_w))))
+            del T, Wq, sw, xq, sx, Tinv
         out[kind] = vals
+        diag[kind] = dk
+    out["diagnostics"] = diag
     status, detail = cat.cat_device_status()
     if status != 0:
         raise DeviceTimeout(f"device status 0x{detail:x} after the transform sweep")
@@ -536,7 +554,9 @@ def ours_arm(args, rank, world, local, retried=None):
     if retried:
         line["retried_after"] = retried
     if sweep:
-        line["sqnr_sweep"] = dict(sweep, unit="dB", over="all n x d_out outputs, y = W x in fp32 as reference")
+        line["sqnr_sweep"] = dict(sweep, unit="dB", over="all n x d_out outputs, y = W x in fp32 as reference",
+                                  diagnostics_note="per transform and k: concentrations C(x'), C(W'), alignment A "
+                                                   "and the Theorem-1 SQNR prediction (N = 14 intervals), in dB")
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = run_cpu_baseline(L, args.kind, k, args.cpu_seconds)
     print(json.dumps(line), flush=True)

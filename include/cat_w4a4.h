@@ -212,6 +212,29 @@ cat_status cat_w4a4_linear_sqnr(const uint8_t* xq, const float* x_scale, const u
 cat_status cat_sqnr(const float* y_ref, const float* y_hat, int64_t numel, double* out3, cat_stream_t stream);
 
 /*
+ * cat_block_row_stats -- per-layer diagnostics (Sec. 2, Lemmas 2 and 3): the row statistics of a
+ * block-transformed matrix that the concentration C(v) = E||v||^2 / E r(v)^2 (symmetric range
+ * r(v) = 2 max_i |v_i|) and the alignment A(x, W) = E||W x||^2 / (||W||_F^2 E||x||^2) are made of.
+ *   V          device [rows][d] in `dtype`: activations x (one token per row) or weights W (one
+ *              output channel per row).
+ *   M_blocks   device [d/k][k][k] float32.  transpose = 0: v'_b = M_b v_b (activations with
+ *              M = T, x' = T x); transpose = 1: v'_b = M_b^T v_b (weight rows with M = T^{-1},
+ *              w' = w T^{-1}).
+ *   row_sumsq  out, device [rows] float32: ||v'_r||^2 (fp32 sums).
+ *   row_amax   out, device [rows] float32: max_i |v'_ri|.
+ *   out3       out, device [3] float64: { sum_r ||v'_r||^2, sum_r (2 max_i |v'_ri|)^2,
+ *              10 log10 of their ratio, i.e. C(v') in dB }.
+ * Then C(x') = out3x[0] / out3x[1], C(W') = out3w[0] / out3w[1], and with sum y^2 over the layer's
+ * outputs (cat_sqnr's first word) A = sum y^2 / (out3w[0] * out3x[0]) (the 1/n of both expectations
+ * cancels).  Diagnostics, off the layer's hot path: a SIMT kernel plus a reduction; the row
+ * outputs are zeroed with two memsets.  Requires rows in [1, 2^31), k in 16..256 (power of two)
+ * dividing d, and 16-byte aligned pointers.
+ */
+cat_status cat_block_row_stats(const void* V, cat_dtype dtype, int64_t rows, int64_t d, int32_t k,
+                               const float* M_blocks, int transpose, float* row_sumsq, float* row_amax, double* out3,
+                               cat_stream_t stream);
+
+/*
  * cat_device_status -- synchronizes `stream`, then reads and clears the device status word.
  * Returns CAT_OK, CAT_ERR_TIMEOUT (a bounded wait in a kernel gave up and the kernel returned
  * early; its outputs are undefined) or CAT_ERR_NUMERIC (a kernel met a non-finite value; the

@@ -66,6 +66,7 @@ def load_library() -> ctypes.CDLL:
         "cat_sqnr": ([P, P, I64, P, P], I),
         "cat_w4a4_linear_sqnr": ([P, P, P, P, I64, I64, I64, P, P, P, P], I),
         "cat_device_status": ([P, P], I),
+        "cat_block_row_stats": ([P, I, I64, I64, I32, P, I, P, P, P, P], I),
     }
     for name, (args, res) in sigs.items():
         f = getattr(lib, name)
@@ -247,6 +248,22 @@ def cat_sqnr(y_ref: torch.Tensor, y_hat: torch.Tensor, out: Optional[torch.Tenso
     _check("cat_sqnr", load_library().cat_sqnr(_ptr(y_ref), _ptr(y_hat), y_ref.numel(), _ptr(out),
                                                _stream(y_ref.device)))
     return out
+
+
+def cat_block_row_stats(V: torch.Tensor, k: int, M: torch.Tensor, transpose: bool = False):
+    """Row statistics of V transformed block by block (v'_b = M_b v_b, or M_b^T v_b when
+    ``transpose``): (row ||v'||^2 float32 [rows], row max |v'| float32 [rows], float64 [3]
+    {sum ||v'||^2, sum (2 max |v'|)^2, 10 log10 of their ratio}) on V's device."""
+    _need(V, "V")
+    _need(M, "M")
+    rows, d = V.shape
+    row_sumsq = torch.empty((rows,), dtype=torch.float32, device=V.device)
+    row_amax = torch.empty((rows,), dtype=torch.float32, device=V.device)
+    out3 = torch.empty((3,), dtype=torch.float64, device=V.device)
+    _check("cat_block_row_stats", load_library().cat_block_row_stats(
+        _ptr(V), _dtype(V), rows, d, k, _ptr(M), 1 if transpose else 0, _ptr(row_sumsq), _ptr(row_amax), _ptr(out3),
+        _stream(V.device)))
+    return row_sumsq, row_amax, out3
 
 
 def cat_device_status(device: Optional[torch.device] = None) -> Tuple[int, int]:

@@ -20,6 +20,9 @@ cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_
 cudaError_t launch_w4a4_gemm_decode(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
                                     int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, const float* y_ref,
                                     double* sums3, uint32_t* status, cudaStream_t stream);
+cudaError_t launch_block_row_stats(const void* V, int dtype, int64_t rows, int64_t d, int k, const float* M,
+                                   int transpose, float* row_sumsq, float* row_amax, double* out3,
+                                   cudaStream_t stream);
 }  // namespace cat
 
 namespace {
@@ -434,3 +437,22 @@ cat_status cat_device_status(cat_stream_t stream, uint32_t* detail) {
 }
 
 }  // extern "C"
+
+cat_status cat_block_row_stats(const void* V, cat_dtype dtype, int64_t rows, int64_t d, int32_t k,
+                               const float* M_blocks, int transpose, float* row_sumsq, float* row_amax, double* out3,
+                               cat_stream_t stream) {
+  if (dtype != CAT_F32 && dtype != CAT_BF16) return fail(CAT_ERR_INVALID_ARG, "unknown dtype");
+  if (rows < 1 || rows > 0x7FFFFFFF) return fail(CAT_ERR_SHAPE, "rows must be in [1, 2^31)");
+  cat_status st = check_din(d);
+  if (st != CAT_OK) return st;
+  if (!valid_k(k) || d % k != 0) return fail(CAT_ERR_SHAPE, "k must be one of 16..256 (power of two) and divide d");
+  if (transpose != 0 && transpose != 1) return fail(CAT_ERR_INVALID_ARG, "transpose must be 0 or 1");
+  if (!V || !M_blocks || !row_sumsq || !row_amax || !out3) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(V) || !aligned16(M_blocks) || !aligned16(row_sumsq) || !aligned16(row_amax) || !aligned16(out3))
+    return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  if ((st = check_device()) != CAT_OK) return st;
+  cudaError_t e = cat::launch_block_row_stats(V, (int)dtype, rows, d, k, M_blocks, transpose, row_sumsq, row_amax, out3,
+                                              (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cat_block_row_stats launch");
+  return ok();
+}

@@ -1,0 +1,179 @@
+// Per-layer diagnostics (Sec. 2): the row statistics that the concentration C(v) = E||v||^2 / E r(v)^2
+// (Lemmas 2 and 3, symmetric range r(v) = 2 max_i |v_i|) and the alignment
+// A(x, W) = E||W x||^2 / (||W||_F^2 E||x||^2) are made of, for rows transformed block by block:
+//   v'_b = M_b v_b          (activations, M = T: x' = T x)
+//   v'_b = M_b^T v_b        (weight rows, M = T^{-1}: w' = w T^{-1})
+// Off the timed path; a plain SIMT kernel.  A CTA takes 64 rows of one block: the rows' block
+// slice and one 64-output slab of M_b at a time sit in shared memory, every thread accumulates a
+// 4-row x (JT / 16)-output register tile in fp32, and each row's partial sum of squares and
+// maximum go to per-row accumulators (float atomics; the maximum on the float bits, which order
+// like the values for non-negative floats).  A second kernel adds the rows' sums of squares and
+// squared ranges through the cross-CTA reduction of sqnr_slot.cuh, which also forms
+// 10 log10(sum ||v'||^2 / sum r^2) = C in dB.
+#include <cstring>
+#include <mutex>
+
+#include "common.cuh"
+#include "sqnr_slot.cuh"
+
+namespace cat {
+namespace {
+
+constexpr int kRows = 64;        // rows per CTA
+constexpr int kThreads = 256;    // 16 row groups of 4 x 16 output groups
+
+template <int K>
+struct DiagCfg {
+  static constexpr int JT = K < 64 ? K : 64;     // outputs per slab
+  static constexpr int OJ = JT / 16;             // outputs per thread
+  static constexpr size_t SMEM = (size_t)K * kRows * 4 + (size_t)K * JT * 4;
+};
+
+__device__ __forceinline__ float load_elem(const void* V, int dtype, size_t idx) {
+  if (dtype == 0) return reinterpret_cast<const float*>(V)[idx];
+  return __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(V)[idx]);
+}
+
+template <int K>
+__global__ void __launch_bounds__(kThreads)
+    block_row_stats_kernel(const void* __restrict__ V, int dtype, int rows, int d, const float* __restrict__ M,
+                           int transpose, float* __restrict__ row_sumsq, uint32_t* __restrict__ row_amax_bits) {
+  using C = DiagCfg<K>;
+  extern __shared__ float sm[];
+  float* vs = sm;                       // [K][kRows]: the rows' block slice, transposed
+  float* ms = sm + K * kRows;           // [K][JT]: ms[i][j] is the weight of input i in output j of the slab
+  const int tid = threadIdx.x, r0 = blockIdx.x * kRows, b = blockIdx.y;
+  const float* Mb = M + (size_t)b * K * K;
+  for (int e = tid; e < K * kRows; e += kThreads) {   // i fastest: coalesced along the row
+    const int r = e / K, i = e % K;
+    vs[i * kRows + r] = (r0 + r < rows) ? load_elem(V, dtype, (size_t)(r0 + r) * d + (size_t)b * K + i) : 0.f;
+  }
+  const int tr = tid >> 4, tj = tid & 15;
+  float sumsq[4] = {0.f, 0.f, 0.f, 0.f}, amax[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int j0 = 0; j0 < K; j0 += C::JT) {
+    __syncthreads();                                   // the previous slab is no longer read
+    for (int e = tid; e < K * C::JT; e += kThreads) {
+      if (transpose) {                                 // ms[i][j] = M_b[i][j0 + j]
+        const int i = e / C::JT, j = e % C::JT;
+        ms[i * C::JT + j] = Mb[(size_t)i * K + j0 + j];
+      } else {                                         // ms[i][j] = M_b[j0 + j][i]
+        const int j = e / K, i = e % K;
+        ms[i * C::JT + j] = Mb[(size_t)(j0 + j) * K + i];
+      }
+    }
+    __syncthreads();
+    float acc[4][C::OJ];
+#pragma unroll
+    for (int rr = 0; rr < 4; ++rr)
+#pragma unroll
+      for (int oj = 0; oj < C::OJ; ++oj) acc[rr][oj] = 0.f;
+#pragma unroll 4
+    for (int i = 0; i < K; ++i) {
+      const float4 v4 = *reinterpret_cast<const float4*>(&vs[i * kRows + 4 * tr]);
+      const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
+#pragma unroll
+      for (int oj = 0; oj < C::OJ; ++oj) {
+        const float m = ms[i * C::JT + tj * C::OJ + oj];
+#pragma unroll
+        for (int rr = 0; rr < 4; ++rr) acc[rr][oj] = fmaf(vv[rr], m, acc[rr][oj]);
+      }
+    }
+#pragma unroll
+    for (int rr = 0; rr < 4; ++rr)
+#pragma unroll
+      for (int oj = 0; oj < C::OJ; ++oj) {
+        sumsq[rr] = fmaf(acc[rr][oj], acc[rr][oj], sumsq[rr]);
+        amax[rr] = fmaxf(amax[rr], fabsf(acc[rr][oj]));
+      }
+  }
+  // the 16 output groups of a row group are the 16 lanes that differ in bits 0..3 of the lane index
+#pragma unroll
+  for (int rr = 0; rr < 4; ++rr) {
+#pragma unroll
+    for (int off = 8; off > 0; off >>= 1) {
+      sumsq[rr] += __shfl_xor_sync(0xFFFFFFFFu, sumsq[rr], off);
+      amax[rr] = fmaxf(amax[rr], __shfl_xor_sync(0xFFFFFFFFu, amax[rr], off));
+    }
+    const int r = r0 + 4 * tr + rr;
+    if (tj == 0 && r < rows) {
+      atomicAdd(&row_sumsq[r], sumsq[rr]);
+      atomicMax(&row_amax_bits[r], __float_as_uint(amax[rr]));
+    }
+  }
+}
+
+// sum_r ||v'_r||^2 and sum_r (2 max_i |v'_ri|)^2 over all rows, and 10 log10 of their ratio.
+__global__ void __launch_bounds__(kThreads)
+    row_stats_reduce_kernel(const float* __restrict__ row_sumsq, const float* __restrict__ row_amax, int rows,
+                            double* __restrict__ out3, int slot) {
+  f32x2 s = {0.f, 0.f}, r2 = {0.f, 0.f};
+  for (int r = blockIdx.x * kThreads + threadIdx.x; r < rows; r += gridDim.x * kThreads) {
+    const float a = 2.f * row_amax[r];
+    s = f2_add(s, row_sumsq[r]);
+    r2 = f2_add(r2, a * a);
+  }
+  s = f2_warp_sum(s);
+  r2 = f2_warp_sum(r2);
+  __shared__ f32x2 ws[kThreads / 32][2];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) {
+    ws[warp][0] = s;
+    ws[warp][1] = r2;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    f32x2 a = {0.f, 0.f}, b = {0.f, 0.f};
+    for (int w = 0; w < kThreads / 32; ++w) {
+      a = f2_add(a, ws[w][0]);
+      b = f2_add(b, ws[w][1]);
+    }
+    sqnr_cta_done(slot, a, b, out3);
+  }
+}
+
+template <int K>
+cudaError_t launch_k(const void* V, int dtype, int64_t rows, int64_t d, const float* M, int transpose,
+                     float* row_sumsq, float* row_amax, cudaStream_t stream) {
+  using C = DiagCfg<K>;
+  static std::once_flag once;
+  static cudaError_t attr = cudaSuccess;
+  std::call_once(once, [] {
+    attr = cudaFuncSetAttribute(block_row_stats_kernel<K>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
+  });
+  if (attr != cudaSuccess) return attr;
+  dim3 grid((unsigned)((rows + kRows - 1) / kRows), (unsigned)(d / K), 1);
+  note_launch();
+  block_row_stats_kernel<K><<<grid, kThreads, C::SMEM, stream>>>(V, dtype, (int)rows, (int)d, M, transpose, row_sumsq,
+                                                                 reinterpret_cast<uint32_t*>(row_amax));
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+// row_sumsq and row_amax are zeroed here and accumulated by the block kernel; out3 is written by the
+// reduction (no zeroing needed).
+cudaError_t launch_block_row_stats(const void* V, int dtype, int64_t rows, int64_t d, int k, const float* M,
+                                   int transpose, float* row_sumsq, float* row_amax, double* out3,
+                                   cudaStream_t stream) {
+  cudaError_t e = cudaMemsetAsync(row_sumsq, 0, (size_t)rows * sizeof(float), stream);
+  if (e == cudaSuccess) e = cudaMemsetAsync(row_amax, 0, (size_t)rows * sizeof(float), stream);
+  if (e != cudaSuccess) return e;
+  switch (k) {
+    case 16: e = launch_k<16>(V, dtype, rows, d, M, transpose, row_sumsq, row_amax, stream); break;
+    case 32: e = launch_k<32>(V, dtype, rows, d, M, transpose, row_sumsq, row_amax, stream); break;
+    case 64: e = launch_k<64>(V, dtype, rows, d, M, transpose, row_sumsq, row_amax, stream); break;
+    case 128: e = launch_k<128>(V, dtype, rows, d, M, transpose, row_sumsq, row_amax, stream); break;
+    case 256: e = launch_k<256>(V, dtype, rows, d, M, transpose, row_sumsq, row_amax, stream); break;
+    default: return cudaErrorInvalidValue;
+  }
+  if (e != cudaSuccess) return e;
+  int64_t grid = (rows + 4 * kThreads - 1) / (4 * kThreads);
+  if (grid < 1) grid = 1;
+  if (grid > kSqnrMaxCtas) grid = kSqnrMaxCtas;
+  note_launch();
+  row_stats_reduce_kernel<<<(unsigned)grid, kThreads, 0, stream>>>(row_sumsq, row_amax, (int)rows, out3,
+                                                                   next_sqnr_slot());
+  return cudaGetLastError();
+}
+
+}  // namespace cat

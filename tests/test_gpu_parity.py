@@ -290,3 +290,42 @@ def test_block_size_transform_sweep(k):
         res[kind] = float(s3[2])
     assert res["cat"] > res["rht"] + 10.0 and res["cat"] > res["identity"] + 10.0, res
     assert cat.cat_device_status()[0] == 0
+
+
+# ------------------------------------------------------------------------------------------
+# Per-layer diagnostics: concentration, alignment and the Theorem-1 prediction from the library's
+# row statistics of x' = T x and W' = W T^{-1}
+# ------------------------------------------------------------------------------------------
+
+@pytest.mark.parametrize("cfg", [SMALL[0], SMALL[1], SMALL[2], SWEEP_LAYER], ids=lambda c: c.name)
+@pytest.mark.parametrize("kind", ["identity", "rht", "cat"])
+def test_layer_diagnostics(cfg, kind):
+    """C(x') and C(W') (Lemmas 2 and 3), A(x', W') and the Theorem-1 SQNR from cat_block_row_stats
+    match the oracle's analysis functions on the oracle's x' and W' within 1e-4 (fp32 products)."""
+    L = WL.make_layer(cfg)
+    k = cfg.k
+    g = gpu_layer(L, kind, k)
+    ref = O.cat_layer(L.x_eval.values, L.W.values, kind, k, X_calib=L.x_calib.values, signs=L.rht_signs)
+    Xp = O.apply_act_transform(L.x_eval.values, ref["prep"].T)
+    Wp = ref["prep"].Wt
+    # the weight rows need T^{-1}: the inverse of the library's own T blocks, on the host
+    Tinv = np.linalg.inv(g["T"].double().cpu().numpy()).astype(np.float32)
+    xs, xa, x3 = cat.cat_block_row_stats(to_dev(L.x_eval), k, g["T"])
+    ws, wa, w3 = cat.cat_block_row_stats(to_dev(L.W), k, torch.from_numpy(Tinv).to(DEV), transpose=True)
+    x3, w3 = x3.cpu().numpy(), w3.cpu().numpy()
+    np.testing.assert_allclose(xs.cpu().numpy(), np.sum(Xp * Xp, axis=1), rtol=1e-4, atol=1e-12)
+    np.testing.assert_allclose(xa.cpu().numpy(), np.max(np.abs(Xp), axis=1), rtol=1e-4, atol=1e-12)
+    np.testing.assert_allclose(ws.cpu().numpy(), np.sum(Wp * Wp, axis=1), rtol=1e-4, atol=1e-12)
+    np.testing.assert_allclose(wa.cpu().numpy(), np.max(np.abs(Wp), axis=1), rtol=1e-4, atol=1e-12)
+    c_x, c_w = x3[0] / x3[1], w3[0] / w3[1]
+    assert abs(c_x / O.concentration_act(Xp) - 1) < 1e-4
+    assert abs(c_w / O.concentration_weight(Wp) - 1) < 1e-4
+    assert abs(x3[2] - 10 * np.log10(c_x)) < 1e-4
+    y = O.linear(L.x_eval.values, L.W.values)
+    sum_y2 = float(cat.cat_sqnr(torch.from_numpy(y.astype(np.float32)).to(DEV), g["y"]).cpu().numpy()[0])
+    a = sum_y2 / (w3[0] * x3[0])
+    assert abs(a / O.alignment(Xp, Wp) - 1) < 1e-4
+    n2 = O.n_intervals(4) ** 2
+    pred = 12.0 * O.parallel(n2 * c_x, n2 * c_w) * a
+    assert abs(O.db(pred) - O.db(O.theorem1_sqnr(Xp, Wp))) < 1e-3
+    assert cat.cat_device_status()[0] == 0
