@@ -63,6 +63,14 @@ constexpr uint32_t kStageB = BNC * BK;      // 16 KiB of E4M3 per stage (two ato
 constexpr int kThreads = 512;
 constexpr int kProdA = 0, kMmaWarp = 1, kProdB = 2, kFwdWarp = 3;
 constexpr int kDecWarp0 = 8, kGroupWarps = 4, kGroupThreads = kGroupWarps * 32;  // two decode groups
+constexpr int kDecGroups = 2;                // the groups take alternate K steps
+// The packed stages are not a multiple of the groups, so one packed stage is consumed by both groups
+// in turn.  Each group therefore gets its own full-barrier per packed stage: a barrier's phases are
+// then consumed by one group only, which has seen the previous phase complete before it waits for
+// the next one.  (With one barrier per stage, a group could wait for a phase two ahead of the
+// barrier, when the other group's load is late, and the parity wait would return at once.)
+// Loads into barrier (g, s) come every kPFullPeriod K steps.
+constexpr int kPFullPeriod = SP % kDecGroups == 0 ? SP : SP * kDecGroups;
 constexpr int kEpiWarp0 = 4, kEpiWarps = 4;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kAccCols = 2 * BN;       // two accumulators
@@ -83,7 +91,7 @@ static_assert((BNC * 8) % kGroupThreads == 0, "B chunks per decode thread");
 
 
 struct Bars {
-  uint64_t p_full[SP], p_empty[SP], full[SE], ready[SE], empty[SE], acc_full[2], acc_empty[2], mma_done;
+  uint64_t p_full[kDecGroups][SP], p_empty[SP], full[SE], ready[SE], empty[SE], acc_full[2], acc_empty[2], mma_done;
   uint64_t ref_full[kEpiWarps][kEpiBufs];      // y_ref tile loads of each epilogue warp
   uint32_t fwd_word[SE];                         // even CTA: targets of the odd CTA's st.async per stage
   uint32_t tmem_addr;
@@ -228,7 +236,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 
   if (tid == 0) {
     for (int s = 0; s < SP; ++s) {
-      mbar_init(&bars->p_full[s], 2);          // the A and the B producer each arrive with their bytes
+      for (int g = 0; g < kDecGroups; ++g)
+        mbar_init(&bars->p_full[g][s], 2);     // the A and the B producer each arrive with their bytes
       mbar_init(&bars->p_empty[s], kGroupWarps);    // the decode group of that stage
     }
     for (int s = 0; s < SE; ++s) {
@@ -269,14 +278,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           const uint32_t s = it % SP, use = it / SP;
           if (use > 0 && !(ok = mbar_wait_bounded(&bars->p_empty[s], (use - 1) & 1, abort_flag, __LINE__))) break;
           uint8_t* dst = pk + s * kPackedStage + (is_a ? 0 : kPackedA);
-          mbar_arrive_expect_tx(&bars->p_full[s], is_a ? kPackedA : kPackedB);
-          tma_load_2d(dst, map, ks * BKP, is_a ? m * 2 * BM + (int)rank * BM : nn * BN + (int)rank * BNC,
-                      &bars->p_full[s]);
+          uint64_t* pf = &bars->p_full[it % kDecGroups][s];   // the barrier of the group that decodes it
+          mbar_arrive_expect_tx(pf, is_a ? kPackedA : kPackedB);
+          tma_load_2d(dst, map, ks * BKP, is_a ? m * 2 * BM + (int)rank * BM : nn * BN + (int)rank * BNC, pf);
         }
       }
       const uint32_t issued = it, first = issued > SP ? issued - SP : 0;
       volatile int no_abort = 0;
-      for (uint32_t j = first; j < issued; ++j) mbar_wait_bounded(&bars->p_full[j % SP], (j / SP) & 1, &no_abort);
+      for (uint32_t j = first; j < issued; ++j)
+        mbar_wait_bounded(&bars->p_full[j % kDecGroups][j % SP], (j / kPFullPeriod) & 1, &no_abort);
     }
   } else if ((warp == kMmaWarp || warp == kFwdWarp) && rank == 1) {
     // ---------------------------------------------------------------- odd CTA: forward stage readiness
@@ -647,7 +657,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       for (int ks = w.k0; ks < w.k1; ++ks, ++it) {
         if ((it & 1u) != (uint32_t)grp) continue;
         const uint32_t ps = it % SP, s = it % SE;
-        if (!(ok = mbar_wait_bounded(&bars->p_full[ps], (it / SP) & 1, abort_flag, __LINE__))) break;
+        if (!(ok = mbar_wait_bounded(&bars->p_full[grp][ps], (it / kPFullPeriod) & 1, abort_flag, __LINE__))) break;
         if (it >= SE && !(ok = mbar_wait_bounded(&bars->empty[s], ((it / SE) - 1) & 1, abort_flag, __LINE__))) break;
         tc_fence_after();
         const uint8_t* pa = pk + ps * kPackedStage;
