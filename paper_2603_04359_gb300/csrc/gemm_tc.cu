@@ -195,8 +195,9 @@ __device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
 
 // Work unit u of the launch: the n_split = tail x split parts come first (part u % split of tail
 // tile num_full + u / split, on pairs 0 .. n_split - 1, one each), then the whole tiles (tile
-// u - n_split).  Each part's sibling parts run at the same time, and the part's share of the tile is
-// finished after the pair's first whole tile, when they have long arrived.
+// u - n_split).  All parts run at the same time, as their pairs' first units, and each part's share
+// of the tile is finished while the MMAs of its pair's first whole tile run (the epilogue is idle
+// then).
 struct Unit {
   int tile, k0, k1, part;                     // part < 0: the whole tile
 };
@@ -582,10 +583,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
         ++fcount;
         if (!ok) break;
-        if (split_state == 1) {                     // the split part's siblings have long arrived
-          finish_share(pair);
-          split_state = 2;
-        }
       } else {
         // a K part of a tail tile: this warp's 32 rows of raw accumulators to the part's slice
         const int tj = w.tile - num_full, j = u;
@@ -608,11 +605,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
         arrive_part(tj);
         split_state = 1;
+        // the sibling parts run at the same time, on other pairs, as their first unit: the share is
+        // finished while this pair's first whole tile is still in its MMAs
+        finish_share(pair);
+        split_state = 2;
       }
-    }
-    if (ok && split_state == 1) {                   // no whole tile followed the split part
-      finish_share(pair);
-      split_state = 2;
     }
     if (!ok && pair < n_split) {
       // a wait gave up: settle this warp's split part all the same (without data: the launch's
