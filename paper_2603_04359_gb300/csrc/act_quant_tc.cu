@@ -125,6 +125,28 @@ __device__ __forceinline__ void split_block(const float* __restrict__ Ab, uint8_
   }
 }
 
+// Four two's-complement bytes in [-7, 7] -> the SM4x8 sign-magnitude bytes (sign << 7 | magnitude).
+__device__ __forceinline__ uint32_t twos_to_sm(uint32_t w) {
+  const uint32_t s = (w >> 7) & 0x01010101u;        // 1 in every negative byte
+  const uint32_t m = (s << 8) - s;                   // 0xFF in every negative byte
+  return ((w ^ m) + s) | (s << 7);                   // |q| (no carry leaves a byte) and the sign bit
+}
+
+// One SM4x8 word of the codes rint(fl32(v_e * inv)), e = 0..7 (v_e = r[base + e] as float), for
+// |v_e * inv| <= 7 (inv = 7 / max|v|).  Adding 1.5 * 2^23 to the rounded product rounds it to an
+// integer (half to even, as rint) that sits, two's complement, in the low byte of the sum's bits;
+// the bytes are gathered four to a word and turned into sign-magnitude.  A non-finite product leaves
+// a garbage byte: callers zero the codes of rows whose maximum is not finite.
+__device__ __forceinline__ uint32_t sm4_quant8(const uint32_t (&r)[32], int base, float inv) {
+  constexpr float kMagic = 12582912.0f;
+  uint32_t b[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) b[e] = __float_as_uint(__fadd_rn(__fmul_rn(__uint_as_float(r[base + e]), inv), kMagic));
+  const uint32_t lo = twos_to_sm(__byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410));
+  const uint32_t hi = twos_to_sm(__byte_perm(__byte_perm(b[4], b[5], 0x0040), __byte_perm(b[6], b[7], 0x0040), 0x5410));
+  return lo | __funnelshift_l(hi, hi, 4);
+}
+
 template <int K, int PASS>
 __global__ void __launch_bounds__(kThreads, 1)
     transform_quant_tc_kernel(const __grid_constant__ CUtensorMap tmX, const float* __restrict__ A, int n, int d,
@@ -247,19 +269,25 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int64_t words_per_row = d / 8;
     bool ok = true, finite = true;
     uint32_t j = 0;
+    // pass 1: this lane's row maximum for the next unit is loaded while the current unit is quantized
+    auto row_of = [&](int64_t uu) { return (int)(uu % num_tiles) * TM + quad * 32 + lane; };
+    float a_next = 0.f;
+    if (PASS == 1 && u0 < u1 && row_of(u0) < n) a_next = __uint_as_float(__ldcg(&amax_bits[row_of(u0)]));
     for (int64_t u = u0; u < u1 && ok; ++u, ++j) {
       const int b = (int)(u / num_tiles), tile = (int)(u % num_tiles);
       const uint32_t sd = j & 1;
       const int t = tile * TM + quad * 32 + lane;
       float inv = 0.f;
-      if (PASS == 1 && t < n) {
-        const float a = __uint_as_float(amax_bits[t]);
-        inv = (isfinite(a) && a > 0.f) ? __fdiv_rn(7.0f, a) : 0.f;
+      if (PASS == 1) {
+        const float a = a_next;
+        if (u + 1 < u1 && row_of(u + 1) < n) a_next = __uint_as_float(__ldcg(&amax_bits[row_of(u + 1)]));
+        inv = (t < n && isfinite(a) && a > 0.f) ? __fdiv_rn(7.0f, a) : 0.f;
       }
       if (!(ok = mbar_wait_bounded(&bars->d_full[sd], (j >> 1) & 1, abort_flag, __LINE__))) break;
       __syncwarp();
       tc_fence_after();
       float m = 0.f;
+      bool row_finite = true;
 #pragma unroll 1
       for (int c = 0; c < K / 32; ++c) {
         uint32_t r[32];
@@ -270,22 +298,15 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int e = 0; e < 32; ++e) {
             const float v = __uint_as_float(r[e]);
-            finite &= isfinite(v);
+            row_finite &= isfinite(v);
             m = fmaxf(m, fabsf(v));
           }
         } else if (t < n) {
+          // the row's codes with the final maximum (|v * inv| <= 7 for a finite row; inv = 0 gives
+          // 0 codes for an all-zero or non-finite row)
           uint32_t w[4];
 #pragma unroll
-          for (int g = 0; g < 4; ++g) {
-            int q[8];
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-              const float v = __uint_as_float(r[8 * g + e]) * inv;
-              const int iv = isfinite(v) ? __float2int_rn(v) : 0;
-              q[e] = iv > 7 ? 7 : (iv < -7 ? -7 : iv);
-            }
-            w[g] = sm4_pack(q);
-          }
+          for (int g = 0; g < 4; ++g) w[g] = inv == 0.f ? 0u : sm4_quant8(r, 8 * g, inv);
           *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * K + c * 32) / 8) =
               make_uint4(w[0], w[1], w[2], w[3]);
         }
@@ -293,7 +314,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&bars->d_empty[sd]);
-      if (PASS == 0 && t < n) atomicMax(&amax_bits[t], __float_as_uint(m));
+      // a non-finite value makes the row's maximum the largest NaN pattern: its codes and step become 0
+      finite &= row_finite;
+      if (PASS == 0 && t < n) atomicMax(&amax_bits[t], row_finite ? __float_as_uint(m) : 0x7FFFFFFFu);
     }
     if (PASS == 0 && !finite) report(status, kStatusNonFinite);
   }
@@ -350,27 +373,6 @@ __device__ __forceinline__ void grid_barrier(uint32_t* ctr, uint32_t expected, v
   epi_bar();
 }
 
-// Four two's-complement bytes in [-7, 7] -> the SM4x8 sign-magnitude bytes (sign << 7 | magnitude).
-__device__ __forceinline__ uint32_t twos_to_sm(uint32_t w) {
-  const uint32_t s = (w >> 7) & 0x01010101u;        // 1 in every negative byte
-  const uint32_t m = (s << 8) - s;                   // 0xFF in every negative byte
-  return ((w ^ m) + s) | (s << 7);                   // |q| (no carry leaves a byte) and the sign bit
-}
-
-// One SM4x8 word of the codes rint(fl32(v_e * inv)), e = 0..7 (v_e = r[base + e] as float), for
-// |v_e * inv| <= 7 (inv = 7 / max|v|).  Adding 1.5 * 2^23 to the rounded product rounds it to an
-// integer (half to even, as rint) that sits, two's complement, in the low byte of the sum's bits;
-// the bytes are gathered four to a word and turned into sign-magnitude.  A non-finite product leaves
-// a garbage byte: callers zero the codes of rows whose maximum is not finite.
-__device__ __forceinline__ uint32_t sm4_quant8(const uint32_t (&r)[32], int base, float inv) {
-  constexpr float kMagic = 12582912.0f;
-  uint32_t b[8];
-#pragma unroll
-  for (int e = 0; e < 8; ++e) b[e] = __float_as_uint(__fadd_rn(__fmul_rn(__uint_as_float(r[base + e]), inv), kMagic));
-  const uint32_t lo = twos_to_sm(__byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410));
-  const uint32_t hi = twos_to_sm(__byte_perm(__byte_perm(b[4], b[5], 0x0040), __byte_perm(b[6], b[7], 0x0040), 0x5410));
-  return lo | __funnelshift_l(hi, hi, 4);
-}
 
 // Named barrier of the 12 warps that quantize (4 epilogue + 8 converter warps).
 __device__ __forceinline__ void quant_bar() { asm volatile("bar.sync 3, 384;" ::: "memory"); }

@@ -87,7 +87,9 @@ def _cat_T(rng, d, k):
 
 @pytest.mark.parametrize("n,d,k,dtype", [(130, 256, 32, "f32"), (67, 384, 128, "bf16"), (200, 512, 256, "bf16"),
                                          (5, 64, 16, "bf16"), (300, 1024, 64, "f32"), (300, 1024, 64, "bf16"),
-                                         (300, 640, 128, "bf16"), (1000, 256, 128, "bf16")])
+                                         (300, 640, 128, "bf16"), (1000, 256, 128, "bf16"),
+                                         # more than four 128-row units per CTA: the two-pass kernel
+                                         (2560, 4096, 128, "bf16"), (1300, 8192, 64, "bf16")])
 def test_transform_quantize_act(n, d, k, dtype):
     rng = np.random.default_rng(7 * n + d)
     X = rng.standard_normal((n, d)) * rng.lognormal(0, 1.0, d)
@@ -120,6 +122,34 @@ def test_nonfinite_activation_reports_numeric():
     assert sx[3].item() == 0.0
     assert sx[4].item() == pytest.approx(1.0 / 7.0, rel=1e-6)
     assert cat.cat_device_status()[0] == 0  # cleared
+
+
+def test_nonfinite_activation_two_pass():
+    """bf16 rows on the two-pass tensor-core kernel: a row holding inf or NaN gets step 0 and all
+    codes 0, the status reports it, and the other rows are unaffected."""
+    n, d, k = 2560, 4096, 128
+    rng = np.random.default_rng(11)
+    X = rng.standard_normal((n, d))
+    Xt = WL.cast(X, "bf16")
+    raw = Xt.raw.copy()
+    raw[5, 17] = 0x7F80                     # +inf
+    raw[900, 4000] = 0x7FC0                 # NaN
+    bad = WL.Tensor(values=WL.bf16_bits_to_f32(raw), raw=raw, dtype="bf16")
+    T32 = _cat_T(rng, d, k)
+    cat.cat_device_status()  # clear
+    xq, sx = cat.cat_transform_quantize_act(to_dev(bad), torch.from_numpy(T32).to(DEV), k)
+    st, word = cat.cat_device_status()
+    assert st == 4 and word & 2
+    q = sm4x8.unpack(xq.cpu().numpy())
+    sxg = sx.cpu().numpy()
+    for r in (5, 900):
+        assert sxg[r] == 0.0 and np.all(q[r] == 0)
+    good = np.ones(n, dtype=bool)
+    good[[5, 900]] = False
+    ref = O.transform_quantize_act(Xt.values[good], T32.astype(np.float64))
+    check_codes(q[good], ref.qx, ref.pre_x)
+    np.testing.assert_allclose(sxg[good].astype(np.float64), ref.sx, rtol=1e-5, atol=0)
+    assert cat.cat_device_status()[0] == 0
 
 
 # ------------------------------------------------------------------------------------------
