@@ -175,6 +175,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bars->d_full[s], 1);
       mbar_init(&bars->d_empty[s], 4);
     }
+    mbar_init(&bars->t_first, kCvtWarps);
     mbar_init(&bars->t_full, kCvtWarps);
     mbar_init(&bars->t_empty, 1);
     mbar_init(&bars->mma_done, 1);
@@ -197,6 +198,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int64_t u = u0; u < u1 && ok; ++u, ++j) {
         const int b = (int)(u / num_tiles), tile = (int)(u % num_tiles);
         const uint32_t s = j % kXStages;
+        // the first unit's x tile goes out with T_b's loads, the others once T_b is split (T_b would
+        // otherwise queue behind them in HBM)
+        if (j == 1 && !(ok = mbar_wait_bounded(&bars->t_first, 0, abort_flag, __LINE__))) break;
         if (j >= kXStages && !(ok = mbar_wait_bounded(&bars->x_empty[s], ((j / kXStages) - 1) & 1, abort_flag, __LINE__))) break;
         mbar_arrive_expect_tx(&bars->x_full[s], C::X_STAGE);
 #pragma unroll
@@ -260,7 +264,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       split_block<K>(A + (size_t)b * K * K, ts, ct);
       fence_proxy_async_smem();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->t_full);
+      if (lane == 0) {
+        mbar_arrive(&bars->t_full);
+        if (version == 0) mbar_arrive(&bars->t_first);
+      }
       ++version;
     }
   } else if (warp >= kEpiWarp0) {
