@@ -151,7 +151,10 @@ template <int K, int PASS>
 __global__ void __launch_bounds__(kThreads, 1)
     transform_quant_tc_kernel(const __grid_constant__ CUtensorMap tmX, const float* __restrict__ A, int n, int d,
                               uint32_t* __restrict__ amax_bits, uint32_t* __restrict__ codes,
+                              float* __restrict__ scale, uint32_t* __restrict__ exit_ctr,
                               uint32_t* __restrict__ status) {
+  // scale != nullptr (pass 1 with the maxima in a scratch slot): the CTAs holding block 0 write the
+  // steps s = max / 7, and the last CTA out zeroes the slot's maxima and its exit counter
   using C = TcCfg<K>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -289,6 +292,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float a = a_next;
         if (u + 1 < u1 && row_of(u + 1) < n) a_next = __uint_as_float(__ldcg(&amax_bits[row_of(u + 1)]));
         inv = (t < n && isfinite(a) && a > 0.f) ? __fdiv_rn(7.0f, a) : 0.f;
+        if (scale && b == 0 && t < n) {               // each row's one unit of block 0 writes its step
+          float sc = 0.f;
+          if (isfinite(a))
+            sc = __fdiv_rn(a, 7.0f);
+          else
+            report(status, kStatusNonFinite);
+          scale[t] = sc;
+        }
       }
       if (!(ok = mbar_wait_bounded(&bars->d_full[sd], (j >> 1) & 1, abort_flag, __LINE__))) break;
       __syncwarp();
@@ -329,6 +340,22 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   __syncthreads();
+  if (PASS == 1 && exit_ctr) {
+    // the last CTA out returns the slot to zero: every CTA has read its maxima before it counts out
+    __shared__ int last_out;
+    if (tid == 0) {
+      __threadfence();
+      last_out = atomicAdd(exit_ctr, 1u) == gridDim.x - 1;
+    }
+    __syncthreads();
+    if (last_out) {
+      __threadfence();
+      for (int t = tid; t < n; t += kThreads) amax_bits[t] = 0u;
+      __threadfence();
+      __syncthreads();
+      if (tid == 0) *exit_ctr = 0u;
+    }
+  }
   if (bars->abort && tid == 0) report(status, timeout_bits(kWhereTransform2Pass, bars->abort));
   if (warp == 0) {
     tc_fence_after();
@@ -667,9 +694,21 @@ int num_sms() {
   return sms;
 }
 
+uint32_t* sync_slots(cudaError_t* err, uint32_t** amax_slots);
+
+// Slots of the transform's device scratch, handed out round robin to every launch that uses one
+// (fused or two-pass), so that up to kSyncSlots such launches may be in flight at once.
+uint32_t next_tq_slot() {
+  static std::atomic<uint32_t> next{0};
+  return next.fetch_add(1) % kSyncSlots;
+}
+
+// scale != nullptr and n <= kAmaxRows: the maxima go to a slot of device scratch and pass 1 writes
+// the steps and returns the slot to zero (no memset, no finalize launch); cudaErrorNotSupported
+// otherwise, when the caller zeroes `amax` (its scale buffer) and finalizes the steps itself.
 template <int K>
 cudaError_t launch_k(const __nv_bfloat16* x, int64_t n, int64_t d, const float* A, uint32_t* amax, uint32_t* words,
-                     uint32_t* status, cudaStream_t stream) {
+                     float* scale, uint32_t* status, cudaStream_t stream) {
   using C = TcCfg<K>;
   EncodeTiledFn fn = encode_fn();
   if (!fn) return cudaErrorNotSupported;
@@ -694,12 +733,23 @@ cudaError_t launch_k(const __nv_bfloat16* x, int64_t n, int64_t d, const float* 
   if (attr != cudaSuccess) return attr;
   const int64_t units = (d / K) * ((n + TM - 1) / TM);
   const int grid = (int)(units < num_sms() ? units : num_sms());
+  uint32_t* exit_ctr = nullptr;
+  if (scale) {
+    if (n > kAmaxRows) return cudaErrorNotSupported;
+    cudaError_t es;
+    uint32_t* amax_slots = nullptr;
+    uint32_t* slots = sync_slots(&es, &amax_slots);
+    if (!slots) return es;
+    const uint32_t slot = next_tq_slot();
+    exit_ctr = slots + 4 * slot + 1;
+    amax = amax_slots + (size_t)kAmaxRows * slot;
+  }
   note_launch();
-  k0<<<grid, kThreads, C::SMEM, stream>>>(map, A, (int)n, (int)d, amax, words, status);
+  k0<<<grid, kThreads, C::SMEM, stream>>>(map, A, (int)n, (int)d, amax, words, nullptr, nullptr, status);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   note_launch();
-  k1<<<grid, kThreads, C::SMEM, stream>>>(map, A, (int)n, (int)d, amax, words, status);
+  k1<<<grid, kThreads, C::SMEM, stream>>>(map, A, (int)n, (int)d, amax, words, scale, exit_ctr, status);
   return cudaGetLastError();
 }
 
@@ -756,8 +806,7 @@ cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, const f
   uint32_t* amax_slots = nullptr;
   uint32_t* slots = sync_slots(&e, &amax_slots);
   if (!slots) return e;
-  static std::atomic<uint32_t> next_slot{0};
-  const uint32_t slot = next_slot.fetch_add(1) % kSyncSlots;
+  const uint32_t slot = next_tq_slot();
   uint32_t* sync = slots + 4 * slot;
   uint32_t* amax_bits = amax_slots + (size_t)kAmaxRows * slot;
   CUtensorMap map;
@@ -803,10 +852,10 @@ bool transform_quantize_tc_supported(int dtype, int k, int64_t n, int64_t d) {
 
 // Passes 0 and 1; the caller zeroes the scale buffer before and finalizes it after.
 cudaError_t launch_transform_quantize_tc(const void* x, int64_t n, int64_t d, int k, const float* A, uint32_t* amax,
-                                         uint32_t* words, uint32_t* status, cudaStream_t stream) {
+                                         uint32_t* words, float* scale, uint32_t* status, cudaStream_t stream) {
   const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
-  if (k == 64) return launch_k<64>(xb, n, d, A, amax, words, status, stream);
-  if (k == 128) return launch_k<128>(xb, n, d, A, amax, words, status, stream);
+  if (k == 64) return launch_k<64>(xb, n, d, A, amax, words, scale, status, stream);
+  if (k == 128) return launch_k<128>(xb, n, d, A, amax, words, scale, status, stream);
   return cudaErrorInvalidValue;
 }
 
