@@ -392,6 +392,20 @@ def test_concentration_bounds():
     assert abs(O.concentration_act(V * 7.5) - O.concentration_act(V)) < 1e-14
 
 
+def test_weight_concentration_closed_forms():
+    """Sec. 2, Lemma 3: C(W) = sum_o ||w_o||^2 / sum_o (2 max_i |w_oi|)^2 over output rows.  Rows
+    of equal magnitudes c in d entries give d c^2 / (4 c^2) = d / 4; one-hot rows give 1/4; a
+    mix weights each row by its squared range (a ratio of sums, not a mean of ratios)."""
+    d = 12
+    flat = np.where(np.arange(3 * d).reshape(3, d) % 2 == 0, 1.0, -1.0) * np.array([[0.5], [2.0], [3.0]])
+    assert O.concentration_weight(flat) == d / 4
+    onehot = np.zeros((4, d))
+    onehot[np.arange(4), [0, 3, 7, 11]] = [1.0, -2.0, 0.25, 9.0]
+    assert O.concentration_weight(onehot) == 0.25
+    mix = np.vstack([flat[:1], onehot[:1] * 0.5])   # ||.||^2 = 12 * 0.25 and 0.25; ranges 1 and 1
+    assert abs(O.concentration_weight(mix) - (3.0 + 0.25) / (1.0 + 1.0)) < 1e-15
+
+
 def test_lemmas_and_theorem1_on_gaussian_layer():
     """Lemma 1-3 / Theorem 1 are approximations; the paper reports them accurate between 5 and
     50 dB (Sec. 2).  On a Gaussian layer: within 0.2 dB at 8 bits, 1 dB at 4 bits, and about
