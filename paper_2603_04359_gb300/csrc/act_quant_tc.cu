@@ -513,9 +513,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int64_t u = u0; u < u1 && ok; ++u, ++j) {
         const int b = (int)(u / num_tiles), tile = (int)(u % num_tiles);
         const uint32_t st = j % kXStages;
-        // the first unit's x tile goes out with T_b's loads; the others wait until T_b is split, so
-        // that T_b does not queue behind them in HBM and unit 0's MMAs start as early as they can
-        if (j == 1 && !(ok = mbar_wait_bounded(&bars->t_first, 0, abort_flag, __LINE__))) break;
+        // the first two units' x tiles go out with T_b's loads; the others wait until T_b is split,
+        // so that T_b does not queue behind them in HBM and unit 0's MMAs start as early as they can
+        if (j == 2 && !(ok = mbar_wait_bounded(&bars->t_first, 0, abort_flag, __LINE__))) break;
         if (j >= kXStages && !(ok = mbar_wait_bounded(&bars->x_empty[st], ((j / kXStages) - 1) & 1, abort_flag, __LINE__))) break;
         mbar_arrive_expect_tx(&bars->x_full[st], C::X_STAGE);
 #pragma unroll
