@@ -327,7 +327,7 @@ def test_block_size_transform_sweep(k):
 # row statistics of x' = T x and W' = W T^{-1}
 # ------------------------------------------------------------------------------------------
 
-@pytest.mark.parametrize("cfg", [SMALL[0], SMALL[1], SMALL[2], SWEEP_LAYER], ids=lambda c: c.name)
+@pytest.mark.parametrize("cfg", SMALL + [SWEEP_LAYER], ids=lambda c: c.name)
 @pytest.mark.parametrize("kind", ["identity", "rht", "cat"])
 def test_layer_diagnostics(cfg, kind):
     """C(x') and C(W') (Lemmas 2 and 3), A(x', W') and the Theorem-1 SQNR from cat_block_row_stats
