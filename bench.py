@@ -298,14 +298,25 @@ class BufferSet:
                                                           self.sigma, self.xq, self.sx, self.y, self.out3))
 
 
+def diagnostics_from_sums(x3, w3, sum_y2, bits: int = 4):
+    """C(x'), C(W'), A and the Theorem-1 SQNR prediction (Sec. 2, Lemmas 2-3, Theorem 1), in dB, from
+    the row-statistics sums of cat_block_row_stats for x' (x3) and W' (w3) and sum y^2 over the
+    outputs: C = sum ||v||^2 / sum r^2, A = sum y^2 / (sum ||w'||^2 sum ||x'||^2), and
+    SQNR ~ 12 (N^2 C(x') || N^2 C(W')) A with N = 2 (2^(b-1) - 1) intervals."""
+    n2 = float((2 * (2 ** (bits - 1) - 1)) ** 2)
+    c_x, c_w = float(x3[0]) / float(x3[1]), float(w3[0]) / float(w3[1])
+    a = float(sum_y2) / (float(w3[0]) * float(x3[0]))
+    pred = 12.0 * a / (1.0 / (n2 * c_x) + 1.0 / (n2 * c_w))
+    db = lambda v: 10.0 * float(np.log10(v))
+    return {"C_x_db": db(c_x), "C_w_db": db(c_w), "A_db": db(a), "theorem1_db": db(pred)}
+
+
 def transform_sweep(cat, L, x, W, xc, y_ref):
     """SQNR (dB) of the library's W4A4 output against y = W x in fp32, over all n x d_out outputs,
     for every block size in SWEEP_K and every transform kind (Sec. 4: identity, the block
     randomized Hadamard rotation, CAT), each prepared from the same calibration split."""
     out = {"k": list(SWEEP_K)}
     diag = {}
-    n2 = float((2 * (2 ** 3 - 1)) ** 2)           # 14 intervals of the restricted INT4 grid, squared
-    db = lambda v: round(10.0 * float(np.log10(v)), 3)
     for kind in ("identity", "rht", "cat"):
         vals = []
         dk = {"C_x_db": [], "C_w_db": [], "A_db": [], "theorem1_db": []}
@@ -321,13 +332,9 @@ def transform_sweep(cat, L, x, W, xc, y_ref):
             Tinv = torch.linalg.inv(T.double()).float().contiguous()
             _, _, x3 = cat.cat_block_row_stats(x, k, T)
             _, _, w3 = cat.cat_block_row_stats(W, k, Tinv, transpose=True)
-            sx2, rx2 = float(x3[0].item()), float(x3[1].item())
-            sw2, rw2 = float(w3[0].item()), float(w3[1].item())
-            c_x, c_w, a = sx2 / rx2, sw2 / rw2, float(out3[0].item()) / (sw2 * sx2)
-            dk["C_x_db"].append(db(c_x))
-            dk["C_w_db"].append(db(c_w))
-            dk["A_db"].append(db(a))
-            dk["theorem1_db"].append(db(12.0 * a / (1.0 / (n2 * c_x) + 1.0 / (n2 * c_w))))
+            dg = diagnostics_from_sums(x3.cpu().numpy(), w3.cpu().numpy(), float(out3[0].item()))
+            for key in dk:
+                dk[key].append(round(dg[key], 3))
             del T, Wq, sw, xq, sx, Tinv
         out[kind] = vals
         diag[kind] = dk

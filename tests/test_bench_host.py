@@ -76,3 +76,23 @@ def test_reference_arm_under_torchrun_prints_once_from_rank0():
     assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["value"] > 0
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["value"] == d["value"]
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["d2h_bytes_per_step"] == 0
+
+
+def test_diagnostics_from_sums_matches_the_oracle():
+    """The bench's concentration / alignment / Theorem-1 arithmetic on row-statistics sums (the
+    quantities cat_block_row_stats returns) equals the oracle's analysis functions."""
+    import numpy as np
+
+    import bench
+    import oracle as O
+    rng = np.random.default_rng(3)
+    X = rng.standard_normal((40, 24)) * rng.lognormal(0, 1, 24)
+    W = rng.standard_normal((30, 24)) * 0.1
+    x3 = [float(np.sum(X * X)), float(np.sum((2 * np.abs(X).max(axis=1)) ** 2))]
+    w3 = [float(np.sum(W * W)), float(np.sum((2 * np.abs(W).max(axis=1)) ** 2))]
+    y = X @ W.T
+    dg = bench.diagnostics_from_sums(x3, w3, float(np.sum(y * y)))
+    assert abs(dg["C_x_db"] - O.db(O.concentration_act(X))) < 1e-9
+    assert abs(dg["C_w_db"] - O.db(O.concentration_weight(W))) < 1e-9
+    assert abs(dg["A_db"] - O.db(O.alignment(X, W))) < 1e-9
+    assert abs(dg["theorem1_db"] - O.db(O.theorem1_sqnr(X, W))) < 1e-9
