@@ -322,8 +322,15 @@ def transform_sweep(cat, L, x, W, xc, y_ref):
         dk = {"C_x_db": [], "C_w_db": [], "A_db": [], "theorem1_db": []}
         for k in SWEEP_K:
             sigma = cat.cat_calib_cov(xc, k) if kind == "cat" else None
-            T, Wq, sw = cat.cat_quantize_weights(W, k, kind, sigma_x=sigma, n_calib=L.cfg.n_calib,
-                                                 rht_signs=L.rht_signs if kind == "rht" else None)
+            try:
+                T, Wq, sw = cat.cat_quantize_weights(W, k, kind, sigma_x=sigma, n_calib=L.cfg.n_calib,
+                                                     rht_signs=L.rht_signs if kind == "rht" else None)
+            except cat.CatError as err:           # e.g. fewer calibration tokens than k: singular Sigma_x blocks
+                vals.append(None)
+                for key in dk:
+                    dk[key].append(None)
+                out.setdefault("skipped", []).append(f"{kind} k={k}: {err}")
+                continue
             xq, sx = cat.cat_transform_quantize_act(x, T, k)
             _, out3 = cat.cat_w4a4_linear_sqnr(xq, sx, Wq, sw, y_ref)
             vals.append(round(float(out3[2].item()), 3))
