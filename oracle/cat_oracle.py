@@ -48,25 +48,23 @@ def quantize_rows_symmetric(V: np.ndarray, bits: int = 4):
     """Quantize every row of ``V`` on its own symmetric uniform grid.
 
     Returns ``(q, s, pre)``: integer codes (int64), the per-row step ``s = max|v| / qmax`` and
-    the exact pre-rounding values ``v / s`` (float64).  An all-zero row gets ``s = 0`` and codes 0.
+    the pre-rounding values ``v / s = qmax * v / max|v|`` (float64).  An all-zero row gets
+    ``s = 0`` and codes 0.
 
-    The paper does not fix the precision in which a value is rounded to its code.  The code is
-    decided in float32, the precision of the kernels: ``rint(f32(v) * f32(qmax / f32(max|v|)))``
-    with IEEE round-to-nearest operations and ties to even.  Deciding in the same precision on
-    both sides matters for inputs on a coarse grid (bf16 weights with T = I), where many values
-    sit exactly on a rounding boundary and float64 would break those ties by its own rounding."""
+    The code is ``clamp(round_half_even(qmax * v / max|v|), -qmax, qmax)``, evaluated in float64
+    as ``(qmax * v) / max|v|``.  For values with at most 24 significant bits (bf16 or fp32 inputs,
+    e.g. weights or activations under T = I) the product is exact and the quotient correctly
+    rounded, so a real tie (a quotient of exactly m + 1/2) stays an exact tie and is broken to
+    even, and every other quotient lies at least 2^-29 away from a tie, far beyond float64's
+    rounding; the code is then the exact round-to-nearest of the definition."""
     V = np.asarray(V, dtype=np.float64)
     qmax = 2 ** (bits - 1) - 1
     a = np.max(np.abs(V), axis=1) if V.shape[1] else np.zeros(V.shape[0])
     s = a / qmax
     pre = np.zeros_like(V)
-    nz = s > 0
-    pre[nz] = V[nz] / s[nz, None]
-    a32 = a.astype(np.float32)
-    inv32 = np.zeros_like(a32)
-    inv32[nz] = np.float32(qmax) / a32[nz]
-    pre32 = V.astype(np.float32) * inv32[:, None]
-    q = np.clip(np.rint(pre32), -qmax, qmax).astype(np.int64)
+    nz = a > 0
+    pre[nz] = (qmax * V[nz]) / a[nz, None]
+    q = np.clip(np.rint(pre), -qmax, qmax).astype(np.int64)
     return q, s, pre
 
 

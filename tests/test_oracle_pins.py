@@ -2,6 +2,8 @@
 routines and brute force.  None of them reuses the oracle's own formula to check itself."""
 import os
 
+from fractions import Fraction
+
 import numpy as np
 import pytest
 import scipy.linalg
@@ -38,17 +40,33 @@ def _read_quant_golden():
             if not line or line.startswith("#"):
                 continue
             row, s, codes = [p.strip() for p in line.split("|")]
-            cases.append((np.array([float(v) for v in row.split()]), float(s),
+            # a step written as a fraction "a/7" is compared with its correctly rounded float64 value
+            num, _, den = s.partition("/")
+            s_val = float(Fraction(num) / Fraction(den or "1"))
+            cases.append((np.array([float(v) for v in row.split()]), s_val,
                           np.array([int(v) for v in codes.split()])))
     return cases
 
 
-@pytest.mark.parametrize("case", range(5))
+@pytest.mark.parametrize("case", range(8))
 def test_quantizer_hand_worked_rows(case):
     row, s_exp, q_exp = _read_quant_golden()[case]
     q, s, pre = O.quantize_rows_symmetric(row[None, :])
     assert s[0] == s_exp
     np.testing.assert_array_equal(q[0], q_exp)
+
+
+def test_quantizer_golden_covers_ties_that_float32_breaks_the_wrong_way():
+    """The tie rows are chosen so that deciding the code as rint(f32(v) * f32(7 / a)) gives a
+    different code than the definition: the fixture can tell the two apart."""
+    diff = 0
+    for row, _, q_exp in _read_quant_golden():
+        a = np.float32(np.max(np.abs(row)))
+        if a == 0:
+            continue
+        q32 = np.rint(row.astype(np.float32) * (np.float32(7) / a)).astype(np.int64)
+        diff += int(np.sum(q32 != q_exp))
+    assert diff >= 3
 
 
 def test_quantizer_ranges_and_error_bound():
@@ -66,10 +84,10 @@ def test_quantizer_ranges_and_error_bound():
     assert s[3] == 0 and np.all(q[3] == 0)
     # |v - s q| <= s / 2 (no clipping: the range covers the row)
     err = np.abs(V - q * s[:, None])
-    assert np.all(err <= s[:, None] / 2 * (1 + 1e-6) + 1e-300)  # float32 code decision
-    # away from rounding boundaries the code is the float64 round-to-nearest of v / s
-    far = np.abs(np.abs(pre) - np.floor(np.abs(pre)) - 0.5) > 1e-5
-    np.testing.assert_array_equal(q[far], np.rint(pre[far]))
+    assert np.all(err <= s[:, None] / 2 * (1 + 1e-12) + 1e-300)
+    # away from rounding boundaries the code is the round-to-nearest of v / s
+    far = (np.abs(np.abs(pre) - np.floor(np.abs(pre)) - 0.5) > 1e-9) & (s[:, None] > 0)
+    np.testing.assert_array_equal(q[far], np.rint(V[far] / np.repeat(s[:, None], V.shape[1], 1)[far]))
     # step size is max|v| / 7 exactly
     np.testing.assert_array_equal(s, np.max(np.abs(V), axis=1) / 7)
 
