@@ -41,7 +41,10 @@ import torch  # noqa: E402
 import workloads as WL  # noqa: E402
 
 METRIC = "CAT W4A4 linear tokens/s & effective TOPS, % of int8/HBM roofline; SQNR dB"
-DEFAULT_CONFIG = "c2_qkv_4096x6144_k128_bf16"
+DEFAULT_CONFIG = "c5_gateup_8192x28672_bf16"     # the largest configuration that fits one GPU
+# measured in the same run and reported under "secondary": the prefill QKV layer (tensor roofline)
+# and the decode layer (HBM roofline of the weight stream)
+SECONDARY = ("c2_qkv_4096x6144_k128_bf16", "c4_decode_up_4096x14336_k128_bf16")
 FP8_PER_BF16 = 2.0          # nominal dense FP8 / BF16 tensor throughput ratio (4.5 / 2.25 PFLOP/s)
 FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}
 DECODE_TOKENS = 32          # cat_w4a4_linear streams the weights (HBM-bound) up to this many tokens
@@ -59,6 +62,7 @@ def parse_args():
     p.add_argument("--k", type=int, default=0, help="block size (default: the config's)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-secondary", action="store_true", help="skip the secondary configurations")
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="budget of the CPU-baseline sample")
     p.add_argument("--sweep", action="store_true",
                    help="also report the layer's SQNR for every block size in SWEEP_K and every transform "
@@ -193,27 +197,6 @@ class OracleRunner:
         ac = O.transform_quantize_act(self.X, self.prep.T)
         _, y_hat = O.w4a4_linear(ac.qx, ac.sx, self.prep.qw, self.prep.sw)
         return O.sqnr_sums(self.y_ref, y_hat)
-
-
-def int8_peak_tops(dev, size=8192, reps=5):
-    """The int8 tensor-core peak of this GPU, measured with cuBLAS (outside any timed region)."""
-    try:
-        g = torch.Generator(device=dev).manual_seed(0)
-        a = torch.randint(-8, 8, (size, size), dtype=torch.int8, device=dev, generator=g)
-        b = torch.randint(-8, 8, (size, size), dtype=torch.int8, device=dev, generator=g)
-        for _ in range(2):
-            torch._int_mm(a, b)
-        best = float("inf")
-        for _ in range(reps):
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record()
-            torch._int_mm(a, b)
-            e1.record()
-            torch.cuda.synchronize()
-            best = min(best, e0.elapsed_time(e1))
-        return 2.0 * size ** 3 / (best / 1e3) / 1e12
-    except Exception:
-        return None
 
 
 def cpu_cores():
@@ -357,35 +340,32 @@ class DeviceTimeout(RuntimeError):
     16..31 the source line of the first wait that gave up)."""
 
 
-def ours_arm(args, rank, world, local, retried=None):
-    import paper_2603_04359_gb300 as cat
-    cat.load_library()
-    dev = torch.device("cuda", local)
-    torch.cuda.set_device(dev)
-    cfg = WL.CONFIGS[args.config]
-    k = args.k or cfg.k
+def measure_config(cat, cfg, k, kind, args, dev, world, rank, with_e2e, sweep=False):
+    """Prepare one layer, time its step (CUDA graph of `steps` steps over an L2-exceeding operand
+    rotation), each call alone, and optionally the host-buffer e2e path.  Returns the raw numbers."""
     L = WL.make_layer(cfg)
     x, W, xc = to_dev(L.x_eval, dev), to_dev(L.W, dev), to_dev(L.x_calib, dev)
     n, d_in, d_out = cfg.n_eval, cfg.d_in, cfg.d_out
 
     # offline: calibration statistics and weight preparation
     sigma = cat.cat_calib_cov(xc, k)
-    T, Wq, sw = cat.cat_quantize_weights(W, k, args.kind, sigma_x=sigma, n_calib=cfg.n_calib,
-                                         rht_signs=L.rht_signs if args.kind == "rht" else None)
+    T, Wq, sw = cat.cat_quantize_weights(W, k, kind, sigma_x=sigma, n_calib=cfg.n_calib,
+                                         rht_signs=L.rht_signs if kind == "rht" else None)
     torch.backends.cuda.matmul.allow_tf32 = False
     y_ref = (x.float() @ W.float().t()).contiguous()
-    sweep = transform_sweep(cat, L, x, W, xc, y_ref) if args.sweep and rank == 0 else None
+    sweep_res = transform_sweep(cat, L, x, W, xc, y_ref) if sweep else None
     del W
     l2 = torch.cuda.get_device_properties(dev).L2_cache_size
     first = BufferSet(cat, x, xc, y_ref, T, Wq, sw, k, dev)
     n_sets = max(2, -(-3 * l2 // first.nbytes()))         # >= 3x L2 of operands in rotation
     sets = [first] + [BufferSet(cat, x, xc, y_ref, T, Wq, sw, k, dev) for _ in range(n_sets - 1)]
+    del x, xc, y_ref, T, Wq, sw, sigma
     stream = torch.cuda.current_stream(dev)
 
     calls = {
         "cat_calib_cov": lambda b: cat.cat_calib_cov(b.xc, k, out=b.sigma),
         "cat_transform_quantize_act": lambda b: cat.cat_transform_quantize_act(b.x, b.T, k, xq=b.xq, x_scale=b.sx),
-        # the integer GEMM, dequantization and SQNR sums (fused in the GEMM epilogue for n > 32)
+        # the integer GEMM, dequantization and SQNR sums (fused in the GEMM epilogue)
         "cat_w4a4_linear_sqnr": lambda b: cat.cat_w4a4_linear_sqnr(b.xq, b.sx, b.Wq, b.sw, b.y_ref, y=b.y, out=b.out3),
     }
 
@@ -422,7 +402,7 @@ def ours_arm(args, rank, world, local, retried=None):
 
     barrier(world)
     torch.cuda.synchronize()
-    clocks = ClockSampler(local)
+    clocks = ClockSampler(dev.index)
     t_heat = time.perf_counter()
     while time.perf_counter() - t_heat < 0.3:               # untimed replays: the clock sampler sees the load
         g_step.replay()
@@ -434,8 +414,7 @@ def ours_arm(args, rank, world, local, retried=None):
     torch.cuda.synchronize()
     clk = clocks.stop()
     barrier(world)
-    step_ms = e0.elapsed_time(e1) / args.steps
-    step_ms_max = max_over_ranks(step_ms, world)
+    step_ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
     call_ms = {}
     for name, g in g_calls.items():                         # each call alone, same rotation, same count
         g.replay()
@@ -445,8 +424,6 @@ def ours_arm(args, rank, world, local, retried=None):
         b.record(stream)
         torch.cuda.synchronize()
         call_ms[name] = a.elapsed_time(b) / args.steps
-    decode = n <= DECODE_TOKENS
-    gemm_ms = call_ms["cat_w4a4_linear (alone)" if decode else "cat_w4a4_linear_sqnr"]
     sqnr_db = float(sets[(args.steps - 1) % n_sets].out3[2].item())
 
     # end to end through the public API with host buffers: every step copies its inputs in from pinned
@@ -455,7 +432,7 @@ def ours_arm(args, rank, world, local, retried=None):
     # i + 1's inputs stream in and step i - 1's outputs stream out while step i computes; events keep
     # each operand set's copies, compute and read-back in order.
     e2e = None
-    if not args.no_e2e:
+    if with_e2e:
         b0 = sets[0]
         x_h = b0.x.cpu().pin_memory()
         xc_h = b0.xc.cpu().pin_memory()
@@ -512,13 +489,27 @@ def ours_arm(args, rank, world, local, retried=None):
         e2e = {"value": world * n / (e2e_ms / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms,
                "overlap": "inputs in, compute, outputs out on three streams (pipelined across steps)"}
+        del x_h, xc_h, yref_h, y_h, o3_h
 
     st, word = cat.cat_device_status(dev)
     if st != 0:
         raise (DeviceTimeout if word & 1 else RuntimeError)(f"device status {st} ({word:#x}) after timing")
+    res = dict(L=L, n=n, d_in=d_in, d_out=d_out, step_ms=step_ms, call_ms=call_ms, launches=int(launches),
+               sqnr_db=sqnr_db, n_sets=n_sets, set_bytes=first.nbytes(), l2=l2, clocks=clk, e2e=e2e,
+               sweep=sweep_res)
+    del sets, first, g_step, g_calls
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    return res
 
-    if rank != 0:
-        return
+
+def roofline_of(cfg, res, steps):
+    """Roofline of the dominant kernel: the prefill GEMM against the FP8 tensor peak, or the decode
+    GEMM's weight stream against HBM."""
+    n, d_in, d_out = res["n"], res["d_in"], res["d_out"]
+    decode = n <= DECODE_TOKENS
+    call_ms = res["call_ms"]
+    gemm_ms = call_ms["cat_w4a4_linear (alone)" if decode else "cat_w4a4_linear_sqnr"]
     peaks = measured_peaks()
     fp8_peak = peaks["bf16_tflops"] * FP8_PER_BF16
     gemm_tflops = 2.0 * n * d_in * d_out / (gemm_ms / 1e3) / 1e12
@@ -528,51 +519,84 @@ def ours_arm(args, rank, world, local, retried=None):
     rec = tr.get(cfg.name, {})
     if rec.get("source_sha1") == source_sha1(kernel_src):     # counters of this very kernel source
         traffic = rec.get("dram_bytes_per_launch")
-    timing = (f"CUDA events around one replay of a CUDA graph of the {args.steps} launches, operand copies "
-              f"rotated over {n_sets} sets ({n_sets * first.nbytes() / 2**20:.0f} MiB > L2)")
+    timing = (f"CUDA events around one replay of a CUDA graph of the {steps} launches, operand copies "
+              f"rotated over {res['n_sets']} sets ({res['n_sets'] * res['set_bytes'] / 2**20:.0f} MiB > L2)")
     if decode:
         # weight stream: packed W + w scales + packed x + x scales + y, once each
         gemm_bytes = d_in * d_out // 2 + 4 * d_out + n * d_in // 2 + 4 * n + 4 * n * d_out
         gbs = gemm_bytes / (gemm_ms / 1e3) / 1e9
-        roofline = {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                    "frac": gbs / peaks["hbm_gbs"], "traffic": traffic, "algorithmic_bytes": gemm_bytes,
-                    "kernel": "w4a4_gemm_decode_tc (cat_w4a4_linear_sqnr, n <= 32)", "timing": timing,
-                    "peak_source": f"{peaks['source']} HBM copy {peaks['hbm_gbs']} GB/s"}
+        roof = {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": gbs / peaks["hbm_gbs"], "traffic": traffic, "algorithmic_bytes": gemm_bytes,
+                "kernel": "w4a4_gemm_decode_tc (cat_w4a4_linear, n <= 32)", "timing": timing,
+                "peak_source": f"{peaks['source']} HBM copy {peaks['hbm_gbs']} GB/s"}
     else:
-        roofline = {"bound": "tensor", "achieved": gemm_tflops, "peak": fp8_peak, "unit": "TFLOP/s",
-                    "frac": gemm_tflops / fp8_peak, "traffic": traffic,
-                    "kernel": "w4a4_gemm_tc (cat_w4a4_linear_sqnr, SQNR sums in the epilogue)", "timing": timing,
-                    "peak_source": f"{peaks['source']} bf16 {peaks['bf16_tflops']} TFLOP/s x {FP8_PER_BF16} "
-                                   "(FP8 engine, nominal FP8/BF16 ratio)"}
+        roof = {"bound": "tensor", "achieved": gemm_tflops, "peak": fp8_peak, "unit": "TFLOP/s",
+                "frac": gemm_tflops / fp8_peak, "traffic": traffic,
+                "algorithmic_ops": 2 * n * d_in * d_out,
+                "kernel": "w4a4_gemm_tc (cat_w4a4_linear_sqnr, SQNR sums in the epilogue)", "timing": timing,
+                "peak_source": f"{peaks['source']} bf16 {peaks['bf16_tflops']} TFLOP/s x {FP8_PER_BF16} "
+                               "(the FP8 engine the GEMM runs on, nominal FP8/BF16 ratio)",
+                "peak_note": "sm_103a has no integer tcgen05 MMA: INT4 codes run exactly as E4M3 operands on the "
+                             "FP8 engine. Beside it: an own kind::f8f6f4 SS-MMA loop reached 4847 TFLOP/s and "
+                             "cuBLAS FP8 8192^3 3344 TFLOP/s on this GPU type; the legacy int8 mma.sync pipe "
+                             "~150 TOP/s"}
+    return roof, gemm_ms, gemm_tflops
+
+
+def ours_arm(args, rank, world, local, retried=None):
+    import paper_2603_04359_gb300 as cat
+    cat.load_library()
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    cfg = WL.CONFIGS[args.config]
+    k = args.k or cfg.k
+    res = measure_config(cat, cfg, k, args.kind, args, dev, world, rank, with_e2e=not args.no_e2e,
+                         sweep=args.sweep and rank == 0)
+    secondary = {}
+    if world == 1 and not args.no_secondary:
+        for name in SECONDARY:
+            if name == cfg.name:
+                continue
+            c2 = WL.CONFIGS[name]
+            r2 = measure_config(cat, c2, c2.k, "cat", args, dev, world, rank, with_e2e=False)
+            roof2, gemm_ms2, tops2 = roofline_of(c2, r2, args.steps)
+            secondary[name] = {
+                "value": r2["n"] / (r2["step_ms"] / 1e3), "unit": "tokens/s", "ms_per_step": r2["step_ms"],
+                "config": {"n_tokens": r2["n"], "d_in": r2["d_in"], "d_out": r2["d_out"], "k": c2.k,
+                           "n_calib": c2.n_calib, "transform": "cat", "input_dtype": c2.dtype,
+                           "l2": f"inputs larger than L2: {r2['n_sets']} operand sets in rotation"},
+                "roofline": roof2, "sqnr_db": r2["sqnr_db"], "gemm_ms": gemm_ms2, "effective_tops": tops2,
+                "call_ms": r2["call_ms"], "gpu_launches": r2["launches"], "clocks": r2["clocks"]}
+    if rank != 0:
+        return
+    roofline, gemm_ms, gemm_tflops = roofline_of(cfg, res, args.steps)
+    n, d_in, d_out = res["n"], res["d_in"], res["d_out"]
     line = {
-        "metric": METRIC, "value": world * n / (step_ms_max / 1e3), "unit": "tokens/s", "n_gpus": world,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms_max, "higher_is_better": True,
+        "metric": METRIC, "value": world * n / (res["step_ms"] / 1e3), "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": res["step_ms"], "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "int4", "data": "synthetic",
         "config": {"workload": cfg.name, "n_tokens": n, "d_in": d_in, "d_out": d_out, "k": k, "n_calib": cfg.n_calib,
                    "transform": args.kind, "input_dtype": cfg.dtype, "parallelism": f"replicas x{world}",
-                   "l2": f"inputs larger than L2: {n_sets} operand sets in rotation "
-                         f"({n_sets * first.nbytes() / 2**20:.0f} MiB, L2 {l2 / 2**20:.0f} MiB)",
+                   "l2": f"inputs larger than L2: {res['n_sets']} operand sets in rotation "
+                         f"({res['n_sets'] * res['set_bytes'] / 2**20:.0f} MiB, L2 {res['l2'] / 2**20:.0f} MiB)",
                    "timing": "device: CUDA graph of the timed steps replayed once between CUDA events; "
                              "e2e: host-issued calls"},
         "roofline": roofline,
-        "sqnr_db": sqnr_db, "gemm_ms": gemm_ms, "effective_tops": gemm_tflops, "call_ms": call_ms,
-        "gpu_launches": int(launches), "clocks": clk,
+        "sqnr_db": res["sqnr_db"], "gemm_ms": gemm_ms, "effective_tops": gemm_tflops, "call_ms": res["call_ms"],
+        "gpu_launches": res["launches"], "clocks": res["clocks"],
     }
-    if not decode:
-        i8 = int8_peak_tops(dev)
-        if i8:
-            line["int8_peak"] = {"tops": i8, "frac": gemm_tflops / i8,
-                                 "source": "measured now: torch._int_mm int8 8192^3, best of 5 (cuBLAS IMMA)"}
-    if e2e:
-        line["e2e"] = e2e
+    if res["e2e"]:
+        line["e2e"] = res["e2e"]
+    if secondary:
+        line["secondary"] = secondary
     if retried:
         line["retried_after"] = retried
-    if sweep:
-        line["sqnr_sweep"] = dict(sweep, unit="dB", over="all n x d_out outputs, y = W x in fp32 as reference",
+    if res["sweep"]:
+        line["sqnr_sweep"] = dict(res["sweep"], unit="dB", over="all n x d_out outputs, y = W x in fp32 as reference",
                                   diagnostics_note="per transform and k: concentrations C(x'), C(W'), alignment A "
                                                    "and the Theorem-1 SQNR prediction (N = 14 intervals), in dB")
     if world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = run_cpu_baseline(L, args.kind, k, args.cpu_seconds)
+        line["cpu_baseline"] = run_cpu_baseline(res["L"], args.kind, k, args.cpu_seconds)
     print(json.dumps(line), flush=True)
 
 

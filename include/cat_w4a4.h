@@ -26,7 +26,9 @@
  *  - Shapes: d_in % 32 == 0 (a packed row is a whole number of 16-byte chunks); k is one of
  *    16, 32, 64, 128, 256 and divides d_in; n, d_out >= 1 (n == 0 is accepted and does nothing).
  *  - Thread safety: calls keep no host state between calls except the error message of the
- *    calling thread.
+ *    calling thread and, per device, the cached device addresses of the library's static device
+ *    scratch (looked up once under a lock).  Exception: cat_quantize_weights_noalloc uses one
+ *    shared device scratch area per device, so its calls must be serialized by the caller.
  *
  * INT4 code format ("SM4x8")
  * --------------------------
@@ -134,7 +136,12 @@ cat_status cat_quantize_weights(const void* W, cat_dtype dtype, int64_t d_out, i
  *   Limit: d_in * k <= CAT_PREP_NOALLOC_MAX_DK; a larger call returns CAT_ERR_SHAPE before any
  *   CUDA call and writes nothing.
  *   Setup: the first call on a device looks up the scratch address (cudaGetSymbolAddress) with
- *   that device current; make that first call before any stream capture.
+ *   that device current; make that first call before any stream capture.  Under CUDA's default
+ *   lazy module loading (CUDA_MODULE_LOADING=LAZY) the 12 MiB array and the kernels this call
+ *   launches are only loaded onto the device by that first call (or by the first use of another
+ *   entry point in the same module), and loading them takes device memory.  A caller that will
+ *   later hand all free device memory to its own pool must therefore make one call (any valid
+ *   size) before reserving it; later calls then take no device memory at all.
  *   Concurrency: every call on a device shares the one scratch area, so calls that overlap in
  *   time (other host threads or streams) race; the caller must serialize them.  Each call
  *   synchronizes its stream before returning, so consecutive calls are safe.
@@ -164,7 +171,8 @@ cat_status cat_build_transform_host(cat_tkind kind, int64_t d_in, int32_t k, con
  *   T_blocks device [d_in/k][k][k] float32 (from cat_quantize_weights).
  *   xq       out, device [n][d_in/2] bytes: SM4x8 codes of x' = T x.
  *   x_scale  out, device [n] float32: per-token step s_x = max_i |x'_i| / 7 (0 for an all-zero token).
- * Codes are q = clamp(rint(x'_i * (7 / max|x'|)), -7, 7), x' accumulated in float32.
+ * Codes are q = clamp(round_half_even(7 x'_i / max|x'|), -7, 7), x' accumulated in float32; the
+ * rounding decision is exact for the float32 x' (ties included), not a float32 approximation of it.
  */
 cat_status cat_transform_quantize_act(const void* x, cat_dtype dtype, int64_t n, int64_t d_in, int32_t k,
                                       const float* T_blocks, uint8_t* xq, float* x_scale,

@@ -109,6 +109,21 @@ def _need(t: torch.Tensor, name: str) -> None:
         raise ValueError(f"{name} must be a contiguous CUDA tensor")
 
 
+def _expect(t: torch.Tensor, name: str, dtype: torch.dtype, shape: tuple, device: torch.device) -> None:
+    """Check a tensor handed to the library (an input it reads or an output it writes): contiguous,
+    on ``device``, of the given dtype and shape.  The library trusts sizes, so a wrong buffer would
+    be read or written past its end; this raises ValueError before any call."""
+    if not isinstance(t, torch.Tensor):
+        raise ValueError(f"{name} must be a torch tensor")
+    _need(t, name)
+    if t.device != device:
+        raise ValueError(f"{name} is on {t.device}, expected {device}")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} has dtype {t.dtype}, expected {dtype}")
+    if tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {tuple(shape)}")
+
+
 def cat_version() -> int:
     return int(load_library().cat_version())
 
@@ -124,6 +139,7 @@ def cat_calib_cov(x: torch.Tensor, k: int, out: Optional[torch.Tensor] = None, a
     n, d = x.shape
     if out is None:
         out = torch.empty((d // k, k, k), dtype=torch.float64, device=x.device)
+    _expect(out, "out", torch.float64, (d // k, k, k), x.device)
     _check("cat_calib_cov", load_library().cat_calib_cov(_ptr(x), _dtype(x), n, d, k, _ptr(out), int(accumulate),
                                                          _stream(x.device)))
     return out
@@ -143,7 +159,9 @@ def cat_quantize_weights(W: torch.Tensor, k: int, kind: str, sigma_x: Optional[t
     if rht_signs is not None:
         signs = np.ascontiguousarray(np.asarray(rht_signs, dtype=np.float32))
     if sigma_x is not None:
-        _need(sigma_x, "sigma_x")
+        _expect(sigma_x, "sigma_x", torch.float64, (d_in // k, k, k), dev)
+    if signs is not None and signs.shape != (d_in,):
+        raise ValueError(f"rht_signs has shape {signs.shape}, expected ({d_in},)")
     st = load_library().cat_quantize_weights(
         _ptr(W), _dtype(W), d_out, d_in, k, KIND[kind], _ptr(sigma_x), int(n_calib),
         None if signs is None else signs.ctypes.data_as(ctypes.c_void_p), _ptr(T), _ptr(Wq), _ptr(sw), _stream(dev))
@@ -163,11 +181,16 @@ def cat_quantize_weights_noalloc(W: torch.Tensor, k: int, kind: str, sigma_x: Op
                torch.empty((d_out, d_in // 2), dtype=torch.uint8, device=dev),
                torch.empty((d_out,), dtype=torch.float32, device=dev))
     T, Wq, sw = out
+    _expect(T, "out[0] (T_blocks)", torch.float32, (d_in // k, k, k), dev)
+    _expect(Wq, "out[1] (Wq)", torch.uint8, (d_out, d_in // 2), dev)
+    _expect(sw, "out[2] (w_scale)", torch.float32, (d_out,), dev)
     signs = None
     if rht_signs is not None:
         signs = np.ascontiguousarray(np.asarray(rht_signs, dtype=np.float32))
+        if signs.shape != (d_in,):
+            raise ValueError(f"rht_signs has shape {signs.shape}, expected ({d_in},)")
     if sigma_x is not None:
-        _need(sigma_x, "sigma_x")
+        _expect(sigma_x, "sigma_x", torch.float64, (d_in // k, k, k), dev)
     st = load_library().cat_quantize_weights_noalloc(
         _ptr(W), _dtype(W), d_out, d_in, k, KIND[kind], _ptr(sigma_x), int(n_calib),
         None if signs is None else signs.ctypes.data_as(ctypes.c_void_p), _ptr(T), _ptr(Wq), _ptr(sw), _stream(dev))
@@ -201,9 +224,23 @@ def cat_transform_quantize_act(x: torch.Tensor, T_blocks: torch.Tensor, k: int, 
         xq = torch.empty((n, d_in // 2), dtype=torch.uint8, device=x.device)
     if x_scale is None:
         x_scale = torch.empty((n,), dtype=torch.float32, device=x.device)
+    _expect(T_blocks, "T_blocks", torch.float32, (d_in // k, k, k), x.device)
+    _expect(xq, "xq", torch.uint8, (n, d_in // 2), x.device)
+    _expect(x_scale, "x_scale", torch.float32, (n,), x.device)
     _check("cat_transform_quantize_act", load_library().cat_transform_quantize_act(
         _ptr(x), _dtype(x), n, d_in, k, _ptr(T_blocks), _ptr(xq), _ptr(x_scale), _stream(x.device)))
     return xq, x_scale
+
+
+def _linear_args(xq, x_scale, Wq, w_scale, y) -> None:
+    n, half = xq.shape
+    d_out = Wq.shape[0]
+    dev = xq.device
+    _expect(xq, "xq", torch.uint8, (n, half), dev)
+    _expect(x_scale, "x_scale", torch.float32, (n,), dev)
+    _expect(Wq, "Wq", torch.uint8, (d_out, half), dev)
+    _expect(w_scale, "w_scale", torch.float32, (d_out,), dev)
+    _expect(y, "y", torch.float32, (n, d_out), dev)
 
 
 def cat_w4a4_linear(xq: torch.Tensor, x_scale: torch.Tensor, Wq: torch.Tensor, w_scale: torch.Tensor,
@@ -215,6 +252,9 @@ def cat_w4a4_linear(xq: torch.Tensor, x_scale: torch.Tensor, Wq: torch.Tensor, w
     d_out = Wq.shape[0]
     if y is None:
         y = torch.empty((n, d_out), dtype=torch.float32, device=xq.device)
+    _linear_args(xq, x_scale, Wq, w_scale, y)
+    if acc_out is not None:
+        _expect(acc_out, "acc_out", torch.int32, (n, d_out), xq.device)
     _check("cat_w4a4_linear", load_library().cat_w4a4_linear(
         _ptr(xq), _ptr(x_scale), _ptr(Wq), _ptr(w_scale), n, 2 * half, d_out, _ptr(y), _ptr(acc_out),
         _stream(xq.device)))
@@ -233,6 +273,9 @@ def cat_w4a4_linear_sqnr(xq: torch.Tensor, x_scale: torch.Tensor, Wq: torch.Tens
         y = torch.empty((n, d_out), dtype=torch.float32, device=xq.device)
     if out is None:
         out = torch.empty((3,), dtype=torch.float64, device=xq.device)
+    _linear_args(xq, x_scale, Wq, w_scale, y)
+    _expect(y_ref, "y_ref", torch.float32, (n, d_out), xq.device)
+    _expect(out, "out", torch.float64, (3,), xq.device)
     _check("cat_w4a4_linear_sqnr", load_library().cat_w4a4_linear_sqnr(
         _ptr(xq), _ptr(x_scale), _ptr(Wq), _ptr(w_scale), n, 2 * half, d_out, _ptr(y), _ptr(y_ref), _ptr(out),
         _stream(xq.device)))
@@ -245,6 +288,10 @@ def cat_sqnr(y_ref: torch.Tensor, y_hat: torch.Tensor, out: Optional[torch.Tenso
     _need(y_hat, "y_hat")
     if out is None:
         out = torch.empty((3,), dtype=torch.float64, device=y_ref.device)
+    _expect(y_hat, "y_hat", torch.float32, tuple(y_ref.shape), y_ref.device)
+    _expect(out, "out", torch.float64, (3,), y_ref.device)
+    if y_ref.dtype != torch.float32:
+        raise ValueError("y_ref must be float32")
     _check("cat_sqnr", load_library().cat_sqnr(_ptr(y_ref), _ptr(y_hat), y_ref.numel(), _ptr(out),
                                                _stream(y_ref.device)))
     return out
@@ -257,6 +304,7 @@ def cat_block_row_stats(V: torch.Tensor, k: int, M: torch.Tensor, transpose: boo
     _need(V, "V")
     _need(M, "M")
     rows, d = V.shape
+    _expect(M, "M", torch.float32, (d // k, k, k), V.device)
     row_sumsq = torch.empty((rows,), dtype=torch.float32, device=V.device)
     row_amax = torch.empty((rows,), dtype=torch.float32, device=V.device)
     out3 = torch.empty((3,), dtype=torch.float64, device=V.device)

@@ -107,16 +107,10 @@ __global__ void __launch_bounds__(ActCfg<K>::THREADS) transform_quant_kernel(
     for (int r = 0; r < 4; ++r) {
       const int64_t t = t0 + 4 * tg + r;
       if (t >= n) continue;
-      const float a = __uint_as_float(amax_bits[t]);
-      const bool ok = isfinite(a);
-      const float inv = (ok && a > 0.f) ? __fdiv_rn(7.0f, a) : 0.f;
+      const QRow qr = qrow_setup(__uint_as_float(amax_bits[t]), 7.0f);
       int q[8];
 #pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        const float v = acc[r][c] * inv;
-        const int iv = isfinite(v) ? __float2int_rn(v) : 0;
-        q[c] = iv > 7 ? 7 : (iv < -7 ? -7 : iv);
-      }
+      for (int c = 0; c < 8; ++c) q[c] = qcode_exact(acc[r][c], qr, 7.0f);
       codes[t * words_per_row + word] = sm4_pack(q);
     }
   }

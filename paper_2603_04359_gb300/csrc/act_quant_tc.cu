@@ -12,7 +12,7 @@
 // units, so it re-splits A_b only when b changes.  D is double-buffered in tensor memory.  The
 // epilogue thread owns one row (TMEM lane), so its row maximum needs no reduction:
 //   pass 0: atomicMax of the row maxima into the scale buffer (float bits, non-negative),
-//   pass 1: recompute, q = clamp(rint(v' * (7 / max)), -7, 7), pack SM4x8, store.
+//   pass 1: recompute, q = clamp(round_half_even(7 v' / max), -7, 7) decided exactly, pack SM4x8, store.
 // Warps: 0 TMA producer + TMEM allocator, 1 MMA issuer, 4..7 epilogue, 8..15 converters.
 #include <atomic>
 #include <cstring>
@@ -132,16 +132,29 @@ __device__ __forceinline__ uint32_t twos_to_sm(uint32_t w) {
   return ((w ^ m) + s) | (s << 7);                   // |q| (no carry leaves a byte) and the sign bit
 }
 
-// One SM4x8 word of the codes rint(fl32(v_e * inv)), e = 0..7 (v_e = r[base + e] as float), for
-// |v_e * inv| <= 7 (inv = 7 / max|v|).  Adding 1.5 * 2^23 to the rounded product rounds it to an
-// integer (half to even, as rint) that sits, two's complement, in the low byte of the sum's bits;
-// the bytes are gathered four to a word and turned into sign-magnitude.  A non-finite product leaves
-// a garbage byte: callers zero the codes of rows whose maximum is not finite.
-__device__ __forceinline__ uint32_t sm4_quant8(const uint32_t (&r)[32], int base, float inv) {
+// One SM4x8 word of the codes of v_e = r[base + e] (as float), e = 0..7, on the row described by qr
+// (|v_e| <= max|v|).  Fast route: adding 1.5 * 2^23 to p = fl(v_e * inv) rounds it to an integer
+// (half to even) that sits, two's complement, in the low byte of the sum's bits; the bytes are
+// gathered four to a word and turned into sign-magnitude.  If any p lies within 2^-18 of a
+// half-integer (an exact tie included), or the row is rescaled, the eight codes are decided
+// exactly instead (qcode_exact).  Callers pass qr.inv == 0 only for rows whose codes are all 0.
+__device__ __forceinline__ uint32_t sm4_quant8(const uint32_t (&r)[32], int base, const QRow& qr) {
   constexpr float kMagic = 12582912.0f;
   uint32_t b[8];
+  bool near = qr.exact;
 #pragma unroll
-  for (int e = 0; e < 8; ++e) b[e] = __float_as_uint(__fadd_rn(__fmul_rn(__uint_as_float(r[base + e]), inv), kMagic));
+  for (int e = 0; e < 8; ++e) {
+    const float p = __fmul_rn(__uint_as_float(r[base + e]), qr.inv);
+    const float rb = __fadd_rn(p, kMagic);
+    near |= fabsf(__fsub_rn(__fsub_rn(rb, kMagic), p)) > kNearTie;
+    b[e] = __float_as_uint(rb);
+  }
+  if (near) {
+    int q[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) q[e] = qcode_exact(__uint_as_float(r[base + e]), qr, 7.0f);
+    return sm4_pack(q);
+  }
   const uint32_t lo = twos_to_sm(__byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410));
   const uint32_t hi = twos_to_sm(__byte_perm(__byte_perm(b[4], b[5], 0x0040), __byte_perm(b[6], b[7], 0x0040), 0x5410));
   return lo | __funnelshift_l(hi, hi, 4);
@@ -287,11 +300,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int b = (int)(u / num_tiles), tile = (int)(u % num_tiles);
       const uint32_t sd = j & 1;
       const int t = tile * TM + quad * 32 + lane;
-      float inv = 0.f;
+      QRow qr = qrow_setup(0.f, 7.0f);
       if (PASS == 1) {
         const float a = a_next;
         if (u + 1 < u1 && row_of(u + 1) < n) a_next = __uint_as_float(__ldcg(&amax_bits[row_of(u + 1)]));
-        inv = (t < n && isfinite(a) && a > 0.f) ? __fdiv_rn(7.0f, a) : 0.f;
+        if (t < n) qr = qrow_setup(a, 7.0f);
         if (scale && b == 0 && t < n) {               // each row's one unit of block 0 writes its step
           float sc = 0.f;
           if (isfinite(a))
@@ -324,7 +337,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           // 0 codes for an all-zero or non-finite row)
           uint32_t w[4];
 #pragma unroll
-          for (int g = 0; g < 4; ++g) w[g] = inv == 0.f ? 0u : sm4_quant8(r, 8 * g, inv);
+          for (int g = 0; g < 4; ++g) w[g] = qr.inv == 0.f ? 0u : sm4_quant8(r, 8 * g, qr);
           *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * K + c * 32) / 8) =
               make_uint4(w[0], w[1], w[2], w[3]);
         }
@@ -425,27 +438,33 @@ __device__ __forceinline__ void quantize_jobs(uint32_t tmem, int64_t u0, int64_t
   const int nu = (int)(u1 - u0);
   const int jobs = nu * (K / 32);
   // this lane's row maxima of every unit, all loads in flight at once
-  float inv_u[kMaxUnits];
+  float a_u[kMaxUnits], inv_u[kMaxUnits];
 #pragma unroll
   for (int j = 0; j < kMaxUnits; ++j) {
     const int t = (int)((u0 + j) % num_tiles) * TM + quad * 32 + lane;
-    inv_u[j] = (j < nu && t < n) ? __uint_as_float(__ldcg(&amax_bits[t])) : 0.f;
+    a_u[j] = (j < nu && t < n) ? __uint_as_float(__ldcg(&amax_bits[t])) : 0.f;
   }
 #pragma unroll
-  for (int j = 0; j < kMaxUnits; ++j) {
-    const float a = inv_u[j];
-    inv_u[j] = (isfinite(a) && a > 0.f) ? __fdiv_rn(7.0f, a) : 0.f;
-  }
+  for (int j = 0; j < kMaxUnits; ++j) inv_u[j] = qrow_setup(a_u[j], 7.0f).inv;
   tc_fence_after();
   for (int job = slot; job < jobs; job += 3) {
     const int j = job / (K / 32), c = job % (K / 32);
     const int64_t u = u0 + j;
     const int b = (int)(u / num_tiles), tile = (int)(u % num_tiles);
     const int t = tile * TM + quad * 32 + lane;
-    float inv = inv_u[0];
+    float inv = inv_u[0], a = a_u[0];
 #pragma unroll
     for (int q = 1; q < kMaxUnits; ++q)
-      if (j == q) inv = inv_u[q];
+      if (j == q) {
+        inv = inv_u[q];
+        a = a_u[q];
+      }
+    QRow qr;
+    qr.inv = inv;
+    qr.a = a;
+    qr.sc = 1.f;
+    qr.exact = false;
+    if (inv != 0.f && (a > 0x1p100f || a < 0x1p-60f)) qr = qrow_setup(a, 7.0f);  // rescaled row
     uint32_t r[32];
     __syncwarp();
     CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + j * K + c * 32, r);
@@ -453,7 +472,7 @@ __device__ __forceinline__ void quantize_jobs(uint32_t tmem, int64_t u0, int64_t
     if (t < n) {
       uint32_t w[4];
 #pragma unroll
-      for (int g = 0; g < 4; ++g) w[g] = inv == 0.f ? 0u : sm4_quant8(r, 8 * g, inv);  // 0: zero or non-finite row
+      for (int g = 0; g < 4; ++g) w[g] = inv == 0.f ? 0u : sm4_quant8(r, 8 * g, qr);  // 0: zero or non-finite row
       *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * K + c * 32) / 8) =
           make_uint4(w[0], w[1], w[2], w[3]);
     }

@@ -82,7 +82,9 @@ constexpr size_t kPrepScratchBytes = kPrepSigmaBytes + (size_t)kPrepMaxDK * size
 
 }  // namespace
 
-// Reserved with the module on each device that loads the library (12 MiB).
+// 12 MiB on each device where this module is loaded.  With lazy module loading (CUDA's default)
+// that happens at the first use of this translation unit on the device -- in practice the first
+// entry-point call there -- not when the library is loaded into the process.
 static __device__ __align__(256) unsigned char g_prep_scratch[kPrepScratchBytes];
 
 namespace {

@@ -96,6 +96,70 @@ __device__ __forceinline__ uint32_t sm4_pack(const int (&q)[8]) {
 constexpr float kAccScale = 262144.0f;
 
 // ------------------------------------------------------------------------------------------
+// Exact symmetric round-to-nearest code decision (Lemma 2 range, Sec. 6 RTN):
+//   q = clamp(round_half_even(qmax * v / a), -qmax, qmax),   a = max|v| of the row.
+// The fast estimate p = fl(v * fl(qmax / a)) is within qmax * 2^-22 of the quotient, so rint(p) is
+// the exact code unless p lies within 2^-18 of a half-integer; there the decision is redone
+// exactly: with f = floor(p) and the boundary h = f + 1/2, the sign of qmax*|v| - h*a is found from
+// a two-product (qmax*|v| = prod + err, both fp32, err by fma) and one fma for prod - h*a, which
+// is exact whenever it is small and otherwise far from zero, so its sum with err has the true
+// sign, and is zero only on an exact tie.  Rows whose maximum lies outside [2^-60, 2^100] are
+// rescaled by a power of two first (exact), so qmax*|v| cannot overflow and no product loses bits
+// to underflow; such rows always take the exact route.
+// ------------------------------------------------------------------------------------------
+struct QRow {
+  float inv;   // fl(qmax / a_s), 0 for a row whose codes are all 0 (zero or non-finite maximum)
+  float a;     // a_s = a * sc
+  float sc;    // power-of-two rescale (1 for ordinary rows)
+  bool exact;  // always decide exactly (rescaled rows)
+};
+
+__device__ __forceinline__ QRow qrow_setup(float a, float qmax) {
+  QRow r;
+  r.sc = 1.f;
+  r.exact = false;
+  if (!(isfinite(a) && a > 0.f)) {
+    r.inv = 0.f;
+    r.a = 0.f;
+    return r;
+  }
+  if (a > 0x1p100f) {
+    r.sc = 0x1p-64f;
+    r.exact = true;
+  } else if (a < 0x1p-60f) {
+    r.sc = 0x1p64f;
+    r.exact = true;
+  }
+  r.a = a * r.sc;
+  r.inv = __fdiv_rn(qmax, r.a);
+  return r;
+}
+
+// round_half_even(qmax * u / a) for 0 <= u <= a (both already rescaled, a in [2^-60, 2^100]).
+__device__ __forceinline__ int qmag_exact(float u, float a, float inv, float qmax) {
+  const float p = __fmul_rn(u, inv);
+  const float f = floorf(p);
+  const float h = __fadd_rn(f, 0.5f);
+  const float prod = __fmul_rn(qmax, u);
+  const float err = __fmaf_rn(qmax, u, -prod);
+  const float dd = __fmaf_rn(-h, a, prod);
+  const float tot = __fadd_rn(dd, err);
+  int q = (int)f;
+  q += (tot > 0.f || (tot == 0.f && (q & 1))) ? 1 : 0;
+  return q > (int)qmax ? (int)qmax : q;
+}
+
+// The signed code of one value of a row (0 for a non-finite value or a zero row).
+__device__ __forceinline__ int qcode_exact(float v, const QRow& r, float qmax) {
+  if (r.inv == 0.f || !isfinite(v)) return 0;
+  const int m = qmag_exact(fabsf(v) * r.sc, r.a, r.inv, qmax);
+  return v < 0.f ? -m : m;
+}
+
+// |rint(p) - p| beyond this marks a value whose fast code may differ from the exact one.
+constexpr float kNearTie = 0.5f - 0x1p-18f;
+
+// ------------------------------------------------------------------------------------------
 // Shared-memory addresses, mbarriers (all waits bounded).
 // ------------------------------------------------------------------------------------------
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {

@@ -152,6 +152,80 @@ def test_nonfinite_activation_two_pass():
     assert cat.cat_device_status()[0] == 0
 
 
+def _bf16_tie_pairs():
+    """For every bf16 step a in [1, 2): the bf16 values v in [a/14, a] with 7 v / a exactly a
+    half-integer (exact rational arithmetic)."""
+    from fractions import Fraction
+    out = {}
+    for ma in range(128):
+        a = Fraction(128 + ma, 128)
+        vs = []
+        for e in range(-4, 1):
+            for mv in range(128):
+                v = Fraction(128 + mv, 128) * Fraction(2) ** e
+                t = 7 * v / a
+                if v <= a and t.denominator == 2:
+                    vs.append(float(v))
+        if vs:
+            out[float(a)] = vs
+    return out
+
+
+def _tie_rows(rng, n, d):
+    """bf16-representable rows in which many entries make 7 v / max|v| an exact half-integer, at
+    ordinary scales and at scales that take the rescaled route (2^-100, 2^110)."""
+    pairs = _bf16_tie_pairs()
+    steps = np.array(sorted(pairs))
+    X = np.empty((n, d))
+    for r in range(n):
+        a = float(rng.choice(steps))
+        ties = np.array(pairs[a])
+        row = WL.cast(rng.uniform(-a, a, d) * 0.99, "bf16").values.astype(np.float64)  # ordinary values
+        pick = rng.random(d) < 0.5
+        row[pick] = rng.choice(ties, pick.sum()) * rng.choice([-1.0, 1.0], pick.sum())
+        row[rng.integers(d)] = a * rng.choice([-1.0, 1.0])
+        scale = {0: 2.0 ** -100, 1: 2.0 ** 110}.get(r, 2.0 ** int(rng.integers(-12, 12)))
+        X[r] = row * scale
+    Xt = WL.cast(X, "bf16")
+    assert np.array_equal(Xt.values, X)                        # every value is a bf16 number
+    return X
+
+
+@pytest.mark.parametrize("n,d,k,dtype", [(300, 512, 64, "bf16"), (1000, 1024, 128, "bf16"),   # fused
+                                         (2560, 4096, 128, "bf16"),                            # two-pass
+                                         (130, 256, 32, "f32"), (200, 512, 256, "bf16"),       # SIMT
+                                         (70, 64, 16, "bf16")])
+def test_code_decision_exact_on_ties(n, d, k, dtype):
+    """With T = I the transformed row is the input row, so the codes must equal the definition's
+    round-half-to-even of 7 v / max|v| exactly, ties included (Lemma 2 range, Sec. 6 RTN).  The rows
+    are built so that a float32 reciprocal-multiply decision would get many of them wrong."""
+    rng = np.random.default_rng(n + k)
+    X = _tie_rows(rng, n, d)
+    Xt = WL.cast(X, dtype)
+    ref = O.quantize_rows_symmetric(Xt.values)
+    a32 = np.max(np.abs(Xt.values), axis=1).astype(np.float32)
+    q32 = np.clip(np.rint(Xt.values.astype(np.float32) * (np.float32(7) / a32)[:, None]), -7, 7)
+    assert np.sum(q32 != ref[0]) > 10                          # the fixture has teeth
+    T = np.tile(np.eye(k, dtype=np.float32), (d // k, 1, 1))
+    xq, sx = cat.cat_transform_quantize_act(to_dev(Xt), torch.from_numpy(T).to(DEV), k)
+    np.testing.assert_array_equal(sm4x8.unpack(xq.cpu().numpy()), ref[0])
+    np.testing.assert_allclose(sx.cpu().numpy().astype(np.float64), ref[1], rtol=1e-6, atol=0)
+    assert cat.cat_device_status()[0] == 0
+
+
+@pytest.mark.parametrize("k", [32, 128])
+def test_weight_code_decision_exact_on_ties(k):
+    """Weight preparation with T = I quantizes the rows of W itself: exact codes, ties included."""
+    rng = np.random.default_rng(99 + k)
+    W = _tie_rows(rng, 300, 1024)
+    Wt = WL.cast(W, "bf16")
+    T, Wq, sw = cat.cat_quantize_weights(to_dev(Wt), k, "identity")
+    ref = O.quantize_rows_symmetric(Wt.values)
+    np.testing.assert_array_equal(sm4x8.unpack(Wq.cpu().numpy()), ref[0])
+    np.testing.assert_allclose(sw.cpu().numpy().astype(np.float64), ref[1], rtol=1e-6, atol=0)
+    assert cat.cat_device_status()[0] == 0
+
+
 # ------------------------------------------------------------------------------------------
 # cat_w4a4_linear (given identical codes): exact accumulators
 # ------------------------------------------------------------------------------------------
@@ -282,7 +356,10 @@ def test_layer_end_to_end(cfg, kind):
     ref = O.cat_layer(L.x_eval.values, L.W.values, kind, k, X_calib=L.x_calib.values, signs=L.rht_signs)
     # transform blocks
     assert rel_fro(g["T"].cpu().numpy(), ref["prep"].T) < (1e-6 if cfg.dtype == "f32" else 1e-5)
-    # weight and activation codes, steps
+    # weight and activation codes, steps (T = I: the quantizer sees the inputs themselves, exact codes)
+    if kind == "identity":
+        np.testing.assert_array_equal(sm4x8.unpack(g["Wq"].cpu().numpy()), ref["prep"].qw)
+        np.testing.assert_array_equal(sm4x8.unpack(g["xq"].cpu().numpy()), ref["act"].qx)
     check_codes(sm4x8.unpack(g["Wq"].cpu().numpy()), ref["prep"].qw, ref["prep"].pre_w)
     np.testing.assert_allclose(g["sw"].cpu().numpy(), ref["prep"].sw, rtol=1e-5)
     check_codes(sm4x8.unpack(g["xq"].cpu().numpy()), ref["act"].qx, ref["act"].pre_x)

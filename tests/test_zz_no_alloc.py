@@ -74,26 +74,36 @@ class _DefaultPool:
 @pytest.mark.gpu
 def test_noalloc_matches_quantize_weights_on_consecutive_calls():
     pool = _DefaultPool(torch.cuda.current_device())
-    for cfg in LAYERS:
+    if not pool.ok:
+        pytest.fail("the default stream-ordered pool could not be opened through libcuda: the no-allocation "
+                    "check would not run")
+    for i, cfg in enumerate(LAYERS):
         L = WL.make_layer(cfg)
         k = cfg.k
         W, xc = _to_dev(L.W), _to_dev(L.x_calib)
         sig = cat.cat_calib_cov(xc, k)
         torch.cuda.synchronize()
         # control: the allocating entry point raises the pool's high watermark, so the watch works
-        watched = pool.reset()
+        assert pool.reset()
         ref = cat.cat_quantize_weights(W, k, "cat", sigma_x=sig, n_calib=cfg.n_calib)
         torch.cuda.synchronize()
-        control = pool.high() if watched else None
-        watched = bool(control) and pool.reset()
+        control = pool.high()
+        if not control:
+            pytest.fail(f"the allocating entry point left the pool's watermark at {control}: the watch cannot "
+                        "tell an allocation from none")
         # preallocated outputs, so that nothing but the call itself runs between the two readings
         out = (torch.full_like(ref[0], float("nan")), torch.full_like(ref[1], 0xFF), torch.full_like(ref[2], -1.0))
         torch.cuda.synchronize()
-        if watched:
-            watched = pool.reset()
+        assert pool.reset()
+        free_before = torch.cuda.mem_get_info()[0]
         got = cat.cat_quantize_weights_noalloc(W, k, "cat", sigma_x=sig, n_calib=cfg.n_calib, out=out)
-        if watched:
-            assert pool.high() == 0, "the no-alloc entry point took memory from the stream-ordered pool"
+        torch.cuda.synchronize()
+        free_after = torch.cuda.mem_get_info()[0]
+        assert pool.high() == 0, "the no-alloc entry point took memory from the stream-ordered pool"
+        if i > 0:
+            # after the first call (which may load the library's modules and their static scratch onto
+            # the device) no call takes device memory of any kind
+            assert free_after == free_before, f"free device memory moved by {free_before - free_after} bytes"
         assert cat.cat_device_status()[0] == 0
         _compare(got, ref)
 
