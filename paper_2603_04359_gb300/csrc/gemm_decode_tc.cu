@@ -17,8 +17,19 @@
 //     exact products q_x q_w 2^-18 in fp32 (|acc| <= 49 d_in < 2^24);
 //   * four epilogue warps read the double-buffered accumulator (thread = output channel) and write
 //     y[t][o] with consecutive o across a warp; y_ref, when given, is loaded while the MMAs run.
-// A persistent CTA per SM walks 128-row units.  Every mbarrier wait is bounded; a wait that gives up
-// raises the device status word and all roles drain and exit.
+// Work split (stream-K): the (unit, K step) sequence -- unit-major, num_units x num_ks steps of
+// 16 KiB -- is cut into one contiguous, equal range per CTA, one CTA per SM, so every SM streams
+// the same number of weight bytes whatever the number of units (with 128-row units alone, 112 units
+// at d_out = 14336 left 40 of 152 SMs idle).  A unit whose steps fall into one CTA's range is
+// finished there.  A unit cut between CTAs is owned by the CTA holding its first step, where it is
+// the last segment of the range; every other part is the first segment of its CTA's range, so it
+// is done early: it stores its raw accumulators (integers times 2^-18, exact in fp32) to its CTA's
+// slice of device scratch and bumps the unit's per-warp counter.  The owner waits (bounded) for the
+// counter while its own MMAs run, loads the other slices, adds them (an exact sum in any order),
+// writes y and resets the counter.  The launch is cooperative, so all parts are resident while the
+// owners wait.  Every mbarrier wait is bounded; a wait that gives up raises the device status word
+// and all roles drain and exit.
+#include <atomic>
 #include <cstring>
 #include <mutex>
 
@@ -55,6 +66,32 @@ struct TmemPlan {
 };
 constexpr uint32_t kTmemCols = 512;
 constexpr size_t kSmemBudget = 220 * 1024;
+
+// Partial accumulators of the non-owner parts of cut units: slice (slot, CTA) holds [NTOK <= 32][128]
+// floats (a CTA is a non-owner part only of the first unit of its range); counters per (slot, unit,
+// epilogue warp).  Slots are handed out round robin per launch.
+constexpr int kDecSlots = 2;
+constexpr int kDecMaxGrid = 192;
+constexpr int kDecMaxUnits = 4096;
+__device__ float4 g_dec_part[kDecSlots][kDecMaxGrid][32][UM / 4];
+__device__ uint32_t g_dec_cnt[kDecSlots][kDecMaxUnits][kEpiWarps];
+
+__device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Range of (unit, K step) steps of CTA c out of g: [s0, s1).  split: equal cuts of all T steps;
+// otherwise whole units, contiguous.
+__host__ __device__ __forceinline__ int range_begin(int c, int g, int units, int num_ks, bool split) {
+  if (split) return (int)((int64_t)c * units * num_ks / g);
+  return (int)((int64_t)c * units / g) * num_ks;
+}
+// The CTA whose range holds step s (split mode): the largest c with range_begin(c) <= s.
+__device__ __forceinline__ int cta_of_step(int s, int g, int total) {
+  return (int)(((int64_t)(s + 1) * g + total - 1) / total) - 1;
+}
 
 struct DecBars {
   uint64_t p_full[kMaxSP], p_empty[kMaxSP], empty[kMaxSE], acc_full[2], acc_empty[2], tok_ready, mma_done;
@@ -102,19 +139,21 @@ __device__ __forceinline__ void dec_mma_ts(uint32_t d_tmem, uint32_t a_tmem, uin
 // Bytes of the resident token operand: one [NTOK rows x 128 B] block per 128-code slab.
 __host__ __device__ constexpr size_t tok_bytes(int ntok, int num_ks) { return (size_t)num_ks * 2 * ntok * 128; }
 
-template <int NTOK>
+template <int NTOK, bool SPLIT>
 __global__ void __launch_bounds__(kThreads, 1)
     w4a4_gemm_decode_tc_kernel(const __grid_constant__ CUtensorMap tmW, const uint8_t* __restrict__ xq,
                                const float* __restrict__ sx, const float* __restrict__ sw, int n, int d_in, int d_out,
                                int sp, float* __restrict__ y, int32_t* __restrict__ acc_out,
                                const float* __restrict__ y_ref, double* __restrict__ sums3, int sqnr_slot,
-                               uint32_t* __restrict__ status) {
+                               int part_slot, uint32_t* __restrict__ status) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int row_bytes = d_in / 2;
   const int num_ks = (row_bytes + KSB - 1) / KSB;
   const int num_units = (d_out + UM - 1) / UM;
-  const int act_groups = num_ks < kDecGroups ? num_ks : kDecGroups;  // groups with K steps in a unit
+  const int total = num_units * num_ks;
+  const int s0 = range_begin(blockIdx.x, gridDim.x, num_units, num_ks, SPLIT);
+  const int s1 = range_begin(blockIdx.x + 1, gridDim.x, num_units, num_ks, SPLIT);
   constexpr int kSE = TmemPlan<NTOK>::kSE;
   constexpr uint32_t kAStage0 = TmemPlan<NTOK>::kAccCols;
   uint8_t* bst = smem;                                            // tokens, E4M3
@@ -131,11 +170,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int s = 0; s < kSE; ++s) mbar_init(&bars->empty[s], 1);
     for (int b = 0; b < 2; ++b) {
-      mbar_init(&bars->acc_full[b], act_groups);  // the groups with K steps in a unit commit once each
+      mbar_init(&bars->acc_full[b], kDecGroups);  // every group commits once per segment
       mbar_init(&bars->acc_empty[b], kEpiWarps);
     }
     mbar_init(&bars->tok_ready, kThreads / 32 - kStageWarp0);
-    mbar_init(&bars->mma_done, act_groups);
+    mbar_init(&bars->mma_done, kDecGroups);
     bars->abort = 0;
     fence_mbar_init();
   }
@@ -151,24 +190,47 @@ __global__ void __launch_bounds__(kThreads, 1)
     // thread's loads in flight at once: the first MMA waits for the whole operand): slab a (codes
     // 128a .. 128a+127) of token t at a*NTOK*128 + t*128, 16-byte chunk c at c ^ (t % 8); tokens >= n
     // and codes >= d_in are zero
-    const int slabs = 2 * num_ks;
+    // Only the K steps of this CTA's range are staged: with fewer steps than a row has, they are the
+    // num_ks-periodic run starting at s0 % num_ks.  Item e = 16-byte chunk c of token t's packed row
+    // (e = t * row_chunks + c); (t, c) advance incrementally, with no division inside the loops.
+    const int span = s1 - s0, ks_lo = s0 % num_ks;
+    const int row_chunks = 8 * num_ks;                            // 16-byte chunks per (padded) packed row
     const int st = tid - kStageWarp0 * 32, nst = kThreads - kStageWarp0 * 32;
-    const int items = NTOK * slabs * 4;
+    const float sx_pre = (st < NTOK && st < n) ? sx[st] * kAccScale : 0.f;   // loaded beside the token rows
+    const int items = NTOK * row_chunks;
+    const int step_t = nst / row_chunks, step_c = nst % row_chunks;
+    int t_cur = st / row_chunks, c_cur = st % row_chunks;
+    auto needed = [&](int c) {
+      if (!SPLIT) return true;
+      int dk = (c >> 3) - ks_lo;
+      if (dk < 0) dk += num_ks;
+      return span >= num_ks || dk < span;
+    };
     for (int e0 = st; e0 < items; e0 += kTokLoads * nst) {
       uint4 w[kTokLoads];
+      int tc[kTokLoads];                                          // t << 16 | c of each item, -1 past the end
 #pragma unroll
       for (int q = 0; q < kTokLoads; ++q) {
         const int e = e0 + q * nst;
-        const int j = e & 3, a = (e >> 2) % slabs, t = (e >> 2) / slabs;
-        const int off = a * 64 + j * 16;                          // packed byte offset in the row
+        const int t = t_cur, c = c_cur;
+        tc[q] = e < items ? (t << 16 | c) : -1;
+        const int off = c * 16;                                   // packed byte offset in the row
         w[q] = make_uint4(0u, 0u, 0u, 0u);
-        if (e < items && t < n && off < row_bytes) w[q] = *reinterpret_cast<const uint4*>(xq + (int64_t)t * row_bytes + off);
+        if (e < items && t < n && off < row_bytes && needed(c))
+          w[q] = *reinterpret_cast<const uint4*>(xq + (int64_t)t * row_bytes + off);
+        c_cur += step_c;
+        t_cur += step_t;
+        if (c_cur >= row_chunks) {
+          c_cur -= row_chunks;
+          ++t_cur;
+        }
       }
 #pragma unroll
       for (int q = 0; q < kTokLoads; ++q) {
-        const int e = e0 + q * nst;
-        if (e >= items) break;
-        const int j = e & 3, a = (e >> 2) % slabs, t = (e >> 2) / slabs;
+        if (tc[q] < 0) break;
+        const int t = tc[q] >> 16, c = tc[q] & 0xFFFF;
+        if (!needed(c)) continue;
+        const int a = c >> 2, j = c & 3;                          // 64-byte slab a, 16-byte chunk j in it
         uint8_t* dst = bst + (size_t)a * NTOK * 128 + t * 128;
         const int swz = t & 7;
         *reinterpret_cast<uint4*>(dst + (((2 * j) ^ swz) << 4)) =
@@ -177,7 +239,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             make_uint4(sm4_lo(w[q].z), sm4_hi(w[q].z), sm4_lo(w[q].w), sm4_hi(w[q].w));
       }
     }
-    if (st < NTOK) sxs[st] = st < n ? sx[st] * kAccScale : 0.f;
+    if (st < NTOK) sxs[st] = sx_pre;
     fence_proxy_async_smem();                                     // the MMA reads the tokens via the async proxy
     __syncwarp();
     if (lane == 0) mbar_arrive(&bars->tok_ready);
@@ -188,17 +250,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       const uint32_t me = warp == kProd0 ? 0u : 1u;
       if (me == 0) prefetch_tensormap(&tmW);
+      // it = the CTA-local step index (step s0 + it of the (unit, K step) sequence)
       uint32_t it = 0, issued_end = 0;                  // this producer issued every K step of its parity below issued_end
       bool ok = true;
-      for (int u = blockIdx.x; u < num_units && ok; u += gridDim.x)
-        for (int ks = 0; ks < num_ks; ++ks, ++it) {
-          if ((it & 1u) != me) continue;
-          const uint32_t s = it % sp, use = it / sp;
-          if (use > 0 && !(ok = mbar_wait_bounded(&bars->p_empty[s], (use - 1) & 1, abort_flag, __LINE__))) break;
-          mbar_arrive_expect_tx(&bars->p_full[s], kPkStage);
-          tma_load_2d(pk + s * kPkStage, &tmW, ks * KSB, u * UM, &bars->p_full[s]);
-          issued_end = it + 1;
-        }
+      for (int sg = s0; sg < s1 && ok; ++sg, ++it) {
+        if ((it & 1u) != me) continue;
+        const int u = sg / num_ks, ks = sg % num_ks;
+        const uint32_t s = it % sp, use = it / sp;
+        if (use > 0 && !(ok = mbar_wait_bounded(&bars->p_empty[s], (use - 1) & 1, abort_flag, __LINE__))) break;
+        mbar_arrive_expect_tx(&bars->p_full[s], kPkStage);
+        tma_load_2d(pk + s * kPkStage, &tmW, ks * KSB, u * UM, &bars->p_full[s]);
+        issued_end = it + 1;
+      }
       // loads still in flight land before the CTA exits: only the last sp K steps of the whole walk
       // (`it` steps) have stages that were not reused, so only their barriers still hold the phase
       // to wait for; this producer waits for the ones it issued
@@ -208,31 +271,37 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp >= kDecWarp0 && warp < kDecWarp0 + kDecWarps) {
     // ---------------------------------------------------------------- decode + MMA: weight row = TMEM lane
-    // Four groups of four warps (one per TMEM lane quadrant) take every fourth K step.  A thread
-    // decodes its whole 128-byte row (256 codes, 64 TMEM columns); then the group's leader thread
-    // issues the step's eight MMAs into the group's own accumulator.  One thread issues an MMA about
-    // every 55 cycles whatever N is, so four issuers keep the tensor core fed at N = 16; the four
-    // partial accumulators are added in the epilogue (integers times 2^-18: exact).
+    // Four groups of four warps (one per TMEM lane quadrant) take every fourth step of the CTA's
+    // range (group = local step index mod 4, so every stage has one consumer).  A thread decodes its
+    // whole 128-byte row (256 codes, 64 TMEM columns); then the group's leader thread issues the
+    // step's eight MMAs into the group's own accumulator.  One thread issues an MMA about every 55
+    // cycles whatever N is, so four issuers keep the tensor core fed at N = 16; the partial
+    // accumulators of a segment (the range's steps of one unit) are added in the epilogue (integers
+    // times 2^-18: exact).  Every group commits the segment's accumulator barrier once, with or
+    // without steps in it, after waiting for that buffer to be drained.
     const int quad = warp & 3, grp = (warp - kDecWarp0) >> 2;
     const bool leader = quad == 0 && lane == 0;
     const int r = quad * 32 + lane;
     constexpr uint32_t kIdesc = idesc_e4m3_f32(UM, NTOK);
     const uint32_t bbase = smem_u32(bst);
-    uint32_t it = 0, tcount = 0;
     bool stop = false;
     if (leader) {
       mbar_wait_bounded(&bars->tok_ready, 0, abort_flag, __LINE__);
       tc_fence_after();
     }
-    for (int u = blockIdx.x; u < num_units && !stop; u += gridDim.x, ++tcount) {
-      const uint32_t ab = tcount & 1;
+    uint32_t seg = 0;
+    for (int sb = s0; sb < s1 && !stop; ++seg) {
+      const int u = sb / num_ks;
+      const int se = min(s1, (u + 1) * num_ks);        // segment [sb, se): the range's steps of unit u
+      const uint32_t ab = seg & 1;
       const uint32_t d_acc = tmem + (ab * kDecGroups + grp) * NTOK;
-      bool first = true;                                 // the group's first K step of the unit
-      for (int ks = 0; ks < num_ks; ++ks, ++it) {
-        if (ks % kDecGroups != grp) continue;          // group g takes the steps ks = g (mod 4) of every unit
-        const uint32_t ps = it % sp, s = it % kSE;
+      bool first = true;                                 // the group's first step of the segment
+      for (int sg = sb + ((grp - (sb - s0)) % kDecGroups + kDecGroups) % kDecGroups; sg < se; sg += kDecGroups) {
+        const uint32_t it = (uint32_t)(sg - s0);         // it % kDecGroups == grp
+        const int ks = sg % num_ks;
+        const uint32_t ps = it % sp, sa = it % kSE;
         const bool good = mbar_wait_bounded(&bars->p_full[ps], (it / sp) & 1, abort_flag, __LINE__) &&
-                          (it < (uint32_t)kSE || mbar_wait_bounded(&bars->empty[s], ((it / kSE) - 1) & 1, abort_flag, __LINE__));
+                          (it < (uint32_t)kSE || mbar_wait_bounded(&bars->empty[sa], ((it / kSE) - 1) & 1, abort_flag, __LINE__));
         if (good) {
           tc_fence_after();
           const uint8_t* prow = pk + ps * kPkStage + r * 128;
@@ -249,7 +318,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               av[8 * jj + 6] = sm4_lo(w.w); av[8 * jj + 7] = sm4_hi(w.w);
             }
             __syncwarp();
-            DEC_TMEM_ST32(tmem + ((uint32_t)(quad * 32) << 16) + kAStage0 + 64u * s + 32u * half, av);
+            DEC_TMEM_ST32(tmem + ((uint32_t)(quad * 32) << 16) + kAStage0 + 64u * sa + 32u * half, av);
           }
           dec_tmem_st_wait();
         }
@@ -261,21 +330,28 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (stop) break;
         if (leader) {
           tc_fence_after();
-          if (first && tcount >= 2) mbar_wait_bounded(&bars->acc_empty[ab], ((tcount >> 1) - 1) & 1, abort_flag, __LINE__);
+          if (first && seg >= 2) mbar_wait_bounded(&bars->acc_empty[ab], ((seg >> 1) - 1) & 1, abort_flag, __LINE__);
           tc_fence_after();
-          const uint32_t ta = tmem + kAStage0 + 64u * s;
+          const uint32_t ta = tmem + kAStage0 + 64u * sa;
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {  // K = 32 codes per MMA: 8 TMEM columns of A; B slab 2ks + kk/4, +32 B
             const uint64_t db = sdesc_kmajor_sw128(bbase + (uint32_t)((2 * ks + (kk >> 2)) * NTOK * 128)) + 2 * (kk & 3);
             dec_mma_ts(d_acc, ta + 8u * kk, db, kIdesc, (first && kk == 0) ? 0u : 1u);
           }
-          mma_commit(&bars->empty[s]);
-          if (ks + kDecGroups >= num_ks) mma_commit(&bars->acc_full[ab]);  // the group's last step of the unit
+          mma_commit(&bars->empty[sa]);
         }
         first = false;
       }
+      if (stop) break;
+      if (leader) {
+        // a group without steps in this segment still waits for the buffer to be drained before it
+        // commits, so its arrivals can never run a phase ahead
+        if (first && seg >= 2) mbar_wait_bounded(&bars->acc_empty[ab], ((seg >> 1) - 1) & 1, abort_flag, __LINE__);
+        mma_commit(&bars->acc_full[ab]);
+      }
+      sb = se;
     }
-    if (leader && grp < act_groups) {
+    if (leader) {
       mma_commit(&bars->mma_done);  // all MMAs complete before tensor memory is released
       volatile int no_abort = 0;
       mbar_wait_bounded(&bars->mma_done, 0, &no_abort);
@@ -283,27 +359,86 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp >= kEpiWarp0) {
     // ---------------------------------------------------------------- epilogue: output channel = TMEM lane
     const int quad = warp & 3;
-    uint32_t tcount = 0;
+    const int ch = quad * 32 + lane;                 // channel within the unit
     bool ok = true;
     f32x2 sig = {0.f, 0.f}, err = {0.f, 0.f};      // SQNR sums (Sec. 2, Eq. 1) when y_ref is given
-    for (int u = blockIdx.x; u < num_units && ok; u += gridDim.x, ++tcount) {
-      const uint32_t ab = tcount & 1;
-      const int o = u * UM + quad * 32 + lane;
+    uint32_t seg = 0;
+    for (int sb = s0; sb < s1 && ok; ++seg) {
+      const int u = sb / num_ks;
+      const int se = min(s1, (u + 1) * num_ks);
+      const uint32_t ab = seg & 1;
+      const bool whole = !SPLIT || se - sb == num_ks;  // the unit is finished in this CTA
+      const int o = u * UM + ch;
       const bool o_ok = o < d_out;
       const float swo = o_ok ? sw[o] : 0.f;
-      float yr[NTOK];                                // y_ref in flight while the MMAs of the unit run
+      const int cf = whole ? (int)blockIdx.x : cta_of_step(u * num_ks, gridDim.x, total);
+      const int cl = whole ? (int)blockIdx.x : cta_of_step((u + 1) * num_ks - 1, gridDim.x, total);
+      const bool owner = cf == (int)blockIdx.x;       // writes the unit's outputs
+      // y_ref in flight while the MMAs of the segment run, where this CTA writes the unit
+      const bool pre = y_ref && o_ok && owner;
+      float yr[NTOK];
 #pragma unroll
-      for (int t = 0; t < NTOK; ++t) yr[t] = (y_ref && o_ok && t < n) ? __ldcs(y_ref + (int64_t)t * d_out + o) : 0.f;
-      if (!(ok = mbar_wait_bounded(&bars->acc_full[ab], (tcount >> 1) & 1, abort_flag, __LINE__))) break;
+      for (int t = 0; t < NTOK; ++t) yr[t] = (pre && t < n) ? __ldcs(y_ref + (int64_t)t * d_out + o) : 0.f;
+      if (!(ok = mbar_wait_bounded(&bars->acc_full[ab], (seg >> 1) & 1, abort_flag, __LINE__))) break;
       __syncwarp();
       tc_fence_after();
+      // the groups with steps in the segment: local steps sb - s0 .. se - s0 - 1, group = step % 4
+      const int nact = se - sb < kDecGroups ? se - sb : kDecGroups;
+      uint32_t* cnt = &g_dec_cnt[part_slot][u][quad];
       float s_run = 0.f, e_run = 0.f;
+      auto emit = [&](int t, float a) {                // y (and acc_out, SQNR terms) of token t
+        const float v = a * sxs[t] * swo;              // consecutive o across the warp: coalesced stores
+        y[(int64_t)t * d_out + o] = v;
+        if (acc_out) acc_out[(int64_t)t * d_out + o] = __float2int_rn(a * kAccScale);
+        const float e = yr[t] - v;
+        s_run += yr[t] * yr[t];
+        e_run += e * e;
+      };
+      // owner of a cut unit: the other parts ran first in their CTAs; wait for their counts and
+      // sum their slices while this segment's MMAs run (16 tokens), or after them (32)
+      constexpr bool kEarly = SPLIT && NTOK == 16;
+      float ext[kEarly ? NTOK : 1];
+      auto wait_parts = [&]() -> bool {              // warp-uniform
+        uint32_t good = 1u;
+        if (lane == 0) {
+          const uint64_t t0 = globaltimer_ns();
+          for (uint32_t it = 0; ld_acquire_u32(cnt) < (uint32_t)(cl - cf); ++it) {
+            __nanosleep(32);
+            if ((it & 63u) == 63u && (*abort_flag || globaltimer_ns() - t0 > kWaitLimitNs)) {
+              if (*abort_flag == 0) *abort_flag = __LINE__;
+              good = 0u;
+              break;
+            }
+          }
+          if (good) *cnt = 0u;                         // every part has counted: clean for the next launch
+        }
+        good = __shfl_sync(0xFFFFFFFFu, good, 0);
+        __threadfence();
+        return good != 0u;
+      };
+      auto slice_of = [&](int c) { return reinterpret_cast<const float*>(&g_dec_part[part_slot][c][0][0]) + ch; };
+      if (kEarly && !whole && owner) {
+        if (!(ok = wait_parts())) break;
+#pragma unroll
+        for (int t = 0; t < (kEarly ? NTOK : 1); ++t) ext[t] = 0.f;
+        for (int c = cf + 1; c <= cl; ++c) {
+          const float* src = slice_of(c);
+#pragma unroll
+          for (int t = 0; t < (kEarly ? NTOK : 1); ++t) ext[t] += __ldcg(src + t * UM);  // exact in any order
+        }
+      }
+      if (!(ok = mbar_wait_bounded(&bars->acc_full[ab], (seg >> 1) & 1, abort_flag, __LINE__))) break;
+      __syncwarp();
+      tc_fence_after();
+      if (!kEarly && !whole && owner && !(ok = wait_parts())) break;
+      float* my_slice = reinterpret_cast<float*>(&g_dec_part[part_slot][blockIdx.x][0][0]) + ch;
 #pragma unroll
       for (int c = 0; c < NTOK / 16; ++c) {          // 16 accumulator columns at a time
         float acc[16];
 #pragma unroll
         for (int j = 0; j < 16; ++j) acc[j] = 0.f;
-        for (int g = 0; g < act_groups; ++g) {         // the decode groups' partial accumulators
+        for (int i = 0; i < nact; ++i) {
+          const int g = (sb - s0 + i) % kDecGroups;
           uint32_t part[16];
           DEC_TMEM_LD16(tmem + ((uint32_t)(quad * 32) << 16) + (ab * kDecGroups + g) * NTOK + 16u * c, part);
           tmem_ld_wait();
@@ -315,24 +450,37 @@ __global__ void __launch_bounds__(kThreads, 1)
           __syncwarp();
           if (lane == 0) mbar_arrive(&bars->acc_empty[ab]);
         }
-        if (o_ok) {
+        if (owner) {
+          if (!whole) {
+            if constexpr (kEarly) {
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const int t = 16 * c + j;
-            if (t < n) {
-              const float a = acc[j];
-              const float v = a * sxs[t] * swo;        // consecutive o across the warp: coalesced stores
-              y[(int64_t)t * d_out + o] = v;
-              if (acc_out) acc_out[(int64_t)t * d_out + o] = __float2int_rn(a * kAccScale);
-              const float e = yr[t] - v;
-              s_run += yr[t] * yr[t];
-              e_run += e * e;
+              for (int j = 0; j < 16; ++j) acc[j] += ext[16 * c + j];
+            } else {
+              for (int p = cf + 1; p <= cl; ++p) {
+                const float* src = slice_of(p);
+#pragma unroll
+                for (int j = 0; j < 16; ++j) acc[j] += __ldcg(src + (16 * c + j) * UM);
+              }
             }
           }
+          if (o_ok) {
+#pragma unroll
+            for (int j = 0; j < 16; ++j)
+              if (16 * c + j < n) emit(16 * c + j, acc[j]);
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 16; ++j) __stcg(my_slice + (16 * c + j) * UM, acc[j]);
         }
+      }
+      if (!owner) {                                    // a non-owner part: stored; count it
+        __threadfence();
+        __syncwarp();
+        if (lane == 0) atomicAdd(cnt, 1u);
       }
       sig = f2_add(sig, s_run);
       err = f2_add(err, e_run);
+      sb = se;
     }
     if (y_ref) {
       // the four warps' sums meet in shared memory; one warp hands the CTA's pair to the slot
@@ -387,6 +535,28 @@ size_t smem_bytes(int ntok, int num_ks, int sp) {
   return 1024 + tok_bytes(ntok, num_ks) + (size_t)sp * kPkStage + sizeof(DecBars) + 32 * sizeof(float);
 }
 
+// Whether one CTA per SM of the kernel is resident at once on this device under a cooperative launch
+// (checked once per token count; the grid never exceeds the SM count).
+template <int NTOK>
+bool coop_fits(size_t smem) {
+  static int ok = -1;
+  static std::mutex mu;
+  std::lock_guard<std::mutex> lock(mu);
+  if (ok < 0) {
+    int dev = 0, coop = 0, blocks = 0;
+    ok = cudaGetDevice(&dev) == cudaSuccess &&
+         cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) == cudaSuccess && coop &&
+         cudaFuncSetAttribute(w4a4_gemm_decode_tc_kernel<NTOK, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)kSmemBudget + 4096) == cudaSuccess &&
+         cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks, w4a4_gemm_decode_tc_kernel<NTOK, true>, kThreads,
+                                                       kSmemBudget + 4096) == cudaSuccess &&
+         blocks >= 1;
+    cudaGetLastError();
+  }
+  (void)smem;
+  return ok == 1;
+}
+
 template <int NTOK>
 cudaError_t launch_ntok(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
                         int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, const float* y_ref, double* sums3,
@@ -411,17 +581,30 @@ cudaError_t launch_ntok(const uint8_t* xq, const float* sx, const uint8_t* wq, c
   {
     std::lock_guard<std::mutex> lock(mu);
     if (smem > configured) {
-      cudaError_t e = cudaFuncSetAttribute(w4a4_gemm_decode_tc_kernel<NTOK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           (int)smem);
+      cudaError_t e = cudaFuncSetAttribute(w4a4_gemm_decode_tc_kernel<NTOK, false>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(w4a4_gemm_decode_tc_kernel<NTOK, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)smem);
       if (e != cudaSuccess) return e;
       configured = smem;
     }
   }
   const int64_t units = (d_out + UM - 1) / UM;
-  const int64_t sms = num_sms();
-  const unsigned grid = (unsigned)(units < sms ? units : sms);
+  const int64_t sms = num_sms() < kDecMaxGrid ? num_sms() : kDecMaxGrid;
+  // Stream-K over all (unit, K step) steps when there are more units than SMs: every CTA's range is
+  // then at least one unit long, so no CTA lies inside a unit and every part of a cut unit other
+  // than the owner's is the head of its CTA's range, done early.  With fewer units than SMs a range
+  // would be shorter than a unit; CTAs inside a unit finish together with the unit's owner, and the
+  // exchange through global memory then sits on the tail (measured at 16 tokens, 4096 -> 14336:
+  // 15.8 us on 152 CTAs against 12.8 us for whole units on 112).  Whole units per CTA in that case.
+  const int split = units > sms && units <= kDecMaxUnits && coop_fits<NTOK>(smem) ? 1 : 0;
+  const int64_t work = split ? units * num_ks : units;
+  const unsigned grid = (unsigned)(work < sms ? work : sms);
   if (grid > (unsigned)kSqnrMaxCtas) return cudaErrorInvalidConfiguration;
   const int slot = y_ref ? next_sqnr_slot() : 0;
+  static std::atomic<unsigned> next_part{0};
+  const int part_slot = split ? (int)(next_part.fetch_add(1, std::memory_order_relaxed) % kDecSlots) : 0;
   note_launch();
   cudaLaunchConfig_t cfg;
   memset(&cfg, 0, sizeof(cfg));
@@ -429,11 +612,16 @@ cudaError_t launch_ntok(const uint8_t* xq, const float* sx, const uint8_t* wq, c
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
-  cudaLaunchAttribute attrs[1] = {pdl_attr()};
+  cudaLaunchAttribute attrs[2] = {pdl_attr(), {}};
+  attrs[1].id = cudaLaunchAttributeCooperative;       // the owners of cut units wait for the other parts
+  attrs[1].val.cooperative = 1;
   cfg.attrs = attrs;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, w4a4_gemm_decode_tc_kernel<NTOK>, map, xq, sx, sw, (int)n, (int)d_in, (int)d_out, sp,
-                            y, acc_out, y_ref, sums3, slot, status);
+  cfg.numAttrs = split ? 2 : 1;
+  if (split)
+    return cudaLaunchKernelEx(&cfg, w4a4_gemm_decode_tc_kernel<NTOK, true>, map, xq, sx, sw, (int)n, (int)d_in,
+                              (int)d_out, sp, y, acc_out, y_ref, sums3, slot, part_slot, status);
+  return cudaLaunchKernelEx(&cfg, w4a4_gemm_decode_tc_kernel<NTOK, false>, map, xq, sx, sw, (int)n, (int)d_in,
+                            (int)d_out, sp, y, acc_out, y_ref, sums3, slot, part_slot, status);
 }
 
 }  // namespace

@@ -236,6 +236,9 @@ GEMM_SHAPES = [
     (1, 64, 8), (5, 160, 100), (17, 96, 33), (16, 4096, 520), (32, 384, 300), (8, 8192, 200),
     (24, 2048, 1000), (2, 1024, 17), (3, 4096, 20000), (20, 2048, 40000), (9, 8192, 12000),
     (16, 9216, 300), (32, 4608, 260),
+    # more 128-row units than SMs: the (unit, K step) sequence cut into equal ranges (stream-K), units
+    # cut between CTAs combined exactly; K steps per row not a multiple of the four decode groups
+    (16, 1536, 20000), (32, 4608, 19500),
     (3, 12288, 100),                                  # n <= 32, tokens too large for shared memory: mma.sync
     (33, 128, 256), (128, 256, 256), (129, 160, 300), (300, 384, 520), (257, 4096, 64),  # tcgen05 path
     (512, 1024, 1024), (1024, 512, 6144),                                                # ... several tiles per pair
