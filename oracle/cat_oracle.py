@@ -44,28 +44,92 @@ QMAX4 = 7  # largest INT4 code of the restricted symmetric grid
 # channel, round-to-nearest).
 # ---------------------------------------------------------------------------------------------
 
-def quantize_rows_symmetric(V: np.ndarray, bits: int = 4):
+def quantize_rows_symmetric(V: np.ndarray, bits: int = 4, ratio: Optional[np.ndarray] = None):
     """Quantize every row of ``V`` on its own symmetric uniform grid.
 
-    Returns ``(q, s, pre)``: integer codes (int64), the per-row step ``s = max|v| / qmax`` and
-    the pre-rounding values ``v / s = qmax * v / max|v|`` (float64).  An all-zero row gets
-    ``s = 0`` and codes 0.
+    Returns ``(q, s, pre)``: integer codes (int64), the per-row step ``s = a / qmax`` with
+    ``a = max|v|`` (times the row's clip ratio when ``ratio`` is given, as chosen by the weight
+    range search below) and the pre-rounding values ``v / s = qmax * v / a`` (float64).  An
+    all-zero row gets ``s = 0`` and codes 0.
 
-    The code is ``clamp(round_half_even(qmax * v / max|v|), -qmax, qmax)``, evaluated in float64
-    as ``(qmax * v) / max|v|``.  For values with at most 24 significant bits (bf16 or fp32 inputs,
-    e.g. weights or activations under T = I) the product is exact and the quotient correctly
-    rounded, so a real tie (a quotient of exactly m + 1/2) stays an exact tie and is broken to
-    even, and every other quotient lies at least 2^-29 away from a tie, far beyond float64's
-    rounding; the code is then the exact round-to-nearest of the definition."""
+    The code is ``clamp(round_half_even(qmax * v / a), -qmax, qmax)``, evaluated in float64
+    as ``(qmax * v) / a``.  For values with at most 24 significant bits (bf16 or fp32 inputs,
+    e.g. weights or activations under T = I) and ``a = max|v|`` the product is exact and the
+    quotient correctly rounded, so a real tie (a quotient of exactly m + 1/2) stays an exact tie
+    and is broken to even, and every other quotient lies at least 2^-29 away from a tie, far
+    beyond float64's rounding; the code is then the exact round-to-nearest of the definition."""
     V = np.asarray(V, dtype=np.float64)
     qmax = 2 ** (bits - 1) - 1
     a = np.max(np.abs(V), axis=1) if V.shape[1] else np.zeros(V.shape[0])
+    if ratio is not None:
+        a = a * np.asarray(ratio, dtype=np.float64)
     s = a / qmax
     pre = np.zeros_like(V)
     nz = a > 0
     pre[nz] = (qmax * V[nz]) / a[nz, None]
     q = np.clip(np.rint(pre), -qmax, qmax).astype(np.int64)
     return q, s, pre
+
+
+def quantize_rows_asymmetric(V: np.ndarray, bits: int = 4):
+    """Per-row asymmetric uniform round-to-nearest quantizer (Sec. 6: activations are quantized
+    dynamically per token, asymmetrically; Lemma 2: asymmetric range r = max - min, N(b) = 2^b - 1
+    intervals).  Reading of the details the paper leaves open (the usual integer-zero-point grid):
+    the range includes zero, ``lo = min(min v, 0)``, ``hi = max(max v, 0)``; the step is
+    ``s = (hi - lo) / N``; the zero point is the integer ``z = round(-lo / s)``; the code is
+    ``q = clamp(round(v / s) + z, 0, N)``, so ``Q(v) = s (q - z)`` and zero is exact.  Roundings are
+    half to even; the quotients are evaluated in float64 as ``(N v) / (hi - lo)`` and
+    ``(N (-lo)) / (hi - lo)``.  Returns ``(q, s, z, pre)`` with ``pre = N v / (hi - lo)``.  An
+    all-zero row gets ``s = 0``, ``z = 0`` and codes 0."""
+    V = np.asarray(V, dtype=np.float64)
+    N = 2 ** bits - 1
+    if V.shape[1]:
+        lo = np.minimum(np.min(V, axis=1), 0.0)
+        hi = np.maximum(np.max(V, axis=1), 0.0)
+    else:
+        lo = hi = np.zeros(V.shape[0])
+    r = hi - lo
+    s = r / N
+    nz = r > 0
+    pre = np.zeros_like(V)
+    pre[nz] = (N * V[nz]) / r[nz, None]
+    z = np.zeros(V.shape[0], dtype=np.int64)
+    z[nz] = np.rint((N * -lo[nz]) / r[nz]).astype(np.int64)
+    q = np.clip(np.rint(pre) + z[:, None], 0, N).astype(np.int64)
+    q[~nz] = 0
+    return q, s, z, pre
+
+
+def dequantize_rows_asymmetric(q: np.ndarray, s: np.ndarray, z: np.ndarray) -> np.ndarray:
+    """``Q(v) = s (q - z)`` per row."""
+    return (q.astype(np.float64) - z[:, None]) * s[:, None]
+
+
+def weight_range_lp(W: np.ndarray, bits: int = 4, norm: float = 2.4, grid: int = 100,
+                    maxshrink: float = 0.8) -> np.ndarray:
+    """Per-output-channel range search by the L_p error (Sec. 6: weight ranges are set with the
+    L_2.4 norm, following GPTQ).  Candidates shrink the row's range, ``a_i = (1 - i / grid) max|w|``
+    for ``i = 0 .. maxshrink * grid - 1``; each is scored by ``sum_j |w_j - s_i q_ij|^norm`` with
+    ``s_i = a_i / qmax`` and ``q_ij = clamp(round(w_j / s_i), -qmax, qmax)``; the first candidate (the
+    largest range) with the smallest score wins.  Returns the chosen ratio per row (1 for an
+    all-zero row)."""
+    W = np.asarray(W, dtype=np.float64)
+    qmax = 2 ** (bits - 1) - 1
+    amax = np.max(np.abs(W), axis=1)
+    best = np.full(W.shape[0], np.inf)
+    ratio = np.ones(W.shape[0])
+    for i in range(int(round(maxshrink * grid))):
+        p = 1.0 - i / grid
+        a = amax * p
+        s = a / qmax
+        nz = a > 0
+        q = np.zeros_like(W)
+        q[nz] = np.clip(np.rint((qmax * W[nz]) / a[nz, None]), -qmax, qmax)
+        err = np.sum(np.abs(W - q * s[:, None]) ** norm, axis=1)
+        better = err < best
+        best[better] = err[better]
+        ratio[better] = p
+    return ratio
 
 
 def dequantize_rows(q: np.ndarray, s: np.ndarray) -> np.ndarray:
@@ -243,12 +307,14 @@ class PreparedWeights:
     qw: np.ndarray         # int64 codes [d_out, d_in]
     sw: np.ndarray         # per-output-channel steps [d_out]
     pre_w: np.ndarray      # pre-rounding values
+    ratio: Optional[np.ndarray] = None   # per-row clip ratio of the L_p range search (None: max range)
 
 
 def prepare_weights(W: np.ndarray, kind: str, k: int, X_calib: Optional[np.ndarray] = None,
-                    signs: Optional[np.ndarray] = None, Sigma_x_blocks: Optional[np.ndarray] = None
-                    ) -> PreparedWeights:
-    """Offline part: calibration statistics, transform, ``W T^{-1}`` and its per-channel INT4 codes."""
+                    signs: Optional[np.ndarray] = None, Sigma_x_blocks: Optional[np.ndarray] = None,
+                    bits: int = 4, w_range: str = "max") -> PreparedWeights:
+    """Offline part: calibration statistics, transform, ``W T^{-1}`` and its per-channel b-bit
+    symmetric codes; ``w_range`` = "max" (the row maximum) or "l2.4" (the L_2.4 range search, Sec. 6)."""
     W = np.asarray(W, dtype=np.float64)
     d = W.shape[1]
     Sx = Sw = None
@@ -260,8 +326,9 @@ def prepare_weights(W: np.ndarray, kind: str, k: int, X_calib: Optional[np.ndarr
         Sw = weight_autocorr_blocks(W, k)
     T, Ti = build_transform(kind, d, k, Sx, Sw, signs)
     Wt = apply_weight_transform(W, Ti)
-    qw, sw, pre_w = quantize_rows_symmetric(Wt)
-    return PreparedWeights(T=T, Tinv=Ti, Wt=Wt, qw=qw, sw=sw, pre_w=pre_w)
+    ratio = weight_range_lp(Wt, bits) if w_range == "l2.4" else None
+    qw, sw, pre_w = quantize_rows_symmetric(Wt, bits, ratio=ratio)
+    return PreparedWeights(T=T, Tinv=Ti, Wt=Wt, qw=qw, sw=sw, pre_w=pre_w, ratio=ratio)
 
 
 @dataclasses.dataclass
@@ -270,27 +337,40 @@ class ActCodes:
     qx: np.ndarray        # int64 codes [n, d_in]
     sx: np.ndarray        # per-token steps [n]
     pre_x: np.ndarray
+    zx: Optional[np.ndarray] = None   # per-token zero points (asymmetric), else None
 
 
-def transform_quantize_act(X: np.ndarray, T_blocks: np.ndarray) -> ActCodes:
-    """Online part, first half: ``x' = T x`` and its per-token INT4 codes."""
+def transform_quantize_act(X: np.ndarray, T_blocks: np.ndarray, bits: int = 4,
+                           asymmetric: bool = False) -> ActCodes:
+    """Online part, first half: ``x' = T x`` and its per-token b-bit codes (symmetric, or the
+    asymmetric per-token quantizer of Sec. 6)."""
     Xt = apply_act_transform(X, T_blocks)
-    qx, sx, pre = quantize_rows_symmetric(Xt)
+    if asymmetric:
+        qx, sx, zx, pre = quantize_rows_asymmetric(Xt, bits)
+        return ActCodes(Xt=Xt, qx=qx, sx=sx, pre_x=pre, zx=zx)
+    qx, sx, pre = quantize_rows_symmetric(Xt, bits)
     return ActCodes(Xt=Xt, qx=qx, sx=sx, pre_x=pre)
 
 
-def w4a4_linear(qx, sx, qw, sw):
-    """Online part, second half: integer GEMM and dequantization.  Returns ``(acc, y_hat)``."""
+def w4a4_linear(qx, sx, qw, sw, zx=None):
+    """Online part, second half: integer GEMM and dequantization.  Returns ``(acc, y_hat)`` with
+    ``acc[t, o] = sum_i (qx[t, i] - zx[t]) qw[o, i]`` (``zx`` = 0 for symmetric activations); the name
+    stays from the 4-bit layer, the arithmetic holds for every bit width."""
+    qx = np.asarray(qx, dtype=np.int64)
+    if zx is not None:
+        qx = qx - np.asarray(zx, dtype=np.int64)[:, None]
     acc = int_gemm(qx, qw)
     return acc, dequantize_output(acc, sx, sw)
 
 
 def cat_layer(X: np.ndarray, W: np.ndarray, kind: str, k: int, X_calib: Optional[np.ndarray] = None,
-              signs: Optional[np.ndarray] = None) -> Dict[str, object]:
-    """Every step of the layer, in the paper's order, returning all intermediates."""
-    pw = prepare_weights(W, kind, k, X_calib=X_calib, signs=signs)
-    ac = transform_quantize_act(X, pw.T)
-    acc, y_hat = w4a4_linear(ac.qx, ac.sx, pw.qw, pw.sw)
+              signs: Optional[np.ndarray] = None, bits_x: int = 4, bits_w: int = 4, act_asym: bool = False,
+              w_range: str = "max") -> Dict[str, object]:
+    """Every step of the layer, in the paper's order, returning all intermediates (W{bits_w}A{bits_x};
+    Sec. 6's set-up is ``act_asym=True, w_range="l2.4"``)."""
+    pw = prepare_weights(W, kind, k, X_calib=X_calib, signs=signs, bits=bits_w, w_range=w_range)
+    ac = transform_quantize_act(X, pw.T, bits=bits_x, asymmetric=act_asym)
+    acc, y_hat = w4a4_linear(ac.qx, ac.sx, pw.qw, pw.sw, zx=ac.zx)
     y = linear(X, W)
     sig, err = sqnr_sums(y, y_hat)
     return dict(prep=pw, act=ac, acc=acc, y_hat=y_hat, y=y, sig=sig, err=err,

@@ -468,3 +468,145 @@ def test_cat_improves_sqnr_on_outlier_layer():
     assert res["cat"]["sqnr_db"] > res["rht"]["sqnr_db"]
     for r in res.values():
         assert np.linalg.norm(r["prep"].Wt @ np.eye(256)) > 0
+
+
+# ------------------------------------------------------------------------------------------
+# Asymmetric per-token quantizer (Sec. 6 set-up; Lemma 2 asymmetric range)
+# ------------------------------------------------------------------------------------------
+
+def _read_asym_golden():
+    cases = []
+    with open(os.path.join(GOLDEN, "quantizer_asym_rows.txt")) as f:
+        for line in f:
+            line = line.strip()
+            if not line or line.startswith("#"):
+                continue
+            bits, row, s, z, codes = [p.strip() for p in line.split("|")]
+            num, _, den = s.partition("/")
+            cases.append((int(bits), np.array([float(v) for v in row.split()]), float(Fraction(num) / Fraction(den or "1")),
+                          int(z), np.array([int(v) for v in codes.split()])))
+    return cases
+
+
+@pytest.mark.parametrize("case", range(6))
+def test_asymmetric_quantizer_hand_worked_rows(case):
+    bits, row, s_exp, z_exp, q_exp = _read_asym_golden()[case]
+    q, s, z, pre = O.quantize_rows_asymmetric(row[None, :], bits)
+    assert s[0] == s_exp and z[0] == z_exp
+    np.testing.assert_array_equal(q[0], q_exp)
+
+
+@pytest.mark.parametrize("bits", [2, 4, 8])
+def test_asymmetric_quantizer_range_and_error_bound(bits):
+    rng = _rng(40 + bits)
+    V = rng.standard_normal((300, 77)) * np.exp(rng.standard_normal((300, 1)))
+    V[5] = np.abs(V[5]) + 1.0            # all positive (ReLU-like)
+    V[6] = -np.abs(V[6])                 # all non-positive
+    V[7] = 0.0
+    N = 2 ** bits - 1
+    q, s, z, pre = O.quantize_rows_asymmetric(V, bits)
+    assert q.min() >= 0 and q.max() <= N
+    Qv = O.dequantize_rows_asymmetric(q, s, z)
+    # every value of the (zero-including) range is within half a step: no clipping
+    assert np.all(np.abs(V - Qv) <= s[:, None] / 2 * (1 + 1e-12) + 1e-300)
+    # zero is on the grid, and the extremes of a row use the extreme codes
+    assert np.all((z >= 0) & (z <= N))
+    np.testing.assert_array_equal(O.dequantize_rows_asymmetric(z[:, None], s, z), 0.0)
+    pos, neg = V.max(axis=1) > 0, V.min(axis=1) < 0
+    assert np.all(q[pos].max(axis=1) == N) and np.all(q[neg].min(axis=1) == 0)
+    assert s[7] == 0 and np.all(q[7] == 0)
+    # the step is the asymmetric range over N intervals (Lemma 2), the range taken with zero
+    lo, hi = np.minimum(V.min(axis=1), 0), np.maximum(V.max(axis=1), 0)
+    np.testing.assert_allclose(s, (hi - lo) / N, rtol=1e-15)
+
+
+def test_asymmetric_beats_symmetric_on_shifted_data_only():
+    """Sec. 2 (Concentration): asymmetric quantization helps a lot for shifted data (after a ReLU)
+    and little for zero-centred data.  Here on the activation side of a layer at 4 bits."""
+    rng = _rng(44)
+    W = rng.standard_normal((64, 96)) * 0.05
+    Xc = rng.standard_normal((4000, 96))             # zero-centred
+    Xr = np.maximum(Xc, 0.0) + 0.05                  # shifted, one-sided
+    def act_sqnr(X, asym):
+        if asym:
+            q, s, z, _ = O.quantize_rows_asymmetric(X, 4)
+            Xq = O.dequantize_rows_asymmetric(q, s, z)
+        else:
+            q, s, _ = O.quantize_rows_symmetric(X, 4)
+            Xq = O.dequantize_rows(q, s)
+        return O.sqnr_db(O.linear(X, W), O.linear(Xq, W))
+    assert abs(act_sqnr(Xc, True) - act_sqnr(Xc, False)) < 1.5
+    assert act_sqnr(Xr, True) > act_sqnr(Xr, False) + 4.0
+
+
+# ------------------------------------------------------------------------------------------
+# L_2.4 weight range search (Sec. 6, following GPTQ)
+# ------------------------------------------------------------------------------------------
+
+def test_weight_range_search_properties():
+    rng = _rng(45)
+    W = rng.standard_normal((50, 128)) * 0.02
+    W[3, 7] = 2.0                                   # one outlier 100x the rest: clipping it would cost more
+    W[4] = 0.0                                      # zero row: every candidate scores 0 -> ratio 1
+    W[5] = np.repeat([-7.0, -3.0, 0.0, 2.0, 7.0], 26)[:128] * 0.125   # every value on the ratio-1 grid
+    r = O.weight_range_lp(W, 4)
+    assert r.shape == (50,) and np.all((r > 0.2) & (r <= 1.0))
+    assert r[4] == 1.0 and r[5] == 1.0              # zero error at ratio 1 is the unique minimum / a tie
+    # the chosen range never scores worse than the full range (ratio 1 is a candidate)
+    def score(row, ratio, bits=4, p=2.4):
+        qmax = 2 ** (bits - 1) - 1
+        s = ratio * np.max(np.abs(row)) / qmax
+        q = np.clip(np.round(row / s), -qmax, qmax) if s > 0 else 0 * row
+        return np.sum(np.abs(row - q * s) ** p)
+    for i in range(50):
+        if i == 4:
+            continue
+        assert score(W[i], r[i]) <= score(W[i], 1.0) * (1 + 1e-12)
+    # Gaussian rows at 4 bits clip (the L_2.4 optimum lies inside the max range); the outlier row keeps
+    # its full range (clipping the outlier costs more than rounding the small values to zero)
+    assert np.median(r[6:]) < 1.0 and r[3] == 1.0
+    # scale invariance: a power-of-two scale of a row leaves the chosen ratio
+    np.testing.assert_array_equal(O.weight_range_lp(W * 8.0, 4), r)
+    # codes at the chosen ratio are clamped to the grid
+    q, s, _ = O.quantize_rows_symmetric(W, 4, ratio=r)
+    assert q.min() >= -7 and q.max() <= 7
+    assert q[3, 7] == 7 and np.all(q[3, np.arange(128) != 7] == 0)
+
+
+def test_l24_range_improves_weight_sqnr_at_4_bits():
+    """Weight-only SQNR with the L_2.4 range is at least that of the max range (Sec. 6 uses it)."""
+    rng = _rng(46)
+    W = rng.standard_t(5, (256, 128)) * 0.02
+    X = rng.standard_normal((2000, 128))
+    def w_sqnr(ratio):
+        q, s, _ = O.quantize_rows_symmetric(W, 4, ratio=ratio)
+        return O.sqnr_db(O.linear(X, W), O.linear(X, O.dequantize_rows(q, s)))
+    assert w_sqnr(O.weight_range_lp(W, 4)) >= w_sqnr(None) + 0.5
+
+
+# ------------------------------------------------------------------------------------------
+# Bit widths of the whole layer (Sec. 2: ~6 dB per bit; Fig. 1, Fig. 6: W4A4 vs W6A6)
+# ------------------------------------------------------------------------------------------
+
+def test_layer_bit_widths_gain_about_6db_per_bit():
+    rng = _rng(47)
+    X = rng.standard_normal((3000, 64))
+    W = rng.standard_normal((48, 64)) * 0.05
+    sq = {b: O.cat_layer(X, W, "identity", 32, bits_x=b, bits_w=b)["sqnr_db"] for b in (4, 6, 8)}
+    assert 10.5 < sq[6] - sq[4] < 13.5
+    assert 10.5 < sq[8] - sq[6] < 13.5
+    w4a8 = O.cat_layer(X, W, "identity", 32, bits_x=8, bits_w=4)["sqnr_db"]
+    assert sq[4] < w4a8 < sq[8]
+
+
+def test_layer_asymmetric_accumulators_match_dequantized_product():
+    """With asymmetric activations the integer path sum (q_x - z) q_w times the steps equals the
+    product of the dequantized operands (Sec. 3, Eq. 5)."""
+    rng = _rng(48)
+    X = rng.standard_normal((70, 64)) + 0.7
+    W = rng.standard_normal((33, 64)) * 0.1
+    r = O.cat_layer(X, W, "identity", 16, bits_x=4, bits_w=4, act_asym=True, w_range="l2.4")
+    ac, pw = r["act"], r["prep"]
+    Xq = O.dequantize_rows_asymmetric(ac.qx, ac.sx, ac.zx)
+    Wq = O.dequantize_rows(pw.qw, pw.sw)
+    np.testing.assert_allclose(r["y_hat"], Xq @ Wq.T, rtol=1e-12, atol=1e-12)
