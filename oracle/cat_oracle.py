@@ -44,29 +44,33 @@ QMAX4 = 7  # largest INT4 code of the restricted symmetric grid
 # channel, round-to-nearest).
 # ---------------------------------------------------------------------------------------------
 
-def quantize_rows_symmetric(V: np.ndarray, bits: int = 4, ratio: Optional[np.ndarray] = None):
+RANGE_GRID = 100   # the L_2.4 search's candidate ranges are max|w| (RANGE_GRID - i) / RANGE_GRID
+
+
+def quantize_rows_symmetric(V: np.ndarray, bits: int = 4, shrink: Optional[np.ndarray] = None):
     """Quantize every row of ``V`` on its own symmetric uniform grid.
 
-    Returns ``(q, s, pre)``: integer codes (int64), the per-row step ``s = a / qmax`` with
-    ``a = max|v|`` (times the row's clip ratio when ``ratio`` is given, as chosen by the weight
-    range search below) and the pre-rounding values ``v / s = qmax * v / a`` (float64).  An
-    all-zero row gets ``s = 0`` and codes 0.
+    Returns ``(q, s, pre)``: integer codes (int64), the per-row step ``s = a / qmax`` and the
+    pre-rounding values ``v / s = qmax * v / a`` (float64), where ``a = max|v|`` or, when the row's
+    candidate index ``shrink[r] = i`` of the weight range search is given, the shrunk range
+    ``a = max|v| (G - i) / G`` (G = RANGE_GRID).  An all-zero row gets ``s = 0`` and codes 0.
 
-    The code is ``clamp(round_half_even(qmax * v / a), -qmax, qmax)``, evaluated in float64
-    as ``(qmax * v) / a``.  For values with at most 24 significant bits (bf16 or fp32 inputs,
-    e.g. weights or activations under T = I) and ``a = max|v|`` the product is exact and the
-    quotient correctly rounded, so a real tie (a quotient of exactly m + 1/2) stays an exact tie
-    and is broken to even, and every other quotient lies at least 2^-29 away from a tie, far
-    beyond float64's rounding; the code is then the exact round-to-nearest of the definition."""
+    The code is ``clamp(round_half_even(qmax * v / a), -qmax, qmax)``, evaluated in float64 as
+    ``(G qmax v) / (max|v| (G - i))``.  For values with at most 24 significant bits (bf16 or fp32
+    inputs, e.g. weights or activations under T = I) both operands are exact and the quotient is
+    correctly rounded, so a real tie (a quotient of exactly m + 1/2) stays an exact tie and is broken
+    to even, and every other quotient lies far beyond float64's rounding from a tie; the code is then
+    the exact round-to-nearest of the definition."""
     V = np.asarray(V, dtype=np.float64)
     qmax = 2 ** (bits - 1) - 1
-    a = np.max(np.abs(V), axis=1) if V.shape[1] else np.zeros(V.shape[0])
-    if ratio is not None:
-        a = a * np.asarray(ratio, dtype=np.float64)
+    amax = np.max(np.abs(V), axis=1) if V.shape[1] else np.zeros(V.shape[0])
+    keep = np.full(V.shape[0], RANGE_GRID, dtype=np.float64) if shrink is None else \
+        RANGE_GRID - np.asarray(shrink, dtype=np.float64)
+    a = amax if shrink is None else amax * keep / RANGE_GRID
     s = a / qmax
     pre = np.zeros_like(V)
-    nz = a > 0
-    pre[nz] = (qmax * V[nz]) / a[nz, None]
+    nz = amax > 0
+    pre[nz] = (RANGE_GRID * qmax * V[nz]) / (amax[nz] * keep[nz])[:, None]
     q = np.clip(np.rint(pre), -qmax, qmax).astype(np.int64)
     return q, s, pre
 
@@ -105,36 +109,32 @@ def dequantize_rows_asymmetric(q: np.ndarray, s: np.ndarray, z: np.ndarray) -> n
     return (q.astype(np.float64) - z[:, None]) * s[:, None]
 
 
-def weight_range_lp(W: np.ndarray, bits: int = 4, norm: float = 2.4, grid: int = 100,
-                    maxshrink: float = 0.8) -> np.ndarray:
-    """Per-output-channel range search by the L_p error (Sec. 6: weight ranges are set with the
-    L_2.4 norm, following GPTQ).  Candidates shrink the row's range, ``a_i = (1 - i / grid) max|w|``
-    for ``i = 0 .. maxshrink * grid - 1``; each is scored by ``sum_j |w_j - s_i q_ij|^norm`` with
-    ``s_i = a_i / qmax`` and ``q_ij = clamp(round(w_j / s_i), -qmax, qmax)``; the first candidate (the
-    largest range) with the smallest score wins.  Returns the chosen ratio per row (1 for an
-    all-zero row)."""
-    W = np.asarray(W, dtype=np.float64)
-    qmax = 2 ** (bits - 1) - 1
-    amax = np.max(np.abs(W), axis=1)
-    best = np.full(W.shape[0], np.inf)
-    ratio = np.ones(W.shape[0])
-    for i in range(int(round(maxshrink * grid))):
-        p = 1.0 - i / grid
-        a = amax * p
-        s = a / qmax
-        nz = a > 0
-        q = np.zeros_like(W)
-        q[nz] = np.clip(np.rint((qmax * W[nz]) / a[nz, None]), -qmax, qmax)
-        err = np.sum(np.abs(W - q * s[:, None]) ** norm, axis=1)
-        better = err < best
-        best[better] = err[better]
-        ratio[better] = p
-    return ratio
-
-
 def dequantize_rows(q: np.ndarray, s: np.ndarray) -> np.ndarray:
     """``Q(v) = s * q`` per row."""
     return q.astype(np.float64) * s[:, None]
+
+
+def weight_range_lp(W: np.ndarray, bits: int = 4, norm: float = 2.4, maxshrink: float = 0.8,
+                    return_scores: bool = False):
+    """Per-output-channel range search by the L_p error (Sec. 6: weight ranges are set with the
+    L_2.4 norm, following GPTQ).  Candidates shrink the row's range, ``a_i = max|w| (G - i) / G``
+    for ``i = 0 .. maxshrink * G - 1`` (G = RANGE_GRID); each is scored by
+    ``sum_j |w_j - s_i q_ij|^norm`` with ``s_i = a_i / qmax`` and the codes of that range; the first
+    candidate (the largest range) with the smallest score wins.  Returns the chosen candidate index
+    per row (0 for an all-zero row), and with ``return_scores`` also every candidate's score
+    [rows, candidates]."""
+    W = np.asarray(W, dtype=np.float64)
+    best = np.full(W.shape[0], np.inf)
+    choice = np.zeros(W.shape[0], dtype=np.int64)
+    scores = []
+    for i in range(int(round(maxshrink * RANGE_GRID))):
+        q, s, _ = quantize_rows_symmetric(W, bits, shrink=np.full(W.shape[0], i))
+        err = np.sum(np.abs(W - q * s[:, None]) ** norm, axis=1)
+        scores.append(err)
+        better = err < best
+        best[better] = err[better]
+        choice[better] = i
+    return (choice, np.stack(scores, axis=1)) if return_scores else choice
 
 
 # ---------------------------------------------------------------------------------------------
@@ -307,7 +307,7 @@ class PreparedWeights:
     qw: np.ndarray         # int64 codes [d_out, d_in]
     sw: np.ndarray         # per-output-channel steps [d_out]
     pre_w: np.ndarray      # pre-rounding values
-    ratio: Optional[np.ndarray] = None   # per-row clip ratio of the L_p range search (None: max range)
+    shrink: Optional[np.ndarray] = None  # per-row candidate index of the L_p range search (None: max range)
 
 
 def prepare_weights(W: np.ndarray, kind: str, k: int, X_calib: Optional[np.ndarray] = None,
@@ -326,9 +326,9 @@ def prepare_weights(W: np.ndarray, kind: str, k: int, X_calib: Optional[np.ndarr
         Sw = weight_autocorr_blocks(W, k)
     T, Ti = build_transform(kind, d, k, Sx, Sw, signs)
     Wt = apply_weight_transform(W, Ti)
-    ratio = weight_range_lp(Wt, bits) if w_range == "l2.4" else None
-    qw, sw, pre_w = quantize_rows_symmetric(Wt, bits, ratio=ratio)
-    return PreparedWeights(T=T, Tinv=Ti, Wt=Wt, qw=qw, sw=sw, pre_w=pre_w, ratio=ratio)
+    shrink = weight_range_lp(Wt, bits) if w_range == "l2.4" else None
+    qw, sw, pre_w = quantize_rows_symmetric(Wt, bits, shrink=shrink)
+    return PreparedWeights(T=T, Tinv=Ti, Wt=Wt, qw=qw, sw=sw, pre_w=pre_w, shrink=shrink)
 
 
 @dataclasses.dataclass

@@ -547,30 +547,46 @@ def test_weight_range_search_properties():
     rng = _rng(45)
     W = rng.standard_normal((50, 128)) * 0.02
     W[3, 7] = 2.0                                   # one outlier 100x the rest: clipping it would cost more
-    W[4] = 0.0                                      # zero row: every candidate scores 0 -> ratio 1
-    W[5] = np.repeat([-7.0, -3.0, 0.0, 2.0, 7.0], 26)[:128] * 0.125   # every value on the ratio-1 grid
-    r = O.weight_range_lp(W, 4)
-    assert r.shape == (50,) and np.all((r > 0.2) & (r <= 1.0))
-    assert r[4] == 1.0 and r[5] == 1.0              # zero error at ratio 1 is the unique minimum / a tie
-    # the chosen range never scores worse than the full range (ratio 1 is a candidate)
-    def score(row, ratio, bits=4, p=2.4):
+    W[4] = 0.0                                      # zero row: every candidate scores 0 -> the full range
+    W[5] = np.repeat([-7.0, -3.0, 0.0, 2.0, 7.0], 26)[:128] * 0.125   # every value on the full range's grid
+    i = O.weight_range_lp(W, 4)
+    assert i.shape == (50,) and np.all((i >= 0) & (i < 80))
+    assert i[4] == 0 and i[5] == 0                  # zero error at the full range: the first minimum
+    # the chosen range never scores worse than the full range (it is a candidate)
+    def score(row, shrink, bits=4, p=2.4):
         qmax = 2 ** (bits - 1) - 1
-        s = ratio * np.max(np.abs(row)) / qmax
+        s = (100 - shrink) / 100 * np.max(np.abs(row)) / qmax
         q = np.clip(np.round(row / s), -qmax, qmax) if s > 0 else 0 * row
         return np.sum(np.abs(row - q * s) ** p)
-    for i in range(50):
-        if i == 4:
+    for r in range(50):
+        if r == 4:
             continue
-        assert score(W[i], r[i]) <= score(W[i], 1.0) * (1 + 1e-12)
+        assert score(W[r], i[r]) <= score(W[r], 0) * (1 + 1e-12)
     # Gaussian rows at 4 bits clip (the L_2.4 optimum lies inside the max range); the outlier row keeps
     # its full range (clipping the outlier costs more than rounding the small values to zero)
-    assert np.median(r[6:]) < 1.0 and r[3] == 1.0
-    # scale invariance: a power-of-two scale of a row leaves the chosen ratio
-    np.testing.assert_array_equal(O.weight_range_lp(W * 8.0, 4), r)
-    # codes at the chosen ratio are clamped to the grid
-    q, s, _ = O.quantize_rows_symmetric(W, 4, ratio=r)
+    assert np.median(i[6:]) > 0 and i[3] == 0
+    # scale invariance: a power-of-two scale of a row leaves the chosen range
+    np.testing.assert_array_equal(O.weight_range_lp(W * 8.0, 4), i)
+    # codes at the chosen range are clamped to the grid, and the step is the shrunk range over qmax
+    q, s, _ = O.quantize_rows_symmetric(W, 4, shrink=i)
     assert q.min() >= -7 and q.max() <= 7
     assert q[3, 7] == 7 and np.all(q[3, np.arange(128) != 7] == 0)
+    np.testing.assert_allclose(s, np.max(np.abs(W), axis=1) * (100 - i) / 100 / 7, rtol=1e-15)
+
+
+def test_shrunk_range_ties_are_exact():
+    """With a shrunk range a_i = max|w| (100 - i) / 100 the quotient qmax v / a_i is evaluated from
+    exact operands, (700 v) / (max|w| (100 - i)), so a value exactly half-way between two points of the
+    shrunk grid rounds to even.  Hand-worked: max|w| = 1, i = 30 (a_i = 0.7, step 0.1): v = 0.25 is
+    2.5 steps -> 2, v = -0.25 -> -2, v = 0.35 (not a binary fraction) ~ 3.5 steps -> by the float64
+    quotient of the stored value; v = 0.75 is 7.5 steps -> clamped to 7."""
+    q, s, pre = O.quantize_rows_symmetric(np.array([[1.0, 0.25, -0.25, 0.75, 0.0]]), 4, shrink=np.array([30]))
+    assert pre[0, 1] == 2.5 and pre[0, 2] == -2.5 and pre[0, 3] == 7.5
+    np.testing.assert_array_equal(q[0], [7, 2, -2, 7, 0])
+    assert s[0] == 0.7 / 7
+    # the same values at i = 0 (full range, step 1/7): 7 * 0.25 = 1.75 -> 2, 0.75 -> 5.25 -> 5
+    q0, _, _ = O.quantize_rows_symmetric(np.array([[1.0, 0.25, -0.25, 0.75, 0.0]]), 4, shrink=np.array([0]))
+    np.testing.assert_array_equal(q0[0], [7, 2, -2, 5, 0])
 
 
 def test_l24_range_improves_weight_sqnr_at_4_bits():
@@ -578,8 +594,8 @@ def test_l24_range_improves_weight_sqnr_at_4_bits():
     rng = _rng(46)
     W = rng.standard_t(5, (256, 128)) * 0.02
     X = rng.standard_normal((2000, 128))
-    def w_sqnr(ratio):
-        q, s, _ = O.quantize_rows_symmetric(W, 4, ratio=ratio)
+    def w_sqnr(shrink):
+        q, s, _ = O.quantize_rows_symmetric(W, 4, shrink=shrink)
         return O.sqnr_db(O.linear(X, W), O.linear(X, O.dequantize_rows(q, s)))
     assert w_sqnr(O.weight_range_lp(W, 4)) >= w_sqnr(None) + 0.5
 
