@@ -243,6 +243,74 @@ cat_status cat_block_row_stats(const void* V, cat_dtype dtype, int64_t rows, int
                                cat_stream_t stream);
 
 /*
+ * ---------------------------------------------------------------------------------------------
+ * b-bit codes as E4M3 digit planes: the bit widths of Sec. 2 ("Bit width": each bit ~6 dB; Fig. 1
+ * and Fig. 6 compare W4A4 with W6A6) and the experimental set-up of Sec. 6 (activations per token,
+ * asymmetric; weights per output channel, symmetric, range by the L_2.4 error following GPTQ).
+ *
+ * Code grids (b in 2..8):
+ *   symmetric  q = clamp(round(qmax v / a), -qmax, qmax), qmax = 2^(b-1) - 1, a = max|v| of the row
+ *              (or the L_2.4 range for weights); step s = a / qmax.
+ *   asymmetric lo = min(min v, 0), hi = max(max v, 0), N = 2^b - 1, s = (hi - lo) / N,
+ *              zero point z = round(-lo / s), q = clamp(round(v / s) + z, 0, N); Q(v) = s (q - z).
+ *   Rounding is half to even; every decision is exact for the float32 transformed value.
+ * Digit-plane format: D = cat_dp_planes(b) planes (1 for b <= 4, else 2); a code is q = d0 + 16 d1 with
+ *   symmetric d0 = ((q + 8) mod 16) - 8, d1 = (q - d0) / 16 (|d| <= 8), asymmetric d0 = q mod 16,
+ *   d1 = q div 16 (one plane: d0 = q).  Each digit is one byte, the FP8 E4M3 encoding
+ *   (d < 0) << 7 | |d|, which is exactly d * 2^-9 for |d| <= 16.  Plane p of an [R][d_in] code
+ *   matrix is the [R][d_in] byte matrix at planes + p * R * d_in.
+ * The GEMM accumulates every digit product on the FP8 tensor cores exactly; these calls need
+ * d_in <= 65536 (CAT_ERR_SHAPE otherwise) on top of the shape rules above.
+ * ---------------------------------------------------------------------------------------------
+ */
+
+/* Number of digit planes of b-bit codes (1 or 2); 0 if b is outside 2..8. */
+int32_t cat_dp_planes(int32_t bits);
+
+/*
+ * cat_transform_quantize_act_dp -- online activation path at b bits (Sec. 3 Eq. 5: x' = T x; Sec. 6:
+ * dynamic per-token quantization, symmetric or asymmetric).
+ *   x, T_blocks  as cat_transform_quantize_act.
+ *   planes       out, device [D][n][d_in] bytes (digit planes of the codes of x').
+ *   x_scale      out, device [n] float32 steps (0 for an all-zero or non-finite token).
+ *   x_zero       out, device [n] int32 zero points (asymmetric only; may be NULL when symmetric).
+ * x_scale and x_zero also serve as the row statistics' scratch while the call runs.  Runs on SIMT
+ * cores (transform, row statistics, codes: four launches).
+ */
+cat_status cat_transform_quantize_act_dp(const void* x, cat_dtype dtype, int64_t n, int64_t d_in, int32_t k,
+                                         const float* T_blocks, int32_t bits, int32_t asymmetric, uint8_t* planes,
+                                         float* x_scale, int32_t* x_zero, cat_stream_t stream);
+
+/*
+ * cat_quantize_weights_dp -- cat_quantize_weights at b bits with digit-plane output (Sec. 4 Eq. 7 and
+ * Eq. 10: the transform; Sec. 6: per-output-channel symmetric codes).
+ *   l24_range  0: a = max|w'| per row; 1: the L_2.4 range search (Sec. 6): candidates
+ *              a_i = max|w'| (100 - i) / 100, i = 0..79, scored by sum |w' - s_i q_i|^2.4 (float32 terms
+ *              summed in float64), the first smallest score wins.
+ *   planes     out, device [D][d_out][d_in] bytes; w_scale out, device [d_out] float32.
+ *   w_rowsum   optional out (NULL to skip), device [d_out] int32: sum_i q_w[o][i], the zero-point
+ *              correction that cat_linear_dp needs for asymmetric activations.
+ * Other arguments, synchronization, allocation and errors as cat_quantize_weights.
+ */
+cat_status cat_quantize_weights_dp(const void* W, cat_dtype dtype, int64_t d_out, int64_t d_in, int32_t k,
+                                   cat_tkind kind, const double* sigma_x_blocks, int64_t n_calib,
+                                   const float* rht_signs, int32_t bits, int32_t l24_range, float* T_blocks,
+                                   uint8_t* planes, float* w_scale, int32_t* w_rowsum, cat_stream_t stream);
+
+/*
+ * cat_linear_dp -- integer GEMM of digit-plane codes and dequantization (Sec. 3 Eq. 5).
+ *   acc[t][o] = sum_i (q_x[t][i] - z[t]) q_w[o][i]  (z = 0 unless asym_x), exactly;
+ *   y[t][o]   = acc * x_scale[t] * w_scale[o] (float32, device [n][d_out]);
+ *   acc_out   optional int32 [n][d_out] (NULL to skip).
+ * asym_x = 1 needs x_zero [n] and w_rowsum [d_out] (from cat_quantize_weights_dp).  tcgen05 FP8 MMAs
+ * (kind::f8f6f4) on TMA-loaded digit planes, one fp32 tensor-memory accumulator per digit weight 16^g.
+ */
+cat_status cat_linear_dp(const uint8_t* x_planes, int32_t bits_x, int32_t asym_x, const float* x_scale,
+                         const int32_t* x_zero, const uint8_t* w_planes, int32_t bits_w, const float* w_scale,
+                         const int32_t* w_rowsum, int64_t n, int64_t d_in, int64_t d_out, float* y, int32_t* acc_out,
+                         cat_stream_t stream);
+
+/*
  * cat_device_status -- synchronizes `stream`, then reads and clears the device status word.
  * Returns CAT_OK, CAT_ERR_TIMEOUT (a bounded wait in a kernel gave up and the kernel returned
  * early; its outputs are undefined) or CAT_ERR_NUMERIC (a kernel met a non-finite value; the

@@ -20,6 +20,7 @@ __all__ = [
     "CatError", "library_path", "load_library", "exported_symbols",
     "cat_calib_cov", "cat_quantize_weights", "cat_build_transform_host", "cat_transform_quantize_act",
     "cat_w4a4_linear", "cat_sqnr", "cat_device_status", "cat_version", "KIND",
+    "cat_dp_planes", "cat_transform_quantize_act_dp", "cat_quantize_weights_dp", "cat_linear_dp",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -67,6 +68,10 @@ def load_library() -> ctypes.CDLL:
         "cat_w4a4_linear_sqnr": ([P, P, P, P, I64, I64, I64, P, P, P, P], I),
         "cat_device_status": ([P, P], I),
         "cat_block_row_stats": ([P, I, I64, I64, I32, P, I, P, P, P, P], I),
+        "cat_dp_planes": ([I32], I32),
+        "cat_transform_quantize_act_dp": ([P, I, I64, I64, I32, P, I32, I32, P, P, P, P], I),
+        "cat_quantize_weights_dp": ([P, I, I64, I64, I32, I, P, I64, P, I32, I32, P, P, P, P, P], I),
+        "cat_linear_dp": ([P, I32, I32, P, P, P, I32, P, P, I64, I64, I64, P, P, P], I),
     }
     for name, (args, res) in sigs.items():
         f = getattr(lib, name)
@@ -80,7 +85,7 @@ def exported_symbols() -> list:
     """Names of the entry points declared in ``include/cat_w4a4.h``."""
     with open(_HEADER) as f:
         text = f.read()
-    return sorted(set(re.findall(r"^\s*(?:cat_status|const char\*|int|unsigned long long)\s+(cat_\w+)\s*\(", text,
+    return sorted(set(re.findall(r"^\s*(?:cat_status|const char\*|int|int32_t|unsigned long long)\s+(cat_\w+)\s*\(", text,
                                  re.M)))
 
 
@@ -312,6 +317,95 @@ def cat_block_row_stats(V: torch.Tensor, k: int, M: torch.Tensor, transpose: boo
         _ptr(V), _dtype(V), rows, d, k, _ptr(M), 1 if transpose else 0, _ptr(row_sumsq), _ptr(row_amax), _ptr(out3),
         _stream(V.device)))
     return row_sumsq, row_amax, out3
+
+
+def cat_dp_planes(bits: int) -> int:
+    """Digit planes of b-bit codes (1 for b <= 4, else 2)."""
+    return int(load_library().cat_dp_planes(int(bits)))
+
+
+def cat_transform_quantize_act_dp(x: torch.Tensor, T_blocks: torch.Tensor, k: int, bits: int, asymmetric: bool = False,
+                                  out=None):
+    """x' = T x and its per-token b-bit codes as digit planes: (planes uint8 [D, n, d_in], x_scale float32 [n],
+    x_zero int32 [n] or None)."""
+    _need(x, "x")
+    n, d_in = x.shape
+    D = cat_dp_planes(bits)
+    if D == 0:
+        raise ValueError("bits must be in 2..8")
+    if out is None:
+        out = (torch.empty((D, n, d_in), dtype=torch.uint8, device=x.device),
+               torch.empty((n,), dtype=torch.float32, device=x.device),
+               torch.empty((n,), dtype=torch.int32, device=x.device) if asymmetric else None)
+    planes, sx, zx = out
+    _expect(T_blocks, "T_blocks", torch.float32, (d_in // k, k, k), x.device)
+    _expect(planes, "planes", torch.uint8, (D, n, d_in), x.device)
+    _expect(sx, "x_scale", torch.float32, (n,), x.device)
+    if asymmetric:
+        _expect(zx, "x_zero", torch.int32, (n,), x.device)
+    _check("cat_transform_quantize_act_dp", load_library().cat_transform_quantize_act_dp(
+        _ptr(x), _dtype(x), n, d_in, k, _ptr(T_blocks), int(bits), int(bool(asymmetric)), _ptr(planes), _ptr(sx),
+        _ptr(zx) if asymmetric else None, _stream(x.device)))
+    return planes, sx, (zx if asymmetric else None)
+
+
+def cat_quantize_weights_dp(W: torch.Tensor, k: int, kind: str, bits: int, sigma_x: Optional[torch.Tensor] = None,
+                            n_calib: int = 0, rht_signs=None, l24_range: bool = False, rowsum: bool = False):
+    """Offline weight preparation at b bits: (T_blocks float32 [d_in/k, k, k], planes uint8 [D, d_out, d_in],
+    w_scale float32 [d_out], w_rowsum int32 [d_out] or None)."""
+    _need(W, "W")
+    d_out, d_in = W.shape
+    dev = W.device
+    D = cat_dp_planes(bits)
+    if D == 0:
+        raise ValueError("bits must be in 2..8")
+    T = torch.empty((d_in // k, k, k), dtype=torch.float32, device=dev)
+    planes = torch.empty((D, d_out, d_in), dtype=torch.uint8, device=dev)
+    sw = torch.empty((d_out,), dtype=torch.float32, device=dev)
+    rs = torch.empty((d_out,), dtype=torch.int32, device=dev) if rowsum else None
+    signs = None
+    if rht_signs is not None:
+        signs = np.ascontiguousarray(np.asarray(rht_signs, dtype=np.float32))
+        if signs.shape != (d_in,):
+            raise ValueError(f"rht_signs has shape {signs.shape}, expected ({d_in},)")
+    if sigma_x is not None:
+        _expect(sigma_x, "sigma_x", torch.float64, (d_in // k, k, k), dev)
+    st = load_library().cat_quantize_weights_dp(
+        _ptr(W), _dtype(W), d_out, d_in, k, KIND[kind], _ptr(sigma_x), int(n_calib),
+        None if signs is None else signs.ctypes.data_as(ctypes.c_void_p), int(bits), int(bool(l24_range)), _ptr(T),
+        _ptr(planes), _ptr(sw), _ptr(rs), _stream(dev))
+    _check("cat_quantize_weights_dp", st)
+    return T, planes, sw, rs
+
+
+def cat_linear_dp(x_planes: torch.Tensor, bits_x: int, x_scale: torch.Tensor, w_planes: torch.Tensor, bits_w: int,
+                  w_scale: torch.Tensor, x_zero: Optional[torch.Tensor] = None, w_rowsum: Optional[torch.Tensor] = None,
+                  y: Optional[torch.Tensor] = None, acc_out: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """y[t, o] = (sum_i (q_x - z_t) q_w) * s_x[t] * s_w[o] from digit-plane codes (float32 [n, d_out])."""
+    Dx, n, d_in = x_planes.shape
+    Dw, d_out, d_in_w = w_planes.shape
+    dev = x_planes.device
+    if Dx != cat_dp_planes(bits_x) or Dw != cat_dp_planes(bits_w) or d_in_w != d_in:
+        raise ValueError("digit planes do not match the bit widths or each other")
+    asym = x_zero is not None
+    if asym and w_rowsum is None:
+        raise ValueError("asymmetric activations need w_rowsum")
+    if y is None:
+        y = torch.empty((n, d_out), dtype=torch.float32, device=dev)
+    _expect(x_planes, "x_planes", torch.uint8, (Dx, n, d_in), dev)
+    _expect(w_planes, "w_planes", torch.uint8, (Dw, d_out, d_in), dev)
+    _expect(x_scale, "x_scale", torch.float32, (n,), dev)
+    _expect(w_scale, "w_scale", torch.float32, (d_out,), dev)
+    _expect(y, "y", torch.float32, (n, d_out), dev)
+    if asym:
+        _expect(x_zero, "x_zero", torch.int32, (n,), dev)
+        _expect(w_rowsum, "w_rowsum", torch.int32, (d_out,), dev)
+    if acc_out is not None:
+        _expect(acc_out, "acc_out", torch.int32, (n, d_out), dev)
+    _check("cat_linear_dp", load_library().cat_linear_dp(
+        _ptr(x_planes), int(bits_x), int(asym), _ptr(x_scale), _ptr(x_zero), _ptr(w_planes), int(bits_w), _ptr(w_scale),
+        _ptr(w_rowsum) if asym else None, n, d_in, d_out, _ptr(y), _ptr(acc_out), _stream(dev)))
+    return y
 
 
 def cat_device_status(device: Optional[torch.device] = None) -> Tuple[int, int]:

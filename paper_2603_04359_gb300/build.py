@@ -17,7 +17,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libcatw4a4.so")
-SOURCES = ["api.cu", "calib_cov.cu", "calib_cov_tc.cu", "act_quant.cu", "act_quant_tc.cu", "gemm_tc.cu", "gemm_decode.cu", "gemm_decode_tc.cu", "sqnr.cu", "diag.cu", "transform_host.cpp"]
+SOURCES = ["api.cu", "calib_cov.cu", "calib_cov_tc.cu", "act_quant.cu", "act_quant_tc.cu", "gemm_tc.cu", "gemm_decode.cu", "gemm_decode_tc.cu", "sqnr.cu", "diag.cu", "quant_dp.cu", "gemm_dp.cu", "transform_host.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 COMMON = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-O3,-pthread", "-I", os.path.join(ROOT, "include")]
 

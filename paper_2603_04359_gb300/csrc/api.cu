@@ -23,6 +23,14 @@ cudaError_t launch_w4a4_gemm_decode(const uint8_t* xq, const float* sx, const ui
 cudaError_t launch_block_row_stats(const void* V, int dtype, int64_t rows, int64_t d, int k, const float* M,
                                    int transpose, float* row_sumsq, float* row_amax, double* out3,
                                    cudaStream_t stream);
+int dp_planes(int bits, int asym);
+size_t dp_l24_work_bytes(int64_t n);
+cudaError_t launch_transform_quantize_dp(const void* x, int dtype, int64_t n, int64_t d, int k, const float* A, int bits,
+                                         int asym, int l24, uint8_t* planes, float* scale, int32_t* zero,
+                                         int32_t* rowsum, void* work, uint32_t* status, cudaStream_t stream);
+cudaError_t launch_dp_gemm(const uint8_t* x_planes, int DX, const float* sx, const int32_t* zx, const uint8_t* w_planes,
+                           int DW, const float* sw, const int32_t* w_rowsum, int64_t n, int64_t d_in, int64_t d_out,
+                           float* y, int32_t* acc_out, uint32_t* status, cudaStream_t stream);
 }  // namespace cat
 
 namespace {
@@ -30,6 +38,9 @@ namespace {
 constexpr int kVersion = 10000;        // 1.0.0
 constexpr int64_t kMaxDecodeTokens = 32;   // n <= 32: weight-streaming kernel; else tcgen05 tiles
 constexpr int64_t kMaxDin = 262144;    // 49 * d_in < 2^24 keeps fp32 accumulation exact
+// digit planes: an accumulator sums up to 2 d_in digit products of at most 15 * 8, and the int32
+// result |sum (q_x - z) q_w| <= 255 * 127 * d_in: both bounded for d_in <= 2^16
+constexpr int64_t kMaxDinDp = 65536;
 
 // Device status word (one per device that loads the library).
 __device__ uint32_t g_device_status;
@@ -334,6 +345,140 @@ cat_status cat_quantize_weights_noalloc(const void* W, cat_dtype dtype, int64_t 
   cudaError_t e2 = cudaStreamSynchronize(s);  // host buffers and the scratch are in use until here
   if (e != cudaSuccess) return cuda_fail(e, "weight quantization");
   if (e2 != cudaSuccess) return cuda_fail(e2, "cudaStreamSynchronize");
+  return ok();
+}
+
+// ---- b-bit codes as E4M3 digit planes (bit widths; Sec. 6's asymmetric activations and L_2.4 range)
+
+int32_t cat_dp_planes(int32_t bits) { return (bits >= 2 && bits <= 8) ? (int32_t)cat::dp_planes(bits, 0) : 0; }
+
+cat_status cat_transform_quantize_act_dp(const void* x, cat_dtype dtype, int64_t n, int64_t d_in, int32_t k,
+                                         const float* T_blocks, int32_t bits, int32_t asymmetric, uint8_t* planes,
+                                         float* x_scale, int32_t* x_zero, cat_stream_t stream) {
+  if (dtype != CAT_F32 && dtype != CAT_BF16) return fail(CAT_ERR_INVALID_ARG, "unknown dtype");
+  if (bits < 2 || bits > 8) return fail(CAT_ERR_SHAPE, "bits must be in 2..8");
+  if (asymmetric != 0 && asymmetric != 1) return fail(CAT_ERR_INVALID_ARG, "asymmetric must be 0 or 1");
+  if (n < 0) return fail(CAT_ERR_SHAPE, "n must be >= 0");
+  cat_status st = check_din(d_in);
+  if (st != CAT_OK) return st;
+  if (d_in > kMaxDinDp) return fail(CAT_ERR_SHAPE, "d_in exceeds 65536 (exact digit-plane accumulation bound)");
+  if (!valid_k(k) || d_in % k != 0) return fail(CAT_ERR_SHAPE, "k must be one of 16..256 (power of two) and divide d_in");
+  if (n == 0) return ok();
+  if (!x || !T_blocks || !planes || !x_scale || (asymmetric && !x_zero)) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(x) || !aligned16(T_blocks) || !aligned16(planes) || !aligned16(x_scale) || (x_zero && !aligned16(x_zero)))
+    return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  if ((n + 63) / 64 > 0x7FFFFFFF) return fail(CAT_ERR_SHAPE, "n too large");
+  if ((st = check_device()) != CAT_OK) return st;
+  cudaError_t e;
+  uint32_t* status = status_word(&e);
+  if (!status) return cuda_fail(e, "status word");
+  e = cat::launch_transform_quantize_dp(x, (int)dtype, n, d_in, k, T_blocks, bits, asymmetric, 0, planes, x_scale,
+                                        asymmetric ? x_zero : nullptr, nullptr, nullptr, status, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cat_transform_quantize_act_dp launch");
+  return ok();
+}
+
+cat_status cat_quantize_weights_dp(const void* W, cat_dtype dtype, int64_t d_out, int64_t d_in, int32_t k,
+                                   cat_tkind kind, const double* sigma_x_blocks, int64_t n_calib,
+                                   const float* rht_signs, int32_t bits, int32_t l24_range, float* T_blocks,
+                                   uint8_t* planes, float* w_scale, int32_t* w_rowsum, cat_stream_t stream) {
+  if (dtype != CAT_F32 && dtype != CAT_BF16) return fail(CAT_ERR_INVALID_ARG, "unknown dtype");
+  if (kind != CAT_T_IDENTITY && kind != CAT_T_RHT && kind != CAT_T_CAT) return fail(CAT_ERR_INVALID_ARG, "unknown kind");
+  if (bits < 2 || bits > 8) return fail(CAT_ERR_SHAPE, "bits must be in 2..8");
+  if (l24_range != 0 && l24_range != 1) return fail(CAT_ERR_INVALID_ARG, "l24_range must be 0 or 1");
+  if (d_out <= 0 || d_out > 0x7FFFFFFF) return fail(CAT_ERR_SHAPE, "d_out must be in [1, 2^31)");
+  cat_status st = check_din(d_in);
+  if (st != CAT_OK) return st;
+  if (d_in > kMaxDinDp) return fail(CAT_ERR_SHAPE, "d_in exceeds 65536 (exact digit-plane accumulation bound)");
+  if (!valid_k(k) || d_in % k != 0) return fail(CAT_ERR_SHAPE, "k must be one of 16..256 (power of two) and divide d_in");
+  if (!W || !T_blocks || !planes || !w_scale) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (kind == CAT_T_CAT && (!sigma_x_blocks || n_calib < 1))
+    return fail(CAT_ERR_INVALID_ARG, "CAT needs sigma_x_blocks and n_calib >= 1");
+  if (kind == CAT_T_RHT && !rht_signs) return fail(CAT_ERR_INVALID_ARG, "RHT needs rht_signs");
+  if (!aligned16(W) || !aligned16(T_blocks) || !aligned16(planes) || !aligned16(w_scale) ||
+      (w_rowsum && !aligned16(w_rowsum)) || (sigma_x_blocks && !aligned16(sigma_x_blocks)))
+    return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  if ((st = check_device()) != CAT_OK) return st;
+
+  cudaStream_t s = (cudaStream_t)stream;
+  const int64_t nb = d_in / k;
+  const size_t kk = (size_t)k * k, nblk = (size_t)nb * kk;
+  std::vector<double> sx_h, sw_h;
+  cudaError_t e;
+  if (kind == CAT_T_CAT) {
+    double* sw_d = nullptr;
+    if ((e = cudaMallocAsync((void**)&sw_d, nblk * sizeof(double), s)) != cudaSuccess) return cuda_fail(e, "cudaMallocAsync");
+    uint32_t* st_word = status_word(&e);
+    if (!st_word) return cuda_fail(e, "status word");
+    e = cat::launch_calib_cov(W, (int)dtype, d_out, d_in, k, sw_d, 0, st_word, s);  // Sigma_w = W^T W blocks
+    sx_h.resize(nblk);
+    sw_h.resize(nblk);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(sx_h.data(), sigma_x_blocks, nblk * sizeof(double), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(sw_h.data(), sw_d, nblk * sizeof(double), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    cudaFreeAsync(sw_d, s);
+    if (e != cudaSuccess) return cuda_fail(e, "Sigma_w / Sigma_x readback");
+  }
+  std::vector<double> T(nblk), Ti(nblk);
+  st = cat_build_transform_host(kind, d_in, k, sx_h.empty() ? nullptr : sx_h.data(), n_calib,
+                                sw_h.empty() ? nullptr : sw_h.data(), rht_signs, T.data(), Ti.data());
+  if (st != CAT_OK) return st;
+  std::vector<float> Tf(nblk), Awf(nblk);
+  for (int64_t b = 0; b < nb; ++b)
+    for (int i = 0; i < k; ++i)
+      for (int j = 0; j < k; ++j) {
+        Tf[b * kk + (size_t)i * k + j] = (float)T[b * kk + (size_t)i * k + j];
+        Awf[b * kk + (size_t)i * k + j] = (float)Ti[b * kk + (size_t)j * k + i];
+      }
+  uint32_t* status = status_word(&e);
+  if (!status) return cuda_fail(e, "status word");
+  float* aw_d = nullptr;
+  void* work = nullptr;
+  const size_t work_bytes = l24_range ? cat::dp_l24_work_bytes(d_out) : 0;
+  if ((e = cudaMallocAsync((void**)&aw_d, nblk * sizeof(float), s)) != cudaSuccess) return cuda_fail(e, "cudaMallocAsync");
+  if (work_bytes && (e = cudaMallocAsync(&work, work_bytes, s)) != cudaSuccess) {
+    cudaFreeAsync(aw_d, s);
+    return cuda_fail(e, "cudaMallocAsync");
+  }
+  if (work_bytes) e = cudaMemsetAsync(work, 0, work_bytes, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(T_blocks, Tf.data(), nblk * sizeof(float), cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(aw_d, Awf.data(), nblk * sizeof(float), cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess)
+    e = cat::launch_transform_quantize_dp(W, (int)dtype, d_out, d_in, k, aw_d, bits, 0, l24_range, planes, w_scale,
+                                          nullptr, w_rowsum, work, status, s);
+  cudaFreeAsync(aw_d, s);
+  if (work) cudaFreeAsync(work, s);
+  cudaError_t e2 = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(e, "weight quantization (digit planes)");
+  if (e2 != cudaSuccess) return cuda_fail(e2, "cudaStreamSynchronize");
+  return ok();
+}
+
+cat_status cat_linear_dp(const uint8_t* x_planes, int32_t bits_x, int32_t asym_x, const float* x_scale,
+                         const int32_t* x_zero, const uint8_t* w_planes, int32_t bits_w, const float* w_scale,
+                         const int32_t* w_rowsum, int64_t n, int64_t d_in, int64_t d_out, float* y, int32_t* acc_out,
+                         cat_stream_t stream) {
+  if (bits_x < 2 || bits_x > 8 || bits_w < 2 || bits_w > 8) return fail(CAT_ERR_SHAPE, "bits must be in 2..8");
+  if (asym_x != 0 && asym_x != 1) return fail(CAT_ERR_INVALID_ARG, "asym_x must be 0 or 1");
+  if (n < 0 || d_out <= 0) return fail(CAT_ERR_SHAPE, "n must be >= 0 and d_out >= 1");
+  cat_status st = check_din(d_in);
+  if (st != CAT_OK) return st;
+  if (d_in > kMaxDinDp) return fail(CAT_ERR_SHAPE, "d_in exceeds 65536 (exact digit-plane accumulation bound)");
+  if (n > 0x7FFFFFFF || d_out > 0x7FFFFFFF || (n + 127) / 128 > 65535) return fail(CAT_ERR_SHAPE, "n or d_out too large");
+  if (n == 0) return ok();
+  if (!x_planes || !x_scale || !w_planes || !w_scale || !y || (asym_x && (!x_zero || !w_rowsum)))
+    return fail(CAT_ERR_INVALID_ARG, "NULL pointer (asymmetric activations need x_zero and w_rowsum)");
+  if (!aligned16(x_planes) || !aligned16(x_scale) || !aligned16(w_planes) || !aligned16(w_scale) || !aligned16(y) ||
+      (x_zero && !aligned16(x_zero)) || (w_rowsum && !aligned16(w_rowsum)) || (acc_out && !aligned16(acc_out)))
+    return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  if ((st = check_device()) != CAT_OK) return st;
+  cudaError_t e;
+  uint32_t* status = status_word(&e);
+  if (!status) return cuda_fail(e, "status word");
+  e = cat::launch_dp_gemm(x_planes, cat::dp_planes(bits_x, asym_x), x_scale, asym_x ? x_zero : nullptr, w_planes,
+                          cat::dp_planes(bits_w, 0), w_scale, asym_x ? w_rowsum : nullptr, n, d_in, d_out, y, acc_out,
+                          status, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cat_linear_dp launch");
   return ok();
 }
 
