@@ -329,9 +329,51 @@ def transform_sweep(cat, L, x, W, xc, y_ref):
         out[kind] = vals
         diag[kind] = dk
     out["diagnostics"] = diag
+    out["bits"] = bit_width_sweep(cat, L, x, W, xc, y_ref)
     status, detail = cat.cat_device_status()
     if status != 0:
         raise DeviceTimeout(f"device status 0x{detail:x} after the transform sweep")
+    return out
+
+
+BIT_CONFIGS = (  # (name, bits_x, bits_w, asymmetric activations, L_2.4 weight range)
+    ("W4A4", 4, 4, False, False), ("W4A8", 8, 4, False, False), ("W6A6", 6, 6, False, False),
+    ("W8A8", 8, 8, False, False), ("W4A4 asym+L2.4 (Sec. 6 set-up)", 4, 4, True, True))
+
+
+def bit_width_sweep(cat, L, x, W, xc, y_ref, steps=10):
+    """SQNR (dB) of the layer at other bit widths and with Sec. 6's quantizer set-up, through the
+    digit-plane path (Sec. 2 "Bit width"; Fig. 1 / Fig. 6: CAT W4A4 against W6A6), for the identity and
+    CAT at the configuration's block size; plus the digit-plane GEMM's time per call (CUDA graph of
+    `steps` launches, operands resident)."""
+    k = L.cfg.k
+    n, d_out = y_ref.shape
+    out = {"k": k, "configs": [c[0] for c in BIT_CONFIGS]}
+    sigma = cat.cat_calib_cov(xc, k)
+    for kind in ("identity", "cat"):
+        vals, ms = [], []
+        for name, bx, bw, asym, l24 in BIT_CONFIGS:
+            T, wp, sw, rs = cat.cat_quantize_weights_dp(W, k, kind, bw, sigma_x=sigma if kind == "cat" else None,
+                                                        n_calib=L.cfg.n_calib, l24_range=l24, rowsum=asym)
+            xp, sx, zx = cat.cat_transform_quantize_act_dp(x, T, k, bx, asym)
+            y = torch.empty((n, d_out), dtype=torch.float32, device=x.device)
+            call = lambda: cat.cat_linear_dp(xp, bx, sx, wp, bw, sw, x_zero=zx, w_rowsum=rs, y=y)  # noqa: E731
+            call()
+            vals.append(round(float(cat.cat_sqnr(y_ref, y)[2].item()), 3))
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                for _ in range(steps):
+                    call()
+            g.replay()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            g.replay()
+            b.record()
+            torch.cuda.synchronize()
+            ms.append(round(a.elapsed_time(b) / steps, 4))
+            del T, wp, sw, rs, xp, sx, zx, y, g
+        out[kind] = vals
+        out[kind + "_gemm_ms"] = ms
     return out
 
 
