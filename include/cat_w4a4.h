@@ -311,6 +311,18 @@ cat_status cat_linear_dp(const uint8_t* x_planes, int32_t bits_x, int32_t asym_x
                          cat_stream_t stream);
 
 /*
+ * cat_set_wait_limit_ns -- testing aid, no counterpart in the paper.  Sets, on the current device, the
+ * bound of the pipeline waits of the weight-streaming W4A4 GEMM (cat_w4a4_linear, n <= 32) and of the
+ * digit-plane GEMM (cat_linear_dp); 0 restores the default of 1 s (1e9 ns, also the largest value
+ * accepted).  A wait that exceeds its bound gives up: the kernel drains its copies and MMAs in flight
+ * (those waits keep the 1 s bound), frees its tensor memory, returns, and raises CAT_ERR_TIMEOUT in the
+ * device status word with the kernel's bit (1 << 11 weight-streaming GEMM, 1 << 13 digit-plane GEMM)
+ * and the source line of the first wait that gave up in bits 16..31.  Its outputs are then undefined.
+ * Synchronous (a blocking copy to the device); not for use while those kernels run.
+ */
+cat_status cat_set_wait_limit_ns(uint64_t ns);
+
+/*
  * cat_device_status -- synchronizes `stream`, then reads and clears the device status word.
  * Returns CAT_OK, CAT_ERR_TIMEOUT (a bounded wait in a kernel gave up and the kernel returned
  * early; its outputs are undefined) or CAT_ERR_NUMERIC (a kernel met a non-finite value; the

@@ -69,6 +69,7 @@ def load_library() -> ctypes.CDLL:
         "cat_device_status": ([P, P], I),
         "cat_block_row_stats": ([P, I, I64, I64, I32, P, I, P, P, P, P], I),
         "cat_dp_planes": ([I32], I32),
+        "cat_set_wait_limit_ns": ([ctypes.c_uint64], I),
         "cat_transform_quantize_act_dp": ([P, I, I64, I64, I32, P, I32, I32, P, P, P, P], I),
         "cat_quantize_weights_dp": ([P, I, I64, I64, I32, I, P, I64, P, I32, I32, P, P, P, P, P], I),
         "cat_linear_dp": ([P, I32, I32, P, P, P, I32, P, P, I64, I64, I64, P, P, P], I),
@@ -406,6 +407,12 @@ def cat_linear_dp(x_planes: torch.Tensor, bits_x: int, x_scale: torch.Tensor, w_
         _ptr(x_planes), int(bits_x), int(asym), _ptr(x_scale), _ptr(x_zero), _ptr(w_planes), int(bits_w), _ptr(w_scale),
         _ptr(w_rowsum) if asym else None, n, d_in, d_out, _ptr(y), _ptr(acc_out), _stream(dev)))
     return y
+
+
+def cat_set_wait_limit_ns(ns: int) -> None:
+    """Testing aid: bound (ns) of the pipeline waits of the weight-streaming and digit-plane GEMMs on the
+    current device; 0 restores the default (1 s)."""
+    _check("cat_set_wait_limit_ns", load_library().cat_set_wait_limit_ns(int(ns)))
 
 
 def cat_device_status(device: Optional[torch.device] = None) -> Tuple[int, int]:

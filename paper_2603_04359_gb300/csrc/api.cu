@@ -24,6 +24,8 @@ cudaError_t launch_block_row_stats(const void* V, int dtype, int64_t rows, int64
                                    int transpose, float* row_sumsq, float* row_amax, double* out3,
                                    cudaStream_t stream);
 int dp_planes(int bits, int asym);
+cudaError_t set_decode_wait_limit(uint64_t ns);
+cudaError_t set_dp_wait_limit(uint64_t ns);
 size_t dp_l24_work_bytes(int64_t n);
 cudaError_t launch_transform_quantize_dp(const void* x, int dtype, int64_t n, int64_t d, int k, const float* A, int bits,
                                          int asym, int l24, uint8_t* planes, float* scale, int32_t* zero,
@@ -568,6 +570,17 @@ cat_status cat_sqnr(const float* y_ref, const float* y_hat, int64_t numel, doubl
   if (st != CAT_OK) return st;
   cudaError_t e = cat::launch_sqnr(y_ref, y_hat, numel, out3, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "cat_sqnr launch");
+  return ok();
+}
+
+cat_status cat_set_wait_limit_ns(uint64_t ns) {
+  if (ns > cat::kWaitLimitNs) return fail(CAT_ERR_INVALID_ARG, "the wait limit is at most 1 s (1e9 ns)");
+  const uint64_t v = ns == 0 ? cat::kWaitLimitNs : ns;
+  cat_status st = check_device();
+  if (st != CAT_OK) return st;
+  cudaError_t e = cat::set_decode_wait_limit(v);
+  if (e == cudaSuccess) e = cat::set_dp_wait_limit(v);
+  if (e != cudaSuccess) return cuda_fail(e, "cat_set_wait_limit_ns");
   return ok();
 }
 

@@ -28,6 +28,7 @@ enum : uint32_t {
   kWhereGemm = 1u << 10,
   kWhereGemmDecode = 1u << 11,
   kWhereCalib = 1u << 12,
+  kWhereGemmDp = 1u << 13,
 };
 
 // The status bits a kernel raises when a wait gave up: abort holds the line of the first one.
@@ -187,14 +188,18 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 // Wait until the phase with the given parity has completed.  Returns false (and raises
 // `*abort`, to `site` if it was not raised yet) if `*abort` was already raised by another thread or
 // the wait exceeded the limit.
-__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, volatile int* abort, int site = 1) {
+// `limit`: the wait's bound in ns (kernels whose pipeline waits take a test-settable bound pass it;
+// waits that drain copies or MMAs in flight before exit always keep kWaitLimitNs).
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, volatile int* abort, int site = 1,
+                                                  uint64_t limit = kWaitLimitNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 63u) == 0u) {
+    // the clock is read on the first poll and every 64th (a try_wait may itself suspend for a while)
+    if (it == 1u || (it & 63u) == 0u) {
       if (*abort) return false;
-      if (globaltimer_ns() - t0 > kWaitLimitNs) {
+      if (globaltimer_ns() - t0 > limit) {
         if (*abort == 0) *abort = site;
         return false;
       }

@@ -76,6 +76,9 @@ constexpr int kDecMaxUnits = 4096;
 __device__ float4 g_dec_part[kDecSlots][kDecMaxGrid][32][UM / 4];
 __device__ uint32_t g_dec_cnt[kDecSlots][kDecMaxUnits][kEpiWarps];
 
+// Bound of the pipeline waits (ns); kWaitLimitNs unless a test shortens it (cat_set_wait_limit_ns).
+__device__ uint64_t g_dec_wait_limit = kWaitLimitNs;
+
 __device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* p) {
   uint32_t v;
   asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
@@ -162,6 +165,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   float* sxs = reinterpret_cast<float*>(bars + 1);                // NTOK token steps
   volatile int* abort_flag = &bars->abort;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint64_t lim = g_dec_wait_limit;
 
   if (tid == 0) {
     for (int s = 0; s < sp; ++s) {
@@ -257,7 +261,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if ((it & 1u) != me) continue;
         const int u = sg / num_ks, ks = sg % num_ks;
         const uint32_t s = it % sp, use = it / sp;
-        if (use > 0 && !(ok = mbar_wait_bounded(&bars->p_empty[s], (use - 1) & 1, abort_flag, __LINE__))) break;
+        if (use > 0 && !(ok = mbar_wait_bounded(&bars->p_empty[s], (use - 1) & 1, abort_flag, __LINE__, lim))) break;
         mbar_arrive_expect_tx(&bars->p_full[s], kPkStage);
         tma_load_2d(pk + s * kPkStage, &tmW, ks * KSB, u * UM, &bars->p_full[s]);
         issued_end = it + 1;
@@ -286,7 +290,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t bbase = smem_u32(bst);
     bool stop = false;
     if (leader) {
-      mbar_wait_bounded(&bars->tok_ready, 0, abort_flag, __LINE__);
+      mbar_wait_bounded(&bars->tok_ready, 0, abort_flag, __LINE__, lim);
       tc_fence_after();
     }
     uint32_t seg = 0;
@@ -300,8 +304,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t it = (uint32_t)(sg - s0);         // it % kDecGroups == grp
         const int ks = sg % num_ks;
         const uint32_t ps = it % sp, sa = it % kSE;
-        const bool good = mbar_wait_bounded(&bars->p_full[ps], (it / sp) & 1, abort_flag, __LINE__) &&
-                          (it < (uint32_t)kSE || mbar_wait_bounded(&bars->empty[sa], ((it / kSE) - 1) & 1, abort_flag, __LINE__));
+        const bool good = mbar_wait_bounded(&bars->p_full[ps], (it / sp) & 1, abort_flag, __LINE__, lim) &&
+                          (it < (uint32_t)kSE || mbar_wait_bounded(&bars->empty[sa], ((it / kSE) - 1) & 1, abort_flag, __LINE__, lim));
         if (good) {
           tc_fence_after();
           const uint8_t* prow = pk + ps * kPkStage + r * 128;
@@ -330,7 +334,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (stop) break;
         if (leader) {
           tc_fence_after();
-          if (first && seg >= 2) mbar_wait_bounded(&bars->acc_empty[ab], ((seg >> 1) - 1) & 1, abort_flag, __LINE__);
+          if (first && seg >= 2) mbar_wait_bounded(&bars->acc_empty[ab], ((seg >> 1) - 1) & 1, abort_flag, __LINE__, lim);
           tc_fence_after();
           const uint32_t ta = tmem + kAStage0 + 64u * sa;
 #pragma unroll
@@ -346,7 +350,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (leader) {
         // a group without steps in this segment still waits for the buffer to be drained before it
         // commits, so its arrivals can never run a phase ahead
-        if (first && seg >= 2) mbar_wait_bounded(&bars->acc_empty[ab], ((seg >> 1) - 1) & 1, abort_flag, __LINE__);
+        if (first && seg >= 2) mbar_wait_bounded(&bars->acc_empty[ab], ((seg >> 1) - 1) & 1, abort_flag, __LINE__, lim);
         mma_commit(&bars->acc_full[ab]);
       }
       sb = se;
@@ -379,7 +383,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       float yr[NTOK];
 #pragma unroll
       for (int t = 0; t < NTOK; ++t) yr[t] = (pre && t < n) ? __ldcs(y_ref + (int64_t)t * d_out + o) : 0.f;
-      if (!(ok = mbar_wait_bounded(&bars->acc_full[ab], (seg >> 1) & 1, abort_flag, __LINE__))) break;
+      if (!(ok = mbar_wait_bounded(&bars->acc_full[ab], (seg >> 1) & 1, abort_flag, __LINE__, lim))) break;
       __syncwarp();
       tc_fence_after();
       // the groups with steps in the segment: local steps sb - s0 .. se - s0 - 1, group = step % 4
@@ -404,7 +408,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint64_t t0 = globaltimer_ns();
           for (uint32_t it = 0; ld_acquire_u32(cnt) < (uint32_t)(cl - cf); ++it) {
             __nanosleep(32);
-            if ((it & 63u) == 63u && (*abort_flag || globaltimer_ns() - t0 > kWaitLimitNs)) {
+            if ((it & 63u) == 63u && (*abort_flag || globaltimer_ns() - t0 > lim)) {
               if (*abort_flag == 0) *abort_flag = __LINE__;
               good = 0u;
               break;
@@ -427,7 +431,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int t = 0; t < (kEarly ? NTOK : 1); ++t) ext[t] += __ldcg(src + t * UM);  // exact in any order
         }
       }
-      if (!(ok = mbar_wait_bounded(&bars->acc_full[ab], (seg >> 1) & 1, abort_flag, __LINE__))) break;
+      if (!(ok = mbar_wait_bounded(&bars->acc_full[ab], (seg >> 1) & 1, abort_flag, __LINE__, lim))) break;
       __syncwarp();
       tc_fence_after();
       if (!kEarly && !whole && owner && !(ok = wait_parts())) break;
@@ -625,6 +629,10 @@ cudaError_t launch_ntok(const uint8_t* xq, const float* sx, const uint8_t* wq, c
 }
 
 }  // namespace
+
+cudaError_t set_decode_wait_limit(uint64_t ns) {
+  return cudaMemcpyToSymbol(g_dec_wait_limit, &ns, sizeof(ns));
+}
 
 // Packed stages that fit beside the resident tokens; 0 when this kernel does not apply.
 int decode_tc_stages(int64_t n, int64_t d_in) {

@@ -41,6 +41,9 @@ struct DpGemmCfg {
   static_assert(S >= 2, "stages");
 };
 
+// Bound of the pipeline waits (ns); kWaitLimitNs unless a test shortens it (cat_set_wait_limit_ns).
+__device__ uint64_t g_dp_wait_limit = kWaitLimitNs;
+
 struct DpBars {
   uint64_t full[8], empty[8], acc_full, mma_done;
   uint32_t tmem_addr;
@@ -79,6 +82,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int o0 = blockIdx.x * BN, t0 = blockIdx.y * BM;
   const int num_k = (d_in + KB - 1) / KB;
+  const uint64_t lim = g_dp_wait_limit;
 
   if (tid == 0) {
     for (int s = 0; s < C::S; ++s) {
@@ -105,7 +109,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       int kb = 0;
       for (; kb < num_k; ++kb) {
         const int s = kb % C::S;
-        if (kb >= C::S && !mbar_wait_bounded(&bars->empty[s], ((kb / C::S) - 1) & 1, abort_flag, __LINE__)) break;
+        if (kb >= C::S && !mbar_wait_bounded(&bars->empty[s], ((kb / C::S) - 1) & 1, abort_flag, __LINE__, lim)) break;
         uint8_t* st = smem + (size_t)s * C::STAGE;
         mbar_arrive_expect_tx(&bars->full[s], C::STAGE);
 #pragma unroll
@@ -127,7 +131,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int g = 0; g < C::G; ++g) started[g] = false;
       for (int kb = 0; kb < num_k; ++kb) {
         const int s = kb % C::S;
-        if (!mbar_wait_bounded(&bars->full[s], (kb / C::S) & 1, abort_flag, __LINE__)) break;
+        if (!mbar_wait_bounded(&bars->full[s], (kb / C::S) & 1, abort_flag, __LINE__, lim)) break;
         tc_fence_after();
         const uint32_t base = smem_u32(smem + (size_t)s * C::STAGE);
 #pragma unroll
@@ -157,7 +161,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const bool t_ok = t < n;
     const float sxt = t_ok ? sx[t] : 0.f;
     const int zt = (t_ok && zx) ? zx[t] : 0;
-    if (mbar_wait_bounded(&bars->acc_full, 0, abort_flag, __LINE__)) {
+    if (mbar_wait_bounded(&bars->acc_full, 0, abort_flag, __LINE__, lim)) {
       __syncwarp();
       tc_fence_after();
 #pragma unroll 1
@@ -192,7 +196,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   tc_fence_before();
   __syncthreads();
-  if (bars->abort && tid == 0) report(status, timeout_bits(kWhereGemm, bars->abort));
+  if (bars->abort && tid == 0) report(status, timeout_bits(kWhereGemmDp, bars->abort));
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, C::TMEM_COLS);
@@ -259,6 +263,8 @@ cudaError_t launch_dx_dw(const CUtensorMap& mx, const CUtensorMap& mw, const flo
 }
 
 }  // namespace
+
+cudaError_t set_dp_wait_limit(uint64_t ns) { return cudaMemcpyToSymbol(g_dp_wait_limit, &ns, sizeof(ns)); }
 
 // x_planes [DX][n][d_in], w_planes [DW][d_out][d_in] digit bytes; zx / w_rowsum both given for
 // asymmetric activations (else both NULL).

@@ -128,3 +128,11 @@ def test_host_transform_k256_and_errors(lib):
     assert ei.value.status == 4
     with pytest.raises(cat.CatError):
         cat.cat_build_transform_host("rht", d, k, rht_signs=np.full(d, 0.5))
+
+
+def test_wait_limit_setter_rejects_bounds_above_one_second():
+    """The testing aid refuses a bound above the default before any CUDA call (runs without a GPU)."""
+    import ctypes
+    lib = cat.load_library()
+    assert lib.cat_set_wait_limit_ns(ctypes.c_uint64(2_000_000_000)) == 1      # CAT_ERR_INVALID_ARG
+    assert b"at most 1 s" in lib.cat_last_error()
