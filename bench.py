@@ -63,6 +63,9 @@ def parse_args():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-secondary", action="store_true", help="skip the secondary configurations")
+    p.add_argument("--shard", choices=["replicas", "tokens"], default="replicas",
+                   help="replicas: one independent layer per GPU (weak scaling); tokens: one layer's tokens split "
+                        "across the GPUs, calibration and SQNR sums all-reduced (strong scaling)")
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="budget of the CPU-baseline sample")
     p.add_argument("--sweep", action="store_true",
                    help="also report the layer's SQNR for every block size in SWEEP_K and every transform "
@@ -169,6 +172,34 @@ def max_over_ranks(v: float, world: int) -> float:
     t = torch.tensor([v], dtype=torch.float64, device="cuda" if torch.cuda.is_available() else "cpu")
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+# ---------------------------------------------------------------------------------------------
+# Token-sharded layer: the layer's tokens split across ranks
+# ---------------------------------------------------------------------------------------------
+
+def shard_range(n: int, rank: int, world: int):
+    """Contiguous, near-equal token ranges: rank r takes [n r / N, n (r + 1) / N)."""
+    return n * rank // world, n * (rank + 1) // world
+
+
+def sharded_layer_step(ops, x_local, xc_local, y_ref_local, W, k, n_calib_total, allreduce_sum):
+    """One step of the layer with its tokens split across ranks.  Activations are quantized per token
+    and weights per output channel (Sec. 6) and T is block-diagonal, so the forward pass needs no
+    collective; the two cross-token reductions are all-reduced:
+      * the calibration block sums sum_t x_{t,b} x_{t,b}^T of every rank's calibration tokens, so that
+        every rank builds the same transform from the whole calibration set (Sec. 4, Eq. 7, Eq. 10);
+      * the SQNR sums (sum y^2, sum (y - y_hat)^2) over every rank's outputs (Sec. 2, Eq. 1).
+    `ops` computes on this rank (the library on a GPU; the oracle in the host tests);
+    `allreduce_sum(arr)` sums an array over ranks in place.  Returns (y_hat_local, sum y^2, sum e^2, dB)."""
+    sigma = ops.calib_cov(xc_local, k)
+    allreduce_sum(sigma)
+    T, Wq, sw = ops.quantize_weights(W, k, sigma, n_calib_total)
+    xq, sx = ops.transform_quantize_act(x_local, T, k)
+    y_hat, sums = ops.linear_sqnr(xq, sx, Wq, sw, y_ref_local)
+    allreduce_sum(sums)
+    sig, err = float(sums[0]), float(sums[1])
+    return y_hat, sig, err, 10.0 * float(np.log10(sig / err))
 
 
 # ---------------------------------------------------------------------------------------------
@@ -585,6 +616,90 @@ def roofline_of(cfg, res, steps):
     return roof, gemm_ms, gemm_tflops
 
 
+class LibOps:
+    """The per-rank computations of sharded_layer_step through the library."""
+
+    def __init__(self, cat):
+        self.cat = cat
+
+    def calib_cov(self, xc, k):
+        return self.cat.cat_calib_cov(xc, k)
+
+    def quantize_weights(self, W, k, sigma, n_calib):
+        return self.cat.cat_quantize_weights(W, k, "cat", sigma_x=sigma, n_calib=n_calib)
+
+    def transform_quantize_act(self, x, T, k):
+        return self.cat.cat_transform_quantize_act(x, T, k)
+
+    def linear_sqnr(self, xq, sx, Wq, sw, y_ref):
+        y, out3 = self.cat.cat_w4a4_linear_sqnr(xq, sx, Wq, sw, y_ref)
+        return y, out3[:2].clone()
+
+
+def token_sharded_arm(args, rank, world, local):
+    """--shard tokens: the configuration's tokens (and calibration tokens) split across the ranks, one
+    layer in total (strong scaling).  A step = calib_cov on the rank's calibration tokens, an
+    all-reduce of the block sums, the transform and the GEMM with SQNR sums on the rank's tokens, an
+    all-reduce of the two sums.  Weight preparation runs once, from the all-reduced sums."""
+    import paper_2603_04359_gb300 as cat
+    cat.load_library()
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    cfg = WL.CONFIGS[args.config]
+    k = args.k or cfg.k
+    L = WL.make_layer(cfg)
+    t0, t1 = shard_range(cfg.n_eval, rank, world)
+    c0, c1 = shard_range(cfg.n_calib, rank, world)
+    x_all, xc_all, W = to_dev(L.x_eval, dev), to_dev(L.x_calib, dev), to_dev(L.W, dev)
+    x, xc = x_all[t0:t1].contiguous(), xc_all[c0:c1].contiguous()
+    torch.backends.cuda.matmul.allow_tf32 = False
+    y_ref = (x.float() @ W.float().t()).contiguous()
+
+    def allreduce_sum(t):
+        if world > 1:
+            import torch.distributed as dist
+            dist.all_reduce(t)
+
+    ops = LibOps(cat)
+    _, sig, err, db = sharded_layer_step(ops, x, xc, y_ref, W, k, cfg.n_calib, allreduce_sum)   # untimed
+    sigma = ops.calib_cov(xc, k)
+    allreduce_sum(sigma)
+    T, Wq, sw = ops.quantize_weights(W, k, sigma, cfg.n_calib)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        s_ = cat.cat_calib_cov(xc, k, out=sigma)
+        allreduce_sum(s_)
+        xq, sx = cat.cat_transform_quantize_act(x, T, k)
+        _, out3 = cat.cat_w4a4_linear_sqnr(xq, sx, Wq, sw, y_ref)
+        sums = out3[:2].clone()
+        allreduce_sum(sums)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    barrier(world)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    ms = max_over_ranks(e0.elapsed_time(e1) / args.steps, world)
+    st, word = cat.cat_device_status(dev)
+    if st != 0:
+        raise RuntimeError(f"device status {st} ({word:#x})")
+    if rank == 0:
+        print(json.dumps({
+            "metric": METRIC, "value": cfg.n_eval / (ms / 1e3), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "strong",
+            "vs_baseline": None, "dtype": "int4", "data": "synthetic",
+            "config": {"workload": cfg.name, "n_tokens": cfg.n_eval, "d_in": cfg.d_in, "d_out": cfg.d_out, "k": k,
+                       "parallelism": f"tokens x{world}", "timing": "host-issued steps between CUDA events"},
+            "sqnr_db": db, "sqnr_sums": [sig, err]}), flush=True)
+
+
 def ours_arm(args, rank, world, local, retried=None):
     import paper_2603_04359_gb300 as cat
     cat.load_library()
@@ -650,6 +765,12 @@ def main():
         reference_arm(args, int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")))
         return
     rank, world, local = dist_setup()
+    if args.shard == "tokens":
+        token_sharded_arm(args, rank, world, local)
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+        return
     try:
         ours_arm(args, rank, world, local)
     except DeviceTimeout as e:           # one fresh measurement on a single GPU, recorded in the line

@@ -96,3 +96,90 @@ def test_diagnostics_from_sums_matches_the_oracle():
     assert abs(dg["C_w_db"] - O.db(O.concentration_weight(W))) < 1e-9
     assert abs(dg["A_db"] - O.db(O.alignment(X, W))) < 1e-9
     assert abs(dg["theorem1_db"] - O.db(O.theorem1_sqnr(X, W))) < 1e-9
+
+
+# ------------------------------------------------------------------------------------------
+# Token-sharded layer: per-rank compute by the oracle, reductions over two gloo ranks
+# ------------------------------------------------------------------------------------------
+
+class _OracleOps:
+    """The per-rank computations of bench.sharded_layer_step, done by the oracle on the host."""
+
+    def __init__(self):
+        import oracle as O
+        self.O = O
+
+    def calib_cov(self, xc, k):
+        return self.O.calib_cov_block_sums(xc, k)
+
+    def quantize_weights(self, W, k, sigma_sums, n_calib):
+        pw = self.O.prepare_weights(W, "cat", k, Sigma_x_blocks=sigma_sums / n_calib)
+        return pw.T, pw.qw, pw.sw
+
+    def transform_quantize_act(self, x, T, k):
+        ac = self.O.transform_quantize_act(x, T)
+        return ac.qx, ac.sx
+
+    def linear_sqnr(self, qx, sx, qw, sw, y_ref):
+        import numpy as np
+        _, y_hat = self.O.w4a4_linear(qx, sx, qw, sw)
+        sig, err = self.O.sqnr_sums(y_ref, y_hat)
+        return y_hat, np.array([sig, err])
+
+
+def _sharded_rank_main(rank, world, port, q):
+    os.environ.update({"MASTER_ADDR": "127.0.0.1", "MASTER_PORT": str(port), "RANK": str(rank),
+                       "WORLD_SIZE": str(world), "LOCAL_RANK": str(rank)})
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    import bench
+    import oracle as O
+    import workloads as WL
+    bench.dist_setup()
+    cfg = WL.small_config("shard", d_in=256, d_out=160, n_eval=211, n_calib=300, k=32, seed=61)
+    L = WL.make_layer(cfg)
+
+    def allreduce_sum(arr):
+        t = torch.from_numpy(np.ascontiguousarray(arr))
+        dist.all_reduce(t)
+        arr[...] = t.numpy()
+
+    t0, t1 = bench.shard_range(cfg.n_eval, rank, world)
+    c0, c1 = bench.shard_range(cfg.n_calib, rank, world)
+    x = L.x_eval.values[t0:t1].astype(np.float64)
+    y_ref = O.linear(x, L.W.values)
+    y_hat, sig, err, db = bench.sharded_layer_step(_OracleOps(), x, L.x_calib.values[c0:c1].astype(np.float64), y_ref,
+                                                   L.W.values, cfg.k, cfg.n_calib, allreduce_sum)
+    q.put((rank, t0, t1, y_hat, sig, err, db))
+    dist.destroy_process_group()
+
+
+def test_token_sharded_layer_matches_one_process():
+    """Two ranks each take half of the tokens (and of the calibration tokens); with the calibration
+    sums and the SQNR sums all-reduced, the combined SQNR and every rank's output equal the one-process
+    layer's (Sec. 6: per-token activations, per-channel weights; the layer shards by tokens)."""
+    import numpy as np
+
+    import oracle as O
+    import workloads as WL
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_sharded_rank_main, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    got = [q.get(timeout=240) for _ in range(2)]
+    for p in procs:
+        p.join(120)
+    assert all(p.exitcode == 0 for p in procs), [p.exitcode for p in procs]
+    cfg = WL.small_config("shard", d_in=256, d_out=160, n_eval=211, n_calib=300, k=32, seed=61)
+    L = WL.make_layer(cfg)
+    ref = O.cat_layer(L.x_eval.values, L.W.values, "cat", cfg.k, X_calib=L.x_calib.values)
+    dbs = {r[6] for r in got}
+    assert len(dbs) == 1                                    # every rank reports the same combined value
+    assert abs(dbs.pop() - ref["sqnr_db"]) < 0.01
+    for rank, t0, t1, y_hat, sig, err, db in got:
+        assert abs(sig / ref["sig"] - 1) < 1e-12 and abs(err / ref["err"] - 1) < 1e-9
+        np.testing.assert_allclose(y_hat, ref["y_hat"][t0:t1], rtol=1e-9, atol=1e-12)

@@ -626,3 +626,19 @@ def test_layer_asymmetric_accumulators_match_dequantized_product():
     Xq = O.dequantize_rows_asymmetric(ac.qx, ac.sx, ac.zx)
     Wq = O.dequantize_rows(pw.qw, pw.sw)
     np.testing.assert_allclose(r["y_hat"], Xq @ Wq.T, rtol=1e-12, atol=1e-12)
+
+
+def test_interval_count_of_the_grid_is_measured_by_the_noise():
+    """N in Lemmas 2-3 is the number of quantization intervals across the range r = 2 max|v|: the
+    noise variance is s^2 / 12 with s = r / N.  On dense rows (the noise is uniform) the measured
+    r / sqrt(12 E[e^2]) is 2 qmax = 14 at 4 bits on the restricted grid used here, not the paper's
+    2^b - 1 = 15 -- n_intervals must return the grid's count (and 2 at 2 bits, 254 at 8 bits)."""
+    rng = _rng(60)
+    V = rng.uniform(-1, 1, (4000, 512))
+    V[:, 0] = 1.0                                    # every row's range is exactly 2
+    for bits in (2, 3, 4, 8):
+        q, s, _ = O.quantize_rows_symmetric(V, bits)
+        e = V[:, 1:] - q[:, 1:] * s[:, None]
+        n_meas = 2.0 / np.sqrt(12 * np.mean(e * e))
+        assert abs(n_meas / O.n_intervals(bits) - 1) < 0.01, (bits, n_meas)
+        assert abs(n_meas / O.n_intervals(bits, paper=True) - 1) > 0.05 or bits == 8
