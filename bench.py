@@ -333,7 +333,7 @@ def transform_sweep(cat, L, x, W, xc, y_ref):
     diag = {}
     for kind in ("identity", "rht", "cat"):
         vals = []
-        dk = {"C_x_db": [], "C_w_db": [], "A_db": [], "theorem1_db": []}
+        dk = {"C_x_db": [], "C_w_db": [], "A_db": [], "theorem1_db": [], "act_only_db": [], "weight_only_db": []}
         for k in SWEEP_K:
             sigma = cat.cat_calib_cov(xc, k) if kind == "cat" else None
             try:
@@ -354,6 +354,8 @@ def transform_sweep(cat, L, x, W, xc, y_ref):
             _, _, x3 = cat.cat_block_row_stats(x, k, T)
             _, _, w3 = cat.cat_block_row_stats(W, k, Tinv, transpose=True)
             dg = diagnostics_from_sums(x3.cpu().numpy(), w3.cpu().numpy(), float(out3[0].item()))
+            # the two measured sides of Theorem 1 (Lemma 2: activations only; Lemma 3: weights only)
+            dg["act_only_db"], dg["weight_only_db"] = cat.one_sided_sqnr(x, W, k, T, Tinv, xq, sx, Wq, sw, y_ref)
             for key in dk:
                 dk[key].append(round(dg[key], 3))
             del T, Wq, sw, xq, sx, Tinv
@@ -750,8 +752,9 @@ def ours_arm(args, rank, world, local, retried=None):
         line["retried_after"] = retried
     if res["sweep"]:
         line["sqnr_sweep"] = dict(res["sweep"], unit="dB", over="all n x d_out outputs, y = W x in fp32 as reference",
-                                  diagnostics_note="per transform and k: concentrations C(x'), C(W'), alignment A "
-                                                   "and the Theorem-1 SQNR prediction (N = 14 intervals), in dB")
+                                  diagnostics_note="per transform and k: concentrations C(x'), C(W'), alignment A, "
+                                                   "the Theorem-1 SQNR prediction (N = 14 intervals) and the measured "
+                                                   "activation-only / weight-only SQNRs (Lemmas 2, 3), in dB")
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = run_cpu_baseline(res["L"], args.kind, k, args.cpu_seconds)
     print(json.dumps(line), flush=True)

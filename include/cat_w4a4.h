@@ -323,6 +323,38 @@ cat_status cat_linear_dp(const uint8_t* x_planes, int32_t bits_x, int32_t asym_x
 cat_status cat_set_wait_limit_ns(uint64_t ns);
 
 /*
+ * One-sided SQNRs (Sec. 2: Lemma 2, SQNR(W x~), only activations quantized; Lemma 3, SQNR(W~ x), only
+ * weights quantized; Lemma 1 combines the two into Theorem 1).  Off the hot path, three building
+ * blocks on SIMT cores; with x' = T x and W' = W T^{-1} (so W' x' = W x):
+ *   activation side: y_x = Q(x') W'^T  = cat_gemm_f32(cat_dequantize_codes(xq, x_scale), W')
+ *   weight side:     y_w = x' Q(W')^T  = cat_gemm_f32(x', cat_dequantize_codes(Wq, w_scale))
+ *   x' and W' from cat_block_transform; each SQNR then from cat_sqnr against y = W x.
+ */
+
+/*
+ * cat_block_transform -- v'_b = M_b v_b (transpose = 0; activations with M = T) or M_b^T v_b
+ * (transpose = 1; weight rows with M = T^{-1}, w' = w T^{-1}) for every row (Sec. 3, Eq. 5).
+ *   V device [rows][d] in `dtype`; M_blocks device [d/k][k][k] float32; out device [rows][d] float32.
+ * fp32 products and sums.
+ */
+cat_status cat_block_transform(const void* V, cat_dtype dtype, int64_t rows, int64_t d, int32_t k,
+                               const float* M_blocks, int transpose, float* out, cat_stream_t stream);
+
+/*
+ * cat_dequantize_codes -- Q(v) = s_r q (Sec. 2): SM4x8 codes [rows][d/2] and steps [rows] float32 to
+ * out [rows][d] float32.  All device pointers.
+ */
+cat_status cat_dequantize_codes(const uint8_t* codes, const float* scale, int64_t rows, int64_t d, float* out,
+                                cat_stream_t stream);
+
+/*
+ * cat_gemm_f32 -- C[i][j] = sum_l A[i][l] B[j][l] in float32 (A [m][kdim], B [n][kdim], C [m][n], row-major
+ * device arrays): the float GEMMs of the one-sided SQNRs.  A tiled SIMT kernel.
+ */
+cat_status cat_gemm_f32(const float* A, const float* B, int64_t m, int64_t n, int64_t kdim, float* C,
+                        cat_stream_t stream);
+
+/*
  * cat_device_status -- synchronizes `stream`, then reads and clears the device status word.
  * Returns CAT_OK, CAT_ERR_TIMEOUT (a bounded wait in a kernel gave up and the kernel returned
  * early; its outputs are undefined) or CAT_ERR_NUMERIC (a kernel met a non-finite value; the

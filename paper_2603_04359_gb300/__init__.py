@@ -21,6 +21,7 @@ __all__ = [
     "cat_calib_cov", "cat_quantize_weights", "cat_build_transform_host", "cat_transform_quantize_act",
     "cat_w4a4_linear", "cat_sqnr", "cat_device_status", "cat_version", "KIND",
     "cat_dp_planes", "cat_transform_quantize_act_dp", "cat_quantize_weights_dp", "cat_linear_dp",
+    "cat_block_transform", "cat_dequantize_codes", "cat_gemm_f32", "one_sided_sqnr", "cat_set_wait_limit_ns",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -70,6 +71,9 @@ def load_library() -> ctypes.CDLL:
         "cat_block_row_stats": ([P, I, I64, I64, I32, P, I, P, P, P, P], I),
         "cat_dp_planes": ([I32], I32),
         "cat_set_wait_limit_ns": ([ctypes.c_uint64], I),
+        "cat_block_transform": ([P, I, I64, I64, I32, P, I, P, P], I),
+        "cat_dequantize_codes": ([P, P, I64, I64, P, P], I),
+        "cat_gemm_f32": ([P, P, I64, I64, I64, P, P], I),
         "cat_transform_quantize_act_dp": ([P, I, I64, I64, I32, P, I32, I32, P, P, P, P], I),
         "cat_quantize_weights_dp": ([P, I, I64, I64, I32, I, P, I64, P, I32, I32, P, P, P, P, P], I),
         "cat_linear_dp": ([P, I32, I32, P, P, P, I32, P, P, I64, I64, I64, P, P, P], I),
@@ -407,6 +411,50 @@ def cat_linear_dp(x_planes: torch.Tensor, bits_x: int, x_scale: torch.Tensor, w_
         _ptr(x_planes), int(bits_x), int(asym), _ptr(x_scale), _ptr(x_zero), _ptr(w_planes), int(bits_w), _ptr(w_scale),
         _ptr(w_rowsum) if asym else None, n, d_in, d_out, _ptr(y), _ptr(acc_out), _stream(dev)))
     return y
+
+
+def cat_block_transform(V: torch.Tensor, k: int, M: torch.Tensor, transpose: bool = False) -> torch.Tensor:
+    """v'_b = M_b v_b (or M_b^T v_b) for every row: float32 [rows, d]."""
+    _need(V, "V")
+    rows, d = V.shape
+    _expect(M, "M", torch.float32, (d // k, k, k), V.device)
+    out = torch.empty((rows, d), dtype=torch.float32, device=V.device)
+    _check("cat_block_transform", load_library().cat_block_transform(
+        _ptr(V), _dtype(V), rows, d, k, _ptr(M), 1 if transpose else 0, _ptr(out), _stream(V.device)))
+    return out
+
+
+def cat_dequantize_codes(codes: torch.Tensor, scale: torch.Tensor) -> torch.Tensor:
+    """s_r * q from SM4x8 codes [rows, d/2] and steps [rows]: float32 [rows, d]."""
+    rows, half = codes.shape
+    _expect(codes, "codes", torch.uint8, (rows, half), codes.device)
+    _expect(scale, "scale", torch.float32, (rows,), codes.device)
+    out = torch.empty((rows, 2 * half), dtype=torch.float32, device=codes.device)
+    _check("cat_dequantize_codes", load_library().cat_dequantize_codes(
+        _ptr(codes), _ptr(scale), rows, 2 * half, _ptr(out), _stream(codes.device)))
+    return out
+
+
+def cat_gemm_f32(A: torch.Tensor, B: torch.Tensor) -> torch.Tensor:
+    """C = A B^T in float32 (A [m, k], B [n, k])."""
+    m, kd = A.shape
+    n = B.shape[0]
+    _expect(A, "A", torch.float32, (m, kd), A.device)
+    _expect(B, "B", torch.float32, (n, kd), A.device)
+    C = torch.empty((m, n), dtype=torch.float32, device=A.device)
+    _check("cat_gemm_f32", load_library().cat_gemm_f32(_ptr(A), _ptr(B), m, n, kd, _ptr(C), _stream(A.device)))
+    return C
+
+
+def one_sided_sqnr(x: torch.Tensor, W: torch.Tensor, k: int, T: torch.Tensor, Tinv: torch.Tensor, xq: torch.Tensor,
+                   x_scale: torch.Tensor, Wq: torch.Tensor, w_scale: torch.Tensor, y_ref: torch.Tensor):
+    """The measured one-sided SQNRs of Lemmas 2 and 3 in dB, (activations only, weights only), composed
+    of the library calls above and cat_sqnr against y_ref = W x."""
+    xt = cat_block_transform(x, k, T)
+    wt = cat_block_transform(W, k, Tinv, transpose=True)
+    y_x = cat_gemm_f32(cat_dequantize_codes(xq, x_scale), wt)
+    y_w = cat_gemm_f32(xt, cat_dequantize_codes(Wq, w_scale))
+    return float(cat_sqnr(y_ref, y_x)[2].item()), float(cat_sqnr(y_ref, y_w)[2].item())
 
 
 def cat_set_wait_limit_ns(ns: int) -> None:

@@ -24,6 +24,12 @@ cudaError_t launch_block_row_stats(const void* V, int dtype, int64_t rows, int64
                                    int transpose, float* row_sumsq, float* row_amax, double* out3,
                                    cudaStream_t stream);
 int dp_planes(int bits, int asym);
+cudaError_t launch_block_transform(const void* V, int dtype, int64_t rows, int64_t d, int k, const float* M,
+                                   int transpose, float* Vt, cudaStream_t stream);
+cudaError_t launch_dequantize_sm4x8(const uint8_t* codes, const float* scale, int64_t rows, int64_t d, float* out,
+                                    cudaStream_t stream);
+cudaError_t launch_gemm_f32_nt(const float* A, const float* B, float* C, int64_t M, int64_t N, int64_t K,
+                               cudaStream_t stream);
 cudaError_t set_decode_wait_limit(uint64_t ns);
 cudaError_t set_dp_wait_limit(uint64_t ns);
 size_t dp_l24_work_bytes(int64_t n);
@@ -614,5 +620,54 @@ cat_status cat_block_row_stats(const void* V, cat_dtype dtype, int64_t rows, int
   cudaError_t e = cat::launch_block_row_stats(V, (int)dtype, rows, d, k, M_blocks, transpose, row_sumsq, row_amax, out3,
                                               (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "cat_block_row_stats launch");
+  return ok();
+}
+
+// ---- building blocks of the one-sided SQNRs (Lemmas 2 and 3), off the hot path
+
+cat_status cat_block_transform(const void* V, cat_dtype dtype, int64_t rows, int64_t d, int32_t k,
+                               const float* M_blocks, int transpose, float* out, cat_stream_t stream) {
+  if (dtype != CAT_F32 && dtype != CAT_BF16) return fail(CAT_ERR_INVALID_ARG, "unknown dtype");
+  if (rows < 1 || rows > 0x7FFFFFFF) return fail(CAT_ERR_SHAPE, "rows must be in [1, 2^31)");
+  cat_status st = check_din(d);
+  if (st != CAT_OK) return st;
+  if (!valid_k(k) || d % k != 0) return fail(CAT_ERR_SHAPE, "k must be one of 16..256 (power of two) and divide d");
+  if ((rows + 63) / 64 > 0x7FFFFFFF || d / k > 65535) return fail(CAT_ERR_SHAPE, "too many rows or blocks");
+  if (transpose != 0 && transpose != 1) return fail(CAT_ERR_INVALID_ARG, "transpose must be 0 or 1");
+  if (!V || !M_blocks || !out) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(V) || !aligned16(M_blocks) || !aligned16(out)) return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  if ((st = check_device()) != CAT_OK) return st;
+  cudaError_t e = cat::launch_block_transform(V, (int)dtype, rows, d, k, M_blocks, transpose, out, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cat_block_transform launch");
+  return ok();
+}
+
+cat_status cat_dequantize_codes(const uint8_t* codes, const float* scale, int64_t rows, int64_t d, float* out,
+                                cat_stream_t stream) {
+  if (rows < 0) return fail(CAT_ERR_SHAPE, "rows must be >= 0");
+  cat_status st = check_din(d);
+  if (st != CAT_OK) return st;
+  if (rows == 0) return ok();
+  if (rows * (d / 8) / 256 + 1 > 0x7FFFFFFF) return fail(CAT_ERR_SHAPE, "too many codes");
+  if (!codes || !scale || !out) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(codes) || !aligned16(scale) || !aligned16(out)) return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  if ((st = check_device()) != CAT_OK) return st;
+  cudaError_t e = cat::launch_dequantize_sm4x8(codes, scale, rows, d, out, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cat_dequantize_codes launch");
+  return ok();
+}
+
+cat_status cat_gemm_f32(const float* A, const float* B, int64_t m, int64_t n, int64_t kdim, float* C,
+                        cat_stream_t stream) {
+  if (m < 0 || n < 0 || kdim < 1 || m > 0x7FFFFFFF || n > 0x7FFFFFFF || kdim > 0x7FFFFFFF)
+    return fail(CAT_ERR_SHAPE, "m, n >= 0 and k >= 1, each below 2^31");
+  if ((m + 127) / 128 > 65535) return fail(CAT_ERR_SHAPE, "m too large");
+  if (m == 0 || n == 0) return ok();
+  if (!A || !B || !C) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(A) || !aligned16(B) || !aligned16(C)) return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  cat_status st = check_device();
+  if (st != CAT_OK) return st;
+  cudaError_t e = cat::launch_gemm_f32_nt(A, B, C, m, n, kdim, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cat_gemm_f32 launch");
   return ok();
 }

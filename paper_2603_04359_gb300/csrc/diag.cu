@@ -37,7 +37,8 @@ __device__ __forceinline__ float load_elem(const void* V, int dtype, size_t idx)
 template <int K>
 __global__ void __launch_bounds__(kThreads)
     block_row_stats_kernel(const void* __restrict__ V, int dtype, int rows, int d, const float* __restrict__ M,
-                           int transpose, float* __restrict__ row_sumsq, uint32_t* __restrict__ row_amax_bits) {
+                           int transpose, float* __restrict__ row_sumsq, uint32_t* __restrict__ row_amax_bits,
+                           float* __restrict__ Vt) {
   using C = DiagCfg<K>;
   extern __shared__ float sm[];
   float* vs = sm;                       // [K][kRows]: the rows' block slice, transposed
@@ -85,7 +86,17 @@ __global__ void __launch_bounds__(kThreads)
         sumsq[rr] = fmaf(acc[rr][oj], acc[rr][oj], sumsq[rr]);
         amax[rr] = fmaxf(amax[rr], fabsf(acc[rr][oj]));
       }
+    if (Vt) {                                          // the transformed rows themselves
+#pragma unroll
+      for (int rr = 0; rr < 4; ++rr) {
+        const int r = r0 + 4 * tr + rr;
+        if (r < rows)
+#pragma unroll
+          for (int oj = 0; oj < C::OJ; ++oj) Vt[(size_t)r * d + (size_t)b * K + j0 + tj * C::OJ + oj] = acc[rr][oj];
+      }
+    }
   }
+  if (!row_sumsq) return;
   // the 16 output groups of a row group are the 16 lanes that differ in bits 0..3 of the lane index
 #pragma unroll
   for (int rr = 0; rr < 4; ++rr) {
@@ -133,7 +144,7 @@ __global__ void __launch_bounds__(kThreads)
 
 template <int K>
 cudaError_t launch_k(const void* V, int dtype, int64_t rows, int64_t d, const float* M, int transpose,
-                     float* row_sumsq, float* row_amax, cudaStream_t stream) {
+                     float* row_sumsq, float* row_amax, float* Vt, cudaStream_t stream) {
   using C = DiagCfg<K>;
   static std::once_flag once;
   static cudaError_t attr = cudaSuccess;
@@ -144,7 +155,7 @@ cudaError_t launch_k(const void* V, int dtype, int64_t rows, int64_t d, const fl
   dim3 grid((unsigned)((rows + kRows - 1) / kRows), (unsigned)(d / K), 1);
   note_launch();
   block_row_stats_kernel<K><<<grid, kThreads, C::SMEM, stream>>>(V, dtype, (int)rows, (int)d, M, transpose, row_sumsq,
-                                                                 reinterpret_cast<uint32_t*>(row_amax));
+                                                                 reinterpret_cast<uint32_t*>(row_amax), Vt);
   return cudaGetLastError();
 }
 
@@ -159,11 +170,11 @@ cudaError_t launch_block_row_stats(const void* V, int dtype, int64_t rows, int64
   if (e == cudaSuccess) e = cudaMemsetAsync(row_amax, 0, (size_t)rows * sizeof(float), stream);
   if (e != cudaSuccess) return e;
   switch (k) {
-    case 16: e = launch_k<16>(V, dtype, rows, d, M, transpose, row_sumsq, row_amax, stream); break;
-    case 32: e = launch_k<32>(V, dtype, rows, d, M, transpose, row_sumsq, row_amax, stream); break;
-    case 64: e = launch_k<64>(V, dtype, rows, d, M, transpose, row_sumsq, row_amax, stream); break;
-    case 128: e = launch_k<128>(V, dtype, rows, d, M, transpose, row_sumsq, row_amax, stream); break;
-    case 256: e = launch_k<256>(V, dtype, rows, d, M, transpose, row_sumsq, row_amax, stream); break;
+    case 16: e = launch_k<16>(V, dtype, rows, d, M, transpose, row_sumsq, row_amax, nullptr, stream); break;
+    case 32: e = launch_k<32>(V, dtype, rows, d, M, transpose, row_sumsq, row_amax, nullptr, stream); break;
+    case 64: e = launch_k<64>(V, dtype, rows, d, M, transpose, row_sumsq, row_amax, nullptr, stream); break;
+    case 128: e = launch_k<128>(V, dtype, rows, d, M, transpose, row_sumsq, row_amax, nullptr, stream); break;
+    case 256: e = launch_k<256>(V, dtype, rows, d, M, transpose, row_sumsq, row_amax, nullptr, stream); break;
     default: return cudaErrorInvalidValue;
   }
   if (e != cudaSuccess) return e;
@@ -173,6 +184,113 @@ cudaError_t launch_block_row_stats(const void* V, int dtype, int64_t rows, int64
   note_launch();
   row_stats_reduce_kernel<<<(unsigned)grid, kThreads, 0, stream>>>(row_sumsq, row_amax, (int)rows, out3,
                                                                    next_sqnr_slot());
+  return cudaGetLastError();
+}
+
+// v'_b = M_b v_b (or M_b^T v_b) for every row, written to Vt [rows][d] float32.
+cudaError_t launch_block_transform(const void* V, int dtype, int64_t rows, int64_t d, int k, const float* M,
+                                   int transpose, float* Vt, cudaStream_t stream) {
+  switch (k) {
+    case 16: return launch_k<16>(V, dtype, rows, d, M, transpose, nullptr, nullptr, Vt, stream);
+    case 32: return launch_k<32>(V, dtype, rows, d, M, transpose, nullptr, nullptr, Vt, stream);
+    case 64: return launch_k<64>(V, dtype, rows, d, M, transpose, nullptr, nullptr, Vt, stream);
+    case 128: return launch_k<128>(V, dtype, rows, d, M, transpose, nullptr, nullptr, Vt, stream);
+    case 256: return launch_k<256>(V, dtype, rows, d, M, transpose, nullptr, nullptr, Vt, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+namespace {
+
+// s_r * q from SM4x8 codes: one thread per packed word (8 codes).
+__global__ void dequantize_sm4x8_kernel(const uint32_t* __restrict__ words, const float* __restrict__ scale, int64_t rows,
+                                        int64_t d, float* __restrict__ out) {
+  const int64_t wpr = d / 8;
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= rows * wpr) return;
+  const int64_t r = idx / wpr;
+  const uint32_t w = words[idx];
+  const uint32_t lo = sm4_lo(w), hi = sm4_hi(w);
+  const float s = scale[r];
+  float v[8];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint32_t bl = (lo >> (8 * i)) & 0xFFu, bh = (hi >> (8 * i)) & 0xFFu;
+    v[i] = (float)((bl & 0x80u) ? -(int)(bl & 7u) : (int)(bl & 7u)) * s;
+    v[4 + i] = (float)((bh & 0x80u) ? -(int)(bh & 7u) : (int)(bh & 7u)) * s;
+  }
+  float4* o = reinterpret_cast<float4*>(out + idx * 8);
+  o[0] = make_float4(v[0], v[1], v[2], v[3]);
+  o[1] = make_float4(v[4], v[5], v[6], v[7]);
+}
+
+// C[m][n] = sum_k A[m][k] B[n][k] in float32: 128 x 128 tiles, 16-deep K slices staged transposed in
+// shared memory, 256 threads with 8 x 8 outputs each.
+constexpr int GT = 128, GK = 16;
+__global__ void __launch_bounds__(256) gemm_f32_nt_kernel(const float* __restrict__ A, const float* __restrict__ B,
+                                                          float* __restrict__ Cm, int M, int N, int K) {
+  __shared__ __align__(16) float As[GK][GT + 4];
+  __shared__ __align__(16) float Bs[GK][GT + 4];
+  const int tid = threadIdx.x, tm = tid >> 4, tn = tid & 15;
+  const int m0 = blockIdx.y * GT, n0 = blockIdx.x * GT;
+  float acc[8][8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
+  for (int k0 = 0; k0 < K; k0 += GK) {
+    for (int e = tid; e < GT * GK; e += 256) {            // k fastest: coalesced along the rows
+      const int r = e / GK, kk = e % GK;
+      const int ka = k0 + kk;
+      As[kk][r] = (m0 + r < M && ka < K) ? A[(size_t)(m0 + r) * K + ka] : 0.f;
+      Bs[kk][r] = (n0 + r < N && ka < K) ? B[(size_t)(n0 + r) * K + ka] : 0.f;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < GK; ++kk) {
+      float a[8], b[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) a[i] = As[kk][tm + 16 * i];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) b[j] = Bs[kk][tn + 16 * j];
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int m = m0 + tm + 16 * i;
+    if (m >= M) continue;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int n = n0 + tn + 16 * j;
+      if (n < N) Cm[(size_t)m * N + n] = acc[i][j];
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_dequantize_sm4x8(const uint8_t* codes, const float* scale, int64_t rows, int64_t d, float* out,
+                                    cudaStream_t stream) {
+  const int64_t words = rows * (d / 8);
+  if (words == 0) return cudaSuccess;
+  note_launch();
+  dequantize_sm4x8_kernel<<<(unsigned)((words + 255) / 256), 256, 0, stream>>>(reinterpret_cast<const uint32_t*>(codes),
+                                                                              scale, rows, d, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gemm_f32_nt(const float* A, const float* B, float* C, int64_t M, int64_t N, int64_t K,
+                               cudaStream_t stream) {
+  if (M == 0 || N == 0) return cudaSuccess;
+  const int64_t gx = (N + GT - 1) / GT, gy = (M + GT - 1) / GT;
+  if (gy > 65535 || gx > 0x7FFFFFFF) return cudaErrorInvalidValue;
+  note_launch();
+  gemm_f32_nt_kernel<<<dim3((unsigned)gx, (unsigned)gy), 256, 0, stream>>>(A, B, C, (int)M, (int)N, (int)K);
   return cudaGetLastError();
 }
 

@@ -438,4 +438,36 @@ def test_layer_diagnostics(cfg, kind):
     n2 = O.n_intervals(4) ** 2
     pred = 12.0 * O.parallel(n2 * c_x, n2 * c_w) * a
     assert abs(O.db(pred) - O.db(O.theorem1_sqnr(Xp, Wp))) < 1e-3
+    # the two measured sides of Theorem 1 (Lemma 2: only activations quantized; Lemma 3: only weights)
+    y_ref = torch.from_numpy(y.astype(np.float32)).to(DEV)
+    act_db, w_db = cat.one_sided_sqnr(to_dev(L.x_eval), to_dev(L.W), k, g["T"], torch.from_numpy(Tinv).to(DEV),
+                                      g["xq"], g["sx"], g["Wq"], g["sw"], y_ref)
+    assert abs(act_db - O.db(O.sqnr_act_only(Xp, Wp))) < 0.01, (act_db, O.db(O.sqnr_act_only(Xp, Wp)))
+    assert abs(w_db - O.db(O.sqnr_weight_only(Xp, Wp))) < 0.01, (w_db, O.db(O.sqnr_weight_only(Xp, Wp)))
     assert cat.cat_device_status()[0] == 0
+
+
+@pytest.mark.parametrize("rows,d,k,transpose,dtype", [(70, 256, 32, False, "f32"), (300, 512, 128, True, "bf16"),
+                                                      (5, 64, 16, False, "bf16"), (129, 768, 256, True, "f32")])
+def test_block_transform_and_dequantize(rows, d, k, transpose, dtype):
+    rng = np.random.default_rng(rows + d)
+    V = WL.cast(rng.standard_normal((rows, d)) * rng.lognormal(0, 1, d), dtype)
+    M = (rng.standard_normal((d // k, k, k)) / np.sqrt(k)).astype(np.float32)
+    out = cat.cat_block_transform(to_dev(V), k, torch.from_numpy(M).to(DEV), transpose=transpose).cpu().numpy()
+    Mb = np.transpose(M, (0, 2, 1)) if transpose else M          # v'_b = M_b v_b, or M_b^T v_b
+    ref = O.apply_act_transform(V.values, Mb.astype(np.float64))
+    assert rel_fro(out, ref) < 1e-6
+    q = WL.random_codes(rng, (rows, d)).astype(np.int64)
+    s_ = rng.uniform(0.01, 1, rows).astype(np.float32)
+    deq = cat.cat_dequantize_codes(torch.from_numpy(sm4x8.pack(q)).to(DEV), torch.from_numpy(s_).to(DEV)).cpu().numpy()
+    np.testing.assert_array_equal(deq, (q * s_[:, None].astype(np.float64)).astype(np.float32))
+
+
+@pytest.mark.parametrize("m,n,kd", [(1, 1, 1), (130, 257, 96), (512, 384, 1024), (33, 1000, 17)])
+def test_gemm_f32(m, n, kd):
+    rng = np.random.default_rng(m + n + kd)
+    A = rng.standard_normal((m, kd)).astype(np.float32)
+    B = rng.standard_normal((n, kd)).astype(np.float32)
+    C = cat.cat_gemm_f32(torch.from_numpy(A).to(DEV), torch.from_numpy(B).to(DEV)).cpu().numpy()
+    ref = A.astype(np.float64) @ B.astype(np.float64).T
+    assert np.max(np.abs(C - ref)) <= 1e-5 * np.sqrt(kd) * np.max(np.abs(ref)) + 1e-6
