@@ -241,6 +241,45 @@ def build_transform(kind: str, d: int, k: int, Sigma_x_blocks: Optional[np.ndarr
     return T, Ti
 
 
+def block_diag(blocks: np.ndarray) -> np.ndarray:
+    """The dense d x d matrix of [d/k, k, k] diagonal blocks."""
+    nb, k, _ = blocks.shape
+    out = np.zeros((nb * k, nb * k))
+    for b in range(nb):
+        out[b * k:(b + 1) * k, b * k:(b + 1) * k] = blocks[b]
+    return out
+
+
+def build_transform_full_hadamard(d: int, k: int, Sigma_x_blocks: np.ndarray, Sigma_w_blocks: np.ndarray):
+    """The approximately optimal transform of Sec. 4 with a full-size Hadamard: the block-diagonal
+    alignment-optimal M_hat_block (Eq. 7 on every k x k block, Eq. 10) composed with the orthonormal
+    Sylvester H_d over all d channels (d a power of two): T = H_d M_hat_block (dense d x d),
+    T^{-1} = M_hat_block^{-1} H_d^T.  Returns ``(T, T^{-1}, M blocks, M^{-1} blocks)``."""
+    nb = d // k
+    M = np.empty((nb, k, k))
+    Mi = np.empty((nb, k, k))
+    for b in range(nb):
+        M[b], Mi[b] = alignment_optimal_M(Sigma_x_blocks[b], Sigma_w_blocks[b])
+    H = hadamard(d)
+    return H @ block_diag(M), block_diag(Mi) @ H.T, M, Mi
+
+
+def cat_layer_dense(X: np.ndarray, W: np.ndarray, T: np.ndarray, Tinv: np.ndarray) -> Dict[str, object]:
+    """The layer with a dense transform (Sec. 3, Eq. 5): x' = T x, W' = W T^{-1}, per-token and
+    per-channel symmetric INT4 codes, integer GEMM, SQNR against y = W x."""
+    X = np.asarray(X, dtype=np.float64)
+    W = np.asarray(W, dtype=np.float64)
+    Xt = X @ T.T
+    Wt = W @ Tinv
+    qx, sx, pre_x = quantize_rows_symmetric(Xt)
+    qw, sw, pre_w = quantize_rows_symmetric(Wt)
+    acc, y_hat = w4a4_linear(qx, sx, qw, sw)
+    y = linear(X, W)
+    sig, err = sqnr_sums(y, y_hat)
+    return dict(Xt=Xt, Wt=Wt, qx=qx, sx=sx, pre_x=pre_x, qw=qw, sw=sw, pre_w=pre_w, acc=acc, y_hat=y_hat, y=y,
+                sqnr_db=10.0 * np.log10(sig / err))
+
+
 def apply_act_transform(X: np.ndarray, T_blocks: np.ndarray) -> np.ndarray:
     """``x' = T x`` for every token row: ``X'_b = X_b T_b^T`` block by block."""
     X = np.asarray(X, dtype=np.float64)

@@ -642,3 +642,46 @@ def test_interval_count_of_the_grid_is_measured_by_the_noise():
         n_meas = 2.0 / np.sqrt(12 * np.mean(e * e))
         assert abs(n_meas / O.n_intervals(bits) - 1) < 0.01, (bits, n_meas)
         assert abs(n_meas / O.n_intervals(bits, paper=True) - 1) > 0.05 or bits == 8
+
+
+# ------------------------------------------------------------------------------------------
+# Full-size Hadamard and the alignment ceiling (Sec. 4: T = H M_hat; Eq. 9)
+# ------------------------------------------------------------------------------------------
+
+def test_full_size_hadamard_keeps_alignment_and_function():
+    """Composing the block M_hat with the full-size H_d changes concentration only: A(T x, W T^{-1})
+    equals A(M_hat x, W M_hat^{-1}) exactly (alignment is rotation invariant, Sec. 2 Eq. 4 / Sec. 4),
+    and (W T^{-1})(T x) = W x (Eq. 5)."""
+    rng = _rng(70)
+    d, k = 64, 16
+    X = rng.standard_normal((600, d)) @ (rng.standard_normal((d, d)) * 0.3 + np.eye(d))
+    X[:, 5] *= 30.0
+    W = rng.standard_normal((40, d)) * 0.05
+    Sx = O.calib_cov_block_sums(X, k) / X.shape[0]
+    Sw = O.weight_autocorr_blocks(W, k)
+    T, Ti, M, Mi = O.build_transform_full_hadamard(d, k, Sx, Sw)
+    np.testing.assert_allclose(T @ Ti, np.eye(d), atol=1e-10)
+    np.testing.assert_allclose((W @ Ti) @ (X @ T.T).T, W @ X.T, rtol=1e-9, atol=1e-9)
+    Mb, Mib = O.block_diag(M), O.block_diag(Mi)
+    assert abs(O.alignment(X @ T.T, W @ Ti) / O.alignment(X @ Mb.T, W @ Mib) - 1) < 1e-12
+    # the block-H_k variant has the same alignment too (its rotation is block-diagonal)
+    Tk, Tik = O.build_transform("cat", d, k, Sx, Sw)
+    assert abs(O.alignment(O.apply_act_transform(X, Tk), O.apply_weight_transform(W, Tik)) /
+               O.alignment(X @ T.T, W @ Ti) - 1) < 1e-10
+    # an outlier channel is spread over all d channels by H_d, over its own block only by H_k
+    ct_full = O.concentration_act(X @ T.T)
+    ct_block = O.concentration_act(O.apply_act_transform(X, Tk))
+    assert ct_full > ct_block
+
+
+def test_full_rank_with_full_hadamard_reaches_the_ceiling():
+    """k = d: M_hat is the full-rank optimum and H_d M_hat reaches A_max of Eq. 9 (R11)."""
+    rng = _rng(71)
+    d = 16
+    X = rng.standard_normal((4000, d)) @ rng.standard_normal((d, d))
+    W = rng.standard_normal((24, d))                 # d_out >= d: Sigma_w positive definite
+    Sx = X.T @ X / X.shape[0]
+    T, Ti, _, _ = O.build_transform_full_hadamard(d, d, Sx[None], (W.T @ W)[None])
+    assert abs(O.alignment(X @ T.T, W @ Ti) / O.max_alignment(Sx, W) - 1) < 1e-8
+    r = O.cat_layer_dense(X, W, T, Ti)
+    assert np.isfinite(r["sqnr_db"]) and np.max(np.abs(r["qx"])) == 7
