@@ -24,6 +24,7 @@ step overlapping the compute of its neighbours (three streams).
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import json
 import os
 import statistics
@@ -363,6 +364,7 @@ def transform_sweep(cat, L, x, W, xc, y_ref):
         diag[kind] = dk
     out["diagnostics"] = diag
     out["bits"] = bit_width_sweep(cat, L, x, W, xc, y_ref)
+    out["alignment"] = alignment_sweep(cat, L)
     status, detail = cat.cat_device_status()
     if status != 0:
         raise DeviceTimeout(f"device status 0x{detail:x} after the transform sweep")
@@ -407,6 +409,57 @@ def bit_width_sweep(cat, L, x, W, xc, y_ref, steps=10):
             del T, wp, sw, rs, xp, sx, zx, y, g
         out[kind] = vals
         out[kind + "_gemm_ms"] = ms
+    return out
+
+
+def alignment_sweep(cat, L, max_d=1024):
+    """How far block CAT sits from the alignment ceiling (Sec. 4, Eq. 9): A_max from the full Sigma_x
+    and Sigma_w (Gram matrices on the GPU, eigenvalues on the host), beside the alignment and SQNR of the
+    identity, the k = 1 diagonal optimum, block CAT at every k and block CAT with the full-size Hadamard
+    (d_in = 2^m).  A_max and every A are taken on the evaluation tokens (the transforms come from the
+    calibration split).  The host eigen-decomposition bounds d_in; a larger layer is replaced by one of the
+    same generator with max_d input channels (named in the result)."""
+    cfg = L.cfg
+    if cfg.d_in > max_d:
+        d_out = min(cfg.d_out, 2 * max_d)
+        cfg = dataclasses.replace(cfg, name=f"{cfg.name} reduced to {max_d} -> {d_out}, 2048 tokens", d_in=max_d,
+                                  d_out=d_out, n_eval=min(cfg.n_eval, 2048), n_calib=max(cfg.n_calib, 2 * max_d))
+        L = WL.make_layer(cfg)
+    dev = torch.device("cuda", torch.cuda.current_device())
+    x, W, xc = to_dev(L.x_eval, dev), to_dev(L.W, dev), to_dev(L.x_calib, dev)
+    y_ref = (x.float() @ W.float().t()).contiguous()
+    # the ceiling of the alignment measured below, i.e. on the evaluation tokens' statistics
+    Sx = cat.cat_gram_f32(x).double().cpu().numpy() / cfg.n_eval
+    Sw = cat.cat_gram_f32(W).double().cpu().numpy()
+    a_max, _, _ = cat.cat_alignment_ceiling_host(Sx, Sw)
+    db = lambda v: round(10.0 * float(np.log10(v)), 3)  # noqa: E731
+    out = {"layer": cfg.name, "d_in": cfg.d_in, "A_max_db": db(a_max), "A_db": {}, "sqnr_db": {}}
+    sum_y2 = float(cat.cat_sqnr(y_ref, y_ref)[0].item())
+    pow2 = cfg.d_in & (cfg.d_in - 1) == 0
+    runs = [("identity", "identity", 64), ("cat_diag", "cat_diag", 64)] + \
+           [(f"cat k={k}", "cat", k) for k in (16, 32, 64, 128, 256) if cfg.d_in % k == 0] + \
+           ([("cat_hd k=128", "cat_hd", 128)] if pow2 else [])
+    for name, kind, k in runs:
+        sig = cat.cat_calib_cov(xc, k) if kind != "identity" else None
+        try:
+            T, Wq, sw = cat.cat_quantize_weights(W, k, kind, sigma_x=sig, n_calib=cfg.n_calib)
+        except cat.CatError as err:           # fewer calibration tokens than k: singular Sigma_x blocks
+            out["sqnr_db"][name] = out["A_db"][name] = None
+            out.setdefault("skipped", []).append(f"{name}: {err}")
+            continue
+        if kind == "cat_hd":
+            xq, sx = cat.cat_transform_quantize_act_hd(x, T, k)
+            xt = cat.cat_fwht_rows(cat.cat_block_transform(x, k, T))
+            Minv = torch.linalg.inv(T.double()).float().contiguous()
+            wt = cat.cat_fwht_rows(cat.cat_block_transform(W, k, Minv, transpose=True))
+        else:
+            xq, sx = cat.cat_transform_quantize_act(x, T, k)
+            xt = cat.cat_block_transform(x, k, T)
+            wt = cat.cat_block_transform(W, k, torch.linalg.inv(T.double()).float().contiguous(), transpose=True)
+        y = cat.cat_w4a4_linear(xq, sx, Wq, sw)
+        out["sqnr_db"][name] = round(float(cat.cat_sqnr(y_ref, y)[2].item()), 3)
+        # A = sum y^2 / (||W'||_F^2 sum ||x'||^2) (Lemma 2)
+        out["A_db"][name] = db(sum_y2 / (float((wt.double() ** 2).sum()) * float((xt.double() ** 2).sum())))
     return out
 
 

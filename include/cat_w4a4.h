@@ -72,7 +72,12 @@ typedef enum { CAT_F32 = 0, CAT_BF16 = 1 } cat_dtype;
 typedef enum {
   CAT_T_IDENTITY = 0,        /* T = I: plain W4A4 RTN */
   CAT_T_RHT = 1,             /* T_b = H_k Diag(sigma_b): randomized Hadamard rotation, signs given by the caller */
-  CAT_T_CAT = 2              /* T_b = H_k M_b, M_b = (Sigma_w_b # Sigma_x_b^{-1})^{1/2} (Sec. 4, Eq. 7, Eq. 10) */
+  CAT_T_CAT = 2,             /* T_b = H_k M_b, M_b = (Sigma_w_b # Sigma_x_b^{-1})^{1/2} (Sec. 4, Eq. 7, Eq. 10) */
+  CAT_T_DIAG = 3,            /* the k = 1 optimum (end of Sec. 4): T = Diag(m), m_i = (Sigma_w_ii / Sigma_x_ii)^{1/4},
+                                stored as k x k diagonal blocks */
+  CAT_T_CAT_HD = 4           /* T = H_d M_block (Sec. 4, "approximately optimal transform" with the full-size
+                                Hadamard over all d_in = 2^m channels): T_blocks hold the M_b; the online path
+                                is cat_transform_quantize_act_hd */
 } cat_tkind;
 
 /* Human-readable name of a status code (static string). */
@@ -108,7 +113,9 @@ cat_status cat_calib_cov(const void* x, cat_dtype dtype, int64_t n, int64_t d, i
  * cat_quantize_weights -- offline weight preparation (Sec. 3 Eq. 5: W' = W T^{-1}; Sec. 4 Eq. 7
  * and Eq. 10: the block transform; Sec. 6: per-output-channel symmetric RTN).
  *   W              device [d_out][d_in] in `dtype`.
- *   kind           transform family.
+ *   kind           transform family.  CAT_T_DIAG and CAT_T_CAT_HD need sigma_x_blocks as CAT does;
+ *                  CAT_T_CAT_HD needs d_in = 2^m <= 32768, returns the M_b blocks in T_blocks and the
+ *                  codes of W M^{-1} H_d (through a float32 scratch from the stream-ordered pool).
  *   sigma_x_blocks device [d_in/k][k][k] float64 sums from cat_calib_cov (CAT only; else may be NULL).
  *   n_calib        number of tokens behind sigma_x_blocks (CAT only, >= 1).
  *   rht_signs      HOST [d_in] float32, each +1 or -1 (RHT only; else may be NULL).
@@ -353,6 +360,37 @@ cat_status cat_dequantize_codes(const uint8_t* codes, const float* scale, int64_
  */
 cat_status cat_gemm_f32(const float* A, const float* B, int64_t m, int64_t n, int64_t kdim, float* C,
                         cat_stream_t stream);
+
+/*
+ * The alignment ceiling and the full-size Hadamard (Sec. 4: "Optimizing alignment", Eq. 9; the
+ * approximately optimal transform T = H M with H over all channels).
+ */
+
+/*
+ * cat_transform_quantize_act_hd -- online activations under CAT_T_CAT_HD: x' = H_d (M_block x) with the
+ * orthonormal Sylvester H_d over all d_in = 2^m <= 32768 channels, then per-token symmetric INT4 codes
+ * (as cat_transform_quantize_act).  M_blocks: the T_blocks of cat_quantize_weights(kind = CAT_T_CAT_HD).
+ * Takes float32 scratch from the stream-ordered pool; synchronizes the stream before returning.
+ */
+cat_status cat_transform_quantize_act_hd(const void* x, cat_dtype dtype, int64_t n, int64_t d_in, int32_t k,
+                                         const float* M_blocks, uint8_t* xq, float* x_scale, cat_stream_t stream);
+
+/* cat_fwht_rows -- in place, V[r] <- H_d V[r] / sqrt(d) for every row (Sylvester order), V device [rows][d]
+ * float32, d = 2^m in 2..32768.  One shared-memory row per CTA, log2(d) butterfly stages. */
+cat_status cat_fwht_rows(float* V, int64_t rows, int64_t d, cat_stream_t stream);
+
+/* cat_gram_f32 -- C = X^T X (C[i][j] = sum_t X[t][i] X[t][j]) in float32, X device [n][d] in `dtype`,
+ * C device [d][d]: the full Sigma_x (over n) and Sigma_w that the ceiling needs. */
+cat_status cat_gram_f32(const void* X, cat_dtype dtype, int64_t n, int64_t d, float* C, cat_stream_t stream);
+
+/*
+ * cat_alignment_ceiling_host -- the largest alignment any invertible transform reaches (Eq. 9):
+ *   A_max = sum_i mu_i / (sum_i sqrt(mu_i))^2,  mu = eigenvalues of Sigma_x^{1/2} Sigma_w Sigma_x^{1/2}
+ *   (equivalently of W Sigma_x W^T).  All pointers HOST: Sigma_x, Sigma_w [d][d] float64 (Sigma_x
+ *   positive definite), out3 = { A_max, sum mu, sum sqrt(mu) }.  d <= 4096 (a Jacobi eigen-decomposition
+ *   on the calling thread).  CAT_ERR_NUMERIC if Sigma_x is not positive definite.
+ */
+cat_status cat_alignment_ceiling_host(const double* sigma_x, const double* sigma_w, int64_t d, double* out3);
 
 /*
  * cat_device_status -- synchronizes `stream`, then reads and clears the device status word.

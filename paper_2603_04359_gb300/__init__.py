@@ -22,6 +22,7 @@ __all__ = [
     "cat_w4a4_linear", "cat_sqnr", "cat_device_status", "cat_version", "KIND",
     "cat_dp_planes", "cat_transform_quantize_act_dp", "cat_quantize_weights_dp", "cat_linear_dp",
     "cat_block_transform", "cat_dequantize_codes", "cat_gemm_f32", "one_sided_sqnr", "cat_set_wait_limit_ns",
+    "cat_transform_quantize_act_hd", "cat_fwht_rows", "cat_gram_f32", "cat_alignment_ceiling_host",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -29,7 +30,7 @@ _LIB_PATH = os.path.join(_HERE, "libcatw4a4.so")
 _HEADER = os.path.join(os.path.dirname(_HERE), "include", "cat_w4a4.h")
 _lib: Optional[ctypes.CDLL] = None
 
-KIND = {"identity": 0, "rht": 1, "cat": 2}
+KIND = {"identity": 0, "rht": 1, "cat": 2, "cat_diag": 3, "cat_hd": 4}
 _DTYPE = {torch.float32: 0, torch.bfloat16: 1}
 _STATUS = {0: "CAT_OK", 1: "CAT_ERR_INVALID_ARG", 2: "CAT_ERR_SHAPE", 3: "CAT_ERR_ALIGNMENT", 4: "CAT_ERR_NUMERIC",
            5: "CAT_ERR_UNSUPPORTED", 6: "CAT_ERR_CUDA", 7: "CAT_ERR_TIMEOUT"}
@@ -74,6 +75,10 @@ def load_library() -> ctypes.CDLL:
         "cat_block_transform": ([P, I, I64, I64, I32, P, I, P, P], I),
         "cat_dequantize_codes": ([P, P, I64, I64, P, P], I),
         "cat_gemm_f32": ([P, P, I64, I64, I64, P, P], I),
+        "cat_transform_quantize_act_hd": ([P, I, I64, I64, I32, P, P, P, P], I),
+        "cat_fwht_rows": ([P, I64, I64, P], I),
+        "cat_gram_f32": ([P, I, I64, I64, P, P], I),
+        "cat_alignment_ceiling_host": ([P, P, I64, P], I),
         "cat_transform_quantize_act_dp": ([P, I, I64, I64, I32, P, I32, I32, P, P, P, P], I),
         "cat_quantize_weights_dp": ([P, I, I64, I64, I32, I, P, I64, P, I32, I32, P, P, P, P, P], I),
         "cat_linear_dp": ([P, I32, I32, P, P, P, I32, P, P, I64, I64, I64, P, P, P], I),
@@ -455,6 +460,48 @@ def one_sided_sqnr(x: torch.Tensor, W: torch.Tensor, k: int, T: torch.Tensor, Ti
     y_x = cat_gemm_f32(cat_dequantize_codes(xq, x_scale), wt)
     y_w = cat_gemm_f32(xt, cat_dequantize_codes(Wq, w_scale))
     return float(cat_sqnr(y_ref, y_x)[2].item()), float(cat_sqnr(y_ref, y_w)[2].item())
+
+
+def cat_transform_quantize_act_hd(x: torch.Tensor, M_blocks: torch.Tensor, k: int) -> Tuple[torch.Tensor, torch.Tensor]:
+    """x' = H_d (M_block x) and its per-token INT4 codes (kind "cat_hd"): (SM4x8 uint8 [n, d_in/2], float32 [n])."""
+    _need(x, "x")
+    n, d_in = x.shape
+    _expect(M_blocks, "M_blocks", torch.float32, (d_in // k, k, k), x.device)
+    xq = torch.empty((n, d_in // 2), dtype=torch.uint8, device=x.device)
+    sx = torch.empty((n,), dtype=torch.float32, device=x.device)
+    _check("cat_transform_quantize_act_hd", load_library().cat_transform_quantize_act_hd(
+        _ptr(x), _dtype(x), n, d_in, k, _ptr(M_blocks), _ptr(xq), _ptr(sx), _stream(x.device)))
+    return xq, sx
+
+
+def cat_fwht_rows(V: torch.Tensor) -> torch.Tensor:
+    """In place: every row of the float32 V [rows, d] becomes H_d v / sqrt(d)."""
+    rows, d = V.shape
+    _expect(V, "V", torch.float32, (rows, d), V.device)
+    _check("cat_fwht_rows", load_library().cat_fwht_rows(_ptr(V), rows, d, _stream(V.device)))
+    return V
+
+
+def cat_gram_f32(X: torch.Tensor) -> torch.Tensor:
+    """X^T X in float32 [d, d] for X [n, d] (float32 or bf16)."""
+    _need(X, "X")
+    n, d = X.shape
+    C = torch.empty((d, d), dtype=torch.float32, device=X.device)
+    _check("cat_gram_f32", load_library().cat_gram_f32(_ptr(X), _dtype(X), n, d, _ptr(C), _stream(X.device)))
+    return C
+
+
+def cat_alignment_ceiling_host(sigma_x: np.ndarray, sigma_w: np.ndarray) -> Tuple[float, float, float]:
+    """Eq. 9 on the host from full Sigma_x, Sigma_w [d, d]: (A_max, sum mu, sum sqrt mu)."""
+    sx = np.ascontiguousarray(sigma_x, dtype=np.float64)
+    sw = np.ascontiguousarray(sigma_w, dtype=np.float64)
+    d = sx.shape[0]
+    if sx.shape != (d, d) or sw.shape != (d, d):
+        raise ValueError("sigma_x and sigma_w must be square and of the same size")
+    out = np.zeros(3)
+    vp = lambda a: a.ctypes.data_as(ctypes.c_void_p)  # noqa: E731
+    _check("cat_alignment_ceiling_host", load_library().cat_alignment_ceiling_host(vp(sx), vp(sw), d, vp(out)))
+    return float(out[0]), float(out[1]), float(out[2])
 
 
 def cat_set_wait_limit_ns(ns: int) -> None:

@@ -30,6 +30,8 @@ cudaError_t launch_dequantize_sm4x8(const uint8_t* codes, const float* scale, in
                                     cudaStream_t stream);
 cudaError_t launch_gemm_f32_nt(const float* A, const float* B, float* C, int64_t M, int64_t N, int64_t K,
                                cudaStream_t stream);
+cudaError_t launch_fwht_rows(float* V, int64_t rows, int64_t d, cudaStream_t stream);
+cudaError_t launch_gram_f32(const void* X, int dtype, int64_t n, int64_t d, float* C, cudaStream_t stream);
 cudaError_t set_decode_wait_limit(uint64_t ns);
 cudaError_t set_dp_wait_limit(uint64_t ns);
 size_t dp_l24_work_bytes(int64_t n);
@@ -151,6 +153,33 @@ cat_status check_din(int64_t d_in) {
   return CAT_OK;
 }
 
+// v' = H_d (A_b v_b) for every row (blocks applied as v'_b = A_b v_b, or A_b^T v_b with transpose), then
+// the per-row symmetric INT4 codes of the float32 rows (identity blocks of 16).  Float32 scratch taken
+// from the stream-ordered pool.
+cudaError_t transform_fwht_quantize(const void* V, int dtype, int64_t rows, int64_t d, int k, const float* A,
+                                    int transpose, uint8_t* codes, float* scale, uint32_t* status, cudaStream_t s) {
+  float* tmp = nullptr;
+  float* eye = nullptr;
+  const size_t eye_elems = (size_t)(d / 16) * 256;
+  cudaError_t e = cudaMallocAsync((void**)&tmp, (size_t)rows * d * sizeof(float), s);
+  if (e != cudaSuccess) return e;
+  if ((e = cudaMallocAsync((void**)&eye, eye_elems * sizeof(float), s)) != cudaSuccess) {
+    cudaFreeAsync(tmp, s);
+    return e;
+  }
+  std::vector<float> eye_h(eye_elems, 0.f);
+  for (size_t b = 0; b < (size_t)(d / 16); ++b)
+    for (int i = 0; i < 16; ++i) eye_h[b * 256 + (size_t)i * 16 + i] = 1.f;
+  e = cudaMemcpyAsync(eye, eye_h.data(), eye_elems * sizeof(float), cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cat::launch_block_transform(V, dtype, rows, d, k, A, transpose, tmp, s);
+  if (e == cudaSuccess) e = cat::launch_fwht_rows(tmp, rows, d, s);
+  if (e == cudaSuccess) e = cat::launch_transform_quantize(tmp, 0, rows, d, 16, eye, codes, scale, status, s);
+  cudaError_t e2 = cudaStreamSynchronize(s);   // eye_h is read by the copy above
+  cudaFreeAsync(tmp, s);
+  cudaFreeAsync(eye, s);
+  return e != cudaSuccess ? e : e2;
+}
+
 }  // namespace
 
 extern "C" {
@@ -197,7 +226,8 @@ cat_status cat_calib_cov(const void* x, cat_dtype dtype, int64_t n, int64_t d, i
 cat_status cat_build_transform_host(cat_tkind kind, int64_t d_in, int32_t k, const double* sigma_x_blocks,
                                     int64_t n_calib, const double* sigma_w_blocks, const float* rht_signs,
                                     double* T_out, double* Tinv_out) {
-  if (kind != CAT_T_IDENTITY && kind != CAT_T_RHT && kind != CAT_T_CAT) return fail(CAT_ERR_INVALID_ARG, "unknown kind");
+  if (kind != CAT_T_IDENTITY && kind != CAT_T_RHT && kind != CAT_T_CAT && kind != CAT_T_DIAG && kind != CAT_T_CAT_HD)
+    return fail(CAT_ERR_INVALID_ARG, "unknown kind");
   if (!valid_k(k)) return fail(CAT_ERR_SHAPE, "k must be one of 16, 32, 64, 128, 256");
   if (d_in <= 0 || d_in % k != 0) return fail(CAT_ERR_SHAPE, "d_in must be a positive multiple of k");
   if (!T_out || !Tinv_out) return fail(CAT_ERR_INVALID_ARG, "NULL output");
@@ -206,7 +236,7 @@ cat_status cat_build_transform_host(cat_tkind kind, int64_t d_in, int32_t k, con
     for (int64_t i = 0; i < d_in; ++i)
       if (rht_signs[i] != 1.0f && rht_signs[i] != -1.0f) return fail(CAT_ERR_INVALID_ARG, "rht_signs must be +-1");
   }
-  if (kind == CAT_T_CAT) {
+  if (kind == CAT_T_CAT || kind == CAT_T_DIAG || kind == CAT_T_CAT_HD) {
     if (!sigma_x_blocks || !sigma_w_blocks) return fail(CAT_ERR_INVALID_ARG, "CAT needs sigma_x and sigma_w blocks");
     if (n_calib < 1) return fail(CAT_ERR_INVALID_ARG, "n_calib must be >= 1");
     const size_t cnt = (size_t)d_in * (size_t)k;
@@ -226,13 +256,17 @@ cat_status cat_quantize_weights(const void* W, cat_dtype dtype, int64_t d_out, i
                                 const float* rht_signs, float* T_blocks, uint8_t* Wq, float* w_scale,
                                 cat_stream_t stream) {
   if (dtype != CAT_F32 && dtype != CAT_BF16) return fail(CAT_ERR_INVALID_ARG, "unknown dtype");
-  if (kind != CAT_T_IDENTITY && kind != CAT_T_RHT && kind != CAT_T_CAT) return fail(CAT_ERR_INVALID_ARG, "unknown kind");
+  if (kind != CAT_T_IDENTITY && kind != CAT_T_RHT && kind != CAT_T_CAT && kind != CAT_T_DIAG && kind != CAT_T_CAT_HD)
+    return fail(CAT_ERR_INVALID_ARG, "unknown kind");
+  if (kind == CAT_T_CAT_HD && (d_in & (d_in - 1)) != 0) return fail(CAT_ERR_SHAPE, "the full-size Hadamard needs d_in = 2^m");
+  if (kind == CAT_T_CAT_HD && d_in > 32768) return fail(CAT_ERR_SHAPE, "the full-size Hadamard needs d_in <= 32768");
   if (d_out <= 0) return fail(CAT_ERR_SHAPE, "d_out must be >= 1");
   cat_status st = check_din(d_in);
   if (st != CAT_OK) return st;
   if (!valid_k(k) || d_in % k != 0) return fail(CAT_ERR_SHAPE, "k must be one of 16..256 (power of two) and divide d_in");
   if (!W || !T_blocks || !Wq || !w_scale) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
-  if (kind == CAT_T_CAT && (!sigma_x_blocks || n_calib < 1))
+  const bool cat_like = kind == CAT_T_CAT || kind == CAT_T_DIAG || kind == CAT_T_CAT_HD;
+  if (cat_like && (!sigma_x_blocks || n_calib < 1))
     return fail(CAT_ERR_INVALID_ARG, "CAT needs sigma_x_blocks and n_calib >= 1");
   if (kind == CAT_T_RHT && !rht_signs) return fail(CAT_ERR_INVALID_ARG, "RHT needs rht_signs");
   if (!aligned16(W) || !aligned16(T_blocks) || !aligned16(Wq) || !aligned16(w_scale) ||
@@ -245,7 +279,7 @@ cat_status cat_quantize_weights(const void* W, cat_dtype dtype, int64_t d_out, i
   const size_t kk = (size_t)k * k, nblk = (size_t)nb * kk;
   std::vector<double> sx_h, sw_h;
   cudaError_t e;
-  if (kind == CAT_T_CAT) {
+  if (cat_like) {
     double* sw_d = nullptr;
     if ((e = cudaMallocAsync((void**)&sw_d, nblk * sizeof(double), s)) != cudaSuccess) return cuda_fail(e, "cudaMallocAsync");
     uint32_t* st_word = status_word(&e);
@@ -277,7 +311,13 @@ cat_status cat_quantize_weights(const void* W, cat_dtype dtype, int64_t d_out, i
   if ((e = cudaMallocAsync((void**)&aw_d, nblk * sizeof(float), s)) != cudaSuccess) return cuda_fail(e, "cudaMallocAsync");
   e = cudaMemcpyAsync(T_blocks, Tf.data(), nblk * sizeof(float), cudaMemcpyHostToDevice, s);
   if (e == cudaSuccess) e = cudaMemcpyAsync(aw_d, Awf.data(), nblk * sizeof(float), cudaMemcpyHostToDevice, s);
-  if (e == cudaSuccess) e = cat::launch_transform_quantize(W, (int)dtype, d_out, d_in, k, aw_d, Wq, w_scale, status, s);
+  if (kind == CAT_T_CAT_HD) {
+    // W' = W M^{-1} H_d: the rows through the blocks (M_b^{-1})^T, the full-size Hadamard, then the
+    // codes of the float32 rows (identity blocks)
+    if (e == cudaSuccess) e = transform_fwht_quantize(W, (int)dtype, d_out, d_in, k, aw_d, 1, Wq, w_scale, status, s);
+  } else if (e == cudaSuccess) {
+    e = cat::launch_transform_quantize(W, (int)dtype, d_out, d_in, k, aw_d, Wq, w_scale, status, s);
+  }
   cudaFreeAsync(aw_d, s);
   cudaError_t e2 = cudaStreamSynchronize(s);  // host buffers above must outlive the copies
   if (e != cudaSuccess) return cuda_fail(e, "weight quantization");
@@ -669,5 +709,64 @@ cat_status cat_gemm_f32(const float* A, const float* B, int64_t m, int64_t n, in
   if (st != CAT_OK) return st;
   cudaError_t e = cat::launch_gemm_f32_nt(A, B, C, m, n, kdim, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "cat_gemm_f32 launch");
+  return ok();
+}
+
+// ---- the alignment ceiling and the full-size Hadamard (Sec. 4: Eq. 9; T = H_d M_hat_block)
+
+cat_status cat_transform_quantize_act_hd(const void* x, cat_dtype dtype, int64_t n, int64_t d_in, int32_t k,
+                                         const float* M_blocks, uint8_t* xq, float* x_scale, cat_stream_t stream) {
+  if (dtype != CAT_F32 && dtype != CAT_BF16) return fail(CAT_ERR_INVALID_ARG, "unknown dtype");
+  if (n < 0) return fail(CAT_ERR_SHAPE, "n must be >= 0");
+  cat_status st = check_din(d_in);
+  if (st != CAT_OK) return st;
+  if ((d_in & (d_in - 1)) != 0 || d_in > 32768) return fail(CAT_ERR_SHAPE, "the full-size Hadamard needs d_in = 2^m <= 32768");
+  if (!valid_k(k) || d_in % k != 0) return fail(CAT_ERR_SHAPE, "k must be one of 16..256 (power of two) and divide d_in");
+  if (n == 0) return ok();
+  if (n > 0x7FFFFFFF) return fail(CAT_ERR_SHAPE, "n too large");
+  if (!x || !M_blocks || !xq || !x_scale) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(x) || !aligned16(M_blocks) || !aligned16(xq) || !aligned16(x_scale))
+    return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  if ((st = check_device()) != CAT_OK) return st;
+  cudaError_t e;
+  uint32_t* status = status_word(&e);
+  if (!status) return cuda_fail(e, "status word");
+  e = transform_fwht_quantize(x, (int)dtype, n, d_in, k, M_blocks, 0, xq, x_scale, status, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cat_transform_quantize_act_hd");
+  return ok();
+}
+
+cat_status cat_fwht_rows(float* V, int64_t rows, int64_t d, cat_stream_t stream) {
+  if (rows < 0 || rows > 0x7FFFFFFF) return fail(CAT_ERR_SHAPE, "rows must be in [0, 2^31)");
+  if (d < 2 || (d & (d - 1)) != 0 || d > 32768) return fail(CAT_ERR_SHAPE, "d must be a power of two in 2..32768");
+  if (rows == 0) return ok();
+  if (!V) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(V)) return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  cat_status st = check_device();
+  if (st != CAT_OK) return st;
+  cudaError_t e = cat::launch_fwht_rows(V, rows, d, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cat_fwht_rows launch");
+  return ok();
+}
+
+cat_status cat_gram_f32(const void* X, cat_dtype dtype, int64_t n, int64_t d, float* C, cat_stream_t stream) {
+  if (dtype != CAT_F32 && dtype != CAT_BF16) return fail(CAT_ERR_INVALID_ARG, "unknown dtype");
+  if (n < 1 || n > 0x7FFFFFFF || d < 1 || d > 65536) return fail(CAT_ERR_SHAPE, "n in [1, 2^31), d in [1, 65536]");
+  if (!X || !C) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(X) || !aligned16(C)) return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  cat_status st = check_device();
+  if (st != CAT_OK) return st;
+  cudaError_t e = cat::launch_gram_f32(X, (int)dtype, n, d, C, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cat_gram_f32 launch");
+  return ok();
+}
+
+cat_status cat_alignment_ceiling_host(const double* sigma_x, const double* sigma_w, int64_t d, double* out3) {
+  if (d < 1 || d > 4096) return fail(CAT_ERR_SHAPE, "d must be in [1, 4096] (a host eigen-decomposition of d x d)");
+  if (!sigma_x || !sigma_w || !out3) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  for (int64_t i = 0; i < d * d; ++i)
+    if (!std::isfinite(sigma_x[i]) || !std::isfinite(sigma_w[i])) return fail(CAT_ERR_NUMERIC, "non-finite statistics");
+  if (!cat::alignment_ceiling_host(sigma_x, sigma_w, d, &out3[0], &out3[1], &out3[2]))
+    return fail(CAT_ERR_NUMERIC, "Sigma_x is not positive definite");
   return ok();
 }

@@ -10,6 +10,7 @@
 // like the values for non-negative floats).  A second kernel adds the rows' sums of squares and
 // squared ranges through the cross-CTA reduction of sqnr_slot.cuh, which also forms
 // 10 log10(sum ||v'||^2 / sum r^2) = C in dB.
+#include <cmath>
 #include <cstring>
 #include <mutex>
 
@@ -272,7 +273,101 @@ __global__ void __launch_bounds__(256) gemm_f32_nt_kernel(const float* __restric
   }
 }
 
+// In place, orthonormal: v <- H_d v / sqrt(d) for every row (Sylvester order), d = 2^m <= 32768.  One
+// CTA per row, the row in shared memory, log2(d) butterfly stages.
+__global__ void __launch_bounds__(512) fwht_rows_kernel(float* __restrict__ V, int64_t rows, int d, float scale) {
+  extern __shared__ float buf[];
+  const int64_t r = blockIdx.x;
+  float* row = V + r * d;
+  for (int i = threadIdx.x; i < d; i += blockDim.x) buf[i] = row[i];
+  __syncthreads();
+  for (int h = 1; h < d; h <<= 1) {
+    for (int p = threadIdx.x; p < d / 2; p += blockDim.x) {
+      const int i = (p / h) * 2 * h + (p % h), j = i + h;
+      const float a = buf[i], b = buf[j];
+      buf[i] = a + b;
+      buf[j] = a - b;
+    }
+    __syncthreads();
+  }
+  for (int i = threadIdx.x; i < d; i += blockDim.x) row[i] = buf[i] * scale;
+}
+
+// C[i][j] = sum_t X[t][i] X[t][j] in float32 (the full Gram matrix of the rows of X [n][d]): the
+// 128 x 128 tiles of the GEMM above, operands read down the columns of X (coalesced along i).
+template <typename Tin>
+__global__ void __launch_bounds__(256) gram_f32_kernel(const Tin* __restrict__ X, float* __restrict__ Cm, int n, int d) {
+  __shared__ __align__(16) float As[GK][GT + 4];
+  __shared__ __align__(16) float Bs[GK][GT + 4];
+  const int tid = threadIdx.x, tm = tid >> 4, tn = tid & 15;
+  const int m0 = blockIdx.y * GT, n0 = blockIdx.x * GT;
+  float acc[8][8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
+  for (int k0 = 0; k0 < n; k0 += GK) {
+    for (int e = tid; e < GT * GK; e += 256) {
+      const int kk = e / GT, c = e % GT;
+      const int t = k0 + kk;
+      As[kk][c] = (t < n && m0 + c < d) ? to_f32(X[(size_t)t * d + m0 + c]) : 0.f;
+      Bs[kk][c] = (t < n && n0 + c < d) ? to_f32(X[(size_t)t * d + n0 + c]) : 0.f;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < GK; ++kk) {
+      float a[8], b[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) a[i] = As[kk][tm + 16 * i];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) b[j] = Bs[kk][tn + 16 * j];
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int m = m0 + tm + 16 * i;
+    if (m >= d) continue;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int c = n0 + tn + 16 * j;
+      if (c < d) Cm[(size_t)m * d + c] = acc[i][j];
+    }
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_fwht_rows(float* V, int64_t rows, int64_t d, cudaStream_t stream) {
+  if (rows == 0) return cudaSuccess;
+  const size_t smem = (size_t)d * sizeof(float);
+  static std::once_flag once;
+  static cudaError_t attr = cudaSuccess;
+  std::call_once(once, [] {
+    attr = cudaFuncSetAttribute(fwht_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 32768 * 4);
+  });
+  if (attr != cudaSuccess) return attr;
+  const int threads = d / 2 < 512 ? (int)(d / 2 < 32 ? 32 : d / 2) : 512;
+  note_launch();
+  fwht_rows_kernel<<<(unsigned)rows, threads, smem, stream>>>(V, rows, (int)d, (float)(1.0 / std::sqrt((double)d)));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gram_f32(const void* X, int dtype, int64_t n, int64_t d, float* C, cudaStream_t stream) {
+  const int64_t g = (d + GT - 1) / GT;
+  if (g > 65535) return cudaErrorInvalidValue;
+  note_launch();
+  if (dtype == 0)
+    gram_f32_kernel<float><<<dim3((unsigned)g, (unsigned)g), 256, 0, stream>>>(static_cast<const float*>(X), C, (int)n, (int)d);
+  else
+    gram_f32_kernel<__nv_bfloat16><<<dim3((unsigned)g, (unsigned)g), 256, 0, stream>>>(
+        static_cast<const __nv_bfloat16*>(X), C, (int)n, (int)d);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_dequantize_sm4x8(const uint8_t* codes, const float* scale, int64_t rows, int64_t d, float* out,
                                     cudaStream_t stream) {

@@ -118,8 +118,10 @@ double hadamard_entry(int i, int j, double inv_sqrt_k) {
   return (__builtin_popcount((unsigned)(i & j)) & 1) ? -inv_sqrt_k : inv_sqrt_k;
 }
 
-// One CAT block: T = H M, Tinv = M^{-1} H^T.  Returns false if a block is not positive definite.
-bool cat_block(const double* sx_sum, double inv_n, const double* sw, int k, double* T, double* Ti) {
+// One CAT block: T = H M, Tinv = M^{-1} H^T (with_h), or T = M, Tinv = M^{-1} (the full-size
+// Hadamard variant, whose H_d is applied across all blocks afterwards).  Returns false if a block is
+// not positive definite.
+bool cat_block(const double* sx_sum, double inv_n, const double* sw, int k, double* T, double* Ti, bool with_h = true) {
   const size_t kk = (size_t)k * k;
   std::vector<double> Sx(kk), Sw(sw, sw + kk);
   for (size_t e = 0; e < kk; ++e) Sx[e] = sx_sum[e] * inv_n;
@@ -135,6 +137,11 @@ bool cat_block(const double* sx_sum, double inv_n, const double* sw, int k, doub
   matmul(tmp, Sxih, k, G);         // G = Sigma_w # Sigma_x^{-1}
   std::vector<double> M, Mi;
   if (!spd_powers(G, k, 0.5, M, -0.5, Mi)) return false;
+  if (!with_h) {
+    std::copy(M.begin(), M.end(), T);
+    std::copy(Mi.begin(), Mi.end(), Ti);
+    return true;
+  }
   const double h = 1.0 / std::sqrt((double)k);
   for (int i = 0; i < k; ++i)
     for (int j = 0; j < k; ++j) {
@@ -146,6 +153,21 @@ bool cat_block(const double* sx_sum, double inv_n, const double* sw, int k, doub
       T[(size_t)i * k + j] = t;
       Ti[(size_t)i * k + j] = ti;
     }
+  return true;
+}
+
+// The k = 1 optimum (end of Sec. 4): m_i = (Sigma_w_ii / Sigma_x_ii)^{1/4}, from the diagonals of the
+// k x k blocks.  Returns false for a non-positive diagonal entry.
+bool diag_block(const double* sx_sum, double inv_n, const double* sw, int k, double* T, double* Ti) {
+  for (int i = 0; i < k; ++i) {
+    const double sx = sx_sum[(size_t)i * k + i] * inv_n, swi = sw[(size_t)i * k + i];
+    if (!(sx > 0.0) || !(swi > 0.0) || !std::isfinite(sx) || !std::isfinite(swi)) return false;
+    const double m = std::pow(swi / sx, 0.25);
+    for (int j = 0; j < k; ++j) {
+      T[(size_t)i * k + j] = i == j ? m : 0.0;
+      Ti[(size_t)i * k + j] = i == j ? 1.0 / m : 0.0;
+    }
+  }
   return true;
 }
 
@@ -181,7 +203,10 @@ int build_transform_host(int kind, int64_t d_in, int k, const double* sigma_x, i
     for (;;) {
       const int64_t b = next.fetch_add(1);
       if (b >= nb) return;
-      if (!cat_block(sigma_x + b * kk, inv_n, sigma_w + b * kk, k, T_out + b * kk, Tinv_out + b * kk)) {
+      const bool good = kind == 3 ? diag_block(sigma_x + b * kk, inv_n, sigma_w + b * kk, k, T_out + b * kk, Tinv_out + b * kk)
+                                  : cat_block(sigma_x + b * kk, inv_n, sigma_w + b * kk, k, T_out + b * kk,
+                                              Tinv_out + b * kk, kind != 4);
+      if (!good) {
         int64_t expected = -1;
         bad.compare_exchange_strong(expected, b);
       }
@@ -198,6 +223,35 @@ int build_transform_host(int kind, int64_t d_in, int k, const double* sigma_x, i
     return 1;
   }
   return 0;
+}
+
+// A_max = Tr(P) / Tr(P^{1/2})^2, P = Sigma_x^{1/2} Sigma_w Sigma_x^{1/2} (Eq. 9, R11): the eigenvalues mu of
+// P are those of W Sigma_x W^T.  Full d x d matrices; Sigma_x must be positive definite, Sigma_w
+// positive semi-definite.  Returns false if not.
+bool alignment_ceiling_host(const double* sigma_x, const double* sigma_w, int64_t d, double* a_max, double* sum_mu,
+                            double* sum_sqrt_mu) {
+  const int k = (int)d;
+  std::vector<double> Sx(sigma_x, sigma_x + (size_t)k * k), Sw(sigma_w, sigma_w + (size_t)k * k);
+  std::vector<double> Sxh, unused;
+  if (!spd_powers(Sx, k, 0.5, Sxh, 1.0, unused)) return false;
+  std::vector<double> tmp, P;
+  matmul(Sxh, Sw, k, tmp);
+  matmul(tmp, Sxh, k, P);
+  std::vector<double> A((size_t)k * k), w, V;
+  for (int i = 0; i < k; ++i)
+    for (int j = 0; j < k; ++j) A[(size_t)i * k + j] = 0.5 * (P[(size_t)i * k + j] + P[(size_t)j * k + i]);
+  jacobi_eig(A, k, w, V);
+  double s = 0.0, r = 0.0;
+  for (double m : w) {
+    const double mu = m > 0.0 ? m : 0.0;   // rounding can leave tiny negative eigenvalues of a PSD P
+    s += mu;
+    r += std::sqrt(mu);
+  }
+  if (!(r > 0.0)) return false;
+  *a_max = s / (r * r);
+  if (sum_mu) *sum_mu = s;
+  if (sum_sqrt_mu) *sum_sqrt_mu = r;
+  return true;
 }
 
 }  // namespace cat

@@ -136,3 +136,40 @@ def test_wait_limit_setter_rejects_bounds_above_one_second():
     lib = cat.load_library()
     assert lib.cat_set_wait_limit_ns(ctypes.c_uint64(2_000_000_000)) == 1      # CAT_ERR_INVALID_ARG
     assert b"at most 1 s" in lib.cat_last_error()
+
+
+def test_host_builder_diagonal_and_full_hadamard_kinds_match_the_oracle():
+    """kind 3 (k = 1 optimum in k-blocks) and kind 4 (the M_b blocks of CAT with the full-size
+    Hadamard) against the oracle (host only)."""
+    rng = np.random.default_rng(81)
+    d, k = 64, 16
+    X = rng.standard_normal((500, d)) @ (rng.standard_normal((d, d)) * 0.3 + np.eye(d))
+    W = rng.standard_normal((80, d)) * 0.05
+    sx = O.calib_cov_block_sums(X, k)
+    sw = O.weight_autocorr_blocks(W, k)
+    T3, Ti3 = cat.cat_build_transform_host("cat_diag", d, k, sigma_x=sx, n_calib=X.shape[0], sigma_w=sw)
+    m = (np.sum(W * W, axis=0) / np.mean(X * X, axis=0)) ** 0.25          # end of Sec. 4 (R9)
+    np.testing.assert_allclose(O.block_diag(T3), np.diag(m), rtol=1e-12, atol=1e-15)
+    np.testing.assert_allclose(O.block_diag(Ti3), np.diag(1 / m), rtol=1e-12, atol=1e-15)
+    Tk1, _ = O.build_transform("cat", d, 1, O.calib_cov_block_sums(X, 1) / X.shape[0], O.weight_autocorr_blocks(W, 1))
+    np.testing.assert_allclose(np.diag(O.block_diag(T3)), Tk1[:, 0, 0], rtol=1e-10)
+    T4, Ti4 = cat.cat_build_transform_host("cat_hd", d, k, sigma_x=sx, n_calib=X.shape[0], sigma_w=sw)
+    _, _, M, Mi = O.build_transform_full_hadamard(d, k, sx / X.shape[0], sw)
+    np.testing.assert_allclose(T4, M, rtol=1e-8, atol=1e-10)
+    np.testing.assert_allclose(Ti4, Mi, rtol=1e-8, atol=1e-10)
+
+
+def test_alignment_ceiling_host_matches_eq9():
+    rng = np.random.default_rng(82)
+    d = 48
+    X = rng.standard_normal((3000, d)) @ rng.standard_normal((d, d))
+    W = rng.standard_normal((30, d))                       # rank-deficient Sigma_w is allowed
+    Sx = X.T @ X / X.shape[0]
+    a, s_mu, s_sq = cat.cat_alignment_ceiling_host(Sx, W.T @ W)
+    # P = Sx^1/2 Sw Sx^1/2 is 48 x 48 of rank 30: its 18 zero eigenvalues come out of the float64
+    # eigen-decomposition at ~1e-14 of the largest, whose square roots add ~1e-8 to sum sqrt(mu)
+    assert abs(a / O.max_alignment(Sx, W) - 1) < 1e-7
+    mu = np.clip(np.linalg.eigvalsh(W @ Sx @ W.T), 0, None)
+    assert abs(s_mu / mu.sum() - 1) < 1e-9 and abs(s_sq / np.sqrt(mu).sum() - 1) < 1e-7
+    with pytest.raises(cat.CatError):
+        cat.cat_alignment_ceiling_host(-np.eye(4), np.eye(4))
