@@ -302,6 +302,8 @@ class BufferSet:
         d_out = Wq.shape[0]
         self.x, self.xc, self.y_ref = x.clone(), xc.clone(), y_ref.clone()
         self.T, self.Wq, self.sw = T.clone(), Wq.clone(), sw.clone()
+        # T's bf16 planes, split once per layer (the tensor-core transform's k = 64, 128)
+        self.T_planes = cat.cat_split_transform(self.T, k) if (k in (64, 128) and x.dtype == torch.bfloat16) else None
         self.sigma = torch.empty((d_in // k, k, k), dtype=torch.float64, device=dev)
         self.xq = torch.empty((n, d_in // 2), dtype=torch.uint8, device=dev)
         self.sx = torch.empty((n,), dtype=torch.float32, device=dev)
@@ -310,7 +312,8 @@ class BufferSet:
 
     def nbytes(self):
         return sum(t.numel() * t.element_size() for t in (self.x, self.xc, self.y_ref, self.T, self.Wq, self.sw,
-                                                          self.sigma, self.xq, self.sx, self.y, self.out3))
+                                                          self.sigma, self.xq, self.sx, self.y, self.out3)) + \
+            (self.T_planes.numel() if self.T_planes is not None else 0)
 
 
 def diagnostics_from_sums(x3, w3, sum_y2, bits: int = 4):
@@ -492,7 +495,8 @@ def measure_config(cat, cfg, k, kind, args, dev, world, rank, with_e2e, sweep=Fa
 
     calls = {
         "cat_calib_cov": lambda b: cat.cat_calib_cov(b.xc, k, out=b.sigma),
-        "cat_transform_quantize_act": lambda b: cat.cat_transform_quantize_act(b.x, b.T, k, xq=b.xq, x_scale=b.sx),
+        "cat_transform_quantize_act": lambda b: cat.cat_transform_quantize_act_split(b.x, b.T, b.T_planes, k, xq=b.xq,
+                                                                                     x_scale=b.sx),
         # the integer GEMM, dequantization and SQNR sums (fused in the GEMM epilogue)
         "cat_w4a4_linear_sqnr": lambda b: cat.cat_w4a4_linear_sqnr(b.xq, b.sx, b.Wq, b.sw, b.y_ref, y=b.y, out=b.out3),
     }

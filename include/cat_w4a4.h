@@ -186,6 +186,25 @@ cat_status cat_transform_quantize_act(const void* x, cat_dtype dtype, int64_t n,
                                       cat_stream_t stream);
 
 /*
+ * cat_split_transform -- T_blocks [d_in/k][k][k] float32 into the three bf16 planes of every block,
+ * T_b = H + M + L with H = bf16(T_b), M = bf16(T_b - H), L = bf16(T_b - H - M) (24 significant bits:
+ * the tensor-core transform's fp32-accurate products), laid out exactly as that kernel's shared-memory
+ * operand (K-major, 128-byte swizzle).  planes: device, 6 * d_in * k bytes.  k = 64 or 128 (the
+ * tensor-core transform's block sizes; CAT_ERR_UNSUPPORTED otherwise).  Run once per layer after
+ * weight preparation; no counterpart in the paper (a layout of T).
+ */
+cat_status cat_split_transform(const float* T_blocks, int64_t d_in, int32_t k, uint8_t* planes, cat_stream_t stream);
+
+/*
+ * cat_transform_quantize_act_split -- cat_transform_quantize_act with T's pre-split planes
+ * (cat_split_transform; may be NULL): on the tensor-core path (bf16 rows, k = 64 or 128) each CTA
+ * fetches its block's planes with three bulk copies instead of splitting T_b itself.  Same results.
+ */
+cat_status cat_transform_quantize_act_split(const void* x, cat_dtype dtype, int64_t n, int64_t d_in, int32_t k,
+                                            const float* T_blocks, const uint8_t* T_planes, uint8_t* xq, float* x_scale,
+                                            cat_stream_t stream);
+
+/*
  * cat_w4a4_linear -- integer GEMM and dequantization (Sec. 3 Eq. 5: y ~ Q(W T^{-1}) Q(T x)).
  *   xq [n][d_in/2], x_scale [n]; Wq [d_out][d_in/2], w_scale [d_out]  (SM4x8 codes and steps).
  *   y        out, device [n][d_out] float32: y[t][o] = acc[t][o] * x_scale[t] * w_scale[o], with

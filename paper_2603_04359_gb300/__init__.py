@@ -23,6 +23,7 @@ __all__ = [
     "cat_dp_planes", "cat_transform_quantize_act_dp", "cat_quantize_weights_dp", "cat_linear_dp",
     "cat_block_transform", "cat_dequantize_codes", "cat_gemm_f32", "one_sided_sqnr", "cat_set_wait_limit_ns",
     "cat_transform_quantize_act_hd", "cat_fwht_rows", "cat_gram_f32", "cat_alignment_ceiling_host",
+    "cat_split_transform", "cat_transform_quantize_act_split",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -76,6 +77,8 @@ def load_library() -> ctypes.CDLL:
         "cat_dequantize_codes": ([P, P, I64, I64, P, P], I),
         "cat_gemm_f32": ([P, P, I64, I64, I64, P, P], I),
         "cat_transform_quantize_act_hd": ([P, I, I64, I64, I32, P, P, P, P], I),
+        "cat_split_transform": ([P, I64, I32, P, P], I),
+        "cat_transform_quantize_act_split": ([P, I, I64, I64, I32, P, P, P, P, P], I),
         "cat_fwht_rows": ([P, I64, I64, P], I),
         "cat_gram_f32": ([P, I, I64, I64, P, P], I),
         "cat_alignment_ceiling_host": ([P, P, I64, P], I),
@@ -256,6 +259,37 @@ def _linear_args(xq, x_scale, Wq, w_scale, y) -> None:
     _expect(Wq, "Wq", torch.uint8, (d_out, half), dev)
     _expect(w_scale, "w_scale", torch.float32, (d_out,), dev)
     _expect(y, "y", torch.float32, (n, d_out), dev)
+
+
+def cat_split_transform(T_blocks: torch.Tensor, k: int) -> torch.Tensor:
+    """T's three bf16 planes per block in the tensor-core transform's layout: uint8 [d_in * k * 6]."""
+    nb = T_blocks.shape[0]
+    d_in = nb * k
+    _expect(T_blocks, "T_blocks", torch.float32, (nb, k, k), T_blocks.device)
+    planes = torch.empty((6 * d_in * k,), dtype=torch.uint8, device=T_blocks.device)
+    _check("cat_split_transform", load_library().cat_split_transform(_ptr(T_blocks), d_in, k, _ptr(planes),
+                                                                     _stream(T_blocks.device)))
+    return planes
+
+
+def cat_transform_quantize_act_split(x: torch.Tensor, T_blocks: torch.Tensor, T_planes: Optional[torch.Tensor], k: int,
+                                     xq: Optional[torch.Tensor] = None,
+                                     x_scale: Optional[torch.Tensor] = None) -> Tuple[torch.Tensor, torch.Tensor]:
+    """cat_transform_quantize_act with T's pre-split planes (cat_split_transform)."""
+    _need(x, "x")
+    n, d_in = x.shape
+    if xq is None:
+        xq = torch.empty((n, d_in // 2), dtype=torch.uint8, device=x.device)
+    if x_scale is None:
+        x_scale = torch.empty((n,), dtype=torch.float32, device=x.device)
+    _expect(T_blocks, "T_blocks", torch.float32, (d_in // k, k, k), x.device)
+    if T_planes is not None:
+        _expect(T_planes, "T_planes", torch.uint8, (6 * d_in * k,), x.device)
+    _expect(xq, "xq", torch.uint8, (n, d_in // 2), x.device)
+    _expect(x_scale, "x_scale", torch.float32, (n,), x.device)
+    _check("cat_transform_quantize_act_split", load_library().cat_transform_quantize_act_split(
+        _ptr(x), _dtype(x), n, d_in, k, _ptr(T_blocks), _ptr(T_planes), _ptr(xq), _ptr(x_scale), _stream(x.device)))
+    return xq, x_scale
 
 
 def cat_w4a4_linear(xq: torch.Tensor, x_scale: torch.Tensor, Wq: torch.Tensor, w_scale: torch.Tensor,

@@ -173,28 +173,32 @@ cudaError_t launch_t(const Tin* x, int64_t n, int64_t d, int k, const float* A, 
 }  // namespace
 
 bool transform_quantize_tc_supported(int dtype, int k, int64_t n, int64_t d);
-cudaError_t launch_transform_quantize_tc(const void* x, int64_t n, int64_t d, int k, const float* A, uint32_t* amax,
-                                         uint32_t* words, float* scale, uint32_t* status, cudaStream_t stream);
+cudaError_t launch_transform_quantize_tc(const void* x, int64_t n, int64_t d, int k, const float* A,
+                                         const uint8_t* planes, uint32_t* amax, uint32_t* words, float* scale,
+                                         uint32_t* status, cudaStream_t stream);
 
 cudaError_t launch_transform_quantize_tc_fused(const void* x, int64_t n, int64_t d, int k, const float* A,
-                                               uint32_t* amax, uint32_t* words, uint32_t* status, cudaStream_t stream);
+                                               const uint8_t* planes, uint32_t* amax, uint32_t* words,
+                                               uint32_t* status, cudaStream_t stream);
 
+// planes (optional): T's pre-split bf16 planes (cat_split_transform), used by the tensor-core path.
 cudaError_t launch_transform_quantize(const void* x, int dtype, int64_t n, int64_t d, int k, const float* A,
-                                      uint8_t* codes, float* scale, uint32_t* status, cudaStream_t stream) {
+                                      uint8_t* codes, float* scale, uint32_t* status, cudaStream_t stream,
+                                      const uint8_t* planes) {
   if (n == 0) return cudaSuccess;
   if (transform_quantize_tc_supported(dtype, k, n, d)) {  // bf16 rows: tensor-core path
     uint32_t* amax = reinterpret_cast<uint32_t*>(scale);
-    const cudaError_t ef = launch_transform_quantize_tc_fused(x, n, d, k, A, amax, reinterpret_cast<uint32_t*>(codes),
-                                                              status, stream);
+    const cudaError_t ef = launch_transform_quantize_tc_fused(x, n, d, k, A, planes, amax,
+                                                              reinterpret_cast<uint32_t*>(codes), status, stream);
     if (ef != cudaErrorNotSupported) return ef;  // done (or failed) in one launch
     // two passes with the maxima in device scratch: pass 1 writes the steps
-    const cudaError_t es = launch_transform_quantize_tc(x, n, d, k, A, nullptr, reinterpret_cast<uint32_t*>(codes),
-                                                        scale, status, stream);
+    const cudaError_t es = launch_transform_quantize_tc(x, n, d, k, A, planes, nullptr,
+                                                        reinterpret_cast<uint32_t*>(codes), scale, status, stream);
     if (es != cudaErrorNotSupported) return es;
     // more rows than the scratch holds: the maxima in the scale buffer, then a finalize launch
     cudaError_t e = cudaMemsetAsync(scale, 0, (size_t)n * sizeof(float), stream);
-    if (e == cudaSuccess) e = launch_transform_quantize_tc(x, n, d, k, A, amax, reinterpret_cast<uint32_t*>(codes),
-                                                           nullptr, status, stream);
+    if (e == cudaSuccess) e = launch_transform_quantize_tc(x, n, d, k, A, planes, amax,
+                                                           reinterpret_cast<uint32_t*>(codes), nullptr, status, stream);
     if (e != cudaSuccess) return e;
     note_launch();
     finalize_scale_kernel<<<(unsigned)((n + 255) / 256), 256, 0, stream>>>(amax, n, status);

@@ -125,6 +125,27 @@ __device__ __forceinline__ void split_block(const float* __restrict__ Ab, uint8_
   }
 }
 
+// The three planes of T_b, pre-split by cat_split_transform into exactly the shared-memory image
+// split_block writes, fetched with one bulk copy per plane (counted on `bar`).
+template <int K>
+__device__ __forceinline__ void fetch_planes(const uint8_t* __restrict__ planes, int b, uint8_t* ts, uint64_t* bar) {
+  using C = TcCfg<K>;
+  mbar_arrive_expect_tx(bar, 3 * C::SPLIT);
+  const uint8_t* src = planes + (size_t)b * 3 * C::SPLIT;
+#pragma unroll
+  for (int sp = 0; sp < 3; ++sp)
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     smem_u32(ts + sp * C::SPLIT)),
+                 "l"(reinterpret_cast<uint64_t>(src + sp * C::SPLIT)), "r"(C::SPLIT), "r"(smem_u32(bar))
+                 : "memory");
+}
+
+// The three bf16 planes of every block, in the MMA's shared-memory layout (cat_split_transform).
+template <int K>
+__global__ void __launch_bounds__(kCvtWarps * 32) split_planes_kernel(const float* __restrict__ A, uint8_t* __restrict__ planes) {
+  split_block<K>(A + (size_t)blockIdx.x * K * K, planes + (size_t)blockIdx.x * 3 * TcCfg<K>::SPLIT, threadIdx.x);
+}
+
 // Four two's-complement bytes in [-7, 7] -> the SM4x8 sign-magnitude bytes (sign << 7 | magnitude).
 __device__ __forceinline__ uint32_t twos_to_sm(uint32_t w) {
   const uint32_t s = (w >> 7) & 0x01010101u;        // 1 in every negative byte
@@ -162,9 +183,9 @@ __device__ __forceinline__ uint32_t sm4_quant8(const uint32_t (&r)[32], int base
 
 template <int K, int PASS>
 __global__ void __launch_bounds__(kThreads, 1)
-    transform_quant_tc_kernel(const __grid_constant__ CUtensorMap tmX, const float* __restrict__ A, int n, int d,
-                              uint32_t* __restrict__ amax_bits, uint32_t* __restrict__ codes,
-                              float* __restrict__ scale, uint32_t* __restrict__ exit_ctr,
+    transform_quant_tc_kernel(const __grid_constant__ CUtensorMap tmX, const float* __restrict__ A,
+                              const uint8_t* __restrict__ planes, int n, int d, uint32_t* __restrict__ amax_bits,
+                              uint32_t* __restrict__ codes, float* __restrict__ scale, uint32_t* __restrict__ exit_ctr,
                               uint32_t* __restrict__ status) {
   // scale != nullptr (pass 1 with the maxima in a scratch slot): the CTAs holding block 0 write the
   // steps s = max / 7, and the last CTA out zeroes the slot's maxima and its exit counter
@@ -191,8 +212,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bars->d_full[s], 1);
       mbar_init(&bars->d_empty[s], 4);
     }
-    mbar_init(&bars->t_first, kCvtWarps);
-    mbar_init(&bars->t_full, kCvtWarps);
+    mbar_init(&bars->t_first, planes ? 1 : kCvtWarps);   // pre-split planes: one copying thread
+    mbar_init(&bars->t_full, planes ? 1 : kCvtWarps);
     mbar_init(&bars->t_empty, 1);
     mbar_init(&bars->mma_done, 1);
     bars->abort = 0;
@@ -277,12 +298,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (b == cur_b) continue;
       if (version > 0 && !(ok = mbar_wait_bounded(&bars->t_empty, (version - 1) & 1, abort_flag, __LINE__))) break;
       cur_b = b;
-      split_block<K>(A + (size_t)b * K * K, ts, ct);
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(&bars->t_full);
-        if (version == 0) mbar_arrive(&bars->t_first);
+      if (planes) {                                    // one thread copies the pre-split planes
+        if (ct == 0) {
+          fetch_planes<K>(planes, b, ts, &bars->t_full);
+          if (version == 0) mbar_arrive(&bars->t_first);
+        }
+      } else {
+        split_block<K>(A + (size_t)b * K * K, ts, ct);
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(&bars->t_full);
+          if (version == 0) mbar_arrive(&bars->t_first);
+        }
       }
       ++version;
     }
@@ -481,10 +509,10 @@ __device__ __forceinline__ void quantize_jobs(uint32_t tmem, int64_t u0, int64_t
 
 template <int K>
 __global__ void __launch_bounds__(kThreads, 1)
-    transform_quant_tc_fused_kernel(const __grid_constant__ CUtensorMap tmX, const float* __restrict__ A, int n,
-                                    int d, float* __restrict__ scale, uint32_t* __restrict__ codes,
-                                    uint32_t* __restrict__ sync, uint32_t* __restrict__ amax_bits,
-                                    uint32_t* __restrict__ status) {
+    transform_quant_tc_fused_kernel(const __grid_constant__ CUtensorMap tmX, const float* __restrict__ A,
+                                    const uint8_t* __restrict__ planes, int n, int d, float* __restrict__ scale,
+                                    uint32_t* __restrict__ codes, uint32_t* __restrict__ sync,
+                                    uint32_t* __restrict__ amax_bits, uint32_t* __restrict__ status) {
   using C = TcCfg<K>;
   constexpr int kMaxUnits = 512 / K;
   extern __shared__ uint8_t smem_raw[];
@@ -508,8 +536,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bars->x_empty[st], 1);
     }
     for (int j = 0; j < kMaxUnits; ++j) mbar_init(&unit_full[j], 1);
-    mbar_init(&bars->t_first, kCvtWarps);
-    mbar_init(&bars->t_full, kCvtWarps);
+    mbar_init(&bars->t_first, planes ? 1 : kCvtWarps);   // pre-split planes: one copying thread
+    mbar_init(&bars->t_full, planes ? 1 : kCvtWarps);
     mbar_init(&bars->t_empty, 1);
     mbar_init(&bars->mma_done, 1);
     bars->abort = 0;
@@ -594,12 +622,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (b == cur_b) continue;
       if (version > 0 && !(ok = mbar_wait_bounded(&bars->t_empty, (version - 1) & 1, abort_flag, __LINE__))) break;
       cur_b = b;
-      split_block<K>(A + (size_t)b * K * K, ts, ct);
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(&bars->t_full);
-        if (version == 0) mbar_arrive(&bars->t_first);
+      if (planes) {                                    // one thread copies the pre-split planes
+        if (ct == 0) {
+          fetch_planes<K>(planes, b, ts, &bars->t_full);
+          if (version == 0) mbar_arrive(&bars->t_first);
+        }
+      } else {
+        split_block<K>(A + (size_t)b * K * K, ts, ct);
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(&bars->t_full);
+          if (version == 0) mbar_arrive(&bars->t_first);
+        }
       }
       ++version;
     }
@@ -726,8 +761,8 @@ uint32_t next_tq_slot() {
 // the steps and returns the slot to zero (no memset, no finalize launch); cudaErrorNotSupported
 // otherwise, when the caller zeroes `amax` (its scale buffer) and finalizes the steps itself.
 template <int K>
-cudaError_t launch_k(const __nv_bfloat16* x, int64_t n, int64_t d, const float* A, uint32_t* amax, uint32_t* words,
-                     float* scale, uint32_t* status, cudaStream_t stream) {
+cudaError_t launch_k(const __nv_bfloat16* x, int64_t n, int64_t d, const float* A, const uint8_t* planes, uint32_t* amax,
+                     uint32_t* words, float* scale, uint32_t* status, cudaStream_t stream) {
   using C = TcCfg<K>;
   EncodeTiledFn fn = encode_fn();
   if (!fn) return cudaErrorNotSupported;
@@ -764,11 +799,11 @@ cudaError_t launch_k(const __nv_bfloat16* x, int64_t n, int64_t d, const float* 
     amax = amax_slots + (size_t)kAmaxRows * slot;
   }
   note_launch();
-  k0<<<grid, kThreads, C::SMEM, stream>>>(map, A, (int)n, (int)d, amax, words, nullptr, nullptr, status);
+  k0<<<grid, kThreads, C::SMEM, stream>>>(map, A, planes, (int)n, (int)d, amax, words, nullptr, nullptr, status);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   note_launch();
-  k1<<<grid, kThreads, C::SMEM, stream>>>(map, A, (int)n, (int)d, amax, words, scale, exit_ctr, status);
+  k1<<<grid, kThreads, C::SMEM, stream>>>(map, A, planes, (int)n, (int)d, amax, words, scale, exit_ctr, status);
   return cudaGetLastError();
 }
 
@@ -805,8 +840,8 @@ bool cooperative_ok() {
 }
 
 template <int K>
-cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, const float* A, uint32_t* amax,
-                           uint32_t* words, uint32_t* status, cudaStream_t stream) {
+cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, const float* A, const uint8_t* planes,
+                           uint32_t* amax, uint32_t* words, uint32_t* status, cudaStream_t stream) {
   using C = TcCfg<K>;
   const int nb = (int)(d / K);
   const int tiles = (int)((n + TM - 1) / TM);
@@ -859,7 +894,7 @@ cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, const f
   cfg.attrs = attrs;
   cfg.numAttrs = 1;
   note_launch();
-  return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<K>, map, A, (int)n, (int)d,
+  return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<K>, map, A, planes, (int)n, (int)d,
                             reinterpret_cast<float*>(amax), words, sync, amax_bits, status);
 }
 
@@ -870,12 +905,24 @@ bool transform_quantize_tc_supported(int dtype, int k, int64_t n, int64_t d) {
 }
 
 // Passes 0 and 1; the caller zeroes the scale buffer before and finalizes it after.
-cudaError_t launch_transform_quantize_tc(const void* x, int64_t n, int64_t d, int k, const float* A, uint32_t* amax,
-                                         uint32_t* words, float* scale, uint32_t* status, cudaStream_t stream) {
+cudaError_t launch_transform_quantize_tc(const void* x, int64_t n, int64_t d, int k, const float* A,
+                                         const uint8_t* planes, uint32_t* amax, uint32_t* words, float* scale,
+                                         uint32_t* status, cudaStream_t stream) {
   const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
-  if (k == 64) return launch_k<64>(xb, n, d, A, amax, words, scale, status, stream);
-  if (k == 128) return launch_k<128>(xb, n, d, A, amax, words, scale, status, stream);
+  if (k == 64) return launch_k<64>(xb, n, d, A, planes, amax, words, scale, status, stream);
+  if (k == 128) return launch_k<128>(xb, n, d, A, planes, amax, words, scale, status, stream);
   return cudaErrorInvalidValue;
+}
+
+// T_blocks -> the three bf16 planes of every block in the transform kernels' shared-memory layout
+// ([d/k][3][k*k] bf16, 6 d k bytes); k = 64 or 128.
+cudaError_t launch_split_transform(const float* A, int64_t d, int k, uint8_t* planes, cudaStream_t stream) {
+  const unsigned nb = (unsigned)(d / k);
+  note_launch();
+  if (k == 64) split_planes_kernel<64><<<nb, kCvtWarps * 32, 0, stream>>>(A, planes);
+  else if (k == 128) split_planes_kernel<128><<<nb, kCvtWarps * 32, 0, stream>>>(A, planes);
+  else return cudaErrorNotSupported;
+  return cudaGetLastError();
 }
 
 }  // namespace cat
@@ -885,10 +932,11 @@ namespace cat {
 // (the row maxima go to a slot of device scratch that the launch leaves zeroed); cudaErrorNotSupported
 // otherwise (the caller takes the two-pass path).
 cudaError_t launch_transform_quantize_tc_fused(const void* x, int64_t n, int64_t d, int k, const float* A,
-                                               uint32_t* amax, uint32_t* words, uint32_t* status, cudaStream_t stream) {
+                                               const uint8_t* planes, uint32_t* amax, uint32_t* words,
+                                               uint32_t* status, cudaStream_t stream) {
   const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
-  if (k == 64) return launch_fused_k<64>(xb, n, d, A, amax, words, status, stream);
-  if (k == 128) return launch_fused_k<128>(xb, n, d, A, amax, words, status, stream);
+  if (k == 64) return launch_fused_k<64>(xb, n, d, A, planes, amax, words, status, stream);
+  if (k == 128) return launch_fused_k<128>(xb, n, d, A, planes, amax, words, status, stream);
   return cudaErrorNotSupported;
 }
 }  // namespace cat

@@ -551,6 +551,42 @@ cat_status cat_transform_quantize_act(const void* x, cat_dtype dtype, int64_t n,
   return ok();
 }
 
+cat_status cat_split_transform(const float* T_blocks, int64_t d_in, int32_t k, uint8_t* planes, cat_stream_t stream) {
+  cat_status st = check_din(d_in);
+  if (st != CAT_OK) return st;
+  if (!valid_k(k) || d_in % k != 0) return fail(CAT_ERR_SHAPE, "k must be one of 16..256 (power of two) and divide d_in");
+  if (k != 64 && k != 128) return fail(CAT_ERR_UNSUPPORTED, "pre-split planes serve the tensor-core transform: k = 64 or 128");
+  if (!T_blocks || !planes) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(T_blocks) || !aligned16(planes)) return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  if ((st = check_device()) != CAT_OK) return st;
+  cudaError_t e = cat::launch_split_transform(T_blocks, d_in, k, planes, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cat_split_transform launch");
+  return ok();
+}
+
+cat_status cat_transform_quantize_act_split(const void* x, cat_dtype dtype, int64_t n, int64_t d_in, int32_t k,
+                                            const float* T_blocks, const uint8_t* T_planes, uint8_t* xq, float* x_scale,
+                                            cat_stream_t stream) {
+  if (dtype != CAT_F32 && dtype != CAT_BF16) return fail(CAT_ERR_INVALID_ARG, "unknown dtype");
+  if (n < 0) return fail(CAT_ERR_SHAPE, "n must be >= 0");
+  cat_status st = check_din(d_in);
+  if (st != CAT_OK) return st;
+  if (!valid_k(k) || d_in % k != 0) return fail(CAT_ERR_SHAPE, "k must be one of 16..256 (power of two) and divide d_in");
+  if (n == 0) return ok();
+  if (!x || !T_blocks || !xq || !x_scale) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(x) || !aligned16(T_blocks) || !aligned16(xq) || !aligned16(x_scale) || (T_planes && !aligned16(T_planes)))
+    return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  if ((n + 63) / 64 > 0x7FFFFFFF) return fail(CAT_ERR_SHAPE, "n too large");
+  if ((st = check_device()) != CAT_OK) return st;
+  cudaError_t e;
+  uint32_t* status = status_word(&e);
+  if (!status) return cuda_fail(e, "status word");
+  e = cat::launch_transform_quantize(x, (int)dtype, n, d_in, k, T_blocks, xq, x_scale, status, (cudaStream_t)stream,
+                                     (k == 64 || k == 128) ? T_planes : nullptr);
+  if (e != cudaSuccess) return cuda_fail(e, "cat_transform_quantize_act_split launch");
+  return ok();
+}
+
 cat_status cat_w4a4_linear(const uint8_t* xq, const float* x_scale, const uint8_t* Wq, const float* w_scale,
                            int64_t n, int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, cat_stream_t stream) {
   if (n < 0 || d_out <= 0) return fail(CAT_ERR_SHAPE, "n must be >= 0 and d_out >= 1");

@@ -110,6 +110,22 @@ def test_transform_quantize_act(n, d, k, dtype):
     assert cat.cat_device_status()[0] == 0
 
 
+@pytest.mark.parametrize("n,d,k,dtype", [(67, 384, 128, "bf16"), (300, 1024, 64, "bf16"), (1000, 256, 128, "bf16"),
+                                         (2560, 4096, 128, "bf16"), (1300, 8192, 64, "bf16"), (130, 256, 32, "f32")])
+def test_transform_with_presplit_planes_is_identical(n, d, k, dtype):
+    """T's bf16 planes split once (cat_split_transform) and bulk-copied by the kernels give the same
+    codes and steps, bit for bit, as the kernels' own split (fused, two-pass, and the SIMT path that
+    ignores the planes)."""
+    rng = np.random.default_rng(5 * n + d)
+    X = WL.cast(rng.standard_normal((n, d)) * rng.lognormal(0, 1.0, d), dtype)
+    T32 = torch.from_numpy(_cat_T(rng, d, k)).to(DEV)
+    planes = cat.cat_split_transform(T32, k) if k in (64, 128) else None
+    xq0, sx0 = cat.cat_transform_quantize_act(to_dev(X), T32, k)
+    xq1, sx1 = cat.cat_transform_quantize_act_split(to_dev(X), T32, planes, k)
+    assert torch.equal(xq0, xq1) and torch.equal(sx0, sx1)
+    assert cat.cat_device_status()[0] == 0
+
+
 def test_nonfinite_activation_reports_numeric():
     d, k = 128, 32
     X = np.ones((70, d), dtype=np.float32)
