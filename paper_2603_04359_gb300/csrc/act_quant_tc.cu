@@ -38,6 +38,15 @@ struct TcCfg {
   static constexpr uint32_t T_OFF = kXStages * X_STAGE;
   static constexpr uint32_t BAR_OFF = T_OFF + 3 * SPLIT;
   static constexpr size_t SMEM = BAR_OFF + 256 + 1024;
+  // fused kernel: the final row maxima of unit j (128 floats).  At k = 128 a CTA has at most
+  // kXStages units, so unit j's x stage is free once its MMAs are done and holds them; at k = 64
+  // they get their own room after the barriers.
+  static constexpr uint32_t FUSED_BAR_BYTES = 512;
+  static constexpr uint32_t AMAX_DEDICATED = BAR_OFF + FUSED_BAR_BYTES;
+  static constexpr size_t FUSED_SMEM = BAR_OFF + FUSED_BAR_BYTES + (K == 128 ? 0 : (512 / K) * TM * 4) + 1024;
+  __device__ static uint8_t* amax_tile(uint8_t* smem, int j) {
+    return K == 128 ? smem + X_OFF + j * X_STAGE : smem + AMAX_DEDICATED + j * TM * 4;
+  }
   static constexpr uint32_t TMEM_COLS = 2 * K;               // double-buffered accumulator
   // kind::f16: D fp32 (bit 4), A = B = BF16 (format 1 at bits 7 and 10), K-major, M = 128, N = K
   static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(K >> 3) << 17) |
@@ -50,8 +59,8 @@ struct TcBars {
   uint32_t tmem_addr;
   int abort;
 };
-// the barrier block and the fused kernel's per-unit barriers (<= 8) fit the 256 bytes reserved for them
-static_assert(sizeof(TcBars) + 8 * sizeof(uint64_t) <= 256, "barrier room");
+// the barrier block fits the 256 bytes reserved for it (the fused kernel reserves FUSED_BAR_BYTES)
+static_assert(sizeof(TcBars) <= 256, "barrier room");
 
 __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
                                          uint32_t accumulate) {
@@ -77,6 +86,50 @@ __host__ __device__ inline void unit_range(int c, int grid, int nb, int tiles, i
     const int64_t units = (int64_t)nb * tiles;
     *u0 = units * c / grid;
     *u1 = units * (c + 1) / grid;
+  }
+}
+
+// The fused kernel's units of CTA c.  With at least as many CTAs as blocks, the m CTAs of block b
+// take its row tiles round robin (the i-th of them: tiles i, i + m, i + 2m, ...), so that tile t sits
+// at position t / m in its CTA in every block, and the tiles' row maxima become final in ascending
+// tile order across the grid; otherwise contiguous block-major ranges as unit_range.
+struct FusedUnits {
+  int64_t u0;        // contiguous ranges: the first unit (block-major index)
+  int b, first, step;
+  int count;         // units of the CTA
+  bool round_robin;
+};
+__host__ __device__ inline FusedUnits fused_units(int c, int grid, int nb, int tiles) {
+  FusedUnits f;
+  f.u0 = 0;
+  f.b = 0;
+  f.first = 0;
+  f.step = 1;
+  f.round_robin = grid >= nb;
+  if (f.round_robin) {
+    const int b = (int)((int64_t)c * nb / grid);
+    const int c_lo = (int)(((int64_t)b * grid + nb - 1) / nb);
+    const int c_hi = (int)(((int64_t)(b + 1) * grid + nb - 1) / nb);
+    const int m = c_hi - c_lo, i = c - c_lo;
+    f.b = b;
+    f.first = i;
+    f.step = m;
+    f.count = i < tiles ? (tiles - i + m - 1) / m : 0;
+  } else {
+    int64_t u1;
+    unit_range(c, grid, nb, tiles, &f.u0, &u1);
+    f.count = (int)(u1 - f.u0);
+  }
+  return f;
+}
+__host__ __device__ inline void fused_unit(const FusedUnits& f, int j, int tiles, int* b, int* tile) {
+  if (f.round_robin) {
+    *b = f.b;
+    *tile = f.first + j * f.step;
+  } else {
+    const int64_t u = f.u0 + j;
+    *b = (int)(u / tiles);
+    *tile = (int)(u % tiles);
   }
 }
 
@@ -127,17 +180,19 @@ __device__ __forceinline__ void split_block(const float* __restrict__ Ab, uint8_
 
 // The three planes of T_b, pre-split by cat_split_transform into exactly the shared-memory image
 // split_block writes, fetched with one bulk copy per plane (counted on `bar`).
+__device__ __forceinline__ void bulk_copy_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_u32(dst)),
+               "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
+}
 template <int K>
 __device__ __forceinline__ void fetch_planes(const uint8_t* __restrict__ planes, int b, uint8_t* ts, uint64_t* bar) {
   using C = TcCfg<K>;
   mbar_arrive_expect_tx(bar, 3 * C::SPLIT);
   const uint8_t* src = planes + (size_t)b * 3 * C::SPLIT;
 #pragma unroll
-  for (int sp = 0; sp < 3; ++sp)
-    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                     smem_u32(ts + sp * C::SPLIT)),
-                 "l"(reinterpret_cast<uint64_t>(src + sp * C::SPLIT)), "r"(C::SPLIT), "r"(smem_u32(bar))
-                 : "memory");
+  for (int sp = 0; sp < 3; ++sp) bulk_copy_g2s(ts + sp * C::SPLIT, src + sp * C::SPLIT, C::SPLIT, bar);
 }
 
 // The three bf16 planes of every block, in the MMA's shared-memory layout (cat_split_transform).
@@ -153,32 +208,55 @@ __device__ __forceinline__ uint32_t twos_to_sm(uint32_t w) {
   return ((w ^ m) + s) | (s << 7);                   // |q| (no carry leaves a byte) and the sign bit
 }
 
-// One SM4x8 word of the codes of v_e = r[base + e] (as float), e = 0..7, on the row described by qr
-// (|v_e| <= max|v|).  Fast route: adding 1.5 * 2^23 to p = fl(v_e * inv) rounds it to an integer
+// The four SM4x8 words of the codes of the 32 values v_e = r[e] (as float) on the row described by
+// qr (|v_e| <= max|v|).  Fast route: adding 1.5 * 2^23 to p = fl(v_e * inv) rounds it to an integer
 // (half to even) that sits, two's complement, in the low byte of the sum's bits; the bytes are
-// gathered four to a word and turned into sign-magnitude.  If any p lies within 2^-18 of a
-// half-integer (an exact tie included), or the row is rescaled, the eight codes are decided
-// exactly instead (qcode_exact).  Callers pass qr.inv == 0 only for rows whose codes are all 0.
-__device__ __forceinline__ uint32_t sm4_quant8(const uint32_t (&r)[32], int base, const QRow& qr) {
+// gathered four to a word and turned into sign-magnitude.  One near-tie test covers the chunk (one
+// branch, so the 32 products overlap): if any p lies within 2^-18 of a half-integer (an exact tie
+// included), or the row is rescaled, the 32 codes are decided exactly instead (qcode_exact).
+// qr.inv == 0 (an all-zero or non-finite row): all codes 0.
+__device__ __forceinline__ uint4 sm4_quant32(const uint32_t (&r)[32], const QRow& qr) {
   constexpr float kMagic = 12582912.0f;
-  uint32_t b[8];
+  if (qr.inv == 0.f) return make_uint4(0u, 0u, 0u, 0u);
+  uint32_t b[32];
   bool near = qr.exact;
 #pragma unroll
-  for (int e = 0; e < 8; ++e) {
-    const float p = __fmul_rn(__uint_as_float(r[base + e]), qr.inv);
+  for (int e = 0; e < 32; ++e) {
+    const float p = __fmul_rn(__uint_as_float(r[e]), qr.inv);
     const float rb = __fadd_rn(p, kMagic);
     near |= fabsf(__fsub_rn(__fsub_rn(rb, kMagic), p)) > kNearTie;
     b[e] = __float_as_uint(rb);
   }
+  uint32_t w[4];
   if (near) {
-    int q[8];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) q[e] = qcode_exact(__uint_as_float(r[base + e]), qr, 7.0f);
-    return sm4_pack(q);
+    for (int g = 0; g < 4; ++g) {
+      int q[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) q[e] = qcode_exact(__uint_as_float(r[8 * g + e]), qr, 7.0f);
+      w[g] = sm4_pack(q);
+    }
+  } else {
+#pragma unroll
+    for (int g = 0; g < 4; ++g) {
+      const uint32_t* bg = b + 8 * g;
+      const uint32_t lo =
+          twos_to_sm(__byte_perm(__byte_perm(bg[0], bg[1], 0x0040), __byte_perm(bg[2], bg[3], 0x0040), 0x5410));
+      const uint32_t hi =
+          twos_to_sm(__byte_perm(__byte_perm(bg[4], bg[5], 0x0040), __byte_perm(bg[6], bg[7], 0x0040), 0x5410));
+      w[g] = lo | __funnelshift_l(hi, hi, 4);
+    }
   }
-  const uint32_t lo = twos_to_sm(__byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410));
-  const uint32_t hi = twos_to_sm(__byte_perm(__byte_perm(b[4], b[5], 0x0040), __byte_perm(b[6], b[7], 0x0040), 0x5410));
-  return lo | __funnelshift_l(hi, hi, 4);
+  return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+// Running maximum of |v| over 32 values, on their bit patterns: for non-negative floats the bit
+// order is the value order, and every NaN pattern lies above the infinity 0x7F800000, so the result
+// is below 0x7F800000 exactly when all 32 values are finite.
+__device__ __forceinline__ uint32_t absmax_bits32(const uint32_t (&r)[32], uint32_t m) {
+#pragma unroll
+  for (int e = 0; e < 32; ++e) m = max(m, r[e] & 0x7FFFFFFFu);
+  return m;
 }
 
 template <int K, int PASS>
@@ -363,11 +441,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         } else if (t < n) {
           // the row's codes with the final maximum (|v * inv| <= 7 for a finite row; inv = 0 gives
           // 0 codes for an all-zero or non-finite row)
-          uint32_t w[4];
-#pragma unroll
-          for (int g = 0; g < 4; ++g) w[g] = qr.inv == 0.f ? 0u : sm4_quant8(r, 8 * g, qr);
           *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * K + c * 32) / 8) =
-              make_uint4(w[0], w[1], w[2], w[3]);
+              sm4_quant32(r, qr);
         }
       }
       tc_fence_before();
@@ -407,102 +482,112 @@ __global__ void __launch_bounds__(kThreads, 1)
 // ---- single-launch variant: x' stays in tensor memory between the two row-wide phases ---------
 //
 // When every CTA's units fit in tensor memory at once (units per CTA x K <= 512 columns), one
-// cooperative launch does both passes: phase A runs the MMAs once, keeps each unit's x' tile in its
-// own TMEM columns and records the row maxima in the launch's scratch slot; a grid-wide barrier;
-// phase B reads the final maxima, quantizes the tiles still in TMEM and writes the codes, and the
-// CTAs holding block 0 write the steps s = max / 7.  The last CTA to leave zeroes the slot (maxima
-// and counters) for the next launch.  Every wait is bounded.
-// Per-launch state of the fused kernel, one slot per launch in flight (slots are handed out round
-// robin, so up to kSyncSlots launches may run at once on different streams): the grid-barrier and
-// exit counters, and the row maxima (float bits).  The last CTA to leave a launch returns its slot to
-// zero, so a launch, a graph replay of it included, always starts from a clean slot.
+// cooperative launch does both passes.  Phase A runs the MMAs once, keeps each unit's x' tile in its
+// own TMEM columns and publishes the tile's row maxima (atomicMax into the launch's scratch slot,
+// then one count per epilogue warp on the tile's record).  Phase B needs a row's maximum over all
+// blocks, i.e. all nb units of a row tile, but not the rest of the grid: a watcher warp per CTA waits
+// for each of its tiles' counts in turn, copies the final maxima to shared memory and releases the
+// quantizer warps for that unit, while later units are still in phase A.  The CTAs holding block 0
+// write the steps s = max / 7; the last CTA to read a tile's maxima returns them and the tile's
+// record to zero, so a launch, a graph replay of it included, always starts from a clean slot.
+// Every wait is bounded; a launch that gave up somewhere has its whole slot zeroed by the last CTA
+// to leave.  Slots are handed out round robin, so up to kSyncSlots launches may run at once on
+// different streams.
 constexpr int kSyncSlots = 8;
-constexpr int kAmaxRows = 1 << 17;             // rows the fused path can have (<= 608 units of 128 rows)
+constexpr int kAmaxRows = 1 << 17;             // rows the fused path can have (<= 1024 tiles of 128 rows)
+constexpr int kAmaxTiles = kAmaxRows / TM;
+constexpr int kTileWords = 32;                 // per tile: [0] maxima published (counts), [16] maxima read
 __device__ __align__(16) uint32_t g_tq_sync[kSyncSlots][4];
 __device__ uint32_t g_tq_amax[kSyncSlots][kAmaxRows];
+__device__ __align__(128) uint32_t g_tq_tiles[kSyncSlots][kAmaxTiles * kTileWords];
 
 __device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
   uint32_t v;
   asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
   return v;
 }
-__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 2, 128;" ::: "memory"); }
 
-// All CTAs' epilogue warps meet here (the other warps of a CTA never wait on it).  Bounded: a
-// barrier that has not filled in kWaitLimitNs raises the abort flag.
-__device__ __forceinline__ void grid_barrier(uint32_t* ctr, uint32_t expected, volatile int* abort_flag, bool leader) {
-  __threadfence();
-  epi_bar();
-  if (leader) {
-    atomicAdd(ctr, 1u);
-    const uint64_t t0 = globaltimer_ns();
-    for (uint32_t it = 0; ld_acquire_gpu(ctr) < expected; ++it) {
-      __nanosleep(64);                                  // keep the polls off the counter's L2 slice
-      if ((it & 63u) == 63u && (*abort_flag || globaltimer_ns() - t0 > kWaitLimitNs)) {
-        if (*abort_flag == 0) *abort_flag = __LINE__;
-        break;
-      }
+// Bounded poll of a counter in global memory until it reaches `expected` (one thread).
+__device__ __forceinline__ bool wait_count(const uint32_t* ctr, uint32_t expected, volatile int* abort_flag, int site) {
+  if (ld_acquire_gpu(ctr) >= expected) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t it = 1;; ++it) {
+    __nanosleep(32);
+    if (ld_acquire_gpu(ctr) >= expected) return true;
+    if ((it & 63u) == 0u && (*abort_flag || globaltimer_ns() - t0 > kWaitLimitNs)) {
+      if (*abort_flag == 0) *abort_flag = site;
+      return false;
     }
-    __threadfence();
   }
-  epi_bar();
 }
 
+// Phase B of one quantizer warp (slot 0: the quadrant's epilogue warp, 1 and 2: its converter
+// warps).  Units are taken in order, each once the watcher has put its final row maxima in shared
+// memory; a unit's 32-column chunk c goes to slot 1 + (c & 1) except in the CTA's last unit, which the
+// three warps share (slot (c + 1) % 3): the epilogue warp joins when its phase A is done.
+__device__ __forceinline__ int chunk_slot(int c, bool last) { return last ? (c + 1) % 3 : 1 + (c & 1); }
 
-// Named barrier of the 12 warps that quantize (4 epilogue + 8 converter warps).
-__device__ __forceinline__ void quant_bar() { asm volatile("bar.sync 3, 384;" ::: "memory"); }
-
-// Phase B jobs of one warp: job = (unit j, 32-column chunk c), taken round-robin by the three warps
-// of a TMEM lane quadrant (slot 0: the epilogue warp, 1 and 2: converter warps).
 template <int K>
-__device__ __forceinline__ void quantize_jobs(uint32_t tmem, int64_t u0, int64_t u1, int num_tiles, int n, int d,
-                                              const uint32_t* __restrict__ amax_bits, uint32_t* __restrict__ codes,
-                                              volatile int* abort_flag, int slot) {
-  // amax_bits: the launch's row maxima (float bits) in its scratch slot
-  if (__any_sync(0xFFFFFFFFu, *abort_flag)) return;
-  constexpr int kMaxUnits = 512 / K;
+__device__ __forceinline__ void quantize_units(uint32_t tmem, uint8_t* smem, const FusedUnits& fu, int num_tiles,
+                                               int n, int d, uint64_t* maxima_ready, uint32_t* __restrict__ codes,
+                                               volatile int* abort_flag, int slot) {
+  using C = TcCfg<K>;
   const int lane = threadIdx.x & 31, quad = (threadIdx.x >> 5) & 3;
   const int64_t words_per_row = d / 8;
-  const int nu = (int)(u1 - u0);
-  const int jobs = nu * (K / 32);
-  // this lane's row maxima of every unit, all loads in flight at once
-  float a_u[kMaxUnits], inv_u[kMaxUnits];
+  const int nu = fu.count;
+  for (int j = 0; j < nu; ++j) {
+    const bool last = j == nu - 1;
+    bool mine = false;
 #pragma unroll
-  for (int j = 0; j < kMaxUnits; ++j) {
-    const int t = (int)((u0 + j) % num_tiles) * TM + quad * 32 + lane;
-    a_u[j] = (j < nu && t < n) ? __uint_as_float(__ldcg(&amax_bits[t])) : 0.f;
-  }
-#pragma unroll
-  for (int j = 0; j < kMaxUnits; ++j) inv_u[j] = qrow_setup(a_u[j], 7.0f).inv;
-  tc_fence_after();
-  for (int job = slot; job < jobs; job += 3) {
-    const int j = job / (K / 32), c = job % (K / 32);
-    const int64_t u = u0 + j;
-    const int b = (int)(u / num_tiles), tile = (int)(u % num_tiles);
+    for (int c = 0; c < K / 32; ++c) mine |= chunk_slot(c, last) == slot;
+    if (!mine) continue;
+    const bool got = !*abort_flag && mbar_wait_bounded(&maxima_ready[j], 0, abort_flag, __LINE__);
+    if (!__all_sync(0xFFFFFFFFu, got)) return;
+    int b, tile;
+    fused_unit(fu, j, num_tiles, &b, &tile);
     const int t = tile * TM + quad * 32 + lane;
-    float inv = inv_u[0], a = a_u[0];
-#pragma unroll
-    for (int q = 1; q < kMaxUnits; ++q)
-      if (j == q) {
-        inv = inv_u[q];
-        a = a_u[q];
-      }
-    QRow qr;
-    qr.inv = inv;
-    qr.a = a;
-    qr.sc = 1.f;
-    qr.exact = false;
-    if (inv != 0.f && (a > 0x1p100f || a < 0x1p-60f)) qr = qrow_setup(a, 7.0f);  // rescaled row
-    uint32_t r[32];
-    __syncwarp();
-    CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + j * K + c * 32, r);
-    tmem_ld_wait();
-    if (t < n) {
-      uint32_t w[4];
-#pragma unroll
-      for (int g = 0; g < 4; ++g) w[g] = inv == 0.f ? 0u : sm4_quant8(r, 8 * g, qr);  // 0: zero or non-finite row
-      *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * K + c * 32) / 8) =
-          make_uint4(w[0], w[1], w[2], w[3]);
+    const float a = reinterpret_cast<const float*>(C::amax_tile(smem, j))[quad * 32 + lane];
+    const QRow qr = qrow_setup(a, 7.0f);       // inv == 0: zero or non-finite row, all codes 0
+    tc_fence_after();
+#pragma unroll 1
+    for (int c = 0; c < K / 32; ++c) {
+      if (chunk_slot(c, last) != slot) continue;
+      uint32_t r[32];
+      __syncwarp();
+      CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + j * K + c * 32, r);
+      tmem_ld_wait();
+      if (t < n)
+        *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * K + c * 32) / 8) =
+            sm4_quant32(r, qr);
+    }
+  }
+}
+
+// Counts the CTA out of the launch's slot; called by every thread of a group of NT threads (the
+// watcher warp, NT = 32, or the whole CTA), id = 0 .. NT - 1.  The last CTA out resets the exit
+// counter and, if some CTA gave up (a tile's maxima and record may then be left behind), first zeroes
+// the slot's maxima and tile records.
+template <int NT>
+__device__ __forceinline__ void exit_slot(uint32_t* sync, uint32_t* amax_bits, uint32_t* tile_rec, int num_tiles, int id,
+                                          bool gave_up, volatile int* last_out) {
+  if (id == 0) {
+    __threadfence();
+    if (gave_up) atomicOr(&sync[2], 1u);
+    __threadfence();
+    *last_out = atomicAdd(&sync[1], 1u) == gridDim.x - 1;
+  }
+  if (NT == 32) __syncwarp(); else __syncthreads();
+  if (*last_out) {
+    __threadfence();
+    if (ld_acquire_gpu(&sync[2]) != 0u) {
+      for (int t = id; t < num_tiles * TM; t += NT) amax_bits[t] = 0u;
+      for (int i = id; i < num_tiles * kTileWords; i += NT) tile_rec[i] = 0u;
+    }
+    __threadfence();
+    if (NT == 32) __syncwarp(); else __syncthreads();
+    if (id == 0) {
+      sync[2] = 0u;
+      sync[1] = 0u;
     }
   }
 }
@@ -512,35 +597,54 @@ __global__ void __launch_bounds__(kThreads, 1)
     transform_quant_tc_fused_kernel(const __grid_constant__ CUtensorMap tmX, const float* __restrict__ A,
                                     const uint8_t* __restrict__ planes, int n, int d, float* __restrict__ scale,
                                     uint32_t* __restrict__ codes, uint32_t* __restrict__ sync,
-                                    uint32_t* __restrict__ amax_bits, uint32_t* __restrict__ status) {
+                                    uint32_t* __restrict__ amax_bits, uint32_t* __restrict__ tile_rec,
+                                    uint32_t* __restrict__ status) {
+  // sync: [1] exit counter, [2] set by a CTA that gave up; amax_bits: the row maxima (float bits);
+  // tile_rec: kTileWords words per row tile (maxima published, maxima read)
   using C = TcCfg<K>;
   constexpr int kMaxUnits = 512 / K;
+  static_assert(sizeof(TcBars) + (3 * kMaxUnits + 3) * sizeof(uint64_t) + 16 <= C::FUSED_BAR_BYTES, "barrier room");
+  static_assert(K != 128 || kMaxUnits <= kXStages, "at k = 128 unit j's x stage holds its maxima");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* xs = smem + C::X_OFF;
   uint8_t* ts = smem + C::T_OFF;
   TcBars* bars = reinterpret_cast<TcBars*>(smem + C::BAR_OFF);
-  uint64_t* unit_full = reinterpret_cast<uint64_t*>(bars + 1);   // one per unit (each used once)
+  uint64_t* unit_full = reinterpret_cast<uint64_t*>(bars + 1);   // per unit, used once: its MMAs are done
+  uint64_t* epi_done = unit_full + kMaxUnits;                     // per unit, used once: its atomics are issued
+  uint64_t* maxima_ready = epi_done + kMaxUnits;                  // per unit, used once: final maxima in smem
+  uint64_t* plane_full = maxima_ready + kMaxUnits;                // per plane of T_b (producer-fetched planes)
+  volatile int* exit_counted = reinterpret_cast<int*>(plane_full + 3);  // [0] the watcher counted the CTA out,
+                                                                         // [1] the CTA was the last out
   volatile int* abort_flag = &bars->abort;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int nb = d / K;
   const int num_tiles = (n + TM - 1) / TM;
-  int64_t u0, u1;
-  unit_range(blockIdx.x, gridDim.x, nb, num_tiles, &u0, &u1);
-  if (u1 - u0 > kMaxUnits) u1 = u0 + kMaxUnits;          // the launcher guarantees this never cuts
+  FusedUnits fu = fused_units(blockIdx.x, gridDim.x, nb, num_tiles);
+  if (fu.count > kMaxUnits) fu.count = kMaxUnits;      // the launcher guarantees this never cuts
+  const int nu = fu.count;
+  // With pre-split planes and one block per CTA, the producer fetches the planes itself, in the order
+  // H, (unit 0's x tile), M, L, and unit 0's MMAs start on H while M and L are still on their way.
+  const bool own_planes = planes != nullptr && fu.round_robin;
 
   if (tid == 0) {
     for (int st = 0; st < kXStages; ++st) {
       mbar_init(&bars->x_full[st], 1);
       mbar_init(&bars->x_empty[st], 1);
     }
-    for (int j = 0; j < kMaxUnits; ++j) mbar_init(&unit_full[j], 1);
+    for (int j = 0; j < kMaxUnits; ++j) {
+      mbar_init(&unit_full[j], 1);
+      mbar_init(&epi_done[j], 4);                       // the four epilogue warps
+      mbar_init(&maxima_ready[j], 1);
+    }
+    for (int sp = 0; sp < 3; ++sp) mbar_init(&plane_full[sp], 1);
     mbar_init(&bars->t_first, planes ? 1 : kCvtWarps);   // pre-split planes: one copying thread
     mbar_init(&bars->t_full, planes ? 1 : kCvtWarps);
     mbar_init(&bars->t_empty, 1);
     mbar_init(&bars->mma_done, 1);
     bars->abort = 0;
+    *exit_counted = 0;
     fence_mbar_init();
   }
   __syncwarp();
@@ -556,34 +660,56 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       prefetch_tensormap(&tmX);
       bool ok = true;
-      uint32_t j = 0;
-      for (int64_t u = u0; u < u1 && ok; ++u, ++j) {
-        const int b = (int)(u / num_tiles), tile = (int)(u % num_tiles);
+      int j = 0;
+      const uint8_t* src = own_planes ? planes + (size_t)fu.b * 3 * C::SPLIT : nullptr;
+      if (own_planes) {
+        mbar_arrive_expect_tx(&plane_full[0], C::SPLIT);
+        bulk_copy_g2s(ts, src, C::SPLIT, &plane_full[0]);
+      }
+      for (; j < nu; ++j) {
+        int b, tile;
+        fused_unit(fu, j, num_tiles, &b, &tile);
         const uint32_t st = j % kXStages;
-        // the first two units' x tiles go out with T_b's loads; the others wait until T_b is split,
-        // so that T_b does not queue behind them in HBM and unit 0's MMAs start as early as they can
-        if (j == 2 && !(ok = mbar_wait_bounded(&bars->t_first, 0, abort_flag, __LINE__))) break;
+        if (own_planes) {
+          // M and L after unit 0's tile; the tiles from unit 2 on after all of T_b is in
+          if (j == 2 && !(ok = mbar_wait_bounded(&plane_full[2], 0, abort_flag, __LINE__))) break;
+        } else {
+          // the first two units' x tiles go out with T_b's loads; the others wait until T_b is in shared
+          // memory, so that T_b does not queue behind them and unit 0's MMAs start as early as they can
+          if (j == 2 && !(ok = mbar_wait_bounded(&bars->t_first, 0, abort_flag, __LINE__))) break;
+        }
         if (j >= kXStages && !(ok = mbar_wait_bounded(&bars->x_empty[st], ((j / kXStages) - 1) & 1, abort_flag, __LINE__))) break;
         mbar_arrive_expect_tx(&bars->x_full[st], C::X_STAGE);
 #pragma unroll
         for (int a = 0; a < C::ATOMS; ++a)
           tma_load_2d(xs + st * C::X_STAGE + a * (TM * 128), &tmX, b * K + 64 * a, tile * TM, &bars->x_full[st]);
+        if (own_planes && j == 0) {
+#pragma unroll
+          for (int sp = 1; sp < 3; ++sp) {
+            mbar_arrive_expect_tx(&plane_full[sp], C::SPLIT);
+            bulk_copy_g2s(ts + sp * C::SPLIT, src + sp * C::SPLIT, C::SPLIT, &plane_full[sp]);
+          }
+        }
       }
-      const uint32_t issued = j, first = issued > kXStages ? issued - kXStages : 0;
+      const int issued = j, first = issued > kXStages ? issued - kXStages : 0;
       volatile int no_abort = 0;
-      for (uint32_t q = first; q < issued; ++q)
-        mbar_wait_bounded(&bars->x_full[q % kXStages], (q / kXStages) & 1, &no_abort);
+      for (int q = first; q < issued; ++q) mbar_wait_bounded(&bars->x_full[q % kXStages], (q / kXStages) & 1, &no_abort);
+      if (own_planes)
+        for (int sp = 0; sp < 3; ++sp) mbar_wait_bounded(&plane_full[sp], 0, &no_abort);
+      (void)ok;
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer: unit j -> columns j K
+    // D = V H^T + V M^T + V L^T, plane by plane
     if (lane == 0) {
       bool ok = true;
-      uint32_t j = 0, version = 0;
+      uint32_t version = 0;
       int cur_b = -1;
-      for (int64_t u = u0; u < u1 && ok; ++u, ++j) {
-        const int b = (int)(u / num_tiles);
+      for (int j = 0; j < nu && ok; ++j) {
+        int b, tile;
+        fused_unit(fu, j, num_tiles, &b, &tile);
         if (b != cur_b) {
-          if (!(ok = mbar_wait_bounded(&bars->t_full, version & 1, abort_flag, __LINE__))) break;
+          if (!own_planes && !(ok = mbar_wait_bounded(&bars->t_full, version & 1, abort_flag, __LINE__))) break;
           ++version;
           cur_b = b;
         }
@@ -594,129 +720,177 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t xbase = smem_u32(xs + st * C::X_STAGE);
         const uint32_t tbase = smem_u32(ts);
 #pragma unroll
-        for (int kk = 0; kk < K / 16; ++kk) {
-          const uint32_t a_off = (kk >> 2) * (TM * 128) + (kk & 3) * 32;
-          const uint32_t b_off = (kk >> 2) * (K * 128) + (kk & 3) * 32;
-          const uint64_t da = sdesc_kmajor_sw128(xbase + a_off);
+        for (int sp = 0; sp < 3; ++sp) {
+          if (own_planes && j == 0) {                   // later units find every plane in place
+            if (!(ok = mbar_wait_bounded(&plane_full[sp], 0, abort_flag, __LINE__))) break;
+            tc_fence_after();
+          }
 #pragma unroll
-          for (int sp = 0; sp < 3; ++sp)
-            mma_bf16(dcol, da, sdesc_kmajor_sw128(tbase + sp * C::SPLIT + b_off), C::IDESC, (kk | sp) != 0);
+          for (int kk = 0; kk < K / 16; ++kk) {
+            const uint32_t a_off = (kk >> 2) * (TM * 128) + (kk & 3) * 32;
+            const uint32_t b_off = (kk >> 2) * (K * 128) + (kk & 3) * 32;
+            mma_bf16(dcol, sdesc_kmajor_sw128(xbase + a_off), sdesc_kmajor_sw128(tbase + sp * C::SPLIT + b_off), C::IDESC,
+                     (kk | sp) != 0);
+          }
         }
+        if (!ok) break;
         mma_commit(&bars->x_empty[st]);
         mma_commit(&unit_full[j]);
-        const bool last_of_block = (u + 1 >= u1) || ((int)((u + 1) / num_tiles) != b);
-        if (last_of_block) mma_commit(&bars->t_empty);
+        int nb_next = -1, tile_next;
+        if (j + 1 < nu) fused_unit(fu, j + 1, num_tiles, &nb_next, &tile_next);
+        if (nb_next != b) mma_commit(&bars->t_empty);     // the CTA's last unit of block b
       }
       mma_commit(&bars->mma_done);
       volatile int no_abort = 0;
       mbar_wait_bounded(&bars->mma_done, 0, &no_abort);
     }
-  } else if (warp >= kCvtWarp0) {
-    // ---------------------------------------------------------------- split A_b into bf16 H, M, L
-    const int ct = tid - kCvtWarp0 * 32;
-    bool ok = true;
-    uint32_t version = 0;
-    int cur_b = -1;
-    for (int64_t u = u0; u < u1 && ok; ++u) {
-      const int b = (int)(u / num_tiles);
-      if (b == cur_b) continue;
-      if (version > 0 && !(ok = mbar_wait_bounded(&bars->t_empty, (version - 1) & 1, abort_flag, __LINE__))) break;
-      cur_b = b;
-      if (planes) {                                    // one thread copies the pre-split planes
-        if (ct == 0) {
-          fetch_planes<K>(planes, b, ts, &bars->t_full);
-          if (version == 0) mbar_arrive(&bars->t_first);
-        }
-      } else {
-        split_block<K>(A + (size_t)b * K * K, ts, ct);
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) {
-          mbar_arrive(&bars->t_full);
-          if (version == 0) mbar_arrive(&bars->t_first);
+  } else if (warp == 2) {
+    // ---------------------------------------------------------------- watcher: final maxima, unit by unit
+    int done = 0;
+    for (; done < nu; ++done) {
+      const int j = done;
+      int b, tile;
+      fused_unit(fu, j, num_tiles, &b, &tile);
+      bool ok = true;
+      if (lane == 0) ok = wait_count(tile_rec + (size_t)tile * kTileWords, 4u * (uint32_t)nb, abort_flag, __LINE__);
+      if (!__shfl_sync(0xFFFFFFFFu, (int)ok, 0)) break;
+      // unit j's MMAs are done (this CTA counted the tile after them): at k = 128 its x stage is free
+      if (!__all_sync(0xFFFFFFFFu, mbar_wait_bounded(&unit_full[j], 0, abort_flag, __LINE__))) break;
+      fence_proxy_async_smem();
+      uint32_t v[TM / 32];
+#pragma unroll
+      for (int i = 0; i < TM / 32; ++i) v[i] = __ldcg(&amax_bits[tile * TM + 32 * i + lane]);  // < kAmaxRows
+      float* am = reinterpret_cast<float*>(C::amax_tile(smem, j));
+#pragma unroll
+      for (int i = 0; i < TM / 32; ++i) am[32 * i + lane] = __uint_as_float(v[i]);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&maxima_ready[j]);
+      if (b == 0) {                                      // the CTAs holding block 0 write the steps
+#pragma unroll
+        for (int i = 0; i < TM / 32; ++i) {
+          const int t = tile * TM + 32 * i + lane;
+          const float a = __uint_as_float(v[i]);
+          if (t >= n) continue;
+          float sc = 0.f;
+          if (isfinite(a))
+            sc = __fdiv_rn(a, 7.0f);
+          else
+            report(status, kStatusNonFinite);
+          scale[t] = sc;
         }
       }
-      ++version;
     }
-    quant_bar();                                       // the epilogue warps have passed the first grid barrier
-    quantize_jobs<K>(tmem, u0, u1, num_tiles, n, d, amax_bits, codes, abort_flag, 1 + ((warp - kCvtWarp0) >> 2));
-    quant_bar();
+    // This CTA has read the maxima of its first `done` tiles: the last of a tile's nb readers returns
+    // them and the tile's record to zero.  Off the units' path: every unit is released by now.
+    __syncwarp();
+    uint32_t last = 0;
+    if (lane < done) {
+      int b, tile;
+      fused_unit(fu, lane, num_tiles, &b, &tile);
+      last = atomicAdd(tile_rec + (size_t)tile * kTileWords + kTileWords / 2, 1u) == (uint32_t)nb - 1u;
+    }
+    uint32_t lasts = __ballot_sync(0xFFFFFFFFu, last);
+    while (lasts) {
+      const int j = __ffs(lasts) - 1;
+      lasts &= lasts - 1;
+      int b, tile;
+      fused_unit(fu, j, num_tiles, &b, &tile);
+      __threadfence();
+#pragma unroll
+      for (int i = 0; i < TM / 32; ++i) amax_bits[tile * TM + 32 * i + lane] = 0u;
+      if (lane == 0) {
+        tile_rec[(size_t)tile * kTileWords] = 0u;
+        tile_rec[(size_t)tile * kTileWords + kTileWords / 2] = 0u;
+      }
+    }
+    // With every unit released, no warp of this CTA touches the slot again (the epilogue's atomics and
+    // the publisher's counts came before the last tile's count was complete): count the CTA out now,
+    // while the quantizer warps finish.  A CTA that gave up counts itself out at the end instead.
+    if (__shfl_sync(0xFFFFFFFFu, (int)(done == nu && !*abort_flag), 0)) {
+      exit_slot<32>(sync, amax_bits, tile_rec, num_tiles, lane, false, exit_counted + 1);
+      if (lane == 0) *exit_counted = 1;
+    }
+  } else if (warp == 3) {
+    // ---------------------------------------------------------------- publisher: a unit's count
+    // The four epilogue warps of unit j arrive on epi_done[j] after issuing the unit's atomicMax; the
+    // fence here (after that CTA-scope synchronization) orders them before the count at GPU scope, so
+    // the epilogue warps never wait on a fence themselves.
+    if (lane == 0) {
+      for (int j = 0; j < nu; ++j) {
+        int b, tile;
+        fused_unit(fu, j, num_tiles, &b, &tile);
+        if (!mbar_wait_bounded(&epi_done[j], 0, abort_flag, __LINE__)) break;
+        __threadfence();
+        atomicAdd(&tile_rec[(size_t)tile * kTileWords], 4u);
+      }
+    }
+  } else if (warp >= kCvtWarp0) {
+    // ---------------------------------------------------------------- T_b into shared memory, then phase B
+    if (!own_planes) {
+      const int ct = tid - kCvtWarp0 * 32;
+      bool ok = true;
+      uint32_t version = 0;
+      int cur_b = -1;
+      for (int j = 0; j < nu && ok; ++j) {
+        int b, tile;
+        fused_unit(fu, j, num_tiles, &b, &tile);
+        if (b == cur_b) continue;
+        if (version > 0 && !(ok = mbar_wait_bounded(&bars->t_empty, (version - 1) & 1, abort_flag, __LINE__))) break;
+        cur_b = b;
+        if (planes) {                                  // one thread copies the pre-split planes
+          if (ct == 0) {
+            fetch_planes<K>(planes, b, ts, &bars->t_full);
+            if (version == 0) mbar_arrive(&bars->t_first);
+          }
+        } else {
+          split_block<K>(A + (size_t)b * K * K, ts, ct);
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            mbar_arrive(&bars->t_full);
+            if (version == 0) mbar_arrive(&bars->t_first);
+          }
+        }
+        ++version;
+      }
+    }
+    quantize_units<K>(tmem, smem, fu, num_tiles, n, d, maxima_ready, codes, abort_flag, 1 + ((warp - kCvtWarp0) >> 2));
     tc_fence_before();
   } else if (warp >= kEpiWarp0) {
-    // ---------------------------------------------------------------- epilogue: one row per thread
+    // ---------------------------------------------------------------- phase A: one row per thread
     const int quad = warp & 3;
-    const bool leader = warp == kEpiWarp0 && lane == 0;
-    const int nu = (int)(u1 - u0);
     bool finite = true;
-    // phase A: row maxima of every unit's tile
     for (int j = 0; j < nu; ++j) {
-      const int tile = (int)((u0 + j) % num_tiles);
+      int b, tile;
+      fused_unit(fu, j, num_tiles, &b, &tile);
       const int t = tile * TM + quad * 32 + lane;
       const bool got = !*abort_flag && mbar_wait_bounded(&unit_full[j], 0, abort_flag, __LINE__);
       if (!__all_sync(0xFFFFFFFFu, got)) break;        // warp-uniform: TMEM loads need the whole warp
       tc_fence_after();
-      float m = 0.f;
-      bool row_finite = true;
+      uint32_t mb = 0;
 #pragma unroll 1
-      for (int c = 0; c < K / 32; ++c) {
-        uint32_t r[32];
+      for (int c = 0; c < K / 32; c += 2) {            // two loads in flight
+        uint32_t r0[32], r1[32];
         __syncwarp();
-        CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + j * K + c * 32, r);
+        CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + j * K + c * 32, r0);
+        CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + j * K + (c + 1) * 32, r1);
         tmem_ld_wait();
-#pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          const float v = __uint_as_float(r[e]);
-          row_finite &= isfinite(v);
-          m = fmaxf(m, fabsf(v));
-        }
+        mb = absmax_bits32(r1, absmax_bits32(r0, mb));
       }
+      const bool row_finite = mb < 0x7F800000u;
       finite &= row_finite;
       // a non-finite value makes the row's maximum the largest NaN pattern: its codes and step become 0
-      if (t < n) atomicMax(&amax_bits[t], row_finite ? __float_as_uint(m) : 0x7FFFFFFFu);
+      if (t < n) atomicMax(&amax_bits[t], row_finite ? mb : 0x7FFFFFFFu);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&epi_done[j]);
     }
     if (!finite) report(status, kStatusNonFinite);
-    grid_barrier(&sync[0], gridDim.x, abort_flag, leader);
-    // phase B: the tiles still in tensor memory, quantized with the final row maxima by the 12 warps
-    // that own TMEM lane quadrants (4 epilogue + 8 converter warps), a 32-column chunk per job
-    quant_bar();
-    quantize_jobs<K>(tmem, u0, u1, num_tiles, n, d, amax_bits, codes, abort_flag, 0);
-    quant_bar();
-    // the steps of the rows this CTA holds in block 0 (the maxima are final since the grid barrier)
-    if (!__any_sync(0xFFFFFFFFu, *abort_flag)) {
-      for (int64_t u = u0; u < u1; ++u) {
-        const int tile = (int)(u % num_tiles);
-        const int t = tile * TM + quad * 32 + lane;
-        if (u / num_tiles != 0 || t >= n) continue;
-        const float a = __uint_as_float(__ldcg(&amax_bits[t]));
-        float sc = 0.f;
-        if (isfinite(a))
-          sc = __fdiv_rn(a, 7.0f);
-        else
-          report(status, kStatusNonFinite);
-        scale[t] = sc;
-      }
-    }
+    quantize_units<K>(tmem, smem, fu, num_tiles, n, d, maxima_ready, codes, abort_flag, 0);
     tc_fence_before();
   }
 
-  // the last CTA out returns the launch's slot to zero: every CTA has passed the grid barrier and read
-  // its maxima before it counts itself out
-  __shared__ int last_out;
   __syncthreads();
-  if (tid == 0) {
-    __threadfence();
-    last_out = atomicAdd(&sync[1], 1u) == gridDim.x - 1;
-  }
-  __syncthreads();
-  if (last_out) {
-    __threadfence();
-    for (int t = tid; t < n; t += kThreads) amax_bits[t] = 0u;
-    if (tid == 0) sync[0] = 0u;
-    __threadfence();
-    __syncthreads();
-    if (tid == 0) sync[1] = 0u;
-  }
-  __syncthreads();
+  if (!*exit_counted) exit_slot<kThreads>(sync, amax_bits, tile_rec, num_tiles, tid, bars->abort != 0, exit_counted + 1);
   if (bars->abort && tid == 0) report(status, timeout_bits(kWhereTransformFused, bars->abort));
   if (warp == 0) {
     tc_fence_after();
@@ -748,7 +922,7 @@ int num_sms() {
   return sms;
 }
 
-uint32_t* sync_slots(cudaError_t* err, uint32_t** amax_slots);
+uint32_t* sync_slots(cudaError_t* err, uint32_t** amax_slots, uint32_t** tile_slots = nullptr);
 
 // Slots of the transform's device scratch, handed out round robin to every launch that uses one
 // (fused or two-pass), so that up to kSyncSlots such launches may be in flight at once.
@@ -807,12 +981,13 @@ cudaError_t launch_k(const __nv_bfloat16* x, int64_t n, int64_t d, const float* 
   return cudaGetLastError();
 }
 
-// Address of this device's barrier slots (looked up once per device).
-// The device's slot arrays (grid-barrier and exit counters; row maxima), looked up once per device.
-uint32_t* sync_slots(cudaError_t* err, uint32_t** amax_slots) {
+// The device's slot arrays (exit counters and flags; row maxima; row-tile records), looked up once
+// per device.
+uint32_t* sync_slots(cudaError_t* err, uint32_t** amax_slots, uint32_t** tile_slots) {
   static std::mutex mu;
   static uint32_t* cache[64] = {nullptr};
   static uint32_t* amax_cache[64] = {nullptr};
+  static uint32_t* tile_cache[64] = {nullptr};
   int dev = 0;
   *err = cudaGetDevice(&dev);
   if (*err != cudaSuccess) return nullptr;
@@ -824,12 +999,16 @@ uint32_t* sync_slots(cudaError_t* err, uint32_t** amax_slots) {
   if (!cache[dev]) {
     void* p = nullptr;
     void* q = nullptr;
+    void* r = nullptr;
     if ((*err = cudaGetSymbolAddress(&p, g_tq_sync)) != cudaSuccess) return nullptr;
     if ((*err = cudaGetSymbolAddress(&q, g_tq_amax)) != cudaSuccess) return nullptr;
+    if ((*err = cudaGetSymbolAddress(&r, g_tq_tiles)) != cudaSuccess) return nullptr;
     cache[dev] = static_cast<uint32_t*>(p);
     amax_cache[dev] = static_cast<uint32_t*>(q);
+    tile_cache[dev] = static_cast<uint32_t*>(r);
   }
   *amax_slots = amax_cache[dev];
+  if (tile_slots) *tile_slots = tile_cache[dev];
   return cache[dev];
 }
 
@@ -847,22 +1026,21 @@ cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, const f
   const int tiles = (int)((n + TM - 1) / TM);
   const int64_t units = (int64_t)nb * tiles;
   const int grid = (int)(units < num_sms() ? units : num_sms());
-  for (int c = 0; c < grid; ++c) {  // every CTA's units must fit in tensor memory at once
-    int64_t u0, u1;
-    unit_range(c, grid, nb, tiles, &u0, &u1);
-    if (u1 - u0 > 512 / K) return cudaErrorNotSupported;
-  }
+  for (int c = 0; c < grid; ++c)  // every CTA's units must fit in tensor memory at once
+    if (fused_units(c, grid, nb, tiles).count > 512 / K) return cudaErrorNotSupported;
   if (!cooperative_ok()) return cudaErrorNotSupported;
   EncodeTiledFn fn = encode_fn();
   if (!fn) return cudaErrorNotSupported;
   if (n > kAmaxRows) return cudaErrorNotSupported;
   cudaError_t e;
   uint32_t* amax_slots = nullptr;
-  uint32_t* slots = sync_slots(&e, &amax_slots);
+  uint32_t* tile_slots = nullptr;
+  uint32_t* slots = sync_slots(&e, &amax_slots, &tile_slots);
   if (!slots) return e;
   const uint32_t slot = next_tq_slot();
   uint32_t* sync = slots + 4 * slot;
   uint32_t* amax_bits = amax_slots + (size_t)kAmaxRows * slot;
+  uint32_t* tile_rec = tile_slots + (size_t)kAmaxTiles * kTileWords * slot;
   CUtensorMap map;
   memset(&map, 0, sizeof(map));
   cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)n};
@@ -877,14 +1055,14 @@ cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, const f
   static cudaError_t attr = cudaSuccess;
   std::call_once(once, [] {
     attr = cudaFuncSetAttribute(transform_quant_tc_fused_kernel<K>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)C::SMEM);
+                                (int)C::FUSED_SMEM);
   });
   if (attr != cudaSuccess) return attr;
   cudaLaunchConfig_t cfg;
   memset(&cfg, 0, sizeof(cfg));
   cfg.gridDim = dim3((unsigned)grid, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = C::SMEM;
+  cfg.dynamicSmemBytes = C::FUSED_SMEM;
   cfg.stream = stream;
   // not a programmatic dependent launch: measured, one cost the c2 step ~4 us (the kernel still
   // releases its dependents early, so a programmatic GEMM launch after it gets going sooner)
@@ -895,7 +1073,7 @@ cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, const f
   cfg.numAttrs = 1;
   note_launch();
   return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<K>, map, A, planes, (int)n, (int)d,
-                            reinterpret_cast<float*>(amax), words, sync, amax_bits, status);
+                            reinterpret_cast<float*>(amax), words, sync, amax_bits, tile_rec, status);
 }
 
 }  // namespace
