@@ -208,44 +208,70 @@ __device__ __forceinline__ uint32_t twos_to_sm(uint32_t w) {
   return ((w ^ m) + s) | (s << 7);                   // |q| (no carry leaves a byte) and the sign bit
 }
 
-// The four SM4x8 words of the codes of the 32 values v_e = r[e] (as float) on the row described by
-// qr (|v_e| <= max|v|).  Fast route: adding 1.5 * 2^23 to p = fl(v_e * inv) rounds it to an integer
-// (half to even) that sits, two's complement, in the low byte of the sum's bits; the bytes are
-// gathered four to a word and turned into sign-magnitude.  One near-tie test covers the chunk (one
-// branch, so the 32 products overlap): if any p lies within 2^-18 of a half-integer (an exact tie
-// included), or the row is rescaled, the 32 codes are decided exactly instead (qcode_exact).
+// qcode_exact out of line: the rare near-tie route then costs a call, not 32 inlined copies.
+__device__ __noinline__ int qcode_exact_call(float v, QRow qr) { return qcode_exact(v, qr, 7.0f); }
+
+// The four SM4x8 words of the codes of the 32 values v_e in tensor memory at taddr (this lane's row,
+// 32 columns) on the row described by qr (|v_e| <= max|v|); called by the whole warp.  Fast route:
+// adding 1.5 * 2^23 to p = fl(v_e * inv) rounds it to an integer (half to even) that sits, two's
+// complement, in the low byte of the sum's bits; the bytes are gathered four to a word and turned
+// into sign-magnitude.  The products and sums run as f32x2 pairs, with the same rounding as the scalar
+// operations.  If any lane has a p within 2^-18 of a half-integer (an exact tie included), or a
+// rescaled row, the warp reloads the chunk and the lanes concerned decide those values' codes exactly
+// (qcode_exact): the values are not kept live across that rare branch, which leaves the fast route
+// its registers, and the branch costs about one exact decision rather than 32.
 // qr.inv == 0 (an all-zero or non-finite row): all codes 0.
-__device__ __forceinline__ uint4 sm4_quant32(const uint32_t (&r)[32], const QRow& qr) {
+__device__ __forceinline__ uint4 quant_chunk(uint32_t taddr, const QRow& qr) {
   constexpr float kMagic = 12582912.0f;
-  if (qr.inv == 0.f) return make_uint4(0u, 0u, 0u, 0u);
-  uint32_t b[32];
+  uint32_t bq[32];
   bool near = qr.exact;
+  {
+    uint32_t r[32];
+    __syncwarp();
+    CAT_TMEM_LD32(taddr, r);
+    tmem_ld_wait();
+    uint64_t inv2, mg2;
+    asm("mov.b64 %0, {%1, %1};" : "=l"(inv2) : "f"(qr.inv));
+    asm("mov.b64 %0, {%1, %1};" : "=l"(mg2) : "f"(kMagic));
 #pragma unroll
-  for (int e = 0; e < 32; ++e) {
-    const float p = __fmul_rn(__uint_as_float(r[e]), qr.inv);
-    const float rb = __fadd_rn(p, kMagic);
-    near |= fabsf(__fsub_rn(__fsub_rn(rb, kMagic), p)) > kNearTie;
-    b[e] = __float_as_uint(rb);
+    for (int e = 0; e < 32; e += 2) {
+      uint64_t v2, p2, rb2, d2;
+      asm("mov.b64 %0, {%1, %2};" : "=l"(v2) : "r"(r[e]), "r"(r[e + 1]));
+      asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(p2) : "l"(v2), "l"(inv2));
+      asm("add.rn.f32x2 %0, %1, %2;" : "=l"(rb2) : "l"(p2), "l"(mg2));
+      asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d2) : "l"(rb2), "l"(mg2));
+      asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d2) : "l"(d2), "l"(p2));
+      float d0, d1;
+      asm("mov.b64 {%0, %1}, %2;" : "=f"(d0), "=f"(d1) : "l"(d2));
+      asm("mov.b64 {%0, %1}, %2;" : "=r"(bq[e]), "=r"(bq[e + 1]) : "l"(rb2));
+      near |= fmaxf(fabsf(d0), fabsf(d1)) > kNearTie;
+    }
   }
+  if (__any_sync(0xFFFFFFFFu, near)) {
+    uint32_t r[32];
+    __syncwarp();
+    CAT_TMEM_LD32(taddr, r);
+    tmem_ld_wait();
+    if (near) {                                  // patch the codes of this lane's near values only
+#pragma unroll
+      for (int e = 0; e < 32; ++e) {
+        const float v = __uint_as_float(r[e]);
+        const float p = __fmul_rn(v, qr.inv);
+        if (qr.exact || fabsf(__fsub_rn(__fsub_rn(__fadd_rn(p, kMagic), kMagic), p)) > kNearTie)
+          bq[e] = (bq[e] & ~0xFFu) | ((uint32_t)qcode_exact_call(v, qr) & 0xFFu);
+      }
+    }
+  }
+  if (qr.inv == 0.f) return make_uint4(0u, 0u, 0u, 0u);
   uint32_t w[4];
-  if (near) {
 #pragma unroll
-    for (int g = 0; g < 4; ++g) {
-      int q[8];
-#pragma unroll
-      for (int e = 0; e < 8; ++e) q[e] = qcode_exact(__uint_as_float(r[8 * g + e]), qr, 7.0f);
-      w[g] = sm4_pack(q);
-    }
-  } else {
-#pragma unroll
-    for (int g = 0; g < 4; ++g) {
-      const uint32_t* bg = b + 8 * g;
-      const uint32_t lo =
-          twos_to_sm(__byte_perm(__byte_perm(bg[0], bg[1], 0x0040), __byte_perm(bg[2], bg[3], 0x0040), 0x5410));
-      const uint32_t hi =
-          twos_to_sm(__byte_perm(__byte_perm(bg[4], bg[5], 0x0040), __byte_perm(bg[6], bg[7], 0x0040), 0x5410));
-      w[g] = lo | __funnelshift_l(hi, hi, 4);
-    }
+  for (int g = 0; g < 4; ++g) {
+    const uint32_t* bg = bq + 8 * g;
+    const uint32_t lo =
+        twos_to_sm(__byte_perm(__byte_perm(bg[0], bg[1], 0x0040), __byte_perm(bg[2], bg[3], 0x0040), 0x5410));
+    const uint32_t hi =
+        twos_to_sm(__byte_perm(__byte_perm(bg[4], bg[5], 0x0040), __byte_perm(bg[6], bg[7], 0x0040), 0x5410));
+    w[g] = lo | __funnelshift_l(hi, hi, 4);
   }
   return make_uint4(w[0], w[1], w[2], w[3]);
 }
@@ -427,22 +453,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool row_finite = true;
 #pragma unroll 1
       for (int c = 0; c < K / 32; ++c) {
-        uint32_t r[32];
-        __syncwarp();
-        CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + sd * K + c * 32, r);
-        tmem_ld_wait();
+        const uint32_t taddr = tmem + ((uint32_t)(quad * 32) << 16) + sd * K + c * 32;
         if (PASS == 0) {
+          uint32_t r[32];
+          __syncwarp();
+          CAT_TMEM_LD32(taddr, r);
+          tmem_ld_wait();
 #pragma unroll
           for (int e = 0; e < 32; ++e) {
             const float v = __uint_as_float(r[e]);
             row_finite &= isfinite(v);
             m = fmaxf(m, fabsf(v));
           }
-        } else if (t < n) {
+        } else {
           // the row's codes with the final maximum (|v * inv| <= 7 for a finite row; inv = 0 gives
           // 0 codes for an all-zero or non-finite row)
-          *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * K + c * 32) / 8) =
-              sm4_quant32(r, qr);
+          const uint4 w = quant_chunk(taddr, qr);
+          if (t < n) *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * K + c * 32) / 8) = w;
         }
       }
       tc_fence_before();
@@ -483,23 +510,29 @@ __global__ void __launch_bounds__(kThreads, 1)
 //
 // When every CTA's units fit in tensor memory at once (units per CTA x K <= 512 columns), one
 // cooperative launch does both passes.  Phase A runs the MMAs once, keeps each unit's x' tile in its
-// own TMEM columns and publishes the tile's row maxima (atomicMax into the launch's scratch slot,
-// then one count per epilogue warp on the tile's record).  Phase B needs a row's maximum over all
-// blocks, i.e. all nb units of a row tile, but not the rest of the grid: a watcher warp per CTA waits
-// for each of its tiles' counts in turn, copies the final maxima to shared memory and releases the
-// quantizer warps for that unit, while later units are still in phase A.  The CTAs holding block 0
-// write the steps s = max / 7; the last CTA to read a tile's maxima returns them and the tile's
-// record to zero, so a launch, a graph replay of it included, always starts from a clean slot.
-// Every wait is bounded; a launch that gave up somewhere has its whole slot zeroed by the last CTA
-// to leave.  Slots are handed out round robin, so up to kSyncSlots launches may run at once on
-// different streams.
+// own TMEM columns and publishes the tile's row maxima (atomicMax into the launch's scratch, then a
+// count on the tile's record).  Phase B needs a row's maximum over all blocks, i.e. all nb units of a
+// row tile, but not the rest of the grid: a watcher warp per CTA waits for each of its tiles' counts
+// in turn, copies the final maxima to shared memory and releases the quantizer warps for that unit,
+// while later units are still in phase A.  The CTAs holding block 0 write the steps s = max / 7.
+//
+// Scratch: each slot (up to kSyncSlots launches may run at once on different streams; slots are
+// handed out round robin) has two sets of maxima and tile records, used by alternate launches on the
+// slot.  A launch reads the slot's epoch at start (parity = its set), zeroes the other set (left by
+// the previous launch on the slot, which has finished: a launch that gave up is cleaned up the same
+// way), and the last of its CTAs to start moves the epoch on and records how many tiles its set
+// holds.  The state lives on the device, so graph replays alternate too, and no CTA has to wait for
+// the others at the end.  Every wait is bounded.
 constexpr int kSyncSlots = 8;
 constexpr int kAmaxRows = 1 << 17;             // rows the fused path can have (<= 1024 tiles of 128 rows)
 constexpr int kAmaxTiles = kAmaxRows / TM;
-constexpr int kTileWords = 32;                 // per tile: [0] maxima published (counts), [16] maxima read
-__device__ __align__(16) uint32_t g_tq_sync[kSyncSlots][4];
-__device__ uint32_t g_tq_amax[kSyncSlots][kAmaxRows];
-__device__ __align__(128) uint32_t g_tq_tiles[kSyncSlots][kAmaxTiles * kTileWords];
+constexpr int kTileWords = 32;                 // a tile's record ([0]: units' maxima published, 4 per unit)
+__device__ __align__(16) uint32_t g_tq_sync[kSyncSlots][4];          // two-pass kernel: [1] exit counter
+__device__ uint32_t g_tq_amax[kSyncSlots][kAmaxRows];                // two-pass kernel: row maxima
+// fused kernel: [0] epoch, [1] CTAs started, [2 + s] tiles set s holds
+__device__ __align__(16) uint32_t g_tqf_state[kSyncSlots][4];
+__device__ uint32_t g_tqf_amax[kSyncSlots][2][kAmaxRows];
+__device__ __align__(128) uint32_t g_tqf_tiles[kSyncSlots][2][kAmaxTiles * kTileWords];
 
 __device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
   uint32_t v;
@@ -552,42 +585,8 @@ __device__ __forceinline__ void quantize_units(uint32_t tmem, uint8_t* smem, con
 #pragma unroll 1
     for (int c = 0; c < K / 32; ++c) {
       if (chunk_slot(c, last) != slot) continue;
-      uint32_t r[32];
-      __syncwarp();
-      CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + j * K + c * 32, r);
-      tmem_ld_wait();
-      if (t < n)
-        *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * K + c * 32) / 8) =
-            sm4_quant32(r, qr);
-    }
-  }
-}
-
-// Counts the CTA out of the launch's slot; called by every thread of a group of NT threads (the
-// watcher warp, NT = 32, or the whole CTA), id = 0 .. NT - 1.  The last CTA out resets the exit
-// counter and, if some CTA gave up (a tile's maxima and record may then be left behind), first zeroes
-// the slot's maxima and tile records.
-template <int NT>
-__device__ __forceinline__ void exit_slot(uint32_t* sync, uint32_t* amax_bits, uint32_t* tile_rec, int num_tiles, int id,
-                                          bool gave_up, volatile int* last_out) {
-  if (id == 0) {
-    __threadfence();
-    if (gave_up) atomicOr(&sync[2], 1u);
-    __threadfence();
-    *last_out = atomicAdd(&sync[1], 1u) == gridDim.x - 1;
-  }
-  if (NT == 32) __syncwarp(); else __syncthreads();
-  if (*last_out) {
-    __threadfence();
-    if (ld_acquire_gpu(&sync[2]) != 0u) {
-      for (int t = id; t < num_tiles * TM; t += NT) amax_bits[t] = 0u;
-      for (int i = id; i < num_tiles * kTileWords; i += NT) tile_rec[i] = 0u;
-    }
-    __threadfence();
-    if (NT == 32) __syncwarp(); else __syncthreads();
-    if (id == 0) {
-      sync[2] = 0u;
-      sync[1] = 0u;
+      const uint4 w = quant_chunk(tmem + ((uint32_t)(quad * 32) << 16) + j * K + c * 32, qr);
+      if (t < n) *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * K + c * 32) / 8) = w;
     }
   }
 }
@@ -596,14 +595,14 @@ template <int K>
 __global__ void __launch_bounds__(kThreads, 1)
     transform_quant_tc_fused_kernel(const __grid_constant__ CUtensorMap tmX, const float* __restrict__ A,
                                     const uint8_t* __restrict__ planes, int n, int d, float* __restrict__ scale,
-                                    uint32_t* __restrict__ codes, uint32_t* __restrict__ sync,
-                                    uint32_t* __restrict__ amax_bits, uint32_t* __restrict__ tile_rec,
+                                    uint32_t* __restrict__ codes, uint32_t* __restrict__ state,
+                                    uint32_t* __restrict__ amax_sets, uint32_t* __restrict__ rec_sets,
                                     uint32_t* __restrict__ status) {
-  // sync: [1] exit counter, [2] set by a CTA that gave up; amax_bits: the row maxima (float bits);
-  // tile_rec: kTileWords words per row tile (maxima published, maxima read)
+  // state: the slot's epoch, start counter and tiles per set; amax_sets: two sets of kAmaxRows row
+  // maxima (float bits); rec_sets: two sets of kAmaxTiles tile records
   using C = TcCfg<K>;
   constexpr int kMaxUnits = 512 / K;
-  static_assert(sizeof(TcBars) + (3 * kMaxUnits + 3) * sizeof(uint64_t) + 16 <= C::FUSED_BAR_BYTES, "barrier room");
+  static_assert(sizeof(TcBars) + (3 * kMaxUnits + 4) * sizeof(uint64_t) + 8 <= C::FUSED_BAR_BYTES, "barrier room");
   static_assert(K != 128 || kMaxUnits <= kXStages, "at k = 128 unit j's x stage holds its maxima");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -614,8 +613,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* epi_done = unit_full + kMaxUnits;                     // per unit, used once: its atomics are issued
   uint64_t* maxima_ready = epi_done + kMaxUnits;                  // per unit, used once: final maxima in smem
   uint64_t* plane_full = maxima_ready + kMaxUnits;                // per plane of T_b (producer-fetched planes)
-  volatile int* exit_counted = reinterpret_cast<int*>(plane_full + 3);  // [0] the watcher counted the CTA out,
-                                                                         // [1] the CTA was the last out
+  uint64_t* set_ready = plane_full + 3;                           // the launch's scratch set is known
+  volatile int* set_sel = reinterpret_cast<int*>(set_ready + 1);  // ... and it is set_sel (0 or 1)
   volatile int* abort_flag = &bars->abort;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -639,12 +638,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&maxima_ready[j], 1);
     }
     for (int sp = 0; sp < 3; ++sp) mbar_init(&plane_full[sp], 1);
+    mbar_init(set_ready, 1);
     mbar_init(&bars->t_first, planes ? 1 : kCvtWarps);   // pre-split planes: one copying thread
     mbar_init(&bars->t_full, planes ? 1 : kCvtWarps);
     mbar_init(&bars->t_empty, 1);
     mbar_init(&bars->mma_done, 1);
     bars->abort = 0;
-    *exit_counted = 0;
     fence_mbar_init();
   }
   __syncwarp();
@@ -746,9 +745,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 2) {
     // ---------------------------------------------------------------- watcher: final maxima, unit by unit
-    int done = 0;
-    for (; done < nu; ++done) {
-      const int j = done;
+    const bool have_set = __all_sync(0xFFFFFFFFu, mbar_wait_bounded(set_ready, 0, abort_flag, __LINE__));
+    const int P = *set_sel;
+    const uint32_t* amax_bits = amax_sets + (size_t)P * kAmaxRows;
+    const uint32_t* tile_rec = rec_sets + (size_t)P * kAmaxTiles * kTileWords;
+    for (int j = 0; j < nu && have_set; ++j) {
       int b, tile;
       fused_unit(fu, j, num_tiles, &b, &tile);
       bool ok = true;
@@ -780,42 +781,43 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-    // This CTA has read the maxima of its first `done` tiles: the last of a tile's nb readers returns
-    // them and the tile's record to zero.  Off the units' path: every unit is released by now.
-    __syncwarp();
-    uint32_t last = 0;
-    if (lane < done) {
-      int b, tile;
-      fused_unit(fu, lane, num_tiles, &b, &tile);
-      last = atomicAdd(tile_rec + (size_t)tile * kTileWords + kTileWords / 2, 1u) == (uint32_t)nb - 1u;
-    }
-    uint32_t lasts = __ballot_sync(0xFFFFFFFFu, last);
-    while (lasts) {
-      const int j = __ffs(lasts) - 1;
-      lasts &= lasts - 1;
-      int b, tile;
-      fused_unit(fu, j, num_tiles, &b, &tile);
-      __threadfence();
-#pragma unroll
-      for (int i = 0; i < TM / 32; ++i) amax_bits[tile * TM + 32 * i + lane] = 0u;
-      if (lane == 0) {
-        tile_rec[(size_t)tile * kTileWords] = 0u;
-        tile_rec[(size_t)tile * kTileWords + kTileWords / 2] = 0u;
-      }
-    }
-    // With every unit released, no warp of this CTA touches the slot again (the epilogue's atomics and
-    // the publisher's counts came before the last tile's count was complete): count the CTA out now,
-    // while the quantizer warps finish.  A CTA that gave up counts itself out at the end instead.
-    if (__shfl_sync(0xFFFFFFFFu, (int)(done == nu && !*abort_flag), 0)) {
-      exit_slot<32>(sync, amax_bits, tile_rec, num_tiles, lane, false, exit_counted + 1);
-      if (lane == 0) *exit_counted = 1;
-    }
   } else if (warp == 3) {
-    // ---------------------------------------------------------------- publisher: a unit's count
-    // The four epilogue warps of unit j arrive on epi_done[j] after issuing the unit's atomicMax; the
-    // fence here (after that CTA-scope synchronization) orders them before the count at GPU scope, so
-    // the epilogue warps never wait on a fence themselves.
+    // ---------------------------------------------------------------- publisher
+    // Start: the slot's epoch gives this launch's scratch set; this CTA's share of the other set (left
+    // by the previous launch on the slot, finished) goes back to zero; the last CTA to start moves the
+    // epoch on (every CTA has read it by then) and records the tiles this launch's set holds.
+    uint32_t E = 0, prev_tiles = 0;
+    if (lane == 0) E = ld_acquire_gpu(&state[0]);
+    E = __shfl_sync(0xFFFFFFFFu, E, 0);
+    const int P = (int)(E & 1u);
     if (lane == 0) {
+      *set_sel = P;
+      mbar_arrive(set_ready);
+      prev_tiles = state[2 + (P ^ 1)];
+    }
+    prev_tiles = min(__shfl_sync(0xFFFFFFFFu, prev_tiles, 0), (uint32_t)kAmaxTiles);
+    {
+      uint32_t* amax_o = amax_sets + (size_t)(P ^ 1) * kAmaxRows;
+      uint32_t* rec_o = rec_sets + (size_t)(P ^ 1) * kAmaxTiles * kTileWords;
+      const int64_t rows = (int64_t)prev_tiles * TM, words = (int64_t)prev_tiles * kTileWords;
+      const int64_t r0 = rows * blockIdx.x / gridDim.x, r1 = rows * (blockIdx.x + 1) / gridDim.x;
+      const int64_t w0 = words * blockIdx.x / gridDim.x, w1 = words * (blockIdx.x + 1) / gridDim.x;
+      for (int64_t i = r0 + lane; i < r1; i += 32) amax_o[i] = 0u;
+      for (int64_t i = w0 + lane; i < w1; i += 32) rec_o[i] = 0u;
+    }
+    __syncwarp();
+    uint32_t* tile_rec = rec_sets + (size_t)P * kAmaxTiles * kTileWords;
+    if (lane == 0) {
+      __threadfence();
+      if (atomicAdd(&state[1], 1u) == gridDim.x - 1) {
+        state[2 + P] = (uint32_t)num_tiles;
+        state[1] = 0u;
+        __threadfence();
+        state[0] = E + 1u;
+      }
+      // A unit's count: the four epilogue warps of unit j arrive on epi_done[j] after issuing the
+      // unit's atomicMax; the fence here (after that CTA-scope synchronization) orders them before the
+      // count at GPU scope, so the epilogue warps never wait on a fence themselves.
       for (int j = 0; j < nu; ++j) {
         int b, tile;
         fused_unit(fu, j, num_tiles, &b, &tile);
@@ -860,7 +862,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---------------------------------------------------------------- phase A: one row per thread
     const int quad = warp & 3;
     bool finite = true;
-    for (int j = 0; j < nu; ++j) {
+    const bool have_set = __all_sync(0xFFFFFFFFu, mbar_wait_bounded(set_ready, 0, abort_flag, __LINE__));
+    uint32_t* amax_bits = amax_sets + (size_t)(*set_sel) * kAmaxRows;
+    for (int j = 0; j < nu && have_set; ++j) {
       int b, tile;
       fused_unit(fu, j, num_tiles, &b, &tile);
       const int t = tile * TM + quad * 32 + lane;
@@ -890,7 +894,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   __syncthreads();
-  if (!*exit_counted) exit_slot<kThreads>(sync, amax_bits, tile_rec, num_tiles, tid, bars->abort != 0, exit_counted + 1);
   if (bars->abort && tid == 0) report(status, timeout_bits(kWhereTransformFused, bars->abort));
   if (warp == 0) {
     tc_fence_after();
@@ -922,7 +925,15 @@ int num_sms() {
   return sms;
 }
 
-uint32_t* sync_slots(cudaError_t* err, uint32_t** amax_slots, uint32_t** tile_slots = nullptr);
+// The device's scratch arrays, looked up once per device.
+struct TqScratch {
+  uint32_t* sync;       // two-pass kernel: [kSyncSlots][4]
+  uint32_t* amax;       // two-pass kernel: [kSyncSlots][kAmaxRows]
+  uint32_t* state;      // fused kernel: [kSyncSlots][4]
+  uint32_t* amax_sets;  // fused kernel: [kSyncSlots][2][kAmaxRows]
+  uint32_t* rec_sets;   // fused kernel: [kSyncSlots][2][kAmaxTiles * kTileWords]
+};
+const TqScratch* tq_scratch(cudaError_t* err);
 
 // Slots of the transform's device scratch, handed out round robin to every launch that uses one
 // (fused or two-pass), so that up to kSyncSlots such launches may be in flight at once.
@@ -965,12 +976,11 @@ cudaError_t launch_k(const __nv_bfloat16* x, int64_t n, int64_t d, const float* 
   if (scale) {
     if (n > kAmaxRows) return cudaErrorNotSupported;
     cudaError_t es;
-    uint32_t* amax_slots = nullptr;
-    uint32_t* slots = sync_slots(&es, &amax_slots);
-    if (!slots) return es;
+    const TqScratch* sc = tq_scratch(&es);
+    if (!sc) return es;
     const uint32_t slot = next_tq_slot();
-    exit_ctr = slots + 4 * slot + 1;
-    amax = amax_slots + (size_t)kAmaxRows * slot;
+    exit_ctr = sc->sync + 4 * slot + 1;
+    amax = sc->amax + (size_t)kAmaxRows * slot;
   }
   note_launch();
   k0<<<grid, kThreads, C::SMEM, stream>>>(map, A, planes, (int)n, (int)d, amax, words, nullptr, nullptr, status);
@@ -981,13 +991,10 @@ cudaError_t launch_k(const __nv_bfloat16* x, int64_t n, int64_t d, const float* 
   return cudaGetLastError();
 }
 
-// The device's slot arrays (exit counters and flags; row maxima; row-tile records), looked up once
-// per device.
-uint32_t* sync_slots(cudaError_t* err, uint32_t** amax_slots, uint32_t** tile_slots) {
+const TqScratch* tq_scratch(cudaError_t* err) {
   static std::mutex mu;
-  static uint32_t* cache[64] = {nullptr};
-  static uint32_t* amax_cache[64] = {nullptr};
-  static uint32_t* tile_cache[64] = {nullptr};
+  static TqScratch cache[64];
+  static bool have[64] = {false};
   int dev = 0;
   *err = cudaGetDevice(&dev);
   if (*err != cudaSuccess) return nullptr;
@@ -996,20 +1003,18 @@ uint32_t* sync_slots(cudaError_t* err, uint32_t** amax_slots, uint32_t** tile_sl
     return nullptr;
   }
   std::lock_guard<std::mutex> lock(mu);
-  if (!cache[dev]) {
-    void* p = nullptr;
-    void* q = nullptr;
-    void* r = nullptr;
-    if ((*err = cudaGetSymbolAddress(&p, g_tq_sync)) != cudaSuccess) return nullptr;
-    if ((*err = cudaGetSymbolAddress(&q, g_tq_amax)) != cudaSuccess) return nullptr;
-    if ((*err = cudaGetSymbolAddress(&r, g_tq_tiles)) != cudaSuccess) return nullptr;
-    cache[dev] = static_cast<uint32_t*>(p);
-    amax_cache[dev] = static_cast<uint32_t*>(q);
-    tile_cache[dev] = static_cast<uint32_t*>(r);
+  if (!have[dev]) {
+    void* p[5] = {nullptr, nullptr, nullptr, nullptr, nullptr};
+    if ((*err = cudaGetSymbolAddress(&p[0], g_tq_sync)) != cudaSuccess) return nullptr;
+    if ((*err = cudaGetSymbolAddress(&p[1], g_tq_amax)) != cudaSuccess) return nullptr;
+    if ((*err = cudaGetSymbolAddress(&p[2], g_tqf_state)) != cudaSuccess) return nullptr;
+    if ((*err = cudaGetSymbolAddress(&p[3], g_tqf_amax)) != cudaSuccess) return nullptr;
+    if ((*err = cudaGetSymbolAddress(&p[4], g_tqf_tiles)) != cudaSuccess) return nullptr;
+    cache[dev] = TqScratch{static_cast<uint32_t*>(p[0]), static_cast<uint32_t*>(p[1]), static_cast<uint32_t*>(p[2]),
+                           static_cast<uint32_t*>(p[3]), static_cast<uint32_t*>(p[4])};
+    have[dev] = true;
   }
-  *amax_slots = amax_cache[dev];
-  if (tile_slots) *tile_slots = tile_cache[dev];
-  return cache[dev];
+  return &cache[dev];
 }
 
 bool cooperative_ok() {
@@ -1033,14 +1038,12 @@ cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, const f
   if (!fn) return cudaErrorNotSupported;
   if (n > kAmaxRows) return cudaErrorNotSupported;
   cudaError_t e;
-  uint32_t* amax_slots = nullptr;
-  uint32_t* tile_slots = nullptr;
-  uint32_t* slots = sync_slots(&e, &amax_slots, &tile_slots);
-  if (!slots) return e;
+  const TqScratch* sc = tq_scratch(&e);
+  if (!sc) return e;
   const uint32_t slot = next_tq_slot();
-  uint32_t* sync = slots + 4 * slot;
-  uint32_t* amax_bits = amax_slots + (size_t)kAmaxRows * slot;
-  uint32_t* tile_rec = tile_slots + (size_t)kAmaxTiles * kTileWords * slot;
+  uint32_t* state = sc->state + 4 * slot;
+  uint32_t* amax_sets = sc->amax_sets + (size_t)2 * kAmaxRows * slot;
+  uint32_t* rec_sets = sc->rec_sets + (size_t)2 * kAmaxTiles * kTileWords * slot;
   CUtensorMap map;
   memset(&map, 0, sizeof(map));
   cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)n};
@@ -1073,7 +1076,7 @@ cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, const f
   cfg.numAttrs = 1;
   note_launch();
   return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<K>, map, A, planes, (int)n, (int)d,
-                            reinterpret_cast<float*>(amax), words, sync, amax_bits, tile_rec, status);
+                            reinterpret_cast<float*>(amax), words, state, amax_sets, rec_sets, status);
 }
 
 }  // namespace
