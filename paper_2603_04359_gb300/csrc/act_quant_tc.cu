@@ -14,6 +14,7 @@
 //   pass 0: atomicMax of the row maxima into the scale buffer (float bits, non-negative),
 //   pass 1: recompute, q = clamp(round_half_even(7 v' / max), -7, 7) decided exactly, pack SM4x8, store.
 // Warps: 0 TMA producer + TMEM allocator, 1 MMA issuer, 4..7 epilogue, 8..15 converters.
+#include <algorithm>
 #include <atomic>
 #include <cstring>
 #include <mutex>
@@ -38,20 +39,34 @@ struct TcCfg {
   static constexpr uint32_t T_OFF = kXStages * X_STAGE;
   static constexpr uint32_t BAR_OFF = T_OFF + 3 * SPLIT;
   static constexpr size_t SMEM = BAR_OFF + 256 + 1024;
-  // fused kernel: the final row maxima of unit j (128 floats).  At k = 128 a CTA has at most
-  // kXStages units, so unit j's x stage is free once its MMAs are done and holds them; at k = 64
-  // they get their own room after the barriers.
-  static constexpr uint32_t FUSED_BAR_BYTES = 512;
-  static constexpr uint32_t AMAX_DEDICATED = BAR_OFF + FUSED_BAR_BYTES;
-  static constexpr size_t FUSED_SMEM = BAR_OFF + FUSED_BAR_BYTES + (K == 128 ? 0 : (512 / K) * TM * 4) + 1024;
-  __device__ static uint8_t* amax_tile(uint8_t* smem, int j) {
-    return K == 128 ? smem + X_OFF + j * X_STAGE : smem + AMAX_DEDICATED + j * TM * 4;
-  }
   static constexpr uint32_t TMEM_COLS = 2 * K;               // double-buffered accumulator
   // kind::f16: D fp32 (bit 4), A = B = BF16 (format 1 at bits 7 and 10), K-major, M = 128, N = K
   static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(K >> 3) << 17) |
                                     ((uint32_t)(TM >> 4) << 24);
 };
+
+// Shared-memory layout of the fused kernel.  U units' x' tiles are resident in tensor memory at once
+// (their slots); with WAVES a CTA has more units than slots and reuses a slot once the unit in it is
+// quantized.  A slot's final row maxima (128 floats): in a single wave at k = 128 (at most kXStages
+// units) in the unit's x stage, free once its MMAs are done; otherwise in their own room, with one x
+// stage fewer at k = 128 to make room.
+template <int K, bool WAVES>
+struct FusedCfg {
+  using C = TcCfg<K>;
+  static constexpr int U = 512 / K;
+  static constexpr int XS = (WAVES && K == 128) ? kXStages - 1 : kXStages;
+  static constexpr uint32_t X_OFF = 0;
+  static constexpr uint32_t T_OFF = XS * C::X_STAGE;
+  static constexpr uint32_t BAR_OFF = T_OFF + 3 * C::SPLIT;
+  static constexpr uint32_t BAR_BYTES = 512;
+  static constexpr bool AMAX_IN_X = !WAVES && K == 128;
+  static constexpr uint32_t AMAX_OFF = BAR_OFF + BAR_BYTES;
+  static constexpr size_t SMEM = AMAX_OFF + (AMAX_IN_X ? 0 : U * TM * 4) + 1024;
+  __device__ static float* amax_slot(uint8_t* smem, int slot) {
+    return reinterpret_cast<float*>(AMAX_IN_X ? smem + X_OFF + slot * C::X_STAGE : smem + AMAX_OFF + slot * TM * 4);
+  }
+};
+static_assert(FusedCfg<128, false>::SMEM <= 227 * 1024 && FusedCfg<128, true>::SMEM <= 227 * 1024, "shared memory");
 
 struct TcBars {
   uint64_t x_full[kXStages], x_empty[kXStages], d_full[2], d_empty[2], t_full, t_empty, mma_done;
@@ -59,7 +74,7 @@ struct TcBars {
   uint32_t tmem_addr;
   int abort;
 };
-// the barrier block fits the 256 bytes reserved for it (the fused kernel reserves FUSED_BAR_BYTES)
+// the barrier block fits the 256 bytes reserved for it (the fused kernel reserves FusedCfg::BAR_BYTES)
 static_assert(sizeof(TcBars) <= 256, "barrier room");
 
 __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
@@ -560,38 +575,48 @@ __device__ __forceinline__ bool wait_count(const uint32_t* ctr, uint32_t expecte
 // three warps share (slot (c + 1) % 3): the epilogue warp joins when its phase A is done.
 __device__ __forceinline__ int chunk_slot(int c, bool last) { return last ? (c + 1) % 3 : 1 + (c & 1); }
 
-template <int K>
+template <int K, bool WAVES>
 __device__ __forceinline__ void quantize_units(uint32_t tmem, uint8_t* smem, const FusedUnits& fu, int num_tiles,
-                                               int n, int d, uint64_t* maxima_ready, uint32_t* __restrict__ codes,
-                                               volatile int* abort_flag, int slot) {
-  using C = TcCfg<K>;
+                                               int n, int d, uint64_t* maxima_ready, uint64_t* tmem_free,
+                                               uint32_t* __restrict__ codes, volatile int* abort_flag, int slot) {
+  // unit j sits in tensor-memory slot j % U (phase (j / U) & 1 of the slot's barriers); with WAVES the
+  // converter warps (slots 1 and 2) hand the slot back once their chunks of the unit are done
+  using F = FusedCfg<K, WAVES>;
   const int lane = threadIdx.x & 31, quad = (threadIdx.x >> 5) & 3;
   const int64_t words_per_row = d / 8;
   const int nu = fu.count;
   for (int j = 0; j < nu; ++j) {
+    const int us = j % F::U;
+    const uint32_t ph = (uint32_t)(j / F::U) & 1u;
     const bool last = j == nu - 1;
     bool mine = false;
 #pragma unroll
     for (int c = 0; c < K / 32; ++c) mine |= chunk_slot(c, last) == slot;
-    if (!mine) continue;
-    const bool got = !*abort_flag && mbar_wait_bounded(&maxima_ready[j], 0, abort_flag, __LINE__);
-    if (!__all_sync(0xFFFFFFFFu, got)) return;
-    int b, tile;
-    fused_unit(fu, j, num_tiles, &b, &tile);
-    const int t = tile * TM + quad * 32 + lane;
-    const float a = reinterpret_cast<const float*>(C::amax_tile(smem, j))[quad * 32 + lane];
-    const QRow qr = qrow_setup(a, 7.0f);       // inv == 0: zero or non-finite row, all codes 0
-    tc_fence_after();
+    if (mine) {
+      const bool got = !*abort_flag && mbar_wait_bounded(&maxima_ready[us], ph, abort_flag, __LINE__);
+      if (!__all_sync(0xFFFFFFFFu, got)) return;
+      int b, tile;
+      fused_unit(fu, j, num_tiles, &b, &tile);
+      const int t = tile * TM + quad * 32 + lane;
+      const float a = F::amax_slot(smem, us)[quad * 32 + lane];
+      const QRow qr = qrow_setup(a, 7.0f);     // inv == 0: zero or non-finite row, all codes 0
+      tc_fence_after();
 #pragma unroll 1
-    for (int c = 0; c < K / 32; ++c) {
-      if (chunk_slot(c, last) != slot) continue;
-      const uint4 w = quant_chunk(tmem + ((uint32_t)(quad * 32) << 16) + j * K + c * 32, qr);
-      if (t < n) *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * K + c * 32) / 8) = w;
+      for (int c = 0; c < K / 32; ++c) {
+        if (chunk_slot(c, last) != slot) continue;
+        const uint4 w = quant_chunk(tmem + ((uint32_t)(quad * 32) << 16) + us * K + c * 32, qr);
+        if (t < n) *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * K + c * 32) / 8) = w;
+      }
+    }
+    if (WAVES && slot != 0) {                  // the slot's tensor memory (and maxima) are free again
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tmem_free[us]);
     }
   }
 }
 
-template <int K>
+template <int K, bool WAVES>
 __global__ void __launch_bounds__(kThreads, 1)
     transform_quant_tc_fused_kernel(const __grid_constant__ CUtensorMap tmX, const float* __restrict__ A,
                                     const uint8_t* __restrict__ planes, int n, int d, float* __restrict__ scale,
@@ -601,18 +626,21 @@ __global__ void __launch_bounds__(kThreads, 1)
   // state: the slot's epoch, start counter and tiles per set; amax_sets: two sets of kAmaxRows row
   // maxima (float bits); rec_sets: two sets of kAmaxTiles tile records
   using C = TcCfg<K>;
-  constexpr int kMaxUnits = 512 / K;
-  static_assert(sizeof(TcBars) + (3 * kMaxUnits + 4) * sizeof(uint64_t) + 8 <= C::FUSED_BAR_BYTES, "barrier room");
-  static_assert(K != 128 || kMaxUnits <= kXStages, "at k = 128 unit j's x stage holds its maxima");
+  using F = FusedCfg<K, WAVES>;
+  constexpr int U = F::U;                              // tensor-memory slots (units resident at once)
+  static_assert(sizeof(TcBars) + (4 * U + 4) * sizeof(uint64_t) + 8 <= F::BAR_BYTES, "barrier room");
+  static_assert(!F::AMAX_IN_X || U <= F::XS, "in one wave at k = 128 unit j's x stage holds its maxima");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* xs = smem + C::X_OFF;
-  uint8_t* ts = smem + C::T_OFF;
-  TcBars* bars = reinterpret_cast<TcBars*>(smem + C::BAR_OFF);
-  uint64_t* unit_full = reinterpret_cast<uint64_t*>(bars + 1);   // per unit, used once: its MMAs are done
-  uint64_t* epi_done = unit_full + kMaxUnits;                     // per unit, used once: its atomics are issued
-  uint64_t* maxima_ready = epi_done + kMaxUnits;                  // per unit, used once: final maxima in smem
-  uint64_t* plane_full = maxima_ready + kMaxUnits;                // per plane of T_b (producer-fetched planes)
+  uint8_t* xs = smem + F::X_OFF;
+  uint8_t* ts = smem + F::T_OFF;
+  TcBars* bars = reinterpret_cast<TcBars*>(smem + F::BAR_OFF);
+  // per tensor-memory slot (unit j: slot j % U, phase (j / U) & 1)
+  uint64_t* unit_full = reinterpret_cast<uint64_t*>(bars + 1);   // the unit's MMAs are done
+  uint64_t* epi_done = unit_full + U;                             // its row maxima's atomics are issued
+  uint64_t* maxima_ready = epi_done + U;                          // its final maxima are in shared memory
+  uint64_t* tmem_free = maxima_ready + U;                         // WAVES: quantized, the slot is free
+  uint64_t* plane_full = tmem_free + U;                           // per plane of T_b (producer-fetched planes)
   uint64_t* set_ready = plane_full + 3;                           // the launch's scratch set is known
   volatile int* set_sel = reinterpret_cast<int*>(set_ready + 1);  // ... and it is set_sel (0 or 1)
   volatile int* abort_flag = &bars->abort;
@@ -621,7 +649,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int nb = d / K;
   const int num_tiles = (n + TM - 1) / TM;
   FusedUnits fu = fused_units(blockIdx.x, gridDim.x, nb, num_tiles);
-  if (fu.count > kMaxUnits) fu.count = kMaxUnits;      // the launcher guarantees this never cuts
+  if (!WAVES && fu.count > U) fu.count = U;            // the launcher guarantees this never cuts
   const int nu = fu.count;
   // With pre-split planes and one block per CTA, the producer fetches the planes itself, in the order
   // H, (unit 0's x tile), M, L, and unit 0's MMAs start on H while M and L are still on their way.
@@ -632,10 +660,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bars->x_full[st], 1);
       mbar_init(&bars->x_empty[st], 1);
     }
-    for (int j = 0; j < kMaxUnits; ++j) {
+    for (int j = 0; j < U; ++j) {
       mbar_init(&unit_full[j], 1);
       mbar_init(&epi_done[j], 4);                       // the four epilogue warps
       mbar_init(&maxima_ready[j], 1);
+      mbar_init(&tmem_free[j], kCvtWarps);              // the converter warps, after their chunks
     }
     for (int sp = 0; sp < 3; ++sp) mbar_init(&plane_full[sp], 1);
     mbar_init(set_ready, 1);
@@ -668,7 +697,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (; j < nu; ++j) {
         int b, tile;
         fused_unit(fu, j, num_tiles, &b, &tile);
-        const uint32_t st = j % kXStages;
+        const uint32_t st = j % F::XS;
         if (own_planes) {
           // M and L after unit 0's tile; the tiles from unit 2 on after all of T_b is in
           if (j == 2 && !(ok = mbar_wait_bounded(&plane_full[2], 0, abort_flag, __LINE__))) break;
@@ -677,7 +706,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           // memory, so that T_b does not queue behind them and unit 0's MMAs start as early as they can
           if (j == 2 && !(ok = mbar_wait_bounded(&bars->t_first, 0, abort_flag, __LINE__))) break;
         }
-        if (j >= kXStages && !(ok = mbar_wait_bounded(&bars->x_empty[st], ((j / kXStages) - 1) & 1, abort_flag, __LINE__))) break;
+        if (j >= F::XS && !(ok = mbar_wait_bounded(&bars->x_empty[st], ((j / F::XS) - 1) & 1, abort_flag, __LINE__))) break;
         mbar_arrive_expect_tx(&bars->x_full[st], C::X_STAGE);
 #pragma unroll
         for (int a = 0; a < C::ATOMS; ++a)
@@ -690,9 +719,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
-      const int issued = j, first = issued > kXStages ? issued - kXStages : 0;
+      const int issued = j, first = issued > F::XS ? issued - F::XS : 0;
       volatile int no_abort = 0;
-      for (int q = first; q < issued; ++q) mbar_wait_bounded(&bars->x_full[q % kXStages], (q / kXStages) & 1, &no_abort);
+      for (int q = first; q < issued; ++q) mbar_wait_bounded(&bars->x_full[q % F::XS], (q / F::XS) & 1, &no_abort);
       if (own_planes)
         for (int sp = 0; sp < 3; ++sp) mbar_wait_bounded(&plane_full[sp], 0, &no_abort);
       (void)ok;
@@ -712,10 +741,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           ++version;
           cur_b = b;
         }
-        const uint32_t st = j % kXStages;
-        if (!(ok = mbar_wait_bounded(&bars->x_full[st], (j / kXStages) & 1, abort_flag, __LINE__))) break;
+        const uint32_t st = j % F::XS;
+        // WAVES: the unit U back in this slot must be quantized before its columns are overwritten
+        if (WAVES && j >= U && !(ok = mbar_wait_bounded(&tmem_free[j % U], ((j / U) - 1) & 1, abort_flag, __LINE__))) break;
+        if (!(ok = mbar_wait_bounded(&bars->x_full[st], (j / F::XS) & 1, abort_flag, __LINE__))) break;
         tc_fence_after();
-        const uint32_t dcol = tmem + j * K;
+        const uint32_t dcol = tmem + (j % U) * K;
         const uint32_t xbase = smem_u32(xs + st * C::X_STAGE);
         const uint32_t tbase = smem_u32(ts);
 #pragma unroll
@@ -734,7 +765,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (!ok) break;
         mma_commit(&bars->x_empty[st]);
-        mma_commit(&unit_full[j]);
+        mma_commit(&unit_full[j % U]);
         int nb_next = -1, tile_next;
         if (j + 1 < nu) fused_unit(fu, j + 1, num_tiles, &nb_next, &tile_next);
         if (nb_next != b) mma_commit(&bars->t_empty);     // the CTA's last unit of block b
@@ -755,17 +786,20 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       if (lane == 0) ok = wait_count(tile_rec + (size_t)tile * kTileWords, 4u * (uint32_t)nb, abort_flag, __LINE__);
       if (!__shfl_sync(0xFFFFFFFFu, (int)ok, 0)) break;
-      // unit j's MMAs are done (this CTA counted the tile after them): at k = 128 its x stage is free
-      if (!__all_sync(0xFFFFFFFFu, mbar_wait_bounded(&unit_full[j], 0, abort_flag, __LINE__))) break;
-      fence_proxy_async_smem();
+      // unit j's MMAs are done (this CTA counted the tile after them): in one wave at k = 128 its x
+      // stage is free for the maxima
+      if (F::AMAX_IN_X) {
+        if (!__all_sync(0xFFFFFFFFu, mbar_wait_bounded(&unit_full[j], 0, abort_flag, __LINE__))) break;
+        fence_proxy_async_smem();
+      }
       uint32_t v[TM / 32];
 #pragma unroll
       for (int i = 0; i < TM / 32; ++i) v[i] = __ldcg(&amax_bits[tile * TM + 32 * i + lane]);  // < kAmaxRows
-      float* am = reinterpret_cast<float*>(C::amax_tile(smem, j));
+      float* am = F::amax_slot(smem, j % U);
 #pragma unroll
       for (int i = 0; i < TM / 32; ++i) am[32 * i + lane] = __uint_as_float(v[i]);
       __syncwarp();
-      if (lane == 0) mbar_arrive(&maxima_ready[j]);
+      if (lane == 0) mbar_arrive(&maxima_ready[j % U]);
       if (b == 0) {                                      // the CTAs holding block 0 write the steps
 #pragma unroll
         for (int i = 0; i < TM / 32; ++i) {
@@ -821,7 +855,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int j = 0; j < nu; ++j) {
         int b, tile;
         fused_unit(fu, j, num_tiles, &b, &tile);
-        if (!mbar_wait_bounded(&epi_done[j], 0, abort_flag, __LINE__)) break;
+        if (!mbar_wait_bounded(&epi_done[j % U], (j / U) & 1, abort_flag, __LINE__)) break;
         __threadfence();
         atomicAdd(&tile_rec[(size_t)tile * kTileWords], 4u);
       }
@@ -856,7 +890,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         ++version;
       }
     }
-    quantize_units<K>(tmem, smem, fu, num_tiles, n, d, maxima_ready, codes, abort_flag, 1 + ((warp - kCvtWarp0) >> 2));
+    quantize_units<K, WAVES>(tmem, smem, fu, num_tiles, n, d, maxima_ready, tmem_free, codes, abort_flag,
+                             1 + ((warp - kCvtWarp0) >> 2));
     tc_fence_before();
   } else if (warp >= kEpiWarp0) {
     // ---------------------------------------------------------------- phase A: one row per thread
@@ -868,7 +903,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       int b, tile;
       fused_unit(fu, j, num_tiles, &b, &tile);
       const int t = tile * TM + quad * 32 + lane;
-      const bool got = !*abort_flag && mbar_wait_bounded(&unit_full[j], 0, abort_flag, __LINE__);
+      const bool got = !*abort_flag && mbar_wait_bounded(&unit_full[j % U], (j / U) & 1, abort_flag, __LINE__);
       if (!__all_sync(0xFFFFFFFFu, got)) break;        // warp-uniform: TMEM loads need the whole warp
       tc_fence_after();
       uint32_t mb = 0;
@@ -876,8 +911,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int c = 0; c < K / 32; c += 2) {            // two loads in flight
         uint32_t r0[32], r1[32];
         __syncwarp();
-        CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + j * K + c * 32, r0);
-        CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + j * K + (c + 1) * 32, r1);
+        CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + (j % U) * K + c * 32, r0);
+        CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + (j % U) * K + (c + 1) * 32, r1);
         tmem_ld_wait();
         mb = absmax_bits32(r1, absmax_bits32(r0, mb));
       }
@@ -886,10 +921,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       // a non-finite value makes the row's maximum the largest NaN pattern: its codes and step become 0
       if (t < n) atomicMax(&amax_bits[t], row_finite ? mb : 0x7FFFFFFFu);
       __syncwarp();
-      if (lane == 0) mbar_arrive(&epi_done[j]);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&epi_done[j % U]);
     }
     if (!finite) report(status, kStatusNonFinite);
-    quantize_units<K>(tmem, smem, fu, num_tiles, n, d, maxima_ready, codes, abort_flag, 0);
+    quantize_units<K, WAVES>(tmem, smem, fu, num_tiles, n, d, maxima_ready, tmem_free, codes, abort_flag, 0);
     tc_fence_before();
   }
 
@@ -1026,13 +1063,23 @@ bool cooperative_ok() {
 template <int K>
 cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, const float* A, const uint8_t* planes,
                            uint32_t* amax, uint32_t* words, uint32_t* status, cudaStream_t stream) {
-  using C = TcCfg<K>;
   const int nb = (int)(d / K);
   const int tiles = (int)((n + TM - 1) / TM);
   const int64_t units = (int64_t)nb * tiles;
-  const int grid = (int)(units < num_sms() ? units : num_sms());
-  for (int c = 0; c < grid; ++c)  // every CTA's units must fit in tensor memory at once
-    if (fused_units(c, grid, nb, tiles).count > 512 / K) return cudaErrorNotSupported;
+  const int sms = num_sms();
+  // One wave when every CTA's units fit in tensor memory at once; otherwise waves, with the same
+  // number m of CTAs on every block (then a tile sits at the same position t / m in every CTA that
+  // holds it, and no CTA can wait on a tile that another CTA reaches only after a later wave of its
+  // own); beyond one CTA per block the caller takes the two-pass path.
+  int grid = (int)(units < sms ? units : sms);
+  bool waves = false;
+  for (int c = 0; c < grid && !waves; ++c)
+    if (fused_units(c, grid, nb, tiles).count > 512 / K) waves = true;
+  if (waves) {
+    if (nb > sms) return cudaErrorNotSupported;
+    const int m = std::min(sms / nb, tiles);
+    grid = m * nb;
+  }
   if (!cooperative_ok()) return cudaErrorNotSupported;
   EncodeTiledFn fn = encode_fn();
   if (!fn) return cudaErrorNotSupported;
@@ -1057,15 +1104,18 @@ cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, const f
   static std::once_flag once;
   static cudaError_t attr = cudaSuccess;
   std::call_once(once, [] {
-    attr = cudaFuncSetAttribute(transform_quant_tc_fused_kernel<K>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)C::FUSED_SMEM);
+    attr = cudaFuncSetAttribute(transform_quant_tc_fused_kernel<K, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)FusedCfg<K, false>::SMEM);
+    if (attr == cudaSuccess)
+      attr = cudaFuncSetAttribute(transform_quant_tc_fused_kernel<K, true>,
+                                  cudaFuncAttributeMaxDynamicSharedMemorySize, (int)FusedCfg<K, true>::SMEM);
   });
   if (attr != cudaSuccess) return attr;
   cudaLaunchConfig_t cfg;
   memset(&cfg, 0, sizeof(cfg));
   cfg.gridDim = dim3((unsigned)grid, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = C::FUSED_SMEM;
+  cfg.dynamicSmemBytes = waves ? FusedCfg<K, true>::SMEM : FusedCfg<K, false>::SMEM;
   cfg.stream = stream;
   // not a programmatic dependent launch: measured, one cost the c2 step ~4 us (the kernel still
   // releases its dependents early, so a programmatic GEMM launch after it gets going sooner)
@@ -1075,7 +1125,10 @@ cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, const f
   cfg.attrs = attrs;
   cfg.numAttrs = 1;
   note_launch();
-  return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<K>, map, A, planes, (int)n, (int)d,
+  if (waves)
+    return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<K, true>, map, A, planes, (int)n, (int)d,
+                              reinterpret_cast<float*>(amax), words, state, amax_sets, rec_sets, status);
+  return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<K, false>, map, A, planes, (int)n, (int)d,
                             reinterpret_cast<float*>(amax), words, state, amax_sets, rec_sets, status);
 }
 

@@ -88,8 +88,11 @@ def _cat_T(rng, d, k):
 @pytest.mark.parametrize("n,d,k,dtype", [(130, 256, 32, "f32"), (67, 384, 128, "bf16"), (200, 512, 256, "bf16"),
                                          (5, 64, 16, "bf16"), (300, 1024, 64, "f32"), (300, 1024, 64, "bf16"),
                                          (300, 640, 128, "bf16"), (1000, 256, 128, "bf16"),
-                                         # more than four 128-row units per CTA: the two-pass kernel
-                                         (2560, 4096, 128, "bf16"), (1300, 8192, 64, "bf16")])
+                                         # more units per CTA than tensor memory holds: the fused kernel
+                                         # in waves (5 and 11 units per CTA, ragged last tile)
+                                         (2560, 4096, 128, "bf16"), (1300, 8192, 64, "bf16"),
+                                         # more blocks than SMs and more than one wave: the two-pass kernel
+                                         (1100, 10240, 64, "bf16")])
 def test_transform_quantize_act(n, d, k, dtype):
     rng = np.random.default_rng(7 * n + d)
     X = rng.standard_normal((n, d)) * rng.lognormal(0, 1.0, d)
@@ -111,7 +114,8 @@ def test_transform_quantize_act(n, d, k, dtype):
 
 
 @pytest.mark.parametrize("n,d,k,dtype", [(67, 384, 128, "bf16"), (300, 1024, 64, "bf16"), (1000, 256, 128, "bf16"),
-                                         (2560, 4096, 128, "bf16"), (1300, 8192, 64, "bf16"), (130, 256, 32, "f32")])
+                                         (2560, 4096, 128, "bf16"), (1300, 8192, 64, "bf16"),
+                                         (1100, 10240, 64, "bf16"), (130, 256, 32, "f32")])
 def test_transform_with_presplit_planes_is_identical(n, d, k, dtype):
     """T's bf16 planes split once (cat_split_transform) and bulk-copied by the kernels give the same
     codes and steps, bit for bit, as the kernels' own split (fused, two-pass, and the SIMT path that
@@ -140,16 +144,17 @@ def test_nonfinite_activation_reports_numeric():
     assert cat.cat_device_status()[0] == 0  # cleared
 
 
-def test_nonfinite_activation_two_pass():
-    """bf16 rows on the two-pass tensor-core kernel: a row holding inf or NaN gets step 0 and all
-    codes 0, the status reports it, and the other rows are unaffected."""
-    n, d, k = 2560, 4096, 128
+@pytest.mark.parametrize("n,d,k", [(2560, 4096, 128),    # the fused kernel in waves
+                                   (1100, 10240, 64)])   # the two-pass kernel
+def test_nonfinite_activation_many_units(n, d, k):
+    """bf16 rows with more units per CTA than tensor memory holds: a row holding inf or NaN gets step 0
+    and all codes 0, the status reports it, and the other rows are unaffected."""
     rng = np.random.default_rng(11)
     X = rng.standard_normal((n, d))
     Xt = WL.cast(X, "bf16")
     raw = Xt.raw.copy()
     raw[5, 17] = 0x7F80                     # +inf
-    raw[900, 4000] = 0x7FC0                 # NaN
+    raw[900, d - 96] = 0x7FC0               # NaN
     bad = WL.Tensor(values=WL.bf16_bits_to_f32(raw), raw=raw, dtype="bf16")
     T32 = _cat_T(rng, d, k)
     cat.cat_device_status()  # clear
@@ -208,7 +213,8 @@ def _tie_rows(rng, n, d):
 
 
 @pytest.mark.parametrize("n,d,k,dtype", [(300, 512, 64, "bf16"), (1000, 1024, 128, "bf16"),   # fused
-                                         (2560, 4096, 128, "bf16"),                            # two-pass
+                                         (2560, 4096, 128, "bf16"),                            # waves
+                                         (1100, 10240, 64, "bf16"),                            # two-pass
                                          (130, 256, 32, "f32"), (200, 512, 256, "bf16"),       # SIMT
                                          (70, 64, 16, "bf16")])
 def test_code_decision_exact_on_ties(n, d, k, dtype):
