@@ -1,27 +1,28 @@
 // Calibration autocorrelation blocks on tensor cores (bf16 rows; Sec. 4: Sigma_x = E[x x^T], Eq. 10
 // keeps the k x k diagonal blocks):  sigma[b] (+)= sum_t x_{t,b} x_{t,b}^T.
 //
-// D = X_G^T X_G for a group of G = max(k, 128) consecutive channels is one MMA chain contracting
-// over tokens: both operands are the same token-by-channel tile, read MN-major (channels
-// contiguous) straight from the TMA-loaded layout, so nothing is transposed.  bf16 products are
-// exact; tokens accumulate in fp32 in tensor memory.  The tensor cores' fp32 accumulation rounds
-// more coarsely than round-to-nearest, with an error that grows with the number of MMA steps, so
-// for k <= 128 the 16-token MMA steps go round-robin to NACC = 4 accumulators (512 TMEM columns),
-// each summing a quarter of the tokens, and the epilogue adds them (fp32) before widening them to
-// float64 with integer operations (the FP64 pipe of this GPU is ~60x slower than FP32).  The result is
-// within ~1e-6 of a float64 sum, which moves the block transform by ~1e-6 (its square roots damp
-// the calibration error) -- far below the INT4 step.  Only the diagonal k x k blocks are written.
+// A group of G = max(k, 128) consecutive channels is contracted over tokens on tensor cores: both
+// operands are slices of the same token-by-channel tile, read MN-major (channels contiguous) straight
+// from the TMA-loaded layout, so nothing is transposed.  bf16 products are exact; tokens accumulate in
+// fp32 in tensor memory.  The tensor cores' fp32 accumulation rounds more coarsely than
+// round-to-nearest, with an error that grows with the number of MMA steps, so the 16-token MMA steps
+// go round-robin to 4 accumulators (runs of up to 1024 tokens) or 8 (longer runs), and the epilogue
+// adds them (fp32) before widening them to float64 with integer operations (the FP64 pipe of this GPU is
+// ~60x slower than FP32).  The result is within ~1e-6 of a float64 sum, which moves the block
+// transform by ~1e-6 (its square roots damp the calibration error) -- far below the INT4 step.
 //
-// CTA = (channel group, token split).  The token splits of a group form a thread-block cluster of
-// S <= 4 CTAs: each CTA sums its accumulators into an fp32 tile in its own shared memory, and after
-// a cluster barrier CTA r reduces rows [r 128/S, (r+1) 128/S) of the S tiles through distributed
-// shared memory and writes them as coalesced float64 rows.  More splits than one cluster (large
-// token counts) add their clusters' results with float64 atomics.  Since D = X^T X is symmetric,
-// the staged tile is the transpose of the TMEM tile (thread = TMEM row writes one shared-memory
-// column, so the stores are conflict-free) and the written blocks are D^T, equal to D up to the
-// rounding of the accumulation order.
-// Warps: 0 TMA producer + TMEM allocator, 1 MMA issuer, 2..5 epilogue (one TMEM lane quadrant
-// each).  Tokens arrive in 64-row chunks of 64-channel, 128B-swizzled boxes through a 4-stage ring.
+// CTA = (channel group, 128-row half of the group (k = 256), 64-column slice of the group, token
+// split): D = X_rows^T X_cols over its tokens, M = 128, N = 64 (one 128-byte swizzle atom of
+// channels).  No reduction between CTAs: the column slices of a group are separate CTAs, and only
+// long calibration runs split the tokens (their CTAs add their results with float64 atomics).  Only
+// the diagonal k x k blocks are written, and through the symmetry of X^T X: lane r of a warp holds
+// row r of D and writes it as column r of the block, so a warp's stores of one D column are 32
+// consecutive doubles (256 bytes) -- the written blocks are D^T, equal to D up to the rounding of
+// the accumulation order.
+// Warps: 0 TMA producer + TMEM allocator, 1 MMA issuer, 2..9 epilogue (a TMEM lane quadrant and a
+// 32-column half of the slice each).  Tokens arrive in 64-row chunks of 64-channel, 128B-swizzled
+// boxes; with up to kStages chunks in flight, the 512-token calibration split of the configurations
+// is read in one go.
 #include <cstring>
 #include <mutex>
 
@@ -31,28 +32,29 @@ namespace cat {
 namespace {
 
 constexpr int kChunk = 64;      // tokens per stage
-constexpr int kStages = 4;
-constexpr int kThreads = 192;
+constexpr int kStages = 8;      // 512 tokens in flight at once
+constexpr int kThreads = 320;         // producer, MMA issuer, 8 epilogue warps
 constexpr uint32_t kBox = kChunk * 128;  // one 64-token x 64-channel bf16 box, 8 KiB
-constexpr int kMaxCluster = 4;           // token splits reduced on chip
-constexpr uint32_t kRedTile = 128 * 128 * 4;  // fp32 128 x 128 reduction tile (reuses the stage ring)
-static_assert(kStages * 2 * kBox >= kRedTile, "the reduction tile must fit in the stage ring");
+constexpr int NACC = 8;                  // round-robin accumulators: all 512 TMEM columns
+constexpr int kSliceN = 64;              // columns of a CTA's tile: one 128-byte swizzle atom
+constexpr uint32_t kTmemCols = NACC * kSliceN;
 
-template <int G2>  // 128-channel tiles per dimension of a group (1: k <= 128, 2: k = 256)
+template <int G2>  // 128-row halves per group (1: k <= 128, 2: k = 256)
 struct CovCfg {
   static constexpr int G = 128 * G2;
-  static constexpr int BOXES = G / 64;
+  static constexpr int SLICES = G / kSliceN;               // column slices per group
+  static constexpr int CTAS = G2 * SLICES;                 // CTAs per group (per token split)
+  // per stage: the two 64-channel boxes of the CTA's 128 rows (their first holds the column slice
+  // when k <= 128), and at k = 256 the column slice's own box
+  static constexpr int BOXES = G2 == 1 ? 2 : 3;
   static constexpr uint32_t STAGE = BOXES * kBox;
   static constexpr uint32_t BAR_OFF = kStages * STAGE;
-  // more than half of an SM's shared memory: one CTA per SM, so that a CTA waiting at a cluster
-  // barrier never holds tensor memory that a CTA of another cluster on the same SM is waiting for
-  static constexpr size_t SMEM = (BAR_OFF + 256 + 1024) > 120 * 1024 ? (BAR_OFF + 256 + 1024) : 120 * 1024;
-  static constexpr int NACC = G2 == 1 ? 4 : 1;              // round-robin accumulators per tile
-  static constexpr uint32_t TMEM_COLS = G2 * G2 * 128 * NACC;
-  // kind::f16, D fp32, A = B = BF16, both MN-major (bits 15, 16), M = N = 128
+  static constexpr size_t SMEM = BAR_OFF + 256 + 1024;
+  // kind::f16, D fp32, A = B = BF16, both MN-major (bits 15, 16), M = 128, N = 64
   static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) | (1u << 16) |
-                                    ((uint32_t)(128 >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+                                    ((uint32_t)(kSliceN >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
 };
+static_assert(CovCfg<2>::SMEM <= 227 * 1024, "shared memory budget");
 
 struct CovBars {
   uint64_t full[kStages], empty[kStages], acc_full, mma_done;
@@ -89,32 +91,20 @@ __device__ __forceinline__ double f32_to_f64_exact(float f) {
   return __longlong_as_double((long long)bits);
 }
 
-__device__ __forceinline__ uint32_t cluster_ctarank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
+
+// The same widening on its common route: a normal float re-biases its exponent by 1023 - 127 = 896
+// (exponent and mantissa shift right by 3 into the high word, the mantissa's low 3 bits go to the
+// top of the low word) and a zero keeps its sign -- a few integer operations, no branch.  Subnormals,
+// inf and nan (`rare`) must take the exact function above.
+__device__ __forceinline__ bool f32_widen_rare(float f) {
+  const uint32_t u = __float_as_uint(f), e = u & 0x7F800000u;
+  return (u & 0x7FFFFFFFu) != 0u && (e == 0u || e == 0x7F800000u);
 }
-__device__ __forceinline__ uint32_t cluster_nctarank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
-  return r;
-}
-// all threads of all CTAs of the cluster; release / acquire orders the shared-memory tiles
-__device__ __forceinline__ void cluster_sync_all() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-__device__ __forceinline__ uint32_t map_cluster(uint32_t saddr, uint32_t rank) {
-  uint32_t r;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
-  return r;
-}
-__device__ __forceinline__ float4 ld_cluster_f32x4(uint32_t caddr) {
-  float4 v;
-  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
-               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-               : "r"(caddr)
-               : "memory");
-  return v;
+__device__ __forceinline__ double f32_to_f64_fast(float f) {
+  const uint32_t u = __float_as_uint(f);
+  const uint32_t mag = u & 0x7FFFFFFFu;
+  const uint32_t hi = (u & 0x80000000u) | (mag == 0u ? 0u : (mag >> 3) + (896u << 20));
+  return __hiloint2double((int)hi, (int)(u << 29));
 }
 
 __device__ __forceinline__ void mma_bf16_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
@@ -137,11 +127,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   CovBars* bars = reinterpret_cast<CovBars*>(smem + C::BAR_OFF);
   volatile int* abort_flag = &bars->abort;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int c0 = blockIdx.x * C::G;
+  const int g = blockIdx.x / C::CTAS;                 // channel group
+  const int ih = (blockIdx.x % C::CTAS) / C::SLICES;  // its 128-row half (k = 256)
+  const int h = blockIdx.x % C::SLICES;               // its 64-column slice
+  const int c0 = g * C::G;                            // first channel of the group
   const int t_begin = blockIdx.y * tok_per_split;
   const int t_end = min(n, t_begin + tok_per_split);
   const int chunks = (t_end - t_begin + kChunk - 1) / kChunk;
   const int total_steps = chunks * (kChunk / 16);
+  // accumulators in use: 4 (16 MMA steps each at most) for short runs, 8 beyond -- fewer
+  // accumulators are fewer tensor-memory reads in the epilogue, more keep each one's sum short
+  const int nacc = total_steps > 4 * 16 ? NACC : NACC / 2;
+  // the column slice's box within a stage: one of the row boxes, or its own (k = 256, other half)
+  const int b_box = G2 == 1 ? h : ((h >> 1) == ih ? (h & 1) : 2);
 
   if (tid == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -155,7 +153,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   __syncwarp();
   pdl_wait_then_release();                        // nothing global or in tensor memory before this
-  if (warp == 0) tmem_alloc(&bars->tmem_addr, C::TMEM_COLS);
+  if (warp == 0) tmem_alloc(&bars->tmem_addr, kTmemCols);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -170,8 +168,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t s = c % kStages;
         if (c >= kStages && !(ok = mbar_wait_bounded(&bars->empty[s], ((c / kStages) - 1) & 1, abort_flag, __LINE__))) break;
         mbar_arrive_expect_tx(&bars->full[s], C::STAGE);
-        for (int bx = 0; bx < C::BOXES; ++bx)
-          tma_load_2d(smem + s * C::STAGE + bx * kBox, &tmX, c0 + 64 * bx, t_begin + c * kChunk, &bars->full[s]);
+        const int t0 = t_begin + c * kChunk;
+        for (int bx = 0; bx < 2; ++bx)            // the CTA's 128 rows
+          tma_load_2d(smem + s * C::STAGE + bx * kBox, &tmX, c0 + ih * 128 + 64 * bx, t0, &bars->full[s]);
+        if (G2 == 2)                              // the column slice's box
+          tma_load_2d(smem + s * C::STAGE + 2 * kBox, &tmX, c0 + kSliceN * h, t0, &bars->full[s]);
       }
       const int first = c > kStages ? c - kStages : 0;
       volatile int no_abort = 0;
@@ -188,15 +189,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int kk = 0; kk < kChunk / 16; ++kk) {  // 16 tokens per MMA: 16 rows of 128 B
           const int step = c * (kChunk / 16) + kk;
-          const int acc = step % C::NACC;            // accumulator of this 16-token step
-#pragma unroll
-          for (int ih = 0; ih < G2; ++ih)
-#pragma unroll
-            for (int jh = 0; jh < G2; ++jh) {
-              const uint64_t da = sdesc_mnmajor_sw128(base + 2 * ih * kBox + kk * 2048, kBox);
-              const uint64_t db = sdesc_mnmajor_sw128(base + 2 * jh * kBox + kk * 2048, kBox);
-              mma_bf16_ss(tmem + ((acc * G2 + ih) * G2 + jh) * 128, da, db, C::IDESC, step >= C::NACC);
-            }
+          const uint64_t da = sdesc_mnmajor_sw128(base + kk * 2048, kBox);
+          const uint64_t db = sdesc_mnmajor_sw128(base + b_box * kBox + kk * 2048, kBox);
+          mma_bf16_ss(tmem + (step % nacc) * kSliceN, da, db, C::IDESC, step >= nacc);
         }
         mma_commit(&bars->empty[s]);
       }
@@ -205,134 +200,86 @@ __global__ void __launch_bounds__(kThreads, 1)
       volatile int no_abort = 0;
       mbar_wait_bounded(&bars->mma_done, 0, &no_abort);
     }
+  } else {
+    // ---------------------------------------------------------------- epilogue: one tile row per lane
+    const int quad = warp & 3;                        // the TMEM lane quadrant this warp may access
+    const int lk = 31 - __clz(k);                     // k = 2^lk
+    const int rg = ih * 128 + quad * 32 + lane;       // this lane's row within the group
+    const bool live = chunks > 0 && mbar_wait_bounded(&bars->acc_full, 0, abort_flag, __LINE__);
+    const int used = total_steps < nacc ? total_steps : nacc;   // accumulators written
+    if (__all_sync(0xFFFFFFFFu, live)) {              // warp-uniform: TMEM loads need the whole warp
+      tc_fence_after();
+      {
+        const int cc = (warp - 2) >> 2;               // this warp's 32-column chunk of the slice
+        const int cg0 = kSliceN * h + 32 * cc;        // first column (within the group) of this chunk
+        // the chunk's columns share a diagonal block with some lane's row
+        const bool need = (rg / k) * k < cg0 + 32 && cg0 < (rg / k + 1) * k;
+        if (__any_sync(0xFFFFFFFFu, need)) {
+        float v[32];
+#pragma unroll
+        for (int e = 0; e < 32; ++e) v[e] = 0.f;
+#pragma unroll 1
+        for (int a = 0; a < used; a += 2) {           // two accumulators per tensor-memory round trip
+          uint32_t rr[32], rq[32];
+          __syncwarp();
+          CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + a * kSliceN + 32 * cc, rr);
+          if (a + 1 < used) CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + (a + 1) * kSliceN + 32 * cc, rq);
+          tmem_ld_wait();
+#pragma unroll
+          for (int e = 0; e < 32; ++e) v[e] += __uint_as_float(rr[e]);
+          if (a + 1 < used) {
+#pragma unroll
+            for (int e = 0; e < 32; ++e) v[e] += __uint_as_float(rq[e]);
+          }
+        }
+        // D[rg][cg] = sigma entry (cg, rg) of their block (the symmetry): for each column the lanes
+        // of a block write consecutive doubles.  k is a power of two (shifts, no divisions), and the
+        // store mode is chosen once per chunk: inside the element loop the compiler would turn the
+        // read-modify-write of `add` (an FP64 add and a global load per element) into work every
+        // element pays for.
+        const int row = c0 + rg;
+        double* rowbase = sigma + ((int64_t)(row >> lk) << (2 * lk)) + (row & (k - 1));
+        const int rblk = rg >> lk;
+        uint32_t ok_mask = 0u;                        // columns of the chunk this lane writes
+        bool rare = false;
+        double w[32];
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          const int cg = cg0 + e;
+          if ((cg >> lk) == rblk && row < d && c0 + cg < d) ok_mask |= 1u << e;
+          rare |= f32_widen_rare(v[e]);
+          w[e] = f32_to_f64_fast(v[e]);
+        }
+        if (__any_sync(0xFFFFFFFFu, rare)) {         // a subnormal, inf or nan in the warp's chunk
+#pragma unroll
+          for (int e = 0; e < 32; ++e) w[e] = f32_to_f64_exact(v[e]);
+        }
+        // entry (col % k, row % k) of the block sits (col % k) k doubles after its row's base
+        const int cbase = (c0 + cg0) & (k - 1);
+        if (mode == 0) {
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (ok_mask >> e & 1u) rowbase[(int64_t)((cbase + e) & (k - 1)) << lk] = w[e];
+        } else if (mode == 1) {
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (ok_mask >> e & 1u) rowbase[(int64_t)((cbase + e) & (k - 1)) << lk] += w[e];
+        } else {
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (ok_mask >> e & 1u) atomicAdd(rowbase + ((int64_t)((cbase + e) & (k - 1)) << lk), w[e]);
+        }
+        }
+      }
+    }
+    tc_fence_before();
   }
 
-  // ---- reduction over the cluster's token splits and the float64 store ---------------------
   __syncthreads();
-  const bool epi = warp >= 2;
-  const int ew = warp - 2;                            // epilogue warp 0..3
-  const int quad = warp & 3;                          // the TMEM lane quadrant this warp may access
-  const uint32_t S = cluster_nctarank();
-  const uint32_t rank = cluster_ctarank();
-  const bool have_acc = chunks > 0 && !bars->abort;
-  if (epi && have_acc) {
-    if (!mbar_wait_bounded(&bars->acc_full, 0, abort_flag, __LINE__)) {
-      // gave up: the tile below is not written; the status word reports it
-    }
-    __syncwarp();
-    tc_fence_after();
-  }
-  float* red = reinterpret_cast<float*>(smem);        // the stage ring is idle once acc_full fired
-  const int used = total_steps < C::NACC ? total_steps : C::NACC;  // accumulators written
-  const int kw = G2 == 2 ? 128 : k;                   // needed columns per row within a tile
-#pragma unroll 1
-  for (int ih = 0; ih < G2; ++ih)
-#pragma unroll 1
-    for (int jh = 0; jh < G2; ++jh) {
-      if (epi) {
-        // phase 1: this CTA's partial tile, summed over its accumulators, stored transposed
-        const int r = quad * 32 + lane;               // TMEM lane = tile row
-        const int cw = kw < 32 ? 32 : kw;             // columns a warp's 32 rows need
-        const int col0 = G2 == 2 ? 0 : ((quad * 32) / cw) * cw;
-        const bool live = have_acc && !__any_sync(0xFFFFFFFFu, *abort_flag);  // warp-uniform
-#pragma unroll 1
-        for (int cc = 0; cc < cw / 32; ++cc) {
-          const int col = col0 + 32 * cc;
-          float v32[32];
-#pragma unroll
-          for (int e = 0; e < 32; ++e) v32[e] = 0.f;
-          if (live) {
-#pragma unroll 1
-            for (int a = 0; a < used; a += 2) {      // two accumulators per tensor-memory round trip
-              uint32_t rr[32], rq[32];
-              __syncwarp();
-              CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + ((a * G2 + ih) * G2 + jh) * 128 + col, rr);
-              if (a + 1 < used)
-                CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + (((a + 1) * G2 + ih) * G2 + jh) * 128 + col, rq);
-              tmem_ld_wait();
-#pragma unroll
-              for (int e = 0; e < 32; ++e) v32[e] += __uint_as_float(rr[e]);
-              if (a + 1 < used) {
-#pragma unroll
-                for (int e = 0; e < 32; ++e) v32[e] += __uint_as_float(rq[e]);
-              }
-            }
-          }
-#pragma unroll
-          for (int e = 0; e < 32; ++e) red[(col + e) * 128 + r] = v32[e];
-        }
-      }
-      __syncwarp();
-      tc_fence_before();
-      cluster_sync_all();                             // every CTA's tile is written
-      if (epi) {
-        // phase 2: rows [rank 128/S, (rank+1) 128/S) of the S tiles; lanes_per_row lanes cover a
-        // row's kw needed columns 4 at a time
-        const int rows = 128 / (int)S;
-        const int r_lo = (int)rank * rows;
-        const int lpr = kw / 4 < 32 ? kw / 4 : 32;
-        const int rpp = 32 / lpr;                     // rows per warp pass
-        const int sub = lane / lpr, l4 = lane % lpr;
-        const uint32_t red_addr = smem_u32(red);
-        // kRowsInFlight rows per round: all their remote loads (S per row and 4-column group) are in
-        // flight before the first sum (remote shared-memory loads are slow); the sums run in a fixed
-        // source order, so they are deterministic
-        constexpr int kRowsInFlight = 4;
-#pragma unroll 1
-        for (int R0 = r_lo + ew * rpp + sub; R0 < r_lo + rows; R0 += kRowsInFlight * 4 * rpp) {
-#pragma unroll 1
-          for (int C4i = 4 * l4; C4i < kw; C4i += 4 * lpr) {
-            float4 part[kRowsInFlight][kMaxCluster];
-#pragma unroll
-            for (int q = 0; q < kRowsInFlight; ++q) {
-              const int R = R0 + q * 4 * rpp;
-              const int cb = G2 == 2 ? 0 : (R / k) * k;   // first column of R's diagonal block in the tile
-              const uint32_t off = red_addr + (uint32_t)(R * 128 + cb + C4i) * 4u;
-#pragma unroll
-              for (int src = 0; src < kMaxCluster; ++src)
-                part[q][src] = (R < r_lo + rows && (uint32_t)src < S) ? ld_cluster_f32x4(map_cluster(off, (uint32_t)src))
-                                                                       : make_float4(0.f, 0.f, 0.f, 0.f);
-            }
-#pragma unroll
-            for (int q = 0; q < kRowsInFlight; ++q) {
-              const int R = R0 + q * 4 * rpp;
-              if (R >= r_lo + rows) break;
-              const int cb = G2 == 2 ? 0 : (R / k) * k;
-              const int C4 = cb + C4i;
-              float4 acc = part[q][0];
-#pragma unroll
-              for (int src = 1; src < kMaxCluster; ++src)
-                if ((uint32_t)src < S) {
-                  acc.x += part[q][src].x; acc.y += part[q][src].y; acc.z += part[q][src].z; acc.w += part[q][src].w;
-                }
-              // staged tile (ih, jh) is transposed: entry (R, C) belongs to group row jh*128 + R
-              const int grow = c0 + jh * 128 + R;
-              if (grow >= d) continue;
-              double* dst = sigma + (int64_t)grow * k + ((ih * 128 + C4) % k);
-              const double v[4] = {f32_to_f64_exact(acc.x), f32_to_f64_exact(acc.y), f32_to_f64_exact(acc.z),
-                                   f32_to_f64_exact(acc.w)};
-              if (mode == 2) {
-#pragma unroll
-                for (int e = 0; e < 4; ++e) atomicAdd(dst + e, v[e]);
-              } else if (mode == 1) {
-#pragma unroll
-                for (int e = 0; e < 4; ++e) dst[e] += v[e];
-              } else {
-                reinterpret_cast<double2*>(dst)[0] = make_double2(v[0], v[1]);
-                reinterpret_cast<double2*>(dst)[1] = make_double2(v[2], v[3]);
-              }
-            }
-          }
-        }
-      }
-      __syncwarp();
-      cluster_sync_all();                             // the tiles may be overwritten / released
-    }
-
   if (bars->abort && tid == 0) report(status, timeout_bits(kWhereCalib, bars->abort));
   if (warp == 0) {
     tc_fence_after();
-    tmem_dealloc(tmem, C::TMEM_COLS);
+    tmem_dealloc(tmem, kTmemCols);
   }
 }
 
@@ -385,15 +332,12 @@ cudaError_t launch_g(const void* x, int64_t n, int64_t d, int k, double* sigma, 
   const int64_t groups = (d + C::G - 1) / C::G;
   const int64_t chunks = (n + kChunk - 1) / kChunk;
   const int sms = num_sms();
-  // S token splits per group reduced on chip (a cluster), while the grid stays within one wave
-  int S = 1;
-  while (S < kMaxCluster && groups * S * 2 <= sms && chunks >= S * 2) S *= 2;
-  // more clusters per group (float64 atomics) only for long calibration runs: >= 2048 tokens per CTA
-  const int64_t per_cta = (chunks + S - 1) / S;
-  int64_t ysplits = (sms + groups * S - 1) / (groups * S);
-  if (ysplits > per_cta / 32) ysplits = per_cta / 32;
+  // token splits (their CTAs add with float64 atomics) only for long calibration runs: >= 2048 tokens
+  // per CTA, within one wave
+  int64_t ysplits = sms / (groups * C::CTAS);
+  if (ysplits > chunks / 32) ysplits = chunks / 32;
   if (ysplits < 1) ysplits = 1;
-  const int64_t tps = ((chunks + S * ysplits - 1) / (S * ysplits)) * kChunk;
+  const int64_t tps = ((chunks + ysplits - 1) / ysplits) * kChunk;
   int mode = accumulate ? 1 : 0;
   if (ysplits > 1) {
     mode = 2;
@@ -404,19 +348,12 @@ cudaError_t launch_g(const void* x, int64_t n, int64_t d, int k, double* sigma, 
   }
   cudaLaunchConfig_t cfg;
   memset(&cfg, 0, sizeof(cfg));
-  cfg.gridDim = dim3((unsigned)groups, (unsigned)(S * ysplits), 1);
+  cfg.gridDim = dim3((unsigned)(groups * C::CTAS), (unsigned)ysplits, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = C::SMEM;
   cfg.stream = stream;
   // not a programmatic dependent launch: measured, one gained ~0.4 us per c4 step and lost ~0.7 us per
   // c2 step (the kernel still releases its dependents early)
-  cudaLaunchAttribute attr_cluster[1];
-  attr_cluster[0].id = cudaLaunchAttributeClusterDimension;
-  attr_cluster[0].val.clusterDim.x = 1;
-  attr_cluster[0].val.clusterDim.y = (unsigned)S;
-  attr_cluster[0].val.clusterDim.z = 1;
-  cfg.attrs = attr_cluster;
-  cfg.numAttrs = 1;
   note_launch();
   cudaError_t e = cudaLaunchKernelEx(&cfg, calib_cov_tc_kernel<G2>, map, (int)n, (int)d, k, (int)tps, sigma, mode,
                                      status);
