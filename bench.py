@@ -303,7 +303,9 @@ class BufferSet:
         self.x, self.xc, self.y_ref = x.clone(), xc.clone(), y_ref.clone()
         self.T, self.Wq, self.sw = T.clone(), Wq.clone(), sw.clone()
         # T's bf16 planes, split once per layer (the tensor-core transform's k = 64, 128)
-        self.T_planes = cat.cat_split_transform(self.T, k) if (k in (64, 128) and x.dtype == torch.bfloat16) else None
+        self.T_planes = (cat.cat_split_transform(self.T, k)
+                         if (x.dtype == torch.bfloat16 and cat.cat_split_transform_bytes(self.T.shape[0] * k, k) > 0)
+                         else None)
         self.sigma = torch.empty((d_in // k, k, k), dtype=torch.float64, device=dev)
         self.xq = torch.empty((n, d_in // 2), dtype=torch.uint8, device=dev)
         self.sx = torch.empty((n,), dtype=torch.float32, device=dev)

@@ -186,19 +186,30 @@ cat_status cat_transform_quantize_act(const void* x, cat_dtype dtype, int64_t n,
                                       cat_stream_t stream);
 
 /*
- * cat_split_transform -- T_blocks [d_in/k][k][k] float32 into the three bf16 planes of every block,
- * T_b = H + M + L with H = bf16(T_b), M = bf16(T_b - H), L = bf16(T_b - H - M) (24 significant bits:
- * the tensor-core transform's fp32-accurate products), laid out exactly as that kernel's shared-memory
- * operand (K-major, 128-byte swizzle).  planes: device, 6 * d_in * k bytes.  k = 64 or 128 (the
- * tensor-core transform's block sizes; CAT_ERR_UNSUPPORTED otherwise).  Run once per layer after
- * weight preparation; no counterpart in the paper (a layout of T).
+ * cat_split_transform_bytes -- the size of cat_split_transform's planes for d_in channels and block
+ * size k: 6 * d_in * K bytes, K the width of the tensor-core transform's channel groups (128 when
+ * 128 divides d_in and k <= 128; 64 for k = 64 otherwise); 0 when no tensor-core transform applies
+ * (k = 256, or a shape the arguments do not allow).  No device access.
+ */
+int64_t cat_split_transform_bytes(int64_t d_in, int32_t k);
+
+/*
+ * cat_split_transform -- T_blocks [d_in/k][k][k] float32 into the three bf16 planes of every K-wide
+ * channel group (K as in cat_split_transform_bytes; a group holds K/k blocks of the block-diagonal T
+ * on its diagonal and zeros elsewhere), T = H + M + L with H = bf16(T), M = bf16(T - H),
+ * L = bf16(T - H - M) (24 significant bits: the tensor-core transform's fp32-accurate products),
+ * laid out exactly as that kernel's shared-memory operand (K-major, 128-byte swizzle).
+ *   planes: device, cat_split_transform_bytes(d_in, k) bytes.
+ * CAT_ERR_UNSUPPORTED when that size is 0.  Run once per layer after weight preparation; no
+ * counterpart in the paper (a layout of T).
  */
 cat_status cat_split_transform(const float* T_blocks, int64_t d_in, int32_t k, uint8_t* planes, cat_stream_t stream);
 
 /*
  * cat_transform_quantize_act_split -- cat_transform_quantize_act with T's pre-split planes
- * (cat_split_transform; may be NULL): on the tensor-core path (bf16 rows, k = 64 or 128) each CTA
- * fetches its block's planes with three bulk copies instead of splitting T_b itself.  Same results.
+ * (cat_split_transform; may be NULL): on the tensor-core path (bf16 rows, cat_split_transform_bytes
+ * nonzero) each CTA fetches its group's planes with three bulk copies instead of splitting them
+ * itself.  Same results.
  */
 cat_status cat_transform_quantize_act_split(const void* x, cat_dtype dtype, int64_t n, int64_t d_in, int32_t k,
                                             const float* T_blocks, const uint8_t* T_planes, uint8_t* xq, float* x_scale,

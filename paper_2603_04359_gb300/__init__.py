@@ -23,7 +23,7 @@ __all__ = [
     "cat_dp_planes", "cat_transform_quantize_act_dp", "cat_quantize_weights_dp", "cat_linear_dp",
     "cat_block_transform", "cat_dequantize_codes", "cat_gemm_f32", "one_sided_sqnr", "cat_set_wait_limit_ns",
     "cat_transform_quantize_act_hd", "cat_fwht_rows", "cat_gram_f32", "cat_alignment_ceiling_host",
-    "cat_split_transform", "cat_transform_quantize_act_split",
+    "cat_split_transform", "cat_split_transform_bytes", "cat_transform_quantize_act_split",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -78,6 +78,7 @@ def load_library() -> ctypes.CDLL:
         "cat_gemm_f32": ([P, P, I64, I64, I64, P, P], I),
         "cat_transform_quantize_act_hd": ([P, I, I64, I64, I32, P, P, P, P], I),
         "cat_split_transform": ([P, I64, I32, P, P], I),
+        "cat_split_transform_bytes": ([I64, I32], I64),
         "cat_transform_quantize_act_split": ([P, I, I64, I64, I32, P, P, P, P, P], I),
         "cat_fwht_rows": ([P, I64, I64, P], I),
         "cat_gram_f32": ([P, I, I64, I64, P, P], I),
@@ -98,7 +99,7 @@ def exported_symbols() -> list:
     """Names of the entry points declared in ``include/cat_w4a4.h``."""
     with open(_HEADER) as f:
         text = f.read()
-    return sorted(set(re.findall(r"^\s*(?:cat_status|const char\*|int|int32_t|unsigned long long)\s+(cat_\w+)\s*\(", text,
+    return sorted(set(re.findall(r"^\s*(?:cat_status|const char\*|int|int32_t|int64_t|unsigned long long)\s+(cat_\w+)\s*\(", text,
                                  re.M)))
 
 
@@ -261,12 +262,21 @@ def _linear_args(xq, x_scale, Wq, w_scale, y) -> None:
     _expect(y, "y", torch.float32, (n, d_out), dev)
 
 
+def cat_split_transform_bytes(d_in: int, k: int) -> int:
+    """Bytes of cat_split_transform's planes (0: no tensor-core transform for this d_in and k)."""
+    return int(load_library().cat_split_transform_bytes(d_in, k))
+
+
 def cat_split_transform(T_blocks: torch.Tensor, k: int) -> torch.Tensor:
-    """T's three bf16 planes per block in the tensor-core transform's layout: uint8 [d_in * k * 6]."""
+    """T's three bf16 planes per channel group in the tensor-core transform's layout: uint8
+    [cat_split_transform_bytes(d_in, k)]."""
     nb = T_blocks.shape[0]
     d_in = nb * k
     _expect(T_blocks, "T_blocks", torch.float32, (nb, k, k), T_blocks.device)
-    planes = torch.empty((6 * d_in * k,), dtype=torch.uint8, device=T_blocks.device)
+    nbytes = cat_split_transform_bytes(d_in, k)
+    if nbytes <= 0:
+        raise CatError("cat_split_transform", 5, f"no tensor-core transform for d_in = {d_in}, k = {k}")
+    planes = torch.empty((nbytes,), dtype=torch.uint8, device=T_blocks.device)
     _check("cat_split_transform", load_library().cat_split_transform(_ptr(T_blocks), d_in, k, _ptr(planes),
                                                                      _stream(T_blocks.device)))
     return planes
@@ -284,7 +294,7 @@ def cat_transform_quantize_act_split(x: torch.Tensor, T_blocks: torch.Tensor, T_
         x_scale = torch.empty((n,), dtype=torch.float32, device=x.device)
     _expect(T_blocks, "T_blocks", torch.float32, (d_in // k, k, k), x.device)
     if T_planes is not None:
-        _expect(T_planes, "T_planes", torch.uint8, (6 * d_in * k,), x.device)
+        _expect(T_planes, "T_planes", torch.uint8, (cat_split_transform_bytes(d_in, k),), x.device)
     _expect(xq, "xq", torch.uint8, (n, d_in // 2), x.device)
     _expect(x_scale, "x_scale", torch.float32, (n,), x.device)
     _check("cat_transform_quantize_act_split", load_library().cat_transform_quantize_act_split(

@@ -153,20 +153,28 @@ __device__ __forceinline__ uint32_t bf16x2_bits(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
-// Split the fp32 block A_b (row-major k x k, row i = output i) into bf16 H, M, L in the MMA's
-// 128B-swizzled K-major layout; `ct` is the thread's index among the converter threads.
+// Split the fp32 K x K group matrix into bf16 H, M, L in the MMA's 128B-swizzled K-major layout;
+// `ct` is the thread's index among the converter threads.  The group matrix is block-diagonal with
+// kb x kb blocks (kb divides K; kb = K: one block): Ab points to the group's K rows in the [rows][kb]
+// layout of the blocks (row i = output i), and entry (i, j) is Ab[i][j % kb] when i and j lie in the
+// same block, 0 otherwise.  A block-diagonal T thus runs on the K-wide kernels exactly: the zeros
+// add exact zeros to the fp32 sums.
 template <int K>
-__device__ __forceinline__ void split_block(const float* __restrict__ Ab, uint8_t* ts, int ct) {
+__device__ __forceinline__ void split_block(const float* __restrict__ Ab, int kb, uint8_t* ts, int ct) {
   using C = TcCfg<K>;
   // all loads first (the block is read from L2/HBM once per block change: keep them in flight together)
   constexpr int kIt = K * K / 8 / (kCvtWarps * 32);
   float4 pv[kIt], qv[kIt];
 #pragma unroll
-  for (int it = 0; it < kIt; ++it) {  // 8 consecutive inputs of one output row per item
+  for (int it = 0; it < kIt; ++it) {  // 8 consecutive inputs of one output row per item (kb >= 16)
     const int ch = ct + it * kCvtWarps * 32;
     const int i = ch / (K / 8), j0 = (ch % (K / 8)) * 8;
-    pv[it] = __ldg(reinterpret_cast<const float4*>(Ab + (size_t)i * K + j0));
-    qv[it] = __ldg(reinterpret_cast<const float4*>(Ab + (size_t)i * K + j0 + 4));
+    if (i / kb == j0 / kb) {
+      pv[it] = __ldg(reinterpret_cast<const float4*>(Ab + (size_t)i * kb + (j0 % kb)));
+      qv[it] = __ldg(reinterpret_cast<const float4*>(Ab + (size_t)i * kb + (j0 % kb) + 4));
+    } else {
+      pv[it] = qv[it] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
   }
 #pragma unroll
   for (int it = 0; it < kIt; ++it) {
@@ -210,10 +218,11 @@ __device__ __forceinline__ void fetch_planes(const uint8_t* __restrict__ planes,
   for (int sp = 0; sp < 3; ++sp) bulk_copy_g2s(ts + sp * C::SPLIT, src + sp * C::SPLIT, C::SPLIT, bar);
 }
 
-// The three bf16 planes of every block, in the MMA's shared-memory layout (cat_split_transform).
+// The three bf16 planes of every K-wide group, in the MMA's shared-memory layout (cat_split_transform).
 template <int K>
-__global__ void __launch_bounds__(kCvtWarps * 32) split_planes_kernel(const float* __restrict__ A, uint8_t* __restrict__ planes) {
-  split_block<K>(A + (size_t)blockIdx.x * K * K, planes + (size_t)blockIdx.x * 3 * TcCfg<K>::SPLIT, threadIdx.x);
+__global__ void __launch_bounds__(kCvtWarps * 32)
+    split_planes_kernel(const float* __restrict__ A, int kb, uint8_t* __restrict__ planes) {
+  split_block<K>(A + (size_t)blockIdx.x * K * kb, kb, planes + (size_t)blockIdx.x * 3 * TcCfg<K>::SPLIT, threadIdx.x);
 }
 
 // Four two's-complement bytes in [-7, 7] -> the SM4x8 sign-magnitude bytes (sign << 7 | magnitude).
@@ -303,7 +312,7 @@ __device__ __forceinline__ uint32_t absmax_bits32(const uint32_t (&r)[32], uint3
 template <int K, int PASS>
 __global__ void __launch_bounds__(kThreads, 1)
     transform_quant_tc_kernel(const __grid_constant__ CUtensorMap tmX, const float* __restrict__ A,
-                              const uint8_t* __restrict__ planes, int n, int d, uint32_t* __restrict__ amax_bits,
+                              const uint8_t* __restrict__ planes, int n, int d, int kb, uint32_t* __restrict__ amax_bits,
                               uint32_t* __restrict__ codes, float* __restrict__ scale, uint32_t* __restrict__ exit_ctr,
                               uint32_t* __restrict__ status) {
   // scale != nullptr (pass 1 with the maxima in a scratch slot): the CTAs holding block 0 write the
@@ -423,7 +432,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (version == 0) mbar_arrive(&bars->t_first);
         }
       } else {
-        split_block<K>(A + (size_t)b * K * K, ts, ct);
+        split_block<K>(A + (size_t)b * K * kb, kb, ts, ct);
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) {
@@ -619,7 +628,7 @@ __device__ __forceinline__ void quantize_units(uint32_t tmem, uint8_t* smem, con
 template <int K, bool WAVES>
 __global__ void __launch_bounds__(kThreads, 1)
     transform_quant_tc_fused_kernel(const __grid_constant__ CUtensorMap tmX, const float* __restrict__ A,
-                                    const uint8_t* __restrict__ planes, int n, int d, float* __restrict__ scale,
+                                    const uint8_t* __restrict__ planes, int n, int d, int kb, float* __restrict__ scale,
                                     uint32_t* __restrict__ codes, uint32_t* __restrict__ state,
                                     uint32_t* __restrict__ amax_sets, uint32_t* __restrict__ rec_sets,
                                     uint32_t* __restrict__ status) {
@@ -879,7 +888,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (version == 0) mbar_arrive(&bars->t_first);
           }
         } else {
-          split_block<K>(A + (size_t)b * K * K, ts, ct);
+          split_block<K>(A + (size_t)b * K * kb, kb, ts, ct);
           fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) {
@@ -983,8 +992,8 @@ uint32_t next_tq_slot() {
 // the steps and returns the slot to zero (no memset, no finalize launch); cudaErrorNotSupported
 // otherwise, when the caller zeroes `amax` (its scale buffer) and finalizes the steps itself.
 template <int K>
-cudaError_t launch_k(const __nv_bfloat16* x, int64_t n, int64_t d, const float* A, const uint8_t* planes, uint32_t* amax,
-                     uint32_t* words, float* scale, uint32_t* status, cudaStream_t stream) {
+cudaError_t launch_k(const __nv_bfloat16* x, int64_t n, int64_t d, int kb, const float* A, const uint8_t* planes,
+                     uint32_t* amax, uint32_t* words, float* scale, uint32_t* status, cudaStream_t stream) {
   using C = TcCfg<K>;
   EncodeTiledFn fn = encode_fn();
   if (!fn) return cudaErrorNotSupported;
@@ -1020,11 +1029,11 @@ cudaError_t launch_k(const __nv_bfloat16* x, int64_t n, int64_t d, const float* 
     amax = sc->amax + (size_t)kAmaxRows * slot;
   }
   note_launch();
-  k0<<<grid, kThreads, C::SMEM, stream>>>(map, A, planes, (int)n, (int)d, amax, words, nullptr, nullptr, status);
+  k0<<<grid, kThreads, C::SMEM, stream>>>(map, A, planes, (int)n, (int)d, kb, amax, words, nullptr, nullptr, status);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   note_launch();
-  k1<<<grid, kThreads, C::SMEM, stream>>>(map, A, planes, (int)n, (int)d, amax, words, scale, exit_ctr, status);
+  k1<<<grid, kThreads, C::SMEM, stream>>>(map, A, planes, (int)n, (int)d, kb, amax, words, scale, exit_ctr, status);
   return cudaGetLastError();
 }
 
@@ -1061,7 +1070,7 @@ bool cooperative_ok() {
 }
 
 template <int K>
-cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, const float* A, const uint8_t* planes,
+cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, int kb, const float* A, const uint8_t* planes,
                            uint32_t* amax, uint32_t* words, uint32_t* status, cudaStream_t stream) {
   const int nb = (int)(d / K);
   const int tiles = (int)((n + TM - 1) / TM);
@@ -1126,16 +1135,27 @@ cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, const f
   cfg.numAttrs = 1;
   note_launch();
   if (waves)
-    return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<K, true>, map, A, planes, (int)n, (int)d,
+    return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<K, true>, map, A, planes, (int)n, (int)d, kb,
                               reinterpret_cast<float*>(amax), words, state, amax_sets, rec_sets, status);
-  return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<K, false>, map, A, planes, (int)n, (int)d,
+  return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<K, false>, map, A, planes, (int)n, (int)d, kb,
                             reinterpret_cast<float*>(amax), words, state, amax_sets, rec_sets, status);
 }
 
 }  // namespace
 
+// The K-wide kernel that runs blocks of size k on d channels: 128 when 128 divides d (a k < 128
+// runs block-diagonal inside each 128-channel group: twice to eight times the MMAs of a k-wide
+// kernel, but the 128-wide kernels are the faster ones, e.g. c5 at k = 64: 64 against 87 us), 64
+// for k = 64 otherwise, 0 when no tensor-core kernel applies (k = 256: three bf16 planes of a
+// 256 x 256 block do not fit in shared memory beside the x tiles).
+int transform_tc_group(int k, int64_t d) {
+  if ((k == 16 || k == 32 || k == 64 || k == 128) && d % 128 == 0) return 128;
+  if (k == 64 && d % 64 == 0) return 64;
+  return 0;
+}
+
 bool transform_quantize_tc_supported(int dtype, int k, int64_t n, int64_t d) {
-  return dtype == 1 && (k == 64 || k == 128) && n <= 0x7FFFFFFF && d <= 0x7FFFFFFF;
+  return dtype == 1 && transform_tc_group(k, d) != 0 && n <= 0x7FFFFFFF && d <= 0x7FFFFFFF;
 }
 
 // Passes 0 and 1; the caller zeroes the scale buffer before and finalizes it after.
@@ -1143,19 +1163,21 @@ cudaError_t launch_transform_quantize_tc(const void* x, int64_t n, int64_t d, in
                                          const uint8_t* planes, uint32_t* amax, uint32_t* words, float* scale,
                                          uint32_t* status, cudaStream_t stream) {
   const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
-  if (k == 64) return launch_k<64>(xb, n, d, A, planes, amax, words, scale, status, stream);
-  if (k == 128) return launch_k<128>(xb, n, d, A, planes, amax, words, scale, status, stream);
+  const int K = transform_tc_group(k, d);
+  if (K == 64) return launch_k<64>(xb, n, d, k, A, planes, amax, words, scale, status, stream);
+  if (K == 128) return launch_k<128>(xb, n, d, k, A, planes, amax, words, scale, status, stream);
   return cudaErrorInvalidValue;
 }
 
-// T_blocks -> the three bf16 planes of every block in the transform kernels' shared-memory layout
-// ([d/k][3][k*k] bf16, 6 d k bytes); k = 64 or 128.
+// T_blocks -> the three bf16 planes of every K-wide group (K = transform_tc_group(k, d)) in the
+// transform kernels' shared-memory layout ([d/K][3][K*K] bf16, 6 d K bytes).
 cudaError_t launch_split_transform(const float* A, int64_t d, int k, uint8_t* planes, cudaStream_t stream) {
-  const unsigned nb = (unsigned)(d / k);
+  const int K = transform_tc_group(k, d);
+  if (K == 0) return cudaErrorNotSupported;
+  const unsigned groups = (unsigned)(d / K);
   note_launch();
-  if (k == 64) split_planes_kernel<64><<<nb, kCvtWarps * 32, 0, stream>>>(A, planes);
-  else if (k == 128) split_planes_kernel<128><<<nb, kCvtWarps * 32, 0, stream>>>(A, planes);
-  else return cudaErrorNotSupported;
+  if (K == 64) split_planes_kernel<64><<<groups, kCvtWarps * 32, 0, stream>>>(A, k, planes);
+  else split_planes_kernel<128><<<groups, kCvtWarps * 32, 0, stream>>>(A, k, planes);
   return cudaGetLastError();
 }
 
@@ -1169,8 +1191,9 @@ cudaError_t launch_transform_quantize_tc_fused(const void* x, int64_t n, int64_t
                                                const uint8_t* planes, uint32_t* amax, uint32_t* words,
                                                uint32_t* status, cudaStream_t stream) {
   const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
-  if (k == 64) return launch_fused_k<64>(xb, n, d, A, planes, amax, words, status, stream);
-  if (k == 128) return launch_fused_k<128>(xb, n, d, A, planes, amax, words, status, stream);
+  const int K = transform_tc_group(k, d);
+  if (K == 64) return launch_fused_k<64>(xb, n, d, k, A, planes, amax, words, status, stream);
+  if (K == 128) return launch_fused_k<128>(xb, n, d, k, A, planes, amax, words, status, stream);
   return cudaErrorNotSupported;
 }
 }  // namespace cat

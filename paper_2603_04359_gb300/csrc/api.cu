@@ -551,11 +551,17 @@ cat_status cat_transform_quantize_act(const void* x, cat_dtype dtype, int64_t n,
   return ok();
 }
 
+int64_t cat_split_transform_bytes(int64_t d_in, int32_t k) {
+  if (d_in <= 0 || !valid_k(k) || d_in % k != 0) return 0;
+  return 6 * d_in * (int64_t)cat::transform_tc_group(k, d_in);
+}
+
 cat_status cat_split_transform(const float* T_blocks, int64_t d_in, int32_t k, uint8_t* planes, cat_stream_t stream) {
   cat_status st = check_din(d_in);
   if (st != CAT_OK) return st;
   if (!valid_k(k) || d_in % k != 0) return fail(CAT_ERR_SHAPE, "k must be one of 16..256 (power of two) and divide d_in");
-  if (k != 64 && k != 128) return fail(CAT_ERR_UNSUPPORTED, "pre-split planes serve the tensor-core transform: k = 64 or 128");
+  if (cat::transform_tc_group(k, d_in) == 0)
+    return fail(CAT_ERR_UNSUPPORTED, "pre-split planes serve the tensor-core transform: k <= 128 with 128 | d_in, or k = 64");
   if (!T_blocks || !planes) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
   if (!aligned16(T_blocks) || !aligned16(planes)) return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
   if ((st = check_device()) != CAT_OK) return st;
@@ -582,7 +588,7 @@ cat_status cat_transform_quantize_act_split(const void* x, cat_dtype dtype, int6
   uint32_t* status = status_word(&e);
   if (!status) return cuda_fail(e, "status word");
   e = cat::launch_transform_quantize(x, (int)dtype, n, d_in, k, T_blocks, xq, x_scale, status, (cudaStream_t)stream,
-                                     (k == 64 || k == 128) ? T_planes : nullptr);
+                                     cat::transform_tc_group(k, d_in) != 0 ? T_planes : nullptr);
   if (e != cudaSuccess) return cuda_fail(e, "cat_transform_quantize_act_split launch");
   return ok();
 }

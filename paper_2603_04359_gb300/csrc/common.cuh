@@ -302,6 +302,9 @@ cudaError_t launch_transform_quantize(const void* x, int dtype, int64_t n, int64
                                       uint8_t* codes, float* scale, uint32_t* status, cudaStream_t stream,
                                       const uint8_t* planes = nullptr);
 cudaError_t launch_split_transform(const float* T, int64_t d, int k, uint8_t* planes, cudaStream_t stream);
+// the group width K of the tensor-core transform for block size k on d channels (0: none applies);
+// the pre-split planes take 6 d K bytes
+int transform_tc_group(int k, int64_t d);
 cudaError_t launch_w4a4_gemm(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
                              int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, uint32_t* status,
                              cudaStream_t stream);

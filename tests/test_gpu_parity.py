@@ -91,8 +91,13 @@ def _cat_T(rng, d, k):
                                          # more units per CTA than tensor memory holds: the fused kernel
                                          # in waves (5 and 11 units per CTA, ragged last tile)
                                          (2560, 4096, 128, "bf16"), (1300, 8192, 64, "bf16"),
-                                         # more blocks than SMs and more than one wave: the two-pass kernel
-                                         (1100, 10240, 64, "bf16")])
+                                         # k < 128 block-diagonal inside 128-channel groups (one wave, waves)
+                                         (300, 512, 32, "bf16"), (130, 384, 16, "bf16"), (2560, 4096, 32, "bf16"),
+                                         (1100, 10240, 64, "bf16"),
+                                         # 64 | d but not 128: the 64-wide kernels (one wave, two passes)
+                                         (300, 192, 64, "bf16"), (1100, 9920, 64, "bf16"),
+                                         # more groups than SMs and more than one wave: two passes
+                                         (520, 20480, 128, "bf16")])
 def test_transform_quantize_act(n, d, k, dtype):
     rng = np.random.default_rng(7 * n + d)
     X = rng.standard_normal((n, d)) * rng.lognormal(0, 1.0, d)
@@ -115,7 +120,8 @@ def test_transform_quantize_act(n, d, k, dtype):
 
 @pytest.mark.parametrize("n,d,k,dtype", [(67, 384, 128, "bf16"), (300, 1024, 64, "bf16"), (1000, 256, 128, "bf16"),
                                          (2560, 4096, 128, "bf16"), (1300, 8192, 64, "bf16"),
-                                         (1100, 10240, 64, "bf16"), (130, 256, 32, "f32")])
+                                         (300, 512, 32, "bf16"), (130, 384, 16, "bf16"), (300, 192, 64, "bf16"),
+                                         (1100, 9920, 64, "bf16"), (130, 256, 32, "f32")])
 def test_transform_with_presplit_planes_is_identical(n, d, k, dtype):
     """T's bf16 planes split once (cat_split_transform) and bulk-copied by the kernels give the same
     codes and steps, bit for bit, as the kernels' own split (fused, two-pass, and the SIMT path that
@@ -123,7 +129,7 @@ def test_transform_with_presplit_planes_is_identical(n, d, k, dtype):
     rng = np.random.default_rng(5 * n + d)
     X = WL.cast(rng.standard_normal((n, d)) * rng.lognormal(0, 1.0, d), dtype)
     T32 = torch.from_numpy(_cat_T(rng, d, k)).to(DEV)
-    planes = cat.cat_split_transform(T32, k) if k in (64, 128) else None
+    planes = cat.cat_split_transform(T32, k) if (dtype == "bf16" and cat.cat_split_transform_bytes(d, k) > 0) else None
     xq0, sx0 = cat.cat_transform_quantize_act(to_dev(X), T32, k)
     xq1, sx1 = cat.cat_transform_quantize_act_split(to_dev(X), T32, planes, k)
     assert torch.equal(xq0, xq1) and torch.equal(sx0, sx1)
@@ -145,7 +151,8 @@ def test_nonfinite_activation_reports_numeric():
 
 
 @pytest.mark.parametrize("n,d,k", [(2560, 4096, 128),    # the fused kernel in waves
-                                   (1100, 10240, 64)])   # the two-pass kernel
+                                   (1100, 9920, 64),     # the two-pass kernel (64-wide)
+                                   (2560, 4096, 32)])    # waves, k = 32 block-diagonal in 128-channel groups
 def test_nonfinite_activation_many_units(n, d, k):
     """bf16 rows with more units per CTA than tensor memory holds: a row holding inf or NaN gets step 0
     and all codes 0, the status reports it, and the other rows are unaffected."""
@@ -214,7 +221,8 @@ def _tie_rows(rng, n, d):
 
 @pytest.mark.parametrize("n,d,k,dtype", [(300, 512, 64, "bf16"), (1000, 1024, 128, "bf16"),   # fused
                                          (2560, 4096, 128, "bf16"),                            # waves
-                                         (1100, 10240, 64, "bf16"),                            # two-pass
+                                         (1100, 9920, 64, "bf16"),                             # two-pass
+                                         (300, 512, 32, "bf16"),                               # k = 32 in groups
                                          (130, 256, 32, "f32"), (200, 512, 256, "bf16"),       # SIMT
                                          (70, 64, 16, "bf16")])
 def test_code_decision_exact_on_ties(n, d, k, dtype):
