@@ -191,18 +191,22 @@ cudaError_t launch_transform_quantize(const void* x, int dtype, int64_t n, int64
     const cudaError_t ef = launch_transform_quantize_tc_fused(x, n, d, k, A, planes, amax,
                                                               reinterpret_cast<uint32_t*>(codes), status, stream);
     if (ef != cudaErrorNotSupported) return ef;  // done (or failed) in one launch
-    // two passes with the maxima in device scratch: pass 1 writes the steps
-    const cudaError_t es = launch_transform_quantize_tc(x, n, d, k, A, planes, nullptr,
-                                                        reinterpret_cast<uint32_t*>(codes), scale, status, stream);
-    if (es != cudaErrorNotSupported) return es;
-    // more rows than the scratch holds: the maxima in the scale buffer, then a finalize launch
-    cudaError_t e = cudaMemsetAsync(scale, 0, (size_t)n * sizeof(float), stream);
-    if (e == cudaSuccess) e = launch_transform_quantize_tc(x, n, d, k, A, planes, amax,
-                                                           reinterpret_cast<uint32_t*>(codes), nullptr, status, stream);
-    if (e != cudaSuccess) return e;
-    note_launch();
-    finalize_scale_kernel<<<(unsigned)((n + 255) / 256), 256, 0, stream>>>(amax, n, status);
-    return cudaGetLastError();
+    if (k != 256) {                               // k = 256 has the fused kernel only
+      // two passes with the maxima in device scratch: pass 1 writes the steps
+      const cudaError_t es = launch_transform_quantize_tc(x, n, d, k, A, planes, nullptr,
+                                                          reinterpret_cast<uint32_t*>(codes), scale, status, stream);
+      if (es != cudaErrorNotSupported) return es;
+      // more rows than the scratch holds: the maxima in the scale buffer, then a finalize launch
+      cudaError_t e = cudaMemsetAsync(scale, 0, (size_t)n * sizeof(float), stream);
+      if (e == cudaSuccess) e = launch_transform_quantize_tc(x, n, d, k, A, planes, amax,
+                                                             reinterpret_cast<uint32_t*>(codes), nullptr, status, stream);
+      if (e != cudaSuccess) return e;
+      note_launch();
+      finalize_scale_kernel<<<(unsigned)((n + 255) / 256), 256, 0, stream>>>(amax, n, status);
+      return cudaGetLastError();
+    }
+    // k = 256 beyond the fused kernel (more 64-output groups than SMs, more rows than its scratch):
+    // the SIMT kernel below
   }
   if (dtype == 0) return launch_t(static_cast<const float*>(x), n, d, k, A, codes, scale, status, stream);
   return launch_t(static_cast<const __nv_bfloat16*>(x), n, d, k, A, codes, scale, status, stream);

@@ -45,28 +45,41 @@ struct TcCfg {
                                     ((uint32_t)(TM >> 4) << 24);
 };
 
-// Shared-memory layout of the fused kernel.  U units' x' tiles are resident in tensor memory at once
-// (their slots); with WAVES a CTA has more units than slots and reuses a slot once the unit in it is
-// quantized.  A slot's final row maxima (128 floats): in a single wave at k = 128 (at most kXStages
-// units) in the unit's x stage, free once its MMAs are done; otherwise in their own room, with one x
-// stage fewer at k = 128 to make room.
-template <int K, bool WAVES>
+// Shared-memory layout of the fused kernel.  A unit is (group of N output channels, 128-row tile);
+// the group's block has KD input channels (N = KD = 128 or 64; N = 64, KD = 256 for 256-blocks, whose
+// three bf16 planes would not fit whole: a group is a quarter of the block's outputs).  An x stage
+// holds 128 rows x min(KD, 128) channels; a unit takes XH = KD / 128 stages (1 below 256).  U units'
+// x' tiles are resident in tensor memory at once (their slots, N columns each); with WAVES a CTA has
+// more units than slots and reuses a slot once the unit in it is quantized.  A slot's final row
+// maxima (128 floats): in a single wave at N = KD = 128 (at most kXStages units) in the unit's x
+// stage, free once its MMAs are done; otherwise in their own room, with one x stage fewer at 128 in
+// waves, and three at KD = 256, to make room.
+template <int N, int KD, bool WAVES>
 struct FusedCfg {
-  using C = TcCfg<K>;
-  static constexpr int U = 512 / K;
-  static constexpr int XS = (WAVES && K == 128) ? kXStages - 1 : kXStages;
+  static constexpr int U = 512 / N;
+  static constexpr int XH = KD > 128 ? KD / 128 : 1;
+  static constexpr int XW = KD > 128 ? 128 : KD;
+  static constexpr int XATOMS = XW / 64;                     // 128-byte channel atoms of an x stage
+  static constexpr uint32_t X_STAGE = TM * XW * 2;
+  static constexpr int XS = KD > 128 ? 3 : ((WAVES && N == 128) ? kXStages - 1 : kXStages);
+  static constexpr uint32_t SPLIT = N * KD * 2;              // one bf16 plane of a group
   static constexpr uint32_t X_OFF = 0;
-  static constexpr uint32_t T_OFF = XS * C::X_STAGE;
-  static constexpr uint32_t BAR_OFF = T_OFF + 3 * C::SPLIT;
+  static constexpr uint32_t T_OFF = XS * X_STAGE;
+  static constexpr uint32_t BAR_OFF = T_OFF + 3 * SPLIT;
   static constexpr uint32_t BAR_BYTES = 512;
-  static constexpr bool AMAX_IN_X = !WAVES && K == 128;
+  static constexpr bool AMAX_IN_X = !WAVES && N == 128 && KD == 128;
   static constexpr uint32_t AMAX_OFF = BAR_OFF + BAR_BYTES;
   static constexpr size_t SMEM = AMAX_OFF + (AMAX_IN_X ? 0 : U * TM * 4) + 1024;
+  // kind::f16: D fp32 (bit 4), A = B = BF16 (format 1 at bits 7 and 10), K-major, M = 128, N
+  static constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) |
+                                    ((uint32_t)(TM >> 4) << 24);
   __device__ static float* amax_slot(uint8_t* smem, int slot) {
-    return reinterpret_cast<float*>(AMAX_IN_X ? smem + X_OFF + slot * C::X_STAGE : smem + AMAX_OFF + slot * TM * 4);
+    return reinterpret_cast<float*>(AMAX_IN_X ? smem + X_OFF + slot * X_STAGE : smem + AMAX_OFF + slot * TM * 4);
   }
 };
-static_assert(FusedCfg<128, false>::SMEM <= 227 * 1024 && FusedCfg<128, true>::SMEM <= 227 * 1024, "shared memory");
+static_assert(FusedCfg<128, 128, false>::SMEM <= 227 * 1024 && FusedCfg<128, 128, true>::SMEM <= 227 * 1024 &&
+                  FusedCfg<64, 256, true>::SMEM <= 227 * 1024,
+              "shared memory");
 
 struct TcBars {
   uint64_t x_full[kXStages], x_empty[kXStages], d_full[2], d_empty[2], t_full, t_empty, mma_done;
@@ -159,16 +172,17 @@ __device__ __forceinline__ uint32_t bf16x2_bits(float lo, float hi) {
 // layout of the blocks (row i = output i), and entry (i, j) is Ab[i][j % kb] when i and j lie in the
 // same block, 0 otherwise.  A block-diagonal T thus runs on the K-wide kernels exactly: the zeros
 // add exact zeros to the fp32 sums.
-template <int K>
+template <int N, int KD>
 __device__ __forceinline__ void split_block(const float* __restrict__ Ab, int kb, uint8_t* ts, int ct) {
-  using C = TcCfg<K>;
+  constexpr uint32_t kSplit = N * KD * 2;                     // one plane
+  static_assert((N * KD / 8) % (kCvtWarps * 32) == 0, "converter items must divide evenly");
   // all loads first (the block is read from L2/HBM once per block change: keep them in flight together)
-  constexpr int kIt = K * K / 8 / (kCvtWarps * 32);
+  constexpr int kIt = N * KD / 8 / (kCvtWarps * 32);
   float4 pv[kIt], qv[kIt];
 #pragma unroll
   for (int it = 0; it < kIt; ++it) {  // 8 consecutive inputs of one output row per item (kb >= 16)
     const int ch = ct + it * kCvtWarps * 32;
-    const int i = ch / (K / 8), j0 = (ch % (K / 8)) * 8;
+    const int i = ch / (KD / 8), j0 = (ch % (KD / 8)) * 8;
     if (i / kb == j0 / kb) {
       pv[it] = __ldg(reinterpret_cast<const float4*>(Ab + (size_t)i * kb + (j0 % kb)));
       qv[it] = __ldg(reinterpret_cast<const float4*>(Ab + (size_t)i * kb + (j0 % kb) + 4));
@@ -179,7 +193,7 @@ __device__ __forceinline__ void split_block(const float* __restrict__ Ab, int kb
 #pragma unroll
   for (int it = 0; it < kIt; ++it) {
     const int ch = ct + it * kCvtWarps * 32;
-    const int i = ch / (K / 8), j0 = (ch % (K / 8)) * 8;
+    const int i = ch / (KD / 8), j0 = (ch % (KD / 8)) * 8;
     const float4 p = pv[it], q = qv[it];
     const float v[8] = {p.x, p.y, p.z, p.w, q.x, q.y, q.z, q.w};
     uint32_t hw[4], mw[4], lw[4];
@@ -194,10 +208,10 @@ __device__ __forceinline__ void split_block(const float* __restrict__ Ab, int kb
       lw[e] = bf16x2_bits(r0 - m0, r1 - m1);
     }
     const int atom = j0 / 64, chunk = (j0 % 64) / 8;
-    const uint32_t off = atom * (K * 128) + i * 128 + ((chunk ^ (i & 7)) << 4);
+    const uint32_t off = atom * (N * 128) + i * 128 + ((chunk ^ (i & 7)) << 4);
     *reinterpret_cast<uint4*>(ts + off) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-    *reinterpret_cast<uint4*>(ts + C::SPLIT + off) = make_uint4(mw[0], mw[1], mw[2], mw[3]);
-    *reinterpret_cast<uint4*>(ts + 2 * C::SPLIT + off) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+    *reinterpret_cast<uint4*>(ts + kSplit + off) = make_uint4(mw[0], mw[1], mw[2], mw[3]);
+    *reinterpret_cast<uint4*>(ts + 2 * kSplit + off) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
   }
 }
 
@@ -209,20 +223,21 @@ __device__ __forceinline__ void bulk_copy_g2s(void* dst, const void* src, uint32
                "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
                : "memory");
 }
-template <int K>
-__device__ __forceinline__ void fetch_planes(const uint8_t* __restrict__ planes, int b, uint8_t* ts, uint64_t* bar) {
-  using C = TcCfg<K>;
-  mbar_arrive_expect_tx(bar, 3 * C::SPLIT);
-  const uint8_t* src = planes + (size_t)b * 3 * C::SPLIT;
+template <int N, int KD>
+__device__ __forceinline__ void fetch_planes(const uint8_t* __restrict__ planes, int g, uint8_t* ts, uint64_t* bar) {
+  constexpr uint32_t kSplit = N * KD * 2;
+  mbar_arrive_expect_tx(bar, 3 * kSplit);
+  const uint8_t* src = planes + (size_t)g * 3 * kSplit;
 #pragma unroll
-  for (int sp = 0; sp < 3; ++sp) bulk_copy_g2s(ts + sp * C::SPLIT, src + sp * C::SPLIT, C::SPLIT, bar);
+  for (int sp = 0; sp < 3; ++sp) bulk_copy_g2s(ts + sp * kSplit, src + sp * kSplit, kSplit, bar);
 }
 
-// The three bf16 planes of every K-wide group, in the MMA's shared-memory layout (cat_split_transform).
-template <int K>
+// The three bf16 planes of every group (N outputs x KD inputs), in the MMA's shared-memory layout
+// (cat_split_transform).
+template <int N, int KD>
 __global__ void __launch_bounds__(kCvtWarps * 32)
     split_planes_kernel(const float* __restrict__ A, int kb, uint8_t* __restrict__ planes) {
-  split_block<K>(A + (size_t)blockIdx.x * K * kb, kb, planes + (size_t)blockIdx.x * 3 * TcCfg<K>::SPLIT, threadIdx.x);
+  split_block<N, KD>(A + (size_t)blockIdx.x * N * kb, kb, planes + (size_t)blockIdx.x * 3 * N * KD * 2, threadIdx.x);
 }
 
 // Four two's-complement bytes in [-7, 7] -> the SM4x8 sign-magnitude bytes (sign << 7 | magnitude).
@@ -428,11 +443,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       cur_b = b;
       if (planes) {                                    // one thread copies the pre-split planes
         if (ct == 0) {
-          fetch_planes<K>(planes, b, ts, &bars->t_full);
+          fetch_planes<K, K>(planes, b, ts, &bars->t_full);
           if (version == 0) mbar_arrive(&bars->t_first);
         }
       } else {
-        split_block<K>(A + (size_t)b * K * kb, kb, ts, ct);
+        split_block<K, K>(A + (size_t)b * K * kb, kb, ts, ct);
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) {
@@ -584,13 +599,13 @@ __device__ __forceinline__ bool wait_count(const uint32_t* ctr, uint32_t expecte
 // three warps share (slot (c + 1) % 3): the epilogue warp joins when its phase A is done.
 __device__ __forceinline__ int chunk_slot(int c, bool last) { return last ? (c + 1) % 3 : 1 + (c & 1); }
 
-template <int K, bool WAVES>
+template <int N, int KD, bool WAVES>
 __device__ __forceinline__ void quantize_units(uint32_t tmem, uint8_t* smem, const FusedUnits& fu, int num_tiles,
                                                int n, int d, uint64_t* maxima_ready, uint64_t* tmem_free,
                                                uint32_t* __restrict__ codes, volatile int* abort_flag, int slot) {
   // unit j sits in tensor-memory slot j % U (phase (j / U) & 1 of the slot's barriers); with WAVES the
   // converter warps (slots 1 and 2) hand the slot back once their chunks of the unit are done
-  using F = FusedCfg<K, WAVES>;
+  using F = FusedCfg<N, KD, WAVES>;
   const int lane = threadIdx.x & 31, quad = (threadIdx.x >> 5) & 3;
   const int64_t words_per_row = d / 8;
   const int nu = fu.count;
@@ -600,7 +615,7 @@ __device__ __forceinline__ void quantize_units(uint32_t tmem, uint8_t* smem, con
     const bool last = j == nu - 1;
     bool mine = false;
 #pragma unroll
-    for (int c = 0; c < K / 32; ++c) mine |= chunk_slot(c, last) == slot;
+    for (int c = 0; c < N / 32; ++c) mine |= chunk_slot(c, last) == slot;
     if (mine) {
       const bool got = !*abort_flag && mbar_wait_bounded(&maxima_ready[us], ph, abort_flag, __LINE__);
       if (!__all_sync(0xFFFFFFFFu, got)) return;
@@ -611,10 +626,10 @@ __device__ __forceinline__ void quantize_units(uint32_t tmem, uint8_t* smem, con
       const QRow qr = qrow_setup(a, 7.0f);     // inv == 0: zero or non-finite row, all codes 0
       tc_fence_after();
 #pragma unroll 1
-      for (int c = 0; c < K / 32; ++c) {
+      for (int c = 0; c < N / 32; ++c) {
         if (chunk_slot(c, last) != slot) continue;
-        const uint4 w = quant_chunk(tmem + ((uint32_t)(quad * 32) << 16) + us * K + c * 32, qr);
-        if (t < n) *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * K + c * 32) / 8) = w;
+        const uint4 w = quant_chunk(tmem + ((uint32_t)(quad * 32) << 16) + us * N + c * 32, qr);
+        if (t < n) *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * N + c * 32) / 8) = w;
       }
     }
     if (WAVES && slot != 0) {                  // the slot's tensor memory (and maxima) are free again
@@ -625,7 +640,7 @@ __device__ __forceinline__ void quantize_units(uint32_t tmem, uint8_t* smem, con
   }
 }
 
-template <int K, bool WAVES>
+template <int N, int KD, bool WAVES>
 __global__ void __launch_bounds__(kThreads, 1)
     transform_quant_tc_fused_kernel(const __grid_constant__ CUtensorMap tmX, const float* __restrict__ A,
                                     const uint8_t* __restrict__ planes, int n, int d, int kb, float* __restrict__ scale,
@@ -634,8 +649,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                     uint32_t* __restrict__ status) {
   // state: the slot's epoch, start counter and tiles per set; amax_sets: two sets of kAmaxRows row
   // maxima (float bits); rec_sets: two sets of kAmaxTiles tile records
-  using C = TcCfg<K>;
-  using F = FusedCfg<K, WAVES>;
+  using F = FusedCfg<N, KD, WAVES>;
   constexpr int U = F::U;                              // tensor-memory slots (units resident at once)
   static_assert(sizeof(TcBars) + (4 * U + 4) * sizeof(uint64_t) + 8 <= F::BAR_BYTES, "barrier room");
   static_assert(!F::AMAX_IN_X || U <= F::XS, "in one wave at k = 128 unit j's x stage holds its maxima");
@@ -655,7 +669,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int* abort_flag = &bars->abort;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int nb = d / K;
+  const int nb = d / N;                                // groups of N output channels
   const int num_tiles = (n + TM - 1) / TM;
   FusedUnits fu = fused_units(blockIdx.x, gridDim.x, nb, num_tiles);
   if (!WAVES && fu.count > U) fu.count = U;            // the launcher guarantees this never cuts
@@ -697,46 +711,50 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       prefetch_tensormap(&tmX);
       bool ok = true;
-      int j = 0;
-      const uint8_t* src = own_planes ? planes + (size_t)fu.b * 3 * C::SPLIT : nullptr;
+      const uint8_t* src = own_planes ? planes + (size_t)fu.b * 3 * F::SPLIT : nullptr;
       if (own_planes) {
-        mbar_arrive_expect_tx(&plane_full[0], C::SPLIT);
-        bulk_copy_g2s(ts, src, C::SPLIT, &plane_full[0]);
+        mbar_arrive_expect_tx(&plane_full[0], F::SPLIT);
+        bulk_copy_g2s(ts, src, F::SPLIT, &plane_full[0]);
       }
-      for (; j < nu; ++j) {
-        int b, tile;
-        fused_unit(fu, j, num_tiles, &b, &tile);
-        const uint32_t st = j % F::XS;
+      // stage q = j XH + h: half h of unit j's x tile (the whole tile below KD = 256)
+      int q = 0;
+      const int nq = nu * F::XH;
+      for (; q < nq; ++q) {
+        const int j = q / F::XH, h = q % F::XH;
+        int g, tile;
+        fused_unit(fu, j, num_tiles, &g, &tile);
+        const int in0 = (g * N / KD) * KD + h * F::XW;   // first input channel of this stage
+        const uint32_t st = q % F::XS;
         if (own_planes) {
-          // M and L after unit 0's tile; the tiles from unit 2 on after all of T_b is in
-          if (j == 2 && !(ok = mbar_wait_bounded(&plane_full[2], 0, abort_flag, __LINE__))) break;
+          // M and L after the first stage; the stages from the third on after all of T's planes are in
+          if (q == 2 && !(ok = mbar_wait_bounded(&plane_full[2], 0, abort_flag, __LINE__))) break;
         } else {
-          // the first two units' x tiles go out with T_b's loads; the others wait until T_b is in shared
-          // memory, so that T_b does not queue behind them and unit 0's MMAs start as early as they can
-          if (j == 2 && !(ok = mbar_wait_bounded(&bars->t_first, 0, abort_flag, __LINE__))) break;
+          // the first two stages go out with T's loads; the others wait until T is in shared memory,
+          // so that T does not queue behind them and unit 0's MMAs start as early as they can
+          if (q == 2 && !(ok = mbar_wait_bounded(&bars->t_first, 0, abort_flag, __LINE__))) break;
         }
-        if (j >= F::XS && !(ok = mbar_wait_bounded(&bars->x_empty[st], ((j / F::XS) - 1) & 1, abort_flag, __LINE__))) break;
-        mbar_arrive_expect_tx(&bars->x_full[st], C::X_STAGE);
+        if (q >= F::XS && !(ok = mbar_wait_bounded(&bars->x_empty[st], ((q / F::XS) - 1) & 1, abort_flag, __LINE__))) break;
+        mbar_arrive_expect_tx(&bars->x_full[st], F::X_STAGE);
 #pragma unroll
-        for (int a = 0; a < C::ATOMS; ++a)
-          tma_load_2d(xs + st * C::X_STAGE + a * (TM * 128), &tmX, b * K + 64 * a, tile * TM, &bars->x_full[st]);
-        if (own_planes && j == 0) {
+        for (int a = 0; a < F::XATOMS; ++a)
+          tma_load_2d(xs + st * F::X_STAGE + a * (TM * 128), &tmX, in0 + 64 * a, tile * TM, &bars->x_full[st]);
+        if (own_planes && q == 0) {
 #pragma unroll
           for (int sp = 1; sp < 3; ++sp) {
-            mbar_arrive_expect_tx(&plane_full[sp], C::SPLIT);
-            bulk_copy_g2s(ts + sp * C::SPLIT, src + sp * C::SPLIT, C::SPLIT, &plane_full[sp]);
+            mbar_arrive_expect_tx(&plane_full[sp], F::SPLIT);
+            bulk_copy_g2s(ts + sp * F::SPLIT, src + sp * F::SPLIT, F::SPLIT, &plane_full[sp]);
           }
         }
       }
-      const int issued = j, first = issued > F::XS ? issued - F::XS : 0;
+      const int issued = q, first = issued > F::XS ? issued - F::XS : 0;
       volatile int no_abort = 0;
-      for (int q = first; q < issued; ++q) mbar_wait_bounded(&bars->x_full[q % F::XS], (q / F::XS) & 1, &no_abort);
+      for (int r = first; r < issued; ++r) mbar_wait_bounded(&bars->x_full[r % F::XS], (r / F::XS) & 1, &no_abort);
       if (own_planes)
         for (int sp = 0; sp < 3; ++sp) mbar_wait_bounded(&plane_full[sp], 0, &no_abort);
       (void)ok;
     }
   } else if (warp == 1) {
-    // ---------------------------------------------------------------- MMA issuer: unit j -> columns j K
+    // ---------------------------------------------------------------- MMA issuer: unit j -> slot j % U
     // D = V H^T + V M^T + V L^T, plane by plane
     if (lane == 0) {
       bool ok = true;
@@ -750,30 +768,35 @@ __global__ void __launch_bounds__(kThreads, 1)
           ++version;
           cur_b = b;
         }
-        const uint32_t st = j % F::XS;
         // WAVES: the unit U back in this slot must be quantized before its columns are overwritten
         if (WAVES && j >= U && !(ok = mbar_wait_bounded(&tmem_free[j % U], ((j / U) - 1) & 1, abort_flag, __LINE__))) break;
-        if (!(ok = mbar_wait_bounded(&bars->x_full[st], (j / F::XS) & 1, abort_flag, __LINE__))) break;
-        tc_fence_after();
-        const uint32_t dcol = tmem + (j % U) * K;
-        const uint32_t xbase = smem_u32(xs + st * C::X_STAGE);
+        const uint32_t dcol = tmem + (j % U) * N;
         const uint32_t tbase = smem_u32(ts);
+        for (int h = 0; h < F::XH && ok; ++h) {       // the unit's x stages (two K halves at KD = 256)
+          const int q = j * F::XH + h;
+          const uint32_t st = q % F::XS;
+          if (!(ok = mbar_wait_bounded(&bars->x_full[st], (q / F::XS) & 1, abort_flag, __LINE__))) break;
+          tc_fence_after();
+          const uint32_t xbase = smem_u32(xs + st * F::X_STAGE);
 #pragma unroll
-        for (int sp = 0; sp < 3; ++sp) {
-          if (own_planes && j == 0) {                   // later units find every plane in place
-            if (!(ok = mbar_wait_bounded(&plane_full[sp], 0, abort_flag, __LINE__))) break;
-            tc_fence_after();
-          }
+          for (int sp = 0; sp < 3; ++sp) {
+            if (own_planes && q == 0) {                 // later stages find every plane in place
+              if (!(ok = mbar_wait_bounded(&plane_full[sp], 0, abort_flag, __LINE__))) break;
+              tc_fence_after();
+            }
 #pragma unroll
-          for (int kk = 0; kk < K / 16; ++kk) {
-            const uint32_t a_off = (kk >> 2) * (TM * 128) + (kk & 3) * 32;
-            const uint32_t b_off = (kk >> 2) * (K * 128) + (kk & 3) * 32;
-            mma_bf16(dcol, sdesc_kmajor_sw128(xbase + a_off), sdesc_kmajor_sw128(tbase + sp * C::SPLIT + b_off), C::IDESC,
-                     (kk | sp) != 0);
+            for (int kk = 0; kk < F::XW / 16; ++kk) {
+              const int kg = h * (F::XW / 16) + kk;       // the K step within the group's KD inputs
+              const uint32_t a_off = (kk >> 2) * (TM * 128) + (kk & 3) * 32;
+              const uint32_t b_off = (kg >> 2) * (N * 128) + (kg & 3) * 32;
+              mma_bf16(dcol, sdesc_kmajor_sw128(xbase + a_off), sdesc_kmajor_sw128(tbase + sp * F::SPLIT + b_off),
+                       F::IDESC, (h | kk | sp) != 0);
+            }
           }
+          if (!ok) break;
+          mma_commit(&bars->x_empty[st]);
         }
         if (!ok) break;
-        mma_commit(&bars->x_empty[st]);
         mma_commit(&unit_full[j % U]);
         int nb_next = -1, tile_next;
         if (j + 1 < nu) fused_unit(fu, j + 1, num_tiles, &nb_next, &tile_next);
@@ -884,11 +907,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         cur_b = b;
         if (planes) {                                  // one thread copies the pre-split planes
           if (ct == 0) {
-            fetch_planes<K>(planes, b, ts, &bars->t_full);
+            fetch_planes<N, KD>(planes, b, ts, &bars->t_full);
             if (version == 0) mbar_arrive(&bars->t_first);
           }
         } else {
-          split_block<K>(A + (size_t)b * K * kb, kb, ts, ct);
+          split_block<N, KD>(A + (size_t)b * N * kb, kb, ts, ct);
           fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) {
@@ -899,8 +922,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         ++version;
       }
     }
-    quantize_units<K, WAVES>(tmem, smem, fu, num_tiles, n, d, maxima_ready, tmem_free, codes, abort_flag,
-                             1 + ((warp - kCvtWarp0) >> 2));
+    quantize_units<N, KD, WAVES>(tmem, smem, fu, num_tiles, n, d, maxima_ready, tmem_free, codes, abort_flag,
+                                 1 + ((warp - kCvtWarp0) >> 2));
     tc_fence_before();
   } else if (warp >= kEpiWarp0) {
     // ---------------------------------------------------------------- phase A: one row per thread
@@ -917,11 +940,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       uint32_t mb = 0;
 #pragma unroll 1
-      for (int c = 0; c < K / 32; c += 2) {            // two loads in flight
+      for (int c = 0; c < N / 32; c += 2) {            // two loads in flight
         uint32_t r0[32], r1[32];
         __syncwarp();
-        CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + (j % U) * K + c * 32, r0);
-        CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + (j % U) * K + (c + 1) * 32, r1);
+        CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + (j % U) * N + c * 32, r0);
+        CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + (j % U) * N + (c + 1) * 32, r1);
         tmem_ld_wait();
         mb = absmax_bits32(r1, absmax_bits32(r0, mb));
       }
@@ -935,7 +958,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) mbar_arrive(&epi_done[j % U]);
     }
     if (!finite) report(status, kStatusNonFinite);
-    quantize_units<K, WAVES>(tmem, smem, fu, num_tiles, n, d, maxima_ready, tmem_free, codes, abort_flag, 0);
+    quantize_units<N, KD, WAVES>(tmem, smem, fu, num_tiles, n, d, maxima_ready, tmem_free, codes, abort_flag, 0);
     tc_fence_before();
   }
 
@@ -1069,10 +1092,10 @@ bool cooperative_ok() {
   return cudaDeviceGetAttribute(&v, cudaDevAttrCooperativeLaunch, dev) == cudaSuccess && v != 0;
 }
 
-template <int K>
+template <int N, int KD>
 cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, int kb, const float* A, const uint8_t* planes,
                            uint32_t* amax, uint32_t* words, uint32_t* status, cudaStream_t stream) {
-  const int nb = (int)(d / K);
+  const int nb = (int)(d / N);                         // groups of N output channels
   const int tiles = (int)((n + TM - 1) / TM);
   const int64_t units = (int64_t)nb * tiles;
   const int sms = num_sms();
@@ -1083,7 +1106,7 @@ cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, int kb,
   int grid = (int)(units < sms ? units : sms);
   bool waves = false;
   for (int c = 0; c < grid && !waves; ++c)
-    if (fused_units(c, grid, nb, tiles).count > 512 / K) waves = true;
+    if (fused_units(c, grid, nb, tiles).count > 512 / N) waves = true;
   if (waves) {
     if (nb > sms) return cudaErrorNotSupported;
     const int m = std::min(sms / nb, tiles);
@@ -1113,18 +1136,18 @@ cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, int kb,
   static std::once_flag once;
   static cudaError_t attr = cudaSuccess;
   std::call_once(once, [] {
-    attr = cudaFuncSetAttribute(transform_quant_tc_fused_kernel<K, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)FusedCfg<K, false>::SMEM);
+    attr = cudaFuncSetAttribute(transform_quant_tc_fused_kernel<N, KD, false>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)FusedCfg<N, KD, false>::SMEM);
     if (attr == cudaSuccess)
-      attr = cudaFuncSetAttribute(transform_quant_tc_fused_kernel<K, true>,
-                                  cudaFuncAttributeMaxDynamicSharedMemorySize, (int)FusedCfg<K, true>::SMEM);
+      attr = cudaFuncSetAttribute(transform_quant_tc_fused_kernel<N, KD, true>,
+                                  cudaFuncAttributeMaxDynamicSharedMemorySize, (int)FusedCfg<N, KD, true>::SMEM);
   });
   if (attr != cudaSuccess) return attr;
   cudaLaunchConfig_t cfg;
   memset(&cfg, 0, sizeof(cfg));
   cfg.gridDim = dim3((unsigned)grid, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = waves ? FusedCfg<K, true>::SMEM : FusedCfg<K, false>::SMEM;
+  cfg.dynamicSmemBytes = waves ? FusedCfg<N, KD, true>::SMEM : FusedCfg<N, KD, false>::SMEM;
   cfg.stream = stream;
   // not a programmatic dependent launch: measured, one cost the c2 step ~4 us (the kernel still
   // releases its dependents early, so a programmatic GEMM launch after it gets going sooner)
@@ -1135,22 +1158,24 @@ cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, int kb,
   cfg.numAttrs = 1;
   note_launch();
   if (waves)
-    return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<K, true>, map, A, planes, (int)n, (int)d, kb,
+    return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<N, KD, true>, map, A, planes, (int)n, (int)d, kb,
                               reinterpret_cast<float*>(amax), words, state, amax_sets, rec_sets, status);
-  return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<K, false>, map, A, planes, (int)n, (int)d, kb,
+  return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<N, KD, false>, map, A, planes, (int)n, (int)d, kb,
                             reinterpret_cast<float*>(amax), words, state, amax_sets, rec_sets, status);
 }
 
 }  // namespace
 
-// The K-wide kernel that runs blocks of size k on d channels: 128 when 128 divides d (a k < 128
-// runs block-diagonal inside each 128-channel group: twice to eight times the MMAs of a k-wide
-// kernel, but the 128-wide kernels are the faster ones, e.g. c5 at k = 64: 64 against 87 us), 64
-// for k = 64 otherwise, 0 when no tensor-core kernel applies (k = 256: three bf16 planes of a
-// 256 x 256 block do not fit in shared memory beside the x tiles).
+// The tensor-core transform's input width KD per group (the plane split's group: N = KD outputs,
+// except N = 64 at KD = 256) for block size k on d channels: 128 when 128 divides d and k <= 128 (a
+// k < 128 runs block-diagonal inside each 128-channel group: 2-8x the MMAs of a k-wide kernel, but
+// the 128-wide kernels are the faster ones, e.g. c5 at k = 64: 64 against 87 us), 64 for k = 64
+// otherwise, 256 for k = 256 (a group is a quarter of a block's outputs: a whole block's three bf16
+// planes would not fit in shared memory), 0 when no tensor-core kernel applies.
 int transform_tc_group(int k, int64_t d) {
   if ((k == 16 || k == 32 || k == 64 || k == 128) && d % 128 == 0) return 128;
   if (k == 64 && d % 64 == 0) return 64;
+  if (k == 256 && d % 256 == 0) return 256;
   return 0;
 }
 
@@ -1166,18 +1191,18 @@ cudaError_t launch_transform_quantize_tc(const void* x, int64_t n, int64_t d, in
   const int K = transform_tc_group(k, d);
   if (K == 64) return launch_k<64>(xb, n, d, k, A, planes, amax, words, scale, status, stream);
   if (K == 128) return launch_k<128>(xb, n, d, k, A, planes, amax, words, scale, status, stream);
-  return cudaErrorInvalidValue;
+  return cudaErrorNotSupported;                      // k = 256: the fused kernel only
 }
 
-// T_blocks -> the three bf16 planes of every K-wide group (K = transform_tc_group(k, d)) in the
-// transform kernels' shared-memory layout ([d/K][3][K*K] bf16, 6 d K bytes).
+// T_blocks -> the three bf16 planes of every group (KD = transform_tc_group(k, d) inputs, N outputs)
+// in the transform kernels' shared-memory layout ([d/N][3][N*KD] bf16, 6 d KD bytes).
 cudaError_t launch_split_transform(const float* A, int64_t d, int k, uint8_t* planes, cudaStream_t stream) {
-  const int K = transform_tc_group(k, d);
-  if (K == 0) return cudaErrorNotSupported;
-  const unsigned groups = (unsigned)(d / K);
+  const int KD = transform_tc_group(k, d);
+  if (KD == 0) return cudaErrorNotSupported;
   note_launch();
-  if (K == 64) split_planes_kernel<64><<<groups, kCvtWarps * 32, 0, stream>>>(A, k, planes);
-  else split_planes_kernel<128><<<groups, kCvtWarps * 32, 0, stream>>>(A, k, planes);
+  if (KD == 64) split_planes_kernel<64, 64><<<(unsigned)(d / 64), kCvtWarps * 32, 0, stream>>>(A, k, planes);
+  else if (KD == 128) split_planes_kernel<128, 128><<<(unsigned)(d / 128), kCvtWarps * 32, 0, stream>>>(A, k, planes);
+  else split_planes_kernel<64, 256><<<(unsigned)(d / 64), kCvtWarps * 32, 0, stream>>>(A, k, planes);
   return cudaGetLastError();
 }
 
@@ -1191,9 +1216,10 @@ cudaError_t launch_transform_quantize_tc_fused(const void* x, int64_t n, int64_t
                                                const uint8_t* planes, uint32_t* amax, uint32_t* words,
                                                uint32_t* status, cudaStream_t stream) {
   const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
-  const int K = transform_tc_group(k, d);
-  if (K == 64) return launch_fused_k<64>(xb, n, d, k, A, planes, amax, words, status, stream);
-  if (K == 128) return launch_fused_k<128>(xb, n, d, k, A, planes, amax, words, status, stream);
+  const int KD = transform_tc_group(k, d);
+  if (KD == 64) return launch_fused_k<64, 64>(xb, n, d, k, A, planes, amax, words, status, stream);
+  if (KD == 128) return launch_fused_k<128, 128>(xb, n, d, k, A, planes, amax, words, status, stream);
+  if (KD == 256) return launch_fused_k<64, 256>(xb, n, d, k, A, planes, amax, words, status, stream);
   return cudaErrorNotSupported;
 }
 }  // namespace cat

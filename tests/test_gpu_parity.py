@@ -97,7 +97,11 @@ def _cat_T(rng, d, k):
                                          # 64 | d but not 128: the 64-wide kernels (one wave, two passes)
                                          (300, 192, 64, "bf16"), (1100, 9920, 64, "bf16"),
                                          # more groups than SMs and more than one wave: two passes
-                                         (520, 20480, 128, "bf16")])
+                                         (520, 20480, 128, "bf16"),
+                                         # k = 256: 64-output quarters of a block over its 256 inputs
+                                         # (one wave, waves, contiguous ranges; beyond: the SIMT kernel)
+                                         (2560, 2048, 256, "bf16"), (2560, 4096, 256, "bf16"),
+                                         (300, 10240, 256, "bf16"), (1300, 10240, 256, "bf16")])
 def test_transform_quantize_act(n, d, k, dtype):
     rng = np.random.default_rng(7 * n + d)
     X = rng.standard_normal((n, d)) * rng.lognormal(0, 1.0, d)
@@ -121,7 +125,8 @@ def test_transform_quantize_act(n, d, k, dtype):
 @pytest.mark.parametrize("n,d,k,dtype", [(67, 384, 128, "bf16"), (300, 1024, 64, "bf16"), (1000, 256, 128, "bf16"),
                                          (2560, 4096, 128, "bf16"), (1300, 8192, 64, "bf16"),
                                          (300, 512, 32, "bf16"), (130, 384, 16, "bf16"), (300, 192, 64, "bf16"),
-                                         (1100, 9920, 64, "bf16"), (130, 256, 32, "f32")])
+                                         (1100, 9920, 64, "bf16"), (200, 512, 256, "bf16"), (2560, 4096, 256, "bf16"),
+                                         (130, 256, 32, "f32")])
 def test_transform_with_presplit_planes_is_identical(n, d, k, dtype):
     """T's bf16 planes split once (cat_split_transform) and bulk-copied by the kernels give the same
     codes and steps, bit for bit, as the kernels' own split (fused, two-pass, and the SIMT path that
@@ -152,7 +157,8 @@ def test_nonfinite_activation_reports_numeric():
 
 @pytest.mark.parametrize("n,d,k", [(2560, 4096, 128),    # the fused kernel in waves
                                    (1100, 9920, 64),     # the two-pass kernel (64-wide)
-                                   (2560, 4096, 32)])    # waves, k = 32 block-diagonal in 128-channel groups
+                                   (2560, 4096, 32),     # waves, k = 32 block-diagonal in 128-channel groups
+                                   (2560, 4096, 256)])   # waves, k = 256 in 64-output quarters
 def test_nonfinite_activation_many_units(n, d, k):
     """bf16 rows with more units per CTA than tensor memory holds: a row holding inf or NaN gets step 0
     and all codes 0, the status reports it, and the other rows are unaffected."""
@@ -223,7 +229,8 @@ def _tie_rows(rng, n, d):
                                          (2560, 4096, 128, "bf16"),                            # waves
                                          (1100, 9920, 64, "bf16"),                             # two-pass
                                          (300, 512, 32, "bf16"),                               # k = 32 in groups
-                                         (130, 256, 32, "f32"), (200, 512, 256, "bf16"),       # SIMT
+                                         (200, 512, 256, "bf16"),                              # k = 256
+                                         (130, 256, 32, "f32"),                                # SIMT
                                          (70, 64, 16, "bf16")])
 def test_code_decision_exact_on_ties(n, d, k, dtype):
     """With T = I the transformed row is the input row, so the codes must equal the definition's
