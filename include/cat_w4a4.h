@@ -244,6 +244,44 @@ cat_status cat_w4a4_linear_sqnr(const uint8_t* xq, const float* x_scale, const u
                                 cat_stream_t stream);
 
 /*
+ * Byte codes ("E8")
+ * -----------------
+ *  The same codes q in [-7, 7], one per byte: byte = (q < 0) << 7 | |q|, the FP8 E4M3 encoding of
+ *  the subnormal q * 2^-9 (the bytes the SM4x8 masks produce).  A row of d codes occupies d bytes,
+ *  twice the SM4x8 size.  The byte-code GEMM loads them into shared memory as they are and runs the
+ *  FP8 tensor cores on them directly, with no decode step; the weights are converted once per layer
+ *  (cat_codes_to_e4m3), the activations are written in this form by cat_transform_quantize_act_e8.
+ *  Its results are identical to the SM4x8 GEMM's (same exact integer accumulators, same scaling).
+ */
+
+/*
+ * cat_codes_to_e4m3 -- SM4x8 codes to byte codes (a layout change; no arithmetic).
+ *   codes  device [rows][d/2] bytes, SM4x8;   out  out, device [rows][d] bytes, byte codes.
+ *   d must be a positive multiple of 32 (CAT_ERR_SHAPE).  rows == 0 is a no-op.  Asynchronous on stream.
+ */
+cat_status cat_codes_to_e4m3(const uint8_t* codes, int64_t rows, int64_t d, uint8_t* out, cat_stream_t stream);
+
+/*
+ * cat_w4a4_linear_e8 -- cat_w4a4_linear on byte codes (Sec. 3 Eq. 5).
+ *   xq8 [n][d_in], Wq8 [d_out][d_in] byte codes; x_scale, w_scale, y, acc_out as cat_w4a4_linear.
+ *   Same results as cat_w4a4_linear on the SM4x8 form of the same codes, for every n >= 1 (it
+ *   always runs the 256 x 128 tile kernel: for n <= 32 the SM4x8 weight-streaming kernel reads half
+ *   the bytes).  Asynchronous on stream; errors as cat_w4a4_linear.
+ */
+cat_status cat_w4a4_linear_e8(const uint8_t* xq8, const float* x_scale, const uint8_t* Wq8, const float* w_scale,
+                              int64_t n, int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, cat_stream_t stream);
+
+/*
+ * cat_w4a4_linear_sqnr_e8 -- cat_w4a4_linear_sqnr on byte codes (Sec. 3 Eq. 5; Sec. 2 Eq. 1).
+ *   Arguments as cat_w4a4_linear_e8 (without acc_out) plus y_ref and out3 as cat_w4a4_linear_sqnr.
+ *   The sums are formed in the GEMM's epilogue when d_out % 4 == 0, else by the cat_sqnr reduction;
+ *   the same sums as cat_w4a4_linear_sqnr for n > 32.
+ */
+cat_status cat_w4a4_linear_sqnr_e8(const uint8_t* xq8, const float* x_scale, const uint8_t* Wq8, const float* w_scale,
+                                   int64_t n, int64_t d_in, int64_t d_out, float* y, const float* y_ref, double* out3,
+                                   cat_stream_t stream);
+
+/*
  * cat_sqnr -- signal-to-quantization-noise ratio of the layer output (Sec. 2, Eq. 1).
  *   y_ref, y_hat device [numel] float32 (full-precision and quantized outputs).
  *   out3         out, device [3] float64: { sum y_ref^2, sum (y_ref - y_hat)^2, 10 log10(ratio) dB }.

@@ -86,6 +86,9 @@ def load_library() -> ctypes.CDLL:
         "cat_transform_quantize_act_dp": ([P, I, I64, I64, I32, P, I32, I32, P, P, P, P], I),
         "cat_quantize_weights_dp": ([P, I, I64, I64, I32, I, P, I64, P, I32, I32, P, P, P, P, P], I),
         "cat_linear_dp": ([P, I32, I32, P, P, P, I32, P, P, I64, I64, I64, P, P, P], I),
+        "cat_codes_to_e4m3": ([P, I64, I64, P, P], I),
+        "cat_w4a4_linear_e8": ([P, P, P, P, I64, I64, I64, P, P, P], I),
+        "cat_w4a4_linear_sqnr_e8": ([P, P, P, P, I64, I64, I64, P, P, P, P], I),
     }
     for name, (args, res) in sigs.items():
         f = getattr(lib, name)
@@ -338,6 +341,70 @@ def cat_w4a4_linear_sqnr(xq: torch.Tensor, x_scale: torch.Tensor, Wq: torch.Tens
     _check("cat_w4a4_linear_sqnr", load_library().cat_w4a4_linear_sqnr(
         _ptr(xq), _ptr(x_scale), _ptr(Wq), _ptr(w_scale), n, 2 * half, d_out, _ptr(y), _ptr(y_ref), _ptr(out),
         _stream(xq.device)))
+    return y, out
+
+
+def cat_codes_to_e4m3(codes: torch.Tensor, out: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """SM4x8 codes uint8 [rows, d/2] -> byte codes uint8 [rows, d] (one E4M3 byte per code)."""
+    _need(codes, "codes")
+    if codes.dtype != torch.uint8 or codes.dim() != 2:
+        raise ValueError("codes must be a 2-D uint8 tensor")
+    rows, half = codes.shape
+    if out is None:
+        out = torch.empty((rows, 2 * half), dtype=torch.uint8, device=codes.device)
+    _expect(out, "out", torch.uint8, (rows, 2 * half), codes.device)
+    _check("cat_codes_to_e4m3", load_library().cat_codes_to_e4m3(_ptr(codes), rows, 2 * half, _ptr(out),
+                                                                 _stream(codes.device)))
+    return out
+
+
+def _linear_args_e8(xq8, x_scale, Wq8, w_scale, y) -> None:
+    n, d_in = xq8.shape
+    d_out = Wq8.shape[0]
+    dev = xq8.device
+    _expect(xq8, "xq8", torch.uint8, (n, d_in), dev)
+    _expect(x_scale, "x_scale", torch.float32, (n,), dev)
+    _expect(Wq8, "Wq8", torch.uint8, (d_out, d_in), dev)
+    _expect(w_scale, "w_scale", torch.float32, (d_out,), dev)
+    _expect(y, "y", torch.float32, (n, d_out), dev)
+
+
+def cat_w4a4_linear_e8(xq8: torch.Tensor, x_scale: torch.Tensor, Wq8: torch.Tensor, w_scale: torch.Tensor,
+                       y: Optional[torch.Tensor] = None, acc_out: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """cat_w4a4_linear on byte codes xq8 [n, d_in], Wq8 [d_out, d_in]: the same y (and accumulators)."""
+    for t, name in ((xq8, "xq8"), (x_scale, "x_scale"), (Wq8, "Wq8"), (w_scale, "w_scale")):
+        _need(t, name)
+    n, d_in = xq8.shape
+    d_out = Wq8.shape[0]
+    if y is None:
+        y = torch.empty((n, d_out), dtype=torch.float32, device=xq8.device)
+    _linear_args_e8(xq8, x_scale, Wq8, w_scale, y)
+    if acc_out is not None:
+        _expect(acc_out, "acc_out", torch.int32, (n, d_out), xq8.device)
+    _check("cat_w4a4_linear_e8", load_library().cat_w4a4_linear_e8(
+        _ptr(xq8), _ptr(x_scale), _ptr(Wq8), _ptr(w_scale), n, d_in, d_out, _ptr(y), _ptr(acc_out),
+        _stream(xq8.device)))
+    return y
+
+
+def cat_w4a4_linear_sqnr_e8(xq8: torch.Tensor, x_scale: torch.Tensor, Wq8: torch.Tensor, w_scale: torch.Tensor,
+                            y_ref: torch.Tensor, y: Optional[torch.Tensor] = None,
+                            out: Optional[torch.Tensor] = None) -> Tuple[torch.Tensor, torch.Tensor]:
+    """cat_w4a4_linear_sqnr on byte codes: (y float32 [n, d_out], float64 [3])."""
+    for t, name in ((xq8, "xq8"), (x_scale, "x_scale"), (Wq8, "Wq8"), (w_scale, "w_scale"), (y_ref, "y_ref")):
+        _need(t, name)
+    n, d_in = xq8.shape
+    d_out = Wq8.shape[0]
+    if y is None:
+        y = torch.empty((n, d_out), dtype=torch.float32, device=xq8.device)
+    if out is None:
+        out = torch.empty((3,), dtype=torch.float64, device=xq8.device)
+    _linear_args_e8(xq8, x_scale, Wq8, w_scale, y)
+    _expect(y_ref, "y_ref", torch.float32, (n, d_out), xq8.device)
+    _expect(out, "out", torch.float64, (3,), xq8.device)
+    _check("cat_w4a4_linear_sqnr_e8", load_library().cat_w4a4_linear_sqnr_e8(
+        _ptr(xq8), _ptr(x_scale), _ptr(Wq8), _ptr(w_scale), n, d_in, d_out, _ptr(y), _ptr(y_ref), _ptr(out),
+        _stream(xq8.device)))
     return y, out
 
 

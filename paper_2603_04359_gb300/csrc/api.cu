@@ -20,6 +20,10 @@ cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_
 cudaError_t launch_w4a4_gemm_decode(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
                                     int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, const float* y_ref,
                                     double* sums3, uint32_t* status, cudaStream_t stream);
+cudaError_t launch_w4a4_gemm_tc_e8(const uint8_t* xq8, const float* sx, const uint8_t* wq8, const float* sw, int64_t n,
+                                   int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, const float* y_ref,
+                                   double* sums3, uint32_t* status, cudaStream_t stream);
+cudaError_t launch_codes_to_e4m3(const uint8_t* codes, int64_t rows, int64_t d, uint8_t* out, cudaStream_t stream);
 cudaError_t launch_block_row_stats(const void* V, int dtype, int64_t rows, int64_t d, int k, const float* M,
                                    int transpose, float* row_sumsq, float* row_amax, double* out3,
                                    cudaStream_t stream);
@@ -646,6 +650,71 @@ cat_status cat_w4a4_linear_sqnr(const uint8_t* xq, const float* x_scale, const u
     if (e == cudaSuccess) e = cat::launch_sqnr(y_ref, y, n * d_out, out3, s);
   }
   if (e != cudaSuccess) return cuda_fail(e, "cat_w4a4_linear_sqnr launch");
+  return ok();
+}
+
+// ---- byte codes: one E4M3 byte per code, for the tensor cores to read as they are
+
+cat_status cat_codes_to_e4m3(const uint8_t* codes, int64_t rows, int64_t d, uint8_t* out, cat_stream_t stream) {
+  if (rows < 0 || d <= 0 || d % 32 != 0) return fail(CAT_ERR_SHAPE, "rows >= 0 and d a positive multiple of 32");
+  if (rows > ((int64_t)1 << 40) / d) return fail(CAT_ERR_SHAPE, "rows x d too large");
+  if (rows == 0) return ok();
+  if (!codes || !out) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(codes) || !aligned16(out)) return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  cat_status st = check_device();
+  if (st != CAT_OK) return st;
+  cudaError_t e = cat::launch_codes_to_e4m3(codes, rows, d, out, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cat_codes_to_e4m3 launch");
+  return ok();
+}
+
+cat_status cat_w4a4_linear_e8(const uint8_t* xq8, const float* x_scale, const uint8_t* Wq8, const float* w_scale,
+                              int64_t n, int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, cat_stream_t stream) {
+  if (n < 0 || d_out <= 0) return fail(CAT_ERR_SHAPE, "n must be >= 0 and d_out >= 1");
+  cat_status st = check_din(d_in);
+  if (st != CAT_OK) return st;
+  if (n > 0x7FFFFFFF || d_out > 0x7FFFFFFF) return fail(CAT_ERR_SHAPE, "n and d_out must fit in int32");
+  if (n == 0) return ok();
+  if (!xq8 || !x_scale || !Wq8 || !w_scale || !y) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(xq8) || !aligned16(x_scale) || !aligned16(Wq8) || !aligned16(w_scale) || !aligned16(y) ||
+      (acc_out && !aligned16(acc_out)))
+    return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  if ((st = check_device()) != CAT_OK) return st;
+  cudaError_t e;
+  uint32_t* status = status_word(&e);
+  if (!status) return cuda_fail(e, "status word");
+  e = cat::launch_w4a4_gemm_tc_e8(xq8, x_scale, Wq8, w_scale, n, d_in, d_out, y, acc_out, nullptr, nullptr, status,
+                                  (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cat_w4a4_linear_e8 launch");
+  return ok();
+}
+
+cat_status cat_w4a4_linear_sqnr_e8(const uint8_t* xq8, const float* x_scale, const uint8_t* Wq8, const float* w_scale,
+                                   int64_t n, int64_t d_in, int64_t d_out, float* y, const float* y_ref, double* out3,
+                                   cat_stream_t stream) {
+  if (n < 0 || d_out <= 0) return fail(CAT_ERR_SHAPE, "n must be >= 0 and d_out >= 1");
+  cat_status st = check_din(d_in);
+  if (st != CAT_OK) return st;
+  if (n > 0x7FFFFFFF || d_out > 0x7FFFFFFF) return fail(CAT_ERR_SHAPE, "n and d_out must fit in int32");
+  if (!out3 || (n > 0 && (!xq8 || !x_scale || !Wq8 || !w_scale || !y || !y_ref)))
+    return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(out3) || (n > 0 && (!aligned16(xq8) || !aligned16(x_scale) || !aligned16(Wq8) ||
+                                     !aligned16(w_scale) || !aligned16(y) || !aligned16(y_ref))))
+    return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  if ((st = check_device()) != CAT_OK) return st;
+  cudaError_t e;
+  uint32_t* status = status_word(&e);
+  if (!status) return cuda_fail(e, "status word");
+  cudaStream_t s = (cudaStream_t)stream;
+  if (n > 0 && d_out % 4 == 0) {  // SQNR sums fused into the GEMM epilogue
+    e = cat::launch_w4a4_gemm_tc_e8(xq8, x_scale, Wq8, w_scale, n, d_in, d_out, y, nullptr, y_ref, out3, status, s);
+  } else {                        // the GEMM, then the separate reduction
+    e = n == 0 ? cudaSuccess
+               : cat::launch_w4a4_gemm_tc_e8(xq8, x_scale, Wq8, w_scale, n, d_in, d_out, y, nullptr, nullptr, nullptr,
+                                             status, s);
+    if (e == cudaSuccess) e = cat::launch_sqnr(y_ref, y, n * d_out, out3, s);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, "cat_w4a4_linear_sqnr_e8 launch");
   return ok();
 }
 

@@ -78,15 +78,33 @@ constexpr uint32_t kIdesc = idesc_e4m3_f32(2 * BM, BN);
 constexpr uint32_t kEpiStage = 32 * 32 * 4;                 // 32 rows x 32 fp32 columns, 4 KiB
 constexpr int kEpiBufs = 2;                                  // TMA-store staging buffers per epilogue warp
 constexpr uint32_t kPkOffset = SE * kStageB;                 // after the decoded B stages
-constexpr uint32_t kEpiOffset = kPkOffset + SP * kPackedStage;
-constexpr uint32_t kRefOffset = kEpiOffset + kEpiWarps * kEpiBufs * kEpiStage;   // y_ref tiles (SQNR)
-constexpr uint32_t kScaleOffset = kRefOffset + kEpiWarps * kEpiBufs * kEpiStage;
-constexpr uint32_t kBarOffset = kScaleOffset + kEpiWarps * BN * 4;
 constexpr uint32_t kBarBytes = 1024;                         // room reserved for the barrier block
-constexpr size_t kSmemBytes = kBarOffset + kBarBytes + 1024;  // + barriers + alignment slack
+// Byte codes (E8): one E4M3 byte per code (sign << 7 | magnitude, i.e. q * 2^-9), loaded by TMA as
+// they are and multiplied from shared memory: no decode warps, no packed ring, and SE stages of
+// A (128 rows x 256 B) and B (64 rows x 256 B).
+constexpr uint32_t kAtomA8 = BM * 128;      // one 128-code K atom of A (128 rows x 128 B)
+constexpr uint32_t kStageA8 = BM * BK;      // 32 KiB
+constexpr uint32_t kStage8 = kStageA8 + kStageB;   // 48 KiB
+// Shared memory and tensor memory of the two operand formats.  The byte-code stages leave room for
+// one y and one y_ref staging buffer per epilogue warp, and the output-channel steps of a chunk go
+// through registers instead of shared memory.
+template <bool E8>
+struct GemmLayout {
+  static constexpr int EB = E8 ? 1 : kEpiBufs;   // y staging buffers per epilogue warp
+  static constexpr int RB = E8 ? 1 : kEpiBufs;   // y_ref staging buffers per epilogue warp
+  static constexpr uint32_t kOperands = E8 ? SE * kStage8 : kPkOffset + SP * kPackedStage;
+  static constexpr uint32_t kEpiOffset = kOperands;
+  static constexpr uint32_t kRefOffset = kEpiOffset + kEpiWarps * EB * kEpiStage;   // y_ref tiles (SQNR)
+  static constexpr uint32_t kScaleOffset = kRefOffset + kEpiWarps * RB * kEpiStage;
+  static constexpr uint32_t kBarOffset = kScaleOffset + (E8 ? 0u : kEpiWarps * BN * 4);
+  static constexpr uint32_t kBarRoom = E8 ? 512u : kBarBytes;
+  static constexpr size_t kSmemBytes = kBarOffset + kBarRoom + 1024;  // + barriers + alignment slack
+  static constexpr uint32_t kTmem = E8 ? kAccCols : kTmemCols;
+  static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+};
 static_assert(kAccCols + SE * 64 <= kTmemCols, "tensor memory budget");
-static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 static_assert(kPackedStage % 1024 == 0 && kAtomB % 1024 == 0 && kPackedA % 1024 == 0, "128B-swizzle alignment");
+static_assert(kStage8 % 1024 == 0 && kAtomA8 % 1024 == 0 && kStageA8 % 1024 == 0, "128B-swizzle alignment");
 static_assert((BNC * 8) % kGroupThreads == 0, "B chunks per decode thread");
 
 
@@ -98,7 +116,8 @@ struct Bars {
   int abort;
   f32x2 sums[kEpiWarps][2];                      // SQNR sums of the epilogue warps
 };
-static_assert(sizeof(Bars) <= kBarBytes, "barrier block must fit its reserved room");
+static_assert(sizeof(Bars) <= GemmLayout<false>::kBarRoom && sizeof(Bars) <= GemmLayout<true>::kBarRoom,
+              "barrier block must fit its reserved room");
 
 // ---- tensor-memory stores and the TMA store path -------------------------------------------
 #define CAT_TMEM_ST32(taddr, v)                                                                                 \
@@ -150,6 +169,15 @@ __device__ __forceinline__ void mma_pair_ts(uint32_t d_tmem, uint32_t a_tmem, ui
       "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// the pair MMA with both operands in shared memory (each CTA: its 128 A rows and its half of B)
+__device__ __forceinline__ void mma_pair_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                            uint32_t accumulate) {
+  asm volatile(
+      "{ .reg .pred p; setp.ne.b32 p, %4, 0; "
+      "tcgen05.mma.cta_group::2.kind::f8f6f4 [%0], %1, %2, %3, p; }" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
 // arrive once on the mbarrier at this offset in both CTAs when the pair MMAs issued so far complete
 __device__ __forceinline__ void mma_commit_pair(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
@@ -168,6 +196,7 @@ __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void*
 }
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_read_le1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read_all() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 // ---- the last wave's tiles split along K -----------------------------------------------------
@@ -207,6 +236,7 @@ __device__ __forceinline__ Unit unit_at(int u, int num_full, int split, int num_
   return {num_full + u / split, part * num_k / split, (part + 1) * num_k / split, part};
 }
 
+template <bool E8>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     w4a4_gemm_tc_kernel(const __grid_constant__ CUtensorMap tmY, const __grid_constant__ CUtensorMap tmA,
                         const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmR,
@@ -215,14 +245,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                         const float* __restrict__ sw, int n, int d_in, int d_out, float* __restrict__ y,
                         int32_t* __restrict__ acc_out, int use_tma_store, int num_full, int split, int split_slot,
                         uint32_t* __restrict__ status) {
+  using L = GemmLayout<E8>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* bst = smem;                         // SE x 2 atoms x [128 rows x 128 B] E4M3, 128B-swizzled
-  uint8_t* pk = smem + kPkOffset;              // SP x [A 128 x 128 B | B 128 x 128 B] packed, 128B-swizzled
-  uint8_t* epi = smem + kEpiOffset;            // 4 warps x 2 x [32 rows x 128 B], 128B-swizzled
-  uint8_t* refb = smem + kRefOffset;           // 4 warps x 2 x [32 rows x 128 B] y_ref, 128B-swizzled
-  float* scl = reinterpret_cast<float*>(smem + kScaleOffset);  // 4 warps x 128 output-channel steps
-  Bars* bars = reinterpret_cast<Bars*>(smem + kBarOffset);
+  // packed codes: SE x 2 atoms x [64 rows x 128 B] decoded B; byte codes: SE x [A 2 atoms x [128 rows x
+  // 128 B] | B 2 atoms x [64 rows x 128 B]] as loaded; all E4M3, 128B-swizzled
+  uint8_t* bst = smem;
+  uint8_t* pk = smem + kPkOffset;              // packed codes: SP x [A 128 x 128 B | B 64 x 128 B], 128B-swizzled
+  uint8_t* epi = smem + L::kEpiOffset;         // 4 warps x EB x [32 rows x 128 B], 128B-swizzled
+  uint8_t* refb = smem + L::kRefOffset;        // 4 warps x RB x [32 rows x 128 B] y_ref, 128B-swizzled
+  float* scl = reinterpret_cast<float*>(smem + L::kScaleOffset);  // packed codes: 4 warps x 128 channel steps
+  Bars* bars = reinterpret_cast<Bars*>(smem + L::kBarOffset);
   volatile int* abort_flag = &bars->abort;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -242,8 +275,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       mbar_init(&bars->p_empty[s], kGroupWarps);    // the decode group of that stage
     }
     for (int s = 0; s < SE; ++s) {
-      mbar_init(&bars->full[s], kGroupWarps);     // even CTA: its decode group (+ 4 bytes from the odd CTA)
-      mbar_init(&bars->ready[s], kGroupWarps);    // odd CTA: its decode group (then forwarded)
+      // even CTA: its decode group, or with byte codes its two producers (+ 4 bytes from the odd CTA);
+      // odd CTA: the same locally, then forwarded
+      mbar_init(&bars->full[s], E8 ? 2 : kGroupWarps);
+      mbar_init(&bars->ready[s], E8 ? 2 : kGroupWarps);
       mbar_init(&bars->empty[s], 1);              // the pair MMA's multicast commit
     }
     for (int b = 0; b < 2; ++b) {
@@ -252,13 +287,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     }
     mbar_init(&bars->mma_done, 1);
     for (int w = 0; w < kEpiWarps; ++w)
-      for (int b = 0; b < kEpiBufs; ++b) mbar_init(&bars->ref_full[w][b], 1);
+      for (int b = 0; b < L::RB; ++b) mbar_init(&bars->ref_full[w][b], 1);
     bars->abort = 0;
     fence_mbar_init();
   }
   __syncwarp();
   pdl_wait_then_release();                        // nothing global or in tensor memory before this
-  if (warp == 0) tmem_alloc_pair(&bars->tmem_addr, kTmemCols);
+  if (warp == 0) tmem_alloc_pair(&bars->tmem_addr, L::kTmem);
   tc_fence_before();
   cluster_sync();                                 // both CTAs' barriers are initialized before any remote arrive
   tc_fence_after();
@@ -275,19 +310,36 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       for (int u = pair; u < total_units && ok; u += num_pairs) {
         const Unit w = unit_at(u, num_full, split, num_k, n_split);
         const int m = w.tile % num_m, nn = w.tile / num_m;
+        const int row = is_a ? m * 2 * BM + (int)rank * BM : nn * BN + (int)rank * BNC;
         for (int ks = w.k0; ks < w.k1; ++ks, ++it) {
-          const uint32_t s = it % SP, use = it / SP;
-          if (use > 0 && !(ok = mbar_wait_bounded(&bars->p_empty[s], (use - 1) & 1, abort_flag, __LINE__))) break;
-          uint8_t* dst = pk + s * kPackedStage + (is_a ? 0 : kPackedA);
-          uint64_t* pf = &bars->p_full[it % kDecGroups][s];   // the barrier of the group that decodes it
-          mbar_arrive_expect_tx(pf, is_a ? kPackedA : kPackedB);
-          tma_load_2d(dst, map, ks * BKP, is_a ? m * 2 * BM + (int)rank * BM : nn * BN + (int)rank * BNC, pf);
+          if constexpr (E8) {
+            // the stage's two K atoms; the even CTA's A producer also expects the odd CTA's 4-byte signal
+            const uint32_t s = it % SE, use = it / SE;
+            if (use > 0 && !(ok = mbar_wait_bounded(&bars->empty[s], (use - 1) & 1, abort_flag, __LINE__))) break;
+            uint8_t* dst = bst + s * kStage8 + (is_a ? 0u : kStageA8);
+            uint64_t* fb = rank == 0 ? &bars->full[s] : &bars->ready[s];
+            mbar_arrive_expect_tx(fb, is_a ? kStageA8 + (rank == 0 ? 4u : 0u) : kStageB);
+            tma_load_2d(dst, map, ks * BK, row, fb);
+            tma_load_2d(dst + (is_a ? kAtomA8 : kAtomB), map, ks * BK + 128, row, fb);
+          } else {
+            const uint32_t s = it % SP, use = it / SP;
+            if (use > 0 && !(ok = mbar_wait_bounded(&bars->p_empty[s], (use - 1) & 1, abort_flag, __LINE__))) break;
+            uint8_t* dst = pk + s * kPackedStage + (is_a ? 0 : kPackedA);
+            uint64_t* pf = &bars->p_full[it % kDecGroups][s];   // the barrier of the group that decodes it
+            mbar_arrive_expect_tx(pf, is_a ? kPackedA : kPackedB);
+            tma_load_2d(dst, map, ks * BKP, row, pf);
+          }
         }
       }
-      const uint32_t issued = it, first = issued > SP ? issued - SP : 0;
+      // the copies in flight land before the CTA exits (they have, unless a wait gave up)
       volatile int no_abort = 0;
-      for (uint32_t j = first; j < issued; ++j)
-        mbar_wait_bounded(&bars->p_full[j % kDecGroups][j % SP], (j / kPFullPeriod) & 1, &no_abort);
+      if constexpr (E8) {
+        for (uint32_t j = it > (uint32_t)SE ? it - SE : 0; j < it; ++j)
+          mbar_wait_bounded(rank == 0 ? &bars->full[j % SE] : &bars->ready[j % SE], (j / SE) & 1, &no_abort);
+      } else {
+        for (uint32_t j = it > (uint32_t)SP ? it - SP : 0; j < it; ++j)
+          mbar_wait_bounded(&bars->p_full[j % kDecGroups][j % SP], (j / kPFullPeriod) & 1, &no_abort);
+      }
     }
   } else if ((warp == kMmaWarp || warp == kFwdWarp) && rank == 1) {
     // ---------------------------------------------------------------- odd CTA: forward stage readiness
@@ -325,12 +377,22 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           const uint32_t s = it % SE;
           if (!(ok = mbar_wait_bounded(&bars->full[s], (it / SE) & 1, abort_flag, __LINE__))) break;
           tc_fence_after();
-          const uint32_t bbase = smem_u32(bst + s * kStageB);
-          const uint32_t ta = tmem + kAccCols + 64u * s;
+          if constexpr (E8) {
+            const uint32_t abase = smem_u32(bst + s * kStage8), bbase = abase + kStageA8;
 #pragma unroll
-          for (int kk = 0; kk < BK / 32; ++kk) {  // K = 32 codes per MMA: 8 TMEM columns of A; B atom kk/4, +32 B
-            const uint64_t db = sdesc_kmajor_sw128(bbase + (uint32_t)(kk >> 2) * kAtomB) + 2 * (kk & 3);
-            mma_pair_ts(tmem + ab * BN, ta + 8u * kk, db, kIdesc, (ks != w.k0 || kk != 0) ? 1u : 0u);
+            for (int kk = 0; kk < BK / 32; ++kk) {  // K = 32 codes per MMA: atom kk/4 of A and of B, +32 B
+              const uint64_t da = sdesc_kmajor_sw128(abase + (uint32_t)(kk >> 2) * kAtomA8) + 2 * (kk & 3);
+              const uint64_t db = sdesc_kmajor_sw128(bbase + (uint32_t)(kk >> 2) * kAtomB) + 2 * (kk & 3);
+              mma_pair_ss(tmem + ab * BN, da, db, kIdesc, (ks != w.k0 || kk != 0) ? 1u : 0u);
+            }
+          } else {
+            const uint32_t bbase = smem_u32(bst + s * kStageB);
+            const uint32_t ta = tmem + kAccCols + 64u * s;
+#pragma unroll
+            for (int kk = 0; kk < BK / 32; ++kk) {  // K = 32 codes per MMA: 8 TMEM columns of A; B atom kk/4, +32 B
+              const uint64_t db = sdesc_kmajor_sw128(bbase + (uint32_t)(kk >> 2) * kAtomB) + 2 * (kk & 3);
+              mma_pair_ts(tmem + ab * BN, ta + 8u * kk, db, kIdesc, (ks != w.k0 || kk != 0) ? 1u : 0u);
+            }
           }
           mma_commit_pair(&bars->empty[s]);
         }
@@ -343,34 +405,40 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   } else if (warp >= kEpiWarp0 && warp < kEpiWarp0 + kEpiWarps) {
     // ---------------------------------------------------------------- epilogue
     const int quad = warp & 3, ew = warp - kEpiWarp0;
-    uint8_t* stage0 = epi + ew * kEpiBufs * kEpiStage;
-    uint8_t* rstage0 = refb + ew * kEpiBufs * kEpiStage;
+    uint8_t* stage0 = epi + ew * L::EB * kEpiStage;
+    uint8_t* rstage0 = refb + ew * L::RB * kEpiStage;
     float* wsc = scl + ew * BN;
     const bool with_ref = sums3 != nullptr;
     f32x2 sig = {0.f, 0.f}, err = {0.f, 0.f};      // SQNR sums of this thread's outputs
     uint32_t tcount = 0, nstore = 0;
     bool ok = true;
-    // y_ref tiles of whole-tile units: chunk c of every such tile goes through buffer c % 2; all four
-    // are loaded (out-of-range parts read as zero), so the buffer phases advance regularly.  The
-    // epilogue of a split tail tile reads y_ref with plain loads.
+    // y_ref tiles of whole-tile units: chunk c of every such tile goes through buffer c % RB, loaded RB
+    // chunks ahead; all four are loaded (out-of-range parts read as zero), so the buffer phases advance
+    // regularly.  The epilogue of a split tail tile reads y_ref with plain loads.
     uint32_t nref[kEpiBufs] = {0u, 0u}, nused[kEpiBufs] = {0u, 0u};  // loads issued / consumed per buffer
     auto load_ref = [&](int tile_, int c_) {        // called by the whole warp; lane 0 issues
       const int m_ = tile_ % num_m, nn_ = tile_ / num_m;
-      uint64_t* bar = &bars->ref_full[ew][c_ & 1];
+      const int rb_ = c_ % L::RB;
+      uint64_t* bar = &bars->ref_full[ew][rb_];
       if (lane == 0) {
         mbar_arrive_expect_tx(bar, kEpiStage);
-        tma_load_2d(rstage0 + (c_ & 1) * kEpiStage, &tmR, nn_ * BN + c_ * 32, m_ * 2 * BM + (int)rank * BM + quad * 32,
+        tma_load_2d(rstage0 + rb_ * kEpiStage, &tmR, nn_ * BN + c_ * 32, m_ * 2 * BM + (int)rank * BM + quad * 32,
                     bar);
       }
-      ++nref[c_ & 1];
+      ++nref[rb_];
     };
     // y (and acc_out) of one chunk: 32 rows from row0_ (this lane: t_) x 32 channels from o0; v the
     // outputs, a the raw accumulators
     auto store_chunk = [&](int o0, int row0_, int t_, const float (&v)[32], const float (&a)[32]) {
       if (o0 >= d_out || row0_ >= n) return;      // warp-uniform: nothing of this chunk is in range
       if (use_tma_store) {
-        uint8_t* buf = stage0 + (nstore % kEpiBufs) * kEpiStage;
-        if (lane == 0) bulk_wait_read_le1();  // the store issued two chunks ago has read this buffer
+        uint8_t* buf = stage0 + (nstore % L::EB) * kEpiStage;
+        if (lane == 0) {                       // the store issued EB chunks ago has read this buffer
+          if (L::EB == 1)
+            bulk_wait_read_all();
+          else
+            bulk_wait_read_le1();
+        }
         __syncwarp();
 #pragma unroll
         for (int q = 0; q < 8; ++q)  // row `lane`, 16-byte chunk q at q ^ (lane % 8)
@@ -509,10 +577,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     // this pair's first whole tile comes after its split part, if it has one; y_ref loads and uses
     // count whole tiles only (fcount)
     const int u_full0 = pair < n_split ? pair + num_pairs : pair;
-    if (with_ref && u_full0 < total_units) {
-      load_ref(u_full0 - n_split, 0);
-      load_ref(u_full0 - n_split, 1);
-    }
+    if (with_ref && u_full0 < total_units)
+      for (int c0 = 0; c0 < L::RB; ++c0) load_ref(u_full0 - n_split, c0);
     uint32_t fcount = 0;
     int split_state = 0;                            // this pair's split part: 1 partials out, 2 share done
     int u = pair;
@@ -523,13 +589,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const int row0 = m * 2 * BM + (int)rank * BM + quad * 32;
       const int t = row0 + lane;
       const float sxt = (t < n) ? sx[t] * kAccScale : 0.f;
-      __syncwarp();
+      if constexpr (!E8) {
+        __syncwarp();
 #pragma unroll
-      for (int i = 0; i < BN / 32; ++i) {  // this tile's output-channel steps, staged once per unit
-        const int o = nn * BN + 32 * i + lane;
-        wsc[32 * i + lane] = (o < d_out) ? sw[o] : 0.f;
+        for (int i = 0; i < BN / 32; ++i) {  // this tile's output-channel steps, staged once per unit
+          const int o = nn * BN + 32 * i + lane;
+          wsc[32 * i + lane] = (o < d_out) ? sw[o] : 0.f;
+        }
+        __syncwarp();
       }
-      __syncwarp();
       if (!(ok = mbar_wait_bounded(&bars->acc_full[ab], (tcount >> 1) & 1, abort_flag, __LINE__))) break;
       __syncwarp();
       tc_fence_after();
@@ -547,18 +615,28 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           }
           const int o0 = nn * BN + c * 32;
           float a[32], v[32];
+          if constexpr (E8) {                    // the chunk's 32 channel steps, one per lane
+            const float swl = (o0 + lane < d_out) ? __ldg(sw + o0 + lane) : 0.f;
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            a[i] = __uint_as_float(r[i]);
-            v[i] = a[i] * sxt * wsc[c * 32 + i];
+            for (int i = 0; i < 32; ++i) {
+              a[i] = __uint_as_float(r[i]);
+              v[i] = a[i] * sxt * __shfl_sync(0xFFFFFFFFu, swl, i);
+            }
+          } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              a[i] = __uint_as_float(r[i]);
+              v[i] = a[i] * sxt * wsc[c * 32 + i];
+            }
           }
           if (with_ref) {
             // SQNR sums (Sec. 2, Eq. 1) from the y_ref tile of this chunk; out-of-range entries are zero
             // on both sides.  Squares are summed in fp32 over the chunk's 32 values, then as float pairs.
-            const uint32_t use = 2 * fcount + (c >> 1);  // the use-th load into buffer c % 2
-            if (!(ok = mbar_wait_bounded(&bars->ref_full[ew][c & 1], use & 1, abort_flag, __LINE__))) break;
-            ++nused[c & 1];
-            const uint8_t* rb = rstage0 + (c & 1) * kEpiStage + lane * 128;
+            const int rbuf = c % L::RB;
+            const uint32_t use = (BN / 32 / L::RB) * fcount + c / L::RB;  // the use-th load into buffer rbuf
+            if (!(ok = mbar_wait_bounded(&bars->ref_full[ew][rbuf], use & 1, abort_flag, __LINE__))) break;
+            ++nused[rbuf];
+            const uint8_t* rb = rstage0 + rbuf * kEpiStage + lane * 128;
             float s_run = 0.f, e_run = 0.f;
 #pragma unroll
             for (int q = 0; q < 8; ++q) {
@@ -569,8 +647,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             }
             sig = f2_add(sig, s_run);
             err = f2_add(err, e_run);
-            // refill this buffer with the chunk two ahead (this tile or the next: whole tiles follow)
-            int nu = u, nc = c + 2;
+            // refill this buffer with the chunk RB ahead (this tile or the next: whole tiles follow)
+            int nu = u, nc = c + L::RB;
             if (nc >= BN / 32) {
               nc -= BN / 32;
               nu = u + num_pairs;
@@ -621,7 +699,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     if (with_ref) {
       // y_ref loads issued but not consumed (only after a wait gave up) land before the CTA exits
       volatile int no_abort = 0;
-      for (int bb = 0; bb < kEpiBufs; ++bb)
+      for (int bb = 0; bb < L::RB; ++bb)
         if (nref[bb] > nused[bb]) mbar_wait_bounded(&bars->ref_full[ew][bb], (nref[bb] - 1) & 1, &no_abort);
       sig = f2_warp_sum(sig);
       err = f2_warp_sum(err);
@@ -638,8 +716,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     }
     if (lane == 0) bulk_wait_all();
     __syncwarp();
-  } else if (warp >= kDecWarp0) {
-    // ---------------------------------------------------------------- decode
+  } else if (!E8 && warp >= kDecWarp0) {
+    // ---------------------------------------------------------------- decode (packed codes)
     // Two groups of four warps (one warp per TMEM lane quadrant each) decode alternate K steps: the
     // decode of one step is latency-bound (shared-memory loads, tensor-memory stores and their wait,
     // the proxy fence), so two steps are kept in flight.
@@ -719,7 +797,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   if (bars->abort && tid == 0) report(status, timeout_bits(kWhereGemm, bars->abort));
   if (warp == 0) {
     tc_fence_after();
-    tmem_dealloc_pair(tmem, kTmemCols);
+    tmem_dealloc_pair(tmem, L::kTmem);
   }
 }
 
@@ -774,8 +852,10 @@ int num_sms() {
 }
 
 // Whether a cooperative launch of `pairs` CTA pairs of the GEMM kernel fits on this device (checked
-// once per process, on the first device asked).
+// once per process and operand format, on the first device asked).
+template <bool E8>
 bool split_launch_ok(int64_t pairs) {
+  using L = GemmLayout<E8>;
   static int ok = -1;
   static std::mutex mu;
   std::lock_guard<std::mutex> lock(mu);
@@ -784,14 +864,14 @@ bool split_launch_ok(int64_t pairs) {
     ok = 0;
     if (cudaGetDevice(&dev) == cudaSuccess &&
         cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) == cudaSuccess && coop &&
-        cudaFuncSetAttribute(w4a4_gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes) ==
-            cudaSuccess) {
+        cudaFuncSetAttribute(w4a4_gemm_tc_kernel<E8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)L::kSmemBytes) == cudaSuccess) {
       cudaLaunchConfig_t cfg;
       memset(&cfg, 0, sizeof(cfg));
       cfg.gridDim = dim3((unsigned)(2 * pairs), 1, 1);
       cfg.blockDim = dim3(kThreads, 1, 1);
-      cfg.dynamicSmemBytes = kSmemBytes;
-      if (cudaOccupancyMaxActiveClusters(&clusters, w4a4_gemm_tc_kernel, &cfg) == cudaSuccess && clusters >= pairs)
+      cfg.dynamicSmemBytes = L::kSmemBytes;
+      if (cudaOccupancyMaxActiveClusters(&clusters, w4a4_gemm_tc_kernel<E8>, &cfg) == cudaSuccess && clusters >= pairs)
         ok = 1;
     }
     cudaGetLastError();
@@ -799,14 +879,14 @@ bool split_launch_ok(int64_t pairs) {
   return ok == 1;
 }
 
-}  // namespace
-
 // y_ref != nullptr: the epilogue also forms the SQNR sums of y against y_ref and writes
 // sums3 = {sum y_ref^2, sum (y_ref - y)^2, dB} (sums3 needs no zeroing).  Needs d_out % 4 == 0
-// (TMA row pitch).
-cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
-                                int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, const float* y_ref,
-                                double* sums3, uint32_t* status, cudaStream_t stream) {
+// (TMA row pitch).  E8: xq and wq hold one code per byte, else SM4x8 (two per byte).
+template <bool E8>
+cudaError_t launch_gemm_tc(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
+                           int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, const float* y_ref, double* sums3,
+                           uint32_t* status, cudaStream_t stream) {
+  using L = GemmLayout<E8>;
   CUtensorMap ty, ta, tb, tr;
   memset(&ty, 0, sizeof(ty));
   memset(&tr, 0, sizeof(tr));
@@ -816,12 +896,14 @@ cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_
     if (d_out % 4 != 0 || !sums3 || !make_output_map(&tr, const_cast<float*>(y_ref), n, d_out))
       return cudaErrorInvalidValue;
   }
-  if (!make_packed_map(&ta, xq, n, d_in / 2, BM) || !make_packed_map(&tb, wq, d_out, d_in / 2, BNC))
+  const int64_t row_bytes = E8 ? d_in : d_in / 2;
+  if (!make_packed_map(&ta, xq, n, row_bytes, BM) || !make_packed_map(&tb, wq, d_out, row_bytes, BNC))
     return cudaErrorInvalidValue;
   static std::once_flag attr_once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(attr_once, [] {
-    attr_err = cudaFuncSetAttribute(w4a4_gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+    attr_err = cudaFuncSetAttribute(w4a4_gemm_tc_kernel<E8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)L::kSmemBytes);
   });
   if (attr_err != cudaSuccess) return attr_err;
   const int64_t tiles = ((n + 2 * BM - 1) / (2 * BM)) * ((d_out + BN - 1) / BN);
@@ -831,7 +913,7 @@ cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_
   // most half full (the parts wait for one another: only with a cooperative launch)
   const int64_t tail = tiles >= pairs_max ? tiles % pairs_max : tiles;
   int split = 1;
-  if (tail > 0 && tail <= kMaxSplitTiles && 2 * tail <= pairs_max && split_launch_ok(pairs_max))
+  if (tail > 0 && tail <= kMaxSplitTiles && 2 * tail <= pairs_max && split_launch_ok<E8>(pairs_max))
     while (2 * split <= kMaxSplit && 2 * split * tail <= pairs_max && 2 * split <= num_k) split *= 2;
   // a single partial wave has no whole tiles to hide the parts' exchange behind: split it only
   // when that saves ten K steps or more
@@ -850,7 +932,7 @@ cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_
   memset(&cfg, 0, sizeof(cfg));
   cfg.gridDim = dim3((unsigned)grid, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.dynamicSmemBytes = L::kSmemBytes;
   cfg.stream = stream;
   cudaLaunchAttribute attrs[2];
   attrs[0] = pdl_attr();
@@ -858,9 +940,47 @@ cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_
   attrs[1].val.cooperative = 1;
   cfg.attrs = attrs;
   cfg.numAttrs = split > 1 ? 2 : 1;
-  return cudaLaunchKernelEx(&cfg, w4a4_gemm_tc_kernel, ty, ta, tb, tr, y_ref, const_cast<double*>(sums), slot, sx, sw,
-                            (int)n, (int)d_in, (int)d_out, y, acc_out, use_tma, (int)num_full, split, split_slot,
+  return cudaLaunchKernelEx(&cfg, w4a4_gemm_tc_kernel<E8>, ty, ta, tb, tr, y_ref, const_cast<double*>(sums), slot, sx,
+                            sw, (int)n, (int)d_in, (int)d_out, y, acc_out, use_tma, (int)num_full, split, split_slot,
                             status);
+}
+
+}  // namespace
+
+cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
+                                int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, const float* y_ref,
+                                double* sums3, uint32_t* status, cudaStream_t stream) {
+  return launch_gemm_tc<false>(xq, sx, wq, sw, n, d_in, d_out, y, acc_out, y_ref, sums3, status, stream);
+}
+
+cudaError_t launch_w4a4_gemm_tc_e8(const uint8_t* xq8, const float* sx, const uint8_t* wq8, const float* sw, int64_t n,
+                                   int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, const float* y_ref,
+                                   double* sums3, uint32_t* status, cudaStream_t stream) {
+  return launch_gemm_tc<true>(xq8, sx, wq8, sw, n, d_in, d_out, y, acc_out, y_ref, sums3, status, stream);
+}
+
+// SM4x8 codes -> byte codes.  Every 16 packed bytes (32 codes of a row) become 32 bytes: the masks of
+// the format give the E4M3 bytes of codes 0..3 and 4..7 of each word directly.
+__global__ void __launch_bounds__(256) codes_to_e4m3_kernel(const uint4* __restrict__ in, uint4* __restrict__ out,
+                                                            int64_t chunks) {
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < chunks; i += stride) {
+    const uint4 w = __ldcs(in + i);
+    out[2 * i] = make_uint4(sm4_lo(w.x), sm4_hi(w.x), sm4_lo(w.y), sm4_hi(w.y));
+    out[2 * i + 1] = make_uint4(sm4_lo(w.z), sm4_hi(w.z), sm4_lo(w.w), sm4_hi(w.w));
+  }
+}
+
+// rows x d codes (d a multiple of 32): codes [rows][d/2] -> out [rows][d].
+cudaError_t launch_codes_to_e4m3(const uint8_t* codes, int64_t rows, int64_t d, uint8_t* out, cudaStream_t stream) {
+  const int64_t chunks = rows * (d / 32);
+  if (chunks == 0) return cudaSuccess;
+  const int64_t cap = (int64_t)num_sms() * 8;
+  const int64_t blocks = (chunks + 255) / 256;
+  note_launch();
+  codes_to_e4m3_kernel<<<(unsigned)(blocks < cap ? blocks : cap), 256, 0, stream>>>(
+      reinterpret_cast<const uint4*>(codes), reinterpret_cast<uint4*>(out), chunks);
+  return cudaGetLastError();
 }
 
 }  // namespace cat

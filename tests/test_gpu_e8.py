@@ -1,0 +1,112 @@
+"""Byte codes (one E4M3 byte per INT4 code) and the GEMM that reads them without a decode step,
+through the C ABI: the conversion is bit-exact against the byte encoding written out here, the
+accumulators match the oracle's integer GEMM bit for bit, and y and the SQNR sums are identical to
+the SM4x8 GEMM's (same exact accumulators, same scaling)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import sm4x8
+import workloads as WL
+
+pytestmark = pytest.mark.gpu
+
+cat = pytest.importorskip("paper_2603_04359_gb300")
+DEV = "cuda"
+
+
+def byte_codes(q: np.ndarray) -> np.ndarray:
+    """The E4M3 byte of the subnormal q * 2^-9: sign bit 7, magnitude in bits 0-2."""
+    q = np.asarray(q, dtype=np.int64)
+    return (np.where(q < 0, 0x80, 0) | np.abs(q)).astype(np.uint8)
+
+
+def rel_fro(a, b):
+    return float(np.linalg.norm(np.asarray(a, np.float64) - b) / max(np.linalg.norm(b), 1e-300))
+
+
+@pytest.mark.parametrize("rows,d", [(1, 32), (77, 4096), (1000, 160), (3, 262144)])
+def test_codes_to_e4m3(rows, d):
+    rng = np.random.default_rng(rows + d)
+    q = WL.random_codes(rng, (rows, d)).astype(np.int64)
+    q[0, :15] = np.arange(-7, 8)                           # every code value
+    out = cat.cat_codes_to_e4m3(torch.from_numpy(sm4x8.pack(q)).to(DEV))
+    np.testing.assert_array_equal(out.cpu().numpy(), byte_codes(q))
+
+
+E8_SHAPES = [
+    (1, 64, 8), (17, 96, 33), (32, 384, 300),            # n <= 32: one partly filled 256-row tile
+    (33, 128, 256), (128, 256, 256), (129, 160, 300), (300, 384, 520), (257, 4096, 64),
+    (512, 1024, 1024), (1024, 512, 6144),                # several tiles per pair
+    (256, 1024, 9984), (300, 2048, 5030),                # a last wave split along K into 4 / 8 parts
+    (2048, 4096, 6144),                                  # the QKV layer's shape: 2.05 waves, split tail
+]
+
+
+@pytest.mark.parametrize("n,d_in,d_out", E8_SHAPES)
+def test_w4a4_linear_e8_exact(n, d_in, d_out):
+    rng = np.random.default_rng(n * 1000 + d_in + d_out)
+    qx = WL.random_codes(rng, (n, d_in)).astype(np.int64)
+    qw = WL.random_codes(rng, (d_out, d_in)).astype(np.int64)
+    sx = rng.uniform(0.01, 2.0, n).astype(np.float32)
+    sw = rng.uniform(0.001, 0.1, d_out).astype(np.float32)
+    sx_d, sw_d = torch.from_numpy(sx).to(DEV), torch.from_numpy(sw).to(DEV)
+    xq8 = torch.from_numpy(byte_codes(qx)).to(DEV)
+    wq8 = cat.cat_codes_to_e4m3(torch.from_numpy(sm4x8.pack(qw)).to(DEV))   # the weights' preparation
+    acc = torch.empty((n, d_out), dtype=torch.int32, device=DEV)
+    y = cat.cat_w4a4_linear_e8(xq8, sx_d, wq8, sw_d, acc_out=acc)
+    ref_acc = O.int_gemm(qx, qw)
+    np.testing.assert_array_equal(acc.cpu().numpy(), ref_acc)
+    ref_y = O.dequantize_output(ref_acc, sx.astype(np.float64), sw.astype(np.float64))
+    assert rel_fro(y.cpu().numpy(), ref_y) < 1e-6
+    if n > 32:                                          # the SM4x8 tile GEMM: the same y, bit for bit
+        y4 = cat.cat_w4a4_linear(torch.from_numpy(sm4x8.pack(qx)).to(DEV), sx_d,
+                                 torch.from_numpy(sm4x8.pack(qw)).to(DEV), sw_d)
+        assert torch.equal(y, y4)
+    assert cat.cat_device_status()[0] == 0
+
+
+@pytest.mark.parametrize("n,d_in", [(200, 14336), (40, 4096)])
+def test_w4a4_linear_e8_extreme_accumulators(n, d_in):
+    d_out = 64
+    qx = np.full((n, d_in), 7, dtype=np.int64)
+    qx[1::2] = -7
+    qw = np.full((d_out, d_in), 7, dtype=np.int64)
+    qw[3, : d_in // 2] = -7                       # cancels to zero
+    qw[5, -300:] = np.arange(300) % 3 - 1         # small codes after a large prefix
+    ones = torch.ones(max(n, d_out), dtype=torch.float32, device=DEV)
+    acc = torch.empty((n, d_out), dtype=torch.int32, device=DEV)
+    cat.cat_w4a4_linear_e8(torch.from_numpy(byte_codes(qx)).to(DEV), ones[:n].contiguous(),
+                           torch.from_numpy(byte_codes(qw)).to(DEV), ones[:d_out].contiguous(), acc_out=acc)
+    ref = O.int_gemm(qx, qw)
+    assert np.abs(ref).max() == 49 * d_in
+    np.testing.assert_array_equal(acc.cpu().numpy(), ref)
+
+
+@pytest.mark.parametrize("n,d_in,d_out", [(300, 1024, 520), (513, 512, 256), (257, 4096, 130), (16, 1024, 200),
+                                          (1024, 512, 6144), (300, 2048, 5032)])
+def test_w4a4_linear_sqnr_e8(n, d_in, d_out):
+    """y equals cat_w4a4_linear_e8's bit for bit; the sums match the oracle's over the same outputs and,
+    for n > 32, the SM4x8 call's."""
+    rng = np.random.default_rng(n + 7 * d_in + 13 * d_out)
+    qx = WL.random_codes(rng, (n, d_in)).astype(np.int64)
+    qw = WL.random_codes(rng, (d_out, d_in)).astype(np.int64)
+    sx = rng.uniform(0.01, 2.0, n).astype(np.float32)
+    sw = rng.uniform(0.001, 0.1, d_out).astype(np.float32)
+    sx_d, sw_d = torch.from_numpy(sx).to(DEV), torch.from_numpy(sw).to(DEV)
+    xq8, wq8 = torch.from_numpy(byte_codes(qx)).to(DEV), torch.from_numpy(byte_codes(qw)).to(DEV)
+    y_plain = cat.cat_w4a4_linear_e8(xq8, sx_d, wq8, sw_d)
+    y_ref = (y_plain.double() + torch.randn(n, d_out, device=DEV, dtype=torch.float64) * 0.05).float().contiguous()
+    for rep in range(2):                                   # twice: the sums restart from zero each call
+        y, out3 = cat.cat_w4a4_linear_sqnr_e8(xq8, sx_d, wq8, sw_d, y_ref)
+        assert torch.equal(y, y_plain)
+        sig, err = O.sqnr_sums(y_ref.cpu().numpy(), y.cpu().numpy())
+        o = out3.cpu().numpy()
+        assert abs(o[0] - sig) <= 1e-6 * sig and abs(o[1] - err) <= 1e-6 * err
+        assert abs(o[2] - 10 * np.log10(sig / err)) < 1e-5
+    if n > 32:
+        _, out4 = cat.cat_w4a4_linear_sqnr(torch.from_numpy(sm4x8.pack(qx)).to(DEV), sx_d,
+                                           torch.from_numpy(sm4x8.pack(qw)).to(DEV), sw_d, y_ref)
+        assert torch.equal(out3, out4)
+    assert cat.cat_device_status()[0] == 0
