@@ -3,10 +3,13 @@
 
 A step is one pass of the whole hot path over one batch of synthetic input, through the C ABI:
   cat_calib_cov (calibration Sigma_x blocks of the step's calibration tokens)
-  -> cat_transform_quantize_act (x' = T x, per-token INT4)
-  -> cat_w4a4_linear_sqnr (integer GEMM + dequantization, with the SQNR sums against the
-     full-precision output formed in the GEMM epilogue).
-The weights are prepared once before timing (cat_quantize_weights, an offline step).  The
+  -> cat_transform_quantize_act_e8 (x' = T x, per-token INT4 codes, one byte per code)
+  -> cat_w4a4_linear_sqnr_e8 (integer GEMM + dequantization on the byte codes, with the SQNR sums
+     against the full-precision output formed in the GEMM epilogue).
+For decode batches (n <= 32 tokens) the codes stay SM4x8-packed (cat_transform_quantize_act_split,
+cat_w4a4_linear_sqnr): that GEMM streams the weights and reads half the bytes.
+The weights are prepared once before timing (cat_quantize_weights and, for the byte-code GEMM,
+cat_codes_to_e4m3: offline steps).  The
 full-precision reference y = W x used by the SQNR is computed once by the harness (fp32 GEMM,
 TF32 off) and is an input of every step.
 
@@ -297,17 +300,19 @@ class BufferSet:
     """One copy of every operand of a step.  The timed graphs cycle through several sets whose
     total size exceeds the L2 cache, so no step finds its inputs (weights included) in L2."""
 
-    def __init__(self, cat, x, xc, y_ref, T, Wq, sw, k, dev):
+    def __init__(self, cat, x, xc, y_ref, T, Wq, sw, k, dev, e8=False):
         n, d_in = x.shape
         d_out = Wq.shape[0]
         self.x, self.xc, self.y_ref = x.clone(), xc.clone(), y_ref.clone()
-        self.T, self.Wq, self.sw = T.clone(), Wq.clone(), sw.clone()
+        self.T, self.sw = T.clone(), sw.clone()
+        # byte codes: the weights' codes converted once (offline), the activations' codes one byte each
+        self.Wq = cat.cat_codes_to_e4m3(Wq) if e8 else Wq.clone()
         # T's bf16 planes, split once per layer (the tensor-core transform's k = 64, 128)
         self.T_planes = (cat.cat_split_transform(self.T, k)
                          if (x.dtype == torch.bfloat16 and cat.cat_split_transform_bytes(self.T.shape[0] * k, k) > 0)
                          else None)
         self.sigma = torch.empty((d_in // k, k, k), dtype=torch.float64, device=dev)
-        self.xq = torch.empty((n, d_in // 2), dtype=torch.uint8, device=dev)
+        self.xq = torch.empty((n, d_in if e8 else d_in // 2), dtype=torch.uint8, device=dev)
         self.sx = torch.empty((n,), dtype=torch.float32, device=dev)
         self.y = torch.empty((n, d_out), dtype=torch.float32, device=dev)
         self.out3 = torch.empty((3,), dtype=torch.float64, device=dev)
@@ -489,19 +494,30 @@ def measure_config(cat, cfg, k, kind, args, dev, world, rank, with_e2e, sweep=Fa
     sweep_res = transform_sweep(cat, L, x, W, xc, y_ref) if sweep else None
     del W
     l2 = torch.cuda.get_device_properties(dev).L2_cache_size
-    first = BufferSet(cat, x, xc, y_ref, T, Wq, sw, k, dev)
+    e8 = n > DECODE_TOKENS                                  # prefill: byte codes; decode: SM4x8 codes
+    first = BufferSet(cat, x, xc, y_ref, T, Wq, sw, k, dev, e8)
     n_sets = max(2, -(-3 * l2 // first.nbytes()))         # >= 3x L2 of operands in rotation
-    sets = [first] + [BufferSet(cat, x, xc, y_ref, T, Wq, sw, k, dev) for _ in range(n_sets - 1)]
+    sets = [first] + [BufferSet(cat, x, xc, y_ref, T, Wq, sw, k, dev, e8) for _ in range(n_sets - 1)]
     del x, xc, y_ref, T, Wq, sw, sigma
     stream = torch.cuda.current_stream(dev)
 
-    calls = {
-        "cat_calib_cov": lambda b: cat.cat_calib_cov(b.xc, k, out=b.sigma),
-        "cat_transform_quantize_act": lambda b: cat.cat_transform_quantize_act_split(b.x, b.T, b.T_planes, k, xq=b.xq,
-                                                                                     x_scale=b.sx),
-        # the integer GEMM, dequantization and SQNR sums (fused in the GEMM epilogue)
-        "cat_w4a4_linear_sqnr": lambda b: cat.cat_w4a4_linear_sqnr(b.xq, b.sx, b.Wq, b.sw, b.y_ref, y=b.y, out=b.out3),
-    }
+    if e8:
+        calls = {
+            "cat_calib_cov": lambda b: cat.cat_calib_cov(b.xc, k, out=b.sigma),
+            "cat_transform_quantize_act_e8": lambda b: cat.cat_transform_quantize_act_e8(b.x, b.T, b.T_planes, k,
+                                                                                         xq8=b.xq, x_scale=b.sx),
+            # the integer GEMM, dequantization and SQNR sums (fused in the GEMM epilogue)
+            "cat_w4a4_linear_sqnr_e8": lambda b: cat.cat_w4a4_linear_sqnr_e8(b.xq, b.sx, b.Wq, b.sw, b.y_ref, y=b.y,
+                                                                             out=b.out3),
+        }
+    else:
+        calls = {
+            "cat_calib_cov": lambda b: cat.cat_calib_cov(b.xc, k, out=b.sigma),
+            "cat_transform_quantize_act": lambda b: cat.cat_transform_quantize_act_split(b.x, b.T, b.T_planes, k,
+                                                                                         xq=b.xq, x_scale=b.sx),
+            "cat_w4a4_linear_sqnr": lambda b: cat.cat_w4a4_linear_sqnr(b.xq, b.sx, b.Wq, b.sw, b.y_ref, y=b.y,
+                                                                       out=b.out3),
+        }
 
     def step(b):
         for fn in calls.values():
@@ -526,7 +542,10 @@ def measure_config(cat, cfg, k, kind, args, dev, world, rank, with_e2e, sweep=Fa
     g_step, launches = capture(lambda: [step(sets[i % n_sets]) for i in range(args.steps)])
     alone = dict(calls)
     # the GEMM without the SQNR sums (not part of the step): the decode roofline is the weight stream's
-    alone["cat_w4a4_linear (alone)"] = lambda b: cat.cat_w4a4_linear(b.xq, b.sx, b.Wq, b.sw, y=b.y)
+    if e8:
+        alone["cat_w4a4_linear_e8 (alone)"] = lambda b: cat.cat_w4a4_linear_e8(b.xq, b.sx, b.Wq, b.sw, y=b.y)
+    else:
+        alone["cat_w4a4_linear (alone)"] = lambda b: cat.cat_w4a4_linear(b.xq, b.sx, b.Wq, b.sw, y=b.y)
     g_calls = {name: capture(lambda fn=fn: [fn(sets[i % n_sets]) for i in range(args.steps)])[0]
                for name, fn in alone.items()}
     for _ in range(2):
@@ -643,7 +662,7 @@ def roofline_of(cfg, res, steps):
     n, d_in, d_out = res["n"], res["d_in"], res["d_out"]
     decode = n <= DECODE_TOKENS
     call_ms = res["call_ms"]
-    gemm_ms = call_ms["cat_w4a4_linear (alone)" if decode else "cat_w4a4_linear_sqnr"]
+    gemm_ms = call_ms["cat_w4a4_linear (alone)" if decode else "cat_w4a4_linear_sqnr_e8"]
     peaks = measured_peaks()
     fp8_peak = peaks["bf16_tflops"] * FP8_PER_BF16
     gemm_tflops = 2.0 * n * d_in * d_out / (gemm_ms / 1e3) / 1e12
@@ -667,7 +686,8 @@ def roofline_of(cfg, res, steps):
         roof = {"bound": "tensor", "achieved": gemm_tflops, "peak": fp8_peak, "unit": "TFLOP/s",
                 "frac": gemm_tflops / fp8_peak, "traffic": traffic,
                 "algorithmic_ops": 2 * n * d_in * d_out,
-                "kernel": "w4a4_gemm_tc (cat_w4a4_linear_sqnr, SQNR sums in the epilogue)", "timing": timing,
+                "kernel": "w4a4_gemm_tc_kernel<E8> (cat_w4a4_linear_sqnr_e8: byte codes, SQNR sums in the "
+                          "epilogue)", "timing": timing,
                 "peak_source": f"{peaks['source']} bf16 {peaks['bf16_tflops']} TFLOP/s x {FP8_PER_BF16} "
                                "(the FP8 engine the GEMM runs on, nominal FP8/BF16 ratio)",
                 "peak_note": "sm_103a has no integer tcgen05 MMA: INT4 codes run exactly as E4M3 operands on the "

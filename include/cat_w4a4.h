@@ -262,6 +262,19 @@ cat_status cat_w4a4_linear_sqnr(const uint8_t* xq, const float* x_scale, const u
 cat_status cat_codes_to_e4m3(const uint8_t* codes, int64_t rows, int64_t d, uint8_t* out, cat_stream_t stream);
 
 /*
+ * cat_transform_quantize_act_e8 -- cat_transform_quantize_act_split with byte codes out (Sec. 3 Eq. 5:
+ * x' = T x; Sec. 2 Lemma 2 range, Sec. 6 round to nearest).
+ *   Arguments as cat_transform_quantize_act_split, except
+ *   xq8  out, device [n][d_in] bytes: the codes of x' as byte codes.
+ *   x_scale and the codes are those cat_transform_quantize_act_split writes (the same code decisions).
+ *   bf16 rows on the fused tensor-core kernel write the bytes directly; elsewhere the SM4x8 codes go
+ *   to stream-ordered scratch (n * d_in / 2 bytes, cudaMallocAsync) and are converted.
+ */
+cat_status cat_transform_quantize_act_e8(const void* x, cat_dtype dtype, int64_t n, int64_t d_in, int32_t k,
+                                         const float* T_blocks, const uint8_t* T_planes, uint8_t* xq8, float* x_scale,
+                                         cat_stream_t stream);
+
+/*
  * cat_w4a4_linear_e8 -- cat_w4a4_linear on byte codes (Sec. 3 Eq. 5).
  *   xq8 [n][d_in], Wq8 [d_out][d_in] byte codes; x_scale, w_scale, y, acc_out as cat_w4a4_linear.
  *   Same results as cat_w4a4_linear on the SM4x8 form of the same codes, for every n >= 1 (it

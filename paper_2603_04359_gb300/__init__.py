@@ -87,6 +87,7 @@ def load_library() -> ctypes.CDLL:
         "cat_quantize_weights_dp": ([P, I, I64, I64, I32, I, P, I64, P, I32, I32, P, P, P, P, P], I),
         "cat_linear_dp": ([P, I32, I32, P, P, P, I32, P, P, I64, I64, I64, P, P, P], I),
         "cat_codes_to_e4m3": ([P, I64, I64, P, P], I),
+        "cat_transform_quantize_act_e8": ([P, I, I64, I64, I32, P, P, P, P, P], I),
         "cat_w4a4_linear_e8": ([P, P, P, P, I64, I64, I64, P, P, P], I),
         "cat_w4a4_linear_sqnr_e8": ([P, P, P, P, I64, I64, I64, P, P, P, P], I),
     }
@@ -303,6 +304,26 @@ def cat_transform_quantize_act_split(x: torch.Tensor, T_blocks: torch.Tensor, T_
     _check("cat_transform_quantize_act_split", load_library().cat_transform_quantize_act_split(
         _ptr(x), _dtype(x), n, d_in, k, _ptr(T_blocks), _ptr(T_planes), _ptr(xq), _ptr(x_scale), _stream(x.device)))
     return xq, x_scale
+
+
+def cat_transform_quantize_act_e8(x: torch.Tensor, T_blocks: torch.Tensor, T_planes: Optional[torch.Tensor], k: int,
+                                  xq8: Optional[torch.Tensor] = None,
+                                  x_scale: Optional[torch.Tensor] = None) -> Tuple[torch.Tensor, torch.Tensor]:
+    """cat_transform_quantize_act_split with the codes as byte codes: (xq8 uint8 [n, d_in], x_scale [n])."""
+    _need(x, "x")
+    n, d_in = x.shape
+    if xq8 is None:
+        xq8 = torch.empty((n, d_in), dtype=torch.uint8, device=x.device)
+    if x_scale is None:
+        x_scale = torch.empty((n,), dtype=torch.float32, device=x.device)
+    _expect(T_blocks, "T_blocks", torch.float32, (d_in // k, k, k), x.device)
+    if T_planes is not None:
+        _expect(T_planes, "T_planes", torch.uint8, (cat_split_transform_bytes(d_in, k),), x.device)
+    _expect(xq8, "xq8", torch.uint8, (n, d_in), x.device)
+    _expect(x_scale, "x_scale", torch.float32, (n,), x.device)
+    _check("cat_transform_quantize_act_e8", load_library().cat_transform_quantize_act_e8(
+        _ptr(x), _dtype(x), n, d_in, k, _ptr(T_blocks), _ptr(T_planes), _ptr(xq8), _ptr(x_scale), _stream(x.device)))
+    return xq8, x_scale
 
 
 def cat_w4a4_linear(xq: torch.Tensor, x_scale: torch.Tensor, Wq: torch.Tensor, w_scale: torch.Tensor,

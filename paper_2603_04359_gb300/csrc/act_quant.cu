@@ -178,7 +178,7 @@ cudaError_t launch_transform_quantize_tc(const void* x, int64_t n, int64_t d, in
                                          uint32_t* status, cudaStream_t stream);
 
 cudaError_t launch_transform_quantize_tc_fused(const void* x, int64_t n, int64_t d, int k, const float* A,
-                                               const uint8_t* planes, uint32_t* amax, uint32_t* words,
+                                               const uint8_t* planes, uint32_t* amax, uint32_t* words, int e8,
                                                uint32_t* status, cudaStream_t stream);
 
 // planes (optional): T's pre-split bf16 planes (cat_split_transform), used by the tensor-core path.
@@ -189,7 +189,7 @@ cudaError_t launch_transform_quantize(const void* x, int dtype, int64_t n, int64
   if (transform_quantize_tc_supported(dtype, k, n, d)) {  // bf16 rows: tensor-core path
     uint32_t* amax = reinterpret_cast<uint32_t*>(scale);
     const cudaError_t ef = launch_transform_quantize_tc_fused(x, n, d, k, A, planes, amax,
-                                                              reinterpret_cast<uint32_t*>(codes), status, stream);
+                                                              reinterpret_cast<uint32_t*>(codes), 0, status, stream);
     if (ef != cudaErrorNotSupported) return ef;  // done (or failed) in one launch
     if (k != 256) {                               // k = 256 has the fused kernel only
       // two passes with the maxima in device scratch: pass 1 writes the steps
@@ -210,6 +210,17 @@ cudaError_t launch_transform_quantize(const void* x, int dtype, int64_t n, int64
   }
   if (dtype == 0) return launch_t(static_cast<const float*>(x), n, d, k, A, codes, scale, status, stream);
   return launch_t(static_cast<const __nv_bfloat16*>(x), n, d, k, A, codes, scale, status, stream);
+}
+
+// The same codes as byte codes ([n][d], one E4M3 byte per code), written by the fused tensor-core
+// kernel; cudaErrorNotSupported (nothing launched) where that kernel does not apply.
+cudaError_t launch_transform_quantize_e8(const void* x, int dtype, int64_t n, int64_t d, int k, const float* A,
+                                         uint8_t* codes8, float* scale, uint32_t* status, cudaStream_t stream,
+                                         const uint8_t* planes) {
+  if (n == 0) return cudaSuccess;
+  if (!transform_quantize_tc_supported(dtype, k, n, d)) return cudaErrorNotSupported;
+  return launch_transform_quantize_tc_fused(x, n, d, k, A, planes, reinterpret_cast<uint32_t*>(scale),
+                                            reinterpret_cast<uint32_t*>(codes8), 1, status, stream);
 }
 
 }  // namespace cat

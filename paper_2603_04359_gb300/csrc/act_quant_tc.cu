@@ -250,8 +250,9 @@ __device__ __forceinline__ uint32_t twos_to_sm(uint32_t w) {
 // qcode_exact out of line: the rare near-tie route then costs a call, not 32 inlined copies.
 __device__ __noinline__ int qcode_exact_call(float v, QRow qr) { return qcode_exact(v, qr, 7.0f); }
 
-// The four SM4x8 words of the codes of the 32 values v_e in tensor memory at taddr (this lane's row,
-// 32 columns) on the row described by qr (|v_e| <= max|v|); called by the whole warp.  Fast route:
+// The codes of the 32 values v_e in tensor memory at taddr (this lane's row, 32 columns) on the row
+// described by qr (|v_e| <= max|v|), as eight words of E4M3 code bytes (codes 4i .. 4i+3 in word i,
+// little-endian); called by the whole warp.  Fast route:
 // adding 1.5 * 2^23 to p = fl(v_e * inv) rounds it to an integer (half to even) that sits, two's
 // complement, in the low byte of the sum's bits; the bytes are gathered four to a word and turned
 // into sign-magnitude.  The products and sums run as f32x2 pairs, with the same rounding as the scalar
@@ -260,7 +261,7 @@ __device__ __noinline__ int qcode_exact_call(float v, QRow qr) { return qcode_ex
 // (qcode_exact): the values are not kept live across that rare branch, which leaves the fast route
 // its registers, and the branch costs about one exact decision rather than 32.
 // qr.inv == 0 (an all-zero or non-finite row): all codes 0.
-__device__ __forceinline__ uint4 quant_chunk(uint32_t taddr, const QRow& qr) {
+__device__ __forceinline__ void quant_chunk(uint32_t taddr, const QRow& qr, uint32_t (&out)[8]) {
   constexpr float kMagic = 12582912.0f;
   uint32_t bq[32];
   bool near = qr.exact;
@@ -301,18 +302,20 @@ __device__ __forceinline__ uint4 quant_chunk(uint32_t taddr, const QRow& qr) {
       }
     }
   }
-  if (qr.inv == 0.f) return make_uint4(0u, 0u, 0u, 0u);
-  uint32_t w[4];
+  const bool zero = qr.inv == 0.f;
 #pragma unroll
-  for (int g = 0; g < 4; ++g) {
-    const uint32_t* bg = bq + 8 * g;
-    const uint32_t lo =
+  for (int g = 0; g < 8; ++g) {
+    const uint32_t* bg = bq + 4 * g;
+    const uint32_t e =
         twos_to_sm(__byte_perm(__byte_perm(bg[0], bg[1], 0x0040), __byte_perm(bg[2], bg[3], 0x0040), 0x5410));
-    const uint32_t hi =
-        twos_to_sm(__byte_perm(__byte_perm(bg[4], bg[5], 0x0040), __byte_perm(bg[6], bg[7], 0x0040), 0x5410));
-    w[g] = lo | __funnelshift_l(hi, hi, 4);
+    out[g] = zero ? 0u : e;
   }
-  return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+// The four SM4x8 words of a chunk's 32 code bytes (codes 8g .. 8g+7 in word g).
+__device__ __forceinline__ uint4 sm4_words(const uint32_t (&e)[8]) {
+  return make_uint4(e[0] | __funnelshift_l(e[1], e[1], 4), e[2] | __funnelshift_l(e[3], e[3], 4),
+                    e[4] | __funnelshift_l(e[5], e[5], 4), e[6] | __funnelshift_l(e[7], e[7], 4));
 }
 
 // Running maximum of |v| over 32 values, on their bit patterns: for non-negative floats the bit
@@ -507,8 +510,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         } else {
           // the row's codes with the final maximum (|v * inv| <= 7 for a finite row; inv = 0 gives
           // 0 codes for an all-zero or non-finite row)
-          const uint4 w = quant_chunk(taddr, qr);
-          if (t < n) *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * K + c * 32) / 8) = w;
+          uint32_t e[8];
+          quant_chunk(taddr, qr, e);
+          if (t < n)
+            *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * K + c * 32) / 8) = sm4_words(e);
         }
       }
       tc_fence_before();
@@ -602,7 +607,8 @@ __device__ __forceinline__ int chunk_slot(int c, bool last) { return last ? (c +
 template <int N, int KD, bool WAVES>
 __device__ __forceinline__ void quantize_units(uint32_t tmem, uint8_t* smem, const FusedUnits& fu, int num_tiles,
                                                int n, int d, uint64_t* maxima_ready, uint64_t* tmem_free,
-                                               uint32_t* __restrict__ codes, volatile int* abort_flag, int slot) {
+                                               uint32_t* __restrict__ codes, int e8, volatile int* abort_flag,
+                                               int slot) {
   // unit j sits in tensor-memory slot j % U (phase (j / U) & 1 of the slot's barriers); with WAVES the
   // converter warps (slots 1 and 2) hand the slot back once their chunks of the unit are done
   using F = FusedCfg<N, KD, WAVES>;
@@ -628,8 +634,18 @@ __device__ __forceinline__ void quantize_units(uint32_t tmem, uint8_t* smem, con
 #pragma unroll 1
       for (int c = 0; c < N / 32; ++c) {
         if (chunk_slot(c, last) != slot) continue;
-        const uint4 w = quant_chunk(tmem + ((uint32_t)(quad * 32) << 16) + us * N + c * 32, qr);
-        if (t < n) *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * N + c * 32) / 8) = w;
+        uint32_t e[8];
+        quant_chunk(tmem + ((uint32_t)(quad * 32) << 16) + us * N + c * 32, qr, e);
+        if (t < n) {
+          if (e8) {                            // byte codes: 32 bytes of row t
+            uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<uint8_t*>(codes) + (int64_t)t * d + (int64_t)b * N +
+                                                  c * 32);
+            dst[0] = make_uint4(e[0], e[1], e[2], e[3]);
+            dst[1] = make_uint4(e[4], e[5], e[6], e[7]);
+          } else {
+            *reinterpret_cast<uint4*>(codes + (int64_t)t * words_per_row + ((int64_t)b * N + c * 32) / 8) = sm4_words(e);
+          }
+        }
       }
     }
     if (WAVES && slot != 0) {                  // the slot's tensor memory (and maxima) are free again
@@ -644,7 +660,7 @@ template <int N, int KD, bool WAVES>
 __global__ void __launch_bounds__(kThreads, 1)
     transform_quant_tc_fused_kernel(const __grid_constant__ CUtensorMap tmX, const float* __restrict__ A,
                                     const uint8_t* __restrict__ planes, int n, int d, int kb, float* __restrict__ scale,
-                                    uint32_t* __restrict__ codes, uint32_t* __restrict__ state,
+                                    uint32_t* __restrict__ codes, int e8, uint32_t* __restrict__ state,
                                     uint32_t* __restrict__ amax_sets, uint32_t* __restrict__ rec_sets,
                                     uint32_t* __restrict__ status) {
   // state: the slot's epoch, start counter and tiles per set; amax_sets: two sets of kAmaxRows row
@@ -922,7 +938,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         ++version;
       }
     }
-    quantize_units<N, KD, WAVES>(tmem, smem, fu, num_tiles, n, d, maxima_ready, tmem_free, codes, abort_flag,
+    quantize_units<N, KD, WAVES>(tmem, smem, fu, num_tiles, n, d, maxima_ready, tmem_free, codes, e8, abort_flag,
                                  1 + ((warp - kCvtWarp0) >> 2));
     tc_fence_before();
   } else if (warp >= kEpiWarp0) {
@@ -958,7 +974,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) mbar_arrive(&epi_done[j % U]);
     }
     if (!finite) report(status, kStatusNonFinite);
-    quantize_units<N, KD, WAVES>(tmem, smem, fu, num_tiles, n, d, maxima_ready, tmem_free, codes, abort_flag, 0);
+    quantize_units<N, KD, WAVES>(tmem, smem, fu, num_tiles, n, d, maxima_ready, tmem_free, codes, e8, abort_flag, 0);
     tc_fence_before();
   }
 
@@ -1094,7 +1110,7 @@ bool cooperative_ok() {
 
 template <int N, int KD>
 cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, int kb, const float* A, const uint8_t* planes,
-                           uint32_t* amax, uint32_t* words, uint32_t* status, cudaStream_t stream) {
+                           uint32_t* amax, uint32_t* words, int e8, uint32_t* status, cudaStream_t stream) {
   const int nb = (int)(d / N);                         // groups of N output channels
   const int tiles = (int)((n + TM - 1) / TM);
   const int64_t units = (int64_t)nb * tiles;
@@ -1159,9 +1175,9 @@ cudaError_t launch_fused_k(const __nv_bfloat16* x, int64_t n, int64_t d, int kb,
   note_launch();
   if (waves)
     return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<N, KD, true>, map, A, planes, (int)n, (int)d, kb,
-                              reinterpret_cast<float*>(amax), words, state, amax_sets, rec_sets, status);
+                              reinterpret_cast<float*>(amax), words, e8, state, amax_sets, rec_sets, status);
   return cudaLaunchKernelEx(&cfg, transform_quant_tc_fused_kernel<N, KD, false>, map, A, planes, (int)n, (int)d, kb,
-                            reinterpret_cast<float*>(amax), words, state, amax_sets, rec_sets, status);
+                            reinterpret_cast<float*>(amax), words, e8, state, amax_sets, rec_sets, status);
 }
 
 }  // namespace
@@ -1211,15 +1227,16 @@ cudaError_t launch_split_transform(const float* A, int64_t d, int k, uint8_t* pl
 namespace cat {
 // Both phases and the steps in one cooperative launch when every CTA's units fit in tensor memory
 // (the row maxima go to a slot of device scratch that the launch leaves zeroed); cudaErrorNotSupported
-// otherwise (the caller takes the two-pass path).
+// otherwise (the caller takes the two-pass path).  e8: the codes as bytes ([n][d], one E4M3 byte per
+// code) instead of SM4x8 words.
 cudaError_t launch_transform_quantize_tc_fused(const void* x, int64_t n, int64_t d, int k, const float* A,
-                                               const uint8_t* planes, uint32_t* amax, uint32_t* words,
+                                               const uint8_t* planes, uint32_t* amax, uint32_t* words, int e8,
                                                uint32_t* status, cudaStream_t stream) {
   const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
   const int KD = transform_tc_group(k, d);
-  if (KD == 64) return launch_fused_k<64, 64>(xb, n, d, k, A, planes, amax, words, status, stream);
-  if (KD == 128) return launch_fused_k<128, 128>(xb, n, d, k, A, planes, amax, words, status, stream);
-  if (KD == 256) return launch_fused_k<64, 256>(xb, n, d, k, A, planes, amax, words, status, stream);
+  if (KD == 64) return launch_fused_k<64, 64>(xb, n, d, k, A, planes, amax, words, e8, status, stream);
+  if (KD == 128) return launch_fused_k<128, 128>(xb, n, d, k, A, planes, amax, words, e8, status, stream);
+  if (KD == 256) return launch_fused_k<64, 256>(xb, n, d, k, A, planes, amax, words, e8, status, stream);
   return cudaErrorNotSupported;
 }
 }  // namespace cat

@@ -668,6 +668,40 @@ cat_status cat_codes_to_e4m3(const uint8_t* codes, int64_t rows, int64_t d, uint
   return ok();
 }
 
+cat_status cat_transform_quantize_act_e8(const void* x, cat_dtype dtype, int64_t n, int64_t d_in, int32_t k,
+                                         const float* T_blocks, const uint8_t* T_planes, uint8_t* xq8, float* x_scale,
+                                         cat_stream_t stream) {
+  if (dtype != CAT_F32 && dtype != CAT_BF16) return fail(CAT_ERR_INVALID_ARG, "unknown dtype");
+  if (n < 0) return fail(CAT_ERR_SHAPE, "n must be >= 0");
+  cat_status st = check_din(d_in);
+  if (st != CAT_OK) return st;
+  if (!valid_k(k) || d_in % k != 0) return fail(CAT_ERR_SHAPE, "k must be one of 16..256 (power of two) and divide d_in");
+  if (n == 0) return ok();
+  if (!x || !T_blocks || !xq8 || !x_scale) return fail(CAT_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(x) || !aligned16(T_blocks) || !aligned16(xq8) || !aligned16(x_scale) || (T_planes && !aligned16(T_planes)))
+    return fail(CAT_ERR_ALIGNMENT, "pointers must be 16-byte aligned");
+  if ((n + 63) / 64 > 0x7FFFFFFF) return fail(CAT_ERR_SHAPE, "n too large");
+  if ((st = check_device()) != CAT_OK) return st;
+  cudaError_t e;
+  uint32_t* status = status_word(&e);
+  if (!status) return cuda_fail(e, "status word");
+  cudaStream_t s = (cudaStream_t)stream;
+  const uint8_t* planes = cat::transform_tc_group(k, d_in) != 0 ? T_planes : nullptr;
+  e = cat::launch_transform_quantize_e8(x, (int)dtype, n, d_in, k, T_blocks, xq8, x_scale, status, s, planes);
+  if (e == cudaErrorNotSupported) {
+    // no kernel writes byte codes here: SM4x8 codes into stream-ordered scratch, then converted
+    uint8_t* tmp = nullptr;
+    if ((e = cudaMallocAsync((void**)&tmp, (size_t)n * (size_t)(d_in / 2), s)) != cudaSuccess)
+      return cuda_fail(e, "cudaMallocAsync");
+    e = cat::launch_transform_quantize(x, (int)dtype, n, d_in, k, T_blocks, tmp, x_scale, status, s, planes);
+    if (e == cudaSuccess) e = cat::launch_codes_to_e4m3(tmp, n, d_in, xq8, s);
+    const cudaError_t ef = cudaFreeAsync(tmp, s);
+    if (e == cudaSuccess) e = ef;
+  }
+  if (e != cudaSuccess) return cuda_fail(e, "cat_transform_quantize_act_e8 launch");
+  return ok();
+}
+
 cat_status cat_w4a4_linear_e8(const uint8_t* xq8, const float* x_scale, const uint8_t* Wq8, const float* w_scale,
                               int64_t n, int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, cat_stream_t stream) {
   if (n < 0 || d_out <= 0) return fail(CAT_ERR_SHAPE, "n must be >= 0 and d_out >= 1");

@@ -301,6 +301,9 @@ cudaError_t launch_calib_cov(const void* x, int dtype, int64_t n, int64_t d, int
 cudaError_t launch_transform_quantize(const void* x, int dtype, int64_t n, int64_t d, int k, const float* T,
                                       uint8_t* codes, float* scale, uint32_t* status, cudaStream_t stream,
                                       const uint8_t* planes = nullptr);
+cudaError_t launch_transform_quantize_e8(const void* x, int dtype, int64_t n, int64_t d, int k, const float* A,
+                                         uint8_t* codes8, float* scale, uint32_t* status, cudaStream_t stream,
+                                         const uint8_t* planes);
 cudaError_t launch_split_transform(const float* T, int64_t d, int k, uint8_t* planes, cudaStream_t stream);
 // the group width K of the tensor-core transform for block size k on d channels (0: none applies);
 // the pre-split planes take 6 d K bytes

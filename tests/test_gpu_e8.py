@@ -110,3 +110,38 @@ def test_w4a4_linear_sqnr_e8(n, d_in, d_out):
                                            torch.from_numpy(sm4x8.pack(qw)).to(DEV), sw_d, y_ref)
         assert torch.equal(out3, out4)
     assert cat.cat_device_status()[0] == 0
+
+
+# ------------------------------------------------------------------------------------------
+# cat_transform_quantize_act_e8: the same code decisions, written as byte codes
+# ------------------------------------------------------------------------------------------
+
+@pytest.mark.parametrize("n,d,k,dtype", [(67, 384, 128, "bf16"), (1000, 256, 128, "bf16"),      # fused, one wave
+                                         (2560, 4096, 128, "bf16"), (1300, 8192, 64, "bf16"),   # fused in waves
+                                         (300, 512, 32, "bf16"), (300, 192, 64, "bf16"),        # embedded, 64-wide
+                                         (2560, 4096, 256, "bf16"), (200, 512, 256, "bf16"),    # k = 256 quarters
+                                         (1100, 9920, 64, "bf16"), (520, 20480, 128, "bf16"),   # two passes + convert
+                                         (1300, 10240, 256, "bf16"),                             # SIMT + convert
+                                         (130, 256, 32, "f32"), (5, 64, 16, "bf16")])            # SIMT + convert
+def test_transform_quantize_act_e8(n, d, k, dtype):
+    """The byte codes are the byte form of cat_transform_quantize_act_split's SM4x8 codes and the steps
+    are the same, bit for bit; on the first shape also checked against the oracle directly."""
+    from test_gpu_parity import _cat_T, check_codes, to_dev
+    rng = np.random.default_rng(11 * n + d)
+    X = rng.standard_normal((n, d)) * rng.lognormal(0, 1.0, d)
+    X[0] = 0.0                       # all-zero token
+    X[min(2, n - 1)] *= 1e4          # a huge token
+    Xt = WL.cast(X, dtype)
+    T32 = _cat_T(rng, d, k)
+    Td = torch.from_numpy(T32).to(DEV)
+    planes = cat.cat_split_transform(Td, k) if (dtype == "bf16" and cat.cat_split_transform_bytes(d, k) > 0) else None
+    xq, sx = cat.cat_transform_quantize_act_split(to_dev(Xt), Td, planes, k)
+    xq8, sx8 = cat.cat_transform_quantize_act_e8(to_dev(Xt), Td, planes, k)
+    q = sm4x8.unpack(xq.cpu().numpy())
+    np.testing.assert_array_equal(xq8.cpu().numpy(), byte_codes(q))
+    assert torch.equal(sx, sx8)
+    if (n, d, k) == (67, 384, 128):
+        ref = O.transform_quantize_act(Xt.values, T32.astype(np.float64))
+        b = xq8.cpu().numpy().astype(np.int64)
+        check_codes(np.where(b & 0x80, -(b & 0x7F), b & 0x7F), ref.qx, ref.pre_x)
+    assert cat.cat_device_status()[0] == 0
