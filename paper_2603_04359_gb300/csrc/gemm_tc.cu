@@ -74,7 +74,6 @@ constexpr int kPFullPeriod = SP % kDecGroups == 0 ? SP : SP * kDecGroups;
 constexpr int kEpiWarp0 = 4, kEpiWarps = 4;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kAccCols = 2 * BN;       // two accumulators
-constexpr uint32_t kIdesc = idesc_e4m3_f32(2 * BM, BN);
 constexpr uint32_t kEpiStage = 32 * 32 * 4;                 // 32 rows x 32 fp32 columns, 4 KiB
 constexpr int kEpiBufs = 2;                                  // TMA-store staging buffers per epilogue warp
 constexpr uint32_t kPkOffset = SE * kStageB;                 // after the decoded B stages
@@ -85,22 +84,31 @@ constexpr uint32_t kBarBytes = 1024;                         // room reserved fo
 constexpr uint32_t kAtomA8 = BM * 128;      // one 128-code K atom of A (128 rows x 128 B)
 constexpr uint32_t kStageA8 = BM * BK;      // 32 KiB
 constexpr uint32_t kStage8 = kStageA8 + kStageB;   // 48 KiB
+constexpr int kStages8 = 4;                 // byte-code stages
+constexpr int kEpiBufs8 = 1;                // byte codes: y and y_ref staging buffers per epilogue warp
 // Shared memory and tensor memory of the two operand formats.  The byte-code stages leave room for
 // one y and one y_ref staging buffer per epilogue warp, and the output-channel steps of a chunk go
 // through registers instead of shared memory.
-template <bool E8>
+template <bool E8, int NB = BN>
 struct GemmLayout {
-  static constexpr int EB = E8 ? 1 : kEpiBufs;   // y staging buffers per epilogue warp
-  static constexpr int RB = E8 ? 1 : kEpiBufs;   // y_ref staging buffers per epilogue warp
-  static constexpr uint32_t kOperands = E8 ? SE * kStage8 : kPkOffset + SP * kPackedStage;
+  // byte codes at NB = 256: three 64 KB stages; NB = 128: kStages8 stages of 48 KB
+  static constexpr int S = E8 ? (NB == 256 ? 3 : kStages8) : SE;   // operand stages the MMA consumes
+  static constexpr uint32_t kStageOp = kStageA8 + (uint32_t)(NB / 2) * BK;
+  static constexpr int EB = E8 ? kEpiBufs8 : kEpiBufs;   // y staging buffers per epilogue warp
+  static constexpr int RB = E8 ? kEpiBufs8 : kEpiBufs;   // y_ref staging buffers per epilogue warp
+  static constexpr uint32_t kOperands = E8 ? S * kStageOp : kPkOffset + SP * kPackedStage;
   static constexpr uint32_t kEpiOffset = kOperands;
   static constexpr uint32_t kRefOffset = kEpiOffset + kEpiWarps * EB * kEpiStage;   // y_ref tiles (SQNR)
   static constexpr uint32_t kScaleOffset = kRefOffset + kEpiWarps * RB * kEpiStage;
-  static constexpr uint32_t kBarOffset = kScaleOffset + (E8 ? 0u : kEpiWarps * BN * 4);
+  static constexpr uint32_t kBarOffset = kScaleOffset + (E8 ? 0u : kEpiWarps * NB * 4);
   static constexpr uint32_t kBarRoom = E8 ? 512u : kBarBytes;
   static constexpr size_t kSmemBytes = kBarOffset + kBarRoom + 1024;  // + barriers + alignment slack
-  static constexpr uint32_t kTmem = E8 ? kAccCols : kTmemCols;
+  static constexpr uint32_t kTmem = E8 ? 2 * NB : kTmemCols;   // E8: the two accumulators
   static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+  static_assert(S <= SE && EB <= kEpiBufs && RB <= kEpiBufs, "barrier arrays");
+  static_assert(E8 || S % kDecGroups == 0, "a decode group's steps keep to the stages of one parity");
+  static_assert((E8 && (NB == 128 || NB == 256)) || NB == BN, "tile widths");
+  static_assert(kStageOp % 1024 == 0, "128B-swizzle alignment");
 };
 static_assert(kAccCols + SE * 64 <= kTmemCols, "tensor memory budget");
 static_assert(kPackedStage % 1024 == 0 && kAtomB % 1024 == 0 && kPackedA % 1024 == 0, "128B-swizzle alignment");
@@ -116,7 +124,8 @@ struct Bars {
   int abort;
   f32x2 sums[kEpiWarps][2];                      // SQNR sums of the epilogue warps
 };
-static_assert(sizeof(Bars) <= GemmLayout<false>::kBarRoom && sizeof(Bars) <= GemmLayout<true>::kBarRoom,
+static_assert(sizeof(Bars) <= GemmLayout<false>::kBarRoom && sizeof(Bars) <= GemmLayout<true>::kBarRoom &&
+                  sizeof(Bars) <= GemmLayout<true, 256>::kBarRoom,
               "barrier block must fit its reserved room");
 
 // ---- tensor-memory stores and the TMA store path -------------------------------------------
@@ -236,7 +245,7 @@ __device__ __forceinline__ Unit unit_at(int u, int num_full, int split, int num_
   return {num_full + u / split, part * num_k / split, (part + 1) * num_k / split, part};
 }
 
-template <bool E8>
+template <bool E8, int NB>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     w4a4_gemm_tc_kernel(const __grid_constant__ CUtensorMap tmY, const __grid_constant__ CUtensorMap tmA,
                         const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmR,
@@ -245,7 +254,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                         const float* __restrict__ sw, int n, int d_in, int d_out, float* __restrict__ y,
                         int32_t* __restrict__ acc_out, int use_tma_store, int num_full, int split, int split_slot,
                         uint32_t* __restrict__ status) {
-  using L = GemmLayout<E8>;
+  using L = GemmLayout<E8, NB>;
+  // the pair tile: 256 tokens x NB channels; each CTA holds NB / 2 rows of B
+  constexpr uint32_t kAtomBn = (uint32_t)(NB / 2) * 128;   // one 128-code K atom of B
+  constexpr uint32_t kStageBn = (uint32_t)(NB / 2) * BK;   // a stage's B (two atoms)
+  constexpr uint32_t kIdescN = idesc_e4m3_f32(2 * BM, NB);
+  static_assert(NB == NB || E8, "the packed-code path uses 128-channel tiles");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   // packed codes: SE x 2 atoms x [64 rows x 128 B] decoded B; byte codes: SE x [A 2 atoms x [128 rows x
@@ -262,7 +276,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const uint32_t rank = cluster_rank();         // 0: the pair's MMA issuer
   const int pair = blockIdx.x >> 1, num_pairs = gridDim.x >> 1;
   const int num_m = (n + 2 * BM - 1) / (2 * BM);  // 256-token pair tiles
-  const int num_n = (d_out + BN - 1) / BN;
+  const int num_n = (d_out + NB - 1) / NB;
   const int num_k = (d_in + BK - 1) / BK;
   const int num_tiles = num_m * num_n;
   const int n_split = (num_tiles - num_full) * split;   // 0 without a split
@@ -310,17 +324,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       for (int u = pair; u < total_units && ok; u += num_pairs) {
         const Unit w = unit_at(u, num_full, split, num_k, n_split);
         const int m = w.tile % num_m, nn = w.tile / num_m;
-        const int row = is_a ? m * 2 * BM + (int)rank * BM : nn * BN + (int)rank * BNC;
+        const int row = is_a ? m * 2 * BM + (int)rank * BM : nn * NB + (int)rank * (NB / 2);
         for (int ks = w.k0; ks < w.k1; ++ks, ++it) {
           if constexpr (E8) {
             // the stage's two K atoms; the even CTA's A producer also expects the odd CTA's 4-byte signal
-            const uint32_t s = it % SE, use = it / SE;
+            const uint32_t s = it % L::S, use = it / L::S;
             if (use > 0 && !(ok = mbar_wait_bounded(&bars->empty[s], (use - 1) & 1, abort_flag, __LINE__))) break;
-            uint8_t* dst = bst + s * kStage8 + (is_a ? 0u : kStageA8);
+            uint8_t* dst = bst + s * L::kStageOp + (is_a ? 0u : kStageA8);
             uint64_t* fb = rank == 0 ? &bars->full[s] : &bars->ready[s];
-            mbar_arrive_expect_tx(fb, is_a ? kStageA8 + (rank == 0 ? 4u : 0u) : kStageB);
+            mbar_arrive_expect_tx(fb, is_a ? kStageA8 + (rank == 0 ? 4u : 0u) : kStageBn);
             tma_load_2d(dst, map, ks * BK, row, fb);
-            tma_load_2d(dst + (is_a ? kAtomA8 : kAtomB), map, ks * BK + 128, row, fb);
+            tma_load_2d(dst + (is_a ? kAtomA8 : kAtomBn), map, ks * BK + 128, row, fb);
           } else {
             const uint32_t s = it % SP, use = it / SP;
             if (use > 0 && !(ok = mbar_wait_bounded(&bars->p_empty[s], (use - 1) & 1, abort_flag, __LINE__))) break;
@@ -334,8 +348,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       // the copies in flight land before the CTA exits (they have, unless a wait gave up)
       volatile int no_abort = 0;
       if constexpr (E8) {
-        for (uint32_t j = it > (uint32_t)SE ? it - SE : 0; j < it; ++j)
-          mbar_wait_bounded(rank == 0 ? &bars->full[j % SE] : &bars->ready[j % SE], (j / SE) & 1, &no_abort);
+        for (uint32_t j = it > (uint32_t)L::S ? it - L::S : 0; j < it; ++j)
+          mbar_wait_bounded(rank == 0 ? &bars->full[j % L::S] : &bars->ready[j % L::S], (j / L::S) & 1, &no_abort);
       } else {
         for (uint32_t j = it > (uint32_t)SP ? it - SP : 0; j < it; ++j)
           mbar_wait_bounded(&bars->p_full[j % kDecGroups][j % SP], (j / kPFullPeriod) & 1, &no_abort);
@@ -346,7 +360,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     // An arrive on the even CTA's barrier from a thread that has just written shared and tensor
     // memory stalls it for ~1.5k cycles (the cluster-scope release drains its writes), so the decode
     // warps arrive locally and one thread per decode group carries the stage's readiness over with an
-    // asynchronous 4-byte store that completes bytes on the even CTA's stage barrier.
+    // asynchronous 4-byte store that completes bytes on the even CTA's stage barrier.  Each forwarder
+    // takes the stages of one parity, so every barrier's phases are waited for in order by one thread
+    // (a thread that skipped a phase would wait for one two ahead, which a parity wait returns at
+    // once); with an even number of stages that is also the decode group of the step.
     if (lane == 0) {
       const uint32_t grp = warp == kMmaWarp ? 0u : 1u;
       uint32_t it = 0;
@@ -354,9 +371,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       for (int u = pair; u < total_units && ok; u += num_pairs) {
         const Unit w = unit_at(u, num_full, split, num_k, n_split);
         for (int ks = w.k0; ks < w.k1; ++ks, ++it) {
-          if ((it & 1u) != grp) continue;
-          const uint32_t s = it % SE;
-          if (!(ok = mbar_wait_bounded(&bars->ready[s], (it / SE) & 1, abort_flag, __LINE__))) break;
+          const uint32_t s = it % L::S;
+          if ((s & 1u) != grp) continue;
+          if (!(ok = mbar_wait_bounded(&bars->ready[s], (it / L::S) & 1, abort_flag, __LINE__))) break;
           tc_fence_after();
           st_async_signal(&bars->fwd_word[s], &bars->full[s], 0);
         }
@@ -374,24 +391,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         if (tcount >= 2 && !(ok = mbar_wait_bounded(&bars->acc_empty[ab], ((tcount >> 1) - 1) & 1, abort_flag, __LINE__))) break;
         tc_fence_after();
         for (int ks = w.k0; ks < w.k1; ++ks, ++it) {
-          const uint32_t s = it % SE;
-          if (!(ok = mbar_wait_bounded(&bars->full[s], (it / SE) & 1, abort_flag, __LINE__))) break;
+          const uint32_t s = it % L::S;
+          if (!(ok = mbar_wait_bounded(&bars->full[s], (it / L::S) & 1, abort_flag, __LINE__))) break;
           tc_fence_after();
           if constexpr (E8) {
-            const uint32_t abase = smem_u32(bst + s * kStage8), bbase = abase + kStageA8;
+            const uint32_t abase = smem_u32(bst + s * L::kStageOp), bbase = abase + kStageA8;
 #pragma unroll
             for (int kk = 0; kk < BK / 32; ++kk) {  // K = 32 codes per MMA: atom kk/4 of A and of B, +32 B
               const uint64_t da = sdesc_kmajor_sw128(abase + (uint32_t)(kk >> 2) * kAtomA8) + 2 * (kk & 3);
-              const uint64_t db = sdesc_kmajor_sw128(bbase + (uint32_t)(kk >> 2) * kAtomB) + 2 * (kk & 3);
-              mma_pair_ss(tmem + ab * BN, da, db, kIdesc, (ks != w.k0 || kk != 0) ? 1u : 0u);
+              const uint64_t db = sdesc_kmajor_sw128(bbase + (uint32_t)(kk >> 2) * kAtomBn) + 2 * (kk & 3);
+              mma_pair_ss(tmem + ab * NB, da, db, kIdescN, (ks != w.k0 || kk != 0) ? 1u : 0u);
             }
           } else {
-            const uint32_t bbase = smem_u32(bst + s * kStageB);
+            const uint32_t bbase = smem_u32(bst + s * kStageBn);
             const uint32_t ta = tmem + kAccCols + 64u * s;
 #pragma unroll
             for (int kk = 0; kk < BK / 32; ++kk) {  // K = 32 codes per MMA: 8 TMEM columns of A; B atom kk/4, +32 B
-              const uint64_t db = sdesc_kmajor_sw128(bbase + (uint32_t)(kk >> 2) * kAtomB) + 2 * (kk & 3);
-              mma_pair_ts(tmem + ab * BN, ta + 8u * kk, db, kIdesc, (ks != w.k0 || kk != 0) ? 1u : 0u);
+              const uint64_t db = sdesc_kmajor_sw128(bbase + (uint32_t)(kk >> 2) * kAtomBn) + 2 * (kk & 3);
+              mma_pair_ts(tmem + ab * NB, ta + 8u * kk, db, kIdescN, (ks != w.k0 || kk != 0) ? 1u : 0u);
             }
           }
           mma_commit_pair(&bars->empty[s]);
@@ -407,7 +424,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     const int quad = warp & 3, ew = warp - kEpiWarp0;
     uint8_t* stage0 = epi + ew * L::EB * kEpiStage;
     uint8_t* rstage0 = refb + ew * L::RB * kEpiStage;
-    float* wsc = scl + ew * BN;
+    float* wsc = scl + ew * NB;
     const bool with_ref = sums3 != nullptr;
     f32x2 sig = {0.f, 0.f}, err = {0.f, 0.f};      // SQNR sums of this thread's outputs
     uint32_t tcount = 0, nstore = 0;
@@ -422,7 +439,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       uint64_t* bar = &bars->ref_full[ew][rb_];
       if (lane == 0) {
         mbar_arrive_expect_tx(bar, kEpiStage);
-        tma_load_2d(rstage0 + rb_ * kEpiStage, &tmR, nn_ * BN + c_ * 32, m_ * 2 * BM + (int)rank * BM + quad * 32,
+        tma_load_2d(rstage0 + rb_ * kEpiStage, &tmR, nn_ * NB + c_ * 32, m_ * 2 * BM + (int)rank * BM + quad * 32,
                     bar);
       }
       ++nref[rb_];
@@ -520,7 +537,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
               pq[i] = __ldcg(&g_split_part[split_slot][tj * S + i % S][g0 + b + i / S][my_row]);
 #pragma unroll
             for (int k = 0; k < PB; ++k) {
-              const int o = nn * BN + 4 * (g0 + b + k);
+              const int o = nn * NB + 4 * (g0 + b + k);
               yr[k] = (with_ref && t < n && o < d_out)
                           ? __ldcs(reinterpret_cast<const float4*>(y_ref + (size_t)t * d_out + o))
                           : make_float4(0.f, 0.f, 0.f, 0.f);
@@ -535,7 +552,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 acc4.z += pq[k * S + q].z;
                 acc4.w += pq[k * S + q].w;
               }
-              const int gl = g0 + b + k, o = nn * BN + 4 * gl;
+              const int gl = g0 + b + k, o = nn * NB + 4 * gl;
               const float a[4] = {acc4.x, acc4.y, acc4.z, acc4.w};
               float v[4];
 #pragma unroll
@@ -592,8 +609,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       if constexpr (!E8) {
         __syncwarp();
 #pragma unroll
-        for (int i = 0; i < BN / 32; ++i) {  // this tile's output-channel steps, staged once per unit
-          const int o = nn * BN + 32 * i + lane;
+        for (int i = 0; i < NB / 32; ++i) {  // this tile's output-channel steps, staged once per unit
+          const int o = nn * NB + 32 * i + lane;
           wsc[32 * i + lane] = (o < d_out) ? sw[o] : 0.f;
         }
         __syncwarp();
@@ -603,17 +620,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       tc_fence_after();
       if (w.part < 0) {
 #pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
+        for (int c = 0; c < NB / 32; ++c) {
           uint32_t r[32];
           __syncwarp();
-          CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + ab * BN + c * 32, r);
+          CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + ab * NB + c * 32, r);
           tmem_ld_wait();
-          if (c == BN / 32 - 1) {  // accumulator fully read: the MMAs of unit + 2 may use it
+          if (c == NB / 32 - 1) {  // accumulator fully read: the MMAs of unit + 2 may use it
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive_cluster(&bars->acc_empty[ab], 0);
           }
-          const int o0 = nn * BN + c * 32;
+          const int o0 = nn * NB + c * 32;
           float a[32], v[32];
           if constexpr (E8) {                    // the chunk's 32 channel steps, one per lane
             const float swl = (o0 + lane < d_out) ? __ldg(sw + o0 + lane) : 0.f;
@@ -633,7 +650,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             // SQNR sums (Sec. 2, Eq. 1) from the y_ref tile of this chunk; out-of-range entries are zero
             // on both sides.  Squares are summed in fp32 over the chunk's 32 values, then as float pairs.
             const int rbuf = c % L::RB;
-            const uint32_t use = (BN / 32 / L::RB) * fcount + c / L::RB;  // the use-th load into buffer rbuf
+            const uint32_t use = (NB / 32 / L::RB) * fcount + c / L::RB;  // the use-th load into buffer rbuf
             if (!(ok = mbar_wait_bounded(&bars->ref_full[ew][rbuf], use & 1, abort_flag, __LINE__))) break;
             ++nused[rbuf];
             const uint8_t* rb = rstage0 + rbuf * kEpiStage + lane * 128;
@@ -649,8 +666,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             err = f2_add(err, e_run);
             // refill this buffer with the chunk RB ahead (this tile or the next: whole tiles follow)
             int nu = u, nc = c + L::RB;
-            if (nc >= BN / 32) {
-              nc -= BN / 32;
+            if (nc >= NB / 32) {
+              nc -= NB / 32;
               nu = u + num_pairs;
             }
             fence_proxy_async_smem();
@@ -665,12 +682,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         // a K part of a tail tile: this warp's 32 rows of raw accumulators to the part's slice
         const int tj = w.tile - num_full, j = u;
 #pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
+        for (int c = 0; c < NB / 32; ++c) {
           uint32_t r[32];
           __syncwarp();
-          CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + ab * BN + c * 32, r);
+          CAT_TMEM_LD32(tmem + ((uint32_t)(quad * 32) << 16) + ab * NB + c * 32, r);
           tmem_ld_wait();
-          if (c == BN / 32 - 1) {
+          if (c == NB / 32 - 1) {
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive_cluster(&bars->acc_empty[ab], 0);
@@ -757,13 +774,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         // one 128-byte row.  Chunk j (codes 32j .. 32j+31) becomes the 16-byte E4M3 chunks 2(j%4) and
         // 2(j%4)+1 of atom j/4; threads of atom 1 store their odd chunk first, so the 8 threads of a
         // row never hit the same bank group in one store
-        uint8_t* bs = bst + s * kStageB;
+        uint8_t* bs = bst + s * kStageBn;
 #pragma unroll
-        for (int i = 0; i < BNC * 8 / kGroupThreads; ++i) {
+        for (int i = 0; i < (NB / 2) * 8 / kGroupThreads; ++i) {
           const int id = gt + kGroupThreads * i;
           const int row = id >> 3, j = id & 7, swz = row & 7;
           const uint4 w = *reinterpret_cast<const uint4*>(pb + row * 128 + ((j ^ swz) << 4));
-          uint8_t* dst = bs + (j >> 2) * kAtomB + row * 128;
+          uint8_t* dst = bs + (j >> 2) * kAtomBn + row * 128;
           const uint4 lo = make_uint4(sm4_lo(w.x), sm4_hi(w.x), sm4_lo(w.y), sm4_hi(w.y));
           const uint4 hi = make_uint4(sm4_lo(w.z), sm4_hi(w.z), sm4_lo(w.w), sm4_hi(w.w));
           const int c0 = 2 * (j & 3);
@@ -855,7 +872,7 @@ int num_sms() {
 // once per process and operand format, on the first device asked).
 template <bool E8>
 bool split_launch_ok(int64_t pairs) {
-  using L = GemmLayout<E8>;
+  using L = GemmLayout<E8, BN>;
   static int ok = -1;
   static std::mutex mu;
   std::lock_guard<std::mutex> lock(mu);
@@ -864,14 +881,15 @@ bool split_launch_ok(int64_t pairs) {
     ok = 0;
     if (cudaGetDevice(&dev) == cudaSuccess &&
         cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) == cudaSuccess && coop &&
-        cudaFuncSetAttribute(w4a4_gemm_tc_kernel<E8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaFuncSetAttribute(w4a4_gemm_tc_kernel<E8, BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)L::kSmemBytes) == cudaSuccess) {
       cudaLaunchConfig_t cfg;
       memset(&cfg, 0, sizeof(cfg));
       cfg.gridDim = dim3((unsigned)(2 * pairs), 1, 1);
       cfg.blockDim = dim3(kThreads, 1, 1);
       cfg.dynamicSmemBytes = L::kSmemBytes;
-      if (cudaOccupancyMaxActiveClusters(&clusters, w4a4_gemm_tc_kernel<E8>, &cfg) == cudaSuccess && clusters >= pairs)
+      if (cudaOccupancyMaxActiveClusters(&clusters, w4a4_gemm_tc_kernel<E8, BN>, &cfg) == cudaSuccess &&
+          clusters >= pairs)
         ok = 1;
     }
     cudaGetLastError();
@@ -881,12 +899,13 @@ bool split_launch_ok(int64_t pairs) {
 
 // y_ref != nullptr: the epilogue also forms the SQNR sums of y against y_ref and writes
 // sums3 = {sum y_ref^2, sum (y_ref - y)^2, dB} (sums3 needs no zeroing).  Needs d_out % 4 == 0
-// (TMA row pitch).  E8: xq and wq hold one code per byte, else SM4x8 (two per byte).
-template <bool E8>
+// (TMA row pitch).  E8: xq and wq hold one code per byte, else SM4x8 (two per byte).  NB: channels per
+// pair tile (256 only with byte codes; the last wave is then not split along K).
+template <bool E8, int NB>
 cudaError_t launch_gemm_tc(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
                            int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, const float* y_ref, double* sums3,
                            uint32_t* status, cudaStream_t stream) {
-  using L = GemmLayout<E8>;
+  using L = GemmLayout<E8, NB>;
   CUtensorMap ty, ta, tb, tr;
   memset(&ty, 0, sizeof(ty));
   memset(&tr, 0, sizeof(tr));
@@ -897,23 +916,23 @@ cudaError_t launch_gemm_tc(const uint8_t* xq, const float* sx, const uint8_t* wq
       return cudaErrorInvalidValue;
   }
   const int64_t row_bytes = E8 ? d_in : d_in / 2;
-  if (!make_packed_map(&ta, xq, n, row_bytes, BM) || !make_packed_map(&tb, wq, d_out, row_bytes, BNC))
+  if (!make_packed_map(&ta, xq, n, row_bytes, BM) || !make_packed_map(&tb, wq, d_out, row_bytes, NB / 2))
     return cudaErrorInvalidValue;
   static std::once_flag attr_once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(attr_once, [] {
-    attr_err = cudaFuncSetAttribute(w4a4_gemm_tc_kernel<E8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    attr_err = cudaFuncSetAttribute(w4a4_gemm_tc_kernel<E8, NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                     (int)L::kSmemBytes);
   });
   if (attr_err != cudaSuccess) return attr_err;
-  const int64_t tiles = ((n + 2 * BM - 1) / (2 * BM)) * ((d_out + BN - 1) / BN);
+  const int64_t tiles = ((n + 2 * BM - 1) / (2 * BM)) * ((d_out + NB - 1) / NB);
   const int64_t num_k = (d_in + BK - 1) / BK;
   const int64_t pairs_max = num_sms() / 2;
   // the last wave's tiles, split along K into a power-of-two number of parts when that wave is at
   // most half full (the parts wait for one another: only with a cooperative launch)
   const int64_t tail = tiles >= pairs_max ? tiles % pairs_max : tiles;
   int split = 1;
-  if (tail > 0 && tail <= kMaxSplitTiles && 2 * tail <= pairs_max && split_launch_ok<E8>(pairs_max))
+  if (NB == BN && tail > 0 && tail <= kMaxSplitTiles && 2 * tail <= pairs_max && split_launch_ok<E8>(pairs_max))
     while (2 * split <= kMaxSplit && 2 * split * tail <= pairs_max && 2 * split <= num_k) split *= 2;
   // a single partial wave has no whole tiles to hide the parts' exchange behind: split it only
   // when that saves ten K steps or more
@@ -940,9 +959,26 @@ cudaError_t launch_gemm_tc(const uint8_t* xq, const float* sx, const uint8_t* wq
   attrs[1].val.cooperative = 1;
   cfg.attrs = attrs;
   cfg.numAttrs = split > 1 ? 2 : 1;
-  return cudaLaunchKernelEx(&cfg, w4a4_gemm_tc_kernel<E8>, ty, ta, tb, tr, y_ref, const_cast<double*>(sums), slot, sx,
+  return cudaLaunchKernelEx(&cfg, w4a4_gemm_tc_kernel<E8, NB>, ty, ta, tb, tr, y_ref, const_cast<double*>(sums), slot, sx,
                             sw, (int)n, (int)d_in, (int)d_out, y, acc_out, use_tma, (int)num_full, split, split_slot,
                             status);
+}
+
+// Byte codes: 256-channel pair tiles where they take less time than 128-channel ones.  The MMA thread's
+// wait for each stage idles the tensor core for ~200-300 cycles, whatever the tile width, so a 256-wide
+// tile (twice the MMA work per stage) costs kWideTileCost of two 128-wide tiles (measured: 0.78 on the
+// 8192 x 8192 x 28672 and 4096 x 14336 x 4096 layers); but there are half as many tiles to spread over
+// the pairs, and the last wave is not split along K.
+constexpr double kWideTileCost = 0.78;
+bool e8_wide_tiles(int64_t n, int64_t d_out) {
+  const int64_t pairs = num_sms() / 2, m_tiles = (n + 2 * BM - 1) / (2 * BM);
+  const int64_t t128 = m_tiles * ((d_out + BN - 1) / BN), t256 = m_tiles * ((d_out + 255) / 256);
+  const int64_t tail = t128 % pairs;
+  // 128-wide: a last wave at most half full is split along K over the idle pairs
+  const double w128 = (tail > 0 && 2 * tail <= pairs && tail <= kMaxSplitTiles) ? (double)t128 / pairs
+                                                                                 : (double)((t128 + pairs - 1) / pairs);
+  const double w256 = 2.0 * kWideTileCost * (double)((t256 + pairs - 1) / pairs);
+  return w256 < w128;
 }
 
 }  // namespace
@@ -950,13 +986,15 @@ cudaError_t launch_gemm_tc(const uint8_t* xq, const float* sx, const uint8_t* wq
 cudaError_t launch_w4a4_gemm_tc(const uint8_t* xq, const float* sx, const uint8_t* wq, const float* sw, int64_t n,
                                 int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, const float* y_ref,
                                 double* sums3, uint32_t* status, cudaStream_t stream) {
-  return launch_gemm_tc<false>(xq, sx, wq, sw, n, d_in, d_out, y, acc_out, y_ref, sums3, status, stream);
+  return launch_gemm_tc<false, BN>(xq, sx, wq, sw, n, d_in, d_out, y, acc_out, y_ref, sums3, status, stream);
 }
 
 cudaError_t launch_w4a4_gemm_tc_e8(const uint8_t* xq8, const float* sx, const uint8_t* wq8, const float* sw, int64_t n,
                                    int64_t d_in, int64_t d_out, float* y, int32_t* acc_out, const float* y_ref,
                                    double* sums3, uint32_t* status, cudaStream_t stream) {
-  return launch_gemm_tc<true>(xq8, sx, wq8, sw, n, d_in, d_out, y, acc_out, y_ref, sums3, status, stream);
+  if (e8_wide_tiles(n, d_out))
+    return launch_gemm_tc<true, 256>(xq8, sx, wq8, sw, n, d_in, d_out, y, acc_out, y_ref, sums3, status, stream);
+  return launch_gemm_tc<true, BN>(xq8, sx, wq8, sw, n, d_in, d_out, y, acc_out, y_ref, sums3, status, stream);
 }
 
 // SM4x8 codes -> byte codes.  Every 16 packed bytes (32 codes of a row) become 32 bytes: the masks of
