@@ -5,7 +5,9 @@ computes one by one), and -- where the oracle finishes in seconds -- on the whol
 Tolerances as in test_gpu_parity.py.  The whole-output oracle check covers the QKV, down and
 decode layers.  On every layer, the 70B gate/up layer included, the whole output is also checked by
 a property that holds at any size: the same codes and steps through the independent digit-plane
-GEMM give the packed GEMM's y bit for bit (both accumulate exactly)."""
+GEMM give the packed GEMM's y bit for bit (both accumulate exactly).  For n > 32 the byte-code calls
+that bench.py times for prefill (transform with byte codes out, GEMM with SQNR sums) give the same
+codes, steps and y."""
 import numpy as np
 import pytest
 import torch
@@ -14,7 +16,7 @@ import dp_planes
 import oracle as O
 import sm4x8
 import workloads as WL
-from test_gpu_parity import DEV, check_codes, gpu_layer, rel_fro
+from test_gpu_parity import DEV, check_codes, gpu_layer, rel_fro, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -104,6 +106,18 @@ def test_full_size_layer(name, k, kind):
     np.testing.assert_array_equal(dp_planes.decode(xp[:, ts_d].cpu().numpy()), sm4x8.unpack(g["xq"][ts_d].cpu().numpy()))
     y_dp = cat.cat_linear_dp(xp, 4, g["sx"], _planes_on_device(g["Wq"]), 4, g["sw"])
     assert torch.equal(y_dp, y_gpu)
+    if n > 32:
+        # the byte-code calls bench.py times for prefill: the same codes (as bytes, against the format's
+        # definition above), the same steps, y bit for bit, the same SQNR sums
+        planes = (cat.cat_split_transform(g["T"], k)
+                  if (cfg.dtype == "bf16" and cat.cat_split_transform_bytes(d_in, k) > 0) else None)
+        xq8, sx8 = cat.cat_transform_quantize_act_e8(to_dev(L.x_eval), g["T"], planes, k)
+        assert torch.equal(xq8, xp[0]) and torch.equal(sx8, g["sx"])
+        y8, o3 = cat.cat_w4a4_linear_sqnr_e8(xq8, sx8, cat.cat_codes_to_e4m3(g["Wq"]), g["sw"], y_ref)
+        assert torch.equal(y8, y_gpu)
+        o3 = o3.cpu().numpy()
+        assert abs(o3[1] - s3[1]) <= 1e-6 * s3[1] and abs(o3[2] - s3[2]) < 1e-4
+        del xq8, y8
     if name in FULL_OUTPUT and kind == "cat":
         ref = O.transform_quantize_act(L.x_eval.values, T)
         prep_q, prep_s, _ = O.quantize_rows_symmetric(O.apply_weight_transform(Wv, Ti))
