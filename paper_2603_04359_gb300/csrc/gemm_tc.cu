@@ -231,6 +231,19 @@ __device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
   return v;
 }
 
+// Tile t of the launch -> (token tile m, channel tile nn).  Tiles go in bands of kBandM token tiles,
+// m fastest within a band, so the tiles a wave of pairs works on at once cover ~kBandM token tiles by
+// a few channel tiles rather than every token tile by ~2 channel tiles: at 8192 x 8192 x 28672 on 76
+// pairs, ~35 MB of operand rows per wave instead of ~70 MB, all read from DRAM again each wave.
+constexpr int kBandM = 8;
+__device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int* m, int* nn) {
+  const int m0 = (t / (kBandM * num_n)) * kBandM;     // the band's first token tile
+  const int bm = min(kBandM, num_m - m0);             // token tiles in this band (fewer in the last)
+  const int r = t - m0 * num_n;                       // the tile's index within its band
+  *m = m0 + r % bm;
+  *nn = r / bm;
+}
+
 // Work unit u of the launch: the n_split = tail x split parts come first (part u % split of tail
 // tile num_full + u / split, on pairs 0 .. n_split - 1, one each), then the whole tiles (tile
 // u - n_split).  All parts run at the same time, as their pairs' first units, and each part's share
@@ -323,7 +336,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int u = pair; u < total_units && ok; u += num_pairs) {
         const Unit w = unit_at(u, num_full, split, num_k, n_split);
-        const int m = w.tile % num_m, nn = w.tile / num_m;
+        int m, nn;
+        tile_coords(w.tile, num_m, num_n, &m, &nn);
         const int row = is_a ? m * 2 * BM + (int)rank * BM : nn * NB + (int)rank * (NB / 2);
         for (int ks = w.k0; ks < w.k1; ++ks, ++it) {
           if constexpr (E8) {
@@ -434,7 +448,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     // regularly.  The epilogue of a split tail tile reads y_ref with plain loads.
     uint32_t nref[kEpiBufs] = {0u, 0u}, nused[kEpiBufs] = {0u, 0u};  // loads issued / consumed per buffer
     auto load_ref = [&](int tile_, int c_) {        // called by the whole warp; lane 0 issues
-      const int m_ = tile_ % num_m, nn_ = tile_ / num_m;
+      int m_, nn_;
+      tile_coords(tile_, num_m, num_n, &m_, &nn_);
       const int rb_ = c_ % L::RB;
       uint64_t* bar = &bars->ref_full[ew][rb_];
       if (lane == 0) {
@@ -519,7 +534,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     auto finish_share = [&](int uu) {
       const Unit w = unit_at(uu, num_full, split, num_k, n_split);
       const int tj = w.tile - num_full;
-      const int m = w.tile % num_m, nn = w.tile / num_m;
+      int m, nn;
+      tile_coords(w.tile, num_m, num_n, &m, &nn);
       const int t = m * 2 * BM + (int)rank * BM + quad * 32 + lane;
       const float sxt = (t < n) ? sx[t] * kAccScale : 0.f;
       if (wait_parts(tj)) {
@@ -602,7 +618,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     for (; u < total_units; u += num_pairs, ++tcount) {
       const Unit w = unit_at(u, num_full, split, num_k, n_split);
       const uint32_t ab = tcount & 1;
-      const int m = w.tile % num_m, nn = w.tile / num_m;
+      int m, nn;
+      tile_coords(w.tile, num_m, num_n, &m, &nn);
       const int row0 = m * 2 * BM + (int)rank * BM + quad * 32;
       const int t = row0 + lane;
       const float sxt = (t < n) ? sx[t] * kAccScale : 0.f;
