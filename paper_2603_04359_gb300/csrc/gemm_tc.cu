@@ -214,15 +214,18 @@ __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wa
 // power of two, at most 16), one part per pair.  Every part writes its raw accumulators to its own
 // slice of device scratch with plain stores (float32 atomics from many SMs onto one tile are an
 // order of magnitude slower), waits until all S parts of the tile have arrived (bounded; the launch
-// is cooperative, so all parts are resident), and then finishes 128 / S of the tile's channels:
+// is cooperative, so all parts are resident), and then finishes NB / S of the tile's channels:
 // the sum over the parts (exact in any order: integer multiples of 2^-18 below 2^6 in magnitude),
 // the scaling, y, acc_out and the SQNR sums.  Counters are per (tile, CTA, epilogue warp); the last
 // part to finish sets them back to zero.  Slots of this scratch are handed out round robin per launch.
 constexpr int kSplitSlots = 2;
 constexpr int kMaxSplitTiles = 38;            // half a wave of 76 pairs
-constexpr int kMaxSplitUnits = 80;            // tail tiles x parts <= pairs
+constexpr int kMaxSplitUnits = 80;            // tail tiles x parts x NB / 128 <= pairs
 constexpr int kMaxSplit = 16;
-__device__ float4 g_split_part[kSplitSlots][kMaxSplitUnits][BN / 4][2 * BM];   // [part][channel/4][row]
+// Per slot: [part][channel/4][row] float4 slices of NB / 4 x 2 BM, room for kMaxSplitUnits 128-wide parts
+// (half as many 256-wide ones).
+constexpr size_t kSplitSlotF4 = (size_t)kMaxSplitUnits * (BN / 4) * (2 * BM);
+__device__ float4 g_split_part[kSplitSlots * kSplitSlotF4];
 __device__ uint32_t g_split_cnt[kSplitSlots][kMaxSplitTiles][2][kEpiWarps][2];   // arrived, finished
 
 __device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
@@ -499,6 +502,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     // tail tiles: this lane's row of part j's partial accumulators, the counters of this warp's
     // 32-row slice of tail tile tj, and the bounded wait for all parts of the tile
     const int my_row = (int)rank * BM + quad * 32 + lane;
+    // part j's partial accumulators of channel group g (4 channels), this lane's row
+    auto split_at = [&](int j, int g) {
+      return g_split_part + (size_t)split_slot * kSplitSlotF4 + ((size_t)j * (NB / 4) + g) * (2 * BM) + my_row;
+    };
     auto cnt_of = [&](int tj, int which) { return &g_split_cnt[split_slot][tj][rank][ew][which]; };
     auto arrive_part = [&](int tj) {                // after this lane's partial stores
       __threadfence();
@@ -529,7 +536,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         *cnt_of(tj, 1) = 0u;
       }
     };
-    // the share of split unit uu's tile that its part finishes: channels [128 / S * part, ...) of the
+    // the share of split unit uu's tile that its part finishes: channels [NB / S * part, ...) of the
     // tile, once all S parts' partials are out
     auto finish_share = [&](int uu) {
       const Unit w = unit_at(uu, num_full, split, num_k, n_split);
@@ -543,14 +550,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         auto fixup = [&](auto split_c) {
           constexpr int S = decltype(split_c)::value;
           constexpr int L = S >= 4 ? 16 : 8;      // loads of parts per batch
-          constexpr int G = 32 / S, PB = L / S;   // groups of the share, groups per batch
+          constexpr int G = NB / 4 / S, PB = L / S;   // groups of the share, groups per batch
           const int g0 = w.part * G;
 #pragma unroll 1
           for (int b = 0; b < G; b += PB) {
             float4 pq[L], yr[PB];
 #pragma unroll
             for (int i = 0; i < L; ++i)
-              pq[i] = __ldcg(&g_split_part[split_slot][tj * S + i % S][g0 + b + i / S][my_row]);
+              pq[i] = __ldcg(split_at(tj * S + i % S, g0 + b + i / S));
 #pragma unroll
             for (int k = 0; k < PB; ++k) {
               const int o = nn * NB + 4 * (g0 + b + k);
@@ -711,7 +718,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           }
 #pragma unroll
           for (int q = 0; q < 8; ++q)   // a warp stores 32 consecutive rows of one channel group: 512 B
-            __stcg(&g_split_part[split_slot][j][8 * c + q][my_row],
+            __stcg(split_at(j, 8 * c + q),
                    make_float4(__uint_as_float(r[4 * q]), __uint_as_float(r[4 * q + 1]), __uint_as_float(r[4 * q + 2]),
                                __uint_as_float(r[4 * q + 3])));
         }
@@ -887,9 +894,9 @@ int num_sms() {
 
 // Whether a cooperative launch of `pairs` CTA pairs of the GEMM kernel fits on this device (checked
 // once per process and operand format, on the first device asked).
-template <bool E8>
+template <bool E8, int NB>
 bool split_launch_ok(int64_t pairs) {
-  using L = GemmLayout<E8, BN>;
+  using L = GemmLayout<E8, NB>;
   static int ok = -1;
   static std::mutex mu;
   std::lock_guard<std::mutex> lock(mu);
@@ -898,14 +905,14 @@ bool split_launch_ok(int64_t pairs) {
     ok = 0;
     if (cudaGetDevice(&dev) == cudaSuccess &&
         cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) == cudaSuccess && coop &&
-        cudaFuncSetAttribute(w4a4_gemm_tc_kernel<E8, BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaFuncSetAttribute(w4a4_gemm_tc_kernel<E8, NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)L::kSmemBytes) == cudaSuccess) {
       cudaLaunchConfig_t cfg;
       memset(&cfg, 0, sizeof(cfg));
       cfg.gridDim = dim3((unsigned)(2 * pairs), 1, 1);
       cfg.blockDim = dim3(kThreads, 1, 1);
       cfg.dynamicSmemBytes = L::kSmemBytes;
-      if (cudaOccupancyMaxActiveClusters(&clusters, w4a4_gemm_tc_kernel<E8, BN>, &cfg) == cudaSuccess &&
+      if (cudaOccupancyMaxActiveClusters(&clusters, w4a4_gemm_tc_kernel<E8, NB>, &cfg) == cudaSuccess &&
           clusters >= pairs)
         ok = 1;
     }
@@ -949,14 +956,18 @@ cudaError_t launch_gemm_tc(const uint8_t* xq, const float* sx, const uint8_t* wq
   // most half full (the parts wait for one another: only with a cooperative launch)
   const int64_t tail = tiles >= pairs_max ? tiles % pairs_max : tiles;
   int split = 1;
-  if (NB == BN && tail > 0 && tail <= kMaxSplitTiles && 2 * tail <= pairs_max && split_launch_ok<E8>(pairs_max))
-    while (2 * split <= kMaxSplit && 2 * split * tail <= pairs_max && 2 * split <= num_k) split *= 2;
+  constexpr int64_t kWide = NB / BN;             // a part's scratch, in 128-wide parts
+  if (tail > 0 && tail <= kMaxSplitTiles && 2 * tail <= pairs_max && split_launch_ok<E8, NB>(pairs_max))
+    while (2 * split <= kMaxSplit && 2 * split * tail <= pairs_max && 2 * split <= num_k &&
+           2 * split * tail * kWide <= kMaxSplitUnits)
+      split *= 2;
   // a single partial wave has no whole tiles to hide the parts' exchange behind: split it only
   // when that saves ten K steps or more
   if (split > 1 && tiles < pairs_max && num_k - num_k / split < 10) split = 1;
   const int64_t num_full = split > 1 ? tiles - tail : tiles;
   const int64_t units = num_full + (tiles - num_full) * split;
-  if (split > 1 && (units - num_full > kMaxSplitUnits || num_full % pairs_max != 0)) return cudaErrorInvalidConfiguration;
+  if (split > 1 && ((units - num_full) * kWide > kMaxSplitUnits || num_full % pairs_max != 0))
+    return cudaErrorInvalidConfiguration;
   const int grid = 2 * (int)(units < pairs_max ? units : pairs_max);  // CTA pairs (cluster of 2)
   if (grid > kSqnrMaxCtas) return cudaErrorInvalidConfiguration;
   static std::atomic<unsigned> next_split{0};
@@ -990,11 +1001,13 @@ constexpr double kWideTileCost = 0.78;
 bool e8_wide_tiles(int64_t n, int64_t d_out) {
   const int64_t pairs = num_sms() / 2, m_tiles = (n + 2 * BM - 1) / (2 * BM);
   const int64_t t128 = m_tiles * ((d_out + BN - 1) / BN), t256 = m_tiles * ((d_out + 255) / 256);
-  const int64_t tail = t128 % pairs;
-  // 128-wide: a last wave at most half full is split along K over the idle pairs
-  const double w128 = (tail > 0 && 2 * tail <= pairs && tail <= kMaxSplitTiles) ? (double)t128 / pairs
-                                                                                 : (double)((t128 + pairs - 1) / pairs);
-  const double w256 = 2.0 * kWideTileCost * (double)((t256 + pairs - 1) / pairs);
+  // a last wave at most half full is split along K over the idle pairs (in about that proportion)
+  auto waves = [&](int64_t tiles) {
+    const int64_t tail = tiles % pairs;
+    return (tail > 0 && 2 * tail <= pairs && tail <= kMaxSplitTiles) ? (double)tiles / pairs
+                                                                      : (double)((tiles + pairs - 1) / pairs);
+  };
+  const double w128 = waves(t128), w256 = 2.0 * kWideTileCost * waves(t256);
   return w256 < w128;
 }
 
