@@ -79,13 +79,17 @@ __device__ __forceinline__ void sqnr_cta_done(int slot, f32x2 sig, f32x2 err, do
   unsigned last = 0;
   if (lane == 0) {
     g_sqnr_part[slot][blockIdx.x] = make_float4(sig.hi, sig.lo, err.hi, err.lo);
-    __threadfence();
-    last = atomicAdd(&g_sqnr_count[slot], 1u) == gridDim.x - 1;
+    // one acquire-release increment instead of two GPU-scope fences: its release orders this CTA's row
+    // before the count, and the last CTA's acquire (the counter's increments form one release
+    // sequence) orders every row before its reads
+    unsigned old;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(&g_sqnr_count[slot]) : "memory");
+    last = old == gridDim.x - 1;
   }
   last = __shfl_sync(0xFFFFFFFFu, last, 0);
   if (!last) return;
-  __threadfence();
-  // every other CTA's row has landed (each fenced its row before its counter increment); lane l
+  __syncwarp();   // the other lanes' loads come after lane 0's acquire
+  // every other CTA's row is visible (each released it with its counter increment); lane l
   // adds rows l, l + 32, ... with eight loads in flight at a time
   f32x2 a = {0.f, 0.f}, b = {0.f, 0.f};
   const unsigned rows = gridDim.x;
