@@ -1001,13 +1001,14 @@ constexpr double kWideTileCost = 0.78;
 bool e8_wide_tiles(int64_t n, int64_t d_out) {
   const int64_t pairs = num_sms() / 2, m_tiles = (n + 2 * BM - 1) / (2 * BM);
   const int64_t t128 = m_tiles * ((d_out + BN - 1) / BN), t256 = m_tiles * ((d_out + 255) / 256);
-  // a last wave at most half full is split along K over the idle pairs (in about that proportion)
-  auto waves = [&](int64_t tiles) {
+  // a last wave at most half full is split along K over the idle pairs (in about that proportion),
+  // when the scratch holds at least two parts of each of its tiles (as the launcher decides)
+  auto waves = [&](int64_t tiles, int64_t wide) {
     const int64_t tail = tiles % pairs;
-    return (tail > 0 && 2 * tail <= pairs && tail <= kMaxSplitTiles) ? (double)tiles / pairs
-                                                                      : (double)((tiles + pairs - 1) / pairs);
+    const bool split = tail > 0 && 2 * tail <= pairs && tail <= kMaxSplitTiles && 2 * tail * wide <= kMaxSplitUnits;
+    return split ? (double)tiles / pairs : (double)((tiles + pairs - 1) / pairs);
   };
-  const double w128 = waves(t128), w256 = 2.0 * kWideTileCost * waves(t256);
+  const double w128 = waves(t128, 1), w256 = 2.0 * kWideTileCost * waves(t256, 2);
   return w256 < w128;
 }
 
