@@ -73,6 +73,25 @@ def test_host_validation_without_gpu(lib):
     # cat_sqnr(y_ref, y_hat, numel, out3, stream)
     assert lib.cat_sqnr(P, P, -1, P, None) == 2
     assert lib.cat_sqnr(P, None, 10, P, None) == 1
+    # byte codes: cat_codes_to_e4m3(codes, rows, d, out, stream)
+    assert lib.cat_codes_to_e4m3(P, 4, 48, P, None) == 2                                 # d % 32
+    assert lib.cat_codes_to_e4m3(P, -1, 64, P, None) == 2                                # rows < 0
+    assert lib.cat_codes_to_e4m3(P, 0, 64, None, None) == 0                              # rows == 0: no-op
+    assert lib.cat_codes_to_e4m3(P, 4, 64, None, None) == 1                              # NULL
+    assert lib.cat_codes_to_e4m3(bad, 4, 64, P, None) == 3                               # alignment
+    # cat_transform_quantize_act_e8(x, dtype, n, d_in, k, T, T_planes, xq8, sx, stream)
+    assert lib.cat_transform_quantize_act_e8(P, 1, 4, 48, 16, P, None, P, P, None) == 2  # d_in % 32
+    assert lib.cat_transform_quantize_act_e8(P, 7, 4, 64, 32, P, None, P, P, None) == 1  # dtype
+    assert lib.cat_transform_quantize_act_e8(P, 1, 4, 64, 32, P, None, None, P, None) == 1   # NULL xq8
+    assert lib.cat_transform_quantize_act_e8(P, 1, 4, 64, 32, P, bad, P, P, None) == 3   # planes alignment
+    assert lib.cat_transform_quantize_act_e8(P, 1, 0, 64, 32, None, None, None, None, None) == 0
+    # cat_w4a4_linear_e8(xq8, sx, wq8, sw, n, d_in, d_out, y, acc, stream) and the SQNR variant
+    assert lib.cat_w4a4_linear_e8(P, P, P, P, 4, 300000, 8, P, None, None) == 2         # exactness bound
+    assert lib.cat_w4a4_linear_e8(P, P, P, P, 4, 64, 0, P, None, None) == 2             # d_out
+    assert lib.cat_w4a4_linear_e8(P, P, P, P, 4, 64, 8, None, None, None) == 1          # y NULL
+    assert lib.cat_w4a4_linear_e8(P, P, bad, P, 4, 64, 8, P, None, None) == 3           # alignment
+    assert lib.cat_w4a4_linear_sqnr_e8(P, P, P, P, 4, 64, 8, P, P, None, None) == 1     # out3 NULL
+    assert lib.cat_w4a4_linear_sqnr_e8(P, P, P, P, 4, 96, 8, P, bad, P, None) == 3      # y_ref alignment
 
 
 def test_valid_call_without_device_reports_cuda_error(lib):
