@@ -8,8 +8,18 @@
 // products q_x q_w 2^-18 in fp32 tensor memory (exact: |acc| <= 49 d_in < 2^24), and the epilogue
 // multiplies by 2^18 s_x s_w.
 //
-// Data path.  The tensor cores read their shared-memory operands on a path of their own (their
-// rate does not change under concurrent LSU shared-memory traffic) and an MMA with A in tensor
+// Two operand formats share this kernel (template parameter E8):
+//   * byte codes (E8): the codes are stored one E4M3 byte each, so TMA loads them into 128B-swizzled
+//     shared memory as they are and the pair MMAs read both operands there -- no decode warps.  Tiles
+//     are 256 x 128 (four 48 KB stages) or 256 x 256 (NB = 256: three 64 KB stages, the two
+//     accumulators filling tensor memory), chosen per shape by e8_wide_tiles;
+//   * SM4x8 codes: the packed codes are decoded in the kernel, as described below (tiles 256 x 128).
+// Both walk the tiles in bands of kBandM token tiles, and both split a last wave that is at most half
+// full along K.
+//
+// Data path of the SM4x8 kernel.  The tensor cores read their shared-memory operands on a path of
+// their own (their rate does not change under concurrent LSU shared-memory traffic) and an MMA with
+// A in tensor
 // memory runs at ~93% of peak, while the decode of the packed B operand into shared memory is the
 // costliest step.  So two SMs share each output tile (a cluster pair and tcgen05.mma.cta_group::2):
 //   * the pair tile is 256 tokens x 128 channels; each CTA owns 128 tokens (the A rows, in its own
